@@ -1,0 +1,55 @@
+"""The oracle's pins catch plausible mistakes.
+
+Each case copies the oracle's C source, plants one mistake (a dropped term, a
+wrong sign, a reversed tie order, a wrong rounding ...), compiles the copy and
+runs the pin suite against it: the suite must fail.  Everything runs on the CPU.
+"""
+import os
+import shutil
+import subprocess
+import sys
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+SRC = os.path.join(ROOT, "oracle", "iso_oracle.c")
+
+MUTATIONS = {
+    "tie_order_reversed_sort": ("if (x->pos != y->pos) return (x->pos < y->pos) ? -1 : 1;",
+                                "if (x->pos != y->pos) return (x->pos > y->pos) ? -1 : 1;"),
+    "one_tie_too_many": ("else if (kp == t && taken < need)", "else if (kp == t && taken <= need)"),
+    "signed_key": ("return f32_bits(t) & 0x7FFFFFFFu;", "return f32_bits(t);"),
+    "k_truncates": ("double kk = floor(rho * (double)n + 0.5);", "double kk = floor(rho * (double)n);"),
+    "ties_disagreeing_set": ("if (tt != 0.0f && sign_f(tt) == gamma)", "if (tt != 0.0f && sign_f(tt) != gamma)"),
+    "ties_plain_mean": ("double merged = cnt ? acc / (double)cnt : 0.0;",
+                        "double merged = cnt ? acc / (double)K : 0.0;"),
+    "ties_untrimmed_election": ("float tt = mask[i][p] ? tau32[i][p] : 0.0f;", "float tt = tau32[i][p];"),
+    "ta_drops_lambda": ("out[p] = add_update(theta0[p], lambda * s);", "out[p] = add_update(theta0[p], s);"),
+    "retention_rhs_ones": ("b[r] = gram[idx[r] * K + idx[r]];", "b[r] = 1.0;"),
+    "retention_no_clip": ("if (c > c_max) c = c_max;", ";"),
+    "gram_diagonal_only": ("s += gi * gj;", "s += gi * gi;"),
+    "gram_untrimmed": ("double gi = mask[i][p] ? tau64[i][p] : 0.0;", "double gi = tau64[i][p];"),
+    "iso_1d_no_average": ("out[p] = add_update(theta0[p], s / (double)K);", "out[p] = add_update(theta0[p], s);"),
+    "bf16_round_half_up": ("u += 0x7FFFu + lsb;", "u += 0x8000u;"),
+    "bf16_f64_truncates": ("double q = round_half_even(ldexp(a, -q_exp));", "double q = floor(ldexp(a, -q_exp));"),
+    "zero_update_normalises_sign": ("return (upd == 0.0) ? theta0 : theta0 + upd;", "return theta0 + upd;"),
+}
+
+
+@pytest.mark.parametrize("name", sorted(MUTATIONS))
+def test_pins_catch_mutation(name, tmp_path):
+    old, new = MUTATIONS[name]
+    src = open(SRC).read()
+    assert src.count(old) == 1, f"mutation anchor not found: {name}"
+    mdir = tmp_path / "oracle_mut"
+    mdir.mkdir()
+    shutil.copy(os.path.join(ROOT, "oracle", "iso_oracle.h"), mdir / "iso_oracle.h")
+    (mdir / "iso_oracle.c").write_text(src.replace(old, new))
+    so = mdir / "libmut.so"
+    subprocess.check_call(["gcc", "-O2", "-std=c11", "-ffp-contract=off", "-fPIC", "-shared",
+                           "-o", str(so), str(mdir / "iso_oracle.c"), "-lm"])
+    env = dict(os.environ, ISO_ORACLE_LIB=str(so))
+    r = subprocess.run([sys.executable, "-m", "pytest", "-x", "-q", "-p", "no:cacheprovider",
+                        os.path.join(ROOT, "tests", "test_oracle_pins.py")],
+                       cwd=ROOT, env=env, capture_output=True, text=True, timeout=600)
+    assert r.returncode != 0, f"pins did not catch mutation {name}:\n{r.stdout[-2000:]}"
