@@ -1,0 +1,353 @@
+"""Benchmark of the whole-model delta -> TopKMask -> update/merge pass.
+
+One step = one pass of the hot path over a full synthetic parameter set held
+in HBM.  Default workload: the Qwen2.5-1.5B-shaped masked ISO update (bf16
+base and RL checkpoint, 253 tensors, 1,543,655,424 parameters, per-tensor
+TopKMask density 5 %).  Other workloads (--workload) are for investigation.
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--impl mine|reference]
+
+Prints one JSON line.  Under torchrun (N > 1) every rank runs its own copy of
+the workload (weak scaling, no data-path collective); the step time is the
+maximum over ranks.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import subprocess
+import sys
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "G params/s and achieved HBM GB/s (% of ~8 TB/s) for full-model mask+merge"
+UNIT = "Gparams/s"
+NOMINAL_HBM_GBS = 8000.0
+
+WORKLOADS = {
+    # name: (shape set, K, op, inputs, density, description)
+    "qwen1.5b_update": ("qwen1.5b", 1, "iso", "ckpt_bf16", 0.05,
+                        "Qwen2.5-1.5B-shaped bf16 base + RL checkpoint, masked ISO update, "
+                        "per-tensor TopKMask 5%"),
+    "qwen7b_update": ("qwen7b", 1, "iso", "ckpt_bf16", 0.05,
+                      "Qwen2.5-7B-shaped bf16 base + RL checkpoint, fused delta+mask+update, "
+                      "per-tensor TopKMask 5%"),
+    "qwen7b_ties_k8": ("qwen7b", 8, "ties", "delta_f32", 0.10,
+                       "Qwen2.5-7B-shaped bf16 base, 8 fp32 RL deltas, TopKMask 10% + TIES"),
+    "qwen7b_iso_k8": ("qwen7b", 8, "iso", "delta_f32", 0.10,
+                      "Qwen2.5-7B-shaped bf16 base, 8 fp32 RL deltas, TopKMask 10% + ISO retention"),
+}
+
+
+def algorithmic_bytes(shapes, K, inputs, op):
+    """Bytes a pass must move at minimum: read theta_0 and the K experts once,
+    write the output once.  Returned per kernel kind: (apply, count)."""
+    n_all = sum(r * c for r, c, _ in shapes)
+    n_trim = sum(r * c for r, c, one in shapes if not (one and op == "iso"))
+    if inputs == "ckpt_bf16":
+        per_x, per_base, per_out = 2, 2, 2
+    else:
+        per_x, per_base, per_out = 4, 2, 2
+    apply = n_all * (per_base + K * per_x + per_out)
+    count = n_trim * (K * per_x + (per_base if inputs == "ckpt_bf16" else 0))
+    return {"apply": apply, "count": count}
+
+
+def read_peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(p) as f:
+            d = json.load(f)
+        return float(d["hbm_gbs"]), "measured"
+    except Exception:
+        return 6800.0, "fallback"
+
+
+class Clocks:
+    """nvidia-smi sampler for the timed region."""
+    Q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+         "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+         "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int, path: str):
+        self.path = path
+        self.idx = gpu_index
+        self.p = None
+        try:
+            self.f = open(path, "w")
+            self.p = subprocess.Popen(["nvidia-smi", f"--query-gpu={self.Q}", "--format=csv,noheader,nounits",
+                                       "-i", str(gpu_index), "-lms", "100"], stdout=self.f,
+                                      stderr=subprocess.DEVNULL)
+        except Exception:
+            self.p = None
+
+    def stop(self):
+        if self.p is None:
+            return None
+        self.p.terminate()
+        try:
+            self.p.wait(timeout=5)
+        except Exception:
+            self.p.kill()
+        self.f.close()
+        rows = []
+        for line in open(self.path):
+            parts = [x.strip() for x in line.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                rows.append((float(parts[1]), float(parts[2]), parts[5:9]))
+            except ValueError:
+                continue
+        if not rows:
+            return None
+        sm = sorted(r[0] for r in rows)
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[i] for r in rows for i, v in enumerate(r[2]) if v.lower() == "active"})
+        return {"sm_mhz": sm[len(sm) // 2], "sm_max_mhz": max(r[1] for r in rows),
+                "reasons": reasons, "samples": len(rows)}
+
+
+def make_workload(name, device, seed):
+    import torch
+    import synth
+    shapes_name, K, op, inputs, density, desc = WORKLOADS[name]
+    shapes = synth.qwen_shapes(shapes_name)
+    if inputs == "ckpt_bf16":
+        th0, th1 = synth.rl_update_set(shapes, seed=seed, device=device)
+        experts = [th1]
+    else:
+        th0 = synth.base_weights(shapes, seed=seed, device=device)
+        experts, _ = synth.merge_experts(shapes, seed=seed, K=K, device=device)
+    torch.cuda.synchronize()
+    return shapes, th0, experts
+
+
+def run_mine(args):
+    import torch
+    import torch.distributed as dist
+    import paper_2607_19331_gb300 as iso
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if world > 1:
+        dist.init_process_group("nccl")
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    name = args.workload
+    shapes_name, K, op, inputs, density, desc = WORKLOADS[name]
+    shapes, th0, experts = make_workload(name, dev, seed=rank)
+    n_params = sum(t.numel() for t in th0)
+    ckpt = inputs == "ckpt_bf16"
+    out = [torch.empty_like(t) for t in th0]
+    cfg = iso.merge_cfg(op, density, "tensor")
+    mn, full = iso.iso_workspace_size(th0, K, cfg)
+    free = torch.cuda.mem_get_info(dev)[0]
+    ws_bytes = full if full + (1 << 30) < free else max(mn, free - (2 << 30))
+    ws = iso.Workspace(dev)
+    ws.get(ws_bytes)
+    stream = torch.cuda.current_stream(dev)
+
+    def step():
+        iso.iso_merge(th0, experts, op=op, experts_are_deltas=not ckpt, out=out, density=density,
+                      scope="tensor", lam=1.0, workspace=ws, ws_bytes=ws_bytes, stream=stream)
+
+    def barrier():
+        if world > 1:
+            dist.barrier()
+
+    for _ in range(args.warmup):
+        step()
+    torch.cuda.synchronize()
+    barrier()
+    os.makedirs(os.path.join(ROOT, "gpurun_out"), exist_ok=True)
+    clocks = Clocks(local, os.path.join(ROOT, "gpurun_out", f"clocks_rank{rank}.csv")) if rank == 0 else None
+    time.sleep(0.3 if clocks else 0)
+    l0 = iso.launch_count()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    torch.cuda.synchronize()
+    barrier()
+    e0.record(stream)
+    for _ in range(args.steps):
+        step()
+    e1.record(stream)
+    torch.cuda.synchronize()
+    barrier()
+    launches = (iso.launch_count() - l0) // max(1, args.steps)
+    ms = e0.elapsed_time(e1) / args.steps
+    ck = clocks.stop() if clocks else None
+    if world > 1:
+        t = torch.tensor([ms], device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ms = float(t.item())
+    value = world * n_params / (ms * 1e-3) / 1e9
+
+    # per-kernel device time through the library's event brackets
+    iso.profile_reset()
+    iso.profile_enable(True)
+    prof_steps = max(3, min(args.steps, 10))
+    for _ in range(prof_steps):
+        step()
+    torch.cuda.synchronize()
+    prof = iso.profile_read()
+    iso.profile_enable(False)
+    algo = algorithmic_bytes(shapes, K, inputs, op)
+    peak, peak_src = read_peaks()
+    kernels = {k: {"launches": n // prof_steps, "ms_per_step": tot / prof_steps} for k, (n, tot) in prof.items()}
+    dom = max(("apply", "count"), key=lambda k: prof.get(k, (0, 0.0))[1])
+    n_dom, t_dom = prof.get(dom, (1, 0.0))
+    avg_ms = t_dom / max(1, n_dom)
+    per_launch_bytes = algo[dom] / max(1, n_dom // prof_steps)
+    achieved = per_launch_bytes / (avg_ms * 1e-3) / 1e9 if avg_ms > 0 else 0.0
+    step_gbs = (algo["apply"] + algo["count"]) / (ms * 1e-3) / 1e9
+
+    # end to end through the public API from pinned host memory
+    e2e = None
+    if not args.no_e2e and ckpt:
+        h0 = [t.cpu().pin_memory() for t in th0]
+        h1 = [t.cpu().pin_memory() for t in experts[0]]
+        del th0, experts
+        torch.cuda.empty_cache()
+        stage = iso.HostStaging(h0, h1, dev)
+        for _ in range(2):
+            stage.run(h0, h1, op=op, update_is_delta=False, density=density, workspace=ws, ws_bytes=ws_bytes)
+        torch.cuda.synchronize()
+        f0, f1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        n_e2e = max(2, min(args.steps, 5))
+        f0.record(stream)
+        for _ in range(n_e2e):
+            stage.run(h0, h1, op=op, update_is_delta=False, density=density, workspace=ws, ws_bytes=ws_bytes)
+        f1.record(stream)
+        torch.cuda.synchronize()
+        ms_e2e = f0.elapsed_time(f1) / n_e2e
+        e2e = {"value": round(world * n_params / (ms_e2e * 1e-3) / 1e9, 3), "unit": UNIT,
+               "ms_per_step": round(ms_e2e, 3), "h2d_bytes_per_step": stage.h2d_bytes,
+               "d2h_bytes_per_step": stage.d2h_bytes}
+
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        cpu = cpu_baseline(name, budget_s=args.cpu_budget)
+
+    if rank == 0:
+        line = {
+            "metric": METRIC, "value": round(value, 3), "unit": UNIT, "n_gpus": world,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms, 4),
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+            "dtype": "bf16" if ckpt else "f32", "data": "synthetic (seeded, Qwen-shaped; no checkpoints)",
+            "config": {"workload": name, "description": desc, "params": n_params, "tensors": len(shapes),
+                       "experts": K, "op": op, "density": density, "scope": "tensor",
+                       "l2": "inputs larger than L2 (129 MB); no flush needed",
+                       "parallelism": f"replica x{world}"},
+            "hbm_gbs_step": round(step_gbs, 1),
+            "hbm_pct_of_8tbs_step": round(100 * step_gbs / NOMINAL_HBM_GBS, 1),
+            "roofline": {"bound": "hbm", "kernel": dom, "achieved": round(achieved, 1), "peak": peak,
+                         "peak_source": peak_src, "unit": "GB/s",
+                         "frac": round(achieved / peak, 4) if peak else None, "traffic": None,
+                         "algorithmic_bytes_per_launch": int(per_launch_bytes),
+                         "avg_launch_ms": round(avg_ms, 4)},
+            "kernels": {k: {"launches": v["launches"], "ms_per_step": round(v["ms_per_step"], 4)}
+                        for k, v in sorted(kernels.items(), key=lambda kv: -kv[1]["ms_per_step"])},
+            "gpu_launches": int(launches),
+            "clocks": ck,
+            "e2e": e2e,
+            "cpu_baseline": cpu,
+        }
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        dist.destroy_process_group()
+
+
+def cpu_sample(name, seed=0):
+    """A bounded, deterministic list of tensors of the workload (layer 0 first)."""
+    import synth
+    shapes_name = WORKLOADS[name][0]
+    shapes = synth.qwen_shapes(shapes_name)
+    order = list(range(1, 10)) + list(range(10, len(shapes)))   # layer 0, then onwards
+    return shapes, order
+
+
+def cpu_baseline(name, budget_s=15.0, seed=0):
+    """The oracle, as it stands, on a bounded sample of the workload: tensors
+    are added in a fixed order until budget_s of single-thread CPU time."""
+    import numpy as np
+    import oracle
+    import synth
+    shapes_name, K, op, inputs, density, _ = WORKLOADS[name]
+    shapes, order = cpu_sample(name, seed)
+    orc_op = {"ta": oracle.TA, "ties": oracle.TIES, "iso": oracle.ISO}[op]
+    done, params, spent = [], 0, 0.0
+    for q in order:
+        s = shapes[q]
+        if inputs == "ckpt_bf16":
+            th0, th1 = synth.rl_update_set([s], seed=seed + q)
+            a = [th0[0].view(-1).view(__import__("torch").int16).numpy().view(np.uint16).reshape(s[0], s[1])]
+            ex = [[th1[0].view(-1).view(__import__("torch").int16).numpy().view(np.uint16).reshape(s[0], s[1])]]
+        else:
+            th0 = synth.base_weights([s], seed=seed + q)
+            taus, _ = synth.merge_experts([s], seed=seed + q, K=K)
+            a = [th0[0].view(-1).view(__import__("torch").int16).numpy().view(np.uint16).reshape(s[0], s[1])]
+            ex = [[e[0].reshape(s[0], s[1]).numpy()] for e in taus]
+        t = time.perf_counter()
+        oracle.merge(a, ex, orc_op, experts_are_deltas=(inputs != "ckpt_bf16"), density=density,
+                     is_1d=[s[2]])
+        spent += time.perf_counter() - t
+        params += s[0] * s[1]
+        done.append(q)
+        if spent >= budget_s:
+            break
+    return {"value": round(params / spent / 1e9, 6), "unit": UNIT, "cores": 1, "kind": "oracle",
+            "sample": f"{len(done)} tensors of the workload ({params} params: tensor ids {done[0]}..{done[-1]} "
+                      f"in layer order), timed on this host, single thread",
+            "seconds": round(spent, 2)}
+
+
+def run_reference(args):
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return
+    name = args.workload
+    per_step = max(2.0, args.cpu_budget / max(1, args.steps))
+    for _ in range(args.warmup and 1):
+        cpu_baseline(name, budget_s=0.5)
+    vals = []
+    for _ in range(args.steps):
+        vals.append(cpu_baseline(name, budget_s=per_step))
+    v = sum(x["value"] for x in vals) / len(vals)
+    line = {
+        "impl": "reference", "metric": METRIC, "value": round(v, 6), "unit": UNIT, "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "f64 values / f32 decisions", "data": "synthetic (seeded, Qwen-shaped)",
+        "config": {"workload": name, "description": WORKLOADS[name][5]},
+        "cpu_baseline": {"value": round(v, 6), "unit": UNIT, "cores": 1, "kind": "oracle",
+                         "sample": vals[-1]["sample"]},
+        "e2e": {"value": round(v, 6), "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=30)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", choices=["mine", "reference"], default="mine")
+    ap.add_argument("--workload", choices=sorted(WORKLOADS), default="qwen1.5b_update")
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--cpu-budget", type=float, default=12.0)
+    args = ap.parse_args()
+    if args.warmup < 3 and args.impl == "mine":
+        args.warmup = 3
+    if args.impl == "reference":
+        run_reference(args)
+    else:
+        run_mine(args)
+
+
+if __name__ == "__main__":
+    main()

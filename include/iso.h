@@ -1,0 +1,215 @@
+/*
+ * iso.h -- C ABI of the GB300 delta-merge library (libiso_gb300.so).
+ *
+ * The library implements the element-wise, data-parallel pass over parameter
+ * updates from "ISO: An RLVR-Native Optimization Stack": for every weight
+ * tensor it forms the task vector, trims it with an exact TopKMask, elects
+ * signs where the operator has an election, and writes the merged or updated
+ * weights
+ *
+ *     theta_merge = theta_0 + tau_merge                   (App. F, problem statement)
+ *
+ * for three operators:
+ *   ISO_OP_TA    Task Arithmetic   tau = lambda * sum_i tau_i                (App. F)
+ *   ISO_OP_TIES  TIES              trim, sign election, disjoint mean,
+ *                                  theta_0 + lambda * tau_TIES              (App. F)
+ *   ISO_OP_ISO   ISO retention     Gram of the trimmed task vectors,
+ *                                  (Gamma + ridge I) c = diag Gamma, clip to
+ *                                  [c_min, c_max], theta_0 + sum_i c_i trimmed tau_i;
+ *                                  1-D tensors take the plain task-vector
+ *                                  average                (Sec. 4.2, App. E, Algorithm 1)
+ *
+ * TopKMask(|tau|, rho) (App. F, TIES trim) keeps the k = floor(rho n + 1/2)
+ * entries of largest |tau| in each selection unit; entries with equal |tau|
+ * are taken lowest flat index first (in GLOBAL scope: tensor order, then flat
+ * index).  |tau| is ranked by its binary32 value.
+ *
+ * Conventions for every entry point
+ *   - All tensor data pointers, mask pointers, stats pointers and the workspace
+ *     are DEVICE pointers owned by the caller.  The library never allocates,
+ *     frees or retains device memory; it only reads the inputs, writes the
+ *     outputs, and uses the caller's workspace as scratch for the duration of
+ *     the call.
+ *   - Tensors are row-major and contiguous; data pointers must be 16-byte
+ *     aligned.  A 1-D tensor is passed as rows = 1, cols = n, is_1d = 1.
+ *   - Work is enqueued on `stream` (a cudaStream_t; NULL = legacy default
+ *     stream) and the call returns without waiting.  Inputs must stay valid
+ *     and unmodified, and the workspace untouched, until the stream reaches
+ *     the end of the call's work.  Calls that share a workspace must be
+ *     ordered on one stream.
+ *   - The return value is ISO_OK or a negative iso_status.  Argument errors
+ *     (ARG, SHAPE, DTYPE, ALIGN, WORKSPACE, UNSUPPORTED) are detected on the
+ *     host before anything is enqueued.  ISO_ERR_CUDA means a launch failed.
+ *     ISO_ERR_NONFINITE is detected on the device: it is written to
+ *     stats->status (when given) and is valid once the stream has reached the
+ *     end of the call; the outputs of such a call are unspecified.
+ *   - No C++ exception crosses this interface.  The library keeps no state
+ *     between calls apart from optional profiling counters.
+ */
+#ifndef ISO_H
+#define ISO_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define ISO_ABI_VERSION 1
+
+typedef enum {
+    ISO_OK = 0,
+    ISO_ERR_ARG = -1,          /* NULL where a pointer is required, count or enum out of range,
+                                  density outside [0, 1], non-finite lambda / ridge / clip bounds */
+    ISO_ERR_SHAPE = -2,        /* base, expert, out, mask shapes disagree; negative extents */
+    ISO_ERR_DTYPE = -3,        /* dtype outside iso_dtype, out dtype differs from the base, or
+                                  experts of mixed dtype */
+    ISO_ERR_ALIGN = -4,        /* a data pointer is not 16-byte aligned */
+    ISO_ERR_WORKSPACE = -5,    /* workspace NULL, not 256-byte aligned, or smaller than the
+                                  minimum reported by iso_workspace_size */
+    ISO_ERR_CUDA = -6,         /* a CUDA launch or runtime call failed */
+    ISO_ERR_NONFINITE = -7,    /* (device) an input held NaN or +-Inf */
+    ISO_ERR_UNSUPPORTED = -8   /* valid request outside this build: K > ISO_MAX_EXPERTS,
+                                  a tensor with 2^32 or more entries, GLOBAL scope larger
+                                  than the workspace allows */
+} iso_status;
+
+#define ISO_MAX_EXPERTS 8
+
+typedef enum { ISO_BF16 = 0, ISO_F32 = 1 } iso_dtype;
+
+/* One tensor of a flat parameter list. */
+typedef struct {
+    void*   data;   /* device pointer, 16-byte aligned, rows * cols entries */
+    int64_t rows;   /* >= 0; 1 for a 1-D tensor */
+    int64_t cols;   /* >= 0 */
+    int32_t dtype;  /* iso_dtype */
+    int32_t is_1d;  /* 1 for normalisation scales, biases and other 1-D parameters */
+} iso_tensor;
+
+typedef enum {
+    ISO_SCOPE_TENSOR = 0,  /* one selection unit per tensor */
+    ISO_SCOPE_BLOCK = 1,   /* one unit per block_rows x block_cols tile of each tensor,
+                              tiles in row-major tile order, partial edge tiles allowed */
+    ISO_SCOPE_GLOBAL = 2   /* one unit over the whole task vector (tensor order, then
+                              flat index): the paper's global magnitude density */
+} iso_scope;
+
+typedef struct {
+    double  density;     /* rho in [0, 1]; k = floor(rho * n + 1/2) per unit */
+    int32_t scope;       /* iso_scope */
+    int32_t block_rows;  /* BLOCK scope: 1..256 (the paper-free default is 128) */
+    int32_t block_cols;  /* BLOCK scope: 8..256, a multiple of 8 */
+    int32_t reserved;    /* must be 0 */
+} iso_topk_cfg;
+
+typedef enum { ISO_OP_TA = 0, ISO_OP_TIES = 1, ISO_OP_ISO = 2 } iso_op;
+
+typedef struct {
+    int32_t op;          /* iso_op */
+    int32_t mask_1d;     /* TIES: 1 = 1-D tensors are trimmed like the rest of the task
+                            vector, 0 = used untrimmed.  Ignored by TA (never trims) and
+                            ISO (1-D tensors take the average) */
+    float   lambda;      /* TA / TIES scale (the paper uses 1.0) */
+    float   reserved;    /* must be 0 */
+    double  ridge;       /* ISO lambda_ridge (the paper uses 1e-12), >= 0 */
+    double  c_min;       /* ISO clip range (the paper uses [0, 1.5]) */
+    double  c_max;
+    iso_topk_cfg topk;   /* TopKMask of TIES and ISO; ignored by TA */
+} iso_merge_cfg;
+
+/* Per selection unit, written by the device. */
+typedef struct {
+    uint32_t thresh_key;      /* binary32 bits of the k-th largest |tau|; 0xFFFFFFFF when the
+                                 unit selects nothing (k == 0) or is not trimmed */
+    uint32_t flags;           /* bit 0: resolved by the full-data fallback; diagnostics only */
+    int64_t  k;               /* entries selected; -1 for a unit that is not trimmed */
+    int64_t  count_above;     /* entries with |tau| above the threshold */
+    int64_t  ties_at_thresh;  /* entries with |tau| equal to the threshold */
+    int64_t  ties_taken;      /* of those, how many are selected (lowest index first) */
+} iso_unit_stats;
+
+/* Optional device-side outputs of a call; every pointer may be NULL. */
+typedef struct {
+    int32_t*        status;  /* 1 value: ISO_OK or ISO_ERR_NONFINITE, valid after the stream
+                                reaches the end of the call */
+    iso_unit_stats* units;   /* [K][n_units], n_units from iso_num_units */
+    double*         gram;    /* ISO: [n_tensors][K][K] Gram of the trimmed task vectors
+                                (zero for 1-D tensors) */
+    double*         coef;    /* ISO: [n_tensors][K] retention coefficients c* */
+} iso_merge_stats;
+
+/* Host-only.  Number of selection units per expert for a tensor list under a
+ * TopKMask configuration (TENSOR: n_tensors; BLOCK: sum of tile counts;
+ * GLOBAL: 1). */
+int32_t iso_num_units(const iso_tensor* tensors, int32_t n_tensors, const iso_topk_cfg* topk,
+                      int64_t* n_units);
+
+/* Host-only.  Workspace bytes for iso_update / iso_merge (K experts) and, with
+ * K = 1, for iso_topk_mask.  *bytes_min receives the smallest workspace the
+ * call accepts (tensors are then processed in groups that fit); *bytes_full
+ * the size that processes the whole list in one group.  Either pointer may be
+ * NULL.  The workspace must be 256-byte aligned. */
+int32_t iso_workspace_size(const iso_tensor* tensors, int32_t n_tensors, int32_t K,
+                           const iso_merge_cfg* cfg, size_t* bytes_min, size_t* bytes_full);
+
+/* tau[t] = theta_i[t] - theta_0[t] for every tensor (App. F task vector),
+ * computed as one binary32 subtraction per entry and stored as ISO_F32.
+ * theta_i / theta_0 may be BF16 or F32; tau must be F32 and may not alias the
+ * inputs.  Needs no workspace. */
+int32_t iso_delta(const iso_tensor* theta_i, const iso_tensor* theta_0, const iso_tensor* tau,
+                  int32_t n_tensors, void* stream);
+
+/* TopKMask(|tau|, rho) over a task vector given as n_tensors tensors (BF16 or
+ * F32).  mask_bits[t] (device, may be NULL for a tensor, or mask_bits itself
+ * NULL) receives ceil(numel / 32) uint32 words: bit j of word w is entry
+ * 32 w + j.  stats->units receives [n_units] records; stats->gram / coef are
+ * unused. */
+int32_t iso_topk_mask(const iso_tensor* tau, int32_t n_tensors, const iso_topk_cfg* cfg,
+                      uint32_t* const* mask_bits, const iso_merge_stats* stats,
+                      void* workspace, size_t ws_bytes, void* stream);
+
+/* The K = 1 masked update of a base by one expert:
+ *   out = theta_0 + c * TopKMask(|tau|) * tau,   tau = update (update_is_delta = 1)
+ *                                               or update - theta_0 (a checkpoint)
+ * with c = lambda for TIES, c = clip(Gamma / (Gamma + ridge)) for ISO (Gamma the
+ * squared norm of the trimmed tensor); ISO leaves 1-D tensors at theta_0 + tau.
+ * TA applies lambda * tau untrimmed.  out has the base's dtype and may alias
+ * theta_0 (each entry is read before it is written by the same thread); it may
+ * not alias update. */
+int32_t iso_update(const iso_tensor* theta_0, const iso_tensor* update, int32_t update_is_delta,
+                   const iso_tensor* out, int32_t n_tensors, const iso_merge_cfg* cfg,
+                   void* workspace, size_t ws_bytes, const iso_merge_stats* stats, void* stream);
+
+/* Merge K experts (1 <= K <= ISO_MAX_EXPERTS) into the base.  experts holds
+ * K * n_tensors descriptors, expert-major (experts[i * n_tensors + t]); they
+ * are task vectors (experts_are_deltas = 1) or fine-tuned checkpoints.  All
+ * experts share one dtype.  out has the base's dtype and may alias theta_0. */
+int32_t iso_merge(const iso_tensor* theta_0, const iso_tensor* experts, int32_t K,
+                  int32_t experts_are_deltas, const iso_tensor* out, int32_t n_tensors,
+                  const iso_merge_cfg* cfg, void* workspace, size_t ws_bytes,
+                  const iso_merge_stats* stats, void* stream);
+
+/* Static description of a status code. */
+const char* iso_error_string(int32_t status);
+
+/* Diagnostics: number of kernels this process has launched through the
+ * library (all streams, all devices). */
+uint64_t iso_launch_count(void);
+
+/* Diagnostics: when enabled, each launch is bracketed by CUDA events on its
+ * stream.  iso_profile_read waits for the recorded events and returns, for
+ * kernel `kind` (0 .. iso_profile_kinds()-1), the number of launches and their
+ * summed device time since the last reset.  Profiling is host state, not
+ * thread-safe, and off by default. */
+int32_t     iso_profile_enable(int32_t on);
+int32_t     iso_profile_reset(void);
+int32_t     iso_profile_kinds(void);
+const char* iso_profile_name(int32_t kind);
+int32_t     iso_profile_read(int32_t kind, int64_t* launches, double* total_ms);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* ISO_H */

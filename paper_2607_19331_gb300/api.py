@@ -1,0 +1,267 @@
+"""PyTorch-facing binding of the C ABI (include/iso.h).
+
+Argument marshalling only: every function here builds the ABI descriptors
+from ``torch.Tensor`` objects (device memory and streams come from PyTorch)
+and calls the entry point of the same name in libiso_gb300.so, where every
+step of the computation runs.  There is no CPU path.
+"""
+from __future__ import annotations
+
+import ctypes
+from dataclasses import dataclass
+from typing import List, Optional, Sequence
+
+import numpy as np
+import torch
+
+from . import _abi
+from ._abi import (IsoMergeCfg, IsoMergeStats, IsoTensor, IsoTopkCfg, check, lib)
+
+OPS = {"ta": _abi.ISO_OP_TA, "ties": _abi.ISO_OP_TIES, "iso": _abi.ISO_OP_ISO}
+SCOPES = {"tensor": _abi.ISO_SCOPE_TENSOR, "block": _abi.ISO_SCOPE_BLOCK,
+          "global": _abi.ISO_SCOPE_GLOBAL}
+UNIT_STATS_DTYPE = np.dtype([
+    ("thresh_key", np.uint32), ("flags", np.uint32), ("k", np.int64),
+    ("count_above", np.int64), ("ties_at_thresh", np.int64), ("ties_taken", np.int64),
+])
+assert UNIT_STATS_DTYPE.itemsize == ctypes.sizeof(_abi.IsoUnitStats)
+
+
+def _code(dtype: torch.dtype) -> int:
+    if dtype == torch.bfloat16:
+        return _abi.ISO_BF16
+    if dtype == torch.float32:
+        return _abi.ISO_F32
+    raise TypeError(f"tensors must be bfloat16 or float32, got {dtype}")
+
+
+def _shape2d(t: torch.Tensor):
+    if t.dim() == 2:
+        return int(t.shape[0]), int(t.shape[1]), 0
+    if t.dim() == 1:
+        return 1, int(t.shape[0]), 1
+    raise ValueError("tensors must be 1-D or 2-D")
+
+
+def describe(ts: Sequence[torch.Tensor], is_1d: Optional[Sequence[bool]] = None):
+    """ctypes array of iso_tensor for a list of contiguous tensors."""
+    arr = (IsoTensor * max(1, len(ts)))()
+    for q, t in enumerate(ts):
+        if not t.is_contiguous():
+            raise ValueError("tensors must be contiguous")
+        r, c, one = _shape2d(t)
+        if is_1d is not None:
+            one = int(bool(is_1d[q]))
+        arr[q] = IsoTensor(t.data_ptr() if t.numel() else None, r, c, _code(t.dtype), one)
+    return arr
+
+
+def topk_cfg(density=0.05, scope="tensor", block=(128, 128)) -> IsoTopkCfg:
+    return IsoTopkCfg(float(density), SCOPES[scope], int(block[0]), int(block[1]), 0)
+
+
+def merge_cfg(op="ties", density=0.2, scope="tensor", block=(128, 128), lam=1.0, ridge=1e-12,
+              c_min=0.0, c_max=1.5, mask_1d=True) -> IsoMergeCfg:
+    return IsoMergeCfg(OPS[op], int(bool(mask_1d)), float(lam), 0.0, float(ridge), float(c_min),
+                       float(c_max), topk_cfg(density, scope, block))
+
+
+def _stream(stream) -> ctypes.c_void_p:
+    if stream is None:
+        stream = torch.cuda.current_stream()
+    return ctypes.c_void_p(stream.cuda_stream)
+
+
+@dataclass
+class Stats:
+    """Device-side outputs of one call (see iso_merge_stats)."""
+    status: torch.Tensor          # int32[1]
+    units: torch.Tensor           # uint8[K * n_units * 40]
+    gram: Optional[torch.Tensor]  # float64[n_tensors * K * K]
+    coef: Optional[torch.Tensor]  # float64[n_tensors * K]
+    K: int
+    n_units: int
+
+    def abi(self) -> IsoMergeStats:
+        return IsoMergeStats(self.status.data_ptr(), self.units.data_ptr(),
+                             self.gram.data_ptr() if self.gram is not None else None,
+                             self.coef.data_ptr() if self.coef is not None else None)
+
+    def units_numpy(self) -> np.ndarray:
+        raw = self.units.cpu().numpy()
+        return raw.view(UNIT_STATS_DTYPE).reshape(self.K, self.n_units)
+
+
+def make_stats(tensors, K, topk: IsoTopkCfg, device, with_gram=True) -> Stats:
+    n_units = iso_num_units(tensors, topk)
+    n = len(tensors)
+    return Stats(
+        status=torch.zeros(1, dtype=torch.int32, device=device),
+        units=torch.zeros(max(1, K * n_units) * UNIT_STATS_DTYPE.itemsize, dtype=torch.uint8, device=device),
+        gram=torch.zeros(max(1, n * K * K), dtype=torch.float64, device=device) if with_gram else None,
+        coef=torch.zeros(max(1, n * K), dtype=torch.float64, device=device) if with_gram else None,
+        K=K, n_units=n_units)
+
+
+class Workspace:
+    """Caller-owned scratch for the library, one growing torch buffer."""
+
+    def __init__(self, device=None):
+        self.device = torch.device(device or "cuda")
+        self.buf = torch.empty(0, dtype=torch.uint8, device=self.device)
+
+    def get(self, nbytes: int):
+        if self.buf.numel() < nbytes:
+            self.buf = torch.empty(nbytes + 256, dtype=torch.uint8, device=self.device)
+        ptr = self.buf.data_ptr()
+        off = (-ptr) % 256
+        return ctypes.c_void_p(ptr + off), self.buf.numel() - off
+
+
+_default_ws = {}
+
+
+def _workspace(ws: Optional[Workspace], device) -> Workspace:
+    if ws is not None:
+        return ws
+    key = torch.device(device).index
+    if key not in _default_ws:
+        _default_ws[key] = Workspace(device)
+    return _default_ws[key]
+
+
+# ---------------------------------------------------------------------------
+# entry points
+# ---------------------------------------------------------------------------
+
+def iso_num_units(tensors, topk: IsoTopkCfg) -> int:
+    d = describe(tensors)
+    n = ctypes.c_int64(0)
+    check(lib().iso_num_units(d, len(tensors), ctypes.byref(topk), ctypes.byref(n)), "iso_num_units")
+    return int(n.value)
+
+
+def iso_workspace_size(tensors, K: int, cfg: IsoMergeCfg):
+    """(minimum, full) workspace bytes."""
+    d = describe(tensors)
+    mn, full = ctypes.c_size_t(0), ctypes.c_size_t(0)
+    check(lib().iso_workspace_size(d, len(tensors), int(K), ctypes.byref(cfg), ctypes.byref(mn),
+                                   ctypes.byref(full)), "iso_workspace_size")
+    return int(mn.value), int(full.value)
+
+
+def iso_delta(theta_i: List[torch.Tensor], theta_0: List[torch.Tensor], tau=None, stream=None):
+    if tau is None:
+        tau = [torch.empty(t.shape, dtype=torch.float32, device=t.device) for t in theta_0]
+    check(lib().iso_delta(describe(theta_i), describe(theta_0), describe(tau), len(theta_0),
+                          _stream(stream)), "iso_delta")
+    return tau
+
+
+def iso_topk_mask(tau: List[torch.Tensor], density=0.2, scope="tensor", block=(128, 128),
+                  masks=None, workspace: Optional[Workspace] = None, stats=False, stream=None,
+                  ws_bytes: Optional[int] = None):
+    """Packed TopKMask of a task vector: per tensor ceil(numel/32) int32 words."""
+    dev = tau[0].device
+    cfg = topk_cfg(density, scope, block)
+    if masks is None:
+        masks = [torch.zeros((t.numel() + 31) // 32 + 4, dtype=torch.int32, device=dev) for t in tau]
+    mptrs = (ctypes.c_void_p * max(1, len(tau)))(*[m.data_ptr() for m in masks])
+    mcfg = merge_cfg("ties", density, scope, block)
+    _, full = iso_workspace_size(tau, 1, mcfg)
+    ws = _workspace(workspace, dev)
+    wptr, wlen = ws.get(full if ws_bytes is None else ws_bytes)
+    st = make_stats(tau, 1, cfg, dev, with_gram=False) if stats else None
+    check(lib().iso_topk_mask(describe(tau), len(tau), ctypes.byref(cfg), mptrs,
+                              ctypes.byref(st.abi()) if st else None, wptr,
+                              wlen if ws_bytes is None else ws_bytes, _stream(stream)),
+          "iso_topk_mask")
+    out = [m[: (t.numel() + 31) // 32] for m, t in zip(masks, tau)]
+    return (out, st) if stats else out
+
+
+def iso_merge(theta_0: List[torch.Tensor], experts: List[List[torch.Tensor]], op="ties",
+              experts_are_deltas=True, out=None, density=0.2, scope="tensor", block=(128, 128),
+              lam=1.0, ridge=1e-12, c_min=0.0, c_max=1.5, mask_1d=True, is_1d=None,
+              workspace: Optional[Workspace] = None, stats=False, stream=None,
+              ws_bytes: Optional[int] = None):
+    K = len(experts)
+    n = len(theta_0)
+    dev = theta_0[0].device
+    if out is None:
+        out = [torch.empty_like(t) for t in theta_0]
+    cfg = merge_cfg(op, density, scope, block, lam, ridge, c_min, c_max, mask_1d)
+    flat = [x for e in experts for x in e]
+    d0 = describe(theta_0, is_1d)
+    dx = describe(flat, None if is_1d is None else list(is_1d) * K)
+    do = describe(out, is_1d)
+    _, full = iso_workspace_size(theta_0, K, cfg)
+    ws = _workspace(workspace, dev)
+    wptr, wlen = ws.get(full if ws_bytes is None else ws_bytes)
+    st = make_stats(theta_0, K, cfg.topk, dev) if stats else None
+    fn = lib().iso_update if K == 1 else None
+    if K == 1:
+        rc = fn(d0, dx, int(bool(experts_are_deltas)), do, n, ctypes.byref(cfg), wptr,
+                wlen if ws_bytes is None else ws_bytes, ctypes.byref(st.abi()) if st else None,
+                _stream(stream))
+        check(rc, "iso_update")
+    else:
+        rc = lib().iso_merge(d0, dx, K, int(bool(experts_are_deltas)), do, n, ctypes.byref(cfg),
+                             wptr, wlen if ws_bytes is None else ws_bytes,
+                             ctypes.byref(st.abi()) if st else None, _stream(stream))
+        check(rc, "iso_merge")
+    return (out, st) if stats else out
+
+
+def iso_update(theta_0: List[torch.Tensor], update: List[torch.Tensor], op="iso",
+               update_is_delta=False, **kw):
+    """The K = 1 masked update (iso_update)."""
+    return iso_merge(theta_0, [update], op=op, experts_are_deltas=update_is_delta, **kw)
+
+
+class HostStaging:
+    """End-to-end use from host memory: pinned host inputs are copied to the
+    device, the update runs through iso_update, and the result is copied back
+    into pinned host memory."""
+
+    def __init__(self, theta_0_host, update_host, device="cuda"):
+        self.dev = torch.device(device)
+        self.theta_0 = [torch.empty(t.shape, dtype=t.dtype, device=self.dev) for t in theta_0_host]
+        self.update = [torch.empty(t.shape, dtype=t.dtype, device=self.dev) for t in update_host]
+        self.out = [torch.empty(t.shape, dtype=t.dtype, device=self.dev) for t in theta_0_host]
+        self.out_host = [torch.empty(t.shape, dtype=t.dtype, pin_memory=True) for t in theta_0_host]
+        self.h2d_bytes = sum(t.numel() * t.element_size() for t in list(theta_0_host) + list(update_host))
+        self.d2h_bytes = sum(t.numel() * t.element_size() for t in self.out_host)
+
+    def run(self, theta_0_host, update_host, **kw):
+        for d, h in zip(self.theta_0, theta_0_host):
+            d.copy_(h, non_blocking=True)
+        for d, h in zip(self.update, update_host):
+            d.copy_(h, non_blocking=True)
+        iso_update(self.theta_0, self.update, out=self.out, **kw)
+        for h, d in zip(self.out_host, self.out):
+            h.copy_(d, non_blocking=True)
+        return self.out_host
+
+
+def launch_count() -> int:
+    return int(lib().iso_launch_count())
+
+
+def profile_enable(on=True):
+    check(lib().iso_profile_enable(int(bool(on))), "iso_profile_enable")
+
+
+def profile_reset():
+    check(lib().iso_profile_reset(), "iso_profile_reset")
+
+
+def profile_read():
+    """{kernel kind: (launches, total ms)} since the last reset."""
+    res = {}
+    for k in range(lib().iso_profile_kinds()):
+        n, ms = ctypes.c_int64(0), ctypes.c_double(0.0)
+        check(lib().iso_profile_read(k, ctypes.byref(n), ctypes.byref(ms)), "iso_profile_read")
+        if n.value:
+            res[lib().iso_profile_name(k).decode()] = (int(n.value), float(ms.value))
+    return res

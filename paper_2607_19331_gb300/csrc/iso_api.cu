@@ -1,0 +1,778 @@
+// iso_api.cu -- host side of the C ABI declared in include/iso.h.
+//
+// Responsibilities: argument validation, the workspace layout, splitting a
+// tensor list into groups that fit the caller's workspace, building the
+// per-group tables (uploaded through kernel parameters), and the launch
+// sequence.  No device memory is allocated here.
+#include <algorithm>
+#include <atomic>
+#include <cmath>
+#include <cstring>
+#include <mutex>
+#include <unordered_map>
+#include <vector>
+
+#include "iso_kernels.cuh"
+
+namespace iso {
+namespace {
+
+// ---------------------------------------------------------------------------
+// profiling and launch accounting
+// ---------------------------------------------------------------------------
+enum Kind {
+    KD_UPLOAD, KD_INIT, KD_SAMPLE, KD_COUNT, KD_DECIDE, KD_RADIX_HIST, KD_RADIX_PICK, KD_TIE,
+    KD_CUT, KD_BLOCK_SELECT, KD_GRAM, KD_SOLVE, KD_APPLY, KD_MASK, KD_DELTA, KD_STATUS, KD_MEMSET,
+    KD_COUNT_KINDS
+};
+const char* kKindNames[KD_COUNT_KINDS] = {
+    "upload", "init_units", "sample", "count", "decide", "radix_hist", "radix_pick", "tie",
+    "cut", "block_select", "gram", "solve", "apply", "mask", "delta", "status", "memset"};
+
+std::atomic<uint64_t> g_launches{0};
+
+struct Prof {
+    bool on = false;
+    static constexpr int CAP = 16384;
+    std::vector<cudaEvent_t> ev;     // 2 per slot
+    std::vector<int> kind;
+    int used = 0;
+} g_prof;
+std::mutex g_prof_mu;
+
+struct ProfScope {
+    int slot = -1;
+    cudaStream_t s;
+    ProfScope(int kind, cudaStream_t st) : s(st) {
+        if (!g_prof.on) return;
+        std::lock_guard<std::mutex> lk(g_prof_mu);
+        if (g_prof.used >= Prof::CAP) return;
+        slot = g_prof.used;
+        if ((int)g_prof.ev.size() < 2 * (slot + 1)) {
+            cudaEvent_t a, b;
+            if (cudaEventCreate(&a) != cudaSuccess) { slot = -1; return; }
+            if (cudaEventCreate(&b) != cudaSuccess) { cudaEventDestroy(a); slot = -1; return; }
+            g_prof.ev.push_back(a);
+            g_prof.ev.push_back(b);
+            g_prof.kind.push_back(kind);
+        } else {
+            g_prof.kind[slot] = kind;
+        }
+        g_prof.used++;
+        cudaEventRecord(g_prof.ev[2 * slot], s);
+    }
+    ~ProfScope() {
+        if (slot >= 0) cudaEventRecord(g_prof.ev[2 * slot + 1], s);
+    }
+};
+
+// Launch a kernel; returns ISO_ERR_CUDA if the launch was rejected.
+template <typename F>
+int launch(int kind, cudaStream_t s, F&& f) {
+    {
+        ProfScope ps(kind, s);
+        f();
+    }
+    if (kind != KD_MEMSET) g_launches.fetch_add(1, std::memory_order_relaxed);
+    return (cudaGetLastError() == cudaSuccess) ? ISO_OK : ISO_ERR_CUDA;
+}
+
+#define ISO_TRY(x) do { int _r = (x); if (_r != ISO_OK) return _r; } while (0)
+
+// ---------------------------------------------------------------------------
+// device properties (cached per device)
+// ---------------------------------------------------------------------------
+struct DevInfo { int sms = 0; bool smem_set = false; };
+std::mutex g_dev_mu;
+std::unordered_map<int, DevInfo> g_dev;
+
+int dev_sms(int* sms) {
+    int d = 0;
+    if (cudaGetDevice(&d) != cudaSuccess) return ISO_ERR_CUDA;
+    std::lock_guard<std::mutex> lk(g_dev_mu);
+    DevInfo& di = g_dev[d];
+    if (di.sms == 0) {
+        if (cudaDeviceGetAttribute(&di.sms, cudaDevAttrMultiProcessorCount, d) != cudaSuccess)
+            return ISO_ERR_CUDA;
+    }
+    *sms = di.sms;
+    return ISO_OK;
+}
+
+// Large dynamic shared memory must be opted into once per kernel and device.
+template <typename K>
+int smem_optin(K kernel, int bytes) {
+    int d = 0;
+    if (cudaGetDevice(&d) != cudaSuccess) return ISO_ERR_CUDA;
+    static std::mutex mu;
+    static std::unordered_map<long long, bool> done;
+    const long long key = ((long long)d << 48) ^ (long long)(uintptr_t)(const void*)kernel;
+    std::lock_guard<std::mutex> lk(mu);
+    if (done.count(key)) return ISO_OK;
+    if (cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes) != cudaSuccess)
+        return ISO_ERR_CUDA;
+    done[key] = true;
+    return ISO_OK;
+}
+
+// ---------------------------------------------------------------------------
+// validation
+// ---------------------------------------------------------------------------
+bool aligned16(const void* p) { return ((uintptr_t)p & 15u) == 0; }
+
+long long numel_of(const iso_tensor& t) { return t.rows * t.cols; }
+
+int check_tensor(const iso_tensor& t) {
+    if (t.rows < 0 || t.cols < 0) return ISO_ERR_SHAPE;
+    if (t.dtype != ISO_BF16 && t.dtype != ISO_F32) return ISO_ERR_DTYPE;
+    if (t.is_1d != 0 && t.is_1d != 1) return ISO_ERR_ARG;
+    if (t.rows > 0 && t.cols > (long long)1 << 40) return ISO_ERR_SHAPE;
+    const long long n = numel_of(t);
+    if (n >= (1LL << 32)) return ISO_ERR_UNSUPPORTED;
+    if (n > 0 && t.data == nullptr) return ISO_ERR_ARG;
+    if (n > 0 && !aligned16(t.data)) return ISO_ERR_ALIGN;
+    return ISO_OK;
+}
+
+bool same_shape(const iso_tensor& a, const iso_tensor& b) { return a.rows == b.rows && a.cols == b.cols; }
+
+int check_topk(const iso_topk_cfg& c) {
+    if (!(c.density >= 0.0 && c.density <= 1.0)) return ISO_ERR_ARG;
+    if (c.scope < ISO_SCOPE_TENSOR || c.scope > ISO_SCOPE_GLOBAL) return ISO_ERR_ARG;
+    if (c.reserved != 0) return ISO_ERR_ARG;
+    if (c.scope == ISO_SCOPE_BLOCK) {
+        if (c.block_rows < 1 || c.block_rows > 256) return ISO_ERR_ARG;
+        if (c.block_cols < 8 || c.block_cols > 256 || (c.block_cols % 8) != 0) return ISO_ERR_ARG;
+        if ((long long)c.block_rows * c.block_cols > BLOCK_MAX_ENTRIES) return ISO_ERR_UNSUPPORTED;
+    }
+    return ISO_OK;
+}
+
+int check_merge_cfg(const iso_merge_cfg& c) {
+    if (c.op < ISO_OP_TA || c.op > ISO_OP_ISO) return ISO_ERR_ARG;
+    if (c.mask_1d != 0 && c.mask_1d != 1) return ISO_ERR_ARG;
+    if (!std::isfinite(c.lambda) || c.reserved != 0.0f) return ISO_ERR_ARG;
+    if (!std::isfinite(c.ridge) || c.ridge < 0.0) return ISO_ERR_ARG;
+    if (!std::isfinite(c.c_min) || !std::isfinite(c.c_max) || c.c_min > c.c_max) return ISO_ERR_ARG;
+    if (c.op != ISO_OP_TA) return check_topk(c.topk);
+    return ISO_OK;
+}
+
+// ---------------------------------------------------------------------------
+// a call, described once
+// ---------------------------------------------------------------------------
+struct Call {
+    const iso_tensor* base = nullptr;     // [n] theta_0 (nullptr for mask-only calls)
+    const iso_tensor* x = nullptr;        // [K * n] experts / task vectors
+    const iso_tensor* out = nullptr;      // [n] or nullptr
+    uint32_t* const* masks = nullptr;     // mask-only calls
+    int n = 0, K = 1;
+    bool ckpt = false;
+    int op = ISO_OP_TIES;
+    bool mask_only = false;
+    bool mask_1d = true;
+    float lambda = 1.0f;
+    double ridge = 1e-12, c_min = 0.0, c_max = 1.5;
+    iso_topk_cfg topk{};
+    bool trims = true;                    // some tensor is trimmed
+    std::vector<char> trim;               // per tensor
+    int xdt = ISO_F32, bdt = ISO_F32;
+};
+
+bool tensor_trimmed(const Call& c, int t) { return c.trim[t] != 0; }
+
+long long tiles_of(long long n) { return (n + TILE - 1) / TILE; }
+
+long long blocks_of(const iso_tensor& t, const iso_topk_cfg& c) {
+    if (t.rows == 0 || t.cols == 0) return 0;
+    return ((t.rows + c.block_rows - 1) / c.block_rows) * ((t.cols + c.block_cols - 1) / c.block_cols);
+}
+
+// candidate capacity of one unit of n entries at density rho
+unsigned long long cand_cap_of(long long n, double rho) {
+    if (n <= SAMPLE_MAX) return 0;    // the sample is the whole unit: the band is exact
+    double kk = std::floor(rho * (double)n + 0.5);
+    kk = std::min(std::max(kk, 0.0), (double)n);
+    const double q = kk / (double)n;
+    const double S = SAMPLE_MAX;
+    const double band = 2.0 * (SAMPLE_Z * std::sqrt(S * q * (1.0 - q)) + 2.0) / S;
+    const double cap = 8192.0 + std::ceil((2.0 * band + 0.002) * (double)n);
+    return (unsigned long long)std::min(cap, (double)n);
+}
+
+size_t al256(size_t v) { return (v + 255) & ~(size_t)255; }
+
+struct Layout {
+    size_t hdr, units, trec, tcnt, hist, gram, coef, zero_end;
+    size_t tens, xptr, mptr, table_end;
+    size_t cand, total;
+    long long n_tiles = 0;
+    int n_units = 0;
+    unsigned long long cand_total = 0;
+    long long global_n = 0;
+};
+
+// Layout of the workspace for tensors [t0, t1).
+Layout layout_of(const Call& c, int t0, int t1) {
+    Layout L;
+    const int T = t1 - t0;
+    const int K = c.K;
+    const int scope = c.topk.scope;
+    long long tiles = 0, units = 0, gn = 0;
+    unsigned long long cand = 0;
+    for (int t = t0; t < t1; ++t) {
+        const iso_tensor& d = c.x[t];
+        const long long n = numel_of(d);
+        tiles += tiles_of(n);
+        if (scope == ISO_SCOPE_BLOCK) units += blocks_of(d, c.topk);
+        if (tensor_trimmed(c, t)) {
+            gn += n;
+            if (scope == ISO_SCOPE_TENSOR) cand += (unsigned long long)K * cand_cap_of(n, c.topk.density);
+        }
+    }
+    if (scope == ISO_SCOPE_TENSOR) units = T;
+    if (scope == ISO_SCOPE_GLOBAL) {
+        units = 1;
+        cand = (unsigned long long)K * cand_cap_of(gn, c.topk.density);
+    }
+    const bool select = c.trims;
+    L.n_tiles = tiles;
+    L.n_units = (int)units;
+    L.cand_total = select ? cand : 0;
+    L.global_n = gn;
+    size_t o = 0;
+    L.hdr = o;   o = al256(o + sizeof(Header));
+    L.units = o; o = al256(o + (size_t)K * units * sizeof(Unit));
+    L.trec = o;  o = al256(o + (select && scope != ISO_SCOPE_BLOCK ? (size_t)K * tiles * sizeof(TileRec) : 0));
+    L.tcnt = o;  o = al256(o + (select && scope != ISO_SCOPE_BLOCK ? (size_t)K * tiles * 4 : 0));
+    L.hist = o;  o = al256(o + (select && scope != ISO_SCOPE_BLOCK ? (size_t)K * units * RADIX_BINS * 4 : 0));
+    L.gram = o;  o = al256(o + (size_t)T * K * K * 8);
+    L.coef = o;  o = al256(o + (size_t)T * K * 8);
+    L.zero_end = o;
+    L.tens = o;  o = al256(o + (size_t)T * sizeof(TensorDesc));
+    L.xptr = o;  o = al256(o + (size_t)K * T * sizeof(void*));
+    L.mptr = o;  o = al256(o + (size_t)T * sizeof(void*));
+    L.table_end = o;
+    L.cand = o;  o = al256(o + (size_t)L.cand_total * 4);
+    L.total = o;
+    return L;
+}
+
+// Split [0, n) into groups whose layout fits `ws` bytes (or one group when
+// the scope spans every tensor).
+int plan_groups(const Call& c, size_t ws, std::vector<int>* bounds) {
+    bounds->clear();
+    bounds->push_back(0);
+    if (c.n == 0) return ISO_OK;
+    if (c.topk.scope == ISO_SCOPE_GLOBAL && c.trims) {
+        if (layout_of(c, 0, c.n).total > ws) return ISO_ERR_WORKSPACE;
+        bounds->push_back(c.n);
+        return ISO_OK;
+    }
+    int t0 = 0;
+    while (t0 < c.n) {
+        if (layout_of(c, t0, t0 + 1).total > ws) return ISO_ERR_WORKSPACE;
+        // grow the group while it fits (doubling, then bisection)
+        int good = t0 + 1, step = 1;
+        while (good < c.n) {
+            const int cand = std::min(c.n, good + step);
+            if (layout_of(c, t0, cand).total <= ws) { good = cand; step *= 2; }
+            else if (step == 1) break;
+            else step = 1;
+        }
+        bounds->push_back(good);
+        t0 = good;
+    }
+    return ISO_OK;
+}
+
+// ---------------------------------------------------------------------------
+// dtype dispatch: F is a generic lambda taking (XT*, BT*, bool_constant<CK>)
+// ---------------------------------------------------------------------------
+template <bool V> struct BoolC { static constexpr bool value = V; };
+
+template <typename F>
+int dispatch_src(int xdt, int bdt, bool ckpt, F&& f) {
+    using B = __nv_bfloat16;
+    if (xdt == ISO_BF16 && bdt == ISO_BF16) return ckpt ? f((B*)0, (B*)0, BoolC<true>()) : f((B*)0, (B*)0, BoolC<false>());
+    if (xdt == ISO_BF16 && bdt == ISO_F32) return ckpt ? f((B*)0, (float*)0, BoolC<true>()) : f((B*)0, (float*)0, BoolC<false>());
+    if (xdt == ISO_F32 && bdt == ISO_BF16) return ckpt ? f((float*)0, (B*)0, BoolC<true>()) : f((float*)0, (B*)0, BoolC<false>());
+    return ckpt ? f((float*)0, (float*)0, BoolC<true>()) : f((float*)0, (float*)0, BoolC<false>());
+}
+
+int upload(cudaStream_t s, char* dst_dev, const std::vector<char>& blob) {
+    size_t off = 0;
+    while (off < blob.size()) {
+        UploadChunk ch;
+        const size_t nb = std::min((size_t)UPLOAD_BYTES, blob.size() - off);
+        ch.dst = (unsigned long long)(uintptr_t)(dst_dev + off);
+        ch.nbytes = (uint32_t)((nb + 15) & ~(size_t)15);
+        ch.pad = 0;
+        std::memset(ch.data, 0, sizeof(ch.data));
+        std::memcpy(ch.data, blob.data() + off, nb);
+        ISO_TRY(launch(KD_UPLOAD, s, [&] { k_upload<<<1, 256, 0, s>>>(ch); }));
+        off += nb;
+    }
+    return ISO_OK;
+}
+
+// ---------------------------------------------------------------------------
+// one group
+// ---------------------------------------------------------------------------
+int run_group(const Call& c, int t0, int t1, char* ws, cudaStream_t s, const iso_merge_stats* st,
+              long long units_stride, int unit_base_global) {
+    const Layout L = layout_of(c, t0, t1);
+    const int T = t1 - t0;
+    const int K = c.K;
+    int sms = 0;
+    ISO_TRY(dev_sms(&sms));
+
+    // tables
+    std::vector<char> blob(L.table_end - L.tens, 0);
+    TensorDesc* tens = reinterpret_cast<TensorDesc*>(blob.data());
+    const void** xptr = reinterpret_cast<const void**>(blob.data() + (L.xptr - L.tens));
+    uint32_t** mptr = reinterpret_cast<uint32_t**>(blob.data() + (L.mptr - L.tens));
+    long long tile = 0, uoff = 0;
+    int unit = 0;
+    unsigned long long cand = 0;
+    for (int q = 0; q < T; ++q) {
+        const int t = t0 + q;
+        const iso_tensor& xt = c.x[t];
+        TensorDesc& d = tens[q];
+        d.base = c.base ? c.base[t].data : nullptr;
+        d.out = c.out ? c.out[t].data : nullptr;
+        d.numel = numel_of(xt);
+        d.rows = xt.rows;
+        d.cols = xt.cols;
+        d.tile_base = tile;
+        tile += tiles_of(d.numel);
+        d.flags = (xt.is_1d ? TF_1D : 0) | (tensor_trimmed(c, t) ? TF_TRIM : 0);
+        d.uoff = uoff;
+        if (tensor_trimmed(c, t)) uoff += d.numel;
+        if (c.topk.scope == ISO_SCOPE_BLOCK) {
+            d.unit = unit;
+            d.bpr = (int)((xt.cols + c.topk.block_cols - 1) / c.topk.block_cols);
+            d.nblocks = (int)blocks_of(xt, c.topk);
+            unit += d.nblocks;
+        } else {
+            d.unit = (c.topk.scope == ISO_SCOPE_GLOBAL) ? 0 : q;
+            d.bpr = 0;
+            d.nblocks = 0;
+        }
+        if (c.topk.scope == ISO_SCOPE_TENSOR) {
+            const unsigned long long cap = tensor_trimmed(c, t) ? cand_cap_of(d.numel, c.topk.density) : 0;
+            d.cand_off = cand;
+            d.cand_cap = cap;
+            cand += (unsigned long long)K * cap;
+        } else {
+            d.cand_off = 0;
+            d.cand_cap = (c.topk.scope == ISO_SCOPE_GLOBAL) ? cand_cap_of(L.global_n, c.topk.density) : 0;
+        }
+        for (int i = 0; i < K; ++i) xptr[i * T + q] = c.x[(size_t)i * c.n + t].data;
+        mptr[q] = c.masks ? c.masks[t] : nullptr;
+    }
+
+    Plan P;
+    std::memset(&P, 0, sizeof(P));
+    P.hdr = reinterpret_cast<Header*>(ws + L.hdr);
+    P.tens = reinterpret_cast<TensorDesc*>(ws + L.tens);
+    P.xptr = reinterpret_cast<const void**>(ws + L.xptr);
+    P.units = reinterpret_cast<Unit*>(ws + L.units);
+    P.trec = reinterpret_cast<TileRec*>(ws + L.trec);
+    P.tcnt = reinterpret_cast<uint32_t*>(ws + L.tcnt);
+    P.hist = reinterpret_cast<uint32_t*>(ws + L.hist);
+    P.cand = reinterpret_cast<uint32_t*>(ws + L.cand);
+    P.gram = reinterpret_cast<double*>(ws + L.gram);
+    P.coef = reinterpret_cast<double*>(ws + L.coef);
+    P.n_tensors = T;
+    P.K = K;
+    P.n_units = L.n_units;
+    P.scope = c.topk.scope;
+    P.n_tiles = L.n_tiles;
+    P.xdt = c.xdt;
+    P.bdt = c.bdt;
+    P.ckpt = c.ckpt ? 1 : 0;
+    P.op = c.mask_only ? ISO_OP_TIES : c.op;
+    P.block_rows = c.topk.block_rows;
+    P.block_cols = c.topk.block_cols;
+    P.lambda = c.lambda;
+    P.density = c.topk.density;
+    P.ridge = c.ridge;
+    P.c_min = c.c_min;
+    P.c_max = c.c_max;
+    P.st_units = st ? st->units : nullptr;
+    P.st_units_stride = units_stride;
+    P.st_unit_base = unit_base_global;
+    P.st_tensor_base = t0;
+    P.st_gram = st ? st->gram : nullptr;
+    P.st_coef = st ? st->coef : nullptr;
+
+    // zero the per-group state (the status word at offset 0 persists across groups)
+    ISO_TRY(launch(KD_MEMSET, s, [&] { cudaMemsetAsync(ws + 4, 0, L.zero_end - 4, s); }));
+    ISO_TRY(upload(s, ws + L.tens, blob));
+
+    const int pgrid = sms * 4;
+    const bool select = c.trims && (c.mask_only || c.op != ISO_OP_TA);
+    int gram_mode = GRAM_NONE;
+    if (!c.mask_only && c.op == ISO_OP_ISO) {
+        if (K == 1 && c.topk.scope == ISO_SCOPE_TENSOR) gram_mode = GRAM_UNIT;
+        else gram_mode = GRAM_ACCUM;
+    }
+    const bool need_gram_pass = gram_mode == GRAM_ACCUM && !(K == 1 && c.topk.scope == ISO_SCOPE_BLOCK);
+    const int KU = K * L.n_units;
+
+    int rc = ISO_OK;
+    if (select && c.topk.scope != ISO_SCOPE_BLOCK) {
+        ISO_TRY(launch(KD_INIT, s, [&] { k_init_units<<<(KU + 255) / 256, 256, 0, s>>>(P, L.global_n); }));
+        rc = dispatch_src(c.xdt, c.bdt, c.ckpt, [&](auto* xt, auto* bt, auto ck) -> int {
+            using XT = std::remove_pointer_t<decltype(xt)>;
+            using BT = std::remove_pointer_t<decltype(bt)>;
+            constexpr bool CK = decltype(ck)::value;
+            const int smem = (SAMPLE_MAX + RADIX_BINS) * 4;
+            ISO_TRY(smem_optin(k_sample<XT, BT, CK>, smem));
+            ISO_TRY(launch(KD_SAMPLE, s, [&] { k_sample<XT, BT, CK><<<KU, SAMPLE_TPB, smem, s>>>(P); }));
+            ISO_TRY(launch(KD_COUNT, s, [&] { k_count<XT, BT, CK><<<pgrid, TPB, 0, s>>>(P); }));
+            ISO_TRY(launch(KD_DECIDE, s, [&] { k_decide<<<(KU + 255) / 256, 256, 0, s>>>(P); }));
+            for (int level = 0; level < 3; ++level) {
+                ISO_TRY(launch(KD_RADIX_HIST, s, [&] { k_radix_hist<XT, BT, CK><<<pgrid, TPB, 0, s>>>(P); }));
+                ISO_TRY(launch(KD_RADIX_PICK, s, [&] { k_radix_pick<<<KU, TPB, 0, s>>>(P); }));
+            }
+            ISO_TRY(launch(KD_TIE, s, [&] { k_tie<XT, BT, CK><<<pgrid, TPB, 0, s>>>(P); }));
+            ISO_TRY(launch(KD_CUT, s, [&] { k_cut<XT, BT, CK><<<KU, TPB, 0, s>>>(P); }));
+            return ISO_OK;
+        });
+        ISO_TRY(rc);
+    } else if (select) {
+        rc = dispatch_src(c.xdt, c.bdt, c.ckpt, [&](auto* xt, auto* bt, auto ck) -> int {
+            using XT = std::remove_pointer_t<decltype(xt)>;
+            using BT = std::remove_pointer_t<decltype(bt)>;
+            constexpr bool CK = decltype(ck)::value;
+            const int smem = BLOCK_MAX_ENTRIES * 4;
+            ISO_TRY(smem_optin(k_block_select<XT, BT, CK>, smem));
+            if (KU > 0)
+                ISO_TRY(launch(KD_BLOCK_SELECT, s, [&] { k_block_select<XT, BT, CK><<<KU, BLOCK_TPB, smem, s>>>(P); }));
+            return ISO_OK;
+        });
+        ISO_TRY(rc);
+    }
+
+    if (c.mask_only) {
+        uint32_t* const* mdev = reinterpret_cast<uint32_t* const*>(ws + L.mptr);
+        if (c.xdt == ISO_BF16)
+            ISO_TRY(launch(KD_MASK, s, [&] { k_mask<__nv_bfloat16><<<pgrid, TPB, 0, s>>>(P, mdev); }));
+        else
+            ISO_TRY(launch(KD_MASK, s, [&] { k_mask<float><<<pgrid, TPB, 0, s>>>(P, mdev); }));
+        return ISO_OK;
+    }
+
+    rc = dispatch_src(c.xdt, c.bdt, c.ckpt, [&](auto* xt, auto* bt, auto ck) -> int {
+        using XT = std::remove_pointer_t<decltype(xt)>;
+        using BT = std::remove_pointer_t<decltype(bt)>;
+        constexpr bool CK = decltype(ck)::value;
+        if (gram_mode != GRAM_NONE) {
+            if (need_gram_pass)
+                ISO_TRY(launch(KD_GRAM, s, [&] { k_gram<XT, BT, CK><<<pgrid, TPB, 0, s>>>(P); }));
+            ISO_TRY(launch(KD_SOLVE, s, [&] { k_solve<<<(T + 127) / 128, 128, 0, s>>>(P, gram_mode); }));
+        }
+        if (K == 1)
+            ISO_TRY(launch(KD_APPLY, s, [&] { k_apply<XT, BT, CK, 1><<<pgrid, TPB, 0, s>>>(P); }));
+        else
+            ISO_TRY(launch(KD_APPLY, s, [&] { k_apply<XT, BT, CK, 0><<<pgrid, TPB, 0, s>>>(P); }));
+        return ISO_OK;
+    });
+    return rc;
+}
+
+// ---------------------------------------------------------------------------
+// shared driver for update / merge / mask
+// ---------------------------------------------------------------------------
+int units_per_expert(const iso_tensor* tens, int n, const iso_topk_cfg& c, long long* out) {
+    long long u = 0;
+    if (c.scope == ISO_SCOPE_TENSOR) u = n;
+    else if (c.scope == ISO_SCOPE_GLOBAL) u = 1;
+    else for (int t = 0; t < n; ++t) u += blocks_of(tens[t], c);
+    *out = u;
+    return ISO_OK;
+}
+
+int run_call(Call& c, void* workspace, size_t ws_bytes, const iso_merge_stats* st, cudaStream_t s) {
+    if (c.n > 0) {
+        if (!workspace) return ISO_ERR_WORKSPACE;
+        if (((uintptr_t)workspace & 255u) != 0) return ISO_ERR_WORKSPACE;
+    }
+    std::vector<int> bounds;
+    ISO_TRY(plan_groups(c, ws_bytes, &bounds));
+    char* ws = static_cast<char*>(workspace);
+    if (c.n > 0) ISO_TRY(launch(KD_MEMSET, s, [&] { cudaMemsetAsync(ws, 0, 4, s); }));
+    long long stride = 0;
+    units_per_expert(c.x, c.n, c.topk, &stride);
+    int unit_base = 0;
+    for (size_t g = 0; g + 1 < bounds.size(); ++g) {
+        const int t0 = bounds[g], t1 = bounds[g + 1];
+        ISO_TRY(run_group(c, t0, t1, ws, s, st, stride, unit_base));
+        if (c.topk.scope == ISO_SCOPE_BLOCK)
+            for (int t = t0; t < t1; ++t) unit_base += (int)blocks_of(c.x[t], c.topk);
+        else if (c.topk.scope == ISO_SCOPE_TENSOR)
+            unit_base += t1 - t0;
+    }
+    if (st && st->status) {
+        if (c.n > 0)
+            ISO_TRY(launch(KD_STATUS, s, [&] { k_status<<<1, 32, 0, s>>>(reinterpret_cast<const Header*>(ws), st->status); }));
+        else
+            ISO_TRY(launch(KD_MEMSET, s, [&] { cudaMemsetAsync(st->status, 0, 4, s); }));
+    }
+    return ISO_OK;
+}
+
+void set_trim(Call& c, const iso_tensor* tens) {
+    c.trim.assign(c.n, 0);
+    c.trims = false;
+    for (int t = 0; t < c.n; ++t) {
+        bool tr;
+        if (c.mask_only) tr = true;
+        else if (c.op == ISO_OP_TA) tr = false;
+        else if (c.op == ISO_OP_TIES) tr = c.mask_1d || !tens[t].is_1d;
+        else tr = !tens[t].is_1d;
+        c.trim[t] = tr ? 1 : 0;
+        c.trims |= tr && numel_of(tens[t]) > 0;
+    }
+}
+
+int build_merge_call(Call& c, const iso_tensor* theta_0, const iso_tensor* experts, int K,
+                     int experts_are_deltas, const iso_tensor* out, int n, const iso_merge_cfg* cfg) {
+    if (n < 0 || K < 1) return ISO_ERR_ARG;
+    if (K > ISO_MAX_EXPERTS) return ISO_ERR_UNSUPPORTED;
+    if (!cfg) return ISO_ERR_ARG;
+    if (n > 0 && (!theta_0 || !experts || !out)) return ISO_ERR_ARG;
+    if (experts_are_deltas != 0 && experts_are_deltas != 1) return ISO_ERR_ARG;
+    ISO_TRY(check_merge_cfg(*cfg));
+    for (int t = 0; t < n; ++t) {
+        ISO_TRY(check_tensor(theta_0[t]));
+        ISO_TRY(check_tensor(out[t]));
+        if (!same_shape(theta_0[t], out[t])) return ISO_ERR_SHAPE;
+        if (out[t].dtype != theta_0[t].dtype) return ISO_ERR_DTYPE;
+        if (theta_0[t].dtype != theta_0[0].dtype) return ISO_ERR_DTYPE;
+        if (out[t].is_1d != theta_0[t].is_1d) return ISO_ERR_SHAPE;
+        for (int i = 0; i < K; ++i) {
+            const iso_tensor& x = experts[(size_t)i * n + t];
+            ISO_TRY(check_tensor(x));
+            if (!same_shape(x, theta_0[t])) return ISO_ERR_SHAPE;
+            if (x.dtype != experts[0].dtype) return ISO_ERR_DTYPE;
+            if (numel_of(x) > 0 && x.data == out[t].data) return ISO_ERR_ARG;   // out may alias the base only
+        }
+    }
+    c.base = theta_0;
+    c.x = experts;
+    c.out = out;
+    c.n = n;
+    c.K = K;
+    c.ckpt = experts_are_deltas == 0;
+    c.op = cfg->op;
+    c.mask_1d = cfg->mask_1d != 0;
+    c.lambda = cfg->lambda;
+    c.ridge = cfg->ridge;
+    c.c_min = cfg->c_min;
+    c.c_max = cfg->c_max;
+    c.topk = cfg->topk;
+    if (c.op == ISO_OP_TA) { c.topk.scope = ISO_SCOPE_TENSOR; c.topk.density = 1.0; }
+    c.xdt = n > 0 ? experts[0].dtype : ISO_F32;
+    c.bdt = n > 0 ? theta_0[0].dtype : ISO_F32;
+    set_trim(c, theta_0);
+    return ISO_OK;
+}
+
+}  // namespace
+}  // namespace iso
+
+// ===========================================================================
+// C ABI
+// ===========================================================================
+using namespace iso;
+
+extern "C" {
+
+int32_t iso_num_units(const iso_tensor* tensors, int32_t n_tensors, const iso_topk_cfg* topk,
+                      int64_t* n_units) {
+    if (!topk || !n_units || n_tensors < 0 || (n_tensors > 0 && !tensors)) return ISO_ERR_ARG;
+    ISO_TRY(check_topk(*topk));
+    for (int t = 0; t < n_tensors; ++t)
+        if (tensors[t].rows < 0 || tensors[t].cols < 0) return ISO_ERR_SHAPE;
+    long long u = 0;
+    units_per_expert(tensors, n_tensors, *topk, &u);
+    *n_units = u;
+    return ISO_OK;
+}
+
+int32_t iso_workspace_size(const iso_tensor* tensors, int32_t n_tensors, int32_t K,
+                           const iso_merge_cfg* cfg, size_t* bytes_min, size_t* bytes_full) {
+    if (!cfg || n_tensors < 0 || (n_tensors > 0 && !tensors) || K < 1) return ISO_ERR_ARG;
+    if (K > ISO_MAX_EXPERTS) return ISO_ERR_UNSUPPORTED;
+    ISO_TRY(check_merge_cfg(*cfg));
+    for (int t = 0; t < n_tensors; ++t) {
+        if (tensors[t].rows < 0 || tensors[t].cols < 0) return ISO_ERR_SHAPE;
+        if (numel_of(tensors[t]) >= (1LL << 32)) return ISO_ERR_UNSUPPORTED;
+    }
+    Call c;
+    std::vector<iso_tensor> xs((size_t)K * n_tensors);
+    for (int i = 0; i < K; ++i)
+        for (int t = 0; t < n_tensors; ++t) xs[(size_t)i * n_tensors + t] = tensors[t];
+    c.x = xs.data();
+    c.n = n_tensors;
+    c.K = K;
+    c.op = cfg->op;
+    c.mask_1d = cfg->mask_1d != 0;
+    c.topk = cfg->topk;
+    if (c.op == ISO_OP_TA) { c.topk.scope = ISO_SCOPE_TENSOR; c.topk.density = 1.0; }
+    set_trim(c, tensors);
+    size_t full = n_tensors ? layout_of(c, 0, n_tensors).total : 256;
+    size_t mn = 256;
+    if (c.topk.scope == ISO_SCOPE_GLOBAL && c.trims) mn = full;
+    else for (int t = 0; t < n_tensors; ++t) mn = std::max(mn, layout_of(c, t, t + 1).total);
+    if (bytes_min) *bytes_min = mn;
+    if (bytes_full) *bytes_full = std::max(full, mn);
+    return ISO_OK;
+}
+
+int32_t iso_delta(const iso_tensor* theta_i, const iso_tensor* theta_0, const iso_tensor* tau,
+                  int32_t n_tensors, void* stream) {
+    if (n_tensors < 0) return ISO_ERR_ARG;
+    if (n_tensors == 0) return ISO_OK;
+    if (!theta_i || !theta_0 || !tau) return ISO_ERR_ARG;
+    for (int t = 0; t < n_tensors; ++t) {
+        ISO_TRY(check_tensor(theta_i[t]));
+        ISO_TRY(check_tensor(theta_0[t]));
+        ISO_TRY(check_tensor(tau[t]));
+        if (!same_shape(theta_i[t], theta_0[t]) || !same_shape(tau[t], theta_0[t])) return ISO_ERR_SHAPE;
+        if (tau[t].dtype != ISO_F32) return ISO_ERR_DTYPE;
+        if (theta_i[t].dtype != theta_i[0].dtype || theta_0[t].dtype != theta_0[0].dtype) return ISO_ERR_DTYPE;
+        if (numel_of(tau[t]) > 0 && (tau[t].data == theta_i[t].data || tau[t].data == theta_0[t].data))
+            return ISO_ERR_ARG;
+    }
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    int sms = 0;
+    ISO_TRY(dev_sms(&sms));
+    for (int t0 = 0; t0 < n_tensors; t0 += DELTA_MAXT) {
+        DeltaArgs A;
+        std::memset(&A, 0, sizeof(A));
+        A.n = std::min(DELTA_MAXT, n_tensors - t0);
+        long long tile = 0;
+        for (int q = 0; q < A.n; ++q) {
+            const int t = t0 + q;
+            A.tile_base[q] = tile;
+            A.numel[q] = numel_of(theta_0[t]);
+            tile += tiles_of(A.numel[q]);
+            A.a[q] = theta_i[t].data;
+            A.b[q] = theta_0[t].data;
+            A.out[q] = static_cast<float*>(tau[t].data);
+        }
+        A.tile_base[A.n] = tile;
+        if (tile == 0) continue;
+        const int grid = (int)std::min<long long>(tile, (long long)sms * 4);
+        const int adt = theta_i[0].dtype, bdt = theta_0[0].dtype;
+        using B = __nv_bfloat16;
+        if (adt == ISO_BF16 && bdt == ISO_BF16) ISO_TRY(launch(KD_DELTA, s, [&] { k_delta<B, B><<<grid, TPB, 0, s>>>(A); }));
+        else if (adt == ISO_BF16) ISO_TRY(launch(KD_DELTA, s, [&] { k_delta<B, float><<<grid, TPB, 0, s>>>(A); }));
+        else if (bdt == ISO_BF16) ISO_TRY(launch(KD_DELTA, s, [&] { k_delta<float, B><<<grid, TPB, 0, s>>>(A); }));
+        else ISO_TRY(launch(KD_DELTA, s, [&] { k_delta<float, float><<<grid, TPB, 0, s>>>(A); }));
+    }
+    return ISO_OK;
+}
+
+int32_t iso_topk_mask(const iso_tensor* tau, int32_t n_tensors, const iso_topk_cfg* cfg,
+                      uint32_t* const* mask_bits, const iso_merge_stats* stats,
+                      void* workspace, size_t ws_bytes, void* stream) {
+    if (n_tensors < 0 || !cfg || (n_tensors > 0 && !tau)) return ISO_ERR_ARG;
+    ISO_TRY(check_topk(*cfg));
+    for (int t = 0; t < n_tensors; ++t) {
+        ISO_TRY(check_tensor(tau[t]));
+        if (tau[t].dtype != tau[0].dtype) return ISO_ERR_DTYPE;
+        if (mask_bits && mask_bits[t] && !aligned16(mask_bits[t])) return ISO_ERR_ALIGN;
+    }
+    Call c;
+    c.x = tau;
+    c.n = n_tensors;
+    c.K = 1;
+    c.ckpt = false;
+    c.mask_only = true;
+    c.masks = mask_bits;
+    c.topk = *cfg;
+    c.xdt = n_tensors ? tau[0].dtype : ISO_F32;
+    c.bdt = c.xdt;
+    set_trim(c, tau);
+    std::vector<uint32_t*> mvec;
+    if (!mask_bits) { mvec.assign(n_tensors, nullptr); c.masks = mvec.data(); }
+    return run_call(c, workspace, ws_bytes, stats, static_cast<cudaStream_t>(stream));
+}
+
+int32_t iso_update(const iso_tensor* theta_0, const iso_tensor* update, int32_t update_is_delta,
+                   const iso_tensor* out, int32_t n_tensors, const iso_merge_cfg* cfg,
+                   void* workspace, size_t ws_bytes, const iso_merge_stats* stats, void* stream) {
+    Call c;
+    ISO_TRY(build_merge_call(c, theta_0, update, 1, update_is_delta, out, n_tensors, cfg));
+    return run_call(c, workspace, ws_bytes, stats, static_cast<cudaStream_t>(stream));
+}
+
+int32_t iso_merge(const iso_tensor* theta_0, const iso_tensor* experts, int32_t K,
+                  int32_t experts_are_deltas, const iso_tensor* out, int32_t n_tensors,
+                  const iso_merge_cfg* cfg, void* workspace, size_t ws_bytes,
+                  const iso_merge_stats* stats, void* stream) {
+    Call c;
+    ISO_TRY(build_merge_call(c, theta_0, experts, K, experts_are_deltas, out, n_tensors, cfg));
+    return run_call(c, workspace, ws_bytes, stats, static_cast<cudaStream_t>(stream));
+}
+
+const char* iso_error_string(int32_t status) {
+    switch (status) {
+        case ISO_OK: return "ISO_OK: success";
+        case ISO_ERR_ARG: return "ISO_ERR_ARG: invalid argument";
+        case ISO_ERR_SHAPE: return "ISO_ERR_SHAPE: tensor shapes disagree";
+        case ISO_ERR_DTYPE: return "ISO_ERR_DTYPE: unsupported or mismatched dtype";
+        case ISO_ERR_ALIGN: return "ISO_ERR_ALIGN: data pointer not 16-byte aligned";
+        case ISO_ERR_WORKSPACE: return "ISO_ERR_WORKSPACE: workspace missing, misaligned or too small";
+        case ISO_ERR_CUDA: return "ISO_ERR_CUDA: a CUDA launch or runtime call failed";
+        case ISO_ERR_NONFINITE: return "ISO_ERR_NONFINITE: an input held NaN or Inf";
+        case ISO_ERR_UNSUPPORTED: return "ISO_ERR_UNSUPPORTED: request outside this build's limits";
+        default: return "unknown iso_status";
+    }
+}
+
+uint64_t iso_launch_count(void) { return g_launches.load(); }
+
+int32_t iso_profile_enable(int32_t on) {
+    std::lock_guard<std::mutex> lk(g_prof_mu);
+    g_prof.on = on != 0;
+    return ISO_OK;
+}
+
+int32_t iso_profile_reset(void) {
+    std::lock_guard<std::mutex> lk(g_prof_mu);
+    g_prof.used = 0;
+    return ISO_OK;
+}
+
+int32_t iso_profile_kinds(void) { return KD_COUNT_KINDS; }
+
+const char* iso_profile_name(int32_t kind) {
+    if (kind < 0 || kind >= KD_COUNT_KINDS) return "";
+    return kKindNames[kind];
+}
+
+int32_t iso_profile_read(int32_t kind, int64_t* launches, double* total_ms) {
+    if (kind < 0 || kind >= KD_COUNT_KINDS || !launches || !total_ms) return ISO_ERR_ARG;
+    std::lock_guard<std::mutex> lk(g_prof_mu);
+    long long n = 0;
+    double ms = 0.0;
+    for (int q = 0; q < g_prof.used; ++q) {
+        if (g_prof.kind[q] != kind) continue;
+        if (cudaEventSynchronize(g_prof.ev[2 * q + 1]) != cudaSuccess) return ISO_ERR_CUDA;
+        float f = 0.0f;
+        if (cudaEventElapsedTime(&f, g_prof.ev[2 * q], g_prof.ev[2 * q + 1]) != cudaSuccess) return ISO_ERR_CUDA;
+        ms += f;
+        ++n;
+    }
+    *launches = n;
+    *total_ms = ms;
+    return ISO_OK;
+}
+
+}  // extern "C"

@@ -1,0 +1,202 @@
+// iso_block.cu -- TopKMask with per-block thresholds (BLOCK scope).
+//
+// Each unit is one block_rows x block_cols tile of a row-major tensor, in
+// row-major tile order; entries inside a tile keep the tensor's own index
+// order, so "lowest index first" among equal |tau| is the tile's row-major
+// order.  One CTA holds a whole unit on chip: it loads the unit's keys into
+// shared memory, finds the k-th largest key by an 11/11/9-bit radix select,
+// and resolves the ties by an ordered block scan.  The result (t, cut) feeds
+// the same streaming apply pass as the other scopes.
+#include "iso_kernels.cuh"
+
+namespace iso {
+
+__device__ __forceinline__ long long k_of_density_b(double rho, long long n) {
+    double kk = floor(__dadd_rn(__dmul_rn(rho, (double)n), 0.5));
+    if (kk < 0.0) kk = 0.0;
+    if (kk > (double)n) kk = (double)n;
+    return (long long)kk;
+}
+
+__device__ void block_find_from_top_b(const uint32_t* hist, int nb, long long rank,
+                                      long long* sm_scan, int* res_bin, long long* res_above) {
+    const int per = (nb + blockDim.x - 1) / blockDim.x;
+    const int j0 = threadIdx.x * per;
+    if (threadIdx.x == 0) { *res_bin = 0; *res_above = 0; }
+    long long local = 0;
+    for (int j = j0; j < j0 + per && j < nb; ++j) local += hist[nb - 1 - j];
+    long long total;
+    const long long excl = block_excl_scan(local, sm_scan, &total);
+    if (excl < rank && rank <= excl + local) {
+        long long acc = excl;
+        for (int j = j0; j < j0 + per && j < nb; ++j) {
+            const uint32_t h = hist[nb - 1 - j];
+            if (rank <= acc + h) { *res_bin = nb - 1 - j; *res_above = acc; break; }
+            acc += h;
+        }
+    }
+    __syncthreads();
+}
+
+template <typename XT, typename BT, bool CK>
+__global__ void __launch_bounds__(BLOCK_TPB) k_block_select(Plan P) {
+    extern __shared__ __align__(16) uint32_t s_keys[];      // BLOCK_MAX_ENTRIES
+    __shared__ uint32_t s_hist[RADIX_BINS];
+    __shared__ long long s_scan[33];
+    __shared__ uint32_t s_scan32[33];
+    __shared__ double s_dred[33];
+    __shared__ int s_bin;
+    __shared__ long long s_above;
+    __shared__ long long s_cutq;
+
+    const int idx = blockIdx.x;
+    const int i = idx / P.n_units, u = idx % P.n_units;
+    // owning tensor: last tensor whose first unit is <= u and that has blocks
+    int lo = 0, hi = P.n_tensors - 1;
+    while (lo < hi) {
+        const int mid = (lo + hi + 1) >> 1;
+        if (P.tens[mid].unit <= u) lo = mid; else hi = mid - 1;
+    }
+    while (lo > 0 && P.tens[lo].nblocks == 0) --lo;
+    const int t = lo;
+    const TensorDesc& d = P.tens[t];
+    Unit& U = P.units[idx];
+    const int b = u - d.unit;
+    const int br = b / d.bpr, bc = b % d.bpr;
+    const long long r0 = (long long)br * P.block_rows, c0 = (long long)bc * P.block_cols;
+    const long long h = min((long long)P.block_rows, d.rows - r0);
+    const long long w = min((long long)P.block_cols, d.cols - c0);
+    const int n = (int)(h * w);
+    auto stats = [&](uint32_t tk, long long k, long long above, long long ties, long long need) {
+        if (!P.st_units) return;
+        iso_unit_stats s;
+        s.thresh_key = tk; s.flags = 0; s.k = k; s.count_above = above;
+        s.ties_at_thresh = ties; s.ties_taken = need;
+        P.st_units[(long long)i * P.st_units_stride + P.st_unit_base + u] = s;
+    };
+    if (!(d.flags & TF_TRIM)) {
+        if (threadIdx.x == 0) {
+            U.state = ST_OFF; U.k = -1; U.t = 0; U.cut = CUT_ALL;
+            stats(KEY_NONE, -1, 0, 0, 0);
+        }
+        return;
+    }
+    const long long k = k_of_density_b(P.density, n);
+    if (k == 0) {
+        if (threadIdx.x == 0) {
+            U.state = ST_NONE; U.k = 0; U.t = KEY_NONE; U.cut = 0;
+            stats(KEY_NONE, 0, 0, 0, 0);
+        }
+        return;
+    }
+    const void* x = P.xptr[i * P.n_tensors + t];
+    // keys in block order (row-major inside the block)
+    bool bad = false;
+    const bool vec = (w % VEC == 0) && (d.cols % VEC == 0) && (c0 % VEC == 0);
+    if (vec) {
+        const int w8 = (int)(w / VEC);
+        for (int q8 = threadIdx.x; q8 < n / VEC; q8 += blockDim.x) {
+            const int rr = q8 / w8, cc = (q8 - rr * w8) * VEC;
+            const long long e = (r0 + rr) * d.cols + c0 + cc;
+            float tau[VEC];
+            TauSrc<XT, BT, CK>::load8(x, d.base, e, d.numel, tau);
+#pragma unroll
+            for (int j = 0; j < VEC; ++j) {
+                const uint32_t kk = key_of(tau[j]);
+                bad |= kk >= KEY_INF;
+                s_keys[q8 * VEC + j] = kk;
+            }
+        }
+    } else {
+        for (int q = threadIdx.x; q < n; q += blockDim.x) {
+            const int rr = q / (int)w, cc = q - rr * (int)w;
+            const long long e = (r0 + rr) * d.cols + c0 + cc;
+            const uint32_t kk = key_of(TauSrc<XT, BT, CK>::load1(x, d.base, e));
+            bad |= kk >= KEY_INF;
+            s_keys[q] = kk;
+        }
+    }
+    if (bad) set_status(P.hdr, ISO_ERR_NONFINITE);
+    __syncthreads();
+    // k-th largest key
+    uint32_t prefix = 0;
+    long long rank = k;
+    int pshift = 31;
+    for (;;) {
+        const int shift = pshift > RADIX_BITS ? pshift - RADIX_BITS : 0;
+        const int nb = 1 << (pshift - shift);
+        for (int q = threadIdx.x; q < nb; q += blockDim.x) s_hist[q] = 0;
+        __syncthreads();
+        for (int q = threadIdx.x; q < n; q += blockDim.x) {
+            const uint32_t v = s_keys[q];
+            if ((v >> pshift) == prefix) atomicAdd(&s_hist[(v >> shift) & (nb - 1)], 1u);
+        }
+        __syncthreads();
+        block_find_from_top_b(s_hist, nb, rank, s_scan, &s_bin, &s_above);
+        rank -= s_above;
+        prefix = (prefix << (pshift - shift)) | (uint32_t)s_bin;
+        __syncthreads();
+        if (shift == 0) break;
+        pshift = shift;
+    }
+    const uint32_t tk = prefix;
+    // counts above / at the threshold, and the squared norm of the kept entries
+    const int per = (n + blockDim.x - 1) / blockDim.x;
+    const int q0 = threadIdx.x * per;
+    uint32_t above = 0, ties = 0;
+    double gsum = 0.0;
+    for (int q = q0; q < q0 + per && q < n; ++q) {
+        const uint32_t v = s_keys[q];
+        if (v > tk) {
+            above++;
+            const double f = (double)__uint_as_float(v);
+            gsum += f * f;
+        } else if (v == tk) {
+            ties++;
+        }
+    }
+    uint32_t tot_ties;
+    const uint32_t ties_before = block_excl_scan(ties, s_scan32, &tot_ties);
+    const uint32_t tot_above = block_sum(above, s_scan32);
+    const long long need = k - (long long)tot_above;
+    if (threadIdx.x == 0) s_cutq = -1;
+    __syncthreads();
+    if (need < (long long)tot_ties) {
+        if ((long long)ties_before < need && need <= (long long)(ties_before + ties)) {
+            uint32_t acc = ties_before;
+            for (int q = q0; q < q0 + per && q < n; ++q)
+                if (s_keys[q] == tk && (long long)(++acc) == need) { s_cutq = q; break; }
+        }
+    }
+    __syncthreads();
+    const bool want_gamma = (P.op == ISO_OP_ISO) && (P.K == 1);
+    double g = 0.0;
+    if (want_gamma) g = block_sum(gsum, s_dred);
+    if (threadIdx.x == 0) {
+        long long cut = CUT_ALL;
+        if (s_cutq >= 0) {
+            const long long rr = s_cutq / w, cc = s_cutq - rr * w;
+            cut = (r0 + rr) * d.cols + c0 + cc + 1;
+        }
+        U.n = n; U.k = k; U.t = tk; U.cut = cut;
+        U.count_above = tot_above; U.ties = tot_ties; U.need = need;
+        U.state = ST_DONE;
+        if (want_gamma) {
+            const double ft = (double)__uint_as_float(tk);
+            atomicAdd(&P.gram[t], g + (double)need * ft * ft);
+        }
+        stats(tk, k, tot_above, tot_ties, need);
+    }
+}
+
+#define ISO_BLOCK_INST(XT, BT, CK) template __global__ void k_block_select<XT, BT, CK>(Plan);
+ISO_BLOCK_INST(__nv_bfloat16, __nv_bfloat16, false)
+ISO_BLOCK_INST(__nv_bfloat16, float, false)
+ISO_BLOCK_INST(float, __nv_bfloat16, false)
+ISO_BLOCK_INST(float, float, false)
+ISO_BLOCK_INST(__nv_bfloat16, __nv_bfloat16, true)
+ISO_BLOCK_INST(__nv_bfloat16, float, true)
+ISO_BLOCK_INST(float, __nv_bfloat16, true)
+ISO_BLOCK_INST(float, float, true)
+
+}  // namespace iso

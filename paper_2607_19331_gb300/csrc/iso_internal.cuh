@@ -1,0 +1,291 @@
+// iso_internal.cuh -- device-side data structures and helpers shared by the
+// kernels of the GB300 delta-merge library.
+//
+// Element-wise path (App. F of the paper for TopKMask / TA / TIES; Sec. 4.2,
+// App. E and Algorithm 1 for the retention combiner):
+//   tau   = theta_i - theta_0          (binary32, one subtraction)
+//   key   = bits(|tau|)                (binary32 pattern, sign cleared: monotone in |tau|)
+//   mask  = key > t || (key == t && index < cut)   per selection unit
+#pragma once
+
+#include <cuda_runtime.h>
+#include <cuda_bf16.h>
+#include <stdint.h>
+
+#include "iso.h"
+
+namespace iso {
+
+// ---------------------------------------------------------------------------
+// geometry
+// ---------------------------------------------------------------------------
+constexpr int TILE = 8192;                  // entries per streaming tile
+constexpr int TPB = 256;                    // threads per streaming block
+constexpr int VEC = 8;                      // entries per thread per vector step
+constexpr int NVEC = TILE / (TPB * VEC);    // vector steps per tile (4)
+static_assert(NVEC * TPB * VEC == TILE, "tile geometry");
+
+constexpr int SAMPLE_MAX = 32768;           // sampled keys per unit (128 KB of smem)
+constexpr int SAMPLE_CHUNK = 256;           // contiguous entries per sample chunk
+constexpr int SAMPLE_TPB = 1024;
+constexpr double SAMPLE_Z = 5.0;            // band half-width in sample standard deviations
+
+constexpr int RADIX_BITS = 11;
+constexpr int RADIX_BINS = 1 << RADIX_BITS;
+constexpr int BLOCK_MAX_ENTRIES = 16384;    // BLOCK scope: entries per unit held on chip
+
+constexpr uint32_t KEY_NONE = 0xFFFFFFFFu;  // threshold of a unit that selects nothing
+constexpr uint32_t KEY_MAX = 0x7FFFFFFFu;   // largest key
+constexpr uint32_t KEY_INF = 0x7F800000u;   // keys >= this are not finite
+constexpr long long CUT_ALL = 0x7FFFFFFFFFFFFFFFLL;
+
+// ---------------------------------------------------------------------------
+// tables (in the caller's workspace)
+// ---------------------------------------------------------------------------
+enum TensorFlags : int32_t { TF_1D = 1, TF_TRIM = 2 };
+
+struct TensorDesc {
+    const void* base;        // theta_0 (or tau for iso_topk_mask)
+    void*       out;         // merged output (NULL for mask-only calls)
+    long long   numel;
+    long long   uoff;        // GLOBAL scope: position of entry 0 in the unit order
+    long long   tile_base;   // first tile id (group-local)
+    long long   rows, cols;
+    int32_t     flags;
+    int32_t     unit;        // TENSOR: this tensor's unit; BLOCK: first block unit
+    int32_t     bpr;         // BLOCK: blocks per block row
+    int32_t     nblocks;     // BLOCK: blocks in this tensor
+    unsigned long long cand_off;  // TENSOR: expert 0's candidate segment (expert i adds i*cand_cap)
+    unsigned long long cand_cap;
+};
+
+enum UnitState : int32_t {
+    ST_OFF = 0,      // not trimmed: every entry is kept
+    ST_NONE = 1,     // k == 0: nothing is kept
+    ST_SAMPLE = 2,   // waiting for the band
+    ST_BAND = 3,     // band set; the count pass fills the counters
+    ST_RADIX = 4,    // exact select in progress (interior candidates or full data)
+    ST_TKNOWN = 5,   // threshold known; cut pending
+    ST_DONE = 6
+};
+enum TieSource : int32_t { TIE_EQ_HI = 0, TIE_EQ_LO = 1, TIE_ARRAY = 2 };
+enum RadixSource : int32_t { SRC_CAND = 0, SRC_DATA = 1 };
+
+struct Unit {
+    // static
+    long long n, k;
+    long long tile_begin, tile_end;     // group-local tiles covering the unit
+    unsigned long long cand_off, cand_cap;
+    int32_t tensor;                     // TENSOR / BLOCK: owning tensor; GLOBAL: -1
+    int32_t expert;
+    int32_t state;
+    int32_t want_gamma;                 // accumulate sum of squares of the kept entries
+    // band
+    uint32_t lo, hi;
+    // count-pass accumulators
+    unsigned long long c_gt, c_hi, c_lo, n_int;
+    double gamma_acc;                   // sum tau^2 over key > hi (count pass)
+    double gamma_acc2;                  // sum tau^2 over the radix source above t
+    // radix select
+    int32_t r_src;
+    int32_t r_shift, r_pshift;
+    uint32_t r_base;                    // key offset: lo for candidates, 0 for data
+    uint32_t r_prefix;
+    int32_t fallback;
+    long long r_rank;                   // rank (1-based, from the top) inside the current set
+    long long r_above;                  // entries above the current set
+    // result
+    uint32_t t;
+    int32_t tie_src;
+    long long count_above, ties, need;
+    long long cut;                      // kept iff key > t || (key == t && pos < cut)
+    double gamma;
+};
+
+struct TileRec {            // per (expert, tile) record of the count pass
+    uint32_t start;         // first interior slot in the unit's candidate segment
+    uint32_t count;         // interior keys stored (0 when the segment overflowed)
+    uint32_t eq_lo;         // keys == lo in this tile
+    uint32_t eq_hi;         // keys == hi in this tile
+};
+
+struct Header {             // first bytes of the workspace
+    int32_t status;
+    int32_t n_radix;        // units in ST_RADIX after the last pick
+    int32_t n_tknown;
+    int32_t pad;
+};
+
+// Everything a kernel needs to find its tables.
+struct Plan {
+    Header*       hdr;
+    TensorDesc*   tens;
+    const void**  xptr;     // [K][n_tensors] expert data
+    Unit*         units;    // [K][n_units]
+    TileRec*      trec;     // [K][n_tiles]
+    uint32_t*     tcnt;     // [K][n_tiles] ties at t per tile
+    uint32_t*     hist;     // [K * n_units][RADIX_BINS]
+    uint32_t*     cand;     // candidate pool
+    double*       gram;     // [n_tensors][K][K]
+    double*       coef;     // [n_tensors][K]
+    int32_t n_tensors;
+    int32_t K;
+    int32_t n_units;        // per expert
+    int32_t scope;
+    long long n_tiles;
+    int32_t xdt;            // expert dtype
+    int32_t bdt;            // base dtype
+    int32_t ckpt;           // experts are checkpoints (tau = x - base)
+    int32_t op;
+    int32_t block_rows, block_cols;
+    float lambda;
+    double density, ridge, c_min, c_max;
+    // stats destinations (device, may be NULL) and the unit offset of this group
+    iso_unit_stats* st_units;
+    long long st_units_stride;          // units per expert in the caller's array
+    int32_t st_unit_base;               // this group's first unit in the caller's array
+    int32_t st_tensor_base;             // this group's first tensor
+    double* st_gram;
+    double* st_coef;
+};
+
+// ---------------------------------------------------------------------------
+// element access
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ float bf16_bits_to_f32(uint32_t b16) {
+    return __uint_as_float(b16 << 16);
+}
+__device__ __forceinline__ uint32_t key_of(float tau) {
+    return __float_as_uint(tau) & 0x7FFFFFFFu;
+}
+
+// 8 consecutive entries (16-byte aligned start) of a tensor as binary32.
+template <typename T> struct Load8;
+template <> struct Load8<__nv_bfloat16> {
+    static __device__ __forceinline__ void run(const void* p, long long e, float (&v)[8]) {
+        uint4 u = __ldg(reinterpret_cast<const uint4*>(static_cast<const __nv_bfloat16*>(p) + e));
+        v[0] = bf16_bits_to_f32(u.x & 0xFFFFu); v[1] = bf16_bits_to_f32(u.x >> 16);
+        v[2] = bf16_bits_to_f32(u.y & 0xFFFFu); v[3] = bf16_bits_to_f32(u.y >> 16);
+        v[4] = bf16_bits_to_f32(u.z & 0xFFFFu); v[5] = bf16_bits_to_f32(u.z >> 16);
+        v[6] = bf16_bits_to_f32(u.w & 0xFFFFu); v[7] = bf16_bits_to_f32(u.w >> 16);
+    }
+    static __device__ __forceinline__ float one(const void* p, long long e) {
+        return bf16_bits_to_f32(static_cast<const unsigned short*>(p)[e]);
+    }
+};
+template <> struct Load8<float> {
+    static __device__ __forceinline__ void run(const void* p, long long e, float (&v)[8]) {
+        const float4* q = reinterpret_cast<const float4*>(static_cast<const float*>(p) + e);
+        float4 a = __ldg(q), b = __ldg(q + 1);
+        v[0] = a.x; v[1] = a.y; v[2] = a.z; v[3] = a.w;
+        v[4] = b.x; v[5] = b.y; v[6] = b.z; v[7] = b.w;
+    }
+    static __device__ __forceinline__ float one(const void* p, long long e) {
+        return static_cast<const float*>(p)[e];
+    }
+};
+
+// Task-vector source: tau = x (delta) or x - base (checkpoint), binary32.
+template <typename XT, typename BT, bool CKPT>
+struct TauSrc {
+    // 8 entries starting at e (e % 8 == 0); entries at or beyond n read as 0
+    static __device__ __forceinline__ void load8(const void* x, const void* base, long long e,
+                                                 long long n, float (&tau)[8]) {
+        if (e + 8 <= n) {
+            Load8<XT>::run(x, e, tau);
+            if (CKPT) {
+                float b[8];
+                Load8<BT>::run(base, e, b);
+#pragma unroll
+                for (int j = 0; j < 8; ++j) tau[j] = __fsub_rn(tau[j], b[j]);
+            }
+        } else {
+#pragma unroll
+            for (int j = 0; j < 8; ++j) {
+                float v = 0.0f;
+                if (e + j < n) {
+                    v = Load8<XT>::one(x, e + j);
+                    if (CKPT) v = __fsub_rn(v, Load8<BT>::one(base, e + j));
+                }
+                tau[j] = v;
+            }
+        }
+    }
+    static __device__ __forceinline__ float load1(const void* x, const void* base, long long e) {
+        float v = Load8<XT>::one(x, e);
+        if (CKPT) v = __fsub_rn(v, Load8<BT>::one(base, e));
+        return v;
+    }
+};
+
+// tile id -> tensor (binary search over tile_base)
+__device__ __forceinline__ int tensor_of_tile(const TensorDesc* tens, int n_tensors, long long tile) {
+    int lo = 0, hi = n_tensors - 1;
+    while (lo < hi) {
+        int mid = (lo + hi + 1) >> 1;
+        if (tens[mid].tile_base <= tile) lo = mid; else hi = mid - 1;
+    }
+    return lo;
+}
+
+__device__ __forceinline__ void set_status(Header* h, int32_t code) {
+    atomicCAS(&h->status, 0, code);
+}
+
+// ---------------------------------------------------------------------------
+// block-wide helpers (blockDim.x a multiple of 32, <= 1024)
+// ---------------------------------------------------------------------------
+template <typename T>
+__device__ __forceinline__ T warp_sum(T v) {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xFFFFFFFFu, v, o);
+    return v;
+}
+
+// Sum over the block; result valid in every thread.  `sm` needs 32 slots.
+template <typename T>
+__device__ __forceinline__ T block_sum(T v, T* sm) {
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    v = warp_sum(v);
+    __syncthreads();
+    if (lane == 0) sm[warp] = v;
+    __syncthreads();
+    const int nw = (blockDim.x + 31) >> 5;
+    T r = (lane < nw) ? sm[lane] : T(0);
+    r = warp_sum(r);
+    return r;
+}
+
+// Exclusive prefix over the block in thread order; *total receives the sum.
+// `sm` needs 33 slots.
+template <typename T>
+__device__ __forceinline__ T block_excl_scan(T v, T* sm, T* total) {
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    T x = v;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+        T y = __shfl_up_sync(0xFFFFFFFFu, x, o);
+        if (lane >= o) x += y;
+    }
+    __syncthreads();
+    if (lane == 31) sm[warp] = x;
+    __syncthreads();
+    if (warp == 0) {
+        const int nw = (blockDim.x + 31) >> 5;
+        T w = (lane < nw) ? sm[lane] : T(0);
+        T s = w;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            T y = __shfl_up_sync(0xFFFFFFFFu, s, o);
+            if (lane >= o) s += y;
+        }
+        if (lane < nw) sm[lane] = s - w;   // exclusive warp offsets
+        if (lane == nw - 1) sm[32] = s;
+    }
+    __syncthreads();
+    T r = sm[warp] + x - v;
+    *total = sm[32];
+    return r;
+}
+
+}  // namespace iso

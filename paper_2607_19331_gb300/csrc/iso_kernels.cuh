@@ -1,0 +1,57 @@
+// iso_kernels.cuh -- kernel declarations (definitions and explicit
+// instantiations live in iso_select.cu, iso_apply.cu and iso_block.cu).
+#pragma once
+
+#include "iso_internal.cuh"
+
+namespace iso {
+
+constexpr int MAXK = ISO_MAX_EXPERTS;
+
+// select (TENSOR / GLOBAL scope)
+__global__ void k_init_units(Plan P, long long global_n);
+template <typename XT, typename BT, bool CK> __global__ void k_sample(Plan P);
+template <typename XT, typename BT, bool CK> __global__ void k_count(Plan P);
+__global__ void k_decide(Plan P);
+template <typename XT, typename BT, bool CK> __global__ void k_radix_hist(Plan P);
+__global__ void k_radix_pick(Plan P);
+template <typename XT, typename BT, bool CK> __global__ void k_tie(Plan P);
+template <typename XT, typename BT, bool CK> __global__ void k_cut(Plan P);
+
+// select (BLOCK scope)
+constexpr int BLOCK_TPB = 512;
+template <typename XT, typename BT, bool CK> __global__ void k_block_select(Plan P);
+
+// apply
+template <typename XT, typename BT, bool CK, int KC> __global__ void k_apply(Plan P);
+template <typename XT, typename BT, bool CK> __global__ void k_gram(Plan P);
+__global__ void k_solve(Plan P, int gram_mode);
+template <typename XT> __global__ void k_mask(Plan P, uint32_t* const* mptr);
+__global__ void k_status(const Header* h, int32_t* out);
+
+// upload of host-built tables through kernel parameters (no host staging
+// buffer, capturable, ordered on the stream)
+constexpr int UPLOAD_BYTES = 16384;
+struct UploadChunk {
+    unsigned long long dst;
+    uint32_t nbytes;   // multiple of 16
+    uint32_t pad;
+    uint4 data[UPLOAD_BYTES / 16];
+};
+__global__ void k_upload(UploadChunk c);
+
+// iso_delta: tensors passed by value in chunks
+constexpr int DELTA_MAXT = 64;
+struct DeltaArgs {
+    int n;
+    long long tile_base[DELTA_MAXT + 1];
+    long long numel[DELTA_MAXT];
+    const void* a[DELTA_MAXT];
+    const void* b[DELTA_MAXT];
+    float* out[DELTA_MAXT];
+};
+template <typename AT, typename BT> __global__ void k_delta(DeltaArgs A);
+
+enum GramMode { GRAM_NONE = 0, GRAM_UNIT = 1, GRAM_ACCUM = 2 };
+
+}  // namespace iso

@@ -1,0 +1,117 @@
+"""Host-side checks of the C ABI (no GPU needed): the library loads, exports
+every entry point include/iso.h declares, and rejects bad arguments before
+anything reaches the device."""
+import ctypes
+import os
+import re
+
+import pytest
+
+import paper_2607_19331_gb300 as iso
+from paper_2607_19331_gb300 import _abi
+from paper_2607_19331_gb300._abi import IsoTensor
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _built():
+    from paper_2607_19331_gb300 import build
+    build.build()
+
+
+def _declared():
+    src = open(os.path.join(ROOT, "include", "iso.h")).read()
+    src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+    return sorted(set(re.findall(r"\b(iso_[a-z_]+)\s*\(", src)))
+
+
+def test_every_declared_symbol_is_exported():
+    names = _declared()
+    assert {"iso_delta", "iso_topk_mask", "iso_update", "iso_merge", "iso_workspace_size"} <= set(names)
+    lib = ctypes.CDLL(_abi.LIB_PATH)
+    for n in names:
+        assert hasattr(lib, n), f"{n} declared in iso.h but not exported"
+    assert {p[0] for p in _abi.PROTOTYPES} == set(names)
+
+
+def test_error_strings():
+    L = _abi.lib()
+    for code in range(0, -9, -1):
+        s = L.iso_error_string(code).decode()
+        assert s.startswith("ISO_"), s
+    assert "unknown" in L.iso_error_string(-99).decode()
+
+
+def _fake(rows, cols, dtype=_abi.ISO_BF16, ptr=0x10000, is_1d=0):
+    return IsoTensor(ptr, rows, cols, dtype, is_1d)
+
+
+def _arr(*ts):
+    a = (IsoTensor * len(ts))()
+    for i, t in enumerate(ts):
+        a[i] = t
+    return a
+
+
+def test_num_units_and_workspace():
+    L = _abi.lib()
+    ts = _arr(_fake(300, 1000), _fake(1, 1536, is_1d=1), _fake(257, 129))
+    n = ctypes.c_int64()
+    for scope, want in ((0, 3), (2, 1), (1, 3 * 8 + 12 + 3 * 2)):
+        cfg = iso.topk_cfg(0.1, ["tensor", "block", "global"][scope])
+        assert L.iso_num_units(ts, 3, ctypes.byref(cfg), ctypes.byref(n)) == 0
+        assert n.value == want, (scope, n.value)
+    mn, full = ctypes.c_size_t(), ctypes.c_size_t()
+    for op in ("ta", "ties", "iso"):
+        for scope in ("tensor", "block", "global"):
+            cfg = iso.merge_cfg(op, 0.05, scope)
+            assert L.iso_workspace_size(ts, 3, 2, ctypes.byref(cfg), ctypes.byref(mn), ctypes.byref(full)) == 0
+            assert 0 < mn.value <= full.value
+            if scope == "global" and op != "ta":
+                assert mn.value == full.value
+    cfg = iso.merge_cfg("ties", 0.05)
+    assert L.iso_workspace_size(ts, 3, 9, ctypes.byref(cfg), None, None) == _abi.ISO_ERR_UNSUPPORTED
+
+
+def test_validation_rejects_before_launch():
+    L = _abi.lib()
+    cfg = iso.merge_cfg("ties", 0.2)
+    a, b = _arr(_fake(8, 8)), _arr(_fake(8, 8, ptr=0x20000))
+    o = _arr(_fake(8, 8, ptr=0x30000))
+    ws = ctypes.c_void_p(0x40000)
+    def upd(a_, b_, o_, cfg_=cfg, ws_=ws, n=1):
+        return L.iso_update(a_, b_, 0, o_, n, ctypes.byref(cfg_) if cfg_ is not None else None,
+                            ws_, 1 << 20, None, None)
+    assert upd(a, _arr(_fake(8, 4, ptr=0x20000)), o) == _abi.ISO_ERR_SHAPE
+    assert upd(a, _arr(_fake(8, 8, ptr=0x20002)), o) == _abi.ISO_ERR_ALIGN
+    assert upd(a, _arr(_fake(8, 8, dtype=7, ptr=0x20000)), o) == _abi.ISO_ERR_DTYPE
+    assert upd(a, b, _arr(_fake(8, 8, dtype=_abi.ISO_F32, ptr=0x30000))) == _abi.ISO_ERR_DTYPE
+    assert upd(a, b, _arr(_fake(8, 8, ptr=0x20000))) == _abi.ISO_ERR_ARG        # out aliases expert
+    assert upd(a, b, o, cfg_=None) == _abi.ISO_ERR_ARG
+    assert upd(a, _arr(_fake(8, 8, ptr=0)), o) == _abi.ISO_ERR_ARG               # NULL data
+    assert upd(a, b, o, ws_=ctypes.c_void_p(0x40010)) == _abi.ISO_ERR_WORKSPACE  # misaligned
+    assert upd(a, b, o, ws_=ctypes.c_void_p(0)) == _abi.ISO_ERR_WORKSPACE
+    bad = iso.merge_cfg("ties", 0.2)
+    bad.topk.density = float("nan")
+    assert upd(a, b, o, cfg_=bad) == _abi.ISO_ERR_ARG
+    bad = iso.merge_cfg("iso", 0.2, c_min=2.0, c_max=1.0)
+    assert upd(a, b, o, cfg_=bad) == _abi.ISO_ERR_ARG
+    bad = iso.merge_cfg("ties", 0.2, "block", block=(128, 12))
+    assert upd(a, b, o, cfg_=bad) == _abi.ISO_ERR_ARG
+    bad = iso.merge_cfg("ties", 0.2, "block", block=(256, 256))
+    assert upd(a, b, o, cfg_=bad) == _abi.ISO_ERR_UNSUPPORTED
+    huge = _arr(_fake(1 << 16, 1 << 16))
+    assert upd(huge, _arr(_fake(1 << 16, 1 << 16, ptr=0x20000)), _arr(_fake(1 << 16, 1 << 16, ptr=0x30000))) \
+        == _abi.ISO_ERR_UNSUPPORTED
+    K9 = (IsoTensor * 9)(*[_fake(8, 8, ptr=0x50000 + 0x1000 * i) for i in range(9)])
+    assert L.iso_merge(a, K9, 9, 1, o, 1, ctypes.byref(cfg), ws, 1 << 20, None, None) == _abi.ISO_ERR_UNSUPPORTED
+    # an empty list is a no-op that needs no workspace and no device
+    assert L.iso_update(a, b, 0, o, 0, ctypes.byref(cfg), None, 0, None, None) == 0
+
+
+def test_missing_library_fails_loudly(monkeypatch):
+    monkeypatch.setattr(_abi, "LIB_PATH", "/nonexistent/libiso_gb300.so")
+    monkeypatch.setattr(_abi, "_lib", None)
+    with pytest.raises(RuntimeError, match="not found"):
+        _abi.lib()
