@@ -271,6 +271,9 @@ void orc_retention(int32_t K, const double* gram, double ridge, double c_min, do
 
 static int sign_f(float v) { return (v > 0.0f) - (v < 0.0f); }
 
+/* mask == NULL: the tensor is not trimmed, every entry is kept */
+static int kept(const uint8_t* const* mask, int i, int64_t p) { return mask ? mask[i][p] : 1; }
+
 /* theta = theta_0 + update; an update of exactly zero leaves theta_0 as is
  * (this keeps the sign of a -0 base weight). */
 static double add_update(double theta0, double upd) { return (upd == 0.0) ? theta0 : theta0 + upd; }
@@ -295,14 +298,14 @@ void orc_merge_tensor(int32_t op, int32_t K, int64_t n, int32_t is_1d,
         for (int64_t p = 0; p < n; ++p) {
             float s32 = 0.0f;                     /* election sum in binary32, i = 1..K */
             for (int i = 0; i < K; ++i) {
-                float tt = mask[i][p] ? tau32[i][p] : 0.0f;
+                float tt = kept(mask, i, p) ? tau32[i][p] : 0.0f;
                 s32 = s32 + tt;
             }
             int gamma = sign_f(s32);
             double acc = 0.0;
             int cnt = 0;
             for (int i = 0; i < K; ++i) {
-                if (!mask[i][p]) continue;
+                if (!kept(mask, i, p)) continue;
                 float tt = tau32[i][p];
                 if (tt != 0.0f && sign_f(tt) == gamma) { acc += tau64[i][p]; cnt++; }
             }
@@ -330,8 +333,8 @@ void orc_merge_tensor(int32_t op, int32_t K, int64_t n, int32_t is_1d,
         for (int j = i; j < K; ++j) {
             double s = 0.0;
             for (int64_t p = 0; p < n; ++p) {
-                double gi = mask[i][p] ? tau64[i][p] : 0.0;
-                double gj = mask[j][p] ? tau64[j][p] : 0.0;
+                double gi = kept(mask, i, p) ? tau64[i][p] : 0.0;
+                double gj = kept(mask, j, p) ? tau64[j][p] : 0.0;
                 s += gi * gj;
             }
             G[i * K + j] = s;
@@ -344,7 +347,7 @@ void orc_merge_tensor(int32_t op, int32_t K, int64_t n, int32_t is_1d,
     for (int64_t p = 0; p < n; ++p) {
         double s = 0.0;
         for (int i = 0; i < K; ++i)
-            if (mask[i][p]) s += c[i] * tau64[i][p];
+            if (kept(mask, i, p)) s += c[i] * tau64[i][p];
         out[p] = add_update(theta0[p], s);
     }
 }

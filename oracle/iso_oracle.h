@@ -60,7 +60,8 @@ void orc_topk_select(const float* tau32, int64_t n, int64_t k, uint8_t* mask, or
  *   op      ORC_TA / ORC_TIES / ORC_ISO
  *   tau32   K arrays, decision precision (signs, TIES election)
  *   tau64   K arrays, value precision
- *   mask    K arrays (TIES, ISO 2-D); NULL for TA and for ISO 1-D
+ *   mask    K arrays (TIES, ISO 2-D); NULL = not trimmed (TA, ISO 1-D, and TIES
+ *           tensors left untrimmed)
  *   is_1d   ISO only: 1-D parameters take the plain task-vector average
  *   out     merged values in f64
  *   gram    K*K (ISO 2-D, may be NULL), coef K (ISO 2-D, may be NULL) */

@@ -23,12 +23,12 @@ MUTATIONS = {
     "ties_disagreeing_set": ("if (tt != 0.0f && sign_f(tt) == gamma)", "if (tt != 0.0f && sign_f(tt) != gamma)"),
     "ties_plain_mean": ("double merged = cnt ? acc / (double)cnt : 0.0;",
                         "double merged = cnt ? acc / (double)K : 0.0;"),
-    "ties_untrimmed_election": ("float tt = mask[i][p] ? tau32[i][p] : 0.0f;", "float tt = tau32[i][p];"),
+    "ties_untrimmed_election": ("float tt = kept(mask, i, p) ? tau32[i][p] : 0.0f;", "float tt = tau32[i][p];"),
     "ta_drops_lambda": ("out[p] = add_update(theta0[p], lambda * s);", "out[p] = add_update(theta0[p], s);"),
     "retention_rhs_ones": ("b[r] = gram[idx[r] * K + idx[r]];", "b[r] = 1.0;"),
     "retention_no_clip": ("if (c > c_max) c = c_max;", ";"),
     "gram_diagonal_only": ("s += gi * gj;", "s += gi * gi;"),
-    "gram_untrimmed": ("double gi = mask[i][p] ? tau64[i][p] : 0.0;", "double gi = tau64[i][p];"),
+    "gram_untrimmed": ("double gi = kept(mask, i, p) ? tau64[i][p] : 0.0;", "double gi = tau64[i][p];"),
     "iso_1d_no_average": ("out[p] = add_update(theta0[p], s / (double)K);", "out[p] = add_update(theta0[p], s);"),
     "bf16_round_half_up": ("u += 0x7FFFu + lsb;", "u += 0x8000u;"),
     "bf16_f64_truncates": ("double q = round_half_even(ldexp(a, -q_exp));", "double q = floor(ldexp(a, -q_exp));"),

@@ -393,3 +393,15 @@ def test_ties_election_uses_trimmed_vectors():
     r = oracle.merge([th0], [[t1], [t2]], oracle.TIES, density=0.5, lam=1.0, is_1d=[False])
     assert r["out64"][0][0] == -0.5
     assert r["out64"][0][1] == 5.0
+
+
+def test_ties_untrimmed_tensor_keeps_every_entry():
+    # mask_1d = 0: a 1-D tensor enters TIES untrimmed (m_i = 1 everywhere); with
+    # K = 1 the merge is then theta_0 + lambda tau on every entry.
+    rng = np.random.default_rng(13)
+    th0 = rng.normal(0, 0.02, 64).astype(np.float32)
+    tau = rng.normal(0, 1e-3, 64).astype(np.float32)
+    r = oracle.merge([th0], [[tau]], oracle.TIES, density=0.1, lam=1.0, mask_1d=False, is_1d=[True])
+    np.testing.assert_array_equal(r["out64"][0], th0.astype(np.float64) + tau.astype(np.float64))
+    r = oracle.merge([th0], [[tau]], oracle.TIES, density=0.1, lam=1.0, mask_1d=True, is_1d=[True])
+    assert (r["out64"][0] != th0.astype(np.float64)).sum() == oracle.k_of(0.1, 64)
