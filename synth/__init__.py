@@ -79,7 +79,8 @@ def laplace_(x: torch.Tensor, rate: float, b: float, gen: torch.Generator) -> to
     """Replace a Bernoulli(rate) subset of x by Laplace(0, b) draws."""
     pick = torch.rand(x.numel(), generator=gen, device=x.device) < rate
     u = torch.rand(x.numel(), generator=gen, device=x.device) - 0.5
-    lap = -b * torch.sign(u) * torch.log1p(-2.0 * u.abs())
+    # keep 2|u| < 1 so the inverse CDF stays finite (rand may return exactly 0)
+    lap = -b * torch.sign(u) * torch.log1p(-(2.0 * u.abs()).clamp(max=1.0 - 2.0 ** -24))
     x[pick] = lap[pick]
     return x
 
