@@ -221,6 +221,8 @@ def topk_masks(tau32_list, shapes, density, scope=SCOPE_TENSOR, block=(128, 128)
         return row
 
     if scope == SCOPE_GLOBAL:
+        if not any(participate):
+            return masks, np.array([skipped_row()], UNIT_STATS_DTYPE)
         parts = [np.asarray(tau32_list[t], np.float32).ravel() for t in range(n_t) if participate[t]]
         cat = np.concatenate(parts) if parts else np.zeros(0, np.float32)
         m, row = topk_unit(cat, k_of(density, cat.size), method)
@@ -307,7 +309,7 @@ def merge(theta0, experts, op, *, experts_are_deltas=True, density=0.2,
 
     masks = [None] * K
     units = []
-    if any(participate):
+    if op != TA:   # every trimming operator reports one row per unit (k = -1: not trimmed)
         for i in range(K):
             masks[i], st = topk_masks(tau32[i], shapes, density, scope, block, method, participate)
             units.append(st)

@@ -307,5 +307,7 @@ def test_full_size_qwen15b_update_sampled():
                           oracle.ISO, update_is_delta=False, density=0.05, is_1d=[shapes[q][2]])
         assert_values_close(to_np(out[q]), r["out64"][0], r["mag"][0], f"full-size tensor {q}")
         assert_units_equal(units[q:q + 1], r["units"][0], f"full-size unit {q}")
+        if shapes[q][2]:
+            assert units[q]["k"] == -1      # 1-D tensors take the ISO average, untrimmed
     del th0, th1, out
     torch.cuda.empty_cache()
