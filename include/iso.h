@@ -191,6 +191,31 @@ int32_t iso_merge(const iso_tensor* theta_0, const iso_tensor* experts, int32_t 
                   const iso_merge_cfg* cfg, void* workspace, size_t ws_bytes,
                   const iso_merge_stats* stats, void* stream);
 
+/* iso_update without a caller workspace.  Some callers cannot allocate device
+ * memory where they run the update (an inference-engine plugin whose enqueue
+ * path may not call cudaMalloc, a server that freezes its allocator after
+ * warm-up, a C host without a device allocator); this entry point serves them.
+ * The paper has no counterpart: it is a property of this library's interface.
+ *
+ * Arguments and results are those of iso_update.  Scratch comes from one
+ * static device array of ISO_NOALLOC_SCRATCH_BYTES per device, part of the
+ * library's module image and held until the process exits; nothing is
+ * allocated or freed.  Tensors are processed in groups that fit the array; a
+ * call whose smallest group (one tensor) needs more returns
+ * ISO_ERR_WORKSPACE before anything is enqueued.
+ *   - The first call on a device looks the array's device address up
+ *     (cudaGetSymbolAddress, with that device current) and caches it: make
+ *     that first call before any stream capture.
+ *   - Every call on a device shares the one array, which keeps the last
+ *     call's contents; each call clears what it needs zeroed.  Calls whose
+ *     work overlaps on the GPU (different streams, or different host threads
+ *     without ordering) race on the array and give undefined results: order
+ *     them on one stream. */
+#define ISO_NOALLOC_SCRATCH_BYTES (32u << 20)
+int32_t iso_update_noalloc(const iso_tensor* theta_0, const iso_tensor* update, int32_t update_is_delta,
+                           const iso_tensor* out, int32_t n_tensors, const iso_merge_cfg* cfg,
+                           const iso_merge_stats* stats, void* stream);
+
 /* Static description of a status code. */
 const char* iso_error_string(int32_t status);
 

@@ -22,6 +22,7 @@ ISO_ERR_CUDA = -6
 ISO_ERR_NONFINITE = -7
 ISO_ERR_UNSUPPORTED = -8
 ISO_MAX_EXPERTS = 8
+ISO_NOALLOC_SCRATCH_BYTES = 32 << 20
 
 ISO_BF16, ISO_F32 = 0, 1
 ISO_SCOPE_TENSOR, ISO_SCOPE_BLOCK, ISO_SCOPE_GLOBAL = 0, 1, 2
@@ -71,6 +72,8 @@ PROTOTYPES = [
                          ctypes.POINTER(IsoMergeStats), P]),
     ("iso_merge", I32, [PT, PT, I32, I32, PT, I32, ctypes.POINTER(IsoMergeCfg), P, SZ,
                         ctypes.POINTER(IsoMergeStats), P]),
+    ("iso_update_noalloc", I32, [PT, PT, I32, PT, I32, ctypes.POINTER(IsoMergeCfg),
+                                 ctypes.POINTER(IsoMergeStats), P]),
     ("iso_error_string", ctypes.c_char_p, [I32]),
     ("iso_launch_count", ctypes.c_uint64, []),
     ("iso_profile_enable", I32, [I32]),

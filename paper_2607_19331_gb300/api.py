@@ -265,3 +265,23 @@ def profile_read():
         if n.value:
             res[lib().iso_profile_name(k).decode()] = (int(n.value), float(ms.value))
     return res
+
+
+def iso_update_noalloc(theta_0: List[torch.Tensor], update: List[torch.Tensor], op="iso",
+                       update_is_delta=False, out=None, density=0.05, scope="tensor",
+                       block=(128, 128), lam=1.0, ridge=1e-12, c_min=0.0, c_max=1.5,
+                       mask_1d=True, stats=False, stream=None):
+    """iso_update for callers that cannot allocate device memory: the library
+    runs the update in its own fixed per-device scratch (no workspace
+    argument).  Make the first call on a device before any stream capture;
+    calls that overlap on the GPU race on the shared scratch."""
+    dev = theta_0[0].device
+    if out is None:
+        out = [torch.empty_like(t) for t in theta_0]
+    cfg = merge_cfg(op, density, scope, block, lam, ridge, c_min, c_max, mask_1d)
+    st = make_stats(theta_0, 1, cfg.topk, dev) if stats else None
+    check(lib().iso_update_noalloc(describe(theta_0), describe(update), int(bool(update_is_delta)),
+                                   describe(out), len(theta_0), ctypes.byref(cfg),
+                                   ctypes.byref(st.abi()) if st else None, _stream(stream)),
+          "iso_update_noalloc")
+    return (out, st) if stats else out

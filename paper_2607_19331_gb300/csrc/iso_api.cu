@@ -776,3 +776,58 @@ int32_t iso_profile_read(int32_t kind, int64_t* launches, double* total_ms) {
 }
 
 }  // extern "C"
+
+// ===========================================================================
+// iso_update_noalloc: iso_update on the library's own fixed scratch
+// ===========================================================================
+// Some callers cannot hand the library a workspace: an inference-engine plugin
+// whose enqueue path may not call cudaMalloc, a serving process that freezes
+// its allocator after warm-up, or a C host without a device allocator of its
+// own.  For them the library keeps one fixed scratch array per device in
+// static device memory (ISO_NOALLOC_SCRATCH_BYTES, loaded with the module and
+// held until the process exits) and runs the same update through it.
+namespace iso {
+namespace {
+
+constexpr size_t NOALLOC_SCRATCH_BYTES = (size_t)ISO_NOALLOC_SCRATCH_BYTES;
+
+static __device__ __align__(256) unsigned char g_noalloc_scratch[NOALLOC_SCRATCH_BYTES];
+
+// Device address of the scratch on the current device.  Looked up once per
+// device (with that device current) and cached; the host-side name of the
+// array is only a stand-in and is never passed to a kernel.
+int noalloc_scratch(void** out) {
+    int d = 0;
+    if (cudaGetDevice(&d) != cudaSuccess) return ISO_ERR_CUDA;
+    static std::mutex mu;
+    static std::unordered_map<int, void*> ptrs;
+    std::lock_guard<std::mutex> lk(mu);
+    auto it = ptrs.find(d);
+    if (it != ptrs.end()) { *out = it->second; return ISO_OK; }
+    void* p = nullptr;
+    if (cudaGetSymbolAddress(&p, g_noalloc_scratch) != cudaSuccess || p == nullptr) return ISO_ERR_CUDA;
+    ptrs[d] = p;
+    *out = p;
+    return ISO_OK;
+}
+
+}  // namespace
+}  // namespace iso
+
+extern "C" int32_t iso_update_noalloc(const iso_tensor* theta_0, const iso_tensor* update,
+                                      int32_t update_is_delta, const iso_tensor* out,
+                                      int32_t n_tensors, const iso_merge_cfg* cfg,
+                                      const iso_merge_stats* stats, void* stream) {
+    Call c;
+    ISO_TRY(build_merge_call(c, theta_0, update, 1, update_is_delta, out, n_tensors, cfg));
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    if (n_tensors == 0) return run_call(c, nullptr, 0, stats, s);
+    // reject requests the fixed scratch cannot hold before touching the device
+    std::vector<int> bounds;
+    ISO_TRY(plan_groups(c, NOALLOC_SCRATCH_BYTES, &bounds));
+    void* ws = nullptr;
+    ISO_TRY(noalloc_scratch(&ws));
+    // run_call clears the scratch's status word and every per-group counter
+    // region it uses before the group's kernels run
+    return run_call(c, ws, NOALLOC_SCRATCH_BYTES, stats, s);
+}
