@@ -111,11 +111,11 @@ class Clocks:
                 "reasons": reasons, "samples": len(rows)}
 
 
-def make_workload(name, device, seed):
+def make_workload(name, device, seed, layers=None):
     import torch
     import synth
     shapes_name, K, op, inputs, density, desc = WORKLOADS[name]
-    shapes = synth.qwen_shapes(shapes_name)
+    shapes = synth.qwen_shapes(shapes_name, layers=layers)
     if inputs == "ckpt_bf16":
         th0, th1 = synth.rl_update_set(shapes, seed=seed, device=device)
         experts = [th1]
@@ -140,7 +140,7 @@ def run_mine(args):
     dev = torch.device("cuda", local)
     name = args.workload
     shapes_name, K, op, inputs, density, desc = WORKLOADS[name]
-    shapes, th0, experts = make_workload(name, dev, seed=rank)
+    shapes, th0, experts = make_workload(name, dev, seed=rank, layers=args.layers)
     n_params = sum(t.numel() for t in th0)
     ckpt = inputs == "ckpt_bf16"
     out = [torch.empty_like(t) for t in th0]
@@ -238,7 +238,8 @@ def run_mine(args):
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms, 4),
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
             "dtype": "bf16" if ckpt else "f32", "data": "synthetic (seeded, Qwen-shaped; no checkpoints)",
-            "config": {"workload": name, "description": desc, "params": n_params, "tensors": len(shapes),
+            "config": {"workload": name if args.layers is None else f"{name} ({args.layers} layers)",
+                       "description": desc, "params": n_params, "tensors": len(shapes),
                        "experts": K, "op": op, "density": density, "scope": "tensor",
                        "l2": "inputs larger than L2 (129 MB); no flush needed",
                        "parallelism": f"replica x{world}"},
@@ -340,6 +341,9 @@ def main():
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-budget", type=float, default=12.0)
+    ap.add_argument("--layers", type=int, default=None,
+                    help="decoder layers of the shape set (default: the model's own); "
+                         "smaller cases are for profiling only")
     args = ap.parse_args()
     if args.warmup < 3 and args.impl == "mine":
         args.warmup = 3

@@ -196,14 +196,17 @@ unsigned long long cand_cap_of(long long n, double rho) {
     const double q = kk / (double)n;
     const double S = SAMPLE_MAX;
     const double band = 2.0 * (SAMPLE_Z * std::sqrt(S * q * (1.0 - q)) + 2.0) / S;
-    const double cap = 8192.0 + std::ceil((2.0 * band + 0.002) * (double)n);
+    // interior keys of the band (twice its expected width), plus what the
+    // warps' candidate chunks may leave unused at the end of their ranges
+    const double waste = (double)CHUNK_MAX * (std::ceil((double)n / (TILE * 64.0)) + 2.0);
+    const double cap = 8192.0 + std::ceil((2.0 * band + 0.002) * (double)n) + waste;
     return (unsigned long long)std::min(cap, (double)n);
 }
 
 size_t al256(size_t v) { return (v + 255) & ~(size_t)255; }
 
 struct Layout {
-    size_t hdr, units, trec, tcnt, hist, gram, coef, zero_end;
+    size_t hdr, units, trec, tcnt, hist, fhist, gram, coef, zero_end;
     size_t tens, xptr, mptr, table_end;
     size_t cand, total;
     long long n_tiles = 0;
@@ -246,6 +249,8 @@ Layout layout_of(const Call& c, int t0, int t1) {
     L.trec = o;  o = al256(o + (select && scope != ISO_SCOPE_BLOCK ? (size_t)K * tiles * sizeof(TileRec) : 0));
     L.tcnt = o;  o = al256(o + (select && scope != ISO_SCOPE_BLOCK ? (size_t)K * tiles * 4 : 0));
     L.hist = o;  o = al256(o + (select && scope != ISO_SCOPE_BLOCK ? (size_t)K * units * RADIX_BINS * 4 : 0));
+    const bool want_gamma = select && !c.mask_only && c.op == ISO_OP_ISO && K == 1 && scope == ISO_SCOPE_TENSOR;
+    L.fhist = o; o = al256(o + (want_gamma ? (size_t)K * units * RADIX_BINS * 8 : 0));
     L.gram = o;  o = al256(o + (size_t)T * K * K * 8);
     L.coef = o;  o = al256(o + (size_t)T * K * 8);
     L.zero_end = o;
@@ -381,6 +386,7 @@ int run_group(const Call& c, int t0, int t1, char* ws, cudaStream_t s, const iso
     P.trec = reinterpret_cast<TileRec*>(ws + L.trec);
     P.tcnt = reinterpret_cast<uint32_t*>(ws + L.tcnt);
     P.hist = reinterpret_cast<uint32_t*>(ws + L.hist);
+    P.fhist = reinterpret_cast<double*>(ws + L.fhist);
     P.cand = reinterpret_cast<uint32_t*>(ws + L.cand);
     P.gram = reinterpret_cast<double*>(ws + L.gram);
     P.coef = reinterpret_cast<double*>(ws + L.coef);
@@ -428,7 +434,7 @@ int run_group(const Call& c, int t0, int t1, char* ws, cudaStream_t s, const iso
             using XT = std::remove_pointer_t<decltype(xt)>;
             using BT = std::remove_pointer_t<decltype(bt)>;
             constexpr bool CK = decltype(ck)::value;
-            const int smem = (SAMPLE_MAX + RADIX_BINS) * 4;
+            const int smem = (SAMPLE_MAX + 2 * RADIX_BINS) * 4;
             ISO_TRY(smem_optin(k_sample<XT, BT, CK>, smem));
             ISO_TRY(launch(KD_SAMPLE, s, [&] { k_sample<XT, BT, CK><<<KU, SAMPLE_TPB, smem, s>>>(P); }));
             ISO_TRY(launch(KD_COUNT, s, [&] { k_count<XT, BT, CK><<<pgrid, TPB, 0, s>>>(P); }));

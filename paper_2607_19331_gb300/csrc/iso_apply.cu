@@ -32,40 +32,6 @@ __device__ __forceinline__ void load8_tail(const void* p, long long e, long long
     }
 }
 
-template <typename T> struct Store8;
-template <> struct Store8<__nv_bfloat16> {
-    static __device__ __forceinline__ void run(void* p, long long e, long long n, const float (&v)[8]) {
-        __nv_bfloat16* q = static_cast<__nv_bfloat16*>(p) + e;
-        if (e + 8 <= n) {
-            uint4 u;
-            __nv_bfloat162 a = __floats2bfloat162_rn(v[0], v[1]);
-            __nv_bfloat162 b = __floats2bfloat162_rn(v[2], v[3]);
-            __nv_bfloat162 c = __floats2bfloat162_rn(v[4], v[5]);
-            __nv_bfloat162 d = __floats2bfloat162_rn(v[6], v[7]);
-            u.x = *reinterpret_cast<uint32_t*>(&a);
-            u.y = *reinterpret_cast<uint32_t*>(&b);
-            u.z = *reinterpret_cast<uint32_t*>(&c);
-            u.w = *reinterpret_cast<uint32_t*>(&d);
-            *reinterpret_cast<uint4*>(q) = u;
-        } else {
-            for (int j = 0; j < 8; ++j)
-                if (e + j < n) q[j] = __float2bfloat16_rn(v[j]);
-        }
-    }
-};
-template <> struct Store8<float> {
-    static __device__ __forceinline__ void run(void* p, long long e, long long n, const float (&v)[8]) {
-        float* q = static_cast<float*>(p) + e;
-        if (e + 8 <= n) {
-            reinterpret_cast<float4*>(q)[0] = make_float4(v[0], v[1], v[2], v[3]);
-            reinterpret_cast<float4*>(q)[1] = make_float4(v[4], v[5], v[6], v[7]);
-        } else {
-            for (int j = 0; j < 8; ++j)
-                if (e + j < n) q[j] = v[j];
-        }
-    }
-};
-
 // ---------------------------------------------------------------------------
 // per-entry selection
 // ---------------------------------------------------------------------------
@@ -83,108 +49,259 @@ __device__ __forceinline__ int block_unit(const Plan& P, const TensorDesc& d, lo
 __device__ __forceinline__ int sgn(float v) { return (v > 0.0f) - (v < 0.0f); }
 
 // ---------------------------------------------------------------------------
-// apply
+// apply: one warp per tile, one contiguous tile range per warp
 // ---------------------------------------------------------------------------
+__device__ __forceinline__ void store8(void* p, long long e, long long n, const float (&v)[8], bool bf16) {
+    if (bf16) {
+        __nv_bfloat16* q = static_cast<__nv_bfloat16*>(p) + e;
+        if (e + 8 <= n) {
+            __nv_bfloat162 a = __floats2bfloat162_rn(v[0], v[1]);
+            __nv_bfloat162 b = __floats2bfloat162_rn(v[2], v[3]);
+            __nv_bfloat162 c = __floats2bfloat162_rn(v[4], v[5]);
+            __nv_bfloat162 d = __floats2bfloat162_rn(v[6], v[7]);
+            uint4 u;
+            u.x = *reinterpret_cast<uint32_t*>(&a); u.y = *reinterpret_cast<uint32_t*>(&b);
+            u.z = *reinterpret_cast<uint32_t*>(&c); u.w = *reinterpret_cast<uint32_t*>(&d);
+            __stcs(reinterpret_cast<uint4*>(q), u);
+        } else {
+            for (int j = 0; j < 8; ++j)
+                if (e + j < n) q[j] = __float2bfloat16_rn(v[j]);
+        }
+    } else {
+        float* q = static_cast<float*>(p) + e;
+        if (e + 8 <= n) {
+            __stcs(reinterpret_cast<float4*>(q), make_float4(v[0], v[1], v[2], v[3]));
+            __stcs(reinterpret_cast<float4*>(q) + 1, make_float4(v[4], v[5], v[6], v[7]));
+        } else {
+            for (int j = 0; j < 8; ++j)
+                if (e + j < n) q[j] = v[j];
+        }
+    }
+}
+
+// the K experts' selection parameters and coefficients of one tensor
+struct TensorParams {
+    SelParam sp[MAXK];
+    float cf[MAXK];
+    const void* xs[MAXK];
+    bool blk, iso2d, iso1d;
+    long long pos_off;
+};
+
+__device__ __forceinline__ void tensor_params(const Plan& P, int t, int K, TensorParams& tp) {
+    const TensorDesc& d = P.tens[t];
+    const bool is1d = (d.flags & TF_1D) != 0;
+    tp.iso2d = (P.op == ISO_OP_ISO) && !is1d;
+    tp.iso1d = (P.op == ISO_OP_ISO) && is1d;
+    tp.blk = (P.scope == ISO_SCOPE_BLOCK) && (d.flags & TF_TRIM);
+    tp.pos_off = (P.scope == ISO_SCOPE_GLOBAL) ? d.uoff : 0;
+#pragma unroll
+    for (int i = 0; i < MAXK; ++i) {
+        if (i >= K) break;
+        tp.xs[i] = P.xptr[i * P.n_tensors + t];
+        tp.cf[i] = tp.iso2d ? (float)P.coef[(long long)t * K + i] : 0.0f;
+        if (!tp.blk) {
+            const Unit& U = P.units[(long long)i * P.n_units + ((P.scope == ISO_SCOPE_GLOBAL) ? 0 : d.unit)];
+            tp.sp[i].t = U.t;
+            tp.sp[i].cut = U.cut;
+        }
+    }
+}
+
+// merged value of one entry from its K (masked) task-vector entries
+__device__ __forceinline__ float combine(const Plan& P, const TensorParams& tp, int K, float th0,
+                                         const float* tau, const bool* sel) {
+    float upd;
+    if (P.op == ISO_OP_TA || tp.iso1d) {
+        float s = 0.0f;
+        for (int i = 0; i < K; ++i) s = __fadd_rn(s, tau[i]);
+        upd = tp.iso1d ? __fdiv_rn(s, (float)K) : __fmul_rn(P.lambda, s);
+    } else if (P.op == ISO_OP_TIES) {
+        float s = 0.0f;
+        for (int i = 0; i < K; ++i) s = __fadd_rn(s, sel[i] ? tau[i] : 0.0f);
+        const int gam = sgn(s);
+        float a = 0.0f;
+        int cnt = 0;
+        for (int i = 0; i < K; ++i)
+            if (sel[i] && tau[i] != 0.0f && sgn(tau[i]) == gam) { a = __fadd_rn(a, tau[i]); cnt++; }
+        const float merged = cnt ? __fdiv_rn(a, (float)cnt) : 0.0f;
+        upd = __fmul_rn(P.lambda, merged);
+    } else {
+        float s = 0.0f;
+        for (int i = 0; i < K; ++i)
+            if (sel[i]) s = __fadd_rn(s, __fmul_rn(tp.cf[i], tau[i]));
+        upd = s;
+    }
+    return (upd == 0.0f) ? th0 : __fadd_rn(th0, upd);
+}
+
+// K = 1: the per-tensor scale, whether the tensor is trimmed, and the packed
+// threshold (t, ~cut) for tensor-local positions below 2^32
+__device__ __forceinline__ void k1_params(const Plan& P, const TensorParams& tp, float* a, bool* mask,
+                                          unsigned long long* thr) {
+    if (P.op == ISO_OP_TA) { *a = P.lambda; *mask = false; }
+    else if (tp.iso1d) { *a = 1.0f; *mask = false; }
+    else if (tp.iso2d) { *a = tp.cf[0]; *mask = true; }
+    else { *a = P.lambda; *mask = true; }
+    const long long cut = tp.sp[0].cut;
+    const uint32_t c32 = (cut >= 0xFFFFFFFFLL) ? 0xFFFFFFFFu : (uint32_t)cut;
+    *thr = ((unsigned long long)tp.sp[0].t << 32) | (uint32_t)~c32;
+}
+
+// BLOCK scope: selection parameters of entry (row, col) for expert i
+__device__ __forceinline__ SelParam block_param(const Plan& P, const TensorDesc& d, int i,
+                                                long long row, long long col) {
+    const Unit& U = P.units[(long long)i * P.n_units + block_unit(P, d, row, col)];
+    SelParam s;
+    s.t = U.t;
+    s.cut = U.cut;
+    return s;
+}
+
 template <typename XT, typename BT, bool CK, int KC>
 __global__ void __launch_bounds__(TPB) k_apply(Plan P) {
     const int K = KC ? KC : P.K;
-    for (long long g = blockIdx.x; g < P.n_tiles; g += gridDim.x) {
-        const int t = tensor_of_tile(P.tens, P.n_tensors, g);
+    const int lane = threadIdx.x & 31;
+    const long long W = (long long)gridDim.x * WPB;
+    const long long wid = (long long)blockIdx.x * WPB + (threadIdx.x >> 5);
+    const long long per = (P.n_tiles + W - 1) / W;
+    const long long beg = wid * per;
+    const long long end = (beg + per < P.n_tiles) ? beg + per : P.n_tiles;
+    if (beg >= end) return;
+    const bool obf = sizeof(BT) == 2;
+    int t = tensor_of_tile(P.tens, P.n_tensors, beg);
+    long long t_end = P.tens[t].tile_base + (P.tens[t].numel + TILE - 1) / TILE;
+    TensorParams tp;
+    tensor_params(P, t, K, tp);
+
+    if (KC == 1) {
+        // K = 1: every operator reduces to theta_0 + a * (mask ? tau : 0) with a
+        // per-tensor scale a (TA, TIES: lambda; ISO 2-D: c; ISO 1-D: 1/K = 1)
+        // and the mask off for TA and ISO 1-D.  The whole tile sits in
+        // registers while the next tile's loads are in flight.
+        RawTile<XT, BT, true> cur, nxt;
+        {
+            const TensorDesc& d = P.tens[t];
+            cur.load(tp.xs[0], d.base, (beg - d.tile_base) * TILE, d.numel, lane);
+        }
+        int nt = t;
+        long long nt_end = t_end;
+        float k1_a = 1.0f;
+        bool k1_mask = true;
+        unsigned long long k1_thr = 0;
+        for (long long g = beg; g < end; ++g) {
+            // prefetch tile g + 1
+            if (g + 1 < end) {
+                while (g + 1 >= nt_end) {
+                    ++nt;
+                    nt_end = P.tens[nt].tile_base + (P.tens[nt].numel + TILE - 1) / TILE;
+                }
+                const TensorDesc& nd = P.tens[nt];
+                nxt.load(P.xptr[nt], nd.base, (g + 1 - nd.tile_base) * TILE, nd.numel, lane);
+            }
+            if (g >= t_end || g == beg) {
+                while (g >= t_end) { ++t; t_end = P.tens[t].tile_base + (P.tens[t].numel + TILE - 1) / TILE; }
+                tensor_params(P, t, K, tp);
+                k1_params(P, tp, &k1_a, &k1_mask, &k1_thr);
+            }
+            const TensorDesc& d = P.tens[t];
+            const long long n = d.numel;
+            const long long e0 = (g - d.tile_base) * TILE;
+#pragma unroll
+            for (int v = 0; v < WVEC; ++v) {
+                const long long e = e0 + v * (32 * VEC) + lane * VEC;
+                if (e >= n) continue;
+                float th0[VEC], tau[VEC];
+                raw_to_f32<BT>(reinterpret_cast<const uint4(&)[Lanes<BT>::N]>(cur.b[v]), th0);
+                if (CK) {
+                    cur.tau(v, tau);
+                } else {
+                    raw_to_f32<XT>(cur.x[v], tau);
+                }
+                float o[VEC];
+                if (tp.blk || P.scope == ISO_SCOPE_GLOBAL) {
+                    long long r = 0, cc = 0;
+                    if (tp.blk) { r = e / d.cols; cc = e - r * d.cols; }
+#pragma unroll
+                    for (int j = 0; j < VEC; ++j) {
+                        SelParam s = tp.sp[0];
+                        if (tp.blk) {
+                            s = block_param(P, d, 0, r, cc);
+                            if (++cc == d.cols) { cc = 0; ++r; }
+                        }
+                        const bool sel = !k1_mask || kept(key_of(tau[j]), tp.pos_off + e + j, s);
+                        const float upd = __fmul_rn(k1_a, sel ? tau[j] : 0.0f);
+                        o[j] = (upd == 0.0f) ? th0[j] : __fadd_rn(th0[j], upd);
+                    }
+                } else {
+                    // kept <=> (key, ~pos) > (t, ~cut) as one 64-bit comparison
+                    const uint32_t p0 = ~(uint32_t)e;
+#pragma unroll
+                    for (int j = 0; j < VEC; ++j) {
+                        const unsigned long long kp =
+                            ((unsigned long long)key_of(tau[j]) << 32) | (uint32_t)(p0 - (uint32_t)j);
+                        const bool sel = !k1_mask || kp > k1_thr;
+                        const float upd = __fmul_rn(k1_a, sel ? tau[j] : 0.0f);
+                        o[j] = (upd == 0.0f) ? th0[j] : __fadd_rn(th0[j], upd);
+                    }
+                }
+                store8(d.out, e, n, o, obf);
+            }
+            cur = nxt;
+        }
+        return;
+    }
+
+    // K >= 2: vector by vector, the K experts' loads of a vector in flight together
+    for (long long g = beg; g < end; ++g) {
+        if (g >= t_end) {
+            while (g >= t_end) { ++t; t_end = P.tens[t].tile_base + (P.tens[t].numel + TILE - 1) / TILE; }
+            tensor_params(P, t, K, tp);
+        }
         const TensorDesc& d = P.tens[t];
         const long long n = d.numel;
         const long long e0 = (g - d.tile_base) * TILE;
-        const bool is1d = (d.flags & TF_1D) != 0;
-        const bool iso2d = (P.op == ISO_OP_ISO) && !is1d;
-        const bool iso1d = (P.op == ISO_OP_ISO) && is1d;
-        const bool blk = (P.scope == ISO_SCOPE_BLOCK) && (d.flags & TF_TRIM);
-        const long long pos_off = (P.scope == ISO_SCOPE_GLOBAL) ? d.uoff : 0;
-        SelParam sp[KC ? KC : MAXK];
-        float cf[KC ? KC : MAXK];
-        const void* xs[KC ? KC : MAXK];
-#pragma unroll
-        for (int i = 0; i < (KC ? KC : MAXK); ++i) {
-            if (i >= K) break;
-            xs[i] = P.xptr[i * P.n_tensors + t];
-            cf[i] = iso2d ? (float)P.coef[(long long)t * K + i] : 0.0f;
-            if (!blk) {
-                const Unit& U = P.units[(long long)i * P.n_units + ((P.scope == ISO_SCOPE_GLOBAL) ? 0 : d.unit)];
-                sp[i].t = U.t;
-                sp[i].cut = U.cut;
-            }
-        }
-        for (int v = 0; v < NVEC; ++v) {
-            const long long e = e0 + v * (TPB * VEC) + threadIdx.x * VEC;
+        for (int v = 0; v < WVEC; ++v) {
+            const long long e = e0 + v * (32 * VEC) + lane * VEC;
             if (e >= n) continue;
-            float th0[VEC];
-            load8_tail<BT>(d.base, e, n, th0);
-            float acc0[VEC], acc1[VEC];   // TA / ISO: running sums; TIES: election sum
+            uint4 braw[Lanes<BT>::N];
+            uint4 xraw[MAXK][Lanes<XT>::N];
+            load_raw8<BT>(d.base, e, n, braw);
 #pragma unroll
-            for (int j = 0; j < VEC; ++j) { acc0[j] = 0.0f; acc1[j] = 0.0f; }
-            float tau[KC ? KC : MAXK][VEC];
-            bool sel[KC ? KC : MAXK][VEC];
-            long long row = 0, col = 0;
-            if (blk) { row = e / d.cols; col = e - row * d.cols; }
-#pragma unroll
-            for (int i = 0; i < (KC ? KC : MAXK); ++i) {
+            for (int i = 0; i < MAXK; ++i) {
                 if (i >= K) break;
-                TauSrc<XT, BT, CK>::load8(xs[i], d.base, e, n, tau[i]);
-                long long r = row, c = col;
+                load_raw8<XT>(tp.xs[i], e, n, xraw[i]);
+            }
+            float th0[VEC];
+            raw_to_f32<BT>(braw, th0);
+            float tau[MAXK][VEC];
 #pragma unroll
-                for (int j = 0; j < VEC; ++j) {
-                    SelParam s;
-                    if (blk) {
-                        const Unit& U = P.units[(long long)i * P.n_units + block_unit(P, d, r, c)];
-                        s.t = U.t;
-                        s.cut = U.cut;
-                        if (++c == d.cols) { c = 0; ++r; }
-                    } else {
-                        s = sp[i];
-                    }
-                    sel[i][j] = kept(key_of(tau[i][j]), pos_off + e + j, s);
+            for (int i = 0; i < MAXK; ++i) {
+                if (i >= K) break;
+                raw_to_f32<XT>(xraw[i], tau[i]);
+                if (CK) {
+#pragma unroll
+                    for (int j = 0; j < VEC; ++j) tau[i][j] = __fsub_rn(tau[i][j], th0[j]);
                 }
             }
+            long long r = 0, cc = 0;
+            if (tp.blk) { r = e / d.cols; cc = e - r * d.cols; }
             float o[VEC];
 #pragma unroll
             for (int j = 0; j < VEC; ++j) {
-                float upd;
-                if (P.op == ISO_OP_TA || iso1d) {
-                    float s = 0.0f;
+                float tj[MAXK];
+                bool sj[MAXK];
 #pragma unroll
-                    for (int i = 0; i < (KC ? KC : MAXK); ++i) {
-                        if (i >= K) break;
-                        s = __fadd_rn(s, tau[i][j]);
-                    }
-                    upd = iso1d ? __fdiv_rn(s, (float)K) : __fmul_rn(P.lambda, s);
-                } else if (P.op == ISO_OP_TIES) {
-                    float s = 0.0f;
-#pragma unroll
-                    for (int i = 0; i < (KC ? KC : MAXK); ++i) {
-                        if (i >= K) break;
-                        s = __fadd_rn(s, sel[i][j] ? tau[i][j] : 0.0f);
-                    }
-                    const int gam = sgn(s);
-                    float a = 0.0f;
-                    int cnt = 0;
-#pragma unroll
-                    for (int i = 0; i < (KC ? KC : MAXK); ++i) {
-                        if (i >= K) break;
-                        const float x = tau[i][j];
-                        if (sel[i][j] && x != 0.0f && sgn(x) == gam) { a = __fadd_rn(a, x); cnt++; }
-                    }
-                    const float merged = cnt ? __fdiv_rn(a, (float)cnt) : 0.0f;
-                    upd = __fmul_rn(P.lambda, merged);
-                } else {
-                    float s = 0.0f;
-#pragma unroll
-                    for (int i = 0; i < (KC ? KC : MAXK); ++i) {
-                        if (i >= K) break;
-                        if (sel[i][j]) s = __fadd_rn(s, __fmul_rn(cf[i], tau[i][j]));
-                    }
-                    upd = s;
+                for (int i = 0; i < MAXK; ++i) {
+                    if (i >= K) break;
+                    tj[i] = tau[i][j];
+                    const SelParam s = tp.blk ? block_param(P, d, i, r, cc) : tp.sp[i];
+                    sj[i] = kept(key_of(tj[i]), tp.pos_off + e + j, s);
                 }
-                o[j] = (upd == 0.0f) ? th0[j] : __fadd_rn(th0[j], upd);
+                if (tp.blk && ++cc == d.cols) { cc = 0; ++r; }
+                o[j] = combine(P, tp, K, th0[j], tj, sj);
             }
-            Store8<BT>::run(d.out, e, n, o);
+            store8(d.out, e, n, o, obf);
         }
     }
 }
@@ -195,65 +312,72 @@ __global__ void __launch_bounds__(TPB) k_apply(Plan P) {
 template <typename XT, typename BT, bool CK>
 __global__ void __launch_bounds__(TPB) k_gram(Plan P) {
     constexpr int NP = MAXK * (MAXK + 1) / 2;
-    __shared__ double s_g[NP];
+    __shared__ double s_g[WPB][NP];
     const int K = P.K;
-    const int np = K * (K + 1) / 2;
-    const long long per = (P.n_tiles + gridDim.x - 1) / gridDim.x;
-    const long long g0 = blockIdx.x * per;
-    const long long g1 = (g0 + per < P.n_tiles) ? g0 + per : P.n_tiles;
-    for (int q = threadIdx.x; q < NP; q += blockDim.x) s_g[q] = 0.0;
-    __syncthreads();
-    int cur = -1;
-    for (long long g = g0; g < g1; ++g) {
-        const int t = tensor_of_tile(P.tens, P.n_tensors, g);
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const long long W = (long long)gridDim.x * WPB;
+    const long long wid = (long long)blockIdx.x * WPB + warp;
+    const long long per = (P.n_tiles + W - 1) / W;
+    const long long beg = wid * per;
+    const long long end = (beg + per < P.n_tiles) ? beg + per : P.n_tiles;
+    for (int q = lane; q < NP; q += 32) s_g[warp][q] = 0.0;
+    __syncwarp();
+    if (beg >= end) return;
+    int t = tensor_of_tile(P.tens, P.n_tensors, beg);
+    long long t_end = P.tens[t].tile_base + (P.tens[t].numel + TILE - 1) / TILE;
+    TensorParams tp;
+    tensor_params(P, t, K, tp);
+    auto flush = [&](int tt) {
+        __syncwarp();
+        if (lane == 0) {
+            int q = 0;
+            for (int a = 0; a < K; ++a)
+                for (int b = a; b < K; ++b, ++q)
+                    if (s_g[warp][q] != 0.0) {
+                        atomicAdd(&P.gram[((long long)tt * K + a) * K + b], s_g[warp][q]);
+                        s_g[warp][q] = 0.0;
+                    }
+        }
+        __syncwarp();
+    };
+    for (long long g = beg; g < end; ++g) {
+        if (g >= t_end) {
+            flush(t);
+            while (g >= t_end) { ++t; t_end = P.tens[t].tile_base + (P.tens[t].numel + TILE - 1) / TILE; }
+            tensor_params(P, t, K, tp);
+        }
         const TensorDesc& d = P.tens[t];
         if ((d.flags & TF_1D) || !(d.flags & TF_TRIM)) continue;
-        if (t != cur) {
-            __syncthreads();
-            if (cur >= 0)
-                for (int q = threadIdx.x; q < np; q += blockDim.x) {
-                    if (s_g[q] != 0.0) {
-                        int a = 0, b = q;   // q -> (a, b) in the upper triangle, row-major
-                        while (b >= K - a) { b -= K - a; ++a; }
-                        atomicAdd(&P.gram[((long long)cur * K + a) * K + a + b], s_g[q]);
-                    }
-                    s_g[q] = 0.0;
-                }
-            __syncthreads();
-            cur = t;
-        }
         const long long n = d.numel;
         const long long e0 = (g - d.tile_base) * TILE;
-        const bool blk = (P.scope == ISO_SCOPE_BLOCK);
-        const long long pos_off = (P.scope == ISO_SCOPE_GLOBAL) ? d.uoff : 0;
         float acc[NP];
 #pragma unroll
         for (int q = 0; q < NP; ++q) acc[q] = 0.0f;
-        for (int v = 0; v < NVEC; ++v) {
-            const long long e = e0 + v * (TPB * VEC) + threadIdx.x * VEC;
+        for (int v = 0; v < WVEC; ++v) {
+            const long long e = e0 + v * (32 * VEC) + lane * VEC;
             if (e >= n) continue;
+            float th0[VEC];
+            if (CK) load8_tail<BT>(d.base, e, n, th0);
             float m[MAXK][VEC];
-            long long row = 0, col = 0;
-            if (blk) { row = e / d.cols; col = e - row * d.cols; }
+            long long r = 0, cc = 0;
+            if (tp.blk) { r = e / d.cols; cc = e - r * d.cols; }
 #pragma unroll
             for (int i = 0; i < MAXK; ++i) {
                 if (i >= K) break;
+                uint4 xr[Lanes<XT>::N];
+                load_raw8<XT>(tp.xs[i], e, n, xr);
                 float tau[VEC];
-                TauSrc<XT, BT, CK>::load8(P.xptr[i * P.n_tensors + t], d.base, e, n, tau);
-                SelParam s;
-                if (!blk) {
-                    const Unit& U = P.units[(long long)i * P.n_units + ((P.scope == ISO_SCOPE_GLOBAL) ? 0 : d.unit)];
-                    s.t = U.t; s.cut = U.cut;
-                }
-                long long r = row, c = col;
+                raw_to_f32<XT>(xr, tau);
+                long long rr = r, c2 = cc;
 #pragma unroll
                 for (int j = 0; j < VEC; ++j) {
-                    if (blk) {
-                        const Unit& U = P.units[(long long)i * P.n_units + block_unit(P, d, r, c)];
-                        s.t = U.t; s.cut = U.cut;
-                        if (++c == d.cols) { c = 0; ++r; }
+                    if (CK) tau[j] = __fsub_rn(tau[j], th0[j]);
+                    SelParam s = tp.sp[i];
+                    if (tp.blk) {
+                        s = block_param(P, d, i, rr, c2);
+                        if (++c2 == d.cols) { c2 = 0; ++rr; }
                     }
-                    m[i][j] = kept(key_of(tau[j]), pos_off + e + j, s) ? tau[j] : 0.0f;
+                    m[i][j] = (e + j < n && kept(key_of(tau[j]), tp.pos_off + e + j, s)) ? tau[j] : 0.0f;
                 }
             }
             int q = 0;
@@ -269,34 +393,22 @@ __global__ void __launch_bounds__(TPB) k_gram(Plan P) {
                 }
             }
         }
-        // warp partials in binary32 (<= 1024 entries), then binary64 in shared memory
-        const int lane = threadIdx.x & 31;
-        int q = 0;
+        // tile partials in binary32 (<= 1024 entries), summed in binary64 per warp
+        int q = 0, cq = 0;
 #pragma unroll
         for (int a = 0; a < MAXK; ++a) {
 #pragma unroll
             for (int b = a; b < MAXK; ++b) {
                 if (a < K && b < K) {
                     const float w = warp_sum(acc[q]);
-                    if (lane == 0 && w != 0.0f) {
-                        // compact index over the K x K upper triangle
-                        const int cq = a * K - a * (a - 1) / 2 + (b - a);
-                        atomicAdd(&s_g[cq], (double)w);
-                    }
+                    if (lane == 0) s_g[warp][cq] += (double)w;
+                    ++cq;
                 }
                 ++q;
             }
         }
     }
-    __syncthreads();
-    if (cur >= 0)
-        for (int q = threadIdx.x; q < np; q += blockDim.x) {
-            if (s_g[q] != 0.0) {
-                int a = 0, b = q;
-                while (b >= K - a) { b -= K - a; ++a; }
-                atomicAdd(&P.gram[((long long)cur * K + a) * K + a + b], s_g[q]);
-            }
-        }
+    flush(t);
 }
 
 // ---------------------------------------------------------------------------
@@ -374,7 +486,9 @@ __global__ void k_solve(Plan P, int gram_mode) {
 // ---------------------------------------------------------------------------
 template <typename XT>
 __global__ void __launch_bounds__(TPB) k_mask(Plan P, uint32_t* const* mptr) {
-    for (long long g = blockIdx.x; g < P.n_tiles; g += gridDim.x) {
+    const int lane = threadIdx.x & 31;
+    const long long W = (long long)gridDim.x * WPB;
+    for (long long g = (long long)blockIdx.x * WPB + (threadIdx.x >> 5); g < P.n_tiles; g += W) {
         const int t = tensor_of_tile(P.tens, P.n_tensors, g);
         const TensorDesc& d = P.tens[t];
         uint32_t* mw = mptr[t];
@@ -384,12 +498,13 @@ __global__ void __launch_bounds__(TPB) k_mask(Plan P, uint32_t* const* mptr) {
         const bool blk = (P.scope == ISO_SCOPE_BLOCK);
         const long long pos_off = (P.scope == ISO_SCOPE_GLOBAL) ? d.uoff : 0;
         SelParam s0;
+        s0.t = 0; s0.cut = 0;
         if (!blk) {
             const Unit& U = P.units[(P.scope == ISO_SCOPE_GLOBAL) ? 0 : d.unit];
             s0.t = U.t; s0.cut = U.cut;
         }
-        for (int v = 0; v < NVEC; ++v) {
-            const long long e = e0 + v * (TPB * VEC) + threadIdx.x * VEC;
+        for (int v = 0; v < WVEC; ++v) {
+            const long long e = e0 + v * (32 * VEC) + lane * VEC;
             uint32_t bits = 0;
             if (e < n) {
                 float tau[VEC];
@@ -401,15 +516,14 @@ __global__ void __launch_bounds__(TPB) k_mask(Plan P, uint32_t* const* mptr) {
                     if (e + j >= n) break;
                     SelParam s = s0;
                     if (blk) {
-                        const Unit& U = P.units[block_unit(P, d, r, c)];
-                        s.t = U.t; s.cut = U.cut;
+                        s = block_param(P, d, 0, r, c);
                         if (++c == d.cols) { c = 0; ++r; }
                     }
                     if (kept(key_of(tau[j]), pos_off + e + j, s)) bits |= 1u << j;
                 }
             }
-            // four consecutive threads hold 32 consecutive entries
-            const int sub = threadIdx.x & 3;
+            // four consecutive lanes hold 32 consecutive entries
+            const int sub = lane & 3;
             uint32_t w = bits << (8 * sub);
             w |= __shfl_xor_sync(0xFFFFFFFFu, w, 1);
             w |= __shfl_xor_sync(0xFFFFFFFFu, w, 2);
@@ -432,22 +546,24 @@ __global__ void k_upload(UploadChunk c) {
 // ---------------------------------------------------------------------------
 template <typename AT, typename BT>
 __global__ void __launch_bounds__(TPB) k_delta(DeltaArgs A) {
+    const int lane = threadIdx.x & 31;
     const long long n_tiles = A.tile_base[A.n];
-    for (long long g = blockIdx.x; g < n_tiles; g += gridDim.x) {
+    const long long W = (long long)gridDim.x * WPB;
+    for (long long g = (long long)blockIdx.x * WPB + (threadIdx.x >> 5); g < n_tiles; g += W) {
         int t = 0;
         while (t + 1 < A.n && A.tile_base[t + 1] <= g) ++t;
         const long long n = A.numel[t];
         const long long e0 = (g - A.tile_base[t]) * TILE;
 #pragma unroll
-        for (int v = 0; v < NVEC; ++v) {
-            const long long e = e0 + v * (TPB * VEC) + threadIdx.x * VEC;
+        for (int v = 0; v < WVEC; ++v) {
+            const long long e = e0 + v * (32 * VEC) + lane * VEC;
             if (e >= n) continue;
             float a[VEC], b[VEC], o[VEC];
             load8_tail<AT>(A.a[t], e, n, a);
             load8_tail<BT>(A.b[t], e, n, b);
 #pragma unroll
             for (int j = 0; j < VEC; ++j) o[j] = __fsub_rn(a[j], b[j]);
-            Store8<float>::run(A.out[t], e, n, o);
+            store8(A.out[t], e, n, o, false);
         }
     }
 }

@@ -19,11 +19,16 @@ namespace iso {
 // ---------------------------------------------------------------------------
 // geometry
 // ---------------------------------------------------------------------------
-constexpr int TILE = 8192;                  // entries per streaming tile
+// A tile is 1024 consecutive entries of one tensor, processed by one warp:
+// lane L holds entries e0 + v*256 + 8L .. +8 for v = 0..3 (each warp-wide
+// vector step reads 256 consecutive entries).
+constexpr int TILE = 1024;                  // entries per tile
+constexpr int VEC = 8;                      // entries per lane per vector step
+constexpr int WVEC = TILE / (32 * VEC);     // vector steps per tile (4)
 constexpr int TPB = 256;                    // threads per streaming block
-constexpr int VEC = 8;                      // entries per thread per vector step
-constexpr int NVEC = TILE / (TPB * VEC);    // vector steps per tile (4)
-static_assert(NVEC * TPB * VEC == TILE, "tile geometry");
+constexpr int WPB = TPB / 32;               // warps per streaming block
+static_assert(WVEC * 32 * VEC == TILE, "tile geometry");
+constexpr int CHUNK_MAX = 1024;             // candidate slots a warp reserves at once
 
 constexpr int SAMPLE_MAX = 32768;           // sampled keys per unit (128 KB of smem)
 constexpr int SAMPLE_CHUNK = 256;           // contiguous entries per sample chunk
@@ -84,8 +89,12 @@ struct Unit {
     uint32_t lo, hi;
     // count-pass accumulators
     unsigned long long c_gt, c_hi, c_lo, n_int;
+    unsigned long long n_alloc;         // candidate slots handed out (>= n_int)
+    int32_t overflow;                   // the segment could not hold every interior key
+    int32_t pad0;
     double gamma_acc;                   // sum tau^2 over key > hi (count pass)
-    double gamma_acc2;                  // sum tau^2 over the radix source above t
+    double gamma_int;                   // sum tau^2 over the interior keys (count pass)
+    double gamma_rad;                   // sum tau^2 above the radix-selected bins
     // radix select
     int32_t r_src;
     int32_t r_shift, r_pshift;
@@ -125,6 +134,7 @@ struct Plan {
     TileRec*      trec;     // [K][n_tiles]
     uint32_t*     tcnt;     // [K][n_tiles] ties at t per tile
     uint32_t*     hist;     // [K * n_units][RADIX_BINS]
+    double*       fhist;    // [K * n_units][RADIX_BINS] sums of tau^2 per bin (K = 1 ISO only)
     uint32_t*     cand;     // candidate pool
     double*       gram;     // [n_tensors][K][K]
     double*       coef;     // [n_tensors][K]
@@ -217,6 +227,113 @@ struct TauSrc {
         return v;
     }
 };
+
+// ---------------------------------------------------------------------------
+// streaming loads / stores
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ uint4 ld_stream(const void* p) {
+    uint4 r;
+    asm("ld.global.nc.L1::no_allocate.L2::256B.v4.u32 {%0, %1, %2, %3}, [%4];"
+        : "=r"(r.x), "=r"(r.y), "=r"(r.z), "=r"(r.w) : "l"(p));
+    return r;
+}
+
+template <typename T> struct Lanes;   // uint4 words per 8 entries
+template <> struct Lanes<__nv_bfloat16> { static constexpr int N = 1; };
+template <> struct Lanes<float> { static constexpr int N = 2; };
+
+// 8 entries (start e, e % 8 == 0) as raw words; entries at or beyond n read as 0
+template <typename T>
+__device__ __forceinline__ void load_raw8(const void* p, long long e, long long n, uint4 (&w)[Lanes<T>::N]) {
+    if (e + 8 <= n) {
+#pragma unroll
+        for (int q = 0; q < Lanes<T>::N; ++q)
+            w[q] = ld_stream(static_cast<const char*>(p) + (e * sizeof(T)) + 16 * q);
+    } else {
+        uint32_t u[4 * Lanes<T>::N];
+#pragma unroll
+        for (int q = 0; q < 4 * Lanes<T>::N; ++q) u[q] = 0;
+        if (sizeof(T) == 2) {
+            const unsigned short* s = static_cast<const unsigned short*>(p);
+#pragma unroll
+            for (int j = 0; j < 8; ++j)
+                if (e + j < n) u[j >> 1] |= (uint32_t)s[e + j] << (16 * (j & 1));
+        } else {
+            const uint32_t* s = static_cast<const uint32_t*>(p);
+#pragma unroll
+            for (int j = 0; j < 8; ++j)
+                if (e + j < n) u[j] = s[e + j];
+        }
+#pragma unroll
+        for (int q = 0; q < Lanes<T>::N; ++q) w[q] = make_uint4(u[4 * q], u[4 * q + 1], u[4 * q + 2], u[4 * q + 3]);
+    }
+}
+
+template <typename T>
+__device__ __forceinline__ void raw_to_f32(const uint4 (&w)[Lanes<T>::N], float (&v)[8]) {
+    if (sizeof(T) == 2) {
+        const uint32_t u[4] = {w[0].x, w[0].y, w[0].z, w[0].w};
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+            v[2 * j] = __uint_as_float(u[j] << 16);
+            v[2 * j + 1] = __uint_as_float(u[j] & 0xFFFF0000u);
+        }
+    } else {
+#pragma unroll
+        for (int q = 0; q < Lanes<T>::N; ++q) {
+            v[4 * q] = __uint_as_float(w[q].x); v[4 * q + 1] = __uint_as_float(w[q].y);
+            v[4 * q + 2] = __uint_as_float(w[q].z); v[4 * q + 3] = __uint_as_float(w[q].w);
+        }
+    }
+}
+
+// One lane's share of a tile of a task-vector source, as raw words, so the
+// next tile's loads can be in flight while the current one is processed.
+template <typename XT, typename BT, bool CK>
+struct RawTile {
+    static constexpr int NX = Lanes<XT>::N;
+    static constexpr int NB = CK ? Lanes<BT>::N : 1;
+    uint4 x[WVEC][NX];
+    uint4 b[WVEC][NB];
+    __device__ __forceinline__ void load(const void* xp, const void* bp, long long e0, long long n, int lane) {
+#pragma unroll
+        for (int v = 0; v < WVEC; ++v) {
+            const long long e = e0 + v * (32 * VEC) + lane * VEC;
+            if (e < n) {
+                load_raw8<XT>(xp, e, n, x[v]);
+                if (CK) load_raw8<BT>(bp, e, n, reinterpret_cast<uint4(&)[Lanes<BT>::N]>(b[v]));
+            } else {
+#pragma unroll
+                for (int q = 0; q < NX; ++q) x[v][q] = make_uint4(0, 0, 0, 0);
+#pragma unroll
+                for (int q = 0; q < NB; ++q) b[v][q] = make_uint4(0, 0, 0, 0);
+            }
+        }
+    }
+    // tau = x (delta) or x - base (checkpoint), binary32
+    __device__ __forceinline__ void tau(int v, float (&t)[8]) const {
+        raw_to_f32<XT>(x[v], t);
+        if (CK) {
+            float bb[8];
+            raw_to_f32<BT>(reinterpret_cast<const uint4(&)[Lanes<BT>::N]>(b[v]), bb);
+#pragma unroll
+            for (int j = 0; j < 8; ++j) t[j] = __fsub_rn(t[j], bb[j]);
+        }
+    }
+};
+
+template <typename T>
+__device__ __forceinline__ T warp_excl_scan(T v, T* total) {
+    const int lane = threadIdx.x & 31;
+    T x = v;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+        T y = __shfl_up_sync(0xFFFFFFFFu, x, o);
+        if (lane >= o) x += y;
+    }
+    *total = __shfl_sync(0xFFFFFFFFu, x, 31);
+    return x - v;
+}
 
 // tile id -> tensor (binary search over tile_base)
 __device__ __forceinline__ int tensor_of_tile(const TensorDesc* tens, int n_tensors, long long tile) {

@@ -7,7 +7,7 @@
 //     kept(p)  <=>  key(p) > t  ||  (key(p) == t && pos(p) < cut)
 // which the streaming passes then apply as a pure per-entry predicate.
 //
-// Pipeline (all launches on the caller's stream, no waits between blocks):
+// Pipeline (all launches on the caller's stream; no block waits on another):
 //   k_sample   keys at evenly spaced chunks -> band [lo, hi] around rank k
 //   k_count    one full read: #key > hi, #key == hi / == lo per tile, and the
 //              interior keys lo < key < hi appended to the unit's segment
@@ -15,9 +15,12 @@
 //              segment) switches the unit to a radix select over its data
 //   k_radix_*  up to three 11-bit radix levels over the interior keys (or
 //              over the whole unit on the fallback path)
-//   k_tie      per-tile counts of keys == t where needed, and the sum of
-//              squares of the kept entries (ISO, K = 1)
+//   k_tie      per-tile counts of keys == t when the threshold is interior
 //   k_cut      the tile holding the need-th tie, then the exact position
+//
+// Work layout: a tile is 1024 entries handled by one warp; every warp (or
+// block) walks a contiguous range of (expert, tile) items, so the owning
+// tensor and unit change rarely and are tracked incrementally.
 #include "iso_internal.cuh"
 
 namespace iso {
@@ -31,6 +34,35 @@ __device__ __forceinline__ long long k_of_density(double rho, long long n) {
 }
 
 __device__ __forceinline__ int bitlen32(uint32_t v) { return v ? 32 - __clz(v) : 0; }
+
+__device__ __forceinline__ double sq(uint32_t key) {
+    const double f = (double)__uint_as_float(key);
+    return f * f;
+}
+
+// ---------------------------------------------------------------------------
+// (expert, tile) item cursor: items are expert-major, tiles in tensor order
+// ---------------------------------------------------------------------------
+struct Cursor {
+    long long it;        // current item
+    long long run_end;   // first item after the current (expert, tensor) run
+    long long g;         // tile
+    int i, t;            // expert, tensor
+};
+
+__device__ __forceinline__ void cursor_at(const Plan& P, long long it, Cursor& c) {
+    c.it = it;
+    c.i = (int)(it / P.n_tiles);
+    c.g = it - (long long)c.i * P.n_tiles;
+    c.t = tensor_of_tile(P.tens, P.n_tensors, c.g);
+    const TensorDesc& d = P.tens[c.t];
+    c.run_end = (long long)c.i * P.n_tiles + d.tile_base + (d.numel + TILE - 1) / TILE;
+}
+
+__device__ __forceinline__ Unit* unit_of(const Plan& P, int i, const TensorDesc& d) {
+    const int u = (P.scope == ISO_SCOPE_GLOBAL) ? 0 : d.unit;
+    return &P.units[(long long)i * P.n_units + u];
+}
 
 // ---------------------------------------------------------------------------
 // unit table
@@ -71,19 +103,15 @@ __global__ void k_init_units(Plan P, long long global_n) {
         return;
     }
     U.k = k_of_density(P.density, U.n);
-    if (U.k == 0) {
-        U.state = ST_NONE;
-        return;
-    }
-    U.state = ST_SAMPLE;
+    U.state = (U.k == 0) ? ST_NONE : ST_SAMPLE;
 }
 
 // ---------------------------------------------------------------------------
 // block-level radix select in shared memory
 // ---------------------------------------------------------------------------
 
-// Find, among nb bins taken from the top, the bin b with
-// above(b) < rank <= above(b) + hist[b].  Result broadcast through `res`.
+// Among nb bins taken from the top, the bin b with above(b) < rank <=
+// above(b) + hist[b]; rank <= 0 or beyond the total gives bin 0.
 __device__ void block_find_from_top(const uint32_t* hist, int nb, long long rank,
                                     long long* sm_scan, int* res_bin, long long* res_above) {
     const int per = (nb + blockDim.x - 1) / blockDim.x;
@@ -92,11 +120,11 @@ __device__ void block_find_from_top(const uint32_t* hist, int nb, long long rank
     long long local = 0;
     for (int j = j0; j < j0 + per && j < nb; ++j) local += hist[nb - 1 - j];
     long long total;
-    long long excl = block_excl_scan(local, sm_scan, &total);
+    const long long excl = block_excl_scan(local, sm_scan, &total);
     if (excl < rank && rank <= excl + local) {
         long long acc = excl;
         for (int j = j0; j < j0 + per && j < nb; ++j) {
-            uint32_t h = hist[nb - 1 - j];
+            const uint32_t h = hist[nb - 1 - j];
             if (rank <= acc + h) { *res_bin = nb - 1 - j; *res_above = acc; break; }
             acc += h;
         }
@@ -104,36 +132,45 @@ __device__ void block_find_from_top(const uint32_t* hist, int nb, long long rank
     __syncthreads();
 }
 
-// k-th largest (1-based rank) of the n keys in shared memory.
-__device__ uint32_t block_kth_largest(const uint32_t* keys, int n, long long rank, uint32_t* hist,
-                                      long long* sm_scan, int* sm_bin, long long* sm_above) {
-    uint32_t prefix = 0;
+// The ra-th and rb-th largest (1-based) of n keys in shared memory, one
+// histogram pass per radix level for both ranks.
+__device__ void block_kth_largest2(const uint32_t* keys, int n, long long ra, long long rb,
+                                   uint32_t* ha, uint32_t* hb, long long* sm_scan, int* sm_bin,
+                                   long long* sm_above, uint32_t* ka, uint32_t* kb) {
+    uint32_t pa = 0, pb = 0;
     int pshift = 31;
     for (;;) {
         const int shift = pshift > RADIX_BITS ? pshift - RADIX_BITS : 0;
         const int nb = 1 << (pshift - shift);
-        for (int b = threadIdx.x; b < nb; b += blockDim.x) hist[b] = 0;
+        for (int b = threadIdx.x; b < nb; b += blockDim.x) { ha[b] = 0; hb[b] = 0; }
         __syncthreads();
         for (int p = threadIdx.x; p < n; p += blockDim.x) {
-            uint32_t v = keys[p];
-            if ((v >> pshift) == prefix) atomicAdd(&hist[(v >> shift) & (nb - 1)], 1u);
+            const uint32_t v = keys[p];
+            const uint32_t top = v >> pshift, dig = (v >> shift) & (nb - 1);
+            if (top == pa) atomicAdd(&ha[dig], 1u);
+            if (top == pb) atomicAdd(&hb[dig], 1u);
         }
         __syncthreads();
-        block_find_from_top(hist, nb, rank, sm_scan, sm_bin, sm_above);
-        const int b = *sm_bin;
-        rank -= *sm_above;
-        prefix = (prefix << (pshift - shift)) | (uint32_t)b;
+        block_find_from_top(ha, nb, ra, sm_scan, sm_bin, sm_above);
+        ra -= *sm_above;
+        pa = (pa << (pshift - shift)) | (uint32_t)*sm_bin;
         __syncthreads();
-        if (shift == 0) return prefix;
+        block_find_from_top(hb, nb, rb, sm_scan, sm_bin, sm_above);
+        rb -= *sm_above;
+        pb = (pb << (pshift - shift)) | (uint32_t)*sm_bin;
+        __syncthreads();
+        if (shift == 0) break;
         pshift = shift;
     }
+    *ka = pa;
+    *kb = pb;
 }
 
 // ---------------------------------------------------------------------------
 // sample -> band
 // ---------------------------------------------------------------------------
 
-// unit position -> (tensor, entry) for GLOBAL scope: last tensor with uoff <= pos
+// unit position -> tensor for GLOBAL scope: last tensor with uoff <= pos
 __device__ __forceinline__ int tensor_of_upos(const TensorDesc* tens, int n_tensors, long long pos) {
     int lo = 0, hi = n_tensors - 1;
     while (lo < hi) {
@@ -146,7 +183,8 @@ __device__ __forceinline__ int tensor_of_upos(const TensorDesc* tens, int n_tens
 template <typename XT, typename BT, bool CKPT>
 __global__ void __launch_bounds__(SAMPLE_TPB) k_sample(Plan P) {
     extern __shared__ __align__(16) uint32_t s_keys[];
-    uint32_t* s_hist = s_keys + SAMPLE_MAX;
+    uint32_t* s_ha = s_keys + SAMPLE_MAX;
+    uint32_t* s_hb = s_ha + RADIX_BINS;
     __shared__ long long s_scan[33];
     __shared__ int s_bin;
     __shared__ long long s_above;
@@ -157,40 +195,58 @@ __global__ void __launch_bounds__(SAMPLE_TPB) k_sample(Plan P) {
     const long long n = U.n;
     const int S = (int)(n < SAMPLE_MAX ? n : SAMPLE_MAX);
     const int nch = SAMPLE_MAX / SAMPLE_CHUNK;
-    for (int q = threadIdx.x; q < S; q += blockDim.x) {
-        long long pos;
-        if (S == n) {
-            pos = q;
-        } else {
-            const int c = q / SAMPLE_CHUNK, j = q % SAMPLE_CHUNK;
-            pos = (long long)((double)(n - SAMPLE_CHUNK) * c / (nch - 1)) + j;
+    if (S < n && P.scope != ISO_SCOPE_GLOBAL) {
+        // chunks of 256 contiguous entries at evenly spaced, 8-aligned starts:
+        // one chunk per warp step, 8 entries per lane
+        const int t = U.tensor;
+        const void* x = P.xptr[i * P.n_tensors + t];
+        const void* b = P.tens[t].base;
+        const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nw = blockDim.x >> 5;
+        for (int c = warp; c < nch; c += nw) {
+            const long long start = ((long long)((double)(n - SAMPLE_CHUNK) * c / (nch - 1))) & ~7LL;
+            float tau[VEC];
+            TauSrc<XT, BT, CKPT>::load8(x, b, start + lane * VEC, n, tau);
+#pragma unroll
+            for (int j = 0; j < VEC; ++j) s_keys[c * SAMPLE_CHUNK + lane * VEC + j] = key_of(tau[j]);
         }
-        int t;
-        long long e;
-        if (P.scope == ISO_SCOPE_GLOBAL) {
-            t = tensor_of_upos(P.tens, P.n_tensors, pos);
-            e = pos - P.tens[t].uoff;
-        } else {
-            t = U.tensor;
-            e = pos;
+    } else {
+        for (int q = threadIdx.x; q < S; q += blockDim.x) {
+            long long pos;
+            if (S == n) {
+                pos = q;
+            } else {
+                const int c = q / SAMPLE_CHUNK, j = q % SAMPLE_CHUNK;
+                pos = (long long)((double)(n - SAMPLE_CHUNK) * c / (nch - 1)) + j;
+            }
+            int t;
+            long long e;
+            if (P.scope == ISO_SCOPE_GLOBAL) {
+                t = tensor_of_upos(P.tens, P.n_tensors, pos);
+                e = pos - P.tens[t].uoff;
+            } else {
+                t = U.tensor;
+                e = pos;
+            }
+            const float tau = TauSrc<XT, BT, CKPT>::load1(P.xptr[i * P.n_tensors + t], P.tens[t].base, e);
+            s_keys[q] = key_of(tau);
         }
-        const float tau = TauSrc<XT, BT, CKPT>::load1(P.xptr[i * P.n_tensors + t], P.tens[t].base, e);
-        s_keys[q] = key_of(tau);
     }
     __syncthreads();
     uint32_t lo, hi;
     if (S == n) {
         // the sample is the whole unit: the band is the exact threshold
-        hi = block_kth_largest(s_keys, S, U.k, s_hist, s_scan, &s_bin, &s_above);
-        lo = hi;
+        block_kth_largest2(s_keys, S, U.k, U.k, s_ha, s_hb, s_scan, &s_bin, &s_above, &hi, &lo);
     } else {
         const double q = (double)U.k / (double)n;
         const double r = (double)U.k * (double)S / (double)n;
         const double delta = SAMPLE_Z * sqrt((double)S * q * (1.0 - q)) + 2.0;
         const long long ra = (long long)floor(r - delta);
         const long long rb = (long long)ceil(r + delta);
-        hi = (ra >= 1) ? block_kth_largest(s_keys, S, ra, s_hist, s_scan, &s_bin, &s_above) : KEY_MAX;
-        lo = (rb <= S) ? block_kth_largest(s_keys, S, rb, s_hist, s_scan, &s_bin, &s_above) : 0u;
+        uint32_t ka, kb;
+        block_kth_largest2(s_keys, S, ra >= 1 ? ra : 1, rb <= S ? rb : S, s_ha, s_hb, s_scan,
+                           &s_bin, &s_above, &ka, &kb);
+        hi = (ra >= 1) ? ka : KEY_MAX;
+        lo = (rb <= S) ? kb : 0u;
     }
     if (threadIdx.x == 0) {
         U.lo = lo;
@@ -200,106 +256,198 @@ __global__ void __launch_bounds__(SAMPLE_TPB) k_sample(Plan P) {
 }
 
 // ---------------------------------------------------------------------------
-// count pass: one full read per unit
+// count pass: one warp per tile, one contiguous item range per warp
 // ---------------------------------------------------------------------------
-__device__ __forceinline__ Unit* unit_of_tile(const Plan& P, int i, const TensorDesc& d) {
-    const int u = (P.scope == ISO_SCOPE_GLOBAL) ? 0 : d.unit;
-    return &P.units[(long long)i * P.n_units + u];
+__device__ __forceinline__ Unit* count_unit(const Plan& P, const Cursor& c) {
+    const TensorDesc& d = P.tens[c.t];
+    if (!(d.flags & TF_TRIM)) return nullptr;
+    Unit* U = unit_of(P, c.i, d);
+    return (U->state == ST_BAND) ? U : nullptr;
 }
 
-template <typename XT, typename BT, bool CKPT>
+template <typename XT, typename BT, bool CK>
 __global__ void __launch_bounds__(TPB) k_count(Plan P) {
-    __shared__ unsigned long long s_red[33];
-    __shared__ uint32_t s_scan[33];
-    __shared__ double s_dred[33];
-    __shared__ uint32_t s_slot;
-    __shared__ int s_ok;
-
+    const int lane = threadIdx.x & 31;
+    const long long W = (long long)gridDim.x * WPB;
+    const long long wid = (long long)blockIdx.x * WPB + (threadIdx.x >> 5);
     const long long items = (long long)P.K * P.n_tiles;
-    for (long long it = blockIdx.x; it < items; it += gridDim.x) {
-        const int i = (int)(it / P.n_tiles);
-        const long long g = it % P.n_tiles;
-        const int t = tensor_of_tile(P.tens, P.n_tensors, g);
-        const TensorDesc& d = P.tens[t];
-        if (!(d.flags & TF_TRIM)) continue;
-        Unit* U = unit_of_tile(P, i, d);
-        if (U->state != ST_BAND) continue;
-        const uint32_t lo = U->lo, hi = U->hi;
-        const bool want_gamma = U->want_gamma != 0;
-        const void* x = P.xptr[i * P.n_tensors + t];
-        const long long e0 = (g - d.tile_base) * TILE;
-        const long long n = d.numel;
+    const long long per = (items + W - 1) / W;
+    const long long beg = wid * per;
+    const long long end = (beg + per < items) ? beg + per : items;
+    if (beg >= end) return;
 
-        uint32_t keys[NVEC][VEC];
+    // first valid item
+    Cursor c;
+    cursor_at(P, beg, c);
+    Unit* U = nullptr;
+    for (;;) {
+        U = count_unit(P, c);
+        if (U) break;
+        if (c.run_end >= end) return;
+        cursor_at(P, c.run_end, c);
+    }
+    RawTile<XT, BT, CK> cur;
+    {
+        const TensorDesc& d = P.tens[c.t];
+        cur.load(P.xptr[c.i * P.n_tensors + c.t], d.base, (c.g - d.tile_base) * TILE, d.numel, lane);
+    }
+
+    // per-unit accumulators (warp-uniform) and the candidate chunk
+    Unit* au = nullptr;
+    unsigned long long a_gt = 0, a_hi = 0, a_lo = 0, a_int = 0;
+    double l_gg = 0.0, l_gi = 0.0;                // per-lane partial sums of tau^2
+    unsigned long long ch_pos = 0;
+    uint32_t ch_left = 0;
+    bool ovf = false;
+    uint32_t lo = 0, hi = 0;
+    bool want_gamma = false;
+    unsigned long long cap = 0, coff = 0;
+
+    auto flush = [&]() {
+        if (!au) return;
+        const double gg = warp_sum(l_gg), gi = warp_sum(l_gi);
+        if (lane == 0) {
+            if (a_gt) atomicAdd(&au->c_gt, a_gt);
+            if (a_hi) atomicAdd(&au->c_hi, a_hi);
+            if (a_lo) atomicAdd(&au->c_lo, a_lo);
+            if (a_int) atomicAdd(&au->n_int, a_int);
+            if (want_gamma) {
+                if (gg != 0.0) atomicAdd(&au->gamma_acc, gg);
+                if (gi != 0.0) atomicAdd(&au->gamma_int, gi);
+            }
+            if (ovf) au->overflow = 1;
+        }
+        a_gt = a_hi = a_lo = a_int = 0;
+        l_gg = l_gi = 0.0;
+    };
+
+    for (;;) {
+        // locate and prefetch the next valid item
+        Cursor nc = c;
+        Unit* nU = nullptr;
+        {
+            long long nit = c.it + 1;
+            while (nit < end) {
+                if (nit >= nc.run_end) cursor_at(P, nit, nc);
+                else { nc.it = nit; nc.g++; }
+                nU = count_unit(P, nc);
+                if (nU) break;
+                nit = nc.run_end;
+            }
+            if (nit >= end) nU = nullptr;
+        }
+        RawTile<XT, BT, CK> nxt;
+        if (nU) {
+            const TensorDesc& nd = P.tens[nc.t];
+            nxt.load(P.xptr[nc.i * P.n_tensors + nc.t], nd.base, (nc.g - nd.tile_base) * TILE, nd.numel, lane);
+        }
+
+        // process the current tile
+        if (U != au) {
+            flush();
+            au = U;
+            lo = U->lo;
+            hi = U->hi;
+            want_gamma = U->want_gamma != 0;
+            cap = U->cand_cap;
+            coff = U->cand_off;
+            ch_left = 0;
+            ovf = false;
+        }
+        const TensorDesc& d = P.tens[c.t];
+        const long long n = d.numel;
+        const long long e0 = (c.g - d.tile_base) * TILE;
         uint32_t n_gt = 0, n_hi = 0, n_lo = 0, n_int = 0;
         bool bad = false;
-        double gacc = 0.0;
+        const uint32_t span = hi - lo;
+        float f_gg = 0.0f, f_gi = 0.0f;   // this tile's sums of tau^2, <= 32 terms per lane
+        const bool full = e0 + TILE <= n;
 #pragma unroll
-        for (int v = 0; v < NVEC; ++v) {
-            const long long e = e0 + v * (TPB * VEC) + threadIdx.x * VEC;
+        for (int v = 0; v < WVEC; ++v) {
             float tau[VEC];
-            if (e < n) {
-                TauSrc<XT, BT, CKPT>::load8(x, d.base, e, n, tau);
-            } else {
-#pragma unroll
-                for (int j = 0; j < VEC; ++j) tau[j] = 0.0f;
-            }
+            cur.tau(v, tau);
+            const long long e = e0 + v * (32 * VEC) + lane * VEC;
 #pragma unroll
             for (int j = 0; j < VEC; ++j) {
                 const uint32_t kk = key_of(tau[j]);
-                const bool valid = e + j < n;
-                keys[v][j] = valid ? kk : 0xFFFFFFFFu;   // sentinel: not counted
-                if (!valid) continue;
-                bad |= kk >= KEY_INF;
-                if (kk > hi) {
-                    n_gt++;
-                    if (want_gamma) gacc += (double)tau[j] * (double)tau[j];
-                } else if (kk == hi) n_hi++;
-                else if (kk == lo) n_lo++;
-                else if (kk > lo) n_int++;
+                const bool ok = full || (e + j < n);
+                const bool gt = ok && kk > hi;
+                const bool band = ok && (kk - lo) <= span;     // lo <= kk <= hi
+                n_gt += gt;
+                bad |= ok && kk >= KEY_INF;
+                if (want_gamma) f_gg = __fmaf_rn(gt ? tau[j] : 0.0f, tau[j], f_gg);
+                if (band) {
+                    const bool eh = kk == hi, el = kk == lo;
+                    n_hi += eh;
+                    n_lo += el && !eh;
+                    const bool in = !eh && !el;
+                    n_int += in;
+                    if (want_gamma && in) f_gi = __fmaf_rn(tau[j], tau[j], f_gi);
+                }
             }
         }
-        if (bad) set_status(P.hdr, ISO_ERR_NONFINITE);
-        unsigned long long packed = (unsigned long long)n_gt | ((unsigned long long)n_hi << 16) |
-                                    ((unsigned long long)n_lo << 32) | ((unsigned long long)n_int << 48);
+        if (want_gamma) { l_gg += (double)f_gg; l_gi += (double)f_gi; }
+        if (__any_sync(0xFFFFFFFFu, bad) && lane == 0) set_status(P.hdr, ISO_ERR_NONFINITE);
+        const unsigned long long packed = (unsigned long long)n_gt | ((unsigned long long)n_hi << 16) |
+                                          ((unsigned long long)n_lo << 32);
+        const unsigned long long tot = warp_sum(packed);
         uint32_t int_total;
-        const uint32_t my_off = block_excl_scan(n_int, s_scan, &int_total);
-        const unsigned long long tot = block_sum(packed, s_red);
-        double gtot = 0.0;
-        if (want_gamma) gtot = block_sum(gacc, s_dred);
-        if (threadIdx.x == 0) {
-            const uint32_t t_gt = (uint32_t)(tot & 0xFFFF), t_hi = (uint32_t)((tot >> 16) & 0xFFFF);
-            const uint32_t t_lo = (uint32_t)((tot >> 32) & 0xFFFF);
-            if (t_gt) atomicAdd(&U->c_gt, (unsigned long long)t_gt);
-            if (t_hi) atomicAdd(&U->c_hi, (unsigned long long)t_hi);
-            if (t_lo) atomicAdd(&U->c_lo, (unsigned long long)t_lo);
-            if (want_gamma && gtot != 0.0) atomicAdd(&U->gamma_acc, gtot);
-            unsigned long long slot = 0;
-            if (int_total) slot = atomicAdd(&U->n_int, (unsigned long long)int_total);
-            const int ok = (slot + int_total <= U->cand_cap) ? 1 : 0;
-            TileRec r;
-            r.start = (uint32_t)slot;
-            r.count = ok ? int_total : 0u;
-            r.eq_lo = t_lo;
-            r.eq_hi = t_hi;
-            P.trec[(long long)i * P.n_tiles + g] = r;
-            s_slot = (uint32_t)slot;
-            s_ok = ok;
+        const uint32_t off = warp_excl_scan(n_int, &int_total);
+        const uint32_t t_gt = (uint32_t)(tot & 0xFFFF), t_hi = (uint32_t)((tot >> 16) & 0xFFFF);
+        const uint32_t t_lo = (uint32_t)((tot >> 32) & 0xFFFF);
+        if (int_total > ch_left && !ovf) {
+            unsigned long long start = 0;
+            uint32_t req = 0;
+            if (lane == 0) {
+                const long long run_end = c.run_end < end ? c.run_end : end;
+                const long long left = run_end - c.it;
+                const unsigned long long want = (unsigned long long)int_total * (unsigned long long)left;
+                req = (uint32_t)max((unsigned long long)int_total, min((unsigned long long)CHUNK_MAX, want));
+                start = atomicAdd(&U->n_alloc, (unsigned long long)req);
+            }
+            start = __shfl_sync(0xFFFFFFFFu, start, 0);
+            req = __shfl_sync(0xFFFFFFFFu, req, 0);
+            if (start + req > cap) {
+                ovf = true;
+                ch_left = 0;
+            } else {
+                ch_pos = start;
+                ch_left = req;
+            }
         }
-        __syncthreads();
-        if (s_ok && n_int) {
-            uint32_t* dst = P.cand + U->cand_off + s_slot + my_off;
+        const bool store = !ovf && int_total > 0;
+        if (store && n_int) {
+            uint32_t* dst = P.cand + coff + ch_pos + off;
             uint32_t w = 0;
 #pragma unroll
-            for (int v = 0; v < NVEC; ++v)
+            for (int v = 0; v < WVEC; ++v) {
+                float tau[VEC];
+                cur.tau(v, tau);
+                const long long e = e0 + v * (32 * VEC) + lane * VEC;
 #pragma unroll
                 for (int j = 0; j < VEC; ++j) {
-                    const uint32_t kk = keys[v][j];
-                    if (kk != 0xFFFFFFFFu && kk < hi && kk > lo) dst[w++] = kk;
+                    const uint32_t kk = key_of(tau[j]);
+                    if (e + j < n && kk < hi && kk > lo) dst[w++] = kk;
                 }
+            }
         }
-        __syncthreads();
+        if (lane == 0) {
+            TileRec r;
+            r.start = store ? (uint32_t)ch_pos : 0u;
+            r.count = store ? int_total : 0u;
+            r.eq_lo = t_lo;
+            r.eq_hi = t_hi;
+            P.trec[(long long)c.i * P.n_tiles + c.g] = r;
+        }
+        if (store) { ch_pos += int_total; ch_left -= int_total; }
+        a_gt += t_gt; a_hi += t_hi; a_lo += t_lo; a_int += int_total;
+
+        if (!nU) break;
+        c = nc;
+        U = nU;
+        cur = nxt;
     }
+    flush();
 }
 
 // ---------------------------------------------------------------------------
@@ -314,19 +462,18 @@ __global__ void k_decide(Plan P) {
     const long long c_lo = (long long)U.c_lo, n_int = (long long)U.n_int;
     long long r = U.k - c_gt;
     bool miss = false;
+    U.r_src = SRC_CAND;
     if (r <= 0) {
         miss = true;
     } else if (r <= c_hi) {
         U.t = U.hi; U.count_above = c_gt; U.ties = c_hi; U.need = r; U.tie_src = TIE_EQ_HI;
-        U.r_src = SRC_CAND;
         U.state = ST_TKNOWN;
     } else {
         r -= c_hi;
         if (r <= n_int) {
-            if ((unsigned long long)n_int > U.cand_cap) {
+            if (U.overflow) {
                 miss = true;
             } else {
-                U.r_src = SRC_CAND;
                 U.r_base = U.lo;
                 U.r_pshift = bitlen32(U.hi - U.lo);
                 U.r_prefix = 0;
@@ -339,7 +486,6 @@ __global__ void k_decide(Plan P) {
             if (r <= c_lo) {
                 U.t = U.lo; U.count_above = c_gt + c_hi + n_int; U.ties = c_lo; U.need = r;
                 U.tie_src = TIE_EQ_LO;
-                U.r_src = SRC_CAND;
                 U.state = ST_TKNOWN;
             } else {
                 miss = true;
@@ -349,7 +495,6 @@ __global__ void k_decide(Plan P) {
     if (miss) {
         // exact fallback: radix select over every entry of the unit
         U.fallback = 1;
-        U.gamma_acc = 0.0;
         U.r_src = SRC_DATA;
         U.r_base = 0;
         U.r_pshift = 31;
@@ -358,80 +503,101 @@ __global__ void k_decide(Plan P) {
         U.r_above = 0;
         U.state = ST_RADIX;
     }
-    if (U.state == ST_RADIX) atomicAdd(&P.hdr->n_radix, 1);
-    else atomicAdd(&P.hdr->n_tknown, 1);
+    if (U.state == ST_RADIX) {
+        atomicAdd(&P.hdr->n_radix, 1);
+    } else {
+        atomicAdd(&P.hdr->n_tknown, 1);
+    }
 }
 
 // ---------------------------------------------------------------------------
-// radix levels
+// radix levels: one block per contiguous item range, a shared-memory
+// histogram per (unit, run) flushed to the unit's global histogram
 // ---------------------------------------------------------------------------
-template <typename XT, typename BT, bool CKPT>
+template <typename XT, typename BT, bool CK>
 __global__ void __launch_bounds__(TPB) k_radix_hist(Plan P) {
     __shared__ uint32_t s_hist[RADIX_BINS];
+    __shared__ double s_fh[RADIX_BINS];
     if (*(volatile int32_t*)&P.hdr->n_radix == 0) return;
     const long long items = (long long)P.K * P.n_tiles;
     const long long per = (items + gridDim.x - 1) / gridDim.x;
-    const long long it0 = blockIdx.x * per;
-    const long long it1 = (it0 + per < items) ? it0 + per : items;
-    long long cur = -1;
-    int cur_nb = 0;
-    for (int b = threadIdx.x; b < RADIX_BINS; b += blockDim.x) s_hist[b] = 0;
+    const long long beg = blockIdx.x * per;
+    const long long end = (beg + per < items) ? beg + per : items;
+    for (int b = threadIdx.x; b < RADIX_BINS; b += blockDim.x) { s_hist[b] = 0; s_fh[b] = 0.0; }
     __syncthreads();
-    for (long long it = it0; it < it1; ++it) {
-        const int i = (int)(it / P.n_tiles);
-        const long long g = it % P.n_tiles;
-        const int t = tensor_of_tile(P.tens, P.n_tensors, g);
-        const TensorDesc& d = P.tens[t];
-        if (!(d.flags & TF_TRIM)) continue;
-        Unit* U = unit_of_tile(P, i, d);
-        if (U->state != ST_RADIX) continue;
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    long long it = beg;
+    while (it < end) {
+        Cursor c;
+        cursor_at(P, it, c);
+        const long long run_end = c.run_end < end ? c.run_end : end;
+        const TensorDesc& d = P.tens[c.t];
+        Unit* U = (d.flags & TF_TRIM) ? unit_of(P, c.i, d) : nullptr;
+        if (!U || U->state != ST_RADIX) { it = run_end; continue; }
         const long long ui = U - P.units;
         const int pshift = U->r_pshift;
         const int shift = pshift > RADIX_BITS ? pshift - RADIX_BITS : 0;
         const int nb = 1 << (pshift - shift);
-        if (ui != cur) {
-            __syncthreads();
-            if (cur >= 0)
-                for (int b = threadIdx.x; b < cur_nb; b += blockDim.x)
-                    if (s_hist[b]) { atomicAdd(&P.hist[cur * RADIX_BINS + b], s_hist[b]); s_hist[b] = 0; }
-            __syncthreads();
-            cur = ui;
-            cur_nb = nb;
-        }
         const uint32_t base = U->r_base, prefix = U->r_prefix;
+        const bool wg = U->want_gamma != 0;
+        const long long ntile = run_end - it;
         if (U->r_src == SRC_CAND) {
-            const TileRec r = P.trec[(long long)i * P.n_tiles + g];
-            const uint32_t* c = P.cand + U->cand_off + r.start;
-            for (uint32_t j = threadIdx.x; j < r.count; j += blockDim.x) {
-                const uint32_t v = c[j] - base;
-                if ((v >> pshift) == prefix) atomicAdd(&s_hist[(v >> shift) & (nb - 1)], 1u);
+            // one tile's candidate list per thread
+            for (long long q = threadIdx.x; q < ntile; q += blockDim.x) {
+                const TileRec r = P.trec[(long long)c.i * P.n_tiles + c.g + q];
+                const uint32_t* cp = P.cand + U->cand_off + r.start;
+                for (uint32_t j = 0; j < r.count; ++j) {
+                    const uint32_t kk = cp[j];
+                    const uint32_t v = kk - base;
+                    if ((v >> pshift) == prefix) {
+                        const int bin = (v >> shift) & (nb - 1);
+                        atomicAdd(&s_hist[bin], 1u);
+                        if (wg) atomicAdd(&s_fh[bin], sq(kk));
+                    }
+                }
             }
         } else {
-            const void* x = P.xptr[i * P.n_tensors + t];
-            const long long e0 = (g - d.tile_base) * TILE;
+            // full data, one tile per warp
+            const void* x = P.xptr[c.i * P.n_tensors + c.t];
+            for (long long q = warp; q < ntile; q += WPB) {
+                RawTile<XT, BT, CK> rt;
+                const long long e0 = (c.g + q - d.tile_base) * TILE;
+                rt.load(x, d.base, e0, d.numel, lane);
 #pragma unroll
-            for (int v = 0; v < NVEC; ++v) {
-                const long long e = e0 + v * (TPB * VEC) + threadIdx.x * VEC;
-                if (e >= d.numel) continue;
-                float tau[VEC];
-                TauSrc<XT, BT, CKPT>::load8(x, d.base, e, d.numel, tau);
+                for (int v = 0; v < WVEC; ++v) {
+                    float tau[VEC];
+                    rt.tau(v, tau);
+                    const long long e = e0 + v * (32 * VEC) + lane * VEC;
 #pragma unroll
-                for (int j = 0; j < VEC; ++j) {
-                    if (e + j >= d.numel) continue;
-                    const uint32_t kk = key_of(tau[j]);
-                    if ((kk >> pshift) == prefix) atomicAdd(&s_hist[(kk >> shift) & (nb - 1)], 1u);
+                    for (int j = 0; j < VEC; ++j) {
+                        if (e + j >= d.numel) continue;
+                        const uint32_t kk = key_of(tau[j]);
+                        if ((kk >> pshift) == prefix) {
+                            const int bin = (kk >> shift) & (nb - 1);
+                            atomicAdd(&s_hist[bin], 1u);
+                            if (wg) atomicAdd(&s_fh[bin], (double)tau[j] * (double)tau[j]);
+                        }
+                    }
                 }
             }
         }
+        __syncthreads();
+        for (int b = threadIdx.x; b < nb; b += blockDim.x) {
+            if (s_hist[b]) {
+                atomicAdd(&P.hist[ui * RADIX_BINS + b], s_hist[b]);
+                if (wg) atomicAdd(&P.fhist[ui * RADIX_BINS + b], s_fh[b]);
+                s_hist[b] = 0;
+                s_fh[b] = 0.0;
+            }
+        }
+        __syncthreads();
+        it = run_end;
     }
-    __syncthreads();
-    if (cur >= 0)
-        for (int b = threadIdx.x; b < cur_nb; b += blockDim.x)
-            if (s_hist[b]) atomicAdd(&P.hist[cur * RADIX_BINS + b], s_hist[b]);
 }
 
 __global__ void __launch_bounds__(TPB) k_radix_pick(Plan P) {
     __shared__ long long s_scan[33];
+    __shared__ double s_dred[33];
     __shared__ int s_bin;
     __shared__ long long s_above;
     Unit& U = P.units[blockIdx.x];
@@ -444,9 +610,19 @@ __global__ void __launch_bounds__(TPB) k_radix_pick(Plan P) {
     const int b = s_bin;
     const long long above = s_above;
     const uint32_t cnt = h[b];
+    double fa = 0.0;
+    if (U.want_gamma) {
+        double* fh = P.fhist + (long long)blockIdx.x * RADIX_BINS;
+        double loc = 0.0;
+        for (int q = b + 1 + threadIdx.x; q < nb; q += blockDim.x) loc += fh[q];
+        fa = block_sum(loc, s_dred);
+        __syncthreads();
+        for (int q = threadIdx.x; q < nb; q += blockDim.x) fh[q] = 0.0;
+    }
     __syncthreads();
     for (int q = threadIdx.x; q < nb; q += blockDim.x) h[q] = 0;
     if (threadIdx.x == 0) {
+        U.gamma_rad += fa;
         U.r_rank -= above;
         U.r_above += above;
         U.r_prefix = (U.r_prefix << (pshift - shift)) | (uint32_t)b;
@@ -466,71 +642,58 @@ __global__ void __launch_bounds__(TPB) k_radix_pick(Plan P) {
 }
 
 // ---------------------------------------------------------------------------
-// ties per tile and the sum of squares of the kept entries
+// per-tile counts of keys == t (interior thresholds with partial ties)
 // ---------------------------------------------------------------------------
-__device__ __forceinline__ bool tie_pass_needed(const Unit& U, bool* count, bool* gamma) {
-    *count = (U.tie_src == TIE_ARRAY) && (U.need < U.ties);
-    *gamma = U.want_gamma && (U.tie_src != TIE_EQ_HI);
-    return *count || *gamma;
-}
-
-template <typename XT, typename BT, bool CKPT>
+template <typename XT, typename BT, bool CK>
 __global__ void __launch_bounds__(TPB) k_tie(Plan P) {
-    __shared__ uint32_t s_red[33];
-    __shared__ double s_dred[33];
     if (*(volatile int32_t*)&P.hdr->n_tknown == 0) return;
     const long long items = (long long)P.K * P.n_tiles;
-    for (long long it = blockIdx.x; it < items; it += gridDim.x) {
-        const int i = (int)(it / P.n_tiles);
-        const long long g = it % P.n_tiles;
-        const int t = tensor_of_tile(P.tens, P.n_tensors, g);
-        const TensorDesc& d = P.tens[t];
-        if (!(d.flags & TF_TRIM)) continue;
-        Unit* U = unit_of_tile(P, i, d);
-        if (U->state != ST_TKNOWN) continue;
-        bool want_count, want_gamma;
-        if (!tie_pass_needed(*U, &want_count, &want_gamma)) continue;
+    const long long per = (items + gridDim.x - 1) / gridDim.x;
+    const long long beg = blockIdx.x * per;
+    const long long end = (beg + per < items) ? beg + per : items;
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    long long it = beg;
+    while (it < end) {
+        Cursor c;
+        cursor_at(P, it, c);
+        const long long run_end = c.run_end < end ? c.run_end : end;
+        const TensorDesc& d = P.tens[c.t];
+        Unit* U = (d.flags & TF_TRIM) ? unit_of(P, c.i, d) : nullptr;
+        if (!U || U->state != ST_TKNOWN || U->tie_src != TIE_ARRAY || U->need >= U->ties) {
+            it = run_end;
+            continue;
+        }
         const uint32_t tk = U->t;
-        uint32_t cnt = 0;
-        double gacc = 0.0;
+        const long long ntile = run_end - it;
+        uint32_t* tc = P.tcnt + (long long)c.i * P.n_tiles + c.g;
         if (U->r_src == SRC_CAND) {
-            const TileRec r = P.trec[(long long)i * P.n_tiles + g];
-            const uint32_t* c = P.cand + U->cand_off + r.start;
-            for (uint32_t j = threadIdx.x; j < r.count; j += blockDim.x) {
-                const uint32_t kk = c[j];
-                cnt += (kk == tk);
-                if (want_gamma && kk > tk) {
-                    const double f = (double)__uint_as_float(kk);
-                    gacc += f * f;
-                }
+            for (long long q = threadIdx.x; q < ntile; q += blockDim.x) {
+                const TileRec r = P.trec[(long long)c.i * P.n_tiles + c.g + q];
+                const uint32_t* cp = P.cand + U->cand_off + r.start;
+                uint32_t cnt = 0;
+                for (uint32_t j = 0; j < r.count; ++j) cnt += (cp[j] == tk);
+                tc[q] = cnt;
             }
         } else {
-            const void* x = P.xptr[i * P.n_tensors + t];
-            const long long e0 = (g - d.tile_base) * TILE;
+            const void* x = P.xptr[c.i * P.n_tensors + c.t];
+            for (long long q = warp; q < ntile; q += WPB) {
+                RawTile<XT, BT, CK> rt;
+                const long long e0 = (c.g + q - d.tile_base) * TILE;
+                rt.load(x, d.base, e0, d.numel, lane);
+                uint32_t cnt = 0;
 #pragma unroll
-            for (int v = 0; v < NVEC; ++v) {
-                const long long e = e0 + v * (TPB * VEC) + threadIdx.x * VEC;
-                if (e >= d.numel) continue;
-                float tau[VEC];
-                TauSrc<XT, BT, CKPT>::load8(x, d.base, e, d.numel, tau);
+                for (int v = 0; v < WVEC; ++v) {
+                    float tau[VEC];
+                    rt.tau(v, tau);
+                    const long long e = e0 + v * (32 * VEC) + lane * VEC;
 #pragma unroll
-                for (int j = 0; j < VEC; ++j) {
-                    if (e + j >= d.numel) continue;
-                    const uint32_t kk = key_of(tau[j]);
-                    cnt += (kk == tk);
-                    if (want_gamma && kk > tk) gacc += (double)tau[j] * (double)tau[j];
+                    for (int j = 0; j < VEC; ++j) cnt += (e + j < d.numel && key_of(tau[j]) == tk);
                 }
+                cnt = warp_sum(cnt);
+                if (lane == 0) tc[q] = cnt;
             }
         }
-        if (want_count) {
-            const uint32_t tot = block_sum(cnt, s_red);
-            if (threadIdx.x == 0) P.tcnt[(long long)i * P.n_tiles + g] = tot;
-        }
-        if (want_gamma) {
-            const double gt = block_sum(gacc, s_dred);
-            if (threadIdx.x == 0 && gt != 0.0) atomicAdd(&U->gamma_acc2, gt);
-        }
-        __syncthreads();
+        it = run_end;
     }
 }
 
@@ -572,11 +735,12 @@ __global__ void __launch_bounds__(TPB) k_cut(Plan P) {
         const long long per = (nt + blockDim.x - 1) / blockDim.x;
         const long long j0 = U.tile_begin + threadIdx.x * per;
         const long long j1 = (j0 + per < U.tile_end) ? j0 + per : U.tile_end;
+        const long long row = (long long)i * P.n_tiles;
+        const int src = U.tie_src;
         auto tile_ties = [&](long long g) -> long long {
-            const long long q = (long long)i * P.n_tiles + g;
-            if (U.tie_src == TIE_EQ_HI) return P.trec[q].eq_hi;
-            if (U.tie_src == TIE_EQ_LO) return P.trec[q].eq_lo;
-            return P.tcnt[q];
+            if (src == TIE_EQ_HI) return P.trec[row + g].eq_hi;
+            if (src == TIE_EQ_LO) return P.trec[row + g].eq_lo;
+            return P.tcnt[row + g];
         };
         long long local = 0;
         for (long long g = j0; g < j1; ++g) local += tile_ties(g);
@@ -585,73 +749,65 @@ __global__ void __launch_bounds__(TPB) k_cut(Plan P) {
         if (excl < U.need && U.need <= excl + local) {
             long long acc = excl;
             for (long long g = j0; g < j1; ++g) {
-                const long long c = tile_ties(g);
-                if (U.need <= acc + c) { s_tile = g; s_rem = U.need - acc; break; }
-                acc += c;
+                const long long cnt = tile_ties(g);
+                if (U.need <= acc + cnt) { s_tile = g; s_rem = U.need - acc; break; }
+                acc += cnt;
             }
         }
         __syncthreads();
         if (s_tile < U.tile_begin || s_tile >= U.tile_end) {
             // the tie counts do not reach `need`: inconsistent state, keep every tie
             if (threadIdx.x == 0) { set_status(P.hdr, ISO_ERR_CUDA); U.cut = CUT_ALL; }
-            goto finish;
-        }
-        {
-        // 2. inside that tile, the rem-th entry with key == t in index order
-        const long long g = s_tile;
-        const long long rem = s_rem;
-        const int t = tensor_of_tile(P.tens, P.n_tensors, g);
-        const TensorDesc& d = P.tens[t];
-        const void* x = P.xptr[i * P.n_tensors + t];
-        const long long e0 = (g - d.tile_base) * TILE;
-        constexpr int PER = TILE / TPB;   // 32 consecutive entries per thread
-        const long long eb = e0 + (long long)threadIdx.x * PER;
-        uint32_t mine = 0;
-        for (int j = 0; j < PER; j += VEC) {
-            const long long e = eb + j;
-            if (e >= d.numel) break;
-            float tau[VEC];
-            TauSrc<XT, BT, CKPT>::load8(x, d.base, e, d.numel, tau);
-#pragma unroll
-            for (int q = 0; q < VEC; ++q)
-                if (e + q < d.numel && key_of(tau[q]) == U.t) mine++;
-        }
-        uint32_t tot32;
-        const uint32_t before = block_excl_scan(mine, s_scan32, &tot32);
-        if (before < rem && rem <= before + mine) {
-            uint32_t acc = before;
+        } else {
+            // 2. inside that tile, the rem-th entry with key == t in index order:
+            //    4 consecutive entries per thread, ordered block scan
+            const long long g = s_tile;
+            const long long rem = s_rem;
+            const int t = tensor_of_tile(P.tens, P.n_tensors, g);
+            const TensorDesc& d = P.tens[t];
+            const void* x = P.xptr[i * P.n_tensors + t];
+            constexpr int PER = TILE / TPB;
+            const long long eb = (g - d.tile_base) * TILE + (long long)threadIdx.x * PER;
+            uint32_t mine = 0;
             for (int j = 0; j < PER; ++j) {
                 const long long e = eb + j;
-                if (e >= d.numel) break;
-                if (key_of(TauSrc<XT, BT, CKPT>::load1(x, d.base, e)) == U.t) {
-                    if (++acc == rem) {
+                if (e < d.numel && key_of(TauSrc<XT, BT, CKPT>::load1(x, d.base, e)) == U.t) mine++;
+            }
+            uint32_t tot32;
+            const uint32_t before = block_excl_scan(mine, s_scan32, &tot32);
+            if (before < rem && rem <= before + mine) {
+                uint32_t acc = before;
+                for (int j = 0; j < PER; ++j) {
+                    const long long e = eb + j;
+                    if (e >= d.numel) break;
+                    if (key_of(TauSrc<XT, BT, CKPT>::load1(x, d.base, e)) == U.t && ++acc == rem) {
                         s_pos = ((P.scope == ISO_SCOPE_GLOBAL) ? d.uoff : 0) + e;
                         break;
                     }
                 }
             }
-        }
-        __syncthreads();
-        if (threadIdx.x == 0) {
-            if (s_pos < 0) { set_status(P.hdr, ISO_ERR_CUDA); U.cut = CUT_ALL; }
-            else U.cut = s_pos + 1;
-        }
+            __syncthreads();
+            if (threadIdx.x == 0) {
+                if (s_pos < 0) { set_status(P.hdr, ISO_ERR_CUDA); U.cut = CUT_ALL; }
+                else U.cut = s_pos + 1;
+            }
         }
     } else if (threadIdx.x == 0) {
         U.cut = CUT_ALL;
     }
-finish:
     if (threadIdx.x == 0) {
         if (U.want_gamma) {
-            const double ft = (double)__uint_as_float(U.t);
-            const double fh = (double)__uint_as_float(U.hi);
+            // sum of tau^2 over the kept entries
+            const double ft2 = sq(U.t), fh2 = sq(U.hi);
             double g;
             if (U.r_src == SRC_DATA) {
-                g = U.gamma_acc2 + (double)U.need * ft * ft;
+                g = U.gamma_rad + (double)U.need * ft2;
             } else if (U.tie_src == TIE_EQ_HI) {
-                g = U.gamma_acc + (double)U.need * ft * ft;
+                g = U.gamma_acc + (double)U.need * ft2;
+            } else if (U.tie_src == TIE_EQ_LO) {
+                g = U.gamma_acc + (double)U.c_hi * fh2 + U.gamma_int + (double)U.need * ft2;
             } else {
-                g = U.gamma_acc + (double)U.c_hi * fh * fh + U.gamma_acc2 + (double)U.need * ft * ft;
+                g = U.gamma_acc + (double)U.c_hi * fh2 + U.gamma_rad + (double)U.need * ft2;
             }
             U.gamma = g;
         }
