@@ -17,6 +17,11 @@
 namespace iso {
 namespace {
 
+#ifndef ISO_COUNT_BLOCKS_PER_SM
+#define ISO_COUNT_BLOCKS_PER_SM 3
+#endif
+constexpr int COUNT_GRID_PER_SM = ISO_COUNT_BLOCKS_PER_SM;
+
 // ---------------------------------------------------------------------------
 // profiling and launch accounting
 // ---------------------------------------------------------------------------
@@ -206,7 +211,7 @@ unsigned long long cand_cap_of(long long n, double rho) {
 size_t al256(size_t v) { return (v + 255) & ~(size_t)255; }
 
 struct Layout {
-    size_t hdr, units, trec, tcnt, hist, fhist, gram, coef, zero_end;
+    size_t hdr, units, tcand, teq_lo, teq_hi, tcnt, hist, fhist, gram, coef, zero_end;
     size_t tens, xptr, mptr, table_end;
     size_t cand, total;
     long long n_tiles = 0;
@@ -246,8 +251,11 @@ Layout layout_of(const Call& c, int t0, int t1) {
     size_t o = 0;
     L.hdr = o;   o = al256(o + sizeof(Header));
     L.units = o; o = al256(o + (size_t)K * units * sizeof(Unit));
-    L.trec = o;  o = al256(o + (select && scope != ISO_SCOPE_BLOCK ? (size_t)K * tiles * sizeof(TileRec) : 0));
-    L.tcnt = o;  o = al256(o + (select && scope != ISO_SCOPE_BLOCK ? (size_t)K * tiles * 4 : 0));
+    const size_t trec = (select && scope != ISO_SCOPE_BLOCK) ? (size_t)K * tiles : 0;
+    L.tcand = o;  o = al256(o + trec * 8);
+    L.teq_lo = o; o = al256(o + trec * 4);
+    L.teq_hi = o; o = al256(o + trec * 4);
+    L.tcnt = o;   o = al256(o + trec * 4);
     L.hist = o;  o = al256(o + (select && scope != ISO_SCOPE_BLOCK ? (size_t)K * units * RADIX_BINS * 4 : 0));
     const bool want_gamma = select && !c.mask_only && c.op == ISO_OP_ISO && K == 1 && scope == ISO_SCOPE_TENSOR;
     L.fhist = o; o = al256(o + (want_gamma ? (size_t)K * units * RADIX_BINS * 8 : 0));
@@ -383,7 +391,9 @@ int run_group(const Call& c, int t0, int t1, char* ws, cudaStream_t s, const iso
     P.tens = reinterpret_cast<TensorDesc*>(ws + L.tens);
     P.xptr = reinterpret_cast<const void**>(ws + L.xptr);
     P.units = reinterpret_cast<Unit*>(ws + L.units);
-    P.trec = reinterpret_cast<TileRec*>(ws + L.trec);
+    P.tcand = reinterpret_cast<uint2*>(ws + L.tcand);
+    P.teq_lo = reinterpret_cast<uint32_t*>(ws + L.teq_lo);
+    P.teq_hi = reinterpret_cast<uint32_t*>(ws + L.teq_hi);
     P.tcnt = reinterpret_cast<uint32_t*>(ws + L.tcnt);
     P.hist = reinterpret_cast<uint32_t*>(ws + L.hist);
     P.fhist = reinterpret_cast<double*>(ws + L.fhist);
@@ -419,6 +429,7 @@ int run_group(const Call& c, int t0, int t1, char* ws, cudaStream_t s, const iso
 
     const int pgrid = sms * 4;
     const bool select = c.trims && (c.mask_only || c.op != ISO_OP_TA);
+    if ((long long)K * L.n_tiles >= (1LL << 31)) return ISO_ERR_UNSUPPORTED;   // 32-bit item indices
     int gram_mode = GRAM_NONE;
     if (!c.mask_only && c.op == ISO_OP_ISO) {
         if (K == 1 && c.topk.scope == ISO_SCOPE_TENSOR) gram_mode = GRAM_UNIT;
@@ -437,7 +448,7 @@ int run_group(const Call& c, int t0, int t1, char* ws, cudaStream_t s, const iso
             const int smem = (SAMPLE_MAX + 2 * RADIX_BINS) * 4;
             ISO_TRY(smem_optin(k_sample<XT, BT, CK>, smem));
             ISO_TRY(launch(KD_SAMPLE, s, [&] { k_sample<XT, BT, CK><<<KU, SAMPLE_TPB, smem, s>>>(P); }));
-            ISO_TRY(launch(KD_COUNT, s, [&] { k_count<XT, BT, CK><<<pgrid, TPB, 0, s>>>(P); }));
+            ISO_TRY(launch(KD_COUNT, s, [&] { k_count<XT, BT, CK><<<sms * COUNT_GRID_PER_SM, TPB, 0, s>>>(P); }));
             ISO_TRY(launch(KD_DECIDE, s, [&] { k_decide<<<(KU + 255) / 256, 256, 0, s>>>(P); }));
             for (int level = 0; level < 3; ++level) {
                 ISO_TRY(launch(KD_RADIX_HIST, s, [&] { k_radix_hist<XT, BT, CK><<<pgrid, TPB, 0, s>>>(P); }));

@@ -111,12 +111,11 @@ struct Unit {
     double gamma;
 };
 
-struct TileRec {            // per (expert, tile) record of the count pass
-    uint32_t start;         // first interior slot in the unit's candidate segment
-    uint32_t count;         // interior keys stored (0 when the segment overflowed)
-    uint32_t eq_lo;         // keys == lo in this tile
-    uint32_t eq_hi;         // keys == hi in this tile
-};
+// Per (expert, tile) records of the count pass, as separate arrays:
+//   tcand  (first interior slot in the unit's candidate segment, interior keys
+//          stored; count 0 when the segment overflowed)
+//   teq_lo / teq_hi  keys == lo / == hi in the tile
+//   tcnt   keys == t in the tile (interior thresholds only, written by k_tie)
 
 struct Header {             // first bytes of the workspace
     int32_t status;
@@ -131,7 +130,9 @@ struct Plan {
     TensorDesc*   tens;
     const void**  xptr;     // [K][n_tensors] expert data
     Unit*         units;    // [K][n_units]
-    TileRec*      trec;     // [K][n_tiles]
+    uint2*        tcand;    // [K][n_tiles] (start, count) of the tile's interior keys
+    uint32_t*     teq_lo;   // [K][n_tiles]
+    uint32_t*     teq_hi;   // [K][n_tiles]
     uint32_t*     tcnt;     // [K][n_tiles] ties at t per tile
     uint32_t*     hist;     // [K * n_units][RADIX_BINS]
     double*       fhist;    // [K * n_units][RADIX_BINS] sums of tau^2 per bin (K = 1 ISO only)

@@ -265,52 +265,52 @@ __device__ __forceinline__ Unit* count_unit(const Plan& P, const Cursor& c) {
     return (U->state == ST_BAND) ? U : nullptr;
 }
 
-template <typename XT, typename BT, bool CK>
-__global__ void __launch_bounds__(TPB) k_count(Plan P) {
-    const int lane = threadIdx.x & 31;
-    const long long W = (long long)gridDim.x * WPB;
-    const long long wid = (long long)blockIdx.x * WPB + (threadIdx.x >> 5);
-    const long long items = (long long)P.K * P.n_tiles;
-    const long long per = (items + W - 1) / W;
-    const long long beg = wid * per;
-    const long long end = (beg + per < items) ? beg + per : items;
-    if (beg >= end) return;
+// Per entry the pass does only what every entry needs: tau, its key, the
+// count above the band and a band test.  Band keys (lo <= key <= hi, a few
+// per cent of the entries) are staged in shared memory -- lane L's j-th at
+// slot j*32 + L, conflict-free; every key is written and only a band key
+// advances the lane's slot -- and then classified by the warp together: ties
+// at hi, ties at lo, and interior keys, which are compacted with ballots into
+// the unit's candidate segment.
+#ifndef ISO_COUNT_BLOCKS_PER_SM
+#define ISO_COUNT_BLOCKS_PER_SM 3
+#endif
+constexpr int COUNT_BLOCKS_PER_SM = ISO_COUNT_BLOCKS_PER_SM;
 
-    // first valid item
-    Cursor c;
-    cursor_at(P, beg, c);
-    Unit* U = nullptr;
-    for (;;) {
-        U = count_unit(P, c);
-        if (U) break;
-        if (c.run_end >= end) return;
-        cursor_at(P, c.run_end, c);
-    }
-    RawTile<XT, BT, CK> cur;
-    {
-        const TensorDesc& d = P.tens[c.t];
-        cur.load(P.xptr[c.i * P.n_tensors + c.t], d.base, (c.g - d.tile_base) * TILE, d.numel, lane);
-    }
+template <typename XT, typename BT, bool CK>
+__global__ void __launch_bounds__(TPB, COUNT_BLOCKS_PER_SM) k_count(Plan P) {
+    __shared__ uint32_t s_band[WPB][TILE + 32];
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    uint32_t* sbl = s_band[warp] + lane;
+    // item indices fit 32 bits (the host checks K * n_tiles < 2^31)
+    const uint32_t W = gridDim.x * WPB;
+    const uint32_t wid = blockIdx.x * WPB + warp;
+    const uint32_t items = (uint32_t)(P.K * P.n_tiles);
+    const uint32_t per = (items + W - 1) / W;
+    const uint32_t beg = wid * per;
+    const uint32_t end = min(items, beg + per);
+    if (beg >= end) return;
+    const unsigned FULL = 0xFFFFFFFFu;
+    const unsigned lt_mask = (1u << lane) - 1u;
 
     // per-unit accumulators (warp-uniform) and the candidate chunk
     Unit* au = nullptr;
-    unsigned long long a_gt = 0, a_hi = 0, a_lo = 0, a_int = 0;
-    double l_gg = 0.0, l_gi = 0.0;                // per-lane partial sums of tau^2
-    unsigned long long ch_pos = 0;
-    uint32_t ch_left = 0;
+    uint32_t a_gt = 0, a_hi = 0, a_lo = 0, a_int = 0;
+    double d_gg = 0.0, d_gi = 0.0;                // per-lane sums of tau^2
+    uint32_t* cseg = nullptr;                     // the unit's candidate segment
+    uint32_t ch_pos = 0, ch_left = 0, cap = 0;
     bool ovf = false;
-    uint32_t lo = 0, hi = 0;
+    uint32_t lo = 0, hi = 0, span = 0;
     bool want_gamma = false;
-    unsigned long long cap = 0, coff = 0;
 
     auto flush = [&]() {
         if (!au) return;
-        const double gg = warp_sum(l_gg), gi = warp_sum(l_gi);
+        const double gg = warp_sum(d_gg), gi = warp_sum(d_gi);
         if (lane == 0) {
-            if (a_gt) atomicAdd(&au->c_gt, a_gt);
-            if (a_hi) atomicAdd(&au->c_hi, a_hi);
-            if (a_lo) atomicAdd(&au->c_lo, a_lo);
-            if (a_int) atomicAdd(&au->n_int, a_int);
+            if (a_gt) atomicAdd(&au->c_gt, (unsigned long long)a_gt);
+            if (a_hi) atomicAdd(&au->c_hi, (unsigned long long)a_hi);
+            if (a_lo) atomicAdd(&au->c_lo, (unsigned long long)a_lo);
+            if (a_int) atomicAdd(&au->n_int, (unsigned long long)a_int);
             if (want_gamma) {
                 if (gg != 0.0) atomicAdd(&au->gamma_acc, gg);
                 if (gi != 0.0) atomicAdd(&au->gamma_int, gi);
@@ -318,134 +318,163 @@ __global__ void __launch_bounds__(TPB) k_count(Plan P) {
             if (ovf) au->overflow = 1;
         }
         a_gt = a_hi = a_lo = a_int = 0;
-        l_gg = l_gi = 0.0;
+        d_gg = d_gi = 0.0;
     };
 
-    for (;;) {
-        // locate and prefetch the next valid item
-        Cursor nc = c;
-        Unit* nU = nullptr;
-        {
-            long long nit = c.it + 1;
-            while (nit < end) {
-                if (nit >= nc.run_end) cursor_at(P, nit, nc);
-                else { nc.it = nit; nc.g++; }
-                nU = count_unit(P, nc);
-                if (nU) break;
-                nit = nc.run_end;
-            }
-            if (nit >= end) nU = nullptr;
-        }
-        RawTile<XT, BT, CK> nxt;
-        if (nU) {
-            const TensorDesc& nd = P.tens[nc.t];
-            nxt.load(P.xptr[nc.i * P.n_tensors + nc.t], nd.base, (nc.g - nd.tile_base) * TILE, nd.numel, lane);
-        }
-
-        // process the current tile
-        if (U != au) {
-            flush();
-            au = U;
-            lo = U->lo;
-            hi = U->hi;
-            want_gamma = U->want_gamma != 0;
-            cap = U->cand_cap;
-            coff = U->cand_off;
-            ch_left = 0;
-            ovf = false;
-        }
-        const TensorDesc& d = P.tens[c.t];
-        const long long n = d.numel;
-        const long long e0 = (c.g - d.tile_base) * TILE;
-        uint32_t n_gt = 0, n_hi = 0, n_lo = 0, n_int = 0;
-        bool bad = false;
-        const uint32_t span = hi - lo;
-        float f_gg = 0.0f, f_gi = 0.0f;   // this tile's sums of tau^2, <= 32 terms per lane
-        const bool full = e0 + TILE <= n;
-#pragma unroll
-        for (int v = 0; v < WVEC; ++v) {
-            float tau[VEC];
-            cur.tau(v, tau);
-            const long long e = e0 + v * (32 * VEC) + lane * VEC;
-#pragma unroll
-            for (int j = 0; j < VEC; ++j) {
-                const uint32_t kk = key_of(tau[j]);
-                const bool ok = full || (e + j < n);
-                const bool gt = ok && kk > hi;
-                const bool band = ok && (kk - lo) <= span;     // lo <= kk <= hi
-                n_gt += gt;
-                bad |= ok && kk >= KEY_INF;
-                if (want_gamma) f_gg = __fmaf_rn(gt ? tau[j] : 0.0f, tau[j], f_gg);
-                if (band) {
-                    const bool eh = kk == hi, el = kk == lo;
-                    n_hi += eh;
-                    n_lo += el && !eh;
-                    const bool in = !eh && !el;
-                    n_int += in;
-                    if (want_gamma && in) f_gi = __fmaf_rn(tau[j], tau[j], f_gi);
-                }
-            }
-        }
-        if (want_gamma) { l_gg += (double)f_gg; l_gi += (double)f_gi; }
-        if (__any_sync(0xFFFFFFFFu, bad) && lane == 0) set_status(P.hdr, ISO_ERR_NONFINITE);
-        const unsigned long long packed = (unsigned long long)n_gt | ((unsigned long long)n_hi << 16) |
-                                          ((unsigned long long)n_lo << 32);
-        const unsigned long long tot = warp_sum(packed);
-        uint32_t int_total;
-        const uint32_t off = warp_excl_scan(n_int, &int_total);
-        const uint32_t t_gt = (uint32_t)(tot & 0xFFFF), t_hi = (uint32_t)((tot >> 16) & 0xFFFF);
-        const uint32_t t_lo = (uint32_t)((tot >> 32) & 0xFFFF);
-        if (int_total > ch_left && !ovf) {
-            unsigned long long start = 0;
-            uint32_t req = 0;
-            if (lane == 0) {
-                const long long run_end = c.run_end < end ? c.run_end : end;
-                const long long left = run_end - c.it;
-                const unsigned long long want = (unsigned long long)int_total * (unsigned long long)left;
-                req = (uint32_t)max((unsigned long long)int_total, min((unsigned long long)CHUNK_MAX, want));
-                start = atomicAdd(&U->n_alloc, (unsigned long long)req);
-            }
-            start = __shfl_sync(0xFFFFFFFFu, start, 0);
-            req = __shfl_sync(0xFFFFFFFFu, req, 0);
-            if (start + req > cap) {
-                ovf = true;
+    // the current (expert, tensor) run: items [it0, run_end) are tiles g0.. of one tensor
+    uint32_t run_end = beg, it0 = beg, g0 = 0, row = 0, n = 0, tile_base = 0;
+    const void* xp = nullptr;
+    const void* bp = nullptr;
+    uint32_t it = beg;
+    while (it < end) {
+        if (it >= run_end) {
+            Cursor c;
+            cursor_at(P, it, c);
+            run_end = (uint32_t)c.run_end;
+            Unit* U = count_unit(P, c);
+            if (!U) { it = run_end; continue; }
+            const TensorDesc& d = P.tens[c.t];
+            n = (uint32_t)d.numel;
+            tile_base = (uint32_t)d.tile_base;
+            xp = P.xptr[c.i * P.n_tensors + c.t];
+            bp = d.base;
+            it0 = it;
+            g0 = (uint32_t)c.g;
+            row = (uint32_t)(c.i * P.n_tiles);
+            if (U != au) {
+                flush();
+                au = U;
+                lo = U->lo;
+                hi = U->hi;
+                span = hi - lo;
+                want_gamma = U->want_gamma != 0;
+                cap = (uint32_t)U->cand_cap;
+                cseg = P.cand + U->cand_off;
                 ch_left = 0;
-            } else {
-                ch_pos = start;
-                ch_left = req;
+                ovf = false;
             }
         }
-        const bool store = !ovf && int_total > 0;
-        if (store && n_int) {
-            uint32_t* dst = P.cand + coff + ch_pos + off;
-            uint32_t w = 0;
+        const uint32_t g = g0 + (it - it0);
+        const uint32_t e0 = (g - tile_base) * TILE;
+        RawTile<XT, BT, CK> rt;
+        rt.load(xp, bp, e0, n, lane);
+        const bool full = e0 + TILE <= n;
+
+        // pass 1: every entry (a full tile needs no bounds test)
+        uint32_t n_gt = 0, nb = 0, kmax = 0;
+        float f_gg = 0.0f;
+        if (full) {
 #pragma unroll
             for (int v = 0; v < WVEC; ++v) {
                 float tau[VEC];
-                cur.tau(v, tau);
-                const long long e = e0 + v * (32 * VEC) + lane * VEC;
+                rt.tau(v, tau);
 #pragma unroll
                 for (int j = 0; j < VEC; ++j) {
                     const uint32_t kk = key_of(tau[j]);
-                    if (e + j < n && kk < hi && kk > lo) dst[w++] = kk;
+                    kmax = max(kmax, kk);
+                    const bool gt = kk > hi;
+                    n_gt += gt;
+                    if (want_gamma && gt) f_gg = __fmaf_rn(tau[j], tau[j], f_gg);
+                    sbl[nb * 32] = kk;
+                    nb += (kk - lo <= span);
+                }
+            }
+        } else {
+#pragma unroll
+            for (int v = 0; v < WVEC; ++v) {
+                float tau[VEC];
+                rt.tau(v, tau);
+                const uint32_t e = e0 + v * (32 * VEC) + lane * VEC;
+#pragma unroll
+                for (int j = 0; j < VEC; ++j) {
+                    if (e + j >= n) continue;
+                    const uint32_t kk = key_of(tau[j]);
+                    kmax = max(kmax, kk);
+                    const bool gt = kk > hi;
+                    n_gt += gt;
+                    if (want_gamma && gt) f_gg = __fmaf_rn(tau[j], tau[j], f_gg);
+                    sbl[nb * 32] = kk;
+                    nb += (kk - lo <= span);
                 }
             }
         }
-        if (lane == 0) {
-            TileRec r;
-            r.start = store ? (uint32_t)ch_pos : 0u;
-            r.count = store ? int_total : 0u;
-            r.eq_lo = t_lo;
-            r.eq_hi = t_hi;
-            P.trec[(long long)c.i * P.n_tiles + c.g] = r;
-        }
-        if (store) { ch_pos += int_total; ch_left -= int_total; }
-        a_gt += t_gt; a_hi += t_hi; a_lo += t_lo; a_int += int_total;
+        if (__any_sync(FULL, kmax >= KEY_INF) && lane == 0) set_status(P.hdr, ISO_ERR_NONFINITE);
+        if (want_gamma) d_gg += (double)f_gg;
+        __syncwarp();
 
-        if (!nU) break;
-        c = nc;
-        U = nU;
-        cur = nxt;
+        // pass 2: the staged band keys, one slot per lane per step
+        const uint32_t qmax = __reduce_max_sync(FULL, nb);
+        uint32_t n_hi = 0, n_lo = 0, t_int = 0, tile_start = 0;
+        float f_gi = 0.0f;
+        bool tile_store = true;
+        for (uint32_t q = 0; q < qmax; ++q) {
+            const bool valid = q < nb;
+            const uint32_t kk = valid ? sbl[q * 32] : 0u;
+            const bool eh = valid && kk == hi;
+            const bool el = valid && kk == lo && !eh;
+            const bool in = valid && !eh && !el;
+            n_hi += eh;
+            n_lo += el;
+            if (want_gamma && in) {
+                const float f = __uint_as_float(kk);
+                f_gi = __fmaf_rn(f, f, f_gi);
+            }
+            const unsigned m = __ballot_sync(FULL, in);
+            if (m) {
+                const uint32_t cnt = __popc(m);
+                if (!ovf && cnt > ch_left) {
+                    // new chunk sized for the rest of the run; a tile's keys stay contiguous
+                    unsigned long long start = 0;
+                    uint32_t req = 0;
+                    if (lane == 0) {
+                        const uint32_t left = min(run_end, end) - it;
+                        const unsigned long long want = (unsigned long long)cnt * 16ull * left;
+                        req = (uint32_t)max((unsigned long long)(t_int + cnt),
+                                            min((unsigned long long)CHUNK_MAX, want));
+                        start = atomicAdd(&au->n_alloc, (unsigned long long)req);
+                    }
+                    start = __shfl_sync(FULL, start, 0);
+                    req = __shfl_sync(FULL, req, 0);
+                    if (start + req > cap) {
+                        ovf = true;
+                        ch_left = 0;
+                    } else {
+                        if (t_int && tile_store) {
+                            __syncwarp();
+                            for (uint32_t w = lane; w < t_int; w += 32)
+                                cseg[start + w] = cseg[ch_pos - t_int + w];
+                            __syncwarp();
+                        }
+                        tile_start = (uint32_t)start;
+                        ch_pos = (uint32_t)start + t_int;
+                        ch_left = req - t_int;
+                    }
+                }
+                if (!ovf) {
+                    if (t_int == 0) tile_start = ch_pos;
+                    if (in) cseg[ch_pos + __popc(m & lt_mask)] = kk;
+                    ch_pos += cnt;
+                    ch_left -= cnt;
+                } else {
+                    tile_store = false;
+                }
+                t_int += cnt;
+            }
+        }
+        if (want_gamma) d_gi += (double)f_gi;
+        const uint32_t t_gt = __reduce_add_sync(FULL, n_gt);
+        const uint32_t t_hi = __reduce_add_sync(FULL, n_hi);
+        const uint32_t t_lo = __reduce_add_sync(FULL, n_lo);
+        const bool store = !ovf && tile_store;
+        if (lane == 0) {
+            const uint32_t q = row + g;
+            P.tcand[q] = make_uint2(store ? tile_start : 0u, store ? t_int : 0u);
+            P.teq_lo[q] = t_lo;
+            P.teq_hi[q] = t_hi;
+        }
+        a_gt += t_gt; a_hi += t_hi; a_lo += t_lo; a_int += t_int;
+        __syncwarp();
+        ++it;
     }
     flush();
 }
@@ -544,9 +573,9 @@ __global__ void __launch_bounds__(TPB) k_radix_hist(Plan P) {
         if (U->r_src == SRC_CAND) {
             // one tile's candidate list per thread
             for (long long q = threadIdx.x; q < ntile; q += blockDim.x) {
-                const TileRec r = P.trec[(long long)c.i * P.n_tiles + c.g + q];
-                const uint32_t* cp = P.cand + U->cand_off + r.start;
-                for (uint32_t j = 0; j < r.count; ++j) {
+                const uint2 r = P.tcand[(long long)c.i * P.n_tiles + c.g + q];
+                const uint32_t* cp = P.cand + U->cand_off + r.x;
+                for (uint32_t j = 0; j < r.y; ++j) {
                     const uint32_t kk = cp[j];
                     const uint32_t v = kk - base;
                     if ((v >> pshift) == prefix) {
@@ -668,10 +697,10 @@ __global__ void __launch_bounds__(TPB) k_tie(Plan P) {
         uint32_t* tc = P.tcnt + (long long)c.i * P.n_tiles + c.g;
         if (U->r_src == SRC_CAND) {
             for (long long q = threadIdx.x; q < ntile; q += blockDim.x) {
-                const TileRec r = P.trec[(long long)c.i * P.n_tiles + c.g + q];
-                const uint32_t* cp = P.cand + U->cand_off + r.start;
+                const uint2 r = P.tcand[(long long)c.i * P.n_tiles + c.g + q];
+                const uint32_t* cp = P.cand + U->cand_off + r.x;
                 uint32_t cnt = 0;
-                for (uint32_t j = 0; j < r.count; ++j) cnt += (cp[j] == tk);
+                for (uint32_t j = 0; j < r.y; ++j) cnt += (cp[j] == tk);
                 tc[q] = cnt;
             }
         } else {
@@ -735,15 +764,12 @@ __global__ void __launch_bounds__(TPB) k_cut(Plan P) {
         const long long per = (nt + blockDim.x - 1) / blockDim.x;
         const long long j0 = U.tile_begin + threadIdx.x * per;
         const long long j1 = (j0 + per < U.tile_end) ? j0 + per : U.tile_end;
-        const long long row = (long long)i * P.n_tiles;
-        const int src = U.tie_src;
-        auto tile_ties = [&](long long g) -> long long {
-            if (src == TIE_EQ_HI) return P.trec[row + g].eq_hi;
-            if (src == TIE_EQ_LO) return P.trec[row + g].eq_lo;
-            return P.tcnt[row + g];
-        };
+        const uint32_t* src = ((U.tie_src == TIE_EQ_HI) ? P.teq_hi : (U.tie_src == TIE_EQ_LO) ? P.teq_lo : P.tcnt) +
+                              (long long)i * P.n_tiles;
+        auto tile_ties = [&](long long g) -> long long { return src[g]; };
         long long local = 0;
-        for (long long g = j0; g < j1; ++g) local += tile_ties(g);
+#pragma unroll 8
+        for (long long g = j0; g < j1; ++g) local += src[g];
         long long total;
         const long long excl = block_excl_scan(local, s_scan, &total);
         if (excl < U.need && U.need <= excl + local) {
