@@ -28,11 +28,12 @@ constexpr int COUNT_GRID_PER_SM = ISO_COUNT_BLOCKS_PER_SM;
 enum Kind {
     KD_UPLOAD, KD_INIT, KD_SAMPLE, KD_COUNT, KD_DECIDE, KD_RADIX_HIST, KD_RADIX_PICK, KD_TIE,
     KD_CUT, KD_BLOCK_SELECT, KD_GRAM, KD_SOLVE, KD_APPLY, KD_MASK, KD_DELTA, KD_STATUS, KD_MEMSET,
-    KD_COUNT_KINDS
+    KD_PATCH, KD_REPAIR, KD_COUNT_KINDS
 };
 const char* kKindNames[KD_COUNT_KINDS] = {
     "upload", "init_units", "sample", "count", "decide", "radix_hist", "radix_pick", "tie",
-    "cut", "block_select", "gram", "solve", "apply", "mask", "delta", "status", "memset"};
+    "cut", "block_select", "gram", "solve", "apply", "mask", "delta", "status", "memset",
+    "patch", "repair"};
 
 std::atomic<uint64_t> g_launches{0};
 
@@ -208,12 +209,33 @@ unsigned long long cand_cap_of(long long n, double rho) {
     return (unsigned long long)std::min(cap, (double)n);
 }
 
+// band-record capacity of one unit for the fused K = 1 pass: the band's rank
+// width (twice its expected size) plus room for exact ties at its edges
+unsigned long long brec_cap_of(long long n, double rho) {
+    if (n <= SAMPLE_MAX) return (unsigned long long)n;
+    double kk = std::floor(rho * (double)n + 0.5);
+    kk = std::min(std::max(kk, 0.0), (double)n);
+    const double q = kk / (double)n;
+    const double S = SAMPLE_MAX;
+    const double band = 2.0 * (SAMPLE_Z * std::sqrt(S * q * (1.0 - q)) + 2.0) / S;
+    const double waste = (double)CHUNK_MAX * (std::ceil((double)n / (TILE * 64.0)) + 2.0);
+    const double cap = 8192.0 + std::ceil((2.0 * band + 0.08) * (double)n) + waste;
+    return (unsigned long long)std::min(cap, (double)n);
+}
+
+// the K = 1 update takes the fused single pass (bf16 base and update, per-tensor units)
+bool fused_path(const Call& c) {
+    return c.K == 1 && !c.mask_only && c.op != ISO_OP_TA && c.topk.scope == ISO_SCOPE_TENSOR &&
+           c.xdt == ISO_BF16 && c.bdt == ISO_BF16 && c.trims;
+}
+
 size_t al256(size_t v) { return (v + 255) & ~(size_t)255; }
 
 struct Layout {
     size_t hdr, units, tcand, teq_lo, teq_hi, tcnt, hist, fhist, gram, coef, zero_end;
     size_t tens, xptr, mptr, table_end;
-    size_t cand, total;
+    size_t tband, repair, cand, brec, total;
+    unsigned long long brec_total = 0;
     long long n_tiles = 0;
     int n_units = 0;
     unsigned long long cand_total = 0;
@@ -244,6 +266,10 @@ Layout layout_of(const Call& c, int t0, int t1) {
         cand = (unsigned long long)K * cand_cap_of(gn, c.topk.density);
     }
     const bool select = c.trims;
+    const bool fused = fused_path(c);
+    if (fused)
+        for (int t = t0; t < t1; ++t)
+            if (tensor_trimmed(c, t)) L.brec_total += brec_cap_of(numel_of(c.x[t]), c.topk.density);
     L.n_tiles = tiles;
     L.n_units = (int)units;
     L.cand_total = select ? cand : 0;
@@ -266,7 +292,10 @@ Layout layout_of(const Call& c, int t0, int t1) {
     L.xptr = o;  o = al256(o + (size_t)K * T * sizeof(void*));
     L.mptr = o;  o = al256(o + (size_t)T * sizeof(void*));
     L.table_end = o;
-    L.cand = o;  o = al256(o + (size_t)L.cand_total * 4);
+    L.tband = o;  o = al256(o + (fused ? (size_t)tiles * 8 : 0));
+    L.repair = o; o = al256(o + (fused ? (size_t)T * 4 : 0));
+    L.cand = o;   o = al256(o + (size_t)L.cand_total * 4);
+    L.brec = o;   o = al256(o + (size_t)L.brec_total * 8);
     L.total = o;
     return L;
 }
@@ -347,7 +376,8 @@ int run_group(const Call& c, int t0, int t1, char* ws, cudaStream_t s, const iso
     uint32_t** mptr = reinterpret_cast<uint32_t**>(blob.data() + (L.mptr - L.tens));
     long long tile = 0, uoff = 0;
     int unit = 0;
-    unsigned long long cand = 0;
+    unsigned long long cand = 0, brec = 0;
+    const bool fused = fused_path(c);
     for (int q = 0; q < T; ++q) {
         const int t = t0 + q;
         const iso_tensor& xt = c.x[t];
@@ -381,6 +411,9 @@ int run_group(const Call& c, int t0, int t1, char* ws, cudaStream_t s, const iso
             d.cand_off = 0;
             d.cand_cap = (c.topk.scope == ISO_SCOPE_GLOBAL) ? cand_cap_of(L.global_n, c.topk.density) : 0;
         }
+        d.brec_off = brec;
+        d.brec_cap = (fused && tensor_trimmed(c, t)) ? brec_cap_of(d.numel, c.topk.density) : 0;
+        brec += d.brec_cap;
         for (int i = 0; i < K; ++i) xptr[i * T + q] = c.x[(size_t)i * c.n + t].data;
         mptr[q] = c.masks ? c.masks[t] : nullptr;
     }
@@ -398,6 +431,9 @@ int run_group(const Call& c, int t0, int t1, char* ws, cudaStream_t s, const iso
     P.hist = reinterpret_cast<uint32_t*>(ws + L.hist);
     P.fhist = reinterpret_cast<double*>(ws + L.fhist);
     P.cand = reinterpret_cast<uint32_t*>(ws + L.cand);
+    P.brec = reinterpret_cast<uint2*>(ws + L.brec);
+    P.tband = reinterpret_cast<uint2*>(ws + L.tband);
+    P.repair = fused ? reinterpret_cast<int32_t*>(ws + L.repair) : nullptr;
     P.gram = reinterpret_cast<double*>(ws + L.gram);
     P.coef = reinterpret_cast<double*>(ws + L.coef);
     P.n_tensors = T;
@@ -448,7 +484,12 @@ int run_group(const Call& c, int t0, int t1, char* ws, cudaStream_t s, const iso
             const int smem = (SAMPLE_MAX + 2 * RADIX_BINS) * 4;
             ISO_TRY(smem_optin(k_sample<XT, BT, CK>, smem));
             ISO_TRY(launch(KD_SAMPLE, s, [&] { k_sample<XT, BT, CK><<<KU, SAMPLE_TPB, smem, s>>>(P); }));
-            ISO_TRY(launch(KD_COUNT, s, [&] { k_count<XT, BT, CK><<<sms * COUNT_GRID_PER_SM, TPB, 0, s>>>(P); }));
+            if (fused) {
+                if (CK) ISO_TRY(launch(KD_COUNT, s, [&] { k_count_apply<true><<<sms * 3, TPB, 0, s>>>(P); }));
+                else ISO_TRY(launch(KD_COUNT, s, [&] { k_count_apply<false><<<sms * 3, TPB, 0, s>>>(P); }));
+            } else {
+                ISO_TRY(launch(KD_COUNT, s, [&] { k_count<XT, BT, CK><<<sms * COUNT_GRID_PER_SM, TPB, 0, s>>>(P); }));
+            }
             ISO_TRY(launch(KD_DECIDE, s, [&] { k_decide<<<(KU + 255) / 256, 256, 0, s>>>(P); }));
             for (int level = 0; level < 3; ++level) {
                 ISO_TRY(launch(KD_RADIX_HIST, s, [&] { k_radix_hist<XT, BT, CK><<<pgrid, TPB, 0, s>>>(P); }));
@@ -479,6 +520,20 @@ int run_group(const Call& c, int t0, int t1, char* ws, cudaStream_t s, const iso
             ISO_TRY(launch(KD_MASK, s, [&] { k_mask<__nv_bfloat16><<<pgrid, TPB, 0, s>>>(P, mdev); }));
         else
             ISO_TRY(launch(KD_MASK, s, [&] { k_mask<float><<<pgrid, TPB, 0, s>>>(P, mdev); }));
+        return ISO_OK;
+    }
+
+    if (fused) {
+        // exact coefficients and repair flags, then the kept band entries, then
+        // the full exact apply of any flagged tensor
+        ISO_TRY(launch(KD_SOLVE, s, [&] { k_solve<<<(T + 127) / 128, 128, 0, s>>>(P, gram_mode); }));
+        if (c.ckpt) {
+            ISO_TRY(launch(KD_PATCH, s, [&] { k_patch<true><<<pgrid, TPB, 0, s>>>(P); }));
+            ISO_TRY(launch(KD_REPAIR, s, [&] { k_repair<true><<<pgrid, TPB, 0, s>>>(P); }));
+        } else {
+            ISO_TRY(launch(KD_PATCH, s, [&] { k_patch<false><<<pgrid, TPB, 0, s>>>(P); }));
+            ISO_TRY(launch(KD_REPAIR, s, [&] { k_repair<false><<<pgrid, TPB, 0, s>>>(P); }));
+        }
         return ISO_OK;
     }
 
@@ -640,6 +695,9 @@ int32_t iso_workspace_size(const iso_tensor* tensors, int32_t n_tensors, int32_t
     c.mask_1d = cfg->mask_1d != 0;
     c.topk = cfg->topk;
     if (c.op == ISO_OP_TA) { c.topk.scope = ISO_SCOPE_TENSOR; c.topk.density = 1.0; }
+    // experts are taken to share the base's dtype: for other combinations the
+    // size reported is an upper bound
+    c.xdt = c.bdt = n_tensors ? tensors[0].dtype : ISO_F32;
     set_trim(c, tensors);
     size_t full = n_tensors ? layout_of(c, 0, n_tensors).total : 256;
     size_t mn = 256;

@@ -19,28 +19,6 @@
 
 namespace iso {
 
-// ---------------------------------------------------------------------------
-// vector load / store with a ragged tail
-// ---------------------------------------------------------------------------
-template <typename T>
-__device__ __forceinline__ void load8_tail(const void* p, long long e, long long n, float (&v)[8]) {
-    if (e + 8 <= n) {
-        Load8<T>::run(p, e, v);
-    } else {
-#pragma unroll
-        for (int j = 0; j < 8; ++j) v[j] = (e + j < n) ? Load8<T>::one(p, e + j) : 0.0f;
-    }
-}
-
-// ---------------------------------------------------------------------------
-// per-entry selection
-// ---------------------------------------------------------------------------
-struct SelParam { uint32_t t; long long cut; };
-
-__device__ __forceinline__ bool kept(uint32_t key, long long pos, const SelParam& s) {
-    return key > s.t || (key == s.t && pos < s.cut);
-}
-
 // BLOCK scope: unit of entry e of tensor d
 __device__ __forceinline__ int block_unit(const Plan& P, const TensorDesc& d, long long row, long long col) {
     return d.unit + (int)(row / P.block_rows) * d.bpr + (int)(col / P.block_cols);
@@ -51,34 +29,6 @@ __device__ __forceinline__ int sgn(float v) { return (v > 0.0f) - (v < 0.0f); }
 // ---------------------------------------------------------------------------
 // apply: one warp per tile, one contiguous tile range per warp
 // ---------------------------------------------------------------------------
-__device__ __forceinline__ void store8(void* p, long long e, long long n, const float (&v)[8], bool bf16) {
-    if (bf16) {
-        __nv_bfloat16* q = static_cast<__nv_bfloat16*>(p) + e;
-        if (e + 8 <= n) {
-            __nv_bfloat162 a = __floats2bfloat162_rn(v[0], v[1]);
-            __nv_bfloat162 b = __floats2bfloat162_rn(v[2], v[3]);
-            __nv_bfloat162 c = __floats2bfloat162_rn(v[4], v[5]);
-            __nv_bfloat162 d = __floats2bfloat162_rn(v[6], v[7]);
-            uint4 u;
-            u.x = *reinterpret_cast<uint32_t*>(&a); u.y = *reinterpret_cast<uint32_t*>(&b);
-            u.z = *reinterpret_cast<uint32_t*>(&c); u.w = *reinterpret_cast<uint32_t*>(&d);
-            __stcs(reinterpret_cast<uint4*>(q), u);
-        } else {
-            for (int j = 0; j < 8; ++j)
-                if (e + j < n) q[j] = __float2bfloat16_rn(v[j]);
-        }
-    } else {
-        float* q = static_cast<float*>(p) + e;
-        if (e + 8 <= n) {
-            __stcs(reinterpret_cast<float4*>(q), make_float4(v[0], v[1], v[2], v[3]));
-            __stcs(reinterpret_cast<float4*>(q) + 1, make_float4(v[4], v[5], v[6], v[7]));
-        } else {
-            for (int j = 0; j < 8; ++j)
-                if (e + j < n) q[j] = v[j];
-        }
-    }
-}
-
 // the K experts' selection parameters and coefficients of one tensor
 struct TensorParams {
     SelParam sp[MAXK];
@@ -474,6 +424,16 @@ __global__ void k_solve(Plan P, int gram_mode) {
         }
     }
     for (int i = 0; i < K; ++i) P.coef[(long long)t * K + i] = c[i];
+    if (P.repair) {
+        // fused K = 1 pass: re-apply in full when the speculative outputs may be wrong
+        const Unit& U = P.units[d.unit];
+        int rep = 0;
+        if ((d.flags & TF_TRIM) && U.state == ST_DONE) {
+            const float a = active ? (float)c[0] : P.lambda;
+            rep = (U.fallback || U.b_overflow || a != k1_spec_coef(P)) ? 1 : 0;
+        }
+        P.repair[t] = rep;
+    }
     const long long tg = P.st_tensor_base + t;
     if (P.st_gram)
         for (int q = 0; q < K * K; ++q) P.st_gram[tg * K * K + q] = G[q];

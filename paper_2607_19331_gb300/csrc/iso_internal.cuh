@@ -39,6 +39,7 @@ constexpr int RADIX_BITS = 11;
 constexpr int RADIX_BINS = 1 << RADIX_BITS;
 constexpr int BLOCK_MAX_ENTRIES = 16384;    // BLOCK scope: entries per unit held on chip
 
+constexpr int MAXK = ISO_MAX_EXPERTS;
 constexpr uint32_t KEY_NONE = 0xFFFFFFFFu;  // threshold of a unit that selects nothing
 constexpr uint32_t KEY_MAX = 0x7FFFFFFFu;   // largest key
 constexpr uint32_t KEY_INF = 0x7F800000u;   // keys >= this are not finite
@@ -62,6 +63,8 @@ struct TensorDesc {
     int32_t     nblocks;     // BLOCK: blocks in this tensor
     unsigned long long cand_off;  // TENSOR: expert 0's candidate segment (expert i adds i*cand_cap)
     unsigned long long cand_cap;
+    unsigned long long brec_off;  // fused K = 1 pass: band-record segment
+    unsigned long long brec_cap;
 };
 
 enum UnitState : int32_t {
@@ -92,6 +95,10 @@ struct Unit {
     unsigned long long n_alloc;         // candidate slots handed out (>= n_int)
     int32_t overflow;                   // the segment could not hold every interior key
     int32_t pad0;
+    unsigned long long b_alloc;         // band-record slots handed out (fused K = 1 pass)
+    unsigned long long brec_off, brec_cap;
+    int32_t b_overflow;                 // the band records did not fit
+    int32_t pad1;
     double gamma_acc;                   // sum tau^2 over key > hi (count pass)
     double gamma_int;                   // sum tau^2 over the interior keys (count pass)
     double gamma_rad;                   // sum tau^2 above the radix-selected bins
@@ -137,6 +144,9 @@ struct Plan {
     uint32_t*     hist;     // [K * n_units][RADIX_BINS]
     double*       fhist;    // [K * n_units][RADIX_BINS] sums of tau^2 per bin (K = 1 ISO only)
     uint32_t*     cand;     // candidate pool
+    uint2*        brec;     // fused K = 1 pass: band records (position, theta_0 bits << 16 | x bits)
+    uint2*        tband;    // fused K = 1 pass: [n_tiles] (start, count) of the tile's band records
+    int32_t*      repair;   // fused K = 1 pass: [n_tensors] tensor needs the full exact apply
     double*       gram;     // [n_tensors][K][K]
     double*       coef;     // [n_tensors][K]
     int32_t n_tensors;
@@ -404,6 +414,118 @@ __device__ __forceinline__ T block_excl_scan(T v, T* sm, T* total) {
     T r = sm[warp] + x - v;
     *total = sm[32];
     return r;
+}
+
+// ---------------------------------------------------------------------------
+// selection helpers shared by the select and fused passes
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ long long k_of_density(double rho, long long n) {
+    // floor(rho n + 1/2) with IEEE products and sums (no contraction)
+    double kk = floor(__dadd_rn(__dmul_rn(rho, (double)n), 0.5));
+    if (kk < 0.0) kk = 0.0;
+    if (kk > (double)n) kk = (double)n;
+    return (long long)kk;
+}
+
+__device__ __forceinline__ int bitlen32(uint32_t v) { return v ? 32 - __clz(v) : 0; }
+
+__device__ __forceinline__ double sq(uint32_t key) {
+    const double f = (double)__uint_as_float(key);
+    return f * f;
+}
+
+// ---------------------------------------------------------------------------
+// (expert, tile) item cursor: items are expert-major, tiles in tensor order
+// ---------------------------------------------------------------------------
+struct Cursor {
+    long long it;        // current item
+    long long run_end;   // first item after the current (expert, tensor) run
+    long long g;         // tile
+    int i, t;            // expert, tensor
+};
+
+__device__ __forceinline__ void cursor_at(const Plan& P, long long it, Cursor& c) {
+    c.it = it;
+    c.i = (int)(it / P.n_tiles);
+    c.g = it - (long long)c.i * P.n_tiles;
+    c.t = tensor_of_tile(P.tens, P.n_tensors, c.g);
+    const TensorDesc& d = P.tens[c.t];
+    c.run_end = (long long)c.i * P.n_tiles + d.tile_base + (d.numel + TILE - 1) / TILE;
+}
+
+__device__ __forceinline__ Unit* unit_of(const Plan& P, int i, const TensorDesc& d) {
+    const int u = (P.scope == ISO_SCOPE_GLOBAL) ? 0 : d.unit;
+    return &P.units[(long long)i * P.n_units + u];
+}
+
+__device__ __forceinline__ Unit* count_unit(const Plan& P, const Cursor& c) {
+    const TensorDesc& d = P.tens[c.t];
+    if (!(d.flags & TF_TRIM)) return nullptr;
+    Unit* U = unit_of(P, c.i, d);
+    return (U->state == ST_BAND) ? U : nullptr;
+}
+
+// ---------------------------------------------------------------------------
+// vector load / store with a ragged tail
+// ---------------------------------------------------------------------------
+template <typename T>
+__device__ __forceinline__ void load8_tail(const void* p, long long e, long long n, float (&v)[8]) {
+    if (e + 8 <= n) {
+        Load8<T>::run(p, e, v);
+    } else {
+#pragma unroll
+        for (int j = 0; j < 8; ++j) v[j] = (e + j < n) ? Load8<T>::one(p, e + j) : 0.0f;
+    }
+}
+
+// ---------------------------------------------------------------------------
+// per-entry selection
+// ---------------------------------------------------------------------------
+struct SelParam { uint32_t t; long long cut; };
+
+__device__ __forceinline__ bool kept(uint32_t key, long long pos, const SelParam& s) {
+    return key > s.t || (key == s.t && pos < s.cut);
+}
+
+__device__ __forceinline__ void store8(void* p, long long e, long long n, const float (&v)[8], bool bf16) {
+    if (bf16) {
+        __nv_bfloat16* q = static_cast<__nv_bfloat16*>(p) + e;
+        if (e + 8 <= n) {
+            __nv_bfloat162 a = __floats2bfloat162_rn(v[0], v[1]);
+            __nv_bfloat162 b = __floats2bfloat162_rn(v[2], v[3]);
+            __nv_bfloat162 c = __floats2bfloat162_rn(v[4], v[5]);
+            __nv_bfloat162 d = __floats2bfloat162_rn(v[6], v[7]);
+            uint4 u;
+            u.x = *reinterpret_cast<uint32_t*>(&a); u.y = *reinterpret_cast<uint32_t*>(&b);
+            u.z = *reinterpret_cast<uint32_t*>(&c); u.w = *reinterpret_cast<uint32_t*>(&d);
+            __stcs(reinterpret_cast<uint4*>(q), u);
+        } else {
+            for (int j = 0; j < 8; ++j)
+                if (e + j < n) q[j] = __float2bfloat16_rn(v[j]);
+        }
+    } else {
+        float* q = static_cast<float*>(p) + e;
+        if (e + 8 <= n) {
+            __stcs(reinterpret_cast<float4*>(q), make_float4(v[0], v[1], v[2], v[3]));
+            __stcs(reinterpret_cast<float4*>(q) + 1, make_float4(v[4], v[5], v[6], v[7]));
+        } else {
+            for (int j = 0; j < 8; ++j)
+                if (e + j < n) q[j] = v[j];
+        }
+    }
+}
+
+// the coefficient a unit has unless its retention system is degenerate:
+// lambda for TIES; for ISO clip(Gamma / (Gamma + ridge)) rounds to
+// clip(1, c_min, c_max) in binary32 whenever Gamma >= 2^25 ridge
+__device__ __forceinline__ float k1_spec_coef(const Plan& P) {
+    if (P.op == ISO_OP_ISO) return (float)fmin(fmax(1.0, P.c_min), P.c_max);
+    return P.lambda;
+}
+
+__device__ __forceinline__ float out_of(float th0, float tau, float a) {
+    const float upd = __fmul_rn(a, tau);
+    return (upd == 0.0f) ? th0 : __fadd_rn(th0, upd);
 }
 
 }  // namespace iso

@@ -6,7 +6,7 @@
 
 namespace iso {
 
-constexpr int MAXK = ISO_MAX_EXPERTS;
+
 
 // select (TENSOR / GLOBAL scope)
 __global__ void k_init_units(Plan P, long long global_n);
@@ -21,6 +21,11 @@ template <typename XT, typename BT, bool CK> __global__ void k_cut(Plan P);
 // select (BLOCK scope)
 constexpr int BLOCK_TPB = 512;
 template <typename XT, typename BT, bool CK> __global__ void k_block_select(Plan P);
+
+// fused K = 1 pass (bf16 base and update)
+template <bool CK> __global__ void k_count_apply(Plan P);
+template <bool CK> __global__ void k_patch(Plan P);
+template <bool CK> __global__ void k_repair(Plan P);
 
 // apply
 template <typename XT, typename BT, bool CK, int KC> __global__ void k_apply(Plan P);

@@ -25,45 +25,6 @@
 
 namespace iso {
 
-__device__ __forceinline__ long long k_of_density(double rho, long long n) {
-    // floor(rho n + 1/2) with IEEE products and sums (no contraction)
-    double kk = floor(__dadd_rn(__dmul_rn(rho, (double)n), 0.5));
-    if (kk < 0.0) kk = 0.0;
-    if (kk > (double)n) kk = (double)n;
-    return (long long)kk;
-}
-
-__device__ __forceinline__ int bitlen32(uint32_t v) { return v ? 32 - __clz(v) : 0; }
-
-__device__ __forceinline__ double sq(uint32_t key) {
-    const double f = (double)__uint_as_float(key);
-    return f * f;
-}
-
-// ---------------------------------------------------------------------------
-// (expert, tile) item cursor: items are expert-major, tiles in tensor order
-// ---------------------------------------------------------------------------
-struct Cursor {
-    long long it;        // current item
-    long long run_end;   // first item after the current (expert, tensor) run
-    long long g;         // tile
-    int i, t;            // expert, tensor
-};
-
-__device__ __forceinline__ void cursor_at(const Plan& P, long long it, Cursor& c) {
-    c.it = it;
-    c.i = (int)(it / P.n_tiles);
-    c.g = it - (long long)c.i * P.n_tiles;
-    c.t = tensor_of_tile(P.tens, P.n_tensors, c.g);
-    const TensorDesc& d = P.tens[c.t];
-    c.run_end = (long long)c.i * P.n_tiles + d.tile_base + (d.numel + TILE - 1) / TILE;
-}
-
-__device__ __forceinline__ Unit* unit_of(const Plan& P, int i, const TensorDesc& d) {
-    const int u = (P.scope == ISO_SCOPE_GLOBAL) ? 0 : d.unit;
-    return &P.units[(long long)i * P.n_units + u];
-}
-
 // ---------------------------------------------------------------------------
 // unit table
 // ---------------------------------------------------------------------------
@@ -93,6 +54,8 @@ __global__ void k_init_units(Plan P, long long global_n) {
         U.tile_end = d.tile_base + (d.numel + TILE - 1) / TILE;
         U.cand_cap = d.cand_cap;
         U.cand_off = d.cand_off + (unsigned long long)i * d.cand_cap;
+        U.brec_cap = d.brec_cap;
+        U.brec_off = d.brec_off;
         trimmed = (d.flags & TF_TRIM) != 0;
     }
     if (!trimmed) {
@@ -258,13 +221,6 @@ __global__ void __launch_bounds__(SAMPLE_TPB) k_sample(Plan P) {
 // ---------------------------------------------------------------------------
 // count pass: one warp per tile, one contiguous item range per warp
 // ---------------------------------------------------------------------------
-__device__ __forceinline__ Unit* count_unit(const Plan& P, const Cursor& c) {
-    const TensorDesc& d = P.tens[c.t];
-    if (!(d.flags & TF_TRIM)) return nullptr;
-    Unit* U = unit_of(P, c.i, d);
-    return (U->state == ST_BAND) ? U : nullptr;
-}
-
 // Per entry the pass does only what every entry needs: tau, its key, the
 // count above the band and a band test.  Band keys (lo <= key <= hi, a few
 // per cent of the entries) are staged in shared memory -- lane L's j-th at
