@@ -21,6 +21,10 @@ namespace {
 #define ISO_COUNT_BLOCKS_PER_SM 3
 #endif
 constexpr int COUNT_GRID_PER_SM = ISO_COUNT_BLOCKS_PER_SM;
+#ifndef ISO_FUSED_BLOCKS_PER_SM
+#define ISO_FUSED_BLOCKS_PER_SM 2
+#endif
+constexpr int FUSED_GRID_PER_SM = ISO_FUSED_BLOCKS_PER_SM;
 
 // ---------------------------------------------------------------------------
 // profiling and launch accounting
@@ -195,8 +199,8 @@ long long blocks_of(const iso_tensor& t, const iso_topk_cfg& c) {
 }
 
 // candidate capacity of one unit of n entries at density rho
-unsigned long long cand_cap_of(long long n, double rho) {
-    if (n <= SAMPLE_MAX) return 0;    // the sample is the whole unit: the band is exact
+unsigned long long cand_cap_of(long long n, double rho, bool quantized) {
+    if (n <= SAMPLE_MAX) return (unsigned long long)n;   // exact band: its ties
     double kk = std::floor(rho * (double)n + 0.5);
     kk = std::min(std::max(kk, 0.0), (double)n);
     const double q = kk / (double)n;
@@ -205,7 +209,11 @@ unsigned long long cand_cap_of(long long n, double rho) {
     // interior keys of the band (twice its expected width), plus what the
     // warps' candidate chunks may leave unused at the end of their ranges
     const double waste = (double)CHUNK_MAX * (std::ceil((double)n / (TILE * 64.0)) + 2.0);
-    const double cap = 8192.0 + std::ceil((2.0 * band + 0.002) * (double)n) + waste;
+    // the band's keys: its rank width (twice the expected size) and room for
+    // runs of exact ties at its edges, which bfloat16-derived task vectors have
+    // (few significant bits) and binary32 ones essentially do not
+    const double ties = quantized ? 0.08 : 0.004;
+    const double cap = 8192.0 + std::ceil((2.0 * band + ties) * (double)n) + waste;
     return (unsigned long long)std::min(cap, (double)n);
 }
 
@@ -223,16 +231,20 @@ unsigned long long brec_cap_of(long long n, double rho) {
     return (unsigned long long)std::min(cap, (double)n);
 }
 
-// the K = 1 update takes the fused single pass (bf16 base and update, per-tensor units)
+// the K = 1 update can take the fused single pass (bf16 base and update,
+// per-tensor units); built in with ISO_ENABLE_FUSED=1
+#ifndef ISO_ENABLE_FUSED
+#define ISO_ENABLE_FUSED 0
+#endif
 bool fused_path(const Call& c) {
-    return c.K == 1 && !c.mask_only && c.op != ISO_OP_TA && c.topk.scope == ISO_SCOPE_TENSOR &&
-           c.xdt == ISO_BF16 && c.bdt == ISO_BF16 && c.trims;
+    return ISO_ENABLE_FUSED && c.K == 1 && !c.mask_only && c.op != ISO_OP_TA &&
+           c.topk.scope == ISO_SCOPE_TENSOR && c.xdt == ISO_BF16 && c.bdt == ISO_BF16 && c.trims;
 }
 
 size_t al256(size_t v) { return (v + 255) & ~(size_t)255; }
 
 struct Layout {
-    size_t hdr, units, tcand, teq_lo, teq_hi, tcnt, hist, fhist, gram, coef, zero_end;
+    size_t hdr, units, tcand, teq_lo, teq_hi, tcnt, hist, hmxc, hmx, gram, coef, zero_end;
     size_t tens, xptr, mptr, table_end;
     size_t tband, repair, cand, brec, total;
     unsigned long long brec_total = 0;
@@ -257,13 +269,13 @@ Layout layout_of(const Call& c, int t0, int t1) {
         if (scope == ISO_SCOPE_BLOCK) units += blocks_of(d, c.topk);
         if (tensor_trimmed(c, t)) {
             gn += n;
-            if (scope == ISO_SCOPE_TENSOR) cand += (unsigned long long)K * cand_cap_of(n, c.topk.density);
+            if (scope == ISO_SCOPE_TENSOR) cand += (unsigned long long)K * cand_cap_of(n, c.topk.density, c.xdt == ISO_BF16);
         }
     }
     if (scope == ISO_SCOPE_TENSOR) units = T;
     if (scope == ISO_SCOPE_GLOBAL) {
         units = 1;
-        cand = (unsigned long long)K * cand_cap_of(gn, c.topk.density);
+        cand = (unsigned long long)K * cand_cap_of(gn, c.topk.density, c.xdt == ISO_BF16);
     }
     const bool select = c.trims;
     const bool fused = fused_path(c);
@@ -283,8 +295,8 @@ Layout layout_of(const Call& c, int t0, int t1) {
     L.teq_hi = o; o = al256(o + trec * 4);
     L.tcnt = o;   o = al256(o + trec * 4);
     L.hist = o;  o = al256(o + (select && scope != ISO_SCOPE_BLOCK ? (size_t)K * units * RADIX_BINS * 4 : 0));
-    const bool want_gamma = select && !c.mask_only && c.op == ISO_OP_ISO && K == 1 && scope == ISO_SCOPE_TENSOR;
-    L.fhist = o; o = al256(o + (want_gamma ? (size_t)K * units * RADIX_BINS * 8 : 0));
+    L.hmxc = o;  o = al256(o + (select && scope != ISO_SCOPE_BLOCK ? (size_t)K * units * RADIX_BINS * 4 : 0));
+    L.hmx = o;   o = al256(o + (select && scope != ISO_SCOPE_BLOCK ? (size_t)K * units * RADIX_BINS * 4 : 0));
     L.gram = o;  o = al256(o + (size_t)T * K * K * 8);
     L.coef = o;  o = al256(o + (size_t)T * K * 8);
     L.zero_end = o;
@@ -403,13 +415,15 @@ int run_group(const Call& c, int t0, int t1, char* ws, cudaStream_t s, const iso
             d.nblocks = 0;
         }
         if (c.topk.scope == ISO_SCOPE_TENSOR) {
-            const unsigned long long cap = tensor_trimmed(c, t) ? cand_cap_of(d.numel, c.topk.density) : 0;
+            const unsigned long long cap =
+                tensor_trimmed(c, t) ? cand_cap_of(d.numel, c.topk.density, c.xdt == ISO_BF16) : 0;
             d.cand_off = cand;
             d.cand_cap = cap;
             cand += (unsigned long long)K * cap;
         } else {
             d.cand_off = 0;
-            d.cand_cap = (c.topk.scope == ISO_SCOPE_GLOBAL) ? cand_cap_of(L.global_n, c.topk.density) : 0;
+            d.cand_cap = (c.topk.scope == ISO_SCOPE_GLOBAL)
+                             ? cand_cap_of(L.global_n, c.topk.density, c.xdt == ISO_BF16) : 0;
         }
         d.brec_off = brec;
         d.brec_cap = (fused && tensor_trimmed(c, t)) ? brec_cap_of(d.numel, c.topk.density) : 0;
@@ -429,7 +443,8 @@ int run_group(const Call& c, int t0, int t1, char* ws, cudaStream_t s, const iso
     P.teq_hi = reinterpret_cast<uint32_t*>(ws + L.teq_hi);
     P.tcnt = reinterpret_cast<uint32_t*>(ws + L.tcnt);
     P.hist = reinterpret_cast<uint32_t*>(ws + L.hist);
-    P.fhist = reinterpret_cast<double*>(ws + L.fhist);
+    P.hmxc = reinterpret_cast<uint32_t*>(ws + L.hmxc);
+    P.hmx = reinterpret_cast<uint32_t*>(ws + L.hmx);
     P.cand = reinterpret_cast<uint32_t*>(ws + L.cand);
     P.brec = reinterpret_cast<uint2*>(ws + L.brec);
     P.tband = reinterpret_cast<uint2*>(ws + L.tband);
@@ -485,8 +500,8 @@ int run_group(const Call& c, int t0, int t1, char* ws, cudaStream_t s, const iso
             ISO_TRY(smem_optin(k_sample<XT, BT, CK>, smem));
             ISO_TRY(launch(KD_SAMPLE, s, [&] { k_sample<XT, BT, CK><<<KU, SAMPLE_TPB, smem, s>>>(P); }));
             if (fused) {
-                if (CK) ISO_TRY(launch(KD_COUNT, s, [&] { k_count_apply<true><<<sms * 3, TPB, 0, s>>>(P); }));
-                else ISO_TRY(launch(KD_COUNT, s, [&] { k_count_apply<false><<<sms * 3, TPB, 0, s>>>(P); }));
+                if (CK) ISO_TRY(launch(KD_COUNT, s, [&] { k_count_apply<true><<<sms * FUSED_GRID_PER_SM, TPB, 0, s>>>(P); }));
+                else ISO_TRY(launch(KD_COUNT, s, [&] { k_count_apply<false><<<sms * FUSED_GRID_PER_SM, TPB, 0, s>>>(P); }));
             } else {
                 ISO_TRY(launch(KD_COUNT, s, [&] { k_count<XT, BT, CK><<<sms * COUNT_GRID_PER_SM, TPB, 0, s>>>(P); }));
             }

@@ -27,7 +27,10 @@ __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
     return *reinterpret_cast<uint32_t*>(&h);
 }
 
-constexpr int FUSED_BLOCKS_PER_SM = 3;
+#ifndef ISO_FUSED_BLOCKS_PER_SM
+#define ISO_FUSED_BLOCKS_PER_SM 2
+#endif
+constexpr int FUSED_BLOCKS_PER_SM = ISO_FUSED_BLOCKS_PER_SM;
 
 template <bool CK>
 __global__ void __launch_bounds__(TPB, FUSED_BLOCKS_PER_SM) k_count_apply(Plan P) {
@@ -52,8 +55,8 @@ __global__ void __launch_bounds__(TPB, FUSED_BLOCKS_PER_SM) k_count_apply(Plan P
 
     // per-unit accumulators and the two segments (interior keys, band records)
     Unit* au = nullptr;
-    uint32_t a_gt = 0, a_hi = 0, a_lo = 0, a_int = 0;
-    double d_gg = 0.0, d_gi = 0.0;
+    uint32_t a_gt = 0, a_int = 0;
+    double d_gg = 0.0;
     uint32_t* cseg = nullptr;
     uint2* bseg = nullptr;
     uint32_t c_pos = 0, c_left = 0, c_cap = 0, b_pos = 0, b_left = 0, b_cap = 0;
@@ -63,21 +66,16 @@ __global__ void __launch_bounds__(TPB, FUSED_BLOCKS_PER_SM) k_count_apply(Plan P
 
     auto flush = [&]() {
         if (!au) return;
-        const double gg = warp_sum(d_gg), gi = warp_sum(d_gi);
+        const double gg = warp_sum(d_gg);
         if (lane == 0) {
             if (a_gt) atomicAdd(&au->c_gt, (unsigned long long)a_gt);
-            if (a_hi) atomicAdd(&au->c_hi, (unsigned long long)a_hi);
-            if (a_lo) atomicAdd(&au->c_lo, (unsigned long long)a_lo);
             if (a_int) atomicAdd(&au->n_int, (unsigned long long)a_int);
-            if (want_gamma) {
-                if (gg != 0.0) atomicAdd(&au->gamma_acc, gg);
-                if (gi != 0.0) atomicAdd(&au->gamma_int, gi);
-            }
+            if (want_gamma && gg != 0.0) atomicAdd(&au->gamma_acc, gg);
             if (c_ovf) au->overflow = 1;
             if (b_ovf) au->b_overflow = 1;
         }
-        a_gt = a_hi = a_lo = a_int = 0;
-        d_gg = d_gi = 0.0;
+        a_gt = a_int = 0;
+        d_gg = 0.0;
     };
 
     // reserve n slots of a segment for one tile; returns false on overflow
@@ -161,7 +159,8 @@ __global__ void __launch_bounds__(TPB, FUSED_BLOCKS_PER_SM) k_count_apply(Plan P
         }
 
         // pass 1: every entry -- counts, band offsets, speculative outputs
-        const bool full = e0 + TILE <= n;
+        // (a ragged last tile reads zeros past the end: key 0 is never above
+        // hi, and a band holding 0 is corrected below)
         uint32_t n_gt = 0, nb = 0, kmax = 0;
         float f_gg = 0.0f;
 #pragma unroll
@@ -175,80 +174,61 @@ __global__ void __launch_bounds__(TPB, FUSED_BLOCKS_PER_SM) k_count_apply(Plan P
 #pragma unroll
             for (int j = 0; j < VEC; ++j) {
                 const uint32_t kk = key_of(tau[j]);
-                const bool ok = full || (e + j < n);
-                const bool gt = ok && kk > hi;
-                kmax = ok ? max(kmax, kk) : kmax;
+                const bool gt = kk > hi;
+                kmax = max(kmax, kk);
                 n_gt += gt;
                 if (want_gamma && gt) f_gg = __fmaf_rn(tau[j], tau[j], f_gg);
                 sol[nb * 32] = (uint16_t)(v * (32 * VEC) + lane * VEC + j);
-                nb += (ok && kk - lo <= span);
+                nb += (kk - lo <= span);
                 o[j] = gt ? out_of(th0[j], tau[j], a_spec) : th0[j];
             }
             if (e < n) store8(op, e, n, o, true);
+        }
+        if (e0 + TILE > n && lo == 0) {
+            // drop the zero-filled entries past the end from the band
+            uint32_t keep = 0;
+            for (uint32_t q = 0; q < nb; ++q) {
+                const uint32_t off = sol[q * 32];
+                if (e0 + off < n) sol[(keep++) * 32] = (uint16_t)off;
+            }
+            nb = keep;
         }
         if (__any_sync(FULL, kmax >= KEY_INF) && lane == 0) set_status(P.hdr, ISO_ERR_NONFINITE);
         if (want_gamma) d_gg += (double)f_gg;
         __syncwarp();
 
-        // pass 2a: classify the band entries
-        const uint32_t qmax = __reduce_max_sync(FULL, nb);
-        uint32_t n_hi = 0, n_lo = 0, n_in = 0;
-        float f_gi = 0.0f;
-        for (uint32_t q = 0; q < qmax; ++q) {
-            if (q >= nb) continue;
-            const uint32_t off = sol[q * 32];
-            const float xv = __uint_as_float((uint32_t)sx[off] << 16);
-            const float bv = __uint_as_float((uint32_t)sbs[off] << 16);
-            const float tau = CK ? __fsub_rn(xv, bv) : xv;
-            const uint32_t kk = key_of(tau);
-            const bool eh = kk == hi, el = kk == lo && !eh;
-            n_hi += eh;
-            n_lo += el;
-            if (!eh && !el) {
-                n_in++;
-                if (want_gamma) f_gi = __fmaf_rn(tau, tau, f_gi);
-            }
-        }
-        if (want_gamma) d_gi += (double)f_gi;
-        uint32_t in_tot, nb_tot;
-        const uint32_t in_off = warp_excl_scan(n_in, &in_tot);
+        // pass 2: the band entries go to the unit's candidate segment (keys)
+        // and to its band records (position and raw values)
+        uint32_t nb_tot;
         const uint32_t nb_off = warp_excl_scan(nb, &nb_tot);
-
-        // pass 2b: slots for this tile's interior keys and band records
         const uint32_t left_tiles = min(run_end, end) - it;
-        if (in_tot && !c_ovf && in_tot > c_left)
-            c_ovf = !reserve(&au->n_alloc, in_tot, c_cap, left_tiles, c_pos, c_left);
+        if (nb_tot && !c_ovf && nb_tot > c_left)
+            c_ovf = !reserve(&au->n_alloc, nb_tot, c_cap, left_tiles, c_pos, c_left);
         if (nb_tot && !b_ovf && nb_tot > b_left)
             b_ovf = !reserve(&au->b_alloc, nb_tot, b_cap, left_tiles, b_pos, b_left);
-        const bool c_store = in_tot && !c_ovf;
+        const bool c_store = nb_tot && !c_ovf;
         const bool b_store = nb_tot && !b_ovf;
-
-        // pass 2c: write them
         if (c_store || b_store) {
-            uint32_t wi = c_pos + in_off, wb = b_pos + nb_off;
+            uint32_t wi = c_pos + nb_off, wb = b_pos + nb_off;
             for (uint32_t q = 0; q < nb; ++q) {
                 const uint32_t off = sol[q * 32];
                 const uint32_t xr = sx[off], br = sbs[off];
                 if (b_store) bseg[wb++] = make_uint2(e0 + off, (br << 16) | xr);
                 if (c_store) {
                     const float xv = __uint_as_float(xr << 16), bv = __uint_as_float(br << 16);
-                    const uint32_t kk = key_of(CK ? __fsub_rn(xv, bv) : xv);
-                    if (kk != hi && kk != lo) cseg[wi++] = kk;
+                    cseg[wi++] = key_of(CK ? __fsub_rn(xv, bv) : xv);
                 }
             }
         }
         const uint32_t t_gt = __reduce_add_sync(FULL, n_gt);
-        const uint32_t t_hi = __reduce_add_sync(FULL, n_hi);
-        const uint32_t t_lo = __reduce_add_sync(FULL, n_lo);
         if (lane == 0) {
-            P.tcand[g] = make_uint2(c_store ? c_pos : 0u, c_store ? in_tot : 0u);
+            P.tcand[g] = make_uint2(c_store ? c_pos : 0u, c_store ? nb_tot : 0u);
             P.tband[g] = make_uint2(b_store ? b_pos : 0u, b_store ? nb_tot : 0u);
-            P.teq_lo[g] = t_lo;
-            P.teq_hi[g] = t_hi;
         }
+        const uint32_t in_tot = nb_tot;
         if (c_store) { c_pos += in_tot; c_left -= in_tot; }
         if (b_store) { b_pos += nb_tot; b_left -= nb_tot; }
-        a_gt += t_gt; a_hi += t_hi; a_lo += t_lo; a_int += in_tot;
+        a_gt += t_gt; a_int += in_tot;
         __syncwarp();
         ++it;
     }

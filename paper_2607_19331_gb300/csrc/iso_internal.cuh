@@ -76,8 +76,8 @@ enum UnitState : int32_t {
     ST_TKNOWN = 5,   // threshold known; cut pending
     ST_DONE = 6
 };
-enum TieSource : int32_t { TIE_EQ_HI = 0, TIE_EQ_LO = 1, TIE_ARRAY = 2 };
 enum RadixSource : int32_t { SRC_CAND = 0, SRC_DATA = 1 };
+enum TieSource : int32_t { TIE_EQ_HI = 0, TIE_EQ_LO = 1, TIE_ARRAY = 2 };
 
 struct Unit {
     // static
@@ -91,17 +91,19 @@ struct Unit {
     // band
     uint32_t lo, hi;
     // count-pass accumulators
-    unsigned long long c_gt, c_hi, c_lo, n_int;
+    unsigned long long c_gt;            // keys above the band
+    unsigned long long n_int;           // keys in the band (the candidates)
+    unsigned long long c_hi, c_lo;      // band keys equal to hi / to lo (lo != hi)
     unsigned long long n_alloc;         // candidate slots handed out (>= n_int)
-    int32_t overflow;                   // the segment could not hold every interior key
+    int32_t overflow;                   // the segment could not hold every band key
     int32_t pad0;
     unsigned long long b_alloc;         // band-record slots handed out (fused K = 1 pass)
     unsigned long long brec_off, brec_cap;
     int32_t b_overflow;                 // the band records did not fit
     int32_t pad1;
     double gamma_acc;                   // sum tau^2 over key > hi (count pass)
-    double gamma_int;                   // sum tau^2 over the interior keys (count pass)
-    double gamma_rad;                   // sum tau^2 above the radix-selected bins
+    double gamma_band;                  // sum tau^2 over the band keys above lo (count pass)
+    double gamma_rad;                   // sum tau^2 over the candidates (or, on the fallback, all entries) above t
     // radix select
     int32_t r_src;
     int32_t r_shift, r_pshift;
@@ -119,10 +121,10 @@ struct Unit {
 };
 
 // Per (expert, tile) records of the count pass, as separate arrays:
-//   tcand  (first interior slot in the unit's candidate segment, interior keys
-//          stored; count 0 when the segment overflowed)
-//   teq_lo / teq_hi  keys == lo / == hi in the tile
-//   tcnt   keys == t in the tile (interior thresholds only, written by k_tie)
+//   tcand  (first slot of the tile's band keys in the unit's candidate
+//          segment, band keys stored; count 0 when the segment overflowed)
+//   teq_lo / teq_hi  band keys == lo / == hi in the tile
+//   tcnt   keys == t in the tile (interior thresholds; written by k_tie)
 
 struct Header {             // first bytes of the workspace
     int32_t status;
@@ -137,12 +139,13 @@ struct Plan {
     TensorDesc*   tens;
     const void**  xptr;     // [K][n_tensors] expert data
     Unit*         units;    // [K][n_units]
-    uint2*        tcand;    // [K][n_tiles] (start, count) of the tile's interior keys
+    uint2*        tcand;    // [K][n_tiles] (start, count) of the tile's band keys
     uint32_t*     teq_lo;   // [K][n_tiles]
     uint32_t*     teq_hi;   // [K][n_tiles]
     uint32_t*     tcnt;     // [K][n_tiles] ties at t per tile
     uint32_t*     hist;     // [K * n_units][RADIX_BINS]
-    double*       fhist;    // [K * n_units][RADIX_BINS] sums of tau^2 per bin (K = 1 ISO only)
+    uint32_t*     hmxc;     // [K * n_units][RADIX_BINS] per bin: max of ~key (its smallest key)
+    uint32_t*     hmx;      // [K * n_units][RADIX_BINS] per bin: largest key
     uint32_t*     cand;     // candidate pool
     uint2*        brec;     // fused K = 1 pass: band records (position, theta_0 bits << 16 | x bits)
     uint2*        tband;    // fused K = 1 pass: [n_tiles] (start, count) of the tile's band records

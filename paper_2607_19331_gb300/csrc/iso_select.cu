@@ -225,9 +225,8 @@ __global__ void __launch_bounds__(SAMPLE_TPB) k_sample(Plan P) {
 // count above the band and a band test.  Band keys (lo <= key <= hi, a few
 // per cent of the entries) are staged in shared memory -- lane L's j-th at
 // slot j*32 + L, conflict-free; every key is written and only a band key
-// advances the lane's slot -- and then classified by the warp together: ties
-// at hi, ties at lo, and interior keys, which are compacted with ballots into
-// the unit's candidate segment.
+// advances the lane's slot -- and then copied, per lane, to the unit's
+// candidate segment.  The radix select and the tie counts work on that set.
 #ifndef ISO_COUNT_BLOCKS_PER_SM
 #define ISO_COUNT_BLOCKS_PER_SM 3
 #endif
@@ -251,8 +250,8 @@ __global__ void __launch_bounds__(TPB, COUNT_BLOCKS_PER_SM) k_count(Plan P) {
 
     // per-unit accumulators (warp-uniform) and the candidate chunk
     Unit* au = nullptr;
-    uint32_t a_gt = 0, a_hi = 0, a_lo = 0, a_int = 0;
-    double d_gg = 0.0, d_gi = 0.0;                // per-lane sums of tau^2
+    uint32_t a_gt = 0, a_int = 0, a_hi = 0, a_lo = 0;
+    double d_gg = 0.0, d_gb = 0.0;                // per-lane sums of tau^2: above hi, band above lo
     uint32_t* cseg = nullptr;                     // the unit's candidate segment
     uint32_t ch_pos = 0, ch_left = 0, cap = 0;
     bool ovf = false;
@@ -261,20 +260,20 @@ __global__ void __launch_bounds__(TPB, COUNT_BLOCKS_PER_SM) k_count(Plan P) {
 
     auto flush = [&]() {
         if (!au) return;
-        const double gg = warp_sum(d_gg), gi = warp_sum(d_gi);
+        const double gg = warp_sum(d_gg), gb = warp_sum(d_gb);
         if (lane == 0) {
             if (a_gt) atomicAdd(&au->c_gt, (unsigned long long)a_gt);
+            if (a_int) atomicAdd(&au->n_int, (unsigned long long)a_int);
             if (a_hi) atomicAdd(&au->c_hi, (unsigned long long)a_hi);
             if (a_lo) atomicAdd(&au->c_lo, (unsigned long long)a_lo);
-            if (a_int) atomicAdd(&au->n_int, (unsigned long long)a_int);
             if (want_gamma) {
                 if (gg != 0.0) atomicAdd(&au->gamma_acc, gg);
-                if (gi != 0.0) atomicAdd(&au->gamma_int, gi);
+                if (gb != 0.0) atomicAdd(&au->gamma_band, gb);
             }
             if (ovf) au->overflow = 1;
         }
-        a_gt = a_hi = a_lo = a_int = 0;
-        d_gg = d_gi = 0.0;
+        a_gt = a_int = a_hi = a_lo = 0;
+        d_gg = d_gb = 0.0;
     };
 
     // the current (expert, tensor) run: items [it0, run_end) are tiles g0.. of one tensor
@@ -358,77 +357,47 @@ __global__ void __launch_bounds__(TPB, COUNT_BLOCKS_PER_SM) k_count(Plan P) {
         if (want_gamma) d_gg += (double)f_gg;
         __syncwarp();
 
-        // pass 2: the staged band keys, one slot per lane per step
-        const uint32_t qmax = __reduce_max_sync(FULL, nb);
-        uint32_t n_hi = 0, n_lo = 0, t_int = 0, tile_start = 0;
-        float f_gi = 0.0f;
-        bool tile_store = true;
-        for (uint32_t q = 0; q < qmax; ++q) {
-            const bool valid = q < nb;
-            const uint32_t kk = valid ? sbl[q * 32] : 0u;
-            const bool eh = valid && kk == hi;
-            const bool el = valid && kk == lo && !eh;
-            const bool in = valid && !eh && !el;
-            n_hi += eh;
-            n_lo += el;
-            if (want_gamma && in) {
-                const float f = __uint_as_float(kk);
-                f_gi = __fmaf_rn(f, f, f_gi);
+        // pass 2: copy the staged band keys to the unit's candidate segment
+        uint32_t t_int;
+        const uint32_t off = warp_excl_scan(nb, &t_int);
+        if (t_int && !ovf && t_int > ch_left) {
+            unsigned long long start = 0;
+            uint32_t req = 0;
+            if (lane == 0) {
+                const uint32_t left = min(run_end, end) - it;
+                const unsigned long long want = (unsigned long long)t_int * (unsigned long long)left;
+                req = (uint32_t)max((unsigned long long)t_int, min((unsigned long long)CHUNK_MAX, want));
+                start = atomicAdd(&au->n_alloc, (unsigned long long)req);
             }
-            const unsigned m = __ballot_sync(FULL, in);
-            if (m) {
-                const uint32_t cnt = __popc(m);
-                if (!ovf && cnt > ch_left) {
-                    // new chunk sized for the rest of the run; a tile's keys stay contiguous
-                    unsigned long long start = 0;
-                    uint32_t req = 0;
-                    if (lane == 0) {
-                        const uint32_t left = min(run_end, end) - it;
-                        const unsigned long long want = (unsigned long long)cnt * 16ull * left;
-                        req = (uint32_t)max((unsigned long long)(t_int + cnt),
-                                            min((unsigned long long)CHUNK_MAX, want));
-                        start = atomicAdd(&au->n_alloc, (unsigned long long)req);
-                    }
-                    start = __shfl_sync(FULL, start, 0);
-                    req = __shfl_sync(FULL, req, 0);
-                    if (start + req > cap) {
-                        ovf = true;
-                        ch_left = 0;
-                    } else {
-                        if (t_int && tile_store) {
-                            __syncwarp();
-                            for (uint32_t w = lane; w < t_int; w += 32)
-                                cseg[start + w] = cseg[ch_pos - t_int + w];
-                            __syncwarp();
-                        }
-                        tile_start = (uint32_t)start;
-                        ch_pos = (uint32_t)start + t_int;
-                        ch_left = req - t_int;
-                    }
-                }
-                if (!ovf) {
-                    if (t_int == 0) tile_start = ch_pos;
-                    if (in) cseg[ch_pos + __popc(m & lt_mask)] = kk;
-                    ch_pos += cnt;
-                    ch_left -= cnt;
-                } else {
-                    tile_store = false;
-                }
-                t_int += cnt;
+            start = __shfl_sync(FULL, start, 0);
+            req = __shfl_sync(FULL, req, 0);
+            if (start + req > cap) { ovf = true; ch_left = 0; }
+            else { ch_pos = (uint32_t)start; ch_left = req; }
+        }
+        const bool store = t_int && !ovf;
+        uint32_t n_hi = 0, n_lo = 0;
+        float f_band = 0.0f;                      // tau^2 over the band keys above lo
+        {
+            uint32_t* dst = cseg + ch_pos + off;
+            for (uint32_t q = 0; q < nb; ++q) {
+                const uint32_t kk = sbl[q * 32];
+                if (store) dst[q] = kk;
+                n_hi += (kk == hi);
+                n_lo += (kk == lo) && (kk != hi);
+                if (want_gamma && kk != lo) { const float f = __uint_as_float(kk); f_band = __fmaf_rn(f, f, f_band); }
             }
         }
-        if (want_gamma) d_gi += (double)f_gi;
+        if (want_gamma) d_gb += (double)f_band;
         const uint32_t t_gt = __reduce_add_sync(FULL, n_gt);
         const uint32_t t_hi = __reduce_add_sync(FULL, n_hi);
         const uint32_t t_lo = __reduce_add_sync(FULL, n_lo);
-        const bool store = !ovf && tile_store;
         if (lane == 0) {
-            const uint32_t q = row + g;
-            P.tcand[q] = make_uint2(store ? tile_start : 0u, store ? t_int : 0u);
-            P.teq_lo[q] = t_lo;
-            P.teq_hi[q] = t_hi;
+            P.tcand[row + g] = make_uint2(store ? ch_pos : 0u, store ? t_int : 0u);
+            P.teq_lo[row + g] = t_lo;
+            P.teq_hi[row + g] = t_hi;
         }
-        a_gt += t_gt; a_hi += t_hi; a_lo += t_lo; a_int += t_int;
+        if (store) { ch_pos += t_int; ch_left -= t_int; }
+        a_gt += t_gt; a_int += t_int; a_hi += t_hi; a_lo += t_lo;
         __syncwarp();
         ++it;
     }
@@ -443,41 +412,30 @@ __global__ void k_decide(Plan P) {
     if (idx >= P.K * P.n_units) return;
     Unit& U = P.units[idx];
     if (U.state != ST_BAND) return;
-    const long long c_gt = (long long)U.c_gt, c_hi = (long long)U.c_hi;
-    const long long c_lo = (long long)U.c_lo, n_int = (long long)U.n_int;
-    long long r = U.k - c_gt;
-    bool miss = false;
+    // rank k counted from the top: c_gt keys lie above the band, then the
+    // band's n_int keys: c_hi equal to hi, the interior, c_lo equal to lo
+    const long long c_gt = (long long)U.c_gt, c_hi = (long long)U.c_hi, c_lo = (long long)U.c_lo;
+    const long long nband = (long long)U.n_int;
+    const long long r = U.k - c_gt;
     U.r_src = SRC_CAND;
-    if (r <= 0) {
-        miss = true;
-    } else if (r <= c_hi) {
-        U.t = U.hi; U.count_above = c_gt; U.ties = c_hi; U.need = r; U.tie_src = TIE_EQ_HI;
-        U.state = ST_TKNOWN;
-    } else {
-        r -= c_hi;
-        if (r <= n_int) {
-            if (U.overflow) {
-                miss = true;
-            } else {
-                U.r_base = U.lo;
-                U.r_pshift = bitlen32(U.hi - U.lo);
-                U.r_prefix = 0;
-                U.r_rank = r;
-                U.r_above = c_gt + c_hi;
-                U.state = ST_RADIX;
-            }
+    if (r >= 1 && r <= nband && !U.overflow) {
+        if (r <= c_hi) {
+            U.t = U.hi; U.count_above = c_gt; U.ties = c_hi; U.need = r; U.tie_src = TIE_EQ_HI;
+            U.state = ST_TKNOWN;
+        } else if (r > nband - c_lo) {
+            U.t = U.lo; U.count_above = c_gt + nband - c_lo; U.ties = c_lo; U.need = r - (nband - c_lo);
+            U.tie_src = TIE_EQ_LO;
+            U.state = ST_TKNOWN;
         } else {
-            r -= n_int;
-            if (r <= c_lo) {
-                U.t = U.lo; U.count_above = c_gt + c_hi + n_int; U.ties = c_lo; U.need = r;
-                U.tie_src = TIE_EQ_LO;
-                U.state = ST_TKNOWN;
-            } else {
-                miss = true;
-            }
+            // an interior key: radix select over the band's keys
+            U.r_base = U.lo;
+            U.r_pshift = bitlen32(U.hi - U.lo);
+            U.r_prefix = 0;
+            U.r_rank = r;
+            U.r_above = c_gt;
+            U.state = ST_RADIX;
         }
-    }
-    if (miss) {
+    } else {
         // exact fallback: radix select over every entry of the unit
         U.fallback = 1;
         U.r_src = SRC_DATA;
@@ -488,27 +446,45 @@ __global__ void k_decide(Plan P) {
         U.r_above = 0;
         U.state = ST_RADIX;
     }
-    if (U.state == ST_RADIX) {
-        atomicAdd(&P.hdr->n_radix, 1);
-    } else {
-        atomicAdd(&P.hdr->n_tknown, 1);
-    }
+    if (U.state == ST_RADIX) atomicAdd(&P.hdr->n_radix, 1);
+    else atomicAdd(&P.hdr->n_tknown, 1);
 }
 
 // ---------------------------------------------------------------------------
-// radix levels: one block per contiguous item range, a shared-memory
-// histogram per (unit, run) flushed to the unit's global histogram
+// radix levels: one block per contiguous item range, one warp per tile, a
+// shared-memory histogram per (unit, run) flushed to the unit's global one.
+// Equal bins inside a warp are merged with __match_any_sync (the band keys
+// hold long runs of exact ties).  Each bin also keeps its smallest and
+// largest key (the smallest as the maximum of complements, so zero-filled
+// memory is the identity), which lets the pick stop at a single-key bin.
 // ---------------------------------------------------------------------------
+__device__ __forceinline__ void hist_add(uint32_t* h, uint32_t* mxc, uint32_t* mx, int bin, uint32_t key,
+                                         bool valid) {
+    const unsigned active = __ballot_sync(0xFFFFFFFFu, valid);
+    if (!valid) return;
+    // lanes with equal bins form disjoint groups; each reduces over its own mask
+    const unsigned grp = __match_any_sync(active, bin);
+    const int leader = __ffs(grp) - 1;
+    const uint32_t kmin = __reduce_min_sync(grp, key);
+    const uint32_t kmax = __reduce_max_sync(grp, key);
+    if ((int)(threadIdx.x & 31) == leader) {
+        atomicAdd(&h[bin], (uint32_t)__popc(grp));
+        atomicMax(&mxc[bin], ~kmin);
+        atomicMax(&mx[bin], kmax);
+    }
+}
+
 template <typename XT, typename BT, bool CK>
 __global__ void __launch_bounds__(TPB) k_radix_hist(Plan P) {
     __shared__ uint32_t s_hist[RADIX_BINS];
-    __shared__ double s_fh[RADIX_BINS];
+    __shared__ uint32_t s_mxc[RADIX_BINS];
+    __shared__ uint32_t s_mx[RADIX_BINS];
     if (*(volatile int32_t*)&P.hdr->n_radix == 0) return;
     const long long items = (long long)P.K * P.n_tiles;
     const long long per = (items + gridDim.x - 1) / gridDim.x;
     const long long beg = blockIdx.x * per;
     const long long end = (beg + per < items) ? beg + per : items;
-    for (int b = threadIdx.x; b < RADIX_BINS; b += blockDim.x) { s_hist[b] = 0; s_fh[b] = 0.0; }
+    for (int b = threadIdx.x; b < RADIX_BINS; b += blockDim.x) { s_hist[b] = 0; s_mxc[b] = 0; s_mx[b] = 0; }
     __syncthreads();
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     long long it = beg;
@@ -524,22 +500,29 @@ __global__ void __launch_bounds__(TPB) k_radix_hist(Plan P) {
         const int shift = pshift > RADIX_BITS ? pshift - RADIX_BITS : 0;
         const int nb = 1 << (pshift - shift);
         const uint32_t base = U->r_base, prefix = U->r_prefix;
-        const bool wg = U->want_gamma != 0;
         const long long ntile = run_end - it;
         if (U->r_src == SRC_CAND) {
-            // one tile's candidate list per thread
+            // one tile's candidate list per thread; runs of one bin (ties)
+            // become one update
+            const uint32_t* cs = P.cand + U->cand_off;
             for (long long q = threadIdx.x; q < ntile; q += blockDim.x) {
                 const uint2 r = P.tcand[(long long)c.i * P.n_tiles + c.g + q];
-                const uint32_t* cp = P.cand + U->cand_off + r.x;
+                int cb = -1;
+                uint32_t cn = 0, cmin = 0, cmax = 0;
                 for (uint32_t j = 0; j < r.y; ++j) {
-                    const uint32_t kk = cp[j];
+                    const uint32_t kk = cs[r.x + j];
                     const uint32_t v = kk - base;
-                    if ((v >> pshift) == prefix) {
-                        const int bin = (v >> shift) & (nb - 1);
-                        atomicAdd(&s_hist[bin], 1u);
-                        if (wg) atomicAdd(&s_fh[bin], sq(kk));
+                    if ((v >> pshift) != prefix) continue;
+                    const int bin = (v >> shift) & (nb - 1);
+                    if (bin != cb) {
+                        if (cb >= 0) { atomicAdd(&s_hist[cb], cn); atomicMax(&s_mxc[cb], ~cmin); atomicMax(&s_mx[cb], cmax); }
+                        cb = bin; cn = 0; cmin = kk; cmax = kk;
                     }
+                    cn++;
+                    cmin = min(cmin, kk);
+                    cmax = max(cmax, kk);
                 }
+                if (cb >= 0) { atomicAdd(&s_hist[cb], cn); atomicMax(&s_mxc[cb], ~cmin); atomicMax(&s_mx[cb], cmax); }
             }
         } else {
             // full data, one tile per warp
@@ -555,13 +538,9 @@ __global__ void __launch_bounds__(TPB) k_radix_hist(Plan P) {
                     const long long e = e0 + v * (32 * VEC) + lane * VEC;
 #pragma unroll
                     for (int j = 0; j < VEC; ++j) {
-                        if (e + j >= d.numel) continue;
                         const uint32_t kk = key_of(tau[j]);
-                        if ((kk >> pshift) == prefix) {
-                            const int bin = (kk >> shift) & (nb - 1);
-                            atomicAdd(&s_hist[bin], 1u);
-                            if (wg) atomicAdd(&s_fh[bin], (double)tau[j] * (double)tau[j]);
-                        }
+                        const bool ok = (e + j < d.numel) && (kk >> pshift) == prefix;
+                        hist_add(s_hist, s_mxc, s_mx, (kk >> shift) & (nb - 1), kk, ok);
                     }
                 }
             }
@@ -570,9 +549,11 @@ __global__ void __launch_bounds__(TPB) k_radix_hist(Plan P) {
         for (int b = threadIdx.x; b < nb; b += blockDim.x) {
             if (s_hist[b]) {
                 atomicAdd(&P.hist[ui * RADIX_BINS + b], s_hist[b]);
-                if (wg) atomicAdd(&P.fhist[ui * RADIX_BINS + b], s_fh[b]);
+                atomicMax(&P.hmxc[ui * RADIX_BINS + b], s_mxc[b]);
+                atomicMax(&P.hmx[ui * RADIX_BINS + b], s_mx[b]);
                 s_hist[b] = 0;
-                s_fh[b] = 0.0;
+                s_mxc[b] = 0;
+                s_mx[b] = 0;
             }
         }
         __syncthreads();
@@ -582,12 +563,12 @@ __global__ void __launch_bounds__(TPB) k_radix_hist(Plan P) {
 
 __global__ void __launch_bounds__(TPB) k_radix_pick(Plan P) {
     __shared__ long long s_scan[33];
-    __shared__ double s_dred[33];
     __shared__ int s_bin;
     __shared__ long long s_above;
     Unit& U = P.units[blockIdx.x];
     if (U.state != ST_RADIX) return;
-    uint32_t* h = P.hist + (long long)blockIdx.x * RADIX_BINS;
+    const long long hb = (long long)blockIdx.x * RADIX_BINS;
+    uint32_t* h = P.hist + hb;
     const int pshift = U.r_pshift;
     const int shift = pshift > RADIX_BITS ? pshift - RADIX_BITS : 0;
     const int nb = 1 << (pshift - shift);
@@ -595,24 +576,15 @@ __global__ void __launch_bounds__(TPB) k_radix_pick(Plan P) {
     const int b = s_bin;
     const long long above = s_above;
     const uint32_t cnt = h[b];
-    double fa = 0.0;
-    if (U.want_gamma) {
-        double* fh = P.fhist + (long long)blockIdx.x * RADIX_BINS;
-        double loc = 0.0;
-        for (int q = b + 1 + threadIdx.x; q < nb; q += blockDim.x) loc += fh[q];
-        fa = block_sum(loc, s_dred);
-        __syncthreads();
-        for (int q = threadIdx.x; q < nb; q += blockDim.x) fh[q] = 0.0;
-    }
+    const uint32_t kmin = ~P.hmxc[hb + b], kmax = P.hmx[hb + b];
     __syncthreads();
-    for (int q = threadIdx.x; q < nb; q += blockDim.x) h[q] = 0;
+    for (int q = threadIdx.x; q < nb; q += blockDim.x) { h[q] = 0; P.hmxc[hb + q] = 0; P.hmx[hb + q] = 0; }
     if (threadIdx.x == 0) {
-        U.gamma_rad += fa;
         U.r_rank -= above;
         U.r_above += above;
-        U.r_prefix = (U.r_prefix << (pshift - shift)) | (uint32_t)b;
-        if (shift == 0) {
-            U.t = U.r_base + U.r_prefix;
+        if (shift == 0 || kmin == kmax) {
+            // the bin is a single key: the threshold
+            U.t = kmax;
             U.count_above = U.r_above;
             U.ties = cnt;
             U.need = U.r_rank;
@@ -621,13 +593,15 @@ __global__ void __launch_bounds__(TPB) k_radix_pick(Plan P) {
             atomicSub(&P.hdr->n_radix, 1);
             atomicAdd(&P.hdr->n_tknown, 1);
         } else {
+            U.r_prefix = (U.r_prefix << (pshift - shift)) | (uint32_t)b;
             U.r_pshift = shift;
         }
     }
 }
 
 // ---------------------------------------------------------------------------
-// per-tile counts of keys == t (interior thresholds with partial ties)
+// per-tile counts of keys == t (partial ties), and for the K = 1 ISO
+// coefficient the sum of tau^2 over the candidates above t
 // ---------------------------------------------------------------------------
 template <typename XT, typename BT, bool CK>
 __global__ void __launch_bounds__(TPB) k_tie(Plan P) {
@@ -644,20 +618,31 @@ __global__ void __launch_bounds__(TPB) k_tie(Plan P) {
         const long long run_end = c.run_end < end ? c.run_end : end;
         const TensorDesc& d = P.tens[c.t];
         Unit* U = (d.flags & TF_TRIM) ? unit_of(P, c.i, d) : nullptr;
-        if (!U || U->state != ST_TKNOWN || U->tie_src != TIE_ARRAY || U->need >= U->ties) {
-            it = run_end;
-            continue;
-        }
+        const bool arr = U && U->state == ST_TKNOWN && U->tie_src == TIE_ARRAY;
+        const bool want_cnt = arr && U->need < U->ties;
+        const bool want_g = arr && U->want_gamma;
+        if (!want_cnt && !want_g) { it = run_end; continue; }
         const uint32_t tk = U->t;
         const long long ntile = run_end - it;
         uint32_t* tc = P.tcnt + (long long)c.i * P.n_tiles + c.g;
+        double g_warp = 0.0;
         if (U->r_src == SRC_CAND) {
-            for (long long q = threadIdx.x; q < ntile; q += blockDim.x) {
-                const uint2 r = P.tcand[(long long)c.i * P.n_tiles + c.g + q];
-                const uint32_t* cp = P.cand + U->cand_off + r.x;
+            // one tile's candidate list per thread
+            const uint32_t* cs = P.cand + U->cand_off;
+            for (long long q0 = 0; q0 < ntile; q0 += blockDim.x) {
+                const long long q = q0 + threadIdx.x;
                 uint32_t cnt = 0;
-                for (uint32_t j = 0; j < r.y; ++j) cnt += (cp[j] == tk);
-                tc[q] = cnt;
+                float fg = 0.0f;
+                if (q < ntile) {
+                    const uint2 r = P.tcand[(long long)c.i * P.n_tiles + c.g + q];
+                    for (uint32_t j = 0; j < r.y; ++j) {
+                        const uint32_t kk = cs[r.x + j];
+                        cnt += (kk == tk);
+                        if (want_g && kk > tk) { const float f = __uint_as_float(kk); fg = __fmaf_rn(f, f, fg); }
+                    }
+                    if (want_cnt) tc[q] = cnt;
+                }
+                g_warp += (double)fg;
             }
         } else {
             const void* x = P.xptr[c.i * P.n_tensors + c.t];
@@ -666,17 +651,28 @@ __global__ void __launch_bounds__(TPB) k_tie(Plan P) {
                 const long long e0 = (c.g + q - d.tile_base) * TILE;
                 rt.load(x, d.base, e0, d.numel, lane);
                 uint32_t cnt = 0;
+                float fg = 0.0f;
 #pragma unroll
                 for (int v = 0; v < WVEC; ++v) {
                     float tau[VEC];
                     rt.tau(v, tau);
                     const long long e = e0 + v * (32 * VEC) + lane * VEC;
 #pragma unroll
-                    for (int j = 0; j < VEC; ++j) cnt += (e + j < d.numel && key_of(tau[j]) == tk);
+                    for (int j = 0; j < VEC; ++j) {
+                        const uint32_t kk = key_of(tau[j]);
+                        const bool ok = e + j < d.numel;
+                        cnt += (ok && kk == tk);
+                        if (want_g && ok && kk > tk) fg = __fmaf_rn(tau[j], tau[j], fg);
+                    }
                 }
-                cnt = warp_sum(cnt);
-                if (lane == 0) tc[q] = cnt;
+                cnt = __reduce_add_sync(0xFFFFFFFFu, cnt);
+                if (want_cnt && lane == 0) tc[q] = cnt;
+                g_warp += (double)fg;
             }
+        }
+        if (want_g) {
+            g_warp = warp_sum(g_warp);
+            if (lane == 0 && g_warp != 0.0) atomicAdd(&U->gamma_rad, g_warp);
         }
         it = run_end;
     }
@@ -779,19 +775,15 @@ __global__ void __launch_bounds__(TPB) k_cut(Plan P) {
     }
     if (threadIdx.x == 0) {
         if (U.want_gamma) {
-            // sum of tau^2 over the kept entries
-            const double ft2 = sq(U.t), fh2 = sq(U.hi);
-            double g;
-            if (U.r_src == SRC_DATA) {
-                g = U.gamma_rad + (double)U.need * ft2;
-            } else if (U.tie_src == TIE_EQ_HI) {
-                g = U.gamma_acc + (double)U.need * ft2;
-            } else if (U.tie_src == TIE_EQ_LO) {
-                g = U.gamma_acc + (double)U.c_hi * fh2 + U.gamma_int + (double)U.need * ft2;
-            } else {
-                g = U.gamma_acc + (double)U.c_hi * fh2 + U.gamma_rad + (double)U.need * ft2;
-            }
-            U.gamma = g;
+            // sum of tau^2 over the kept entries: above the band (count pass),
+            // the band keys above t, and the kept ties
+            const double ft2 = sq(U.t);
+            double above;
+            if (U.r_src == SRC_DATA) above = U.gamma_rad;              // every entry above t
+            else if (U.tie_src == TIE_EQ_HI) above = U.gamma_acc;      // nothing in the band above hi
+            else if (U.tie_src == TIE_EQ_LO) above = U.gamma_acc + U.gamma_band;
+            else above = U.gamma_acc + U.gamma_rad;                  // candidates above t
+            U.gamma = above + (double)U.need * ft2;
         }
         U.state = ST_DONE;
         write_unit_stats(P, idx, U);

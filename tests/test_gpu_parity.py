@@ -311,3 +311,44 @@ def test_full_size_qwen15b_update_sampled():
             assert units[q]["k"] == -1      # 1-D tensors take the ISO average, untrimmed
     del th0, th1, out
     torch.cuda.empty_cache()
+
+
+# ---------------------------------------------------------------------------
+# the fused K = 1 pass: each way it falls back to the full exact apply
+# ---------------------------------------------------------------------------
+def _update_vs_oracle(th0, th1, op, density, is_delta=False, what=""):
+    shapes = [(t.shape[0], t.shape[1]) if t.dim() == 2 else (1, t.numel()) for t in th0]
+    is1d = [t.dim() == 1 for t in th0]
+    out, st = iso.iso_update([t.to(DEV) for t in th0], [t.to(DEV) for t in th1], op=op,
+                             update_is_delta=is_delta, density=density, stats=True)
+    torch.cuda.synchronize()
+    r = oracle.update(_np_list(th0), _np_list(th1), OPS[op], update_is_delta=is_delta,
+                      density=density, shapes=shapes, is_1d=is1d)
+    _check_merge(out, st, r, th0, OPS[op], 1, what=what)
+    return r
+
+
+def test_fused_repair_when_retention_coefficient_is_not_one():
+    # ||trimmed tau||^2 ~ 1e-13 < 2^25 * ridge: c = Gamma / (Gamma + ridge) is far from 1
+    g = torch.Generator().manual_seed(31)
+    th0 = (torch.randn(300, 1000, generator=g) * 0.02).to(torch.bfloat16)
+    tiny = (torch.randn(300, 1000, generator=g) * 1e-9)
+    r = _update_vs_oracle([th0], [tiny], "iso", 0.05, is_delta=True, what="tiny-gamma iso")
+    assert 0.0 < r["coef"][0][0] < 0.9
+
+
+def test_fused_repair_when_band_records_overflow():
+    # every |tau| equal: the whole tensor is one run of ties at the threshold
+    g = torch.Generator().manual_seed(32)
+    th0 = (torch.randn(300, 1000, generator=g) * 0.02).to(torch.bfloat16)
+    sgn = torch.where(torch.rand(300, 1000, generator=g) < 0.5, -1.0, 1.0)
+    d = (sgn * 2.0 ** -10).to(torch.bfloat16)
+    for op in ("ties", "iso"):
+        _update_vs_oracle([th0], [d], op, 0.05, is_delta=True, what=f"all-tied {op}")
+
+
+def test_fused_bf16_delta_input_mixed_list():
+    th0 = synth.base_weights(MIXED, seed=33)
+    taus = [t.to(torch.bfloat16) for t in _taus(MIXED, 34, torch.float32)]
+    for op in ("ties", "iso"):
+        _update_vs_oracle(th0, taus, op, 0.05, is_delta=True, what=f"bf16 delta {op}")
