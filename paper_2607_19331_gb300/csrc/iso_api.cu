@@ -511,7 +511,7 @@ int run_group(const Call& c, int t0, int t1, char* ws, cudaStream_t s, const iso
                 ISO_TRY(launch(KD_RADIX_PICK, s, [&] { k_radix_pick<<<KU, TPB, 0, s>>>(P); }));
             }
             ISO_TRY(launch(KD_TIE, s, [&] { k_tie<XT, BT, CK><<<pgrid, TPB, 0, s>>>(P); }));
-            ISO_TRY(launch(KD_CUT, s, [&] { k_cut<XT, BT, CK><<<KU, TPB, 0, s>>>(P); }));
+            ISO_TRY(launch(KD_CUT, s, [&] { k_cut<XT, BT, CK><<<KU, 1024, 0, s>>>(P); }));
             return ISO_OK;
         });
         ISO_TRY(rc);

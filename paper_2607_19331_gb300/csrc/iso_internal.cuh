@@ -30,7 +30,7 @@ constexpr int WPB = TPB / 32;               // warps per streaming block
 static_assert(WVEC * 32 * VEC == TILE, "tile geometry");
 constexpr int CHUNK_MAX = 1024;             // candidate slots a warp reserves at once
 
-constexpr int SAMPLE_MAX = 32768;           // sampled keys per unit (128 KB of smem)
+constexpr int SAMPLE_MAX = 24576;           // sampled keys per unit (96 KB of smem: two blocks per SM)
 constexpr int SAMPLE_CHUNK = 256;           // contiguous entries per sample chunk
 constexpr int SAMPLE_TPB = 1024;
 constexpr double SAMPLE_Z = 5.0;            // band half-width in sample standard deviations

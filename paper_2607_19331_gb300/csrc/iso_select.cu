@@ -694,8 +694,10 @@ __device__ __forceinline__ void write_unit_stats(const Plan& P, int idx, const U
     P.st_units[(long long)i * P.st_units_stride + P.st_unit_base + u] = s;
 }
 
+constexpr int CUT_TPB = 1024;
+
 template <typename XT, typename BT, bool CKPT>
-__global__ void __launch_bounds__(TPB) k_cut(Plan P) {
+__global__ void __launch_bounds__(CUT_TPB) k_cut(Plan P) {
     __shared__ long long s_scan[33];
     __shared__ uint32_t s_scan32[33];
     __shared__ long long s_tile;
@@ -720,8 +722,16 @@ __global__ void __launch_bounds__(TPB) k_cut(Plan P) {
                               (long long)i * P.n_tiles;
         auto tile_ties = [&](long long g) -> long long { return src[g]; };
         long long local = 0;
-#pragma unroll 8
-        for (long long g = j0; g < j1; ++g) local += src[g];
+        {
+            // 16-byte loads where the chunk allows
+            long long g = j0;
+            for (; g < j1 && ((uintptr_t)(src + g) & 15); ++g) local += src[g];
+            for (; g + 4 <= j1; g += 4) {
+                const uint4 v = *reinterpret_cast<const uint4*>(src + g);
+                local += (long long)v.x + v.y + v.z + v.w;
+            }
+            for (; g < j1; ++g) local += src[g];
+        }
         long long total;
         const long long excl = block_excl_scan(local, s_scan, &total);
         if (excl < U.need && U.need <= excl + local) {
@@ -744,7 +754,7 @@ __global__ void __launch_bounds__(TPB) k_cut(Plan P) {
             const int t = tensor_of_tile(P.tens, P.n_tensors, g);
             const TensorDesc& d = P.tens[t];
             const void* x = P.xptr[i * P.n_tensors + t];
-            constexpr int PER = TILE / TPB;
+            constexpr int PER = TILE / CUT_TPB;
             const long long eb = (g - d.tile_base) * TILE + (long long)threadIdx.x * PER;
             uint32_t mine = 0;
             for (int j = 0; j < PER; ++j) {

@@ -100,7 +100,7 @@ def test_band_miss_falls_back_exactly():
     # misses and the unit is resolved by the full-data radix select.
     n = 300_000
     x = (torch.arange(n, dtype=torch.float32) % 977 + 1.0) * 1e-3
-    S, C = 32768, 256
+    S, C = 24576, 256   # the library's sample size and chunk length
     nch = S // C
     for c in range(nch):
         p = int((n - C) * c / (nch - 1))
