@@ -56,6 +56,37 @@ def algorithmic_bytes(shapes, K, inputs, op):
     return {"apply": apply, "count": count}
 
 
+def kernel_source_hash():
+    """sha1 of the kernel sources: a profile's traffic applies only to the
+    kernels it measured."""
+    import glob
+    import hashlib
+    csrc = os.path.join(ROOT, "paper_2607_19331_gb300", "csrc")
+    files = sorted(glob.glob(os.path.join(csrc, "*.cu")) + glob.glob(os.path.join(csrc, "*.cuh")))
+    files.append(os.path.join(ROOT, "include", "iso.h"))
+    h = hashlib.sha1()
+    for f in files:
+        h.update(os.path.basename(f).encode())
+        with open(f, "rb") as fh:
+            h.update(fh.read())
+    return h.hexdigest()[:16]
+
+
+def profiled_traffic(kernel, workload):
+    """DRAM bytes per parameter of `kernel` from the committed ncu summaries in
+    profiles/, if they were taken on the current kernel sources."""
+    import glob
+    sha = kernel_source_hash()
+    for f in glob.glob(os.path.join(ROOT, "profiles", "*.md")):
+        for line in open(f):
+            if not line.startswith("traffic:"):
+                continue
+            kv = dict(x.split("=", 1) for x in line.split()[1:])
+            if kv.get("kernel") == kernel and kv.get("workload") == workload and kv.get("csrc_sha1") == sha:
+                return float(kv["dram_bytes_per_param"])
+    return None
+
+
 def read_peaks():
     p = os.path.join(ROOT, "MEASURED_PEAKS.json")
     try:
@@ -204,6 +235,8 @@ def run_mine(args):
     per_launch_bytes = algo[dom] / max(1, n_dom // prof_steps)
     achieved = per_launch_bytes / (avg_ms * 1e-3) / 1e9 if avg_ms > 0 else 0.0
     step_gbs = (algo["apply"] + algo["count"]) / (ms * 1e-3) / 1e9
+    tb = profiled_traffic(dom, name) if args.layers is None else None
+    traffic = None if tb is None else int(tb * n_params)
 
     # end to end through the public API from pinned host memory
     e2e = None
@@ -247,7 +280,9 @@ def run_mine(args):
             "hbm_pct_of_8tbs_step": round(100 * step_gbs / NOMINAL_HBM_GBS, 1),
             "roofline": {"bound": "hbm", "kernel": dom, "achieved": round(achieved, 1), "peak": peak,
                          "peak_source": peak_src, "unit": "GB/s",
-                         "frac": round(achieved / peak, 4) if peak else None, "traffic": None,
+                         "frac": round(achieved / peak, 4) if peak else None, "traffic": traffic,
+                         "traffic_source": "profiles/ ncu summary (DRAM bytes per param x params)"
+                         if traffic is not None else "no ncu summary for the current kernel sources",
                          "algorithmic_bytes_per_launch": int(per_launch_bytes),
                          "avg_launch_ms": round(avg_ms, 4)},
             "kernels": {k: {"launches": v["launches"], "ms_per_step": round(v["ms_per_step"], 4)}
