@@ -9,6 +9,7 @@
 #include <cmath>
 #include <cstring>
 #include <mutex>
+#include <type_traits>
 #include <unordered_map>
 #include <vector>
 
@@ -25,6 +26,7 @@ constexpr int COUNT_GRID_PER_SM = ISO_COUNT_BLOCKS_PER_SM;
 #define ISO_FUSED_BLOCKS_PER_SM 2
 #endif
 constexpr int FUSED_GRID_PER_SM = ISO_FUSED_BLOCKS_PER_SM;
+constexpr int MERGE_GRID_PER_SM = 2;     // k_merge / k_gramk: 2 resident blocks of 256 per SM
 
 // ---------------------------------------------------------------------------
 // profiling and launch accounting
@@ -556,15 +558,28 @@ int run_group(const Call& c, int t0, int t1, char* ws, cudaStream_t s, const iso
         using XT = std::remove_pointer_t<decltype(xt)>;
         using BT = std::remove_pointer_t<decltype(bt)>;
         constexpr bool CK = decltype(ck)::value;
+        const int mgrid = sms * MERGE_GRID_PER_SM;
         if (gram_mode != GRAM_NONE) {
-            if (need_gram_pass)
-                ISO_TRY(launch(KD_GRAM, s, [&] { k_gram<XT, BT, CK><<<pgrid, TPB, 0, s>>>(P); }));
+            if (need_gram_pass) {
+                auto gram = [&](auto kc) {
+                    constexpr int KC = decltype(kc)::value;
+                    return launch(KD_GRAM, s, [&] { k_gramk<XT, BT, CK, KC><<<mgrid, TPB, 0, s>>>(P); });
+                };
+                if (K == 1) ISO_TRY(gram(std::integral_constant<int, 1>{}));
+                else if (K == 2) ISO_TRY(gram(std::integral_constant<int, 2>{}));
+                else if (K <= 4) ISO_TRY(gram(std::integral_constant<int, 4>{}));
+                else ISO_TRY(gram(std::integral_constant<int, 8>{}));
+            }
             ISO_TRY(launch(KD_SOLVE, s, [&] { k_solve<<<(T + 127) / 128, 128, 0, s>>>(P, gram_mode); }));
         }
-        if (K == 1)
-            ISO_TRY(launch(KD_APPLY, s, [&] { k_apply<XT, BT, CK, 1><<<pgrid, TPB, 0, s>>>(P); }));
-        else
-            ISO_TRY(launch(KD_APPLY, s, [&] { k_apply<XT, BT, CK, 0><<<pgrid, TPB, 0, s>>>(P); }));
+        auto merge = [&](auto kc) {
+            constexpr int KC = decltype(kc)::value;
+            return launch(KD_APPLY, s, [&] { k_merge<XT, BT, CK, KC><<<mgrid, TPB, 0, s>>>(P); });
+        };
+        if (K == 1) ISO_TRY(launch(KD_APPLY, s, [&] { k_apply<XT, BT, CK, 1><<<pgrid, TPB, 0, s>>>(P); }));
+        else if (K == 2) ISO_TRY(merge(std::integral_constant<int, 2>{}));
+        else if (K <= 4) ISO_TRY(merge(std::integral_constant<int, 4>{}));
+        else ISO_TRY(merge(std::integral_constant<int, 8>{}));
         return ISO_OK;
     });
     return rc;

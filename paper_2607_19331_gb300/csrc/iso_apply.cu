@@ -1,14 +1,15 @@
-// iso_apply.cu -- the streaming passes that apply a resolved TopKMask.
+// iso_apply.cu -- the K = 1 update pass, the retention solve and the small
+// passes around them.
 //
-//   k_apply  out = theta_0 + update, one read of theta_0 and the K experts
-//            and one write:                                         (App. F)
-//              TA    update = lambda * sum_i tau_i
-//              TIES  gamma = sign(sum_i m_i tau_i); A = {i : m_i tau_i != 0,
-//                    sign = gamma}; update = lambda * mean_{i in A} tau_i
-//              ISO   2-D: update = sum_i c_i m_i tau_i          (Sec. 4.2, App. E)
-//                    1-D: update = (1/K) sum_i tau_i            (App. E, Algorithm 1)
+//   k_apply  out = theta_0 + update for one expert, one read of theta_0 and
+//            the expert and one write (App. F): every operator reduces to
+//            update = a * m * tau with a per-tensor scale a
+//              TA    a = lambda, no mask
+//              TIES  a = lambda (one expert: the elected sign is its own)
+//              ISO   2-D: a = c, the tensor's retention coefficient (Sec. 4.2)
+//                    1-D: a = 1/K = 1, no mask                 (App. E, Algorithm 1)
 //            An update of exactly zero leaves theta_0 untouched.
-//   k_gram   Gamma_ij = <m_i tau_i, m_j tau_j> per 2-D tensor  (Sec. 4.2 Gram eq.)
+//            (K >= 2 and the Gram pass: iso_merge.cu)
 //   k_solve  (Gamma + ridge I) c = diag Gamma on the non-zero experts, clip
 //   k_mask   the mask itself as a packed bitmask
 //   k_delta  tau = theta_i - theta_0 in binary32
@@ -24,7 +25,6 @@ __device__ __forceinline__ int block_unit(const Plan& P, const TensorDesc& d, lo
     return d.unit + (int)(row / P.block_rows) * d.bpr + (int)(col / P.block_cols);
 }
 
-__device__ __forceinline__ int sgn(float v) { return (v > 0.0f) - (v < 0.0f); }
 
 // ---------------------------------------------------------------------------
 // apply: one warp per tile, one contiguous tile range per warp
@@ -58,33 +58,6 @@ __device__ __forceinline__ void tensor_params(const Plan& P, int t, int K, Tenso
     }
 }
 
-// merged value of one entry from its K (masked) task-vector entries
-__device__ __forceinline__ float combine(const Plan& P, const TensorParams& tp, int K, float th0,
-                                         const float* tau, const bool* sel) {
-    float upd;
-    if (P.op == ISO_OP_TA || tp.iso1d) {
-        float s = 0.0f;
-        for (int i = 0; i < K; ++i) s = __fadd_rn(s, tau[i]);
-        upd = tp.iso1d ? __fdiv_rn(s, (float)K) : __fmul_rn(P.lambda, s);
-    } else if (P.op == ISO_OP_TIES) {
-        float s = 0.0f;
-        for (int i = 0; i < K; ++i) s = __fadd_rn(s, sel[i] ? tau[i] : 0.0f);
-        const int gam = sgn(s);
-        float a = 0.0f;
-        int cnt = 0;
-        for (int i = 0; i < K; ++i)
-            if (sel[i] && tau[i] != 0.0f && sgn(tau[i]) == gam) { a = __fadd_rn(a, tau[i]); cnt++; }
-        const float merged = cnt ? __fdiv_rn(a, (float)cnt) : 0.0f;
-        upd = __fmul_rn(P.lambda, merged);
-    } else {
-        float s = 0.0f;
-        for (int i = 0; i < K; ++i)
-            if (sel[i]) s = __fadd_rn(s, __fmul_rn(tp.cf[i], tau[i]));
-        upd = s;
-    }
-    return (upd == 0.0f) ? th0 : __fadd_rn(th0, upd);
-}
-
 // K = 1: the per-tensor scale, whether the tensor is trimmed, and the packed
 // threshold (t, ~cut) for tensor-local positions below 2^32
 __device__ __forceinline__ void k1_params(const Plan& P, const TensorParams& tp, float* a, bool* mask,
@@ -110,7 +83,8 @@ __device__ __forceinline__ SelParam block_param(const Plan& P, const TensorDesc&
 
 template <typename XT, typename BT, bool CK, int KC>
 __global__ void __launch_bounds__(TPB) k_apply(Plan P) {
-    const int K = KC ? KC : P.K;
+    static_assert(KC == 1, "K >= 2 merges run in k_merge");
+    const int K = 1;
     const int lane = threadIdx.x & 31;
     const long long W = (long long)gridDim.x * WPB;
     const long long wid = (long long)blockIdx.x * WPB + (threadIdx.x >> 5);
@@ -124,7 +98,7 @@ __global__ void __launch_bounds__(TPB) k_apply(Plan P) {
     TensorParams tp;
     tensor_params(P, t, K, tp);
 
-    if (KC == 1) {
+    {
         // K = 1: every operator reduces to theta_0 + a * (mask ? tau : 0) with a
         // per-tensor scale a (TA, TIES: lambda; ISO 2-D: c; ISO 1-D: 1/K = 1)
         // and the mask off for TA and ISO 1-D.  The whole tile sits in
@@ -199,166 +173,7 @@ __global__ void __launch_bounds__(TPB) k_apply(Plan P) {
             }
             cur = nxt;
         }
-        return;
     }
-
-    // K >= 2: vector by vector, the K experts' loads of a vector in flight together
-    for (long long g = beg; g < end; ++g) {
-        if (g >= t_end) {
-            while (g >= t_end) { ++t; t_end = P.tens[t].tile_base + (P.tens[t].numel + TILE - 1) / TILE; }
-            tensor_params(P, t, K, tp);
-        }
-        const TensorDesc& d = P.tens[t];
-        const long long n = d.numel;
-        const long long e0 = (g - d.tile_base) * TILE;
-        for (int v = 0; v < WVEC; ++v) {
-            const long long e = e0 + v * (32 * VEC) + lane * VEC;
-            if (e >= n) continue;
-            uint4 braw[Lanes<BT>::N];
-            uint4 xraw[MAXK][Lanes<XT>::N];
-            load_raw8<BT>(d.base, e, n, braw);
-#pragma unroll
-            for (int i = 0; i < MAXK; ++i) {
-                if (i >= K) break;
-                load_raw8<XT>(tp.xs[i], e, n, xraw[i]);
-            }
-            float th0[VEC];
-            raw_to_f32<BT>(braw, th0);
-            float tau[MAXK][VEC];
-#pragma unroll
-            for (int i = 0; i < MAXK; ++i) {
-                if (i >= K) break;
-                raw_to_f32<XT>(xraw[i], tau[i]);
-                if (CK) {
-#pragma unroll
-                    for (int j = 0; j < VEC; ++j) tau[i][j] = __fsub_rn(tau[i][j], th0[j]);
-                }
-            }
-            long long r = 0, cc = 0;
-            if (tp.blk) { r = e / d.cols; cc = e - r * d.cols; }
-            float o[VEC];
-#pragma unroll
-            for (int j = 0; j < VEC; ++j) {
-                float tj[MAXK];
-                bool sj[MAXK];
-#pragma unroll
-                for (int i = 0; i < MAXK; ++i) {
-                    if (i >= K) break;
-                    tj[i] = tau[i][j];
-                    const SelParam s = tp.blk ? block_param(P, d, i, r, cc) : tp.sp[i];
-                    sj[i] = kept(key_of(tj[i]), tp.pos_off + e + j, s);
-                }
-                if (tp.blk && ++cc == d.cols) { cc = 0; ++r; }
-                o[j] = combine(P, tp, K, th0[j], tj, sj);
-            }
-            store8(d.out, e, n, o, obf);
-        }
-    }
-}
-
-// ---------------------------------------------------------------------------
-// Gram of the trimmed task vectors (per 2-D tensor, upper triangle)
-// ---------------------------------------------------------------------------
-template <typename XT, typename BT, bool CK>
-__global__ void __launch_bounds__(TPB) k_gram(Plan P) {
-    constexpr int NP = MAXK * (MAXK + 1) / 2;
-    __shared__ double s_g[WPB][NP];
-    const int K = P.K;
-    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-    const long long W = (long long)gridDim.x * WPB;
-    const long long wid = (long long)blockIdx.x * WPB + warp;
-    const long long per = (P.n_tiles + W - 1) / W;
-    const long long beg = wid * per;
-    const long long end = (beg + per < P.n_tiles) ? beg + per : P.n_tiles;
-    for (int q = lane; q < NP; q += 32) s_g[warp][q] = 0.0;
-    __syncwarp();
-    if (beg >= end) return;
-    int t = tensor_of_tile(P.tens, P.n_tensors, beg);
-    long long t_end = P.tens[t].tile_base + (P.tens[t].numel + TILE - 1) / TILE;
-    TensorParams tp;
-    tensor_params(P, t, K, tp);
-    auto flush = [&](int tt) {
-        __syncwarp();
-        if (lane == 0) {
-            int q = 0;
-            for (int a = 0; a < K; ++a)
-                for (int b = a; b < K; ++b, ++q)
-                    if (s_g[warp][q] != 0.0) {
-                        atomicAdd(&P.gram[((long long)tt * K + a) * K + b], s_g[warp][q]);
-                        s_g[warp][q] = 0.0;
-                    }
-        }
-        __syncwarp();
-    };
-    for (long long g = beg; g < end; ++g) {
-        if (g >= t_end) {
-            flush(t);
-            while (g >= t_end) { ++t; t_end = P.tens[t].tile_base + (P.tens[t].numel + TILE - 1) / TILE; }
-            tensor_params(P, t, K, tp);
-        }
-        const TensorDesc& d = P.tens[t];
-        if ((d.flags & TF_1D) || !(d.flags & TF_TRIM)) continue;
-        const long long n = d.numel;
-        const long long e0 = (g - d.tile_base) * TILE;
-        float acc[NP];
-#pragma unroll
-        for (int q = 0; q < NP; ++q) acc[q] = 0.0f;
-        for (int v = 0; v < WVEC; ++v) {
-            const long long e = e0 + v * (32 * VEC) + lane * VEC;
-            if (e >= n) continue;
-            float th0[VEC];
-            if (CK) load8_tail<BT>(d.base, e, n, th0);
-            float m[MAXK][VEC];
-            long long r = 0, cc = 0;
-            if (tp.blk) { r = e / d.cols; cc = e - r * d.cols; }
-#pragma unroll
-            for (int i = 0; i < MAXK; ++i) {
-                if (i >= K) break;
-                uint4 xr[Lanes<XT>::N];
-                load_raw8<XT>(tp.xs[i], e, n, xr);
-                float tau[VEC];
-                raw_to_f32<XT>(xr, tau);
-                long long rr = r, c2 = cc;
-#pragma unroll
-                for (int j = 0; j < VEC; ++j) {
-                    if (CK) tau[j] = __fsub_rn(tau[j], th0[j]);
-                    SelParam s = tp.sp[i];
-                    if (tp.blk) {
-                        s = block_param(P, d, i, rr, c2);
-                        if (++c2 == d.cols) { c2 = 0; ++rr; }
-                    }
-                    m[i][j] = (e + j < n && kept(key_of(tau[j]), tp.pos_off + e + j, s)) ? tau[j] : 0.0f;
-                }
-            }
-            int q = 0;
-#pragma unroll
-            for (int a = 0; a < MAXK; ++a) {
-#pragma unroll
-                for (int b = a; b < MAXK; ++b) {
-                    if (a < K && b < K) {
-#pragma unroll
-                        for (int j = 0; j < VEC; ++j) acc[q] = __fadd_rn(acc[q], __fmul_rn(m[a][j], m[b][j]));
-                    }
-                    ++q;
-                }
-            }
-        }
-        // tile partials in binary32 (<= 1024 entries), summed in binary64 per warp
-        int q = 0, cq = 0;
-#pragma unroll
-        for (int a = 0; a < MAXK; ++a) {
-#pragma unroll
-            for (int b = a; b < MAXK; ++b) {
-                if (a < K && b < K) {
-                    const float w = warp_sum(acc[q]);
-                    if (lane == 0) s_g[warp][cq] += (double)w;
-                    ++cq;
-                }
-                ++q;
-            }
-        }
-    }
-    flush(t);
 }
 
 // ---------------------------------------------------------------------------
@@ -532,9 +347,7 @@ __global__ void __launch_bounds__(TPB) k_delta(DeltaArgs A) {
 // instantiations
 // ---------------------------------------------------------------------------
 #define ISO_APPLY_INST(XT, BT, CK)                                             \
-    template __global__ void k_apply<XT, BT, CK, 1>(Plan);                    \
-    template __global__ void k_apply<XT, BT, CK, 0>(Plan);                    \
-    template __global__ void k_gram<XT, BT, CK>(Plan);
+    template __global__ void k_apply<XT, BT, CK, 1>(Plan);
 
 ISO_APPLY_INST(__nv_bfloat16, __nv_bfloat16, false)
 ISO_APPLY_INST(__nv_bfloat16, float, false)

@@ -1,5 +1,6 @@
 // iso_kernels.cuh -- kernel declarations (definitions and explicit
-// instantiations live in iso_select.cu, iso_apply.cu and iso_block.cu).
+// instantiations live in iso_select.cu, iso_apply.cu, iso_merge.cu,
+// iso_block.cu and iso_fused.cu).
 #pragma once
 
 #include "iso_internal.cuh"
@@ -27,9 +28,11 @@ template <bool CK> __global__ void k_count_apply(Plan P);
 template <bool CK> __global__ void k_patch(Plan P);
 template <bool CK> __global__ void k_repair(Plan P);
 
-// apply
+// apply: K = 1 (iso_apply.cu); K >= 2 with a compile-time bound KC >= K on
+// the expert count, and the Gram pass for any K (iso_merge.cu)
 template <typename XT, typename BT, bool CK, int KC> __global__ void k_apply(Plan P);
-template <typename XT, typename BT, bool CK> __global__ void k_gram(Plan P);
+template <typename XT, typename BT, bool CK, int KC> __global__ void k_merge(Plan P);
+template <typename XT, typename BT, bool CK, int KC> __global__ void k_gramk(Plan P);
 __global__ void k_solve(Plan P, int gram_mode);
 template <typename XT> __global__ void k_mask(Plan P, uint32_t* const* mptr);
 __global__ void k_status(const Header* h, int32_t* out);

@@ -181,6 +181,39 @@ def test_merge_bf16_base_fp32_deltas(scope, op, K):
     _check_merge(out, st, r, th0, OPS[op], K, what=f"merge K={K} {op} {scope}")
 
 
+@pytest.mark.parametrize("scope", ["tensor", "block", "global"])
+@pytest.mark.parametrize("op", ["ties", "iso", "ta"])
+@pytest.mark.parametrize("K,experts", [(2, "delta_bf16"), (4, "ckpt_bf16"), (5, "delta_bf16"),
+                                       (5, "ckpt_f32"), (7, "delta_f32")])
+def test_merge_expert_counts_and_dtypes(scope, op, K, experts):
+    # every compile-time expert bound (2, 4, 8) with K below and at it, bf16
+    # and fp32 experts given as task vectors or as checkpoints, on shapes with
+    # ragged tails, 1-D tensors, partial blocks and an empty tensor
+    shapes = MIXED
+    base_dt = torch.float32 if experts == "ckpt_f32" else torch.bfloat16
+    th0 = synth.base_weights(shapes, seed=11, dtype=base_dt)
+    xs = []
+    for i in range(K):
+        d = _taus(shapes, 40 + i, torch.float32, ties=(i % 2 == 1))
+        if experts == "delta_bf16":
+            xs.append([x.to(torch.bfloat16) for x in d])
+        elif experts == "delta_f32":
+            xs.append(d)
+        else:
+            dt = torch.bfloat16 if experts == "ckpt_bf16" else torch.float32
+            xs.append([(b.float() + x).to(dt) for b, x in zip(th0, d)])
+    is_delta = experts.startswith("delta")
+    d0 = [t.to(DEV) for t in th0]
+    dx = [[t.to(DEV) for t in e] for e in xs]
+    out, st = iso.iso_merge(d0, dx, op=op, experts_are_deltas=is_delta, density=0.15, scope=scope,
+                            lam=0.9, stats=True)
+    torch.cuda.synchronize()
+    r = oracle.merge(_np_list(th0), [_np_list(e) for e in xs], OPS[op], experts_are_deltas=is_delta,
+                     density=0.15, scope=SCOPES[scope], lam=0.9, shapes=_shapes(shapes),
+                     is_1d=_is1d(shapes))
+    _check_merge(out, st, r, th0, OPS[op], K, what=f"merge K={K} {experts} {op} {scope}")
+
+
 def test_merge_checkpoints_mask_1d_off():
     shapes = MIXED
     th0 = synth.base_weights(shapes, seed=9, dtype=torch.float32)
