@@ -28,32 +28,45 @@ UNIT = "Gparams/s"
 NOMINAL_HBM_GBS = 8000.0
 
 WORKLOADS = {
-    # name: (shape set, K, op, inputs, density, description)
-    "qwen1.5b_update": ("qwen1.5b", 1, "iso", "ckpt_bf16", 0.05,
+    # name: (shape set, K, op, inputs, density, scope, description)
+    "qwen1.5b_update": ("qwen1.5b", 1, "iso", "ckpt_bf16", 0.05, "tensor",
                         "Qwen2.5-1.5B-shaped bf16 base + RL checkpoint, masked ISO update, "
                         "per-tensor TopKMask 5%"),
-    "qwen7b_update": ("qwen7b", 1, "iso", "ckpt_bf16", 0.05,
+    "qwen7b_update": ("qwen7b", 1, "iso", "ckpt_bf16", 0.05, "tensor",
                       "Qwen2.5-7B-shaped bf16 base + RL checkpoint, fused delta+mask+update, "
                       "per-tensor TopKMask 5%"),
-    "qwen7b_ties_k8": ("qwen7b", 8, "ties", "delta_f32", 0.10,
+    "qwen7b_ties_k8": ("qwen7b", 8, "ties", "delta_f32", 0.10, "tensor",
                        "Qwen2.5-7B-shaped bf16 base, 8 fp32 RL deltas, TopKMask 10% + TIES"),
-    "qwen7b_iso_k8": ("qwen7b", 8, "iso", "delta_f32", 0.10,
+    "qwen7b_iso_k8": ("qwen7b", 8, "iso", "delta_f32", 0.10, "tensor",
                       "Qwen2.5-7B-shaped bf16 base, 8 fp32 RL deltas, TopKMask 10% + ISO retention"),
+    "sweep_tensor": ("sweep", 1, "ties", "delta_bf16", 0.05, "tensor",
+                     "bf16 4096x14336 delta N(0,1e-3^2)+1e-3 t_3 with 1000 threshold ties, "
+                     "per-tensor TopKMask + masked update (--density)"),
+    "sweep_block": ("sweep", 1, "ties", "delta_bf16", 0.05, "block",
+                    "bf16 4096x14336 delta N(0,1e-3^2)+1e-3 t_3 with 1000 threshold ties, "
+                    "per-128x128-block TopKMask + masked update (--density)"),
 }
 
 
-def algorithmic_bytes(shapes, K, inputs, op):
-    """Bytes a pass must move at minimum: read theta_0 and the K experts once,
-    write the output once.  Returned per kernel kind: (apply, count)."""
+def algorithmic_bytes(shapes, K, inputs, op, scope="tensor"):
+    """Bytes each full pass must move at minimum, per kernel kind.
+
+    apply:        read theta_0 and the K experts once, write the output once
+    count:        (per-tensor scope) read the K task vectors once
+    block_select: (per-block scope) read the K task vectors once
+    gram:         (ISO, K >= 2) read the K task vectors once
+    """
     n_all = sum(r * c for r, c, _ in shapes)
     n_trim = sum(r * c for r, c, one in shapes if not (one and op == "iso"))
-    if inputs == "ckpt_bf16":
-        per_x, per_base, per_out = 2, 2, 2
-    else:
-        per_x, per_base, per_out = 4, 2, 2
-    apply = n_all * (per_base + K * per_x + per_out)
-    count = n_trim * (K * per_x + (per_base if inputs == "ckpt_bf16" else 0))
-    return {"apply": apply, "count": count}
+    per_x = {"ckpt_bf16": 2, "delta_bf16": 2, "delta_f32": 4}[inputs]
+    per_base, per_out = 2, 2
+    read_tau = n_trim * (K * per_x + (per_base if inputs == "ckpt_bf16" else 0))
+    out = {"apply": n_all * (per_base + K * per_x + per_out)}
+    if op != "ta":
+        out["block_select" if scope == "block" else "count"] = read_tau
+    if op == "iso" and K >= 2:
+        out["gram"] = read_tau
+    return out
 
 
 def kernel_source_hash():
@@ -142,11 +155,18 @@ class Clocks:
                 "reasons": reasons, "samples": len(rows)}
 
 
-def make_workload(name, device, seed, layers=None):
+def make_workload(name, device, seed, layers=None, density=None, scale=1):
     import torch
     import synth
-    shapes_name, K, op, inputs, density, desc = WORKLOADS[name]
-    shapes = synth.qwen_shapes(shapes_name, layers=layers)
+    shapes_name, K, op, inputs, d0, scope, desc = WORKLOADS[name]
+    if shapes_name == "sweep":
+        shapes = [(4096, 14336, False)]
+        th0 = synth.base_weights(shapes, seed=seed, device=device)
+        experts = [[synth.density_sweep_delta(seed=seed, rho=d0 if density is None else density,
+                                              device=device)]]
+        torch.cuda.synchronize()
+        return shapes, th0, experts
+    shapes = synth.qwen_shapes(shapes_name, layers=layers, scale=scale)
     if inputs == "ckpt_bf16":
         th0, th1 = synth.rl_update_set(shapes, seed=seed, device=device)
         experts = [th1]
@@ -170,12 +190,15 @@ def run_mine(args):
     torch.cuda.set_device(local)
     dev = torch.device("cuda", local)
     name = args.workload
-    shapes_name, K, op, inputs, density, desc = WORKLOADS[name]
-    shapes, th0, experts = make_workload(name, dev, seed=rank, layers=args.layers)
+    shapes_name, K, op, inputs, density, scope, desc = WORKLOADS[name]
+    if args.density is not None:
+        density = args.density
+    shapes, th0, experts = make_workload(name, dev, seed=rank, layers=args.layers, density=density,
+                                         scale=args.scale)
     n_params = sum(t.numel() for t in th0)
     ckpt = inputs == "ckpt_bf16"
     out = [torch.empty_like(t) for t in th0]
-    cfg = iso.merge_cfg(op, density, "tensor")
+    cfg = iso.merge_cfg(op, density, scope)
     mn, full = iso.iso_workspace_size(th0, K, cfg)
     free = torch.cuda.mem_get_info(dev)[0]
     ws_bytes = full if full + (1 << 30) < free else max(mn, free - (2 << 30))
@@ -185,7 +208,7 @@ def run_mine(args):
 
     def step():
         iso.iso_merge(th0, experts, op=op, experts_are_deltas=not ckpt, out=out, density=density,
-                      scope="tensor", lam=1.0, workspace=ws, ws_bytes=ws_bytes, stream=stream)
+                      scope=scope, lam=1.0, workspace=ws, ws_bytes=ws_bytes, stream=stream)
 
     def barrier():
         if world > 1:
@@ -226,34 +249,37 @@ def run_mine(args):
     torch.cuda.synchronize()
     prof = iso.profile_read()
     iso.profile_enable(False)
-    algo = algorithmic_bytes(shapes, K, inputs, op)
+    algo = algorithmic_bytes(shapes, K, inputs, op, scope)
     peak, peak_src = read_peaks()
     kernels = {k: {"launches": n // prof_steps, "ms_per_step": tot / prof_steps} for k, (n, tot) in prof.items()}
-    dom = max(("apply", "count"), key=lambda k: prof.get(k, (0, 0.0))[1])
+    dom = max(algo, key=lambda k: prof.get(k, (0, 0.0))[1])
     n_dom, t_dom = prof.get(dom, (1, 0.0))
     avg_ms = t_dom / max(1, n_dom)
     per_launch_bytes = algo[dom] / max(1, n_dom // prof_steps)
     achieved = per_launch_bytes / (avg_ms * 1e-3) / 1e9 if avg_ms > 0 else 0.0
-    step_gbs = (algo["apply"] + algo["count"]) / (ms * 1e-3) / 1e9
-    tb = profiled_traffic(dom, name) if args.layers is None else None
+    step_gbs = sum(algo.values()) / (ms * 1e-3) / 1e9
+    small = args.layers is not None or args.scale != 1
+    tb = profiled_traffic(dom, name) if not small else None
     traffic = None if tb is None else int(tb * n_params)
 
     # end to end through the public API from pinned host memory
     e2e = None
-    if not args.no_e2e and ckpt:
+    if not args.no_e2e and K == 1:
         h0 = [t.cpu().pin_memory() for t in th0]
         h1 = [t.cpu().pin_memory() for t in experts[0]]
         del th0, experts
         torch.cuda.empty_cache()
         stage = iso.HostStaging(h0, h1, dev)
         for _ in range(2):
-            stage.run(h0, h1, op=op, update_is_delta=False, density=density, workspace=ws, ws_bytes=ws_bytes)
+            stage.run(h0, h1, op=op, update_is_delta=not ckpt, density=density, scope=scope,
+                      workspace=ws, ws_bytes=ws_bytes)
         torch.cuda.synchronize()
         f0, f1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         n_e2e = max(2, min(args.steps, 5))
         f0.record(stream)
         for _ in range(n_e2e):
-            stage.run(h0, h1, op=op, update_is_delta=False, density=density, workspace=ws, ws_bytes=ws_bytes)
+            stage.run(h0, h1, op=op, update_is_delta=not ckpt, density=density, scope=scope,
+                      workspace=ws, ws_bytes=ws_bytes)
         f1.record(stream)
         torch.cuda.synchronize()
         ms_e2e = f0.elapsed_time(f1) / n_e2e
@@ -263,7 +289,7 @@ def run_mine(args):
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        cpu = cpu_baseline(name, budget_s=args.cpu_budget)
+        cpu = cpu_baseline(name, budget_s=args.cpu_budget, rho=density)
 
     if rank == 0:
         line = {
@@ -271,9 +297,9 @@ def run_mine(args):
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms, 4),
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
             "dtype": "bf16" if ckpt else "f32", "data": "synthetic (seeded, Qwen-shaped; no checkpoints)",
-            "config": {"workload": name if args.layers is None else f"{name} ({args.layers} layers)",
+            "config": {"workload": name if not small else f"{name} (layers={args.layers}, widths/{args.scale})",
                        "description": desc, "params": n_params, "tensors": len(shapes),
-                       "experts": K, "op": op, "density": density, "scope": "tensor",
+                       "experts": K, "op": op, "density": density, "scope": scope,
                        "l2": "inputs larger than L2 (129 MB); no flush needed",
                        "parallelism": f"replica x{world}"},
             "hbm_gbs_step": round(step_gbs, 1),
@@ -306,13 +332,17 @@ def cpu_sample(name, seed=0):
     return shapes, order
 
 
-def cpu_baseline(name, budget_s=15.0, seed=0):
+def cpu_baseline(name, budget_s=15.0, seed=0, rho=None):
     """The oracle, as it stands, on a bounded sample of the workload: tensors
     are added in a fixed order until budget_s of single-thread CPU time."""
     import numpy as np
     import oracle
     import synth
-    shapes_name, K, op, inputs, density, _ = WORKLOADS[name]
+    shapes_name, K, op, inputs, density, scope, _ = WORKLOADS[name]
+    if rho is not None:
+        density = rho
+    if shapes_name == "sweep":
+        return cpu_baseline_sweep(name, density, scope, seed)
     shapes, order = cpu_sample(name, seed)
     orc_op = {"ta": oracle.TA, "ties": oracle.TIES, "iso": oracle.ISO}[op]
     done, params, spent = [], 0, 0.0
@@ -341,24 +371,45 @@ def cpu_baseline(name, budget_s=15.0, seed=0):
             "seconds": round(spent, 2)}
 
 
+def cpu_baseline_sweep(name, rho, scope, seed=0):
+    """The oracle on the whole density-sweep tensor (58.7 M entries)."""
+    import numpy as np
+    import torch
+    import oracle
+    import synth
+    s = (4096, 14336, False)
+    d = synth.density_sweep_delta(seed=seed, rho=rho)
+    b = synth.base_weights([s], seed=seed)[0]
+    a = b.view(torch.int16).numpy().view(np.uint16).reshape(s[0], s[1])
+    x = d.view(torch.int16).numpy().view(np.uint16).reshape(s[0], s[1])
+    sc = oracle.SCOPE_BLOCK if scope == "block" else oracle.SCOPE_TENSOR
+    t = time.perf_counter()
+    oracle.merge([a], [[x]], oracle.TIES, experts_are_deltas=True, density=rho, scope=sc)
+    spent = time.perf_counter() - t
+    return {"value": round(s[0] * s[1] / spent / 1e9, 6), "unit": UNIT, "cores": 1, "kind": "oracle",
+            "sample": f"the whole 4096x14336 tensor ({scope} scope, rho={rho}), timed on this host, "
+                      f"single thread", "seconds": round(spent, 2)}
+
+
 def run_reference(args):
     world = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
     if rank != 0:
         return
     name = args.workload
+    rho = args.density if args.density is not None else WORKLOADS[name][4]
     per_step = max(2.0, args.cpu_budget / max(1, args.steps))
     for _ in range(args.warmup and 1):
-        cpu_baseline(name, budget_s=0.5)
+        cpu_baseline(name, budget_s=0.5, rho=rho)
     vals = []
     for _ in range(args.steps):
-        vals.append(cpu_baseline(name, budget_s=per_step))
+        vals.append(cpu_baseline(name, budget_s=per_step, rho=rho))
     v = sum(x["value"] for x in vals) / len(vals)
     line = {
         "impl": "reference", "metric": METRIC, "value": round(v, 6), "unit": UNIT, "n_gpus": world,
         "steps": args.steps, "warmup": args.warmup, "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "f64 values / f32 decisions", "data": "synthetic (seeded, Qwen-shaped)",
-        "config": {"workload": name, "description": WORKLOADS[name][5]},
+        "config": {"workload": name, "description": WORKLOADS[name][6]},
         "cpu_baseline": {"value": round(v, 6), "unit": UNIT, "cores": 1, "kind": "oracle",
                          "sample": vals[-1]["sample"]},
         "e2e": {"value": round(v, 6), "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
@@ -373,12 +424,16 @@ def main():
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", choices=["mine", "reference"], default="mine")
     ap.add_argument("--workload", choices=sorted(WORKLOADS), default="qwen1.5b_update")
+    ap.add_argument("--density", type=float, default=None,
+                    help="TopKMask density (default: the workload's own)")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-budget", type=float, default=12.0)
     ap.add_argument("--layers", type=int, default=None,
                     help="decoder layers of the shape set (default: the model's own); "
                          "smaller cases are for profiling only")
+    ap.add_argument("--scale", type=int, default=1,
+                    help="divide every width of the shape set (profiling of small cases only)")
     args = ap.parse_args()
     if args.warmup < 3 and args.impl == "mine":
         args.warmup = 3

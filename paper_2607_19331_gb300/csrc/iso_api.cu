@@ -18,15 +18,11 @@
 namespace iso {
 namespace {
 
-#ifndef ISO_COUNT_BLOCKS_PER_SM
-#define ISO_COUNT_BLOCKS_PER_SM 3
-#endif
-constexpr int COUNT_GRID_PER_SM = ISO_COUNT_BLOCKS_PER_SM;
+constexpr int COUNT_GRID_PER_SM = COUNT_BLOCKS_PER_SM;
 #ifndef ISO_FUSED_BLOCKS_PER_SM
 #define ISO_FUSED_BLOCKS_PER_SM 2
 #endif
 constexpr int FUSED_GRID_PER_SM = ISO_FUSED_BLOCKS_PER_SM;
-constexpr int MERGE_GRID_PER_SM = 2;     // k_merge / k_gramk: 2 resident blocks of 256 per SM
 
 // ---------------------------------------------------------------------------
 // profiling and launch accounting
@@ -522,7 +518,7 @@ int run_group(const Call& c, int t0, int t1, char* ws, cudaStream_t s, const iso
             using XT = std::remove_pointer_t<decltype(xt)>;
             using BT = std::remove_pointer_t<decltype(bt)>;
             constexpr bool CK = decltype(ck)::value;
-            const int smem = BLOCK_MAX_ENTRIES * 4;
+            const int smem = (BLOCK_MAX_ENTRIES + BLOCK_MAX_ENTRIES / 32) * 4;
             ISO_TRY(smem_optin(k_block_select<XT, BT, CK>, smem));
             if (KU > 0)
                 ISO_TRY(launch(KD_BLOCK_SELECT, s, [&] { k_block_select<XT, BT, CK><<<KU, BLOCK_TPB, smem, s>>>(P); }));
@@ -558,12 +554,13 @@ int run_group(const Call& c, int t0, int t1, char* ws, cudaStream_t s, const iso
         using XT = std::remove_pointer_t<decltype(xt)>;
         using BT = std::remove_pointer_t<decltype(bt)>;
         constexpr bool CK = decltype(ck)::value;
-        const int mgrid = sms * MERGE_GRID_PER_SM;
+        const int mgrid = sms * MERGE_BLOCKS_PER_SM;
         if (gram_mode != GRAM_NONE) {
             if (need_gram_pass) {
                 auto gram = [&](auto kc) {
                     constexpr int KC = decltype(kc)::value;
-                    return launch(KD_GRAM, s, [&] { k_gramk<XT, BT, CK, KC><<<mgrid, TPB, 0, s>>>(P); });
+                    const int ggrid = sms * gram_blocks_per_sm(KC);
+                    return launch(KD_GRAM, s, [&] { k_gramk<XT, BT, CK, KC><<<ggrid, TPB, 0, s>>>(P); });
                 };
                 if (K == 1) ISO_TRY(gram(std::integral_constant<int, 1>{}));
                 else if (K == 2) ISO_TRY(gram(std::integral_constant<int, 2>{}));

@@ -38,9 +38,13 @@ __device__ void block_find_from_top_b(const uint32_t* hist, int nb, long long ra
     __syncthreads();
 }
 
+// keys sit at q + q / 32: a thread walking its own contiguous range and a
+// warp walking consecutive entries are both free of bank conflicts
+__device__ __forceinline__ int kpad(int q) { return q + (q >> 5); }
+
 template <typename XT, typename BT, bool CK>
 __global__ void __launch_bounds__(BLOCK_TPB) k_block_select(Plan P) {
-    extern __shared__ __align__(16) uint32_t s_keys[];      // BLOCK_MAX_ENTRIES
+    extern __shared__ __align__(16) uint32_t s_keys[];      // kpad(BLOCK_MAX_ENTRIES)
     __shared__ uint32_t s_hist[RADIX_BINS];
     __shared__ long long s_scan[33];
     __shared__ uint32_t s_scan32[33];
@@ -48,6 +52,7 @@ __global__ void __launch_bounds__(BLOCK_TPB) k_block_select(Plan P) {
     __shared__ int s_bin;
     __shared__ long long s_above;
     __shared__ long long s_cutq;
+    __shared__ uint32_t s_or;
 
     const int idx = blockIdx.x;
     const int i = idx / P.n_units, u = idx % P.n_units;
@@ -92,6 +97,9 @@ __global__ void __launch_bounds__(BLOCK_TPB) k_block_select(Plan P) {
     const void* x = P.xptr[i * P.n_tensors + t];
     // keys in block order (row-major inside the block)
     bool bad = false;
+    uint32_t kor = 0;                        // OR of the keys: trailing zero bits need no radix level
+    if (threadIdx.x == 0) s_or = 0;
+    __syncthreads();
     const bool vec = (w % VEC == 0) && (d.cols % VEC == 0) && (c0 % VEC == 0);
     if (vec) {
         const int w8 = (int)(w / VEC);
@@ -104,7 +112,8 @@ __global__ void __launch_bounds__(BLOCK_TPB) k_block_select(Plan P) {
             for (int j = 0; j < VEC; ++j) {
                 const uint32_t kk = key_of(tau[j]);
                 bad |= kk >= KEY_INF;
-                s_keys[q8 * VEC + j] = kk;
+                kor |= kk;
+                s_keys[kpad(q8 * VEC + j)] = kk;
             }
         }
     } else {
@@ -113,22 +122,28 @@ __global__ void __launch_bounds__(BLOCK_TPB) k_block_select(Plan P) {
             const long long e = (r0 + rr) * d.cols + c0 + cc;
             const uint32_t kk = key_of(TauSrc<XT, BT, CK>::load1(x, d.base, e));
             bad |= kk >= KEY_INF;
-            s_keys[q] = kk;
+            kor |= kk;
+            s_keys[kpad(q)] = kk;
         }
     }
     if (bad) set_status(P.hdr, ISO_ERR_NONFINITE);
+    kor = __reduce_or_sync(0xFFFFFFFFu, kor);
+    if ((threadIdx.x & 31) == 0 && kor) atomicOr(&s_or, kor);
     __syncthreads();
-    // k-th largest key
+    // k-th largest key: radix levels down to the lowest bit any key has set
+    // (bf16-valued task vectors leave the low 16 bits clear)
+    const int low = s_or ? __ffs(s_or) - 1 : 31;
     uint32_t prefix = 0;
     long long rank = k;
     int pshift = 31;
     for (;;) {
-        const int shift = pshift > RADIX_BITS ? pshift - RADIX_BITS : 0;
+        int shift = pshift > RADIX_BITS ? pshift - RADIX_BITS : 0;
+        if (shift < low) shift = low;
         const int nb = 1 << (pshift - shift);
         for (int q = threadIdx.x; q < nb; q += blockDim.x) s_hist[q] = 0;
         __syncthreads();
         for (int q = threadIdx.x; q < n; q += blockDim.x) {
-            const uint32_t v = s_keys[q];
+            const uint32_t v = s_keys[kpad(q)];
             if ((v >> pshift) == prefix) atomicAdd(&s_hist[(v >> shift) & (nb - 1)], 1u);
         }
         __syncthreads();
@@ -136,23 +151,23 @@ __global__ void __launch_bounds__(BLOCK_TPB) k_block_select(Plan P) {
         rank -= s_above;
         prefix = (prefix << (pshift - shift)) | (uint32_t)s_bin;
         __syncthreads();
-        if (shift == 0) break;
+        if (shift == low) break;
         pshift = shift;
     }
-    const uint32_t tk = prefix;
+    const uint32_t tk = prefix << low;
     // counts above / at the threshold, and the squared norm of the kept entries
     const int per = (n + blockDim.x - 1) / blockDim.x;
     const int q0 = threadIdx.x * per;
+    const bool want_gamma = (P.op == ISO_OP_ISO) && (P.K == 1);
     uint32_t above = 0, ties = 0;
     double gsum = 0.0;
     for (int q = q0; q < q0 + per && q < n; ++q) {
-        const uint32_t v = s_keys[q];
-        if (v > tk) {
-            above++;
+        const uint32_t v = s_keys[kpad(q)];
+        above += v > tk;
+        ties += v == tk;
+        if (want_gamma && v > tk) {
             const double f = (double)__uint_as_float(v);
             gsum += f * f;
-        } else if (v == tk) {
-            ties++;
         }
     }
     uint32_t tot_ties;
@@ -165,11 +180,10 @@ __global__ void __launch_bounds__(BLOCK_TPB) k_block_select(Plan P) {
         if ((long long)ties_before < need && need <= (long long)(ties_before + ties)) {
             uint32_t acc = ties_before;
             for (int q = q0; q < q0 + per && q < n; ++q)
-                if (s_keys[q] == tk && (long long)(++acc) == need) { s_cutq = q; break; }
+                if (s_keys[kpad(q)] == tk && (long long)(++acc) == need) { s_cutq = q; break; }
         }
     }
     __syncthreads();
-    const bool want_gamma = (P.op == ISO_OP_ISO) && (P.K == 1);
     double g = 0.0;
     if (want_gamma) g = block_sum(gsum, s_dred);
     if (threadIdx.x == 0) {

@@ -324,6 +324,31 @@ struct RawTile {
             }
         }
     }
+    // vector step v of the tile starting at tensor entry e0, with rem = numel - e0
+    // entries left in the tensor (32-bit offsets; no bounds tests on a whole tile)
+    __device__ __forceinline__ void load_step(int v, const void* xp, const void* bp, uint32_t e0,
+                                              uint32_t rem, int lane) {
+        const uint32_t o = (uint32_t)(v * (32 * VEC) + lane * VEC);
+        if (rem >= TILE) {
+            const char* xq = static_cast<const char*>(xp) + ((size_t)e0 + o) * sizeof(XT);
+#pragma unroll
+            for (int q = 0; q < NX; ++q) x[v][q] = ld_stream(xq + 16 * q);
+            if (CK) {
+                const char* bq = static_cast<const char*>(bp) + ((size_t)e0 + o) * sizeof(BT);
+#pragma unroll
+                for (int q = 0; q < NB; ++q) b[v][q] = ld_stream(bq + 16 * q);
+            }
+        } else if (o < rem) {
+            load_raw8<XT>(xp, (long long)e0 + o, (long long)e0 + rem, x[v]);
+            if (CK) load_raw8<BT>(bp, (long long)e0 + o, (long long)e0 + rem,
+                                  reinterpret_cast<uint4(&)[Lanes<BT>::N]>(b[v]));
+        } else {
+#pragma unroll
+            for (int q = 0; q < NX; ++q) x[v][q] = make_uint4(0, 0, 0, 0);
+#pragma unroll
+            for (int q = 0; q < NB; ++q) b[v][q] = make_uint4(0, 0, 0, 0);
+        }
+    }
     // tau = x (delta) or x - base (checkpoint), binary32
     __device__ __forceinline__ void tau(int v, float (&t)[8]) const {
         raw_to_f32<XT>(x[v], t);
@@ -428,6 +453,16 @@ __device__ __forceinline__ long long k_of_density(double rho, long long n) {
     if (kk < 0.0) kk = 0.0;
     if (kk > (double)n) kk = (double)n;
     return (long long)kk;
+}
+
+// s + e += x exactly as a binary32 pair (Knuth's two-sum: the rounding
+// error of s + x is carried in e)
+__device__ __forceinline__ void two_sum_add(float& s, float& e, float x) {
+    const float t = __fadd_rn(s, x);
+    const float bp = __fsub_rn(t, s);
+    const float err = __fadd_rn(__fsub_rn(s, __fsub_rn(t, bp)), __fsub_rn(x, bp));
+    s = t;
+    e = __fadd_rn(e, err);
 }
 
 __device__ __forceinline__ int bitlen32(uint32_t v) { return v ? 32 - __clz(v) : 0; }

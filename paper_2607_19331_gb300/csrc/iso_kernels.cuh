@@ -10,6 +10,7 @@ namespace iso {
 
 
 // select (TENSOR / GLOBAL scope)
+constexpr int COUNT_BLOCKS_PER_SM = 2;      // k_count: resident blocks of TPB threads per SM
 __global__ void k_init_units(Plan P, long long global_n);
 template <typename XT, typename BT, bool CK> __global__ void k_sample(Plan P);
 template <typename XT, typename BT, bool CK> __global__ void k_count(Plan P);
@@ -33,6 +34,8 @@ template <bool CK> __global__ void k_repair(Plan P);
 template <typename XT, typename BT, bool CK, int KC> __global__ void k_apply(Plan P);
 template <typename XT, typename BT, bool CK, int KC> __global__ void k_merge(Plan P);
 template <typename XT, typename BT, bool CK, int KC> __global__ void k_gramk(Plan P);
+constexpr int MERGE_BLOCKS_PER_SM = 2;                 // k_merge: resident blocks of TPB threads per SM
+constexpr int gram_blocks_per_sm(int KC) { return KC >= 8 ? 1 : 2; }
 __global__ void k_solve(Plan P, int gram_mode);
 template <typename XT> __global__ void k_mask(Plan P, uint32_t* const* mptr);
 __global__ void k_status(const Header* h, int32_t* out);

@@ -204,41 +204,79 @@ __device__ __forceinline__ uint32_t select_bits(const Plan& P, const TensorDesc&
     return bits;
 }
 
+// the merged output of one entry; every argument is in registers
 template <int KC>
-__device__ __forceinline__ float merged_value(const Plan& P, const MergeParams<KC>& mp, int K, float th0,
-                                              const float (&tau)[KC], uint32_t bits) {
+__device__ __forceinline__ float merged_value(int opk, bool iso1d, float lambda, int K, float th0,
+                                              const float (&tau)[KC], const float (&cf)[KC], uint32_t bits) {
     float upd;
-    if (mp.opk == OPK_SUM) {
+    if (opk == OPK_SUM) {
         float s = 0.0f;
 #pragma unroll
         for (int i = 0; i < KC; ++i)
             if (i < K) s = __fadd_rn(s, tau[i]);
-        upd = mp.iso1d ? __fdiv_rn(s, (float)K) : __fmul_rn(P.lambda, s);
-    } else if (mp.opk == OPK_TIES) {
+        upd = iso1d ? __fdiv_rn(s, (float)K) : __fmul_rn(lambda, s);
+    } else if (opk == OPK_TIES) {
+        // gamma = sign(sum of the trimmed values); the agreeing set holds the
+        // non-zero trimmed values of that sign (none when the sum is 0)
+        float tt[KC];
         float s = 0.0f;
 #pragma unroll
-        for (int i = 0; i < KC; ++i)
-            if (i < K) s = __fadd_rn(s, ((bits >> i) & 1u) ? tau[i] : 0.0f);
-        const int gam = sgnf(s);
+        for (int i = 0; i < KC; ++i) {
+            tt[i] = (i < K && ((bits >> i) & 1u)) ? tau[i] : 0.0f;
+            if (i < K) s = __fadd_rn(s, tt[i]);
+        }
+        const uint32_t sbit = __float_as_uint(s) & 0x80000000u;
         float a = 0.0f;
         int cnt = 0;
 #pragma unroll
         for (int i = 0; i < KC; ++i) {
-            if (i < K && ((bits >> i) & 1u) && tau[i] != 0.0f && sgnf(tau[i]) == gam) {
-                a = __fadd_rn(a, tau[i]);
-                ++cnt;
-            }
+            const bool agree = (i < K) && (tt[i] != 0.0f) && ((__float_as_uint(tt[i]) & 0x80000000u) == sbit);
+            a = agree ? __fadd_rn(a, tt[i]) : a;
+            cnt += agree;
         }
+        if (s == 0.0f) cnt = 0;
         const float m = cnt ? __fdiv_rn(a, (float)cnt) : 0.0f;
-        upd = __fmul_rn(P.lambda, m);
+        upd = __fmul_rn(lambda, m);
     } else {
         float s = 0.0f;
 #pragma unroll
         for (int i = 0; i < KC; ++i)
-            if (i < K && ((bits >> i) & 1u)) s = __fadd_rn(s, __fmul_rn(mp.cf[i], tau[i]));
+            if (i < K && ((bits >> i) & 1u)) s = __fadd_rn(s, __fmul_rn(cf[i], tau[i]));
         upd = s;
     }
     return (upd == 0.0f) ? th0 : __fadd_rn(th0, upd);
+}
+
+// Per-tile thresholds.  Inside a tile that lies wholly before (after) a unit's
+// cut, an entry with key == t is kept (dropped), so the selection is the
+// single comparison  (int)key > T  with T = t - 1 (T = t); keys are below 2^31.
+// A tile holding the cut, and BLOCK scope, take the exact per-entry test.
+template <int KC>
+__device__ __forceinline__ bool tile_thresholds(const MergeParams<KC>& mp, int K, uint32_t e0, uint32_t e1,
+                                                int (&T)[KC]) {
+    bool exact = (mp.sel == SEL_BLOCK);
+#pragma unroll
+    for (int i = 0; i < KC; ++i) {
+        T[i] = -1;
+        if (i < K && mp.sel == SEL_PACKED) {
+            const unsigned long long th = mp.thr[i];
+            const uint32_t tk = (uint32_t)(th >> 32), c32 = ~(uint32_t)th;
+            if (tk > 0x7FFFFFFEu) T[i] = 0x7FFFFFFF;          // nothing is kept
+            else if (e1 <= c32) T[i] = (int)tk - 1;            // ties kept
+            else if (e0 >= c32) T[i] = (int)tk;                // ties dropped
+            else exact = true;
+        }
+    }
+    return exact;
+}
+
+template <int KC>
+__device__ __forceinline__ uint32_t fast_bits(const int (&T)[KC], int K, const float (&tau)[KC]) {
+    uint32_t bits = 0;
+#pragma unroll
+    for (int i = 0; i < KC; ++i)
+        if (i < K && (int)key_of(tau[i]) > T[i]) bits |= 1u << i;
+    return bits;
 }
 
 // the warp's contiguous tile range
@@ -259,19 +297,15 @@ __device__ __forceinline__ long long tensor_tile_end(const Plan& P, int t) {
 
 }  // namespace
 
-// steps of one warp whose loads are issued together: KC 16-byte loads per
-// step, about 4 KB in flight per warp
-template <int KC, int SPT>
-struct Batch {
-    static constexpr int U0 = 8 / KC > 0 ? 8 / KC : 1;
-    static constexpr int U = U0 < SPT ? U0 : SPT;
-};
-
+// One warp per tile, a contiguous tile range per warp.  Each lane takes one
+// 16-byte vector of every expert per step (4 fp32 or 8 bf16 entries); up to
+// four experts, the next step's loads are issued before the current step is
+// merged.
 template <typename XT, typename BT, bool CK, int KC>
-__global__ void __launch_bounds__(TPB, 2) k_merge(Plan P) {
+__global__ void __launch_bounds__(TPB, MERGE_BLOCKS_PER_SM) k_merge(Plan P) {
     constexpr int E = 16 / (int)sizeof(XT);          // entries per lane per step
-    constexpr int SPT = TILE / (32 * E);             // steps per tile
-    constexpr int U = Batch<KC, SPT>::U;
+    constexpr int SPT = TILE / (32 * E);             // steps per tile (4 or 8)
+    static_assert(SPT % 2 == 0, "steps alternate between two buffers");
     const int K = P.K;
     const int lane = threadIdx.x & 31;
     const WarpRange wr = warp_range(P);
@@ -289,60 +323,97 @@ __global__ void __launch_bounds__(TPB, 2) k_merge(Plan P) {
         const TensorDesc& d = P.tens[t];
         const long long n = d.numel;
         const long long e0 = (g - d.tile_base) * TILE;
-#pragma unroll 1
-        for (int s0 = 0; s0 < SPT; s0 += U) {
-            Words<XT, E> xr[U][KC];
-            Words<BT, E> br[U];
+        const long long e1 = (e0 + TILE < n) ? e0 + TILE : n;
+        // this tile's parameters, in registers
+        const void* xs[KC];
+        float cf[KC];
+        int T[KC];
 #pragma unroll
-            for (int u = 0; u < U; ++u) {
-                const long long e = e0 + (long long)(s0 + u) * (32 * E) + lane * E;
-                if (e < n) {
-                    load_words<BT, E>(d.base, e, n, br[u]);
+        for (int i = 0; i < KC; ++i) { xs[i] = mp.xs[i]; cf[i] = mp.cf[i]; }
+        const bool exact = tile_thresholds<KC>(mp, K, (uint32_t)e0, (uint32_t)e1, T);
+        const int opk = mp.opk;
+        const bool iso1d = mp.iso1d;
+        const void* bp = d.base;
+        void* op = d.out;
+
+        Words<XT, E> xa[KC], xb[KC];
+        Words<BT, E> ba, bb;
+        auto load = [&](int st, Words<XT, E> (&x)[KC], Words<BT, E>& b) {
+            const long long e = e0 + (long long)st * (32 * E) + lane * E;
+            if (e < n) {
+                load_words<BT, E>(bp, e, n, b);
 #pragma unroll
-                    for (int i = 0; i < KC; ++i)
-                        if (i < K) load_words<XT, E>(mp.xs[i], e, n, xr[u][i]);
-                }
+                for (int i = 0; i < KC; ++i)
+                    if (i < K) load_words<XT, E>(xs[i], e, n, x[i]);
             }
+        };
+        auto merge_step = [&](int st, const Words<XT, E> (&x)[KC], const Words<BT, E>& b) {
+            const long long e = e0 + (long long)st * (32 * E) + lane * E;
+            if (e >= n) return;
+            long long r = 0, c = 0;
+            if (exact && mp.sel == SEL_BLOCK) { r = e / d.cols; c = e - r * d.cols; }
+            float o[E];
 #pragma unroll
-            for (int u = 0; u < U; ++u) {
-                const long long e = e0 + (long long)(s0 + u) * (32 * E) + lane * E;
-                if (e >= n) continue;
-                long long r = 0, c = 0;
-                if (mp.sel == SEL_BLOCK) { r = e / d.cols; c = e - r * d.cols; }
-                float o[E];
+            for (int j = 0; j < E; ++j) {
+                const float th0 = word_f32<BT, E>(b, j);
+                float tau[KC];
 #pragma unroll
-                for (int j = 0; j < E; ++j) {
-                    const float th0 = word_f32<BT, E>(br[u], j);
-                    float tau[KC];
-#pragma unroll
-                    for (int i = 0; i < KC; ++i) {
-                        tau[i] = (i < K) ? word_f32<XT, E>(xr[u][i], j) : 0.0f;
-                        if (CK) tau[i] = __fsub_rn(tau[i], th0);
-                    }
-                    const uint32_t bits = select_bits<KC>(P, d, mp, K, tau, e + j, r, c);
-                    o[j] = merged_value<KC>(P, mp, K, th0, tau, bits);
+                for (int i = 0; i < KC; ++i) {
+                    tau[i] = (i < K) ? word_f32<XT, E>(x[i], j) : 0.0f;
+                    if (CK) tau[i] = __fsub_rn(tau[i], th0);
                 }
-                store_out<BT, E>(d.out, e, n, o);
+                const uint32_t bits = exact ? select_bits<KC>(P, d, mp, K, tau, e + j, r, c)
+                                            : fast_bits<KC>(T, K, tau);
+                o[j] = merged_value<KC>(opk, iso1d, P.lambda, K, th0, tau, cf, bits);
+            }
+            store_out<BT, E>(op, e, n, o);
+        };
+        if (KC <= 4) {
+            load(0, xa, ba);
+#pragma unroll 1
+            for (int st = 0; st < SPT; st += 2) {
+                load(st + 1, xb, bb);
+                merge_step(st, xa, ba);
+                if (st + 2 < SPT) load(st + 2, xa, ba);
+                merge_step(st + 1, xb, bb);
+            }
+        } else {
+            // eight experts: one buffer (the registers of a second would spill)
+#pragma unroll 1
+            for (int st = 0; st < SPT; ++st) {
+                load(st, xa, ba);
+                merge_step(st, xa, ba);
             }
         }
     }
 }
+
+// steps of one warp whose loads are issued together in the Gram pass: KC
+// 16-byte loads per step, 4 KB in flight per warp; eight experts take two
+// steps (8 KB) and one block per SM, whose registers hold the 36 pair sums
+// and both steps
+template <int KC, int SPT>
+struct Batch {
+    static constexpr int U0 = KC >= 8 ? 2 : 8 / KC;
+    static constexpr int U = U0 < SPT ? U0 : SPT;
+};
 
 // Gram of the trimmed task vectors, upper triangle, per 2-D trimmed tensor.
 // Tile partials in binary32 (fused multiply-add over one lane's entries of
 // the tile, then a warp sum), accumulated per warp in binary64 and added to
 // the tensor's Gamma with one atomic per pair when the warp leaves the tensor.
 template <typename XT, typename BT, bool CK, int KC>
-__global__ void __launch_bounds__(TPB, 2) k_gramk(Plan P) {
+__global__ void __launch_bounds__(TPB, gram_blocks_per_sm(KC)) k_gramk(Plan P) {
     constexpr int E = 16 / (int)sizeof(XT);
     constexpr int SPT = TILE / (32 * E);
     constexpr int U = Batch<KC, SPT>::U;
     constexpr int NP = KC * (KC + 1) / 2;
-    __shared__ double s_g[WPB][NP];
+    static_assert(NP <= 64, "two pair sums per lane");
     const int K = P.K;
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-    for (int q = lane; q < NP; q += 32) s_g[warp][q] = 0.0;
-    __syncwarp();
+    // lane L accumulates pairs L and 32 + L over the warp's tiles of one
+    // tensor as binary32 two-sum pairs (no binary64 arithmetic per tile)
+    float gs0 = 0.0f, ge0 = 0.0f, gs1 = 0.0f, ge1 = 0.0f;
     const WarpRange wr = warp_range(P);
     if (wr.beg >= wr.end) return;
     int t = tensor_of_tile(P.tens, P.n_tensors, wr.beg);
@@ -351,17 +422,18 @@ __global__ void __launch_bounds__(TPB, 2) k_gramk(Plan P) {
     MergeParams<KC>& mp = s_mp[warp];
     merge_params<KC>(P, t, K, mp);
     auto flush = [&](int tt) {
-        __syncwarp();
-        if (lane == 0) {
-            int q = 0;
-            for (int a = 0; a < KC; ++a)
-                for (int b = a; b < KC; ++b, ++q)
-                    if (a < K && b < K && s_g[warp][q] != 0.0) {
-                        atomicAdd(&P.gram[((long long)tt * K + a) * K + b], s_g[warp][q]);
-                        s_g[warp][q] = 0.0;
-                    }
+        int q = 0;
+#pragma unroll
+        for (int a = 0; a < KC; ++a) {
+#pragma unroll
+            for (int b = a; b < KC; ++b, ++q) {
+                if (a < K && b < K && (lane == q || lane + 32 == q)) {
+                    const double v = (lane == q) ? (double)gs0 + (double)ge0 : (double)gs1 + (double)ge1;
+                    if (v != 0.0) atomicAdd(&P.gram[((long long)tt * K + a) * K + b], v);
+                }
+            }
         }
-        __syncwarp();
+        gs0 = ge0 = gs1 = ge1 = 0.0f;
     };
     for (long long g = wr.beg; g < wr.end; ++g) {
         if (g >= t_end) {
@@ -373,6 +445,9 @@ __global__ void __launch_bounds__(TPB, 2) k_gramk(Plan P) {
         if (!mp.trimmed2d) continue;
         const long long n = d.numel;
         const long long e0 = (g - d.tile_base) * TILE;
+        const long long e1 = (e0 + TILE < n) ? e0 + TILE : n;
+        int T[KC];
+        const bool exact = tile_thresholds<KC>(mp, K, (uint32_t)e0, (uint32_t)e1, T);
         float acc[NP];
 #pragma unroll
         for (int q = 0; q < NP; ++q) acc[q] = 0.0f;
@@ -395,7 +470,7 @@ __global__ void __launch_bounds__(TPB, 2) k_gramk(Plan P) {
                 const long long e = e0 + (long long)(s0 + u) * (32 * E) + lane * E;
                 if (e >= n) continue;
                 long long r = 0, c = 0;
-                if (mp.sel == SEL_BLOCK) { r = e / d.cols; c = e - r * d.cols; }
+                if (exact && mp.sel == SEL_BLOCK) { r = e / d.cols; c = e - r * d.cols; }
 #pragma unroll
                 for (int j = 0; j < E; ++j) {
                     float tau[KC];
@@ -405,7 +480,9 @@ __global__ void __launch_bounds__(TPB, 2) k_gramk(Plan P) {
                         tau[i] = (i < K) ? word_f32<XT, E>(xr[u][i], j) : 0.0f;
                         if (CK) tau[i] = __fsub_rn(tau[i], th0);
                     }
-                    const uint32_t bits = (e + j < n) ? select_bits<KC>(P, d, mp, K, tau, e + j, r, c) : 0u;
+                    uint32_t bits = 0;
+                    if (e + j < n) bits = exact ? select_bits<KC>(P, d, mp, K, tau, e + j, r, c)
+                                                : fast_bits<KC>(T, K, tau);
                     float m[KC];
 #pragma unroll
                     for (int i = 0; i < KC; ++i) m[i] = ((bits >> i) & 1u) ? tau[i] : 0.0f;
@@ -417,6 +494,7 @@ __global__ void __launch_bounds__(TPB, 2) k_gramk(Plan P) {
                 }
             }
         }
+        float w0 = 0.0f, w1 = 0.0f;
         int q = 0;
 #pragma unroll
         for (int a = 0; a < KC; ++a) {
@@ -424,10 +502,13 @@ __global__ void __launch_bounds__(TPB, 2) k_gramk(Plan P) {
             for (int b = a; b < KC; ++b, ++q) {
                 if (a < K && b < K) {
                     const float w = warp_sum(acc[q]);
-                    if (lane == 0) s_g[warp][q] += (double)w;
+                    if (q < 32) w0 = (lane == q) ? w : w0;
+                    else w1 = (lane + 32 == q) ? w : w1;
                 }
             }
         }
+        two_sum_add(gs0, ge0, w0);
+        if (NP > 32) two_sum_add(gs1, ge1, w1);
     }
     flush(t);
 }

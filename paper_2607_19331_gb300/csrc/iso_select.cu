@@ -21,7 +21,7 @@
 // Work layout: a tile is 1024 entries handled by one warp; every warp (or
 // block) walks a contiguous range of (expert, tile) items, so the owning
 // tensor and unit change rarely and are tracked incrementally.
-#include "iso_internal.cuh"
+#include "iso_kernels.cuh"
 
 namespace iso {
 
@@ -227,16 +227,54 @@ __global__ void __launch_bounds__(SAMPLE_TPB) k_sample(Plan P) {
 // slot j*32 + L, conflict-free; every key is written and only a band key
 // advances the lane's slot -- and then copied, per lane, to the unit's
 // candidate segment.  The radix select and the tie counts work on that set.
-#ifndef ISO_COUNT_BLOCKS_PER_SM
-#define ISO_COUNT_BLOCKS_PER_SM 3
-#endif
-constexpr int COUNT_BLOCKS_PER_SM = ISO_COUNT_BLOCKS_PER_SM;
+//
+// The warp's tiles stream through two register buffers: the next tile's loads
+// are issued before the current tile is processed.  A non-finite tau has a key
+// above every finite key, so it is either above hi, where it turns the lane's
+// binary32 sum of tau^2 non-finite (then the tile is re-checked key by key),
+// or a band key, checked when the band keys are copied; lo itself is a sampled
+// key, so a non-finite lo is a band key of its own unit.
+
+// consecutive items of one (expert, tensor) that the count pass visits
+struct CountRun {
+    uint32_t it0, end;       // items [it0, end), end clipped to the warp's range
+    uint32_t e0;             // tensor entry of item it0's first element
+    uint32_t n;              // tensor entries
+    uint32_t rec;            // index of item it0 in the per-(expert, tile) arrays
+    const void* xp;
+    const void* bp;
+    Unit* U;
+};
+
+// the first counted run at or after item it (< end); false if there is none
+__device__ __forceinline__ bool count_run_at(const Plan& P, uint32_t it, uint32_t end, CountRun& r) {
+    while (it < end) {
+        Cursor c;
+        cursor_at(P, it, c);
+        const uint32_t re = min((uint32_t)c.run_end, end);
+        Unit* U = count_unit(P, c);
+        if (U) {
+            const TensorDesc& d = P.tens[c.t];
+            r.it0 = it;
+            r.end = re;
+            r.e0 = (uint32_t)(c.g - d.tile_base) * TILE;
+            r.n = (uint32_t)d.numel;
+            r.rec = (uint32_t)((long long)c.i * P.n_tiles + c.g);
+            r.xp = P.xptr[c.i * P.n_tensors + c.t];
+            r.bp = d.base;
+            r.U = U;
+            return true;
+        }
+        it = re;
+    }
+    return false;
+}
 
 template <typename XT, typename BT, bool CK>
 __global__ void __launch_bounds__(TPB, COUNT_BLOCKS_PER_SM) k_count(Plan P) {
     __shared__ uint32_t s_band[WPB][TILE + 32];
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-    uint32_t* sbl = s_band[warp] + lane;
+    uint32_t* const sbl = s_band[warp] + lane;
     // item indices fit 32 bits (the host checks K * n_tiles < 2^31)
     const uint32_t W = gridDim.x * WPB;
     const uint32_t wid = blockIdx.x * WPB + warp;
@@ -246,21 +284,26 @@ __global__ void __launch_bounds__(TPB, COUNT_BLOCKS_PER_SM) k_count(Plan P) {
     const uint32_t end = min(items, beg + per);
     if (beg >= end) return;
     const unsigned FULL = 0xFFFFFFFFu;
-    const unsigned lt_mask = (1u << lane) - 1u;
+
+    CountRun r;
+    if (!count_run_at(P, beg, end, r)) return;
 
     // per-unit accumulators (warp-uniform) and the candidate chunk
     Unit* au = nullptr;
     uint32_t a_gt = 0, a_int = 0, a_hi = 0, a_lo = 0;
-    double d_gg = 0.0, d_gb = 0.0;                // per-lane sums of tau^2: above hi, band above lo
+    // per-lane sums of tau^2 (above hi; band keys above lo) as binary32
+    // pairs: sum + error term, kept exact by two-sum, so no binary64
+    // arithmetic runs per tile
+    float s_gg = 0.0f, e_gg = 0.0f, s_gb = 0.0f, e_gb = 0.0f;
     uint32_t* cseg = nullptr;                     // the unit's candidate segment
     uint32_t ch_pos = 0, ch_left = 0, cap = 0;
     bool ovf = false;
-    uint32_t lo = 0, hi = 0, span = 0;
+    uint32_t lo = 0, hi = 0;
     bool want_gamma = false;
 
     auto flush = [&]() {
         if (!au) return;
-        const double gg = warp_sum(d_gg), gb = warp_sum(d_gb);
+        const double gg = warp_sum((double)s_gg + (double)e_gg), gb = warp_sum((double)s_gb + (double)e_gb);
         if (lane == 0) {
             if (a_gt) atomicAdd(&au->c_gt, (unsigned long long)a_gt);
             if (a_int) atomicAdd(&au->n_int, (unsigned long long)a_int);
@@ -273,65 +316,50 @@ __global__ void __launch_bounds__(TPB, COUNT_BLOCKS_PER_SM) k_count(Plan P) {
             if (ovf) au->overflow = 1;
         }
         a_gt = a_int = a_hi = a_lo = 0;
-        d_gg = d_gb = 0.0;
+        s_gg = e_gg = s_gb = e_gb = 0.0f;
     };
 
-    // the current (expert, tensor) run: items [it0, run_end) are tiles g0.. of one tensor
-    uint32_t run_end = beg, it0 = beg, g0 = 0, row = 0, n = 0, tile_base = 0;
-    const void* xp = nullptr;
-    const void* bp = nullptr;
-    uint32_t it = beg;
-    while (it < end) {
-        if (it >= run_end) {
-            Cursor c;
-            cursor_at(P, it, c);
-            run_end = (uint32_t)c.run_end;
-            Unit* U = count_unit(P, c);
-            if (!U) { it = run_end; continue; }
-            const TensorDesc& d = P.tens[c.t];
-            n = (uint32_t)d.numel;
-            tile_base = (uint32_t)d.tile_base;
-            xp = P.xptr[c.i * P.n_tensors + c.t];
-            bp = d.base;
-            it0 = it;
-            g0 = (uint32_t)c.g;
-            row = (uint32_t)(c.i * P.n_tiles);
-            if (U != au) {
-                flush();
-                au = U;
-                lo = U->lo;
-                hi = U->hi;
-                span = hi - lo;
-                want_gamma = U->want_gamma != 0;
-                cap = (uint32_t)U->cand_cap;
-                cseg = P.cand + U->cand_off;
-                ch_left = 0;
-                ovf = false;
-            }
+    // Count one tile held in registers (item it of run rr).  As each vector
+    // step is converted to tau, its registers are refilled with the same step
+    // of the next tile (item it2 of run r2), so a whole tile of loads is in
+    // flight while this one is counted.
+    RawTile<XT, BT, CK> rt;
+    auto count_tile = [&](const CountRun& rr, uint32_t it, bool more, const CountRun& r2, uint32_t it2) {
+        if (rr.U != au) {
+            flush();
+            au = rr.U;
+            lo = au->lo;
+            hi = au->hi;
+            want_gamma = au->want_gamma != 0;
+            cap = (uint32_t)au->cand_cap;
+            cseg = P.cand + au->cand_off;
+            ch_left = 0;
+            ovf = false;
         }
-        const uint32_t g = g0 + (it - it0);
-        const uint32_t e0 = (g - tile_base) * TILE;
-        RawTile<XT, BT, CK> rt;
-        rt.load(xp, bp, e0, n, lane);
-        const bool full = e0 + TILE <= n;
+        const uint32_t e0 = rr.e0 + (it - rr.it0) * TILE;
+        const uint32_t rem = rr.n - e0;           // > 0
+        const uint32_t rec = rr.rec + (it - rr.it0);
+        const uint32_t ne0 = more ? r2.e0 + (it2 - r2.it0) * TILE : 0u;
+        const uint32_t nrem = more ? r2.n - ne0 : 0u;
 
-        // pass 1: every entry (a full tile needs no bounds test)
-        uint32_t n_gt = 0, nb = 0, kmax = 0;
-        float f_gg = 0.0f;
-        if (full) {
+        // pass 1: every entry
+        uint32_t n_gt = 0;
+        float f_gg = 0.0f;                         // tau^2 above hi (also the non-finite detector)
+        uint32_t* sp = sbl;
+        if (rem >= TILE) {
 #pragma unroll
             for (int v = 0; v < WVEC; ++v) {
                 float tau[VEC];
                 rt.tau(v, tau);
+                if (more) rt.load_step(v, r2.xp, r2.bp, ne0, nrem, lane);
 #pragma unroll
                 for (int j = 0; j < VEC; ++j) {
                     const uint32_t kk = key_of(tau[j]);
-                    kmax = max(kmax, kk);
                     const bool gt = kk > hi;
                     n_gt += gt;
-                    if (want_gamma && gt) f_gg = __fmaf_rn(tau[j], tau[j], f_gg);
-                    sbl[nb * 32] = kk;
-                    nb += (kk - lo <= span);
+                    f_gg = gt ? __fmaf_rn(tau[j], tau[j], f_gg) : f_gg;
+                    *sp = kk;
+                    sp += ((kk >= lo) & !gt) ? 32 : 0;
                 }
             }
         } else {
@@ -339,22 +367,36 @@ __global__ void __launch_bounds__(TPB, COUNT_BLOCKS_PER_SM) k_count(Plan P) {
             for (int v = 0; v < WVEC; ++v) {
                 float tau[VEC];
                 rt.tau(v, tau);
-                const uint32_t e = e0 + v * (32 * VEC) + lane * VEC;
+                if (more) rt.load_step(v, r2.xp, r2.bp, ne0, nrem, lane);
+                const uint32_t o = (uint32_t)(v * (32 * VEC) + lane * VEC);
 #pragma unroll
                 for (int j = 0; j < VEC; ++j) {
-                    if (e + j >= n) continue;
+                    if (o + j >= rem) continue;
                     const uint32_t kk = key_of(tau[j]);
-                    kmax = max(kmax, kk);
                     const bool gt = kk > hi;
                     n_gt += gt;
-                    if (want_gamma && gt) f_gg = __fmaf_rn(tau[j], tau[j], f_gg);
-                    sbl[nb * 32] = kk;
-                    nb += (kk - lo <= span);
+                    f_gg = gt ? __fmaf_rn(tau[j], tau[j], f_gg) : f_gg;
+                    *sp = kk;
+                    sp += ((kk >= lo) & !gt) ? 32 : 0;
                 }
             }
         }
-        if (__any_sync(FULL, kmax >= KEY_INF) && lane == 0) set_status(P.hdr, ISO_ERR_NONFINITE);
-        if (want_gamma) d_gg += (double)f_gg;
+        const uint32_t nb = (uint32_t)(sp - sbl) >> 5;
+        if (__any_sync(FULL, !(fabsf(f_gg) <= 3.402823466e38f))) {
+            // a non-finite (or overflowing) sum: read the tile's keys again
+            uint32_t kmax = 0;
+            for (int v = 0; v < WVEC; ++v) {
+                const uint32_t o = (uint32_t)(v * (32 * VEC) + lane * VEC);
+                if (o >= rem) break;
+                float tau[VEC];
+                TauSrc<XT, BT, CK>::load8(rr.xp, rr.bp, (long long)e0 + o, (long long)rr.n, tau);
+#pragma unroll
+                for (int j = 0; j < VEC; ++j)
+                    if (o + j < rem) kmax = max(kmax, key_of(tau[j]));
+            }
+            if (__any_sync(FULL, kmax >= KEY_INF) && lane == 0) set_status(P.hdr, ISO_ERR_NONFINITE);
+        }
+        if (want_gamma) two_sum_add(s_gg, e_gg, f_gg);
         __syncwarp();
 
         // pass 2: copy the staged band keys to the unit's candidate segment
@@ -364,7 +406,7 @@ __global__ void __launch_bounds__(TPB, COUNT_BLOCKS_PER_SM) k_count(Plan P) {
             unsigned long long start = 0;
             uint32_t req = 0;
             if (lane == 0) {
-                const uint32_t left = min(run_end, end) - it;
+                const uint32_t left = rr.end - it;
                 const unsigned long long want = (unsigned long long)t_int * (unsigned long long)left;
                 req = (uint32_t)max((unsigned long long)t_int, min((unsigned long long)CHUNK_MAX, want));
                 start = atomicAdd(&au->n_alloc, (unsigned long long)req);
@@ -375,7 +417,7 @@ __global__ void __launch_bounds__(TPB, COUNT_BLOCKS_PER_SM) k_count(Plan P) {
             else { ch_pos = (uint32_t)start; ch_left = req; }
         }
         const bool store = t_int && !ovf;
-        uint32_t n_hi = 0, n_lo = 0;
+        uint32_t n_hi = 0, n_lo = 0, kbad = 0;
         float f_band = 0.0f;                      // tau^2 over the band keys above lo
         {
             uint32_t* dst = cseg + ch_pos + off;
@@ -384,22 +426,44 @@ __global__ void __launch_bounds__(TPB, COUNT_BLOCKS_PER_SM) k_count(Plan P) {
                 if (store) dst[q] = kk;
                 n_hi += (kk == hi);
                 n_lo += (kk == lo) && (kk != hi);
+                kbad |= (kk >= KEY_INF);
                 if (want_gamma && kk != lo) { const float f = __uint_as_float(kk); f_band = __fmaf_rn(f, f, f_band); }
             }
         }
-        if (want_gamma) d_gb += (double)f_band;
+        if (__any_sync(FULL, kbad) && lane == 0) set_status(P.hdr, ISO_ERR_NONFINITE);
+        if (want_gamma) two_sum_add(s_gb, e_gb, f_band);
         const uint32_t t_gt = __reduce_add_sync(FULL, n_gt);
         const uint32_t t_hi = __reduce_add_sync(FULL, n_hi);
         const uint32_t t_lo = __reduce_add_sync(FULL, n_lo);
         if (lane == 0) {
-            P.tcand[row + g] = make_uint2(store ? ch_pos : 0u, store ? t_int : 0u);
-            P.teq_lo[row + g] = t_lo;
-            P.teq_hi[row + g] = t_hi;
+            P.tcand[rec] = make_uint2(store ? ch_pos : 0u, store ? t_int : 0u);
+            P.teq_lo[rec] = t_lo;
+            P.teq_hi[rec] = t_hi;
         }
         if (store) { ch_pos += t_int; ch_left -= t_int; }
         a_gt += t_gt; a_int += t_int; a_hi += t_hi; a_lo += t_lo;
         __syncwarp();
-        ++it;
+    };
+
+    uint32_t it = r.it0;
+    {
+        const uint32_t e0 = r.e0;
+#pragma unroll
+        for (int v = 0; v < WVEC; ++v) rt.load_step(v, r.xp, r.bp, e0, r.n - e0, lane);
+    }
+    for (;;) {
+        // the next item: the same run, or the next counted run
+        uint32_t it2 = it + 1;
+        CountRun r2 = r;
+        bool more = true;
+        if (it2 >= r.end) {
+            more = count_run_at(P, r.end, end, r2);
+            it2 = r2.it0;
+        }
+        count_tile(r, it, more, r2, it2);
+        if (!more) break;
+        it = it2;
+        r = r2;
     }
     flush();
 }

@@ -1,0 +1,135 @@
+"""GPU parity at the workloads' full sizes, in the benchmark's launch
+configuration, checked against the oracle on sampled tensors.
+
+* Qwen2.5-7B-shaped masked ISO update (bf16 base + RL checkpoint, 254
+  tensors, per-tensor TopKMask 5 %);
+* the density sweep on one bf16 4096 x 14336 task vector with 1000 entries
+  moved onto the threshold (per-tensor and per-128x128-block TopKMask at
+  rho = 1, 5, 20, 50 %), every entry checked;
+* the Qwen2.5-7B-shaped merge of 8 fp32 RL deltas into a bf16 base (TopKMask
+  10 % per delta, TIES and the ISO retention rule), which holds ~274 GB of
+  inputs and outputs on the device.
+
+Each selection unit is an independent problem, so a tensor checked alone by
+the oracle must match the same tensor inside the whole-model call.
+"""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+import paper_2607_19331_gb300 as iso
+import synth
+from paper_2607_19331_gb300 import _abi
+from parity_util import assert_units_equal, assert_values_close, to_np, unpack_mask
+
+pytestmark = pytest.mark.gpu
+DEV = "cuda:0"
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _cuda():
+    assert torch.cuda.is_available(), "GPU tests need CUDA"
+    torch.cuda.set_device(0)
+    _abi.lib()
+    yield
+    torch.cuda.empty_cache()
+
+
+def _qwen7b_index(layer, which):
+    """Position of a per-layer tensor in the Qwen2.5-7B list (embedding first)."""
+    names = ["q", "k", "v", "o", "gate", "up", "down", "norm1", "norm2"]
+    return 1 + layer * 9 + names.index(which)
+
+
+def _workspace_bytes(tensors, K, op, density):
+    """The benchmark's rule: the full workspace if it fits, else what fits."""
+    mn, full = iso.iso_workspace_size(tensors, K, iso.merge_cfg(op, density, "tensor"))
+    free = torch.cuda.mem_get_info()[0]
+    return full if full + (1 << 30) < free else max(mn, free - (2 << 30))
+
+
+def test_full_size_qwen7b_update_sampled():
+    shapes = synth.qwen_shapes("qwen7b")
+    th0, th1 = synth.rl_update_set(shapes, seed=0, device=DEV)
+    out = [torch.empty_like(t) for t in th0]
+    ws = iso.Workspace(DEV)
+    ws_bytes = _workspace_bytes(th0, 1, "iso", 0.05)
+    ws.get(ws_bytes)
+    out, st = iso.iso_update(th0, th1, op="iso", density=0.05, scope="tensor", stats=True,
+                             out=out, workspace=ws, ws_bytes=ws_bytes)
+    torch.cuda.synchronize()
+    assert int(st.status.item()) == 0
+    units = st.units_numpy()[0]
+    picks = [_qwen7b_index(0, "k"), _qwen7b_index(0, "norm1"), _qwen7b_index(13, "v"),
+             _qwen7b_index(27, "down"), _qwen7b_index(27, "o")]
+    for q in picks:
+        r_, c_, one = shapes[q]
+        a, b = to_np(th0[q]), to_np(th1[q])
+        r = oracle.update([a.reshape(r_, c_)], [b.reshape(r_, c_)], oracle.ISO, update_is_delta=False,
+                          density=0.05, is_1d=[one])
+        assert_values_close(to_np(out[q]), r["out64"][0], r["mag"][0], f"7B tensor {q}")
+        assert_units_equal(units[q:q + 1], r["units"][0], f"7B unit {q}")
+    del th0, th1, out, ws
+    torch.cuda.empty_cache()
+
+
+@pytest.mark.parametrize("rho", [0.01, 0.05, 0.2, 0.5])
+def test_density_sweep_full_size(rho):
+    s = (4096, 14336, False)
+    delta = synth.density_sweep_delta(seed=0, rho=rho, device=DEV)
+    base = synth.base_weights([s], seed=0, device=DEV)[0]
+    d_np, b_np = to_np(delta).reshape(s[0], s[1]), to_np(base).reshape(s[0], s[1])
+    for scope, oscope in (("tensor", oracle.SCOPE_TENSOR), ("block", oracle.SCOPE_BLOCK)):
+        masks, mst = iso.iso_topk_mask([delta], density=rho, scope=scope, stats=True)
+        out, st = iso.iso_update([base], [delta], op="ties", update_is_delta=True, density=rho,
+                                 scope=scope, lam=1.0, stats=True)
+        torch.cuda.synchronize()
+        assert int(mst.status.item()) == 0 and int(st.status.item()) == 0
+        r = oracle.update([b_np], [d_np], oracle.TIES, update_is_delta=True, density=rho,
+                          scope=oscope, lam=1.0)
+        what = f"sweep rho={rho} {scope}"
+        assert np.array_equal(unpack_mask(masks[0], delta.numel()), r["masks"][0][0]), what + " mask"
+        assert_units_equal(mst.units_numpy()[0], r["units"][0], what + " mask units")
+        assert_units_equal(st.units_numpy()[0], r["units"][0], what + " update units")
+        assert_values_close(to_np(out[0]), r["out64"][0], r["mag"][0], what)
+        if scope == "tensor":
+            u = r["units"][0][0]
+            assert u["ties_at_thresh"] >= 1001, "the injected ties sit at the threshold"
+            assert 0 < u["ties_taken"] < u["ties_at_thresh"]
+    del delta, base, masks, out
+    torch.cuda.empty_cache()
+
+
+def test_full_size_qwen7b_merge_k8_sampled():
+    shapes = synth.qwen_shapes("qwen7b")
+    K = 8
+    th0 = synth.base_weights(shapes, seed=0, device=DEV)
+    taus, _ = synth.merge_experts(shapes, seed=0, K=K, device=DEV)
+    torch.cuda.empty_cache()
+    out = [torch.empty_like(t) for t in th0]
+    ws = iso.Workspace(DEV)
+    ws_bytes = _workspace_bytes(th0, K, "iso", 0.1)
+    ws.get(ws_bytes)
+    picks = [_qwen7b_index(0, "k"), _qwen7b_index(0, "norm2"), _qwen7b_index(13, "q"),
+             _qwen7b_index(27, "v")]
+    for op, oop in (("ties", oracle.TIES), ("iso", oracle.ISO)):
+        out, st = iso.iso_merge(th0, taus, op=op, experts_are_deltas=True, out=out, density=0.1,
+                                scope="tensor", lam=1.0, stats=True, workspace=ws, ws_bytes=ws_bytes)
+        torch.cuda.synchronize()
+        assert int(st.status.item()) == 0
+        units = st.units_numpy()
+        coef = st.coef.cpu().numpy().reshape(-1, K) if op == "iso" else None
+        for q in picks:
+            r_, c_, one = shapes[q]
+            a = to_np(th0[q]).reshape(r_, c_)
+            ex = [[to_np(taus[i][q]).reshape(r_, c_)] for i in range(K)]
+            r = oracle.merge([a], ex, oop, experts_are_deltas=True, density=0.1, lam=1.0,
+                             is_1d=[one])
+            what = f"7B K=8 {op} tensor {q}"
+            assert_values_close(to_np(out[q]), r["out64"][0], r["mag"][0], what)
+            assert_units_equal(units[:, q:q + 1], r["units"], what)
+            if op == "iso" and not one:
+                np.testing.assert_allclose(coef[q], r["coef"][0], rtol=1e-5, atol=1e-9)
+    del th0, taus, out, ws
+    torch.cuda.empty_cache()
