@@ -23,6 +23,8 @@ import time
 ROOT = os.path.dirname(os.path.abspath(__file__))
 sys.path.insert(0, ROOT)
 
+from paper_2607_19331_gb300.shard import job_throughput, reduce_step_ms  # noqa: E402
+
 METRIC = "G params/s and achieved HBM GB/s (% of ~8 TB/s) for full-model mask+merge"
 UNIT = "Gparams/s"
 NOMINAL_HBM_GBS = 8000.0
@@ -48,11 +50,20 @@ WORKLOADS = {
 }
 
 
-def algorithmic_bytes(shapes, K, inputs, op, scope="tensor"):
+def fused_pass(K, inputs, op, scope, two_pass=False):
+    """Whether the library runs the K = 1 update as its fused single pass
+    (bf16 base and update, per-tensor TopKMask, a trimming operator)."""
+    return (not two_pass and K == 1 and scope == "tensor" and op != "ta"
+            and inputs in ("ckpt_bf16", "delta_bf16"))
+
+
+def algorithmic_bytes(shapes, K, inputs, op, scope="tensor", two_pass=False):
     """Bytes each full pass must move at minimum, per kernel kind.
 
     apply:        read theta_0 and the K experts once, write the output once
-    count:        (per-tensor scope) read the K task vectors once
+    count:        (per-tensor scope) read the K task vectors once; in the fused
+                  K = 1 pass this kernel is the whole update (read theta_0 and
+                  the expert, write the output) and there is no apply pass
     block_select: (per-block scope) read the K task vectors once
     gram:         (ISO, K >= 2) read the K task vectors once
     """
@@ -60,6 +71,8 @@ def algorithmic_bytes(shapes, K, inputs, op, scope="tensor"):
     n_trim = sum(r * c for r, c, one in shapes if not (one and op == "iso"))
     per_x = {"ckpt_bf16": 2, "delta_bf16": 2, "delta_f32": 4}[inputs]
     per_base, per_out = 2, 2
+    if fused_pass(K, inputs, op, scope, two_pass):
+        return {"count": n_all * (per_base + per_x + per_out)}
     read_tau = n_trim * (K * per_x + (per_base if inputs == "ckpt_bf16" else 0))
     out = {"apply": n_all * (per_base + K * per_x + per_out)}
     if op != "ta":
@@ -155,7 +168,10 @@ class Clocks:
                 "reasons": reasons, "samples": len(rows)}
 
 
-def make_workload(name, device, seed, layers=None, density=None, scale=1):
+def make_workload(name, device, seed, layers=None, density=None, scale=1, shard=None):
+    """The workload's tensors on `device`; with shard = (rank, world) only the
+    tensors shard_tensors assigns to this rank (the same seeded values the
+    whole set would hold)."""
     import torch
     import synth
     shapes_name, K, op, inputs, d0, scope, desc = WORKLOADS[name]
@@ -173,6 +189,13 @@ def make_workload(name, device, seed, layers=None, density=None, scale=1):
     else:
         th0 = synth.base_weights(shapes, seed=seed, device=device)
         experts, _ = synth.merge_experts(shapes, seed=seed, K=K, device=device)
+    if shard is not None:
+        from paper_2607_19331_gb300.shard import shard_tensors
+        mine = shard_tensors([r * c for r, c, _ in shapes], shard[1])[shard[0]]
+        shapes = [shapes[q] for q in mine]
+        th0 = [th0[q] for q in mine]
+        experts = [[e[q] for q in mine] for e in experts]
+        torch.cuda.empty_cache()
     torch.cuda.synchronize()
     return shapes, th0, experts
 
@@ -193,11 +216,18 @@ def run_mine(args):
     shapes_name, K, op, inputs, density, scope, desc = WORKLOADS[name]
     if args.density is not None:
         density = args.density
-    shapes, th0, experts = make_workload(name, dev, seed=rank, layers=args.layers, density=density,
-                                         scale=args.scale)
+    shapes, th0, experts = make_workload(name, dev, seed=0 if args.shard else rank, layers=args.layers,
+                                         density=density, scale=args.scale,
+                                         shard=(rank, world) if args.shard else None)
     n_params = sum(t.numel() for t in th0)
+    n_params_all = n_params
+    if args.shard and world > 1:
+        t_n = torch.tensor([n_params], dtype=torch.int64, device=dev)
+        dist.all_reduce(t_n)
+        n_params_all = int(t_n.item())
     ckpt = inputs == "ckpt_bf16"
     out = [torch.empty_like(t) for t in th0]
+    iso.force_two_pass(args.two_pass)
     cfg = iso.merge_cfg(op, density, scope)
     mn, full = iso.iso_workspace_size(th0, K, cfg)
     free = torch.cuda.mem_get_info(dev)[0]
@@ -234,11 +264,9 @@ def run_mine(args):
     launches = (iso.launch_count() - l0) // max(1, args.steps)
     ms = e0.elapsed_time(e1) / args.steps
     ck = clocks.stop() if clocks else None
-    if world > 1:
-        t = torch.tensor([ms], device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        ms = float(t.item())
-    value = world * n_params / (ms * 1e-3) / 1e9
+    ms = reduce_step_ms(ms, dev)
+    n_job = n_params_all if args.shard else world * n_params
+    value = job_throughput(n_job, ms)
 
     # per-kernel device time through the library's event brackets
     iso.profile_reset()
@@ -249,7 +277,7 @@ def run_mine(args):
     torch.cuda.synchronize()
     prof = iso.profile_read()
     iso.profile_enable(False)
-    algo = algorithmic_bytes(shapes, K, inputs, op, scope)
+    algo = algorithmic_bytes(shapes, K, inputs, op, scope, args.two_pass)
     peak, peak_src = read_peaks()
     kernels = {k: {"launches": n // prof_steps, "ms_per_step": tot / prof_steps} for k, (n, tot) in prof.items()}
     dom = max(algo, key=lambda k: prof.get(k, (0, 0.0))[1])
@@ -282,8 +310,8 @@ def run_mine(args):
                       workspace=ws, ws_bytes=ws_bytes)
         f1.record(stream)
         torch.cuda.synchronize()
-        ms_e2e = f0.elapsed_time(f1) / n_e2e
-        e2e = {"value": round(world * n_params / (ms_e2e * 1e-3) / 1e9, 3), "unit": UNIT,
+        ms_e2e = reduce_step_ms(f0.elapsed_time(f1) / n_e2e, dev)
+        e2e = {"value": round(job_throughput(n_job, ms_e2e), 3), "unit": UNIT,
                "ms_per_step": round(ms_e2e, 3), "h2d_bytes_per_step": stage.h2d_bytes,
                "d2h_bytes_per_step": stage.d2h_bytes}
 
@@ -295,13 +323,15 @@ def run_mine(args):
         line = {
             "metric": METRIC, "value": round(value, 3), "unit": UNIT, "n_gpus": world,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms, 4),
-            "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+            "higher_is_better": True, "scaling": "strong" if args.shard else "weak", "vs_baseline": None,
             "dtype": "bf16" if ckpt else "f32", "data": "synthetic (seeded, Qwen-shaped; no checkpoints)",
             "config": {"workload": name if not small else f"{name} (layers={args.layers}, widths/{args.scale})",
                        "description": desc, "params": n_params, "tensors": len(shapes),
                        "experts": K, "op": op, "density": density, "scope": scope,
+                       "path": "fused single pass" if fused_pass(K, inputs, op, scope, args.two_pass)
+                       else "separate passes",
                        "l2": "inputs larger than L2 (129 MB); no flush needed",
-                       "parallelism": f"replica x{world}"},
+                       "parallelism": (f"tensor shards x{world}" if args.shard else f"replica x{world}")},
             "hbm_gbs_step": round(step_gbs, 1),
             "hbm_pct_of_8tbs_step": round(100 * step_gbs / NOMINAL_HBM_GBS, 1),
             "roofline": {"bound": "hbm", "kernel": dom, "achieved": round(achieved, 1), "peak": peak,
@@ -424,6 +454,12 @@ def main():
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", choices=["mine", "reference"], default="mine")
     ap.add_argument("--workload", choices=sorted(WORKLOADS), default="qwen1.5b_update")
+    ap.add_argument("--two-pass", action="store_true",
+                    help="run the K = 1 update as its two-pass form (count, then apply) "
+                         "instead of the fused single pass")
+    ap.add_argument("--shard", action="store_true",
+                    help="N > 1: split one parameter set's tensors over the ranks (strong scaling) "
+                         "instead of a replica per rank (weak scaling)")
     ap.add_argument("--density", type=float, default=None,
                     help="TopKMask density (default: the workload's own)")
     ap.add_argument("--no-e2e", action="store_true")

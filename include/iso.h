@@ -123,7 +123,11 @@ typedef struct {
 typedef struct {
     uint32_t thresh_key;      /* binary32 bits of the k-th largest |tau|; 0xFFFFFFFF when the
                                  unit selects nothing (k == 0) or is not trimmed */
-    uint32_t flags;           /* bit 0: resolved by the full-data fallback; diagnostics only */
+    uint32_t flags;           /* diagnostics only.  bit 0: resolved by the full-data fallback;
+                                 bit 1: fused K = 1 pass took the sampled run of ties as the
+                                 threshold; bit 2: fused pass re-applied the unit in full;
+                                 bit 3: band keys overflowed their segment; bit 4: fused band
+                                 records overflowed */
     int64_t  k;               /* entries selected; -1 for a unit that is not trimmed */
     int64_t  count_above;     /* entries with |tau| above the threshold */
     int64_t  ties_at_thresh;  /* entries with |tau| equal to the threshold */
@@ -222,6 +226,13 @@ const char* iso_error_string(int32_t status);
 /* Diagnostics: number of kernels this process has launched through the
  * library (all streams, all devices). */
 uint64_t iso_launch_count(void);
+
+/* Diagnostics: the K = 1 update of a bf16 base by a bf16 update under
+ * per-tensor TopKMask normally runs as one fused pass over the inputs
+ * (speculative outputs from the sampled threshold, then an exact correction);
+ * on = 1 makes later calls take the two-pass form instead (a counting pass,
+ * then the apply pass).  Both give the same result.  Process-wide host state. */
+int32_t iso_force_two_pass(int32_t on);
 
 /* Diagnostics: when enabled, each launch is bracketed by CUDA events on its
  * stream.  iso_profile_read waits for the recorded events and returns, for

@@ -248,6 +248,11 @@ def launch_count() -> int:
     return int(lib().iso_launch_count())
 
 
+def force_two_pass(on=True):
+    """Diagnostics: run later K = 1 updates in the two-pass form."""
+    check(lib().iso_force_two_pass(int(bool(on))), "iso_force_two_pass")
+
+
 def profile_enable(on=True):
     check(lib().iso_profile_enable(int(bool(on))), "iso_profile_enable")
 

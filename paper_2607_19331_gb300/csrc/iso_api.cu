@@ -19,10 +19,7 @@ namespace iso {
 namespace {
 
 constexpr int COUNT_GRID_PER_SM = COUNT_BLOCKS_PER_SM;
-#ifndef ISO_FUSED_BLOCKS_PER_SM
-#define ISO_FUSED_BLOCKS_PER_SM 2
-#endif
-constexpr int FUSED_GRID_PER_SM = ISO_FUSED_BLOCKS_PER_SM;
+constexpr int FUSED_GRID_PER_SM = FUSED_BLOCKS_PER_SM;
 
 // ---------------------------------------------------------------------------
 // profiling and launch accounting
@@ -229,14 +226,23 @@ unsigned long long brec_cap_of(long long n, double rho) {
     return (unsigned long long)std::min(cap, (double)n);
 }
 
-// the K = 1 update can take the fused single pass (bf16 base and update,
-// per-tensor units); built in with ISO_ENABLE_FUSED=1
-#ifndef ISO_ENABLE_FUSED
-#define ISO_ENABLE_FUSED 0
-#endif
+std::atomic<int> g_two_pass{0};
+// The K = 1 update takes the fused single pass (bf16 base and update,
+// per-tensor units) unless iso_force_two_pass selected the two-pass form.
+// Its corrections re-read theta_0 after the outputs are written, so an output
+// that aliases theta_0 (an in-place update) takes the two-pass form.
 bool fused_path(const Call& c) {
-    return ISO_ENABLE_FUSED && c.K == 1 && !c.mask_only && c.op != ISO_OP_TA &&
-           c.topk.scope == ISO_SCOPE_TENSOR && c.xdt == ISO_BF16 && c.bdt == ISO_BF16 && c.trims;
+    if (g_two_pass.load(std::memory_order_relaxed) || c.K != 1 || c.mask_only || c.op == ISO_OP_TA ||
+        c.topk.scope != ISO_SCOPE_TENSOR || c.xdt != ISO_BF16 || c.bdt != ISO_BF16 || !c.trims)
+        return false;
+    // (workspace sizing passes no outputs: it sizes for the fused pass)
+    for (int t = 0; c.out && t < c.n; ++t) {
+        const char* b = static_cast<const char*>(c.base[t].data);
+        const char* o = static_cast<const char*>(c.out[t].data);
+        const long long bytes = numel_of(c.base[t]) * 2;
+        if (b && o && b < o + bytes && o < b + bytes) return false;
+    }
+    return true;
 }
 
 size_t al256(size_t v) { return (v + 255) & ~(size_t)255; }
@@ -458,6 +464,7 @@ int run_group(const Call& c, int t0, int t1, char* ws, cudaStream_t s, const iso
     P.bdt = c.bdt;
     P.ckpt = c.ckpt ? 1 : 0;
     P.op = c.mask_only ? ISO_OP_TIES : c.op;
+    P.fused = fused ? 1 : 0;
     P.block_rows = c.topk.block_rows;
     P.block_cols = c.topk.block_cols;
     P.lambda = c.lambda;
@@ -498,8 +505,13 @@ int run_group(const Call& c, int t0, int t1, char* ws, cudaStream_t s, const iso
             ISO_TRY(smem_optin(k_sample<XT, BT, CK>, smem));
             ISO_TRY(launch(KD_SAMPLE, s, [&] { k_sample<XT, BT, CK><<<KU, SAMPLE_TPB, smem, s>>>(P); }));
             if (fused) {
-                if (CK) ISO_TRY(launch(KD_COUNT, s, [&] { k_count_apply<true><<<sms * FUSED_GRID_PER_SM, TPB, 0, s>>>(P); }));
-                else ISO_TRY(launch(KD_COUNT, s, [&] { k_count_apply<false><<<sms * FUSED_GRID_PER_SM, TPB, 0, s>>>(P); }));
+                if (CK) {
+                    ISO_TRY(smem_optin(k_count_apply<true>, FUSED_SMEM));
+                    ISO_TRY(launch(KD_COUNT, s, [&] { k_count_apply<true><<<sms * FUSED_GRID_PER_SM, TPB, FUSED_SMEM, s>>>(P); }));
+                } else {
+                    ISO_TRY(smem_optin(k_count_apply<false>, FUSED_SMEM));
+                    ISO_TRY(launch(KD_COUNT, s, [&] { k_count_apply<false><<<sms * FUSED_GRID_PER_SM, TPB, FUSED_SMEM, s>>>(P); }));
+                }
             } else {
                 ISO_TRY(launch(KD_COUNT, s, [&] { k_count<XT, BT, CK><<<sms * COUNT_GRID_PER_SM, TPB, 0, s>>>(P); }));
             }
@@ -540,12 +552,13 @@ int run_group(const Call& c, int t0, int t1, char* ws, cudaStream_t s, const iso
         // exact coefficients and repair flags, then the kept band entries, then
         // the full exact apply of any flagged tensor
         ISO_TRY(launch(KD_SOLVE, s, [&] { k_solve<<<(T + 127) / 128, 128, 0, s>>>(P, gram_mode); }));
+        ISO_TRY(launch(KD_REPAIR, s, [&] { k_fix_plan<<<1, 1024, 0, s>>>(P); }));
         if (c.ckpt) {
             ISO_TRY(launch(KD_PATCH, s, [&] { k_patch<true><<<pgrid, TPB, 0, s>>>(P); }));
-            ISO_TRY(launch(KD_REPAIR, s, [&] { k_repair<true><<<pgrid, TPB, 0, s>>>(P); }));
+            ISO_TRY(launch(KD_REPAIR, s, [&] { k_fix<true><<<pgrid, TPB, 0, s>>>(P); }));
         } else {
             ISO_TRY(launch(KD_PATCH, s, [&] { k_patch<false><<<pgrid, TPB, 0, s>>>(P); }));
-            ISO_TRY(launch(KD_REPAIR, s, [&] { k_repair<false><<<pgrid, TPB, 0, s>>>(P); }));
+            ISO_TRY(launch(KD_REPAIR, s, [&] { k_fix<false><<<pgrid, TPB, 0, s>>>(P); }));
         }
         return ISO_OK;
     }
@@ -554,13 +567,15 @@ int run_group(const Call& c, int t0, int t1, char* ws, cudaStream_t s, const iso
         using XT = std::remove_pointer_t<decltype(xt)>;
         using BT = std::remove_pointer_t<decltype(bt)>;
         constexpr bool CK = decltype(ck)::value;
-        const int mgrid = sms * MERGE_BLOCKS_PER_SM;
+
         if (gram_mode != GRAM_NONE) {
             if (need_gram_pass) {
                 auto gram = [&](auto kc) {
                     constexpr int KC = decltype(kc)::value;
                     const int ggrid = sms * gram_blocks_per_sm(KC);
-                    return launch(KD_GRAM, s, [&] { k_gramk<XT, BT, CK, KC><<<ggrid, TPB, 0, s>>>(P); });
+                    const int smem = merge_smem_bytes<XT, BT, KC>();
+                    ISO_TRY(smem_optin(k_gramk<XT, BT, CK, KC>, smem));
+                    return launch(KD_GRAM, s, [&] { k_gramk<XT, BT, CK, KC><<<ggrid, TPB, smem, s>>>(P); });
                 };
                 if (K == 1) ISO_TRY(gram(std::integral_constant<int, 1>{}));
                 else if (K == 2) ISO_TRY(gram(std::integral_constant<int, 2>{}));
@@ -571,7 +586,10 @@ int run_group(const Call& c, int t0, int t1, char* ws, cudaStream_t s, const iso
         }
         auto merge = [&](auto kc) {
             constexpr int KC = decltype(kc)::value;
-            return launch(KD_APPLY, s, [&] { k_merge<XT, BT, CK, KC><<<mgrid, TPB, 0, s>>>(P); });
+            const int smem = merge_smem_bytes<XT, BT, KC>();
+            const int mgrid = sms * merge_blocks_per_sm(KC);
+            ISO_TRY(smem_optin(k_merge<XT, BT, CK, KC>, smem));
+            return launch(KD_APPLY, s, [&] { k_merge<XT, BT, CK, KC><<<mgrid, TPB, smem, s>>>(P); });
         };
         if (K == 1) ISO_TRY(launch(KD_APPLY, s, [&] { k_apply<XT, BT, CK, 1><<<pgrid, TPB, 0, s>>>(P); }));
         else if (K == 2) ISO_TRY(merge(std::integral_constant<int, 2>{}));
@@ -839,6 +857,11 @@ const char* iso_error_string(int32_t status) {
 }
 
 uint64_t iso_launch_count(void) { return g_launches.load(); }
+
+int32_t iso_force_two_pass(int32_t on) {
+    g_two_pass.store(on ? 1 : 0);
+    return ISO_OK;
+}
 
 int32_t iso_profile_enable(int32_t on) {
     std::lock_guard<std::mutex> lk(g_prof_mu);

@@ -246,6 +246,8 @@ __global__ void k_solve(Plan P, int gram_mode) {
         if ((d.flags & TF_TRIM) && U.state == ST_DONE) {
             const float a = active ? (float)c[0] : P.lambda;
             rep = (U.fallback || U.b_overflow || a != k1_spec_coef(P)) ? 1 : 0;
+            if (rep && P.st_units)
+                P.st_units[P.st_unit_base + d.unit].flags |= 4u | (U.b_overflow ? 16u : 0u);
         }
         P.repair[t] = rep;
     }

@@ -7,42 +7,36 @@
 // The two-pass form reads the inputs twice: once to count (TopKMask needs the
 // unit's k-th largest |tau| before any entry can be decided) and once to apply.
 //
-// Here a single pass does both.  With the sampled band [lo, hi] around rank k
-// (k_sample) every entry above hi is kept and every entry below lo dropped
-// whatever the exact threshold turns out to be; only band entries are
-// undecided.  The pass therefore writes every output at once -- entries above
-// hi with the coefficient a_spec the unit will have in every ordinary case,
-// band entries as dropped -- and records each band entry (position and raw
-// values).  Once the exact threshold and cut are known (the select chain) and
-// the coefficient is exact, k_patch rewrites the band entries that are kept.
-// A tensor whose band missed, whose records overflowed, or whose exact
-// coefficient differs from a_spec is flagged and re-applied in full by
-// k_apply, so the result is exact in every case.
+// Here a single pass counts and writes every output under a speculative
+// selection taken from the sample (k_sample), and a small exact pass then
+// corrects what the speculation can have got wrong:
+//
+//   run mode  (the sampled band is one key value t^, a run of exact ties, as
+//             bf16-derived task vectors have): kept_spec = key > t^, or
+//             key == t^ before the sampled cut position c^.  If the counts
+//             confirm t = t^, only ties between c^ and the exact cut can be
+//             wrong, and k_fix re-applies that position range exactly.
+//   band mode (a band [lo, hi] of several key values): kept_spec = key > hi;
+//             every band entry is recorded (position and raw values), and
+//             k_patch writes the band entries that the exact cut keeps.
+//
+// The exact threshold and cut come from the same select chain as the two-pass
+// form (k_decide, k_radix_*, k_tie, k_cut), fed by this pass's counters.  A
+// unit whose speculation failed (threshold outside the band, overflowing
+// records) or whose exact coefficient differs from the speculated one is
+// re-applied in full by k_fix, so the result is exact in every case.
 #include "iso_kernels.cuh"
 
 namespace iso {
 
-__device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
-    __nv_bfloat162 h = __floats2bfloat162_rn(lo, hi);
-    return *reinterpret_cast<uint32_t*>(&h);
-}
-
-#ifndef ISO_FUSED_BLOCKS_PER_SM
-#define ISO_FUSED_BLOCKS_PER_SM 2
-#endif
-constexpr int FUSED_BLOCKS_PER_SM = ISO_FUSED_BLOCKS_PER_SM;
-
 template <bool CK>
 __global__ void __launch_bounds__(TPB, FUSED_BLOCKS_PER_SM) k_count_apply(Plan P) {
-    // per warp: the tile's raw update and base values, and the offsets of its
-    // band entries (lane L's j-th at j*32 + L)
-    __shared__ __align__(16) uint16_t s_x[WPB][TILE];
-    __shared__ __align__(16) uint16_t s_b[WPB][TILE];
-    __shared__ uint16_t s_off[WPB][TILE + 32];
+    // per lane, its band entries other than t^ as (tile offset, theta_0 bits
+    // << 16 | x bits), lane L's j-th at j*32 + L; FUSED_SMEM bytes of dynamic
+    // shared memory
+    extern __shared__ uint2 s_stage[];
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-    uint16_t* sx = s_x[warp];
-    uint16_t* sbs = s_b[warp];
-    uint16_t* sol = s_off[warp] + lane;
+    uint2* const sbl = s_stage + warp * (TILE + 32) + lane;
     const uint32_t W = gridDim.x * WPB;
     const uint32_t wid = blockIdx.x * WPB + warp;
     const uint32_t items = (uint32_t)P.n_tiles;
@@ -53,32 +47,77 @@ __global__ void __launch_bounds__(TPB, FUSED_BLOCKS_PER_SM) k_count_apply(Plan P
     const unsigned FULL = 0xFFFFFFFFu;
     const float a_spec = k1_spec_coef(P);
 
-    // per-unit accumulators and the two segments (interior keys, band records)
+    // the current tensor and its unit
+    int t = tensor_of_tile(P.tens, P.n_tensors, beg);
+    uint32_t t_end = 0;                       // first tile after tensor t
+    bool sel = false;                         // the tensor's unit is decided here
+    bool keep_all = false;                    // otherwise: every entry kept (untrimmed) or none (k == 0)
+    float a = 0.0f;                           // coefficient of the kept entries
+    uint32_t lo = 0, hi = 0, th = 0, chat = 0;
     Unit* au = nullptr;
-    uint32_t a_gt = 0, a_int = 0;
-    double d_gg = 0.0;
+    uint32_t a_gt = 0, a_eq = 0, a_int = 0, a_abv = 0;
+    float s_gg = 0.0f, e_gg = 0.0f, s_gb = 0.0f, e_gb = 0.0f;
+    bool want_gamma = false;
     uint32_t* cseg = nullptr;
     uint2* bseg = nullptr;
     uint32_t c_pos = 0, c_left = 0, c_cap = 0, b_pos = 0, b_left = 0, b_cap = 0;
     bool c_ovf = false, b_ovf = false;
-    uint32_t lo = 0, hi = 0, span = 0;
-    bool want_gamma = false;
 
     auto flush = [&]() {
         if (!au) return;
-        const double gg = warp_sum(d_gg);
+        const double gg = warp_sum((double)s_gg + (double)e_gg), gb = warp_sum((double)s_gb + (double)e_gb);
         if (lane == 0) {
             if (a_gt) atomicAdd(&au->c_gt, (unsigned long long)a_gt);
+            if (a_eq) atomicAdd(&au->c_eq, (unsigned long long)a_eq);
             if (a_int) atomicAdd(&au->n_int, (unsigned long long)a_int);
-            if (want_gamma && gg != 0.0) atomicAdd(&au->gamma_acc, gg);
+            if (a_abv) atomicAdd(&au->c_abv, (unsigned long long)a_abv);
+            if (want_gamma) {
+                if (gg != 0.0) atomicAdd(&au->gamma_acc, gg);
+                if (gb != 0.0) atomicAdd(&au->gamma_band, gb);
+            }
             if (c_ovf) au->overflow = 1;
             if (b_ovf) au->b_overflow = 1;
         }
-        a_gt = a_int = 0;
-        d_gg = 0.0;
+        a_gt = a_eq = a_int = a_abv = 0;
+        s_gg = e_gg = s_gb = e_gb = 0.0f;
     };
 
-    // reserve n slots of a segment for one tile; returns false on overflow
+    auto enter_tensor = [&](int tt) {
+        flush();
+        au = nullptr;
+        const TensorDesc& d = P.tens[tt];
+        t_end = (uint32_t)(d.tile_base + (d.numel + TILE - 1) / TILE);
+        const bool is1d = (d.flags & TF_1D) != 0;
+        sel = false;
+        if (!(d.flags & TF_TRIM)) {
+            keep_all = true;
+            a = (P.op == ISO_OP_ISO && is1d) ? 1.0f : P.lambda;
+            return;
+        }
+        Unit* U = &P.units[d.unit];
+        if (U->state != ST_BAND || !U->mode_t) {   // k == 0: nothing kept
+            keep_all = false;
+            a = 0.0f;
+            return;
+        }
+        sel = true;
+        au = U;
+        a = a_spec;
+        lo = U->lo;
+        hi = U->hi;
+        th = U->that;
+        const long long ch = U->chat;
+        chat = (uint32_t)(ch < 0 ? 0 : ch);
+        want_gamma = U->want_gamma != 0;
+        c_cap = (uint32_t)U->cand_cap;
+        cseg = P.cand + U->cand_off;
+        b_cap = (uint32_t)U->brec_cap;
+        bseg = P.brec + U->brec_off;
+        c_left = b_left = 0;
+        c_ovf = b_ovf = false;
+    };
+
+    // reserve slots of a segment for one tile; false on overflow
     auto reserve = [&](unsigned long long* alloc, uint32_t need, uint32_t cap, uint32_t left_tiles,
                        uint32_t& pos, uint32_t& left) -> bool {
         unsigned long long start = 0;
@@ -96,146 +135,194 @@ __global__ void __launch_bounds__(TPB, FUSED_BLOCKS_PER_SM) k_count_apply(Plan P
         return true;
     };
 
-    uint32_t run_end = beg, it0 = beg, g0 = 0, n = 0, tile_base = 0;
-    const void* xp = nullptr;
-    const void* bp = nullptr;
-    void* op = nullptr;
-    bool fuse = false, kept_all = false;
-    float a_fix = 0.0f;
-    uint32_t it = beg;
-    while (it < end) {
-        if (it >= run_end) {
-            Cursor c;
-            cursor_at(P, it, c);
-            run_end = (uint32_t)c.run_end;
-            const TensorDesc& d = P.tens[c.t];
-            n = (uint32_t)d.numel;
-            tile_base = (uint32_t)d.tile_base;
-            xp = P.xptr[c.t];
-            bp = d.base;
-            op = d.out;
-            it0 = it;
-            g0 = (uint32_t)c.g;
-            Unit* U = &P.units[d.unit];
-            fuse = (d.flags & TF_TRIM) && U->state == ST_BAND;
-            // a tensor whose selection is already final: untrimmed (all kept) or k = 0
-            kept_all = !(d.flags & TF_TRIM);
-            a_fix = (P.op == ISO_OP_ISO && (d.flags & TF_1D)) ? 1.0f : P.lambda;
-            if (fuse && U != au) {
-                flush();
-                au = U;
-                lo = U->lo;
-                hi = U->hi;
-                span = hi - lo;
-                want_gamma = U->want_gamma != 0;
-                c_cap = (uint32_t)U->cand_cap;
-                cseg = P.cand + U->cand_off;
-                b_cap = (uint32_t)U->brec_cap;
-                bseg = P.brec + U->brec_off;
-                c_left = b_left = 0;
-                c_ovf = b_ovf = false;
-            }
-        }
-        const uint32_t g = g0 + (it - it0);
-        const uint32_t e0 = (g - tile_base) * TILE;
-        RawTile<__nv_bfloat16, __nv_bfloat16, true> rt;
-        rt.load(xp, bp, e0, n, lane);
+    RawTile<__nv_bfloat16, __nv_bfloat16, true> rt;   // x in rt.x, theta_0 in rt.b
 
-        if (!fuse) {
-            // final selection: plain map
+    // first tile's loads
+    enter_tensor(t);
+    {
+        const TensorDesc& d = P.tens[t];
+        const uint32_t e0 = (uint32_t)(beg - d.tile_base) * TILE;
+#pragma unroll
+        for (int v = 0; v < WVEC; ++v) rt.load_step(v, P.xptr[t], d.base, e0, (uint32_t)d.numel - e0, lane);
+    }
+    int nt = t;                               // tensor of the next tile
+    uint32_t nt_end = t_end;
+    for (uint32_t g = beg; g < end; ++g) {
+        if (g >= t_end) {
+            while (g >= (uint32_t)(P.tens[t].tile_base + (P.tens[t].numel + TILE - 1) / TILE)) ++t;
+            enter_tensor(t);
+        }
+        const TensorDesc& d = P.tens[t];
+        void* op = d.out;
+        const uint32_t n = (uint32_t)d.numel;
+        const uint32_t e0 = (uint32_t)(g - d.tile_base) * TILE;
+        const uint32_t rem = n - e0;
+        // the next tile: its loads replace each step as it is consumed
+        const bool more = g + 1 < end;
+        const void* nxp = nullptr;
+        const void* nbp = nullptr;
+        uint32_t ne0 = 0, nrem = 0;
+        if (more) {
+            while (g + 1 >= nt_end) {
+                ++nt;
+                nt_end = (uint32_t)(P.tens[nt].tile_base + (P.tens[nt].numel + TILE - 1) / TILE);
+            }
+            const TensorDesc& nd = P.tens[nt];
+            nxp = P.xptr[nt];
+            nbp = nd.base;
+            ne0 = (uint32_t)(g + 1 - nd.tile_base) * TILE;
+            nrem = (uint32_t)nd.numel - ne0;
+        }
+
+        if (!sel) {
 #pragma unroll
             for (int v = 0; v < WVEC; ++v) {
-                const uint32_t e = e0 + v * (32 * VEC) + lane * VEC;
-                if (e >= n) continue;
                 float th0[VEC], tau[VEC], o[VEC];
                 raw_to_f32<__nv_bfloat16>(rt.b[v], th0);
                 if (CK) rt.tau(v, tau); else raw_to_f32<__nv_bfloat16>(rt.x[v], tau);
+                if (more) rt.load_step(v, nxp, nbp, ne0, nrem, lane);
+                const uint32_t o8 = (uint32_t)(v * (32 * VEC) + lane * VEC);
+                if (o8 >= rem) continue;
 #pragma unroll
-                for (int j = 0; j < VEC; ++j) o[j] = kept_all ? out_of(th0[j], tau[j], a_fix) : th0[j];
-                store8(op, e, n, o, true);
+                for (int j = 0; j < VEC; ++j) o[j] = keep_all ? out_of(th0[j], tau[j], a) : th0[j];
+                store8(op, (long long)e0 + o8, n, o, true);
             }
-            ++it;
             continue;
         }
 
-        // pass 1: every entry -- counts, band offsets, speculative outputs
-        // (a ragged last tile reads zeros past the end: key 0 is never above
-        // hi, and a band holding 0 is corrected below)
-        uint32_t n_gt = 0, nb = 0, kmax = 0;
-        float f_gg = 0.0f;
+        // speculative selection: kept <=> key > t^, or key == t^ at a
+        // position before chat.  In a whole tile on one side of chat that is
+        // one comparison, key > T; a tile holding chat or the tensor's end
+        // takes the per-entry form.  Band keys other than t^ are rare: their
+        // lanes stage them from the step's raw words, still in registers.
+        const uint32_t tile_hi = e0 + min(rem, (uint32_t)TILE);
+        const bool fast = rem >= TILE && (tile_hi <= chat || e0 >= chat);
+        const uint32_t T = (tile_hi <= chat) ? th - 1u : th;     // th >= 1 whenever ties are kept here
+        uint32_t n_gt = 0, n_eq = 0;
+        float f_gg = 0.0f;                     // tau^2 above hi (also the non-finite detector)
+        uint2* sp = sbl;
 #pragma unroll
         for (int v = 0; v < WVEC; ++v) {
-            const uint32_t e = e0 + v * (32 * VEC) + lane * VEC;
-            *reinterpret_cast<uint4*>(sx + v * (32 * VEC) + lane * VEC) = rt.x[v][0];
-            *reinterpret_cast<uint4*>(sbs + v * (32 * VEC) + lane * VEC) = rt.b[v][0];
             float th0[VEC], tau[VEC], o[VEC];
             raw_to_f32<__nv_bfloat16>(rt.b[v], th0);
             if (CK) rt.tau(v, tau); else raw_to_f32<__nv_bfloat16>(rt.x[v], tau);
+            const uint4 xw = rt.x[v][0], bw = rt.b[v][0];
+            if (more) rt.load_step(v, nxp, nbp, ne0, nrem, lane);
+            const uint32_t o8 = (uint32_t)(v * (32 * VEC) + lane * VEC);
+            uint32_t bm = 0;                   // band entries of this step
+            if (fast) {
 #pragma unroll
-            for (int j = 0; j < VEC; ++j) {
-                const uint32_t kk = key_of(tau[j]);
-                const bool gt = kk > hi;
-                kmax = max(kmax, kk);
-                n_gt += gt;
-                if (want_gamma && gt) f_gg = __fmaf_rn(tau[j], tau[j], f_gg);
-                sol[nb * 32] = (uint16_t)(v * (32 * VEC) + lane * VEC + j);
-                nb += (kk - lo <= span);
-                o[j] = gt ? out_of(th0[j], tau[j], a_spec) : th0[j];
-            }
-            if (e < n) store8(op, e, n, o, true);
-        }
-        if (e0 + TILE > n && lo == 0) {
-            // drop the zero-filled entries past the end from the band
-            uint32_t keep = 0;
-            for (uint32_t q = 0; q < nb; ++q) {
-                const uint32_t off = sol[q * 32];
-                if (e0 + off < n) sol[(keep++) * 32] = (uint16_t)off;
-            }
-            nb = keep;
-        }
-        if (__any_sync(FULL, kmax >= KEY_INF) && lane == 0) set_status(P.hdr, ISO_ERR_NONFINITE);
-        if (want_gamma) d_gg += (double)f_gg;
-        __syncwarp();
-
-        // pass 2: the band entries go to the unit's candidate segment (keys)
-        // and to its band records (position and raw values)
-        uint32_t nb_tot;
-        const uint32_t nb_off = warp_excl_scan(nb, &nb_tot);
-        const uint32_t left_tiles = min(run_end, end) - it;
-        if (nb_tot && !c_ovf && nb_tot > c_left)
-            c_ovf = !reserve(&au->n_alloc, nb_tot, c_cap, left_tiles, c_pos, c_left);
-        if (nb_tot && !b_ovf && nb_tot > b_left)
-            b_ovf = !reserve(&au->b_alloc, nb_tot, b_cap, left_tiles, b_pos, b_left);
-        const bool c_store = nb_tot && !c_ovf;
-        const bool b_store = nb_tot && !b_ovf;
-        if (c_store || b_store) {
-            uint32_t wi = c_pos + nb_off, wb = b_pos + nb_off;
-            for (uint32_t q = 0; q < nb; ++q) {
-                const uint32_t off = sol[q * 32];
-                const uint32_t xr = sx[off], br = sbs[off];
-                if (b_store) bseg[wb++] = make_uint2(e0 + off, (br << 16) | xr);
-                if (c_store) {
-                    const float xv = __uint_as_float(xr << 16), bv = __uint_as_float(br << 16);
-                    cseg[wi++] = key_of(CK ? __fsub_rn(xv, bv) : xv);
+                for (int j = 0; j < VEC; ++j) {
+                    const uint32_t kk = key_of(tau[j]);
+                    const bool gt = kk > hi, eq = kk == th;
+                    const bool kept = (int)kk > (int)T;
+                    n_gt += gt;
+                    n_eq += eq;
+                    if (gt) f_gg = __fmaf_rn(tau[j], tau[j], f_gg);
+                    bm |= (uint32_t)(kk >= lo && !gt && !eq) << j;
+                    const float upd = __fmul_rn(a, tau[j]);
+                    o[j] = (kept && upd != 0.0f) ? __fadd_rn(th0[j], upd) : th0[j];
+                }
+            } else {
+                if (o8 >= rem) continue;
+#pragma unroll
+                for (int j = 0; j < VEC; ++j) {
+                    const bool valid = o8 + j < rem;
+                    const uint32_t kk = key_of(tau[j]);
+                    const bool gt = valid && kk > hi, eq = valid && kk == th;
+                    const bool kept = (kk > th) || (eq && e0 + o8 + j < chat);
+                    n_gt += gt;
+                    n_eq += eq;
+                    if (gt) f_gg = __fmaf_rn(tau[j], tau[j], f_gg);
+                    bm |= (uint32_t)(valid && kk >= lo && !gt && !eq) << j;
+                    const float upd = __fmul_rn(a, tau[j]);
+                    o[j] = (kept && upd != 0.0f) ? __fadd_rn(th0[j], upd) : th0[j];
                 }
             }
+            store8(op, (long long)e0 + o8, n, o, true);
+            if (bm) {
+                const uint32_t xr[4] = {xw.x, xw.y, xw.z, xw.w}, br[4] = {bw.x, bw.y, bw.z, bw.w};
+                do {
+                    const int j = __ffs(bm) - 1;
+                    bm &= bm - 1;
+                    const uint32_t sh = 16u * (uint32_t)(j & 1);
+                    const uint32_t rx = (xr[j >> 1] >> sh) & 0xFFFFu, rb = (br[j >> 1] >> sh) & 0xFFFFu;
+                    *sp = make_uint2(o8 + j, (rb << 16) | rx);
+                    sp += 32;
+                } while (bm);
+            }
         }
+        if (__any_sync(FULL, !(fabsf(f_gg) <= 3.402823466e38f))) {
+            // a non-finite (or overflowing) sum: read the tile's keys again
+            uint32_t kmax = 0;
+            for (int v = 0; v < WVEC; ++v) {
+                const uint32_t o8 = (uint32_t)(v * (32 * VEC) + lane * VEC);
+                if (o8 >= rem) break;
+                float tau[VEC];
+                TauSrc<__nv_bfloat16, __nv_bfloat16, CK>::load8(P.xptr[t], d.base, (long long)e0 + o8, (long long)n, tau);
+#pragma unroll
+                for (int j = 0; j < VEC; ++j)
+                    if (o8 + j < rem) kmax = max(kmax, key_of(tau[j]));
+            }
+            if (__any_sync(FULL, kmax >= KEY_INF) && lane == 0) set_status(P.hdr, ISO_ERR_NONFINITE);
+        }
+        if (want_gamma) two_sum_add(s_gg, e_gg, f_gg);
         const uint32_t t_gt = __reduce_add_sync(FULL, n_gt);
+        const uint32_t t_eq = __reduce_add_sync(FULL, n_eq);
+        a_gt += t_gt;
+        a_eq += t_eq;
+
+        // pass 2: the staged band entries (keys other than t^, a fraction of a
+        // per cent) go to the unit's candidate segment (keys) and its band
+        // records (position and raw values), read again from L2
+        const uint32_t nb = (uint32_t)(sp - sbl) >> 5;
+        uint32_t nb_tot;
+        const uint32_t nb_off = warp_excl_scan(nb, &nb_tot);
+        const uint32_t left_tiles = min(t_end, end) - g;   // this warp's tiles left in the unit
+        if (nb_tot && !c_ovf && nb_tot > c_left) c_ovf = !reserve(&au->n_alloc, nb_tot, c_cap, left_tiles, c_pos, c_left);
+        if (nb_tot && !b_ovf && nb_tot > b_left) b_ovf = !reserve(&au->b_alloc, nb_tot, b_cap, left_tiles, b_pos, b_left);
+        const bool c_store = nb_tot && !c_ovf;
+        const bool b_store = nb_tot && !b_ovf;
+        uint32_t n_abv = 0, kbad = 0;
+        float f_band = 0.0f;                   // tau^2 over the candidates above t^
+        if (nb_tot) {
+            uint32_t wi = c_pos + nb_off, wb = b_pos + nb_off;
+            for (uint32_t q = 0; q < nb; ++q) {
+                const uint2 st = sbl[q * 32];
+                const uint32_t pos = e0 + st.x;
+                const float xv = __uint_as_float(st.y << 16), bv = __uint_as_float(st.y & 0xFFFF0000u);
+                const float tv = CK ? __fsub_rn(xv, bv) : xv;
+                const uint32_t kk = key_of(tv);
+                if (b_store) bseg[wb++] = make_uint2(pos, st.y);
+                if (c_store) cseg[wi++] = kk;
+                const bool ab = kk > th;
+                n_abv += ab;
+                kbad |= (kk >= KEY_INF);
+                if (want_gamma && ab) f_band = __fmaf_rn(tv, tv, f_band);
+            }
+        }
+        if (__any_sync(FULL, kbad) && lane == 0) set_status(P.hdr, ISO_ERR_NONFINITE);
+        if (want_gamma) two_sum_add(s_gb, e_gb, f_band);
+        const uint32_t t_abv = __reduce_add_sync(FULL, n_abv);
         if (lane == 0) {
             P.tcand[g] = make_uint2(c_store ? c_pos : 0u, c_store ? nb_tot : 0u);
             P.tband[g] = make_uint2(b_store ? b_pos : 0u, b_store ? nb_tot : 0u);
+            P.teq_lo[g] = 0;
+            P.teq_hi[g] = t_eq;
         }
-        const uint32_t in_tot = nb_tot;
-        if (c_store) { c_pos += in_tot; c_left -= in_tot; }
+        if (c_store) { c_pos += nb_tot; c_left -= nb_tot; }
         if (b_store) { b_pos += nb_tot; b_left -= nb_tot; }
-        a_gt += t_gt; a_int += in_tot;
+        a_int += nb_tot;
+        a_abv += t_abv;
         __syncwarp();
-        ++it;
     }
     flush();
 }
 
-// Rewrites the kept band entries of every fused tensor that needs no repair.
+// The recorded band entries (keys other than t^): the fused pass kept those
+// above t^; the exact selection decides each again, and an entry whose
+// decision changed is rewritten.  Units re-applied by k_fix in full are
+// skipped.
 template <bool CK>
 __global__ void __launch_bounds__(TPB) k_patch(Plan P) {
     const int lane = threadIdx.x & 31;
@@ -246,28 +333,26 @@ __global__ void __launch_bounds__(TPB) k_patch(Plan P) {
     const uint32_t beg = wid * per;
     const uint32_t end = min(items, beg + per);
     uint32_t it = beg, run_end = beg;
-    const Unit* U = nullptr;
     const uint2* bseg = nullptr;
     __nv_bfloat16* op = nullptr;
-    bool active = false;
     float a = 0.0f;
-    uint32_t tk = 0;
+    uint32_t th = 0;
     unsigned long long thr = 0;
     while (it < end) {
         if (it >= run_end) {
             const int t = tensor_of_tile(P.tens, P.n_tensors, it);
             const TensorDesc& d = P.tens[t];
             run_end = (uint32_t)(d.tile_base + (d.numel + TILE - 1) / TILE);
-            U = &P.units[d.unit];
-            active = (d.flags & TF_TRIM) && U->state == ST_DONE && !P.repair[t];
+            const Unit* U = &P.units[d.unit];
+            const bool active = (d.flags & TF_TRIM) && U->state == ST_DONE && U->mode_t && !P.repair[t];
             if (!active) { it = run_end; continue; }
             bseg = P.brec + U->brec_off;
             op = static_cast<__nv_bfloat16*>(d.out);
             a = (P.op == ISO_OP_ISO) ? (float)P.coef[t] : P.lambda;
-            tk = U->t;
+            th = U->that;
             const long long cut = U->cut;
             const uint32_t c32 = (cut >= 0xFFFFFFFFLL) ? 0xFFFFFFFFu : (uint32_t)cut;
-            thr = ((unsigned long long)tk << 32) | (uint32_t)~c32;
+            thr = ((unsigned long long)U->t << 32) | (uint32_t)~c32;
         }
         const uint2 r = P.tband[it];
         for (uint32_t q = lane; q < r.y; q += 32) {
@@ -275,69 +360,128 @@ __global__ void __launch_bounds__(TPB) k_patch(Plan P) {
             const float xv = __uint_as_float(rec.y << 16);
             const float bv = __uint_as_float(rec.y & 0xFFFF0000u);
             const float tau = CK ? __fsub_rn(xv, bv) : xv;
-            const unsigned long long kp = ((unsigned long long)key_of(tau) << 32) | (uint32_t)~rec.x;
-            if (kp > thr) op[rec.x] = __float2bfloat16_rn(out_of(bv, tau, a));
+            const uint32_t kk = key_of(tau);
+            const bool kept = (((unsigned long long)kk << 32) | (uint32_t)~rec.x) > thr;
+            if (kept != (kk > th)) op[rec.x] = __float2bfloat16_rn(kept ? out_of(bv, tau, a) : bv);
         }
         ++it;
     }
 }
 
-// The exact apply for the fused tensors flagged by k_solve (normally none).
-template <bool CK>
-__global__ void __launch_bounds__(TPB) k_repair(Plan P) {
-    const int lane = threadIdx.x & 31;
-    const uint32_t W = gridDim.x * WPB;
-    const uint32_t wid = blockIdx.x * WPB + (threadIdx.x >> 5);
-    const uint32_t items = (uint32_t)P.n_tiles;
-    const uint32_t per = (items + W - 1) / W;
-    const uint32_t beg = wid * per;
-    const uint32_t end = min(items, beg + per);
-    uint32_t it = beg, run_end = beg, n = 0, tile_base = 0;
-    const void* xp = nullptr;
-    const void* bp = nullptr;
-    void* op = nullptr;
-    float a = 0.0f;
-    unsigned long long thr = 0;
-    while (it < end) {
-        if (it >= run_end) {
-            const int t = tensor_of_tile(P.tens, P.n_tensors, it);
+// The exact apply over a position range per tensor: the whole tensor for a
+// unit flagged by k_solve (normally none); otherwise the keys equal to t^
+// between the sampled cut chat and where the exact selection puts it (the
+// exact cut when t == t^, the tensor's end when t < t^, its start when
+// t > t^), the only entries the fused pass can have decided the wrong way
+// besides the recorded band entries.
+// The position range k_fix re-applies for each unit, and the prefix over
+// units of its tile counts, so that k_fix can spread all ranges evenly over
+// the GPU.  One block; the total goes to the header.
+__global__ void __launch_bounds__(1024) k_fix_plan(Plan P) {
+    __shared__ long long s_scan[33];
+    long long base = 0;
+    for (int t0 = 0; t0 < P.n_tensors; t0 += blockDim.x) {
+        const int t = t0 + threadIdx.x;
+        long long tiles = 0;
+        if (t < P.n_tensors) {
             const TensorDesc& d = P.tens[t];
-            run_end = (uint32_t)(d.tile_base + (d.numel + TILE - 1) / TILE);
-            if (!P.repair[t]) { it = run_end; continue; }
-            const Unit& U = P.units[d.unit];
-            n = (uint32_t)d.numel;
-            tile_base = (uint32_t)d.tile_base;
-            xp = P.xptr[t];
-            bp = d.base;
-            op = d.out;
-            a = (P.op == ISO_OP_ISO) ? (float)P.coef[t] : P.lambda;
-            const long long cut = U.cut;
-            const uint32_t c32 = (cut >= 0xFFFFFFFFLL) ? 0xFFFFFFFFu : (uint32_t)cut;
-            thr = ((unsigned long long)U.t << 32) | (uint32_t)~c32;
-        }
-        const uint32_t e0 = (it - tile_base) * TILE;
-        RawTile<__nv_bfloat16, __nv_bfloat16, true> rt;
-        rt.load(xp, bp, e0, n, lane);
-#pragma unroll
-        for (int v = 0; v < WVEC; ++v) {
-            const uint32_t e = e0 + v * (32 * VEC) + lane * VEC;
-            if (e >= n) continue;
-            float th0[VEC], tau[VEC], o[VEC];
-            raw_to_f32<__nv_bfloat16>(rt.b[v], th0);
-            if (CK) rt.tau(v, tau); else raw_to_f32<__nv_bfloat16>(rt.x[v], tau);
-#pragma unroll
-            for (int j = 0; j < VEC; ++j) {
-                const unsigned long long kp = ((unsigned long long)key_of(tau[j]) << 32) | (uint32_t)~(e + j);
-                o[j] = (kp > thr) ? out_of(th0[j], tau[j], a) : th0[j];
+            Unit& U = P.units[d.unit];
+            long long r0 = 0, r1 = 0;
+            if ((d.flags & TF_TRIM) && U.state == ST_DONE && U.mode_t) {
+                if (P.repair[t]) {
+                    r0 = 0;
+                    r1 = d.numel;
+                } else {
+                    const long long c = (U.t < U.that) ? d.numel
+                                      : (U.t > U.that ? 0 : (U.cut > d.numel ? d.numel : U.cut));
+                    r0 = min(c, U.chat);
+                    r1 = max(c, U.chat);
+                }
             }
-            store8(op, e, n, o, true);
+            if (r1 > r0) tiles = (r1 + TILE - 1) / TILE - r0 / TILE;
+            U.fix0 = r0;
+            U.fix1 = r1;
         }
-        ++it;
+        long long tot;
+        const long long off = block_excl_scan(tiles, s_scan, &tot);
+        if (t < P.n_tensors) P.units[P.tens[t].unit].fix_off = base + off;
+        base += tot;
+        __syncthreads();
+    }
+    if (threadIdx.x == 0) P.hdr->fix_tiles = (int32_t)min(base, (long long)0x7FFFFFFF);
+}
+
+// Re-applies the exact selection on each unit's range (k_fix_plan): the whole
+// tensor for a unit flagged by k_solve (normally none); otherwise the keys
+// equal to t^ between the sampled cut chat and where the exact selection
+// puts it (the exact cut when t == t^, the tensor's end when t < t^, its
+// start when t > t^), the only entries the fused pass can have decided the
+// wrong way besides the recorded band entries.  The ranges' tiles are split
+// evenly over the warps.
+template <bool CK>
+__global__ void __launch_bounds__(TPB) k_fix(Plan P) {
+    const int lane = threadIdx.x & 31;
+    const long long total = *(volatile int32_t*)&P.hdr->fix_tiles;
+    const long long W = (long long)gridDim.x * WPB;
+    const long long wid = (long long)blockIdx.x * WPB + (threadIdx.x >> 5);
+    const long long per = (total + W - 1) / W;
+    const long long fb = wid * per, fe = min(total, fb + per);
+    if (fb >= fe) return;
+    // the unit holding flattened tile fb: last tensor with fix_off <= fb and tiles to fix
+    int t = 0;
+    {
+        int lo = 0, hi = P.n_tensors - 1;
+        while (lo < hi) {
+            const int mid = (lo + hi + 1) >> 1;
+            if (P.units[P.tens[mid].unit].fix_off <= fb) lo = mid; else hi = mid - 1;
+        }
+        t = lo;
+    }
+    long long f = fb;
+    while (f < fe) {
+        const TensorDesc& d = P.tens[t];
+        const Unit& U = P.units[d.unit];
+        const long long r0 = U.fix0, r1 = U.fix1;
+        const long long g_lo = r0 / TILE, nt = (r1 > r0) ? (r1 + TILE - 1) / TILE - g_lo : 0;
+        if (f >= U.fix_off + nt) { ++t; continue; }
+        const bool all = P.repair[t] != 0;
+        const uint32_t n = (uint32_t)d.numel;
+        const uint32_t th = U.that;
+        const void* xp = P.xptr[t];
+        const void* bp = d.base;
+        __nv_bfloat16* q = static_cast<__nv_bfloat16*>(d.out);
+        const float a = (P.op == ISO_OP_ISO) ? (float)P.coef[t] : P.lambda;
+        const long long cut = U.cut;
+        const uint32_t c32 = (cut >= 0xFFFFFFFFLL) ? 0xFFFFFFFFu : (uint32_t)cut;
+        const unsigned long long thr = ((unsigned long long)U.t << 32) | (uint32_t)~c32;
+        const long long f_end = min(fe, U.fix_off + nt);
+        for (; f < f_end; ++f) {
+            const uint32_t e0 = (uint32_t)(g_lo + (f - U.fix_off)) * TILE;
+            RawTile<__nv_bfloat16, __nv_bfloat16, true> rt;
+            rt.load(xp, bp, e0, n, lane);
+#pragma unroll
+            for (int v = 0; v < WVEC; ++v) {
+                const uint32_t e = e0 + v * (32 * VEC) + lane * VEC;
+                if (e >= n) continue;
+                float th0[VEC], tau[VEC];
+                raw_to_f32<__nv_bfloat16>(rt.b[v], th0);
+                if (CK) rt.tau(v, tau); else raw_to_f32<__nv_bfloat16>(rt.x[v], tau);
+#pragma unroll
+                for (int j = 0; j < VEC; ++j) {
+                    const long long pos = (long long)e + j;
+                    const uint32_t kk = key_of(tau[j]);
+                    if (pos >= n || pos < r0 || pos >= r1 || !(all || kk == th)) continue;
+                    const unsigned long long kp = ((unsigned long long)kk << 32) | (uint32_t)~(uint32_t)pos;
+                    q[pos] = __float2bfloat16_rn((kp > thr) ? out_of(th0[j], tau[j], a) : th0[j]);
+                }
+            }
+        }
+        ++t;
     }
 }
 
-template __global__ void k_repair<true>(Plan);
-template __global__ void k_repair<false>(Plan);
+template __global__ void k_fix<true>(Plan);
+template __global__ void k_fix<false>(Plan);
 template __global__ void k_count_apply<true>(Plan);
 template __global__ void k_count_apply<false>(Plan);
 template __global__ void k_patch<true>(Plan);

@@ -34,6 +34,7 @@ constexpr int SAMPLE_MAX = 24576;           // sampled keys per unit (96 KB of s
 constexpr int SAMPLE_CHUNK = 256;           // contiguous entries per sample chunk
 constexpr int SAMPLE_TPB = 1024;
 constexpr double SAMPLE_Z = 5.0;            // band half-width in sample standard deviations
+constexpr double RUN_Z = 3.0;               // fused K = 1 pass: margin of a run of ties taken as the threshold
 
 constexpr int RADIX_BITS = 11;
 constexpr int RADIX_BINS = 1 << RADIX_BITS;
@@ -118,6 +119,16 @@ struct Unit {
     long long count_above, ties, need;
     long long cut;                      // kept iff key > t || (key == t && pos < cut)
     double gamma;
+    // fused K = 1 pass: the sample's estimate t^ of the threshold (that) and
+    // of the cut among its ties (chat); the band's other keys are the
+    // candidates, the keys equal to t^ are counted per tile (teq_hi)
+    int32_t mode_t;
+    uint32_t that;
+    long long chat;
+    unsigned long long c_eq;            // keys == t^
+    unsigned long long c_abv;           // candidates above t^
+    long long fix0, fix1;               // positions k_fix re-applies (k_fix_plan)
+    long long fix_off;                  // tiles to fix in the units before this one
 };
 
 // Per (expert, tile) records of the count pass, as separate arrays:
@@ -130,7 +141,7 @@ struct Header {             // first bytes of the workspace
     int32_t status;
     int32_t n_radix;        // units in ST_RADIX after the last pick
     int32_t n_tknown;
-    int32_t pad;
+    int32_t fix_tiles;      // fused K = 1 pass: tiles k_fix re-applies (k_fix_plan)
 };
 
 // Everything a kernel needs to find its tables.
@@ -161,6 +172,7 @@ struct Plan {
     int32_t bdt;            // base dtype
     int32_t ckpt;           // experts are checkpoints (tau = x - base)
     int32_t op;
+    int32_t fused;          // the K = 1 update runs the fused single pass
     int32_t block_rows, block_cols;
     float lambda;
     double density, ridge, c_min, c_max;

@@ -25,16 +25,22 @@ constexpr int BLOCK_TPB = 512;
 template <typename XT, typename BT, bool CK> __global__ void k_block_select(Plan P);
 
 // fused K = 1 pass (bf16 base and update)
+constexpr int FUSED_BLOCKS_PER_SM = 2;
+constexpr int FUSED_SMEM = WPB * (TILE + 32) * 8;   // band staging, dynamic shared memory
 template <bool CK> __global__ void k_count_apply(Plan P);
 template <bool CK> __global__ void k_patch(Plan P);
-template <bool CK> __global__ void k_repair(Plan P);
+__global__ void k_fix_plan(Plan P);
+template <bool CK> __global__ void k_fix(Plan P);
 
 // apply: K = 1 (iso_apply.cu); K >= 2 with a compile-time bound KC >= K on
 // the expert count, and the Gram pass for any K (iso_merge.cu)
 template <typename XT, typename BT, bool CK, int KC> __global__ void k_apply(Plan P);
 template <typename XT, typename BT, bool CK, int KC> __global__ void k_merge(Plan P);
 template <typename XT, typename BT, bool CK, int KC> __global__ void k_gramk(Plan P);
-constexpr int MERGE_BLOCKS_PER_SM = 2;                 // k_merge: resident blocks of TPB threads per SM
+// k_merge: resident blocks of TPB threads per SM
+constexpr int merge_blocks_per_sm(int KC) { return KC >= 8 ? 1 : 2; }
+// k_merge's dynamic shared memory (its per-warp staging ring)
+template <typename XT, typename BT, int KC> int merge_smem_bytes();
 constexpr int gram_blocks_per_sm(int KC) { return KC >= 8 ? 1 : 2; }
 __global__ void k_solve(Plan P, int gram_mode);
 template <typename XT> __global__ void k_mask(Plan P, uint32_t* const* mptr);

@@ -297,118 +297,223 @@ __device__ __forceinline__ long long tensor_tile_end(const Plan& P, int t) {
 
 }  // namespace
 
-// One warp per tile, a contiguous tile range per warp.  Each lane takes one
-// 16-byte vector of every expert per step (4 fp32 or 8 bf16 entries); up to
-// four experts, the next step's loads are issued before the current step is
-// merged.
-template <typename XT, typename BT, bool CK, int KC>
-__global__ void __launch_bounds__(TPB, MERGE_BLOCKS_PER_SM) k_merge(Plan P) {
-    constexpr int E = 16 / (int)sizeof(XT);          // entries per lane per step
-    constexpr int SPT = TILE / (32 * E);             // steps per tile (4 or 8)
-    static_assert(SPT % 2 == 0, "steps alternate between two buffers");
-    const int K = P.K;
-    const int lane = threadIdx.x & 31;
-    const WarpRange wr = warp_range(P);
-    if (wr.beg >= wr.end) return;
-    int t = tensor_of_tile(P.tens, P.n_tensors, wr.beg);
-    long long t_end = tensor_tile_end(P, t);
-    __shared__ MergeParams<KC> s_mp[WPB];
-    MergeParams<KC>& mp = s_mp[threadIdx.x >> 5];
-    merge_params<KC>(P, t, K, mp);
-    for (long long g = wr.beg; g < wr.end; ++g) {
-        if (g >= t_end) {
-            while (g >= t_end) t_end = tensor_tile_end(P, ++t);
-            merge_params<KC>(P, t, K, mp);
-        }
-        const TensorDesc& d = P.tens[t];
-        const long long n = d.numel;
-        const long long e0 = (g - d.tile_base) * TILE;
-        const long long e1 = (e0 + TILE < n) ? e0 + TILE : n;
-        // this tile's parameters, in registers
-        const void* xs[KC];
-        float cf[KC];
-        int T[KC];
-#pragma unroll
-        for (int i = 0; i < KC; ++i) { xs[i] = mp.xs[i]; cf[i] = mp.cf[i]; }
-        const bool exact = tile_thresholds<KC>(mp, K, (uint32_t)e0, (uint32_t)e1, T);
-        const int opk = mp.opk;
-        const bool iso1d = mp.iso1d;
-        const void* bp = d.base;
-        void* op = d.out;
+// ---------------------------------------------------------------------------
+// Staged streaming of the K experts and the base.  A warp walks its steps
+// (tile, 32 lanes x E entries) in order; each lane copies its own 16-byte
+// vector of every expert, and its base entries, into a per-warp ring of DEPTH
+// stages in shared memory with cp.async, DEPTH - 1 steps ahead of the step it
+// merges.  The data in flight then lives in shared memory instead of
+// registers, which holds enough of it to keep HBM busy with eight experts.
+// Each lane reads back only what it copied itself, so no barrier is needed.
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ void cp_async16(uint32_t dst, const void* src, uint32_t src_bytes) {
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" :: "r"(dst), "l"(src), "r"(src_bytes) : "memory");
+}
+__device__ __forceinline__ void cp_async8(uint32_t dst, const void* src, uint32_t src_bytes) {
+    asm volatile("cp.async.ca.shared.global [%0], [%1], 8, %2;" :: "r"(dst), "l"(src), "r"(src_bytes) : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+template <int N>
+__device__ __forceinline__ void cp_async_wait() { asm volatile("cp.async.wait_group %0;" :: "n"(N) : "memory"); }
 
-        Words<XT, E> xa[KC], xb[KC];
-        Words<BT, E> ba, bb;
-        auto load = [&](int st, Words<XT, E> (&x)[KC], Words<BT, E>& b) {
-            const long long e = e0 + (long long)st * (32 * E) + lane * E;
-            if (e < n) {
-                load_words<BT, E>(bp, e, n, b);
+__device__ __forceinline__ uint32_t clamp_bytes(long long avail, uint32_t cap) {
+    return avail <= 0 ? 0u : (avail >= (long long)cap ? cap : (uint32_t)avail);
+}
+
+template <typename XT, typename BT, int KC>
+struct StageGeom {
+    static constexpr int E = 16 / (int)sizeof(XT);          // entries per lane per step
+    static constexpr int SPT = TILE / (32 * E);              // steps per tile
+    static constexpr int BB = E * (int)sizeof(BT);           // base bytes per lane per step (8, 16, 32)
+    static constexpr int BYTES = KC * 512 + 32 * BB;         // one stage of one warp
+    // up to four experts: about 108 KB per block, two blocks per SM; eight
+    // experts: one block per SM (its registers hold the eight vectors of a
+    // step without spilling) with about 216 KB, a deeper ring
+    static constexpr int BUDGET = merge_blocks_per_sm(KC) == 1 ? 221184 : 110592;
+    static constexpr int DMAX = merge_blocks_per_sm(KC) == 1 ? 6 : 4;
+    static constexpr int D0 = BUDGET / (WPB * BYTES);
+    static constexpr int DEPTH = D0 < 2 ? 2 : (D0 > DMAX ? DMAX : D0);
+    static constexpr int SMEM = WPB * DEPTH * BYTES;
+};
+
+// the tile a step belongs to and where its data comes from (issue side)
+template <int KC>
+struct IssueCursor {
+    long long g = -1;        // tile of the cached tensor data
+    int t = 0;
+    long long t_end = 0, e0 = 0, n = 0;
+    const void* xs[KC];
+    const void* bp = nullptr;
+};
+
+// copy step (g, s) of lane `lane` into stage `st` (shared-space address)
+template <typename XT, typename BT, int KC>
+__device__ __forceinline__ void issue_step(const Plan& P, int K, IssueCursor<KC>& ic, long long g, int s,
+                                           uint32_t st, int lane) {
+    using G = StageGeom<XT, BT, KC>;
+    if (g != ic.g) {
+        if (ic.g < 0 || g >= ic.t_end) {
+            if (ic.g < 0) ic.t = tensor_of_tile(P.tens, P.n_tensors, g);
+            while (g >= P.tens[ic.t].tile_base + (P.tens[ic.t].numel + TILE - 1) / TILE) ++ic.t;
+            const TensorDesc& d = P.tens[ic.t];
+            ic.t_end = d.tile_base + (d.numel + TILE - 1) / TILE;
+            ic.n = d.numel;
+            ic.bp = d.base;
 #pragma unroll
-                for (int i = 0; i < KC; ++i)
-                    if (i < K) load_words<XT, E>(xs[i], e, n, x[i]);
-            }
-        };
-        auto merge_step = [&](int st, const Words<XT, E> (&x)[KC], const Words<BT, E>& b) {
-            const long long e = e0 + (long long)st * (32 * E) + lane * E;
-            if (e >= n) return;
-            long long r = 0, c = 0;
-            if (exact && mp.sel == SEL_BLOCK) { r = e / d.cols; c = e - r * d.cols; }
-            float o[E];
-#pragma unroll
-            for (int j = 0; j < E; ++j) {
-                const float th0 = word_f32<BT, E>(b, j);
-                float tau[KC];
-#pragma unroll
-                for (int i = 0; i < KC; ++i) {
-                    tau[i] = (i < K) ? word_f32<XT, E>(x[i], j) : 0.0f;
-                    if (CK) tau[i] = __fsub_rn(tau[i], th0);
-                }
-                const uint32_t bits = exact ? select_bits<KC>(P, d, mp, K, tau, e + j, r, c)
-                                            : fast_bits<KC>(T, K, tau);
-                o[j] = merged_value<KC>(opk, iso1d, P.lambda, K, th0, tau, cf, bits);
-            }
-            store_out<BT, E>(op, e, n, o);
-        };
-        if (KC <= 4) {
-            load(0, xa, ba);
-#pragma unroll 1
-            for (int st = 0; st < SPT; st += 2) {
-                load(st + 1, xb, bb);
-                merge_step(st, xa, ba);
-                if (st + 2 < SPT) load(st + 2, xa, ba);
-                merge_step(st + 1, xb, bb);
-            }
-        } else {
-            // eight experts: one buffer (the registers of a second would spill)
-#pragma unroll 1
-            for (int st = 0; st < SPT; ++st) {
-                load(st, xa, ba);
-                merge_step(st, xa, ba);
-            }
+            for (int i = 0; i < KC; ++i) ic.xs[i] = (i < K) ? P.xptr[i * P.n_tensors + ic.t] : nullptr;
         }
+        ic.g = g;
+        ic.e0 = (g - P.tens[ic.t].tile_base) * TILE;
+    }
+    const long long e = ic.e0 + (long long)s * (32 * G::E) + lane * G::E;
+    const bool in = e < ic.n;
+    const uint32_t xb = clamp_bytes((ic.n - e) * (long long)sizeof(XT), 16);
+#pragma unroll
+    for (int i = 0; i < KC; ++i) {
+        if (i < K) {
+            const char* src = static_cast<const char*>(ic.xs[i]) + (in ? e * (long long)sizeof(XT) : 0);
+            cp_async16(st + i * 512 + lane * 16, src, xb);
+        }
+    }
+    const uint32_t bdst = st + KC * 512 + lane * G::BB;
+    const char* bsrc = static_cast<const char*>(ic.bp) + (in ? e * (long long)sizeof(BT) : 0);
+    const long long bavail = (ic.n - e) * (long long)sizeof(BT);
+    if (G::BB == 8) {
+        cp_async8(bdst, bsrc, clamp_bytes(bavail, 8));
+    } else {
+#pragma unroll
+        for (int q = 0; q < G::BB / 16; ++q)
+            cp_async16(bdst + 16 * q, bsrc + (in && bavail > 16 * q ? 16 * q : 0), clamp_bytes(bavail - 16 * q, 16));
     }
 }
 
-// steps of one warp whose loads are issued together in the Gram pass: KC
-// 16-byte loads per step, 4 KB in flight per warp; eight experts take two
-// steps (8 KB) and one block per SM, whose registers hold the 36 pair sums
-// and both steps
-template <int KC, int SPT>
-struct Batch {
-    static constexpr int U0 = KC >= 8 ? 2 : 8 / KC;
-    static constexpr int U = U0 < SPT ? U0 : SPT;
-};
+// the step's words back from the stage
+template <typename XT, typename BT, int KC>
+__device__ __forceinline__ void read_step(const char* st, int K, int lane, Words<XT, 16 / (int)sizeof(XT)> (&x)[KC],
+                                          Words<BT, 16 / (int)sizeof(XT)>& b) {
+    using G = StageGeom<XT, BT, KC>;
+    constexpr int E = G::E;
+#pragma unroll
+    for (int i = 0; i < KC; ++i) {
+        if (i < K) {
+            const uint4 v = *reinterpret_cast<const uint4*>(st + i * 512 + lane * 16);
+            x[i].w[0] = v.x; x[i].w[1] = v.y; x[i].w[2] = v.z; x[i].w[3] = v.w;
+        }
+    }
+    const char* bs = st + KC * 512 + lane * G::BB;
+    if (G::BB == 8) {
+        const uint2 v = *reinterpret_cast<const uint2*>(bs);
+        b.w[0] = v.x; b.w[1] = v.y;
+    } else {
+#pragma unroll
+        for (int q = 0; q < G::BB / 16; ++q) {
+            const uint4 v = *reinterpret_cast<const uint4*>(bs + 16 * q);
+            b.w[4 * q] = v.x; b.w[4 * q + 1] = v.y; b.w[4 * q + 2] = v.z; b.w[4 * q + 3] = v.w;
+        }
+    }
+    (void)E;
+}
+
+// One warp per tile, a contiguous tile range per warp; every step staged
+// through shared memory (above).
+template <typename XT, typename BT, bool CK, int KC>
+__global__ void __launch_bounds__(TPB, merge_blocks_per_sm(KC)) k_merge(Plan P) {
+    using G = StageGeom<XT, BT, KC>;
+    constexpr int E = G::E;
+    constexpr int SPT = G::SPT;
+    constexpr int D = G::DEPTH;
+    extern __shared__ __align__(16) char s_stage[];
+    const int K = P.K;
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const WarpRange wr = warp_range(P);
+    if (wr.beg >= wr.end) return;
+    char* ring = s_stage + warp * D * G::BYTES;
+    const uint32_t ring_s = (uint32_t)__cvta_generic_to_shared(ring);
+    const long long NS = (wr.end - wr.beg) * SPT;
+    IssueCursor<KC> ic;
+#pragma unroll
+    for (int p = 0; p < D - 1; ++p) {
+        if (p < NS) issue_step<XT, BT, KC>(P, K, ic, wr.beg + p / SPT, p % SPT, ring_s + p * G::BYTES, lane);
+        cp_async_commit();
+    }
+    int t = tensor_of_tile(P.tens, P.n_tensors, wr.beg);
+    long long t_end = tensor_tile_end(P, t);
+    __shared__ MergeParams<KC> s_mp[WPB];
+    MergeParams<KC>& mp = s_mp[warp];
+    merge_params<KC>(P, t, K, mp);
+    float cf[KC];
+    int T[KC];
+    bool exact = false;
+    int opk = 0;
+    bool iso1d = false;
+    long long n = 0, e0 = 0;
+    void* op = nullptr;
+    const TensorDesc* dp = nullptr;
+#pragma unroll 1
+    for (long long i = 0; i < NS; ++i) {
+        const long long g = wr.beg + i / SPT;
+        const int s = (int)(i % SPT);
+        if (s == 0) {
+            if (g >= t_end) {
+                while (g >= t_end) t_end = tensor_tile_end(P, ++t);
+                merge_params<KC>(P, t, K, mp);
+            }
+            dp = &P.tens[t];
+            n = dp->numel;
+            e0 = (g - dp->tile_base) * TILE;
+            const long long e1 = (e0 + TILE < n) ? e0 + TILE : n;
+#pragma unroll
+            for (int q = 0; q < KC; ++q) cf[q] = mp.cf[q];
+            exact = tile_thresholds<KC>(mp, K, (uint32_t)e0, (uint32_t)e1, T);
+            opk = mp.opk;
+            iso1d = mp.iso1d;
+            op = dp->out;
+        }
+        cp_async_wait<D - 2>();
+        Words<XT, E> x[KC];
+        Words<BT, E> b;
+        read_step<XT, BT, KC>(ring + (int)(i % D) * G::BYTES, K, lane, x, b);
+        const long long ni = i + D - 1;
+        if (ni < NS) issue_step<XT, BT, KC>(P, K, ic, wr.beg + ni / SPT, (int)(ni % SPT), ring_s + (int)(ni % D) * G::BYTES, lane);
+        cp_async_commit();
+        const long long e = e0 + (long long)s * (32 * E) + lane * E;
+        if (e >= n) continue;
+        long long r = 0, c = 0;
+        if (exact && mp.sel == SEL_BLOCK) { r = e / dp->cols; c = e - r * dp->cols; }
+        float o[E];
+#pragma unroll
+        for (int j = 0; j < E; ++j) {
+            const float th0 = word_f32<BT, E>(b, j);
+            float tau[KC];
+#pragma unroll
+            for (int q = 0; q < KC; ++q) {
+                tau[q] = (q < K) ? word_f32<XT, E>(x[q], j) : 0.0f;
+                if (CK) tau[q] = __fsub_rn(tau[q], th0);
+            }
+            const uint32_t bits = exact ? select_bits<KC>(P, *dp, mp, K, tau, e + j, r, c)
+                                        : fast_bits<KC>(T, K, tau);
+            o[j] = merged_value<KC>(opk, iso1d, P.lambda, K, th0, tau, cf, bits);
+        }
+        store_out<BT, E>(op, e, n, o);
+    }
+    cp_async_wait<0>();
+}
 
 // Gram of the trimmed task vectors, upper triangle, per 2-D trimmed tensor.
-// Tile partials in binary32 (fused multiply-add over one lane's entries of
-// the tile, then a warp sum), accumulated per warp in binary64 and added to
-// the tensor's Gamma with one atomic per pair when the warp leaves the tensor.
+// The experts stream through the same shared-memory ring as the merge.  Tile
+// partials in binary32 (fused multiply-add over one lane's entries of the
+// tile, then a warp sum), accumulated per warp as binary32 two-sum pairs and
+// added to the tensor's Gamma with one atomic per pair when the warp leaves
+// the tensor.
 template <typename XT, typename BT, bool CK, int KC>
 __global__ void __launch_bounds__(TPB, gram_blocks_per_sm(KC)) k_gramk(Plan P) {
-    constexpr int E = 16 / (int)sizeof(XT);
-    constexpr int SPT = TILE / (32 * E);
-    constexpr int U = Batch<KC, SPT>::U;
+    using G = StageGeom<XT, BT, KC>;
+    constexpr int E = G::E;
+    constexpr int SPT = G::SPT;
+    constexpr int D = G::DEPTH;
     constexpr int NP = KC * (KC + 1) / 2;
     static_assert(NP <= 64, "two pair sums per lane");
+    extern __shared__ __align__(16) char s_stage[];
     const int K = P.K;
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     // lane L accumulates pairs L and 32 + L over the warp's tiles of one
@@ -416,6 +521,15 @@ __global__ void __launch_bounds__(TPB, gram_blocks_per_sm(KC)) k_gramk(Plan P) {
     float gs0 = 0.0f, ge0 = 0.0f, gs1 = 0.0f, ge1 = 0.0f;
     const WarpRange wr = warp_range(P);
     if (wr.beg >= wr.end) return;
+    char* ring = s_stage + warp * D * G::BYTES;
+    const uint32_t ring_s = (uint32_t)__cvta_generic_to_shared(ring);
+    const long long NS = (wr.end - wr.beg) * SPT;
+    IssueCursor<KC> ic;
+#pragma unroll
+    for (int p = 0; p < D - 1; ++p) {
+        if (p < NS) issue_step<XT, BT, KC>(P, K, ic, wr.beg + p / SPT, p % SPT, ring_s + p * G::BYTES, lane);
+        cp_async_commit();
+    }
     int t = tensor_of_tile(P.tens, P.n_tensors, wr.beg);
     long long t_end = tensor_tile_end(P, t);
     __shared__ MergeParams<KC> s_mp[WPB];
@@ -435,83 +549,98 @@ __global__ void __launch_bounds__(TPB, gram_blocks_per_sm(KC)) k_gramk(Plan P) {
         }
         gs0 = ge0 = gs1 = ge1 = 0.0f;
     };
-    for (long long g = wr.beg; g < wr.end; ++g) {
-        if (g >= t_end) {
-            flush(t);
-            while (g >= t_end) t_end = tensor_tile_end(P, ++t);
-            merge_params<KC>(P, t, K, mp);
-        }
-        const TensorDesc& d = P.tens[t];
-        if (!mp.trimmed2d) continue;
-        const long long n = d.numel;
-        const long long e0 = (g - d.tile_base) * TILE;
-        const long long e1 = (e0 + TILE < n) ? e0 + TILE : n;
-        int T[KC];
-        const bool exact = tile_thresholds<KC>(mp, K, (uint32_t)e0, (uint32_t)e1, T);
-        float acc[NP];
-#pragma unroll
-        for (int q = 0; q < NP; ++q) acc[q] = 0.0f;
+    int T[KC];
+    bool exact = false, active = false;
+    long long n = 0, e0 = 0;
+    const TensorDesc* dp = nullptr;
+    float acc[NP];
 #pragma unroll 1
-        for (int s0 = 0; s0 < SPT; s0 += U) {
-            Words<XT, E> xr[U][KC];
-            Words<BT, E> br[U];
-#pragma unroll
-            for (int u = 0; u < U; ++u) {
-                const long long e = e0 + (long long)(s0 + u) * (32 * E) + lane * E;
-                if (e < n) {
-                    if (CK) load_words<BT, E>(d.base, e, n, br[u]);
-#pragma unroll
-                    for (int i = 0; i < KC; ++i)
-                        if (i < K) load_words<XT, E>(mp.xs[i], e, n, xr[u][i]);
-                }
+    for (long long i = 0; i < NS; ++i) {
+        const long long g = wr.beg + i / SPT;
+        const int s = (int)(i % SPT);
+        if (s == 0) {
+            if (g >= t_end) {
+                flush(t);
+                while (g >= t_end) t_end = tensor_tile_end(P, ++t);
+                merge_params<KC>(P, t, K, mp);
             }
+            dp = &P.tens[t];
+            active = mp.trimmed2d;
+            n = dp->numel;
+            e0 = (g - dp->tile_base) * TILE;
+            const long long e1 = (e0 + TILE < n) ? e0 + TILE : n;
+            exact = tile_thresholds<KC>(mp, K, (uint32_t)e0, (uint32_t)e1, T);
 #pragma unroll
-            for (int u = 0; u < U; ++u) {
-                const long long e = e0 + (long long)(s0 + u) * (32 * E) + lane * E;
-                if (e >= n) continue;
-                long long r = 0, c = 0;
-                if (exact && mp.sel == SEL_BLOCK) { r = e / d.cols; c = e - r * d.cols; }
+            for (int q = 0; q < NP; ++q) acc[q] = 0.0f;
+        }
+        cp_async_wait<D - 2>();
+        Words<XT, E> x[KC];
+        Words<BT, E> b;
+        read_step<XT, BT, KC>(ring + (int)(i % D) * G::BYTES, K, lane, x, b);
+        const long long ni = i + D - 1;
+        if (ni < NS) issue_step<XT, BT, KC>(P, K, ic, wr.beg + ni / SPT, (int)(ni % SPT), ring_s + (int)(ni % D) * G::BYTES, lane);
+        cp_async_commit();
+        const long long e = e0 + (long long)s * (32 * E) + lane * E;
+        if (active && e < n) {
+            long long r = 0, c = 0;
+            if (exact && mp.sel == SEL_BLOCK) { r = e / dp->cols; c = e - r * dp->cols; }
 #pragma unroll
-                for (int j = 0; j < E; ++j) {
-                    float tau[KC];
-                    const float th0 = CK ? word_f32<BT, E>(br[u], j) : 0.0f;
+            for (int j = 0; j < E; ++j) {
+                float tau[KC];
+                const float th0 = CK ? word_f32<BT, E>(b, j) : 0.0f;
 #pragma unroll
-                    for (int i = 0; i < KC; ++i) {
-                        tau[i] = (i < K) ? word_f32<XT, E>(xr[u][i], j) : 0.0f;
-                        if (CK) tau[i] = __fsub_rn(tau[i], th0);
+                for (int q = 0; q < KC; ++q) {
+                    tau[q] = (q < K) ? word_f32<XT, E>(x[q], j) : 0.0f;
+                    if (CK) tau[q] = __fsub_rn(tau[q], th0);
+                }
+                uint32_t bits = 0;
+                if (e + j < n) bits = exact ? select_bits<KC>(P, *dp, mp, K, tau, e + j, r, c)
+                                            : fast_bits<KC>(T, K, tau);
+                float m[KC];
+#pragma unroll
+                for (int q = 0; q < KC; ++q) m[q] = ((bits >> q) & 1u) ? tau[q] : 0.0f;
+                int q = 0;
+#pragma unroll
+                for (int a2 = 0; a2 < KC; ++a2)
+#pragma unroll
+                    for (int b2 = a2; b2 < KC; ++b2, ++q) acc[q] = __fmaf_rn(m[a2], m[b2], acc[q]);
+            }
+        }
+        if (s == SPT - 1 && active) {
+            // the tile's partial sums: warp sums, then one two-sum per lane
+            float w0 = 0.0f, w1 = 0.0f;
+            int q = 0;
+#pragma unroll
+            for (int a2 = 0; a2 < KC; ++a2) {
+#pragma unroll
+                for (int b2 = a2; b2 < KC; ++b2, ++q) {
+                    if (a2 < K && b2 < K) {
+                        const float w = warp_sum(acc[q]);
+                        if (q < 32) w0 = (lane == q) ? w : w0;
+                        else w1 = (lane + 32 == q) ? w : w1;
                     }
-                    uint32_t bits = 0;
-                    if (e + j < n) bits = exact ? select_bits<KC>(P, d, mp, K, tau, e + j, r, c)
-                                                : fast_bits<KC>(T, K, tau);
-                    float m[KC];
-#pragma unroll
-                    for (int i = 0; i < KC; ++i) m[i] = ((bits >> i) & 1u) ? tau[i] : 0.0f;
-                    int q = 0;
-#pragma unroll
-                    for (int a = 0; a < KC; ++a)
-#pragma unroll
-                        for (int b = a; b < KC; ++b, ++q) acc[q] = __fmaf_rn(m[a], m[b], acc[q]);
                 }
             }
+            two_sum_add(gs0, ge0, w0);
+            if (NP > 32) two_sum_add(gs1, ge1, w1);
         }
-        float w0 = 0.0f, w1 = 0.0f;
-        int q = 0;
-#pragma unroll
-        for (int a = 0; a < KC; ++a) {
-#pragma unroll
-            for (int b = a; b < KC; ++b, ++q) {
-                if (a < K && b < K) {
-                    const float w = warp_sum(acc[q]);
-                    if (q < 32) w0 = (lane == q) ? w : w0;
-                    else w1 = (lane + 32 == q) ? w : w1;
-                }
-            }
-        }
-        two_sum_add(gs0, ge0, w0);
-        if (NP > 32) two_sum_add(gs1, ge1, w1);
     }
+    cp_async_wait<0>();
     flush(t);
 }
+
+template <typename XT, typename BT, int KC>
+int merge_smem_bytes() { return StageGeom<XT, BT, KC>::SMEM; }
+
+#define ISO_MERGE_SMEM(XT, BT)                                                 \
+    template int merge_smem_bytes<XT, BT, 1>();                               \
+    template int merge_smem_bytes<XT, BT, 2>();                               \
+    template int merge_smem_bytes<XT, BT, 4>();                               \
+    template int merge_smem_bytes<XT, BT, 8>();
+ISO_MERGE_SMEM(__nv_bfloat16, __nv_bfloat16)
+ISO_MERGE_SMEM(__nv_bfloat16, float)
+ISO_MERGE_SMEM(float, __nv_bfloat16)
+ISO_MERGE_SMEM(float, float)
 
 #define ISO_MERGE_INST(XT, BT, CK)                                             \
     template __global__ void k_merge<XT, BT, CK, 2>(Plan);                    \

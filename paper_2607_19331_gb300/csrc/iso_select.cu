@@ -196,9 +196,11 @@ __global__ void __launch_bounds__(SAMPLE_TPB) k_sample(Plan P) {
     }
     __syncthreads();
     uint32_t lo, hi;
+    uint32_t that = 0;                       // fused pass: the estimate of the threshold
     if (S == n) {
         // the sample is the whole unit: the band is the exact threshold
         block_kth_largest2(s_keys, S, U.k, U.k, s_ha, s_hb, s_scan, &s_bin, &s_above, &hi, &lo);
+        that = hi;
     } else {
         const double q = (double)U.k / (double)n;
         const double r = (double)U.k * (double)S / (double)n;
@@ -210,10 +212,123 @@ __global__ void __launch_bounds__(SAMPLE_TPB) k_sample(Plan P) {
                            &s_bin, &s_above, &ka, &kb);
         hi = (ra >= 1) ? ka : KEY_MAX;
         lo = (rb <= S) ? kb : 0u;
+        if (P.fused && P.scope == ISO_SCOPE_TENSOR) {
+            // t^: of the sampled keys at five ranks across the band (the band
+            // edges, the rank of k and halfway between), the one that occurs
+            // most often in the sample -- a run of ties wider than a fifth
+            // of the band is always among them.  The corrections are then
+            // small whichever side of that run rank k falls on.
+            const long long rk = (long long)floor(r + 0.5);
+            const long long h = (long long)floor(delta / 2.0);
+            auto clampr = [&](long long x) { return x < 1 ? 1LL : (x > S ? (long long)S : x); };
+            uint32_t pv[5];
+            pv[0] = ka;
+            pv[4] = kb;
+            block_kth_largest2(s_keys, S, clampr(rk - h), clampr(rk + h), s_ha, s_hb, s_scan, &s_bin, &s_above,
+                               &pv[1], &pv[3]);
+            if (pv[1] == pv[3]) {
+                pv[2] = pv[1];
+            } else {
+                uint32_t dummy;
+                block_kth_largest2(s_keys, S, clampr(rk), clampr(rk), s_ha, s_hb, s_scan, &s_bin, &s_above,
+                                   &pv[2], &dummy);
+            }
+            unsigned cnt[5] = {0, 0, 0, 0, 0};
+            for (int q = threadIdx.x; q < S; q += blockDim.x) {
+                const uint32_t v = s_keys[q];
+#pragma unroll
+                for (int j = 0; j < 5; ++j) cnt[j] += (v == pv[j]);
+            }
+            __shared__ unsigned s_cnt[5];
+            if (threadIdx.x < 5) s_cnt[threadIdx.x] = 0;
+            __syncthreads();
+#pragma unroll
+            for (int j = 0; j < 5; ++j) {
+                const unsigned w = __reduce_add_sync(0xFFFFFFFFu, cnt[j]);
+                if ((threadIdx.x & 31) == 0 && w) atomicAdd(&s_cnt[j], w);
+            }
+            __syncthreads();
+            int best = 2;
+            for (int j = 0; j < 5; ++j)
+                if (s_cnt[j] > s_cnt[best] || (s_cnt[j] == s_cnt[best] && j == 2)) best = j;
+            that = pv[best];
+            if (that > hi) that = hi;
+            if (that < lo) that = lo;
+        }
+    }
+    // Fused K = 1 pass: the estimate t^ of the threshold (the sample's key at
+    // the rank of k; bf16-derived task vectors hold long runs of ties there)
+    // and of the position before which its ties are kept: exact when the
+    // sample is the whole unit, else interpolated from the sampled ties
+    // chunk by chunk.
+    long long chat = -1;
+    if (P.fused && P.scope == ISO_SCOPE_TENSOR) {
+        __shared__ unsigned long long s_cgt;
+        __shared__ unsigned s_ties[SAMPLE_MAX / SAMPLE_CHUNK];
+        __shared__ long long s_chat;
+        if (threadIdx.x == 0) { s_cgt = 0; s_chat = n; }
+        __syncthreads();
+        const uint32_t tk = that;
+        if (S == n) {
+            // keys in position order: the need-th tie
+            const int per = (S + blockDim.x - 1) / blockDim.x;
+            const int q0 = threadIdx.x * per;
+            long long gt = 0, eq = 0;
+            for (int q = q0; q < q0 + per && q < S; ++q) { gt += s_keys[q] > tk; eq += s_keys[q] == tk; }
+            long long tot;
+            const long long before = block_excl_scan(eq, s_scan, &tot);
+            const long long cgt = block_sum(gt, s_scan);
+            const long long need = U.k - cgt;
+            if (before < need && need <= before + eq) {
+                long long acc = before;
+                for (int q = q0; q < q0 + per && q < S; ++q)
+                    if (s_keys[q] == tk && ++acc == need) { s_chat = q + 1; break; }
+            }
+            __syncthreads();
+        } else {
+            const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nw = blockDim.x >> 5;
+            for (int c = warp; c < nch; c += nw) {
+                unsigned gt = 0, eq = 0;
+#pragma unroll
+                for (int j = 0; j < VEC; ++j) {
+                    const uint32_t v = s_keys[c * SAMPLE_CHUNK + lane * VEC + j];
+                    gt += v > tk;
+                    eq += v == tk;
+                }
+                gt = __reduce_add_sync(0xFFFFFFFFu, gt);
+                eq = __reduce_add_sync(0xFFFFFFFFu, eq);
+                if (lane == 0) { s_ties[c] = eq; atomicAdd(&s_cgt, (unsigned long long)gt); }
+            }
+            __syncthreads();
+            if (threadIdx.x == 0) {
+                const double need_s = (double)U.k * (double)S / (double)n - (double)s_cgt;
+                long long ch = n;
+                if (need_s <= 0.0) {
+                    ch = 0;
+                } else {
+                    double cum = 0.0;
+                    for (int c = 0; c < nch; ++c) {
+                        const long long a = (c == 0) ? 0 : (((long long)((double)(n - SAMPLE_CHUNK) * c / (nch - 1))) & ~7LL);
+                        const long long b = (c + 1 == nch) ? n
+                                            : (((long long)((double)(n - SAMPLE_CHUNK) * (c + 1) / (nch - 1))) & ~7LL);
+                        const double tc = (double)s_ties[c];
+                        if (tc > 0.0 && cum + tc >= need_s) {
+                            ch = a + (long long)((need_s - cum) / tc * (double)(b - a));
+                            break;
+                        }
+                        cum += tc;
+                    }
+                }
+                s_chat = ch < 0 ? 0 : (ch > n ? n : ch);
+            }
+            __syncthreads();
+        }
+        chat = s_chat;
     }
     if (threadIdx.x == 0) {
         U.lo = lo;
         U.hi = hi;
+        if (chat >= 0) { U.mode_t = 1; U.that = that; U.chat = chat; }
         U.state = ST_BAND;
     }
 }
@@ -482,7 +597,34 @@ __global__ void k_decide(Plan P) {
     const long long nband = (long long)U.n_int;
     const long long r = U.k - c_gt;
     U.r_src = SRC_CAND;
-    if (r >= 1 && r <= nband && !U.overflow) {
+    if (U.mode_t) {
+        // fused pass: the band holds A candidates above t^, the E keys equal
+        // to t^ (not candidates), and the candidates below t^
+        const long long A = (long long)U.c_abv, E = (long long)U.c_eq;
+        const long long tot = nband + E;
+        if (r >= 1 && r <= tot && !U.overflow) {
+            if (r > A && r <= A + E) {
+                U.t = U.that; U.count_above = c_gt + A; U.ties = E; U.need = r - A; U.tie_src = TIE_EQ_HI;
+                U.state = ST_TKNOWN;
+            } else {
+                U.r_base = U.lo;
+                U.r_pshift = bitlen32(U.hi - U.lo);
+                U.r_prefix = 0;
+                U.r_rank = (r <= A) ? r : r - E;
+                U.r_above = (r <= A) ? c_gt : c_gt + E;
+                U.state = ST_RADIX;
+            }
+        } else {
+            U.fallback = 1;
+            U.r_src = SRC_DATA;
+            U.r_base = 0;
+            U.r_pshift = 31;
+            U.r_prefix = 0;
+            U.r_rank = U.k;
+            U.r_above = 0;
+            U.state = ST_RADIX;
+        }
+    } else if (r >= 1 && r <= nband && !U.overflow) {
         if (r <= c_hi) {
             U.t = U.hi; U.count_above = c_gt; U.ties = c_hi; U.need = r; U.tie_src = TIE_EQ_HI;
             U.state = ST_TKNOWN;
@@ -750,7 +892,7 @@ __device__ __forceinline__ void write_unit_stats(const Plan& P, int idx, const U
     const int i = idx / P.n_units, u = idx % P.n_units;
     iso_unit_stats s;
     s.thresh_key = (U.state == ST_OFF) ? KEY_NONE : U.t;
-    s.flags = U.fallback ? 1u : 0u;
+    s.flags = (U.fallback ? 1u : 0u) | (U.mode_t ? 2u : 0u) | (U.overflow ? 8u : 0u);
     s.k = U.k;
     s.count_above = (U.state == ST_DONE) ? U.count_above : 0;
     s.ties_at_thresh = (U.state == ST_DONE) ? U.ties : 0;
@@ -854,6 +996,11 @@ __global__ void __launch_bounds__(CUT_TPB) k_cut(Plan P) {
             const double ft2 = sq(U.t);
             double above;
             if (U.r_src == SRC_DATA) above = U.gamma_rad;              // every entry above t
+            else if (U.mode_t) {
+                // fused pass: gamma_band holds the candidates above t^
+                if (U.tie_src == TIE_EQ_HI) above = U.gamma_acc + U.gamma_band;   // t == t^
+                else above = U.gamma_acc + U.gamma_rad + (U.t < U.that ? (double)U.c_eq * sq(U.that) : 0.0);
+            }
             else if (U.tie_src == TIE_EQ_HI) above = U.gamma_acc;      // nothing in the band above hi
             else if (U.tie_src == TIE_EQ_LO) above = U.gamma_acc + U.gamma_band;
             else above = U.gamma_acc + U.gamma_rad;                  // candidates above t
