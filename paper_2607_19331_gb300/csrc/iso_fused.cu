@@ -174,43 +174,27 @@ __global__ void __launch_bounds__(TPB, FUSED_BLOCKS_PER_SM) k_count_apply(Plan P
             nrem = (uint32_t)nd.numel - ne0;
         }
 
-        if (!sel) {
+        // speculative selection: kept <=> key > t^, or key == t^ at a
+        // position before chat.  In a whole tile on one side of chat that is
+        // one comparison, key > T, on the tile held in registers.  A tile of a
+        // tensor whose selection is already final, a tile holding chat and a
+        // tensor's last tile (a few per tensor) take a compact per-entry loop
+        // that reads the tile again from L2.  Band keys other than t^ are
+        // rare: their lanes stage them while the step's words are in registers.
+        const uint32_t tile_hi = e0 + min(rem, (uint32_t)TILE);
+        const bool fast = sel && rem >= TILE && (tile_hi <= chat || e0 >= chat);
+        uint32_t n_gt = 0, n_eq = 0;
+        float f_gg = 0.0f;                     // tau^2 above hi (also the non-finite detector)
+        uint2* sp = sbl;
+        if (fast) {
+            const uint32_t T = (tile_hi <= chat) ? th - 1u : th;     // th >= 1 whenever ties are kept here
 #pragma unroll
             for (int v = 0; v < WVEC; ++v) {
                 float th0[VEC], tau[VEC], o[VEC];
                 raw_to_f32<__nv_bfloat16>(rt.b[v], th0);
                 if (CK) rt.tau(v, tau); else raw_to_f32<__nv_bfloat16>(rt.x[v], tau);
-                if (more) rt.load_step(v, nxp, nbp, ne0, nrem, lane);
                 const uint32_t o8 = (uint32_t)(v * (32 * VEC) + lane * VEC);
-                if (o8 >= rem) continue;
-#pragma unroll
-                for (int j = 0; j < VEC; ++j) o[j] = keep_all ? out_of(th0[j], tau[j], a) : th0[j];
-                store8(op, (long long)e0 + o8, n, o, true);
-            }
-            continue;
-        }
-
-        // speculative selection: kept <=> key > t^, or key == t^ at a
-        // position before chat.  In a whole tile on one side of chat that is
-        // one comparison, key > T; a tile holding chat or the tensor's end
-        // takes the per-entry form.  Band keys other than t^ are rare: their
-        // lanes stage them from the step's raw words, still in registers.
-        const uint32_t tile_hi = e0 + min(rem, (uint32_t)TILE);
-        const bool fast = rem >= TILE && (tile_hi <= chat || e0 >= chat);
-        const uint32_t T = (tile_hi <= chat) ? th - 1u : th;     // th >= 1 whenever ties are kept here
-        uint32_t n_gt = 0, n_eq = 0;
-        float f_gg = 0.0f;                     // tau^2 above hi (also the non-finite detector)
-        uint2* sp = sbl;
-#pragma unroll
-        for (int v = 0; v < WVEC; ++v) {
-            float th0[VEC], tau[VEC], o[VEC];
-            raw_to_f32<__nv_bfloat16>(rt.b[v], th0);
-            if (CK) rt.tau(v, tau); else raw_to_f32<__nv_bfloat16>(rt.x[v], tau);
-            const uint4 xw = rt.x[v][0], bw = rt.b[v][0];
-            if (more) rt.load_step(v, nxp, nbp, ne0, nrem, lane);
-            const uint32_t o8 = (uint32_t)(v * (32 * VEC) + lane * VEC);
-            uint32_t bm = 0;                   // band entries of this step
-            if (fast) {
+                uint32_t bm = 0;               // band entries of this step
 #pragma unroll
                 for (int j = 0; j < VEC; ++j) {
                     const uint32_t kk = key_of(tau[j]);
@@ -223,34 +207,52 @@ __global__ void __launch_bounds__(TPB, FUSED_BLOCKS_PER_SM) k_count_apply(Plan P
                     const float upd = __fmul_rn(a, tau[j]);
                     o[j] = (kept && upd != 0.0f) ? __fadd_rn(th0[j], upd) : th0[j];
                 }
-            } else {
-                if (o8 >= rem) continue;
+                store8(op, (long long)e0 + o8, n, o, true);
+                if (bm) {
+                    const uint4 xw = rt.x[v][0], bw = rt.b[v][0];
+                    const uint32_t xr[4] = {xw.x, xw.y, xw.z, xw.w}, br[4] = {bw.x, bw.y, bw.z, bw.w};
+                    do {
+                        const int j = __ffs(bm) - 1;
+                        bm &= bm - 1;
+                        const uint32_t sh = 16u * (uint32_t)(j & 1);
+                        const uint32_t rx = (xr[j >> 1] >> sh) & 0xFFFFu, rb = (br[j >> 1] >> sh) & 0xFFFFu;
+                        *sp = make_uint2(o8 + j, (rb << 16) | rx);
+                        sp += 32;
+                    } while (bm);
+                }
+                if (more) rt.load_step(v, nxp, nbp, ne0, nrem, lane);
+            }
+        } else {
+            // the next tile's loads first, then this tile entry by entry from L2
 #pragma unroll
-                for (int j = 0; j < VEC; ++j) {
-                    const bool valid = o8 + j < rem;
-                    const uint32_t kk = key_of(tau[j]);
-                    const bool gt = valid && kk > hi, eq = valid && kk == th;
-                    const bool kept = (kk > th) || (eq && e0 + o8 + j < chat);
+            for (int v = 0; v < WVEC; ++v)
+                if (more) rt.load_step(v, nxp, nbp, ne0, nrem, lane);
+            const unsigned short* xs16 = static_cast<const unsigned short*>(P.xptr[t]);
+            const unsigned short* bs16 = static_cast<const unsigned short*>(d.base);
+            __nv_bfloat16* q16 = static_cast<__nv_bfloat16*>(op);
+            const uint32_t cnt = min(rem, (uint32_t)TILE);
+#pragma unroll 1
+            for (uint32_t o1 = lane; o1 < cnt; o1 += 32) {
+                const uint32_t pos = e0 + o1;
+                const uint32_t xr = __ldg(xs16 + pos), br = __ldg(bs16 + pos);
+                const float bv = __uint_as_float(br << 16), xv = __uint_as_float(xr << 16);
+                const float tv = CK ? __fsub_rn(xv, bv) : xv;
+                float ov;
+                if (!sel) {
+                    ov = keep_all ? out_of(bv, tv, a) : bv;
+                } else {
+                    const uint32_t kk = key_of(tv);
+                    const bool gt = kk > hi, eq = kk == th;
+                    const bool kept = kk > th || (eq && pos < chat);
                     n_gt += gt;
                     n_eq += eq;
-                    if (gt) f_gg = __fmaf_rn(tau[j], tau[j], f_gg);
-                    bm |= (uint32_t)(valid && kk >= lo && !gt && !eq) << j;
-                    const float upd = __fmul_rn(a, tau[j]);
-                    o[j] = (kept && upd != 0.0f) ? __fadd_rn(th0[j], upd) : th0[j];
+                    if (gt) f_gg = __fmaf_rn(tv, tv, f_gg);
+                    if (kk >= lo && !gt && !eq) { *sp = make_uint2(o1, (br << 16) | xr); sp += 32; }
+                    ov = kept ? out_of(bv, tv, a) : bv;
                 }
+                q16[pos] = __float2bfloat16_rn(ov);
             }
-            store8(op, (long long)e0 + o8, n, o, true);
-            if (bm) {
-                const uint32_t xr[4] = {xw.x, xw.y, xw.z, xw.w}, br[4] = {bw.x, bw.y, bw.z, bw.w};
-                do {
-                    const int j = __ffs(bm) - 1;
-                    bm &= bm - 1;
-                    const uint32_t sh = 16u * (uint32_t)(j & 1);
-                    const uint32_t rx = (xr[j >> 1] >> sh) & 0xFFFFu, rb = (br[j >> 1] >> sh) & 0xFFFFu;
-                    *sp = make_uint2(o8 + j, (rb << 16) | rx);
-                    sp += 32;
-                } while (bm);
-            }
+            if (!sel) continue;
         }
         if (__any_sync(FULL, !(fabsf(f_gg) <= 3.402823466e38f))) {
             // a non-finite (or overflowing) sum: read the tile's keys again
@@ -307,8 +309,7 @@ __global__ void __launch_bounds__(TPB, FUSED_BLOCKS_PER_SM) k_count_apply(Plan P
         if (lane == 0) {
             P.tcand[g] = make_uint2(c_store ? c_pos : 0u, c_store ? nb_tot : 0u);
             P.tband[g] = make_uint2(b_store ? b_pos : 0u, b_store ? nb_tot : 0u);
-            P.teq_lo[g] = 0;
-            P.teq_hi[g] = t_eq;
+            P.teq_hi[g] = t_eq;                 // teq_lo stays 0 (zeroed with the group's state)
         }
         if (c_store) { c_pos += nb_tot; c_left -= nb_tot; }
         if (b_store) { b_pos += nb_tot; b_left -= nb_tot; }

@@ -257,7 +257,7 @@ __device__ __forceinline__ bool tile_thresholds(const MergeParams<KC>& mp, int K
     bool exact = (mp.sel == SEL_BLOCK);
 #pragma unroll
     for (int i = 0; i < KC; ++i) {
-        T[i] = -1;
+        T[i] = (i < K) ? -1 : 0x7FFFFFFF;                      // experts past K: nothing kept
         if (i < K && mp.sel == SEL_PACKED) {
             const unsigned long long th = mp.thr[i];
             const uint32_t tk = (uint32_t)(th >> 32), c32 = ~(uint32_t)th;
@@ -268,6 +268,56 @@ __device__ __forceinline__ bool tile_thresholds(const MergeParams<KC>& mp, int K
         }
     }
     return exact;
+}
+
+// merged output of one entry inside a tile with per-tile thresholds: the
+// selection of expert q is (int)key > T[q] (never for q >= K), unselected
+// terms enter the sums as +0, which leaves every sum and the output as the
+// skipping form gives them
+template <int KC>
+__device__ __forceinline__ float merged_fast(int opk, bool iso1d, float lambda, int K, float th0,
+                                             const float (&tau)[KC], const float (&cf)[KC], const int (&T)[KC]) {
+    float upd;
+    if (opk == OPK_TIES) {
+        // gamma = sign of the trimmed sum; the agreeing set: the non-zero
+        // trimmed values of that sign.  u = tt with the sign of the sum
+        // cleared is |tt| exactly for the agreeing ones, so their sum in
+        // order is the magnitude of the signed sum, bit for bit.
+        float tt[KC];
+        float s = 0.0f;
+#pragma unroll
+        for (int q = 0; q < KC; ++q) {
+            tt[q] = ((int)key_of(tau[q]) > T[q]) ? tau[q] : 0.0f;
+            s = __fadd_rn(s, tt[q]);
+        }
+        const uint32_t sb = __float_as_uint(s) & 0x80000000u;
+        float a = 0.0f;
+        int cnt = 0;
+#pragma unroll
+        for (int q = 0; q < KC; ++q) {
+            const float u = __uint_as_float(__float_as_uint(tt[q]) ^ sb);
+            const bool ag = u > 0.0f;
+            a = ag ? __fadd_rn(a, u) : a;
+            cnt += ag;
+        }
+        if (s == 0.0f) cnt = 0;
+        float m = cnt ? __fdiv_rn(a, (float)cnt) : 0.0f;
+        m = __uint_as_float(__float_as_uint(m) ^ sb);
+        upd = __fmul_rn(lambda, m);
+    } else if (opk == OPK_ISO) {
+        float s = 0.0f;
+#pragma unroll
+        for (int q = 0; q < KC; ++q)
+            s = __fadd_rn(s, ((int)key_of(tau[q]) > T[q]) ? __fmul_rn(cf[q], tau[q]) : 0.0f);
+        upd = s;
+    } else {
+        float s = 0.0f;
+#pragma unroll
+        for (int q = 0; q < KC; ++q)
+            if (q < K) s = __fadd_rn(s, tau[q]);
+        upd = iso1d ? __fdiv_rn(s, (float)K) : __fmul_rn(lambda, s);
+    }
+    return (upd == 0.0f) ? th0 : __fadd_rn(th0, upd);
 }
 
 template <int KC>
@@ -490,9 +540,12 @@ __global__ void __launch_bounds__(TPB, merge_blocks_per_sm(KC)) k_merge(Plan P) 
                 tau[q] = (q < K) ? word_f32<XT, E>(x[q], j) : 0.0f;
                 if (CK) tau[q] = __fsub_rn(tau[q], th0);
             }
-            const uint32_t bits = exact ? select_bits<KC>(P, *dp, mp, K, tau, e + j, r, c)
-                                        : fast_bits<KC>(T, K, tau);
-            o[j] = merged_value<KC>(opk, iso1d, P.lambda, K, th0, tau, cf, bits);
+            if (exact) {
+                const uint32_t bits = select_bits<KC>(P, *dp, mp, K, tau, e + j, r, c);
+                o[j] = merged_value<KC>(opk, iso1d, P.lambda, K, th0, tau, cf, bits);
+            } else {
+                o[j] = merged_fast<KC>(opk, iso1d, P.lambda, K, th0, tau, cf, T);
+            }
         }
         store_out<BT, E>(op, e, n, o);
     }
@@ -593,12 +646,17 @@ __global__ void __launch_bounds__(TPB, gram_blocks_per_sm(KC)) k_gramk(Plan P) {
                     tau[q] = (q < K) ? word_f32<XT, E>(x[q], j) : 0.0f;
                     if (CK) tau[q] = __fsub_rn(tau[q], th0);
                 }
-                uint32_t bits = 0;
-                if (e + j < n) bits = exact ? select_bits<KC>(P, *dp, mp, K, tau, e + j, r, c)
-                                            : fast_bits<KC>(T, K, tau);
                 float m[KC];
+                if (exact) {
+                    const uint32_t bits = (e + j < n) ? select_bits<KC>(P, *dp, mp, K, tau, e + j, r, c) : 0u;
 #pragma unroll
-                for (int q = 0; q < KC; ++q) m[q] = ((bits >> q) & 1u) ? tau[q] : 0.0f;
+                    for (int q = 0; q < KC; ++q) m[q] = ((bits >> q) & 1u) ? tau[q] : 0.0f;
+                } else {
+                    // past the tensor's end the loads read zeros: key 0 is never selected by T >= 0,
+                    // and T = -1 (everything kept) only leaves zeros in the sums
+#pragma unroll
+                    for (int q = 0; q < KC; ++q) m[q] = ((int)key_of(tau[q]) > T[q]) ? tau[q] : 0.0f;
+                }
                 int q = 0;
 #pragma unroll
                 for (int a2 = 0; a2 < KC; ++a2)
