@@ -37,6 +37,9 @@ __global__ void __launch_bounds__(TPB, FUSED_BLOCKS_PER_SM) k_count_apply(Plan P
     extern __shared__ uint2 s_stage[];
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     uint2* const sbl = s_stage + warp * (TILE + 32) + lane;
+    // the raw words of the tile being decided, per lane and step (x then theta_0)
+    uint32_t* const s_raw = reinterpret_cast<uint32_t*>(s_stage + WPB * (TILE + 32)) +
+                            (warp * WVEC * 32 + lane) * 8;
     const uint32_t W = gridDim.x * WPB;
     const uint32_t wid = blockIdx.x * WPB + warp;
     const uint32_t items = (uint32_t)P.n_tiles;
@@ -188,13 +191,17 @@ __global__ void __launch_bounds__(TPB, FUSED_BLOCKS_PER_SM) k_count_apply(Plan P
         uint2* sp = sbl;
         if (fast) {
             const uint32_t T = (tile_hi <= chat) ? th - 1u : th;     // th >= 1 whenever ties are kept here
+            uint32_t tbm = 0;                  // band entries of the tile: bit 8 v + j
 #pragma unroll
             for (int v = 0; v < WVEC; ++v) {
                 float th0[VEC], tau[VEC], o[VEC];
                 raw_to_f32<__nv_bfloat16>(rt.b[v], th0);
                 if (CK) rt.tau(v, tau); else raw_to_f32<__nv_bfloat16>(rt.x[v], tau);
+                // keep the step's raw words for the band entries, then reuse the registers
+                *reinterpret_cast<uint4*>(s_raw + v * 256) = rt.x[v][0];
+                *reinterpret_cast<uint4*>(s_raw + v * 256 + 4) = rt.b[v][0];
+                if (more) rt.load_step(v, nxp, nbp, ne0, nrem, lane);
                 const uint32_t o8 = (uint32_t)(v * (32 * VEC) + lane * VEC);
-                uint32_t bm = 0;               // band entries of this step
 #pragma unroll
                 for (int j = 0; j < VEC; ++j) {
                     const uint32_t kk = key_of(tau[j]);
@@ -203,24 +210,22 @@ __global__ void __launch_bounds__(TPB, FUSED_BLOCKS_PER_SM) k_count_apply(Plan P
                     n_gt += gt;
                     n_eq += eq;
                     if (gt) f_gg = __fmaf_rn(tau[j], tau[j], f_gg);
-                    bm |= (uint32_t)(kk >= lo && !gt && !eq) << j;
+                    if (kk >= lo && !gt && !eq) tbm |= 1u << (v * VEC + j);
                     const float upd = __fmul_rn(a, tau[j]);
                     o[j] = (kept && upd != 0.0f) ? __fadd_rn(th0[j], upd) : th0[j];
                 }
                 store8(op, (long long)e0 + o8, n, o, true);
-                if (bm) {
-                    const uint4 xw = rt.x[v][0], bw = rt.b[v][0];
-                    const uint32_t xr[4] = {xw.x, xw.y, xw.z, xw.w}, br[4] = {bw.x, bw.y, bw.z, bw.w};
-                    do {
-                        const int j = __ffs(bm) - 1;
-                        bm &= bm - 1;
-                        const uint32_t sh = 16u * (uint32_t)(j & 1);
-                        const uint32_t rx = (xr[j >> 1] >> sh) & 0xFFFFu, rb = (br[j >> 1] >> sh) & 0xFFFFu;
-                        *sp = make_uint2(o8 + j, (rb << 16) | rx);
-                        sp += 32;
-                    } while (bm);
-                }
-                if (more) rt.load_step(v, nxp, nbp, ne0, nrem, lane);
+            }
+            // the lane's band entries into its staging list, raw bits from shared memory
+            while (tbm) {
+                const int b = __ffs(tbm) - 1;
+                tbm &= tbm - 1;
+                const int v = b >> 3, j = b & 7;
+                const uint32_t sh = 16u * (uint32_t)(j & 1);
+                const uint32_t rx = (s_raw[v * 256 + (j >> 1)] >> sh) & 0xFFFFu;
+                const uint32_t rb = (s_raw[v * 256 + 4 + (j >> 1)] >> sh) & 0xFFFFu;
+                *sp = make_uint2((uint32_t)(v * (32 * VEC) + lane * VEC + j), (rb << 16) | rx);
+                sp += 32;
             }
         } else {
             // the next tile's loads first, then this tile entry by entry from L2
@@ -355,8 +360,10 @@ __global__ void __launch_bounds__(TPB) k_patch(Plan P) {
             const uint32_t c32 = (cut >= 0xFFFFFFFFLL) ? 0xFFFFFFFFu : (uint32_t)cut;
             thr = ((unsigned long long)U->t << 32) | (uint32_t)~c32;
         }
-        const uint2 r = P.tband[it];
-        for (uint32_t q = lane; q < r.y; q += 32) {
+        // 32 tiles at a time, one per lane
+        const uint32_t nt = min(32u, min(run_end, end) - it);
+        const uint2 r = (lane < (int)nt) ? P.tband[it + lane] : make_uint2(0u, 0u);
+        for (uint32_t q = 0; q < r.y; ++q) {
             const uint2 rec = bseg[r.x + q];
             const float xv = __uint_as_float(rec.y << 16);
             const float bv = __uint_as_float(rec.y & 0xFFFF0000u);
@@ -365,7 +372,7 @@ __global__ void __launch_bounds__(TPB) k_patch(Plan P) {
             const bool kept = (((unsigned long long)kk << 32) | (uint32_t)~rec.x) > thr;
             if (kept != (kk > th)) op[rec.x] = __float2bfloat16_rn(kept ? out_of(bv, tau, a) : bv);
         }
-        ++it;
+        it += nt;
     }
 }
 

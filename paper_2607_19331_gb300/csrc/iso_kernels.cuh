@@ -26,7 +26,8 @@ template <typename XT, typename BT, bool CK> __global__ void k_block_select(Plan
 
 // fused K = 1 pass (bf16 base and update)
 constexpr int FUSED_BLOCKS_PER_SM = 2;
-constexpr int FUSED_SMEM = WPB * (TILE + 32) * 8;   // band staging, dynamic shared memory
+// dynamic shared memory: band staging (8 B per slot) and the raw words of a tile (4 KB per warp)
+constexpr int FUSED_SMEM = WPB * (TILE + 32) * 8 + WPB * TILE * 4;
 template <bool CK> __global__ void k_count_apply(Plan P);
 template <bool CK> __global__ void k_patch(Plan P);
 __global__ void k_fix_plan(Plan P);
