@@ -191,6 +191,7 @@ __global__ void __launch_bounds__(TPB, FUSED_BLOCKS_PER_SM) k_count_apply(Plan P
         uint2* sp = sbl;
         if (fast) {
             const uint32_t T = (tile_hi <= chat) ? th - 1u : th;     // th >= 1 whenever ties are kept here
+            const uint32_t span = hi - lo;     // band: key - lo <= span (unsigned), key != t^
             uint32_t tbm = 0;                  // band entries of the tile: bit 8 v + j
 #pragma unroll
             for (int v = 0; v < WVEC; ++v) {
@@ -210,9 +211,9 @@ __global__ void __launch_bounds__(TPB, FUSED_BLOCKS_PER_SM) k_count_apply(Plan P
                     n_gt += gt;
                     n_eq += eq;
                     if (gt) f_gg = __fmaf_rn(tau[j], tau[j], f_gg);
-                    if (kk >= lo && !gt && !eq) tbm |= 1u << (v * VEC + j);
+                    if ((kk - lo <= span) & !eq) tbm |= 1u << (v * VEC + j);
                     const float upd = __fmul_rn(a, tau[j]);
-                    o[j] = (kept && upd != 0.0f) ? __fadd_rn(th0[j], upd) : th0[j];
+                    o[j] = (kept & (upd != 0.0f)) ? __fadd_rn(th0[j], upd) : th0[j];
                 }
                 store8(op, (long long)e0 + o8, n, o, true);
             }

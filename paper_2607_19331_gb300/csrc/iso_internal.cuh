@@ -34,7 +34,7 @@ constexpr int SAMPLE_MAX = 24576;           // sampled keys per unit (96 KB of s
 constexpr int SAMPLE_CHUNK = 256;           // contiguous entries per sample chunk
 constexpr int SAMPLE_TPB = 1024;
 constexpr double SAMPLE_Z = 5.0;            // band half-width in sample standard deviations
-constexpr double RUN_Z = 3.0;               // fused K = 1 pass: margin of a run of ties taken as the threshold
+constexpr int COUNT_CHUNKS = 512;           // fused K = 1 pass: 256-entry chunks counted for the cut estimate
 
 constexpr int RADIX_BITS = 11;
 constexpr int RADIX_BINS = 1 << RADIX_BITS;

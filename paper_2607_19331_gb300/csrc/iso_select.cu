@@ -254,6 +254,12 @@ __global__ void __launch_bounds__(SAMPLE_TPB) k_sample(Plan P) {
             that = pv[best];
             if (that > hi) that = hi;
             if (that < lo) that = lo;
+            // run mode: the run of t^ covers the sample rank of k by half the
+            // band on both sides (2.5 sample standard deviations), so the
+            // threshold is t^ but for a small chance, which the counts catch
+            // (then the unit is resolved exactly and re-applied): the band
+            // collapses to t^ and the fused pass needs no band test
+            if (pv[1] == that && pv[3] == that) { lo = that; hi = that; }
         }
     }
     // Fused K = 1 pass: the estimate t^ of the threshold (the sample's key at
@@ -264,7 +270,7 @@ __global__ void __launch_bounds__(SAMPLE_TPB) k_sample(Plan P) {
     long long chat = -1;
     if (P.fused && P.scope == ISO_SCOPE_TENSOR) {
         __shared__ unsigned long long s_cgt;
-        __shared__ unsigned s_ties[SAMPLE_MAX / SAMPLE_CHUNK];
+        __shared__ unsigned s_ties[COUNT_CHUNKS];
         __shared__ long long s_chat;
         if (threadIdx.x == 0) { s_cgt = 0; s_chat = n; }
         __syncthreads();
@@ -286,41 +292,54 @@ __global__ void __launch_bounds__(SAMPLE_TPB) k_sample(Plan P) {
             }
             __syncthreads();
         } else {
+            // a larger count sample for the cut: CX chunks of 256 entries,
+            // contiguous when they cover the unit, else evenly spaced; per
+            // chunk the keys equal to t^, overall the keys above it
+            const long long nchunks = (n + SAMPLE_CHUNK - 1) / SAMPLE_CHUNK;
+            const bool whole = nchunks <= COUNT_CHUNKS;
+            const int CX = whole ? (int)nchunks : COUNT_CHUNKS;
+            auto chunk_start = [&](int c) -> long long {
+                if (whole) return (long long)c * SAMPLE_CHUNK;
+                return (long long)(((unsigned long long)(n - SAMPLE_CHUNK) * (unsigned long long)c) /
+                                   (unsigned long long)(CX - 1)) & ~7LL;
+            };
+            const int t = U.tensor;
+            const void* x = P.xptr[U.expert * P.n_tensors + t];
+            const void* b = P.tens[t].base;
             const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nw = blockDim.x >> 5;
-            for (int c = warp; c < nch; c += nw) {
+            for (int c = warp; c < CX; c += nw) {
+                const long long st = chunk_start(c);
+                const long long e = st + lane * VEC;
+                float tau[VEC];
+                TauSrc<XT, BT, CKPT>::load8(x, b, e, n, tau);
                 unsigned gt = 0, eq = 0;
 #pragma unroll
                 for (int j = 0; j < VEC; ++j) {
-                    const uint32_t v = s_keys[c * SAMPLE_CHUNK + lane * VEC + j];
-                    gt += v > tk;
-                    eq += v == tk;
+                    const uint32_t v = key_of(tau[j]);
+                    const bool in = e + j < n;
+                    gt += in && v > tk;
+                    eq += in && v == tk;
                 }
                 gt = __reduce_add_sync(0xFFFFFFFFu, gt);
                 eq = __reduce_add_sync(0xFFFFFFFFu, eq);
                 if (lane == 0) { s_ties[c] = eq; atomicAdd(&s_cgt, (unsigned long long)gt); }
             }
             __syncthreads();
-            if (threadIdx.x == 0) {
-                const double need_s = (double)U.k * (double)S / (double)n - (double)s_cgt;
-                long long ch = n;
-                if (need_s <= 0.0) {
-                    ch = 0;
-                } else {
-                    double cum = 0.0;
-                    for (int c = 0; c < nch; ++c) {
-                        const long long a = (c == 0) ? 0 : (((long long)((double)(n - SAMPLE_CHUNK) * c / (nch - 1))) & ~7LL);
-                        const long long b = (c + 1 == nch) ? n
-                                            : (((long long)((double)(n - SAMPLE_CHUNK) * (c + 1) / (nch - 1))) & ~7LL);
-                        const double tc = (double)s_ties[c];
-                        if (tc > 0.0 && cum + tc >= need_s) {
-                            ch = a + (long long)((need_s - cum) / tc * (double)(b - a));
-                            break;
-                        }
-                        cum += tc;
-                    }
-                }
+            // the chunk where the sampled ties reach the sampled need, one
+            // thread per chunk (a scan over the chunks' tie counts)
+            const long long SX = whole ? n : (long long)CX * SAMPLE_CHUNK;
+            const double need_s = (double)U.k * (double)SX / (double)n - (double)s_cgt;
+            const int c = threadIdx.x;
+            const long long tcl = (c < CX) ? (long long)s_ties[c] : 0;
+            long long tot_ties;
+            const long long cum = block_excl_scan(tcl, s_scan, &tot_ties);
+            if (c < CX && tcl > 0 && (double)cum < need_s && need_s <= (double)(cum + tcl)) {
+                const long long a = chunk_start(c);
+                const long long bb = (c + 1 == CX) ? n : chunk_start(c + 1);
+                const long long ch = a + (long long)((need_s - (double)cum) / (double)tcl * (double)(bb - a));
                 s_chat = ch < 0 ? 0 : (ch > n ? n : ch);
             }
+            if (c == 0 && need_s <= 0.0) s_chat = 0;
             __syncthreads();
         }
         chat = s_chat;
