@@ -82,13 +82,25 @@ def algorithmic_bytes(shapes, K, inputs, op, scope="tensor", two_pass=False):
     return out
 
 
-def kernel_source_hash():
-    """sha1 of the kernel sources: a profile's traffic applies only to the
-    kernels it measured."""
-    import glob
+# the source files each timed kernel kind is built from (besides the shared headers)
+KERNEL_SOURCES = {
+    "count": ["iso_fused.cu", "iso_select.cu"],   # fused K = 1 pass, or the two-pass counting read
+    "apply": ["iso_apply.cu", "iso_merge.cu"],
+    "gram": ["iso_merge.cu"],
+    "block_select": ["iso_block.cu"],
+}
+
+
+def kernel_source_hash(kind=None):
+    """sha1 of a kernel kind's sources and the shared headers (all sources
+    when kind is None): a profile's traffic applies only to the kernels it
+    measured."""
     import hashlib
     csrc = os.path.join(ROOT, "paper_2607_19331_gb300", "csrc")
-    files = sorted(glob.glob(os.path.join(csrc, "*.cu")) + glob.glob(os.path.join(csrc, "*.cuh")))
+    names = KERNEL_SOURCES.get(kind) if kind else None
+    if names is None:
+        names = sorted(f for f in os.listdir(csrc) if f.endswith(".cu"))
+    files = [os.path.join(csrc, f) for f in sorted(names) + ["iso_internal.cuh", "iso_kernels.cuh"]]
     files.append(os.path.join(ROOT, "include", "iso.h"))
     h = hashlib.sha1()
     for f in files:
@@ -100,9 +112,9 @@ def kernel_source_hash():
 
 def profiled_traffic(kernel, workload):
     """DRAM bytes per parameter of `kernel` from the committed ncu summaries in
-    profiles/, if they were taken on the current kernel sources."""
+    profiles/, if they were taken on the kernel's current sources."""
     import glob
-    sha = kernel_source_hash()
+    sha = kernel_source_hash(kernel)
     for f in glob.glob(os.path.join(ROOT, "profiles", "*.md")):
         for line in open(f):
             if not line.startswith("traffic:"):

@@ -57,6 +57,7 @@ __global__ void __launch_bounds__(TPB, FUSED_BLOCKS_PER_SM) k_count_apply(Plan P
     bool keep_all = false;                    // otherwise: every entry kept (untrimmed) or none (k == 0)
     float a = 0.0f;                           // coefficient of the kept entries
     uint32_t lo = 0, hi = 0, th = 0, chat = 0;
+    bool a_t_normal = false;                  // |a t^| is a normal binary32 number
     Unit* au = nullptr;
     uint32_t a_gt = 0, a_eq = 0, a_int = 0, a_abv = 0;
     float s_gg = 0.0f, e_gg = 0.0f, s_gb = 0.0f, e_gb = 0.0f;
@@ -109,6 +110,7 @@ __global__ void __launch_bounds__(TPB, FUSED_BLOCKS_PER_SM) k_count_apply(Plan P
         lo = U->lo;
         hi = U->hi;
         th = U->that;
+        a_t_normal = fabsf(__fmul_rn(a, __uint_as_float(th))) >= 1.17549435e-38f;
         const long long ch = U->chat;
         chat = (uint32_t)(ch < 0 ? 0 : ch);
         want_gamma = U->want_gamma != 0;
@@ -185,7 +187,10 @@ __global__ void __launch_bounds__(TPB, FUSED_BLOCKS_PER_SM) k_count_apply(Plan P
         // that reads the tile again from L2.  Band keys other than t^ are
         // rare: their lanes stage them while the step's words are in registers.
         const uint32_t tile_hi = e0 + min(rem, (uint32_t)TILE);
-        const bool fast = sel && rem >= TILE && (tile_hi <= chat || e0 >= chat);
+        // the fast form writes theta_0 + (kept ? a tau : -0): exact (theta_0 bits
+        // kept for an update of 0) because every kept |tau| is at least t^'s and
+        // a times that stays a normal number
+        const bool fast = sel && rem >= TILE && (tile_hi <= chat || e0 >= chat) && a_t_normal;
         uint32_t n_gt = 0, n_eq = 0;
         float f_gg = 0.0f;                     // tau^2 above hi (also the non-finite detector)
         uint2* sp = sbl;
@@ -212,8 +217,7 @@ __global__ void __launch_bounds__(TPB, FUSED_BLOCKS_PER_SM) k_count_apply(Plan P
                     n_eq += eq;
                     if (gt) f_gg = __fmaf_rn(tau[j], tau[j], f_gg);
                     if ((kk - lo <= span) & !eq) tbm |= 1u << (v * VEC + j);
-                    const float upd = __fmul_rn(a, tau[j]);
-                    o[j] = (kept & (upd != 0.0f)) ? __fadd_rn(th0[j], upd) : th0[j];
+                    o[j] = __fadd_rn(th0[j], kept ? __fmul_rn(a, tau[j]) : -0.0f);
                 }
                 store8(op, (long long)e0 + o8, n, o, true);
             }

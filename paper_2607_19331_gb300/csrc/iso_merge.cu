@@ -392,7 +392,7 @@ struct IssueCursor {
     long long g = -1;        // tile of the cached tensor data
     int t = 0;
     long long t_end = 0, e0 = 0, n = 0;
-    const void* xs[KC];
+    const void** xs;         // the warp's copy of the tensor's KC expert pointers (shared memory)
     const void* bp = nullptr;
 };
 
@@ -411,6 +411,7 @@ __device__ __forceinline__ void issue_step(const Plan& P, int K, IssueCursor<KC>
             ic.bp = d.base;
 #pragma unroll
             for (int i = 0; i < KC; ++i) ic.xs[i] = (i < K) ? P.xptr[i * P.n_tensors + ic.t] : nullptr;
+            __syncwarp();
         }
         ic.g = g;
         ic.e0 = (g - P.tens[ic.t].tile_base) * TILE;
@@ -480,7 +481,9 @@ __global__ void __launch_bounds__(TPB, merge_blocks_per_sm(KC)) k_merge(Plan P) 
     char* ring = s_stage + warp * D * G::BYTES;
     const uint32_t ring_s = (uint32_t)__cvta_generic_to_shared(ring);
     const long long NS = (wr.end - wr.beg) * SPT;
+    __shared__ const void* s_xs[WPB][KC];
     IssueCursor<KC> ic;
+    ic.xs = s_xs[warp];
 #pragma unroll
     for (int p = 0; p < D - 1; ++p) {
         if (p < NS) issue_step<XT, BT, KC>(P, K, ic, wr.beg + p / SPT, p % SPT, ring_s + p * G::BYTES, lane);
@@ -577,7 +580,9 @@ __global__ void __launch_bounds__(TPB, gram_blocks_per_sm(KC)) k_gramk(Plan P) {
     char* ring = s_stage + warp * D * G::BYTES;
     const uint32_t ring_s = (uint32_t)__cvta_generic_to_shared(ring);
     const long long NS = (wr.end - wr.beg) * SPT;
+    __shared__ const void* s_xs[WPB][KC];
     IssueCursor<KC> ic;
+    ic.xs = s_xs[warp];
 #pragma unroll
     for (int p = 0; p < D - 1; ++p) {
         if (p < NS) issue_step<XT, BT, KC>(P, K, ic, wr.beg + p / SPT, p % SPT, ring_s + p * G::BYTES, lane);
