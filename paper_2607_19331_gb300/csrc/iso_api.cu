@@ -573,7 +573,7 @@ int run_group(const Call& c, int t0, int t1, char* ws, cudaStream_t s, const iso
                 auto gram = [&](auto kc) {
                     constexpr int KC = decltype(kc)::value;
                     const int ggrid = sms * gram_blocks_per_sm(KC);
-                    const int smem = merge_smem_bytes<XT, BT, KC>();
+                    const int smem = gram_smem_bytes<XT, BT, KC>();
                     ISO_TRY(smem_optin(k_gramk<XT, BT, CK, KC>, smem));
                     return launch(KD_GRAM, s, [&] { k_gramk<XT, BT, CK, KC><<<ggrid, TPB, smem, s>>>(P); });
                 };
@@ -586,10 +586,16 @@ int run_group(const Call& c, int t0, int t1, char* ws, cudaStream_t s, const iso
         }
         auto merge = [&](auto kc) {
             constexpr int KC = decltype(kc)::value;
-            const int smem = merge_smem_bytes<XT, BT, KC>();
-            const int mgrid = sms * merge_blocks_per_sm(KC);
-            ISO_TRY(smem_optin(k_merge<XT, BT, CK, KC>, smem));
-            return launch(KD_APPLY, s, [&] { k_merge<XT, BT, CK, KC><<<mgrid, TPB, smem, s>>>(P); });
+            if (c.op == ISO_OP_TIES) {
+                const int smem = merge_smem_bytes<XT, BT, KC, OPF_TIES>();
+                const int mgrid = sms * merge_blocks_per_sm(KC, OPF_TIES);
+                ISO_TRY(smem_optin(k_merge<XT, BT, CK, KC, OPF_TIES>, smem));
+                return launch(KD_APPLY, s, [&] { k_merge<XT, BT, CK, KC, OPF_TIES><<<mgrid, TPB, smem, s>>>(P); });
+            }
+            const int smem = merge_smem_bytes<XT, BT, KC, OPF_OTHER>();
+            const int mgrid = sms * merge_blocks_per_sm(KC, OPF_OTHER);
+            ISO_TRY(smem_optin(k_merge<XT, BT, CK, KC, OPF_OTHER>, smem));
+            return launch(KD_APPLY, s, [&] { k_merge<XT, BT, CK, KC, OPF_OTHER><<<mgrid, TPB, smem, s>>>(P); });
         };
         if (K == 1) ISO_TRY(launch(KD_APPLY, s, [&] { k_apply<XT, BT, CK, 1><<<pgrid, TPB, 0, s>>>(P); }));
         else if (K == 2) ISO_TRY(merge(std::integral_constant<int, 2>{}));

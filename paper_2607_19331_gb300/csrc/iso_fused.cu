@@ -38,8 +38,9 @@ __global__ void __launch_bounds__(TPB, FUSED_BLOCKS_PER_SM) k_count_apply(Plan P
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     uint2* const sbl = s_stage + warp * (TILE + 32) + lane;
     // the raw words of the tile being decided, per lane and step (x then theta_0)
-    uint32_t* const s_raw = reinterpret_cast<uint32_t*>(s_stage + WPB * (TILE + 32)) +
-                            (warp * WVEC * 32 + lane) * 8;
+    // step v's x words of lane L at uint4 (2 v * 32 + L), its theta_0 words at ((2 v + 1) * 32 + L):
+    // each warp-wide store is 512 contiguous bytes
+    uint4* const s_raw = reinterpret_cast<uint4*>(s_stage + WPB * (TILE + 32)) + warp * (WVEC * 2 * 32) + lane;
     const uint32_t W = gridDim.x * WPB;
     const uint32_t wid = blockIdx.x * WPB + warp;
     const uint32_t items = (uint32_t)P.n_tiles;
@@ -204,8 +205,8 @@ __global__ void __launch_bounds__(TPB, FUSED_BLOCKS_PER_SM) k_count_apply(Plan P
                 raw_to_f32<__nv_bfloat16>(rt.b[v], th0);
                 if (CK) rt.tau(v, tau); else raw_to_f32<__nv_bfloat16>(rt.x[v], tau);
                 // keep the step's raw words for the band entries, then reuse the registers
-                *reinterpret_cast<uint4*>(s_raw + v * 256) = rt.x[v][0];
-                *reinterpret_cast<uint4*>(s_raw + v * 256 + 4) = rt.b[v][0];
+                s_raw[(2 * v) * 32] = rt.x[v][0];
+                s_raw[(2 * v + 1) * 32] = rt.b[v][0];
                 if (more) rt.load_step(v, nxp, nbp, ne0, nrem, lane);
                 const uint32_t o8 = (uint32_t)(v * (32 * VEC) + lane * VEC);
 #pragma unroll
@@ -227,8 +228,8 @@ __global__ void __launch_bounds__(TPB, FUSED_BLOCKS_PER_SM) k_count_apply(Plan P
                 tbm &= tbm - 1;
                 const int v = b >> 3, j = b & 7;
                 const uint32_t sh = 16u * (uint32_t)(j & 1);
-                const uint32_t rx = (s_raw[v * 256 + (j >> 1)] >> sh) & 0xFFFFu;
-                const uint32_t rb = (s_raw[v * 256 + 4 + (j >> 1)] >> sh) & 0xFFFFu;
+                const uint32_t rx = (reinterpret_cast<const uint32_t*>(s_raw + (2 * v) * 32)[j >> 1] >> sh) & 0xFFFFu;
+                const uint32_t rb = (reinterpret_cast<const uint32_t*>(s_raw + (2 * v + 1) * 32)[j >> 1] >> sh) & 0xFFFFu;
                 *sp = make_uint2((uint32_t)(v * (32 * VEC) + lane * VEC + j), (rb << 16) | rx);
                 sp += 32;
             }

@@ -36,12 +36,17 @@ template <bool CK> __global__ void k_fix(Plan P);
 // apply: K = 1 (iso_apply.cu); K >= 2 with a compile-time bound KC >= K on
 // the expert count, and the Gram pass for any K (iso_merge.cu)
 template <typename XT, typename BT, bool CK, int KC> __global__ void k_apply(Plan P);
-template <typename XT, typename BT, bool CK, int KC> __global__ void k_merge(Plan P);
+// k_merge is compiled for TIES alone and for the other operators (ISO, whose
+// 1-D tensors take the plain average, and TA): TIES needs no coefficients
+enum MergeOpFamily : int { OPF_TIES = 0, OPF_OTHER = 1 };
+template <typename XT, typename BT, bool CK, int KC, int OPF> __global__ void k_merge(Plan P);
 template <typename XT, typename BT, bool CK, int KC> __global__ void k_gramk(Plan P);
 // k_merge: resident blocks of TPB threads per SM
-constexpr int merge_blocks_per_sm(int KC) { return KC >= 8 ? 1 : 2; }
+// (eight experts and the coefficient-carrying family need more registers: one block)
+constexpr int merge_blocks_per_sm(int KC, int OPF) { return (KC >= 8 && OPF != 0) ? 1 : 2; }
 // k_merge's dynamic shared memory (its per-warp staging ring)
-template <typename XT, typename BT, int KC> int merge_smem_bytes();
+template <typename XT, typename BT, int KC, int OPF> int merge_smem_bytes();
+template <typename XT, typename BT, int KC> int gram_smem_bytes();
 constexpr int gram_blocks_per_sm(int KC) { return KC >= 8 ? 1 : 2; }
 __global__ void k_solve(Plan P, int gram_mode);
 template <typename XT> __global__ void k_mask(Plan P, uint32_t* const* mptr);

@@ -370,7 +370,7 @@ __device__ __forceinline__ uint32_t clamp_bytes(long long avail, uint32_t cap) {
     return avail <= 0 ? 0u : (avail >= (long long)cap ? cap : (uint32_t)avail);
 }
 
-template <typename XT, typename BT, int KC>
+template <typename XT, typename BT, int KC, int BLK = 2>
 struct StageGeom {
     static constexpr int E = 16 / (int)sizeof(XT);          // entries per lane per step
     static constexpr int SPT = TILE / (32 * E);              // steps per tile
@@ -379,26 +379,38 @@ struct StageGeom {
     // up to four experts: about 108 KB per block, two blocks per SM; eight
     // experts: one block per SM (its registers hold the eight vectors of a
     // step without spilling) with about 216 KB, a deeper ring
-    static constexpr int BUDGET = merge_blocks_per_sm(KC) == 1 ? 221184 : 110592;
-    static constexpr int DMAX = merge_blocks_per_sm(KC) == 1 ? 6 : 4;
+    static constexpr int BUDGET = BLK == 1 ? 221184 : 110592;
+    static constexpr int DMAX = BLK == 1 ? 6 : 4;
     static constexpr int D0 = BUDGET / (WPB * BYTES);
     static constexpr int DEPTH = D0 < 2 ? 2 : (D0 > DMAX ? DMAX : D0);
     static constexpr int SMEM = WPB * DEPTH * BYTES;
 };
 
 // the tile a step belongs to and where its data comes from (issue side)
+template <int KC, bool SMEM_PTRS>
+struct IssueCursor;
+// the tensor's expert pointers in registers
 template <int KC>
-struct IssueCursor {
+struct IssueCursor<KC, false> {
     long long g = -1;        // tile of the cached tensor data
     int t = 0;
     long long t_end = 0, e0 = 0, n = 0;
-    const void** xs;         // the warp's copy of the tensor's KC expert pointers (shared memory)
+    const void* xs[KC];
+    const void* bp = nullptr;
+};
+// ... or in the warp's shared-memory copy (frees registers for two blocks per SM)
+template <int KC>
+struct IssueCursor<KC, true> {
+    long long g = -1;
+    int t = 0;
+    long long t_end = 0, e0 = 0, n = 0;
+    const void** xs;
     const void* bp = nullptr;
 };
 
 // copy step (g, s) of lane `lane` into stage `st` (shared-space address)
-template <typename XT, typename BT, int KC>
-__device__ __forceinline__ void issue_step(const Plan& P, int K, IssueCursor<KC>& ic, long long g, int s,
+template <typename XT, typename BT, int KC, bool SP>
+__device__ __forceinline__ void issue_step(const Plan& P, int K, IssueCursor<KC, SP>& ic, long long g, int s,
                                            uint32_t st, int lane) {
     using G = StageGeom<XT, BT, KC>;
     if (g != ic.g) {
@@ -411,7 +423,7 @@ __device__ __forceinline__ void issue_step(const Plan& P, int K, IssueCursor<KC>
             ic.bp = d.base;
 #pragma unroll
             for (int i = 0; i < KC; ++i) ic.xs[i] = (i < K) ? P.xptr[i * P.n_tensors + ic.t] : nullptr;
-            __syncwarp();
+            if (SP) __syncwarp();
         }
         ic.g = g;
         ic.e0 = (g - P.tens[ic.t].tile_base) * TILE;
@@ -467,9 +479,9 @@ __device__ __forceinline__ void read_step(const char* st, int K, int lane, Words
 
 // One warp per tile, a contiguous tile range per warp; every step staged
 // through shared memory (above).
-template <typename XT, typename BT, bool CK, int KC>
-__global__ void __launch_bounds__(TPB, merge_blocks_per_sm(KC)) k_merge(Plan P) {
-    using G = StageGeom<XT, BT, KC>;
+template <typename XT, typename BT, bool CK, int KC, int OPF>
+__global__ void __launch_bounds__(TPB, merge_blocks_per_sm(KC, OPF)) k_merge(Plan P) {
+    using G = StageGeom<XT, BT, KC, merge_blocks_per_sm(KC, OPF)>;
     constexpr int E = G::E;
     constexpr int SPT = G::SPT;
     constexpr int D = G::DEPTH;
@@ -481,12 +493,13 @@ __global__ void __launch_bounds__(TPB, merge_blocks_per_sm(KC)) k_merge(Plan P) 
     char* ring = s_stage + warp * D * G::BYTES;
     const uint32_t ring_s = (uint32_t)__cvta_generic_to_shared(ring);
     const long long NS = (wr.end - wr.beg) * SPT;
+    constexpr bool SP = merge_blocks_per_sm(KC, OPF) == 2 && KC >= 8;
     __shared__ const void* s_xs[WPB][KC];
-    IssueCursor<KC> ic;
-    ic.xs = s_xs[warp];
+    IssueCursor<KC, SP> ic;
+    if constexpr (SP) ic.xs = s_xs[warp];
 #pragma unroll
     for (int p = 0; p < D - 1; ++p) {
-        if (p < NS) issue_step<XT, BT, KC>(P, K, ic, wr.beg + p / SPT, p % SPT, ring_s + p * G::BYTES, lane);
+        if (p < NS) issue_step<XT, BT, KC, SP>(P, K, ic, wr.beg + p / SPT, p % SPT, ring_s + p * G::BYTES, lane);
         cp_async_commit();
     }
     int t = tensor_of_tile(P.tens, P.n_tensors, wr.beg);
@@ -516,9 +529,9 @@ __global__ void __launch_bounds__(TPB, merge_blocks_per_sm(KC)) k_merge(Plan P) 
             e0 = (g - dp->tile_base) * TILE;
             const long long e1 = (e0 + TILE < n) ? e0 + TILE : n;
 #pragma unroll
-            for (int q = 0; q < KC; ++q) cf[q] = mp.cf[q];
+            for (int q = 0; q < KC; ++q) cf[q] = (OPF == OPF_TIES) ? 0.0f : mp.cf[q];
             exact = tile_thresholds<KC>(mp, K, (uint32_t)e0, (uint32_t)e1, T);
-            opk = mp.opk;
+            opk = (OPF == OPF_TIES) ? (int)OPK_TIES : mp.opk;
             iso1d = mp.iso1d;
             op = dp->out;
         }
@@ -527,7 +540,7 @@ __global__ void __launch_bounds__(TPB, merge_blocks_per_sm(KC)) k_merge(Plan P) 
         Words<BT, E> b;
         read_step<XT, BT, KC>(ring + (int)(i % D) * G::BYTES, K, lane, x, b);
         const long long ni = i + D - 1;
-        if (ni < NS) issue_step<XT, BT, KC>(P, K, ic, wr.beg + ni / SPT, (int)(ni % SPT), ring_s + (int)(ni % D) * G::BYTES, lane);
+        if (ni < NS) issue_step<XT, BT, KC, SP>(P, K, ic, wr.beg + ni / SPT, (int)(ni % SPT), ring_s + (int)(ni % D) * G::BYTES, lane);
         cp_async_commit();
         const long long e = e0 + (long long)s * (32 * E) + lane * E;
         if (e >= n) continue;
@@ -563,7 +576,7 @@ __global__ void __launch_bounds__(TPB, merge_blocks_per_sm(KC)) k_merge(Plan P) 
 // the tensor.
 template <typename XT, typename BT, bool CK, int KC>
 __global__ void __launch_bounds__(TPB, gram_blocks_per_sm(KC)) k_gramk(Plan P) {
-    using G = StageGeom<XT, BT, KC>;
+    using G = StageGeom<XT, BT, KC, gram_blocks_per_sm(KC)>;
     constexpr int E = G::E;
     constexpr int SPT = G::SPT;
     constexpr int D = G::DEPTH;
@@ -580,12 +593,11 @@ __global__ void __launch_bounds__(TPB, gram_blocks_per_sm(KC)) k_gramk(Plan P) {
     char* ring = s_stage + warp * D * G::BYTES;
     const uint32_t ring_s = (uint32_t)__cvta_generic_to_shared(ring);
     const long long NS = (wr.end - wr.beg) * SPT;
-    __shared__ const void* s_xs[WPB][KC];
-    IssueCursor<KC> ic;
-    ic.xs = s_xs[warp];
+    constexpr bool SP = false;
+    IssueCursor<KC, SP> ic;
 #pragma unroll
     for (int p = 0; p < D - 1; ++p) {
-        if (p < NS) issue_step<XT, BT, KC>(P, K, ic, wr.beg + p / SPT, p % SPT, ring_s + p * G::BYTES, lane);
+        if (p < NS) issue_step<XT, BT, KC, SP>(P, K, ic, wr.beg + p / SPT, p % SPT, ring_s + p * G::BYTES, lane);
         cp_async_commit();
     }
     int t = tensor_of_tile(P.tens, P.n_tensors, wr.beg);
@@ -636,7 +648,7 @@ __global__ void __launch_bounds__(TPB, gram_blocks_per_sm(KC)) k_gramk(Plan P) {
         Words<BT, E> b;
         read_step<XT, BT, KC>(ring + (int)(i % D) * G::BYTES, K, lane, x, b);
         const long long ni = i + D - 1;
-        if (ni < NS) issue_step<XT, BT, KC>(P, K, ic, wr.beg + ni / SPT, (int)(ni % SPT), ring_s + (int)(ni % D) * G::BYTES, lane);
+        if (ni < NS) issue_step<XT, BT, KC, SP>(P, K, ic, wr.beg + ni / SPT, (int)(ni % SPT), ring_s + (int)(ni % D) * G::BYTES, lane);
         cp_async_commit();
         const long long e = e0 + (long long)s * (32 * E) + lane * E;
         if (active && e < n) {
@@ -692,23 +704,34 @@ __global__ void __launch_bounds__(TPB, gram_blocks_per_sm(KC)) k_gramk(Plan P) {
     flush(t);
 }
 
+template <typename XT, typename BT, int KC, int OPF>
+int merge_smem_bytes() { return StageGeom<XT, BT, KC, merge_blocks_per_sm(KC, OPF)>::SMEM; }
 template <typename XT, typename BT, int KC>
-int merge_smem_bytes() { return StageGeom<XT, BT, KC>::SMEM; }
+int gram_smem_bytes() { return StageGeom<XT, BT, KC, gram_blocks_per_sm(KC)>::SMEM; }
 
 #define ISO_MERGE_SMEM(XT, BT)                                                 \
-    template int merge_smem_bytes<XT, BT, 1>();                               \
-    template int merge_smem_bytes<XT, BT, 2>();                               \
-    template int merge_smem_bytes<XT, BT, 4>();                               \
-    template int merge_smem_bytes<XT, BT, 8>();
+    template int merge_smem_bytes<XT, BT, 2, OPF_TIES>();                     \
+    template int merge_smem_bytes<XT, BT, 4, OPF_TIES>();                     \
+    template int merge_smem_bytes<XT, BT, 8, OPF_TIES>();                     \
+    template int merge_smem_bytes<XT, BT, 2, OPF_OTHER>();                    \
+    template int merge_smem_bytes<XT, BT, 4, OPF_OTHER>();                    \
+    template int merge_smem_bytes<XT, BT, 8, OPF_OTHER>();                    \
+    template int gram_smem_bytes<XT, BT, 1>();                                \
+    template int gram_smem_bytes<XT, BT, 2>();                                \
+    template int gram_smem_bytes<XT, BT, 4>();                                \
+    template int gram_smem_bytes<XT, BT, 8>();
 ISO_MERGE_SMEM(__nv_bfloat16, __nv_bfloat16)
 ISO_MERGE_SMEM(__nv_bfloat16, float)
 ISO_MERGE_SMEM(float, __nv_bfloat16)
 ISO_MERGE_SMEM(float, float)
 
 #define ISO_MERGE_INST(XT, BT, CK)                                             \
-    template __global__ void k_merge<XT, BT, CK, 2>(Plan);                    \
-    template __global__ void k_merge<XT, BT, CK, 4>(Plan);                    \
-    template __global__ void k_merge<XT, BT, CK, 8>(Plan);                    \
+    template __global__ void k_merge<XT, BT, CK, 2, OPF_TIES>(Plan);          \
+    template __global__ void k_merge<XT, BT, CK, 4, OPF_TIES>(Plan);          \
+    template __global__ void k_merge<XT, BT, CK, 8, OPF_TIES>(Plan);          \
+    template __global__ void k_merge<XT, BT, CK, 2, OPF_OTHER>(Plan);         \
+    template __global__ void k_merge<XT, BT, CK, 4, OPF_OTHER>(Plan);         \
+    template __global__ void k_merge<XT, BT, CK, 8, OPF_OTHER>(Plan);         \
     template __global__ void k_gramk<XT, BT, CK, 1>(Plan);                    \
     template __global__ void k_gramk<XT, BT, CK, 2>(Plan);                    \
     template __global__ void k_gramk<XT, BT, CK, 4>(Plan);                    \

@@ -166,7 +166,9 @@ __global__ void __launch_bounds__(SAMPLE_TPB) k_sample(Plan P) {
         const void* b = P.tens[t].base;
         const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nw = blockDim.x >> 5;
         for (int c = warp; c < nch; c += nw) {
-            const long long start = ((long long)((double)(n - SAMPLE_CHUNK) * c / (nch - 1))) & ~7LL;
+            // (n - 256) c / 95, rounded down (exact: integer arithmetic)
+            const long long start = (long long)(((unsigned long long)(n - SAMPLE_CHUNK) * (unsigned long long)c) /
+                                               (unsigned long long)(nch - 1)) & ~7LL;
             float tau[VEC];
             TauSrc<XT, BT, CKPT>::load8(x, b, start + lane * VEC, n, tau);
 #pragma unroll
@@ -202,11 +204,19 @@ __global__ void __launch_bounds__(SAMPLE_TPB) k_sample(Plan P) {
         block_kth_largest2(s_keys, S, U.k, U.k, s_ha, s_hb, s_scan, &s_bin, &s_above, &hi, &lo);
         that = hi;
     } else {
-        const double q = (double)U.k / (double)n;
-        const double r = (double)U.k * (double)S / (double)n;
-        const double delta = SAMPLE_Z * sqrt((double)S * q * (1.0 - q)) + 2.0;
-        const long long ra = (long long)floor(r - delta);
-        const long long rb = (long long)ceil(r + delta);
+        // the band's sample ranks, by one thread (binary64 is slow on this GPU)
+        __shared__ long long s_r[4];
+        if (threadIdx.x == 0) {
+            const double q = (double)U.k / (double)n;
+            const double r = (double)U.k * (double)S / (double)n;
+            const double delta = SAMPLE_Z * sqrt((double)S * q * (1.0 - q)) + 2.0;
+            s_r[0] = (long long)floor(r - delta);
+            s_r[1] = (long long)ceil(r + delta);
+            s_r[2] = (long long)floor(r + 0.5);
+            s_r[3] = (long long)floor(delta / 2.0);
+        }
+        __syncthreads();
+        const long long ra = s_r[0], rb = s_r[1];
         uint32_t ka, kb;
         block_kth_largest2(s_keys, S, ra >= 1 ? ra : 1, rb <= S ? rb : S, s_ha, s_hb, s_scan,
                            &s_bin, &s_above, &ka, &kb);
@@ -218,8 +228,8 @@ __global__ void __launch_bounds__(SAMPLE_TPB) k_sample(Plan P) {
             // most often in the sample -- a run of ties wider than a fifth
             // of the band is always among them.  The corrections are then
             // small whichever side of that run rank k falls on.
-            const long long rk = (long long)floor(r + 0.5);
-            const long long h = (long long)floor(delta / 2.0);
+            const long long rk = s_r[2];
+            const long long h = s_r[3];
             auto clampr = [&](long long x) { return x < 1 ? 1LL : (x > S ? (long long)S : x); };
             uint32_t pv[5];
             pv[0] = ka;
@@ -327,8 +337,13 @@ __global__ void __launch_bounds__(SAMPLE_TPB) k_sample(Plan P) {
             __syncthreads();
             // the chunk where the sampled ties reach the sampled need, one
             // thread per chunk (a scan over the chunks' tie counts)
-            const long long SX = whole ? n : (long long)CX * SAMPLE_CHUNK;
-            const double need_s = (double)U.k * (double)SX / (double)n - (double)s_cgt;
+            __shared__ double s_need;
+            if (threadIdx.x == 0) {
+                const long long SX = whole ? n : (long long)CX * SAMPLE_CHUNK;
+                s_need = (double)U.k * (double)SX / (double)n - (double)s_cgt;
+            }
+            __syncthreads();
+            const double need_s = s_need;
             const int c = threadIdx.x;
             const long long tcl = (c < CX) ? (long long)s_ties[c] : 0;
             long long tot_ties;
@@ -432,7 +447,7 @@ __global__ void __launch_bounds__(TPB, COUNT_BLOCKS_PER_SM) k_count(Plan P) {
     uint32_t* cseg = nullptr;                     // the unit's candidate segment
     uint32_t ch_pos = 0, ch_left = 0, cap = 0;
     bool ovf = false;
-    uint32_t lo = 0, hi = 0;
+    uint32_t lo = 0, hi = 0, span = 0;
     bool want_gamma = false;
 
     auto flush = [&]() {
@@ -464,6 +479,7 @@ __global__ void __launch_bounds__(TPB, COUNT_BLOCKS_PER_SM) k_count(Plan P) {
             au = rr.U;
             lo = au->lo;
             hi = au->hi;
+            span = hi - lo;
             want_gamma = au->want_gamma != 0;
             cap = (uint32_t)au->cand_cap;
             cseg = P.cand + au->cand_off;
@@ -493,7 +509,7 @@ __global__ void __launch_bounds__(TPB, COUNT_BLOCKS_PER_SM) k_count(Plan P) {
                     n_gt += gt;
                     f_gg = gt ? __fmaf_rn(tau[j], tau[j], f_gg) : f_gg;
                     *sp = kk;
-                    sp += ((kk >= lo) & !gt) ? 32 : 0;
+                    sp += (kk - lo <= span) ? 32 : 0;
                 }
             }
         } else {
