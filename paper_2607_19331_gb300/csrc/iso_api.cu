@@ -465,6 +465,10 @@ int run_group(const Call& c, int t0, int t1, char* ws, cudaStream_t s, const iso
     P.ckpt = c.ckpt ? 1 : 0;
     P.op = c.mask_only ? ISO_OP_TIES : c.op;
     P.fused = fused ? 1 : 0;
+    // BLOCK scope, one expert, TIES: the block kernel writes the outputs itself
+    const bool fuse_block = c.trims && !c.mask_only && K == 1 && c.topk.scope == ISO_SCOPE_BLOCK &&
+                            c.op == ISO_OP_TIES;
+    P.fuse_block = fuse_block ? 1 : 0;
     P.block_rows = c.topk.block_rows;
     P.block_cols = c.topk.block_cols;
     P.lambda = c.lambda;
@@ -597,6 +601,7 @@ int run_group(const Call& c, int t0, int t1, char* ws, cudaStream_t s, const iso
             ISO_TRY(smem_optin(k_merge<XT, BT, CK, KC, OPF_OTHER>, smem));
             return launch(KD_APPLY, s, [&] { k_merge<XT, BT, CK, KC, OPF_OTHER><<<mgrid, TPB, smem, s>>>(P); });
         };
+        if (K == 1 && fuse_block) return ISO_OK;
         if (K == 1) ISO_TRY(launch(KD_APPLY, s, [&] { k_apply<XT, BT, CK, 1><<<pgrid, TPB, 0, s>>>(P); }));
         else if (K == 2) ISO_TRY(merge(std::integral_constant<int, 2>{}));
         else if (K <= 4) ISO_TRY(merge(std::integral_constant<int, 4>{}));

@@ -43,7 +43,7 @@ __device__ void block_find_from_top_b(const uint32_t* hist, int nb, long long ra
 __device__ __forceinline__ int kpad(int q) { return q + (q >> 5); }
 
 template <typename XT, typename BT, bool CK>
-__global__ void __launch_bounds__(BLOCK_TPB) k_block_select(Plan P) {
+__global__ void __launch_bounds__(BLOCK_TPB, 1) k_block_select(Plan P) {
     extern __shared__ __align__(16) uint32_t s_keys[];      // kpad(BLOCK_MAX_ENTRIES)
     __shared__ uint32_t s_hist[RADIX_BINS];
     __shared__ long long s_scan[33];
@@ -79,11 +79,48 @@ __global__ void __launch_bounds__(BLOCK_TPB) k_block_select(Plan P) {
         s.ties_at_thresh = ties; s.ties_taken = need;
         P.st_units[(long long)i * P.st_units_stride + P.st_unit_base + u] = s;
     };
+    const void* x = P.xptr[i * P.n_tensors + t];
+    const bool vec = (w % VEC == 0) && (d.cols % VEC == 0) && (c0 % VEC == 0);
+    // fused K = 1 update (TIES / masked update): the block's outputs are
+    // written here, theta_0 + lambda tau for the kept entries, theta_0 else
+    const bool obf = sizeof(BT) == 2;
+    auto apply_block = [&](uint32_t tk, long long cut, bool keep_all) {
+        if (vec) {
+            const int w8 = (int)(w / VEC);
+            for (int q8 = threadIdx.x; q8 < n / VEC; q8 += blockDim.x) {
+                const int rr = q8 / w8, cc = (q8 - rr * w8) * VEC;
+                const long long e = (r0 + rr) * d.cols + c0 + cc;
+                float th0[VEC], tau[VEC], o[VEC];
+                load8_tail<BT>(d.base, e, d.numel, th0);
+                TauSrc<XT, BT, CK>::load8(x, d.base, e, d.numel, tau);
+#pragma unroll
+                for (int j = 0; j < VEC; ++j) {
+                    const uint32_t kk = key_of(tau[j]);
+                    const bool kept = keep_all || kk > tk || (kk == tk && e + j < cut);
+                    o[j] = kept ? out_of(th0[j], tau[j], P.lambda) : th0[j];
+                }
+                store8(d.out, e, d.numel, o, obf);
+            }
+        } else {
+            for (int q = threadIdx.x; q < n; q += blockDim.x) {
+                const int rr = q / (int)w, cc = q - rr * (int)w;
+                const long long e = (r0 + rr) * d.cols + c0 + cc;
+                const float th0 = Load8<BT>::one(d.base, e);
+                const float tau = TauSrc<XT, BT, CK>::load1(x, d.base, e);
+                const uint32_t kk = key_of(tau);
+                const bool kept = keep_all || kk > tk || (kk == tk && e < cut);
+                const float o = kept ? out_of(th0, tau, P.lambda) : th0;
+                if (obf) static_cast<__nv_bfloat16*>(d.out)[e] = __float2bfloat16_rn(o);
+                else static_cast<float*>(d.out)[e] = o;
+            }
+        }
+    };
     if (!(d.flags & TF_TRIM)) {
         if (threadIdx.x == 0) {
             U.state = ST_OFF; U.k = -1; U.t = 0; U.cut = CUT_ALL;
             stats(KEY_NONE, -1, 0, 0, 0);
         }
+        if (P.fuse_block) apply_block(0u, CUT_ALL, true);
         return;
     }
     const long long k = k_of_density_b(P.density, n);
@@ -92,15 +129,123 @@ __global__ void __launch_bounds__(BLOCK_TPB) k_block_select(Plan P) {
             U.state = ST_NONE; U.k = 0; U.t = KEY_NONE; U.cut = 0;
             stats(KEY_NONE, 0, 0, 0, 0);
         }
+        if (P.fuse_block) apply_block(KEY_NONE, 0, false);
         return;
     }
-    const void* x = P.xptr[i * P.n_tensors + t];
+    const bool want_gamma = (P.op == ISO_OP_ISO) && (P.K == 1);
+
+    // Full block of BLOCK_TPB x 16 entries in rows of a multiple of 16: each
+    // thread holds 16 consecutive entries (block order) in registers, and the
+    // threshold is found bit by bit from the top: t is the largest key value v
+    // with #{key >= v} >= k, so a bit is kept when the block still counts k
+    // keys at or above the prefix with that bit set.  No atomics, no bank
+    // conflicts; one block sum per bit below the highest.
+    constexpr int BFE = BLOCK_MAX_ENTRIES / BLOCK_TPB;
+    if (n == BLOCK_TPB * BFE && w % BFE == 0 && (d.cols % VEC) == 0 && (c0 % VEC) == 0 &&
+        blockDim.x == BLOCK_TPB) {
+        const int tq = threadIdx.x * BFE;
+        const int rr = tq / (int)w, cc = tq - rr * (int)w;
+        const long long ea = (r0 + rr) * d.cols + c0 + cc;     // tensor position of the thread's first entry
+        float tau[BFE];
+#pragma unroll
+        for (int g = 0; g < BFE / VEC; ++g) {
+            float t8[VEC];
+            TauSrc<XT, BT, CK>::load8(x, d.base, ea + g * VEC, d.numel, t8);
+#pragma unroll
+            for (int j = 0; j < VEC; ++j) tau[g * VEC + j] = t8[j];
+        }
+        uint32_t kmax = 0, kor = 0;
+#pragma unroll
+        for (int j = 0; j < BFE; ++j) { const uint32_t kk = key_of(tau[j]); kmax = max(kmax, kk); kor |= kk; }
+        if (kmax >= KEY_INF) set_status(P.hdr, ISO_ERR_NONFINITE);
+        kor = __reduce_or_sync(0xFFFFFFFFu, kor);
+        if (threadIdx.x == 0) s_or = 0;
+        __syncthreads();
+        if ((threadIdx.x & 31) == 0 && kor) atomicOr(&s_or, kor);
+        __syncthreads();
+        const int low = s_or ? __ffs(s_or) - 1 : 31;
+        const int top = s_or ? 31 - __clz(s_or) : 0;
+        // one barrier per bit: warp sums go to one of three counters; the
+        // counter of the bit after next is cleared meanwhile (its last reads
+        // were before this bit's barrier, its next adds come after the next one)
+        __shared__ uint32_t s_cnt[3];
+        if (threadIdx.x < 3) s_cnt[threadIdx.x] = 0;
+        __syncthreads();
+        uint32_t prefix = 0;
+        int cur = 0;
+        for (int bit = top; bit >= low; --bit) {
+            const uint32_t cand = prefix | (1u << bit);
+            uint32_t c = 0;
+#pragma unroll
+            for (int j = 0; j < BFE; ++j) c += key_of(tau[j]) >= cand;
+            c = __reduce_add_sync(0xFFFFFFFFu, c);
+            if ((threadIdx.x & 31) == 0 && c) atomicAdd(&s_cnt[cur], c);
+            __syncthreads();
+            if ((long long)s_cnt[cur] >= k) prefix = cand;
+            const int nxt2 = (cur + 2) % 3;
+            if (threadIdx.x == 0) s_cnt[nxt2] = 0;
+            cur = (cur + 1) % 3;
+        }
+        const uint32_t tk = prefix;
+        uint32_t above = 0, ties = 0;
+#pragma unroll
+        for (int j = 0; j < BFE; ++j) { const uint32_t kk = key_of(tau[j]); above += kk > tk; ties += kk == tk; }
+        uint32_t tot_ties;
+        const uint32_t ties_before = block_excl_scan(ties, s_scan32, &tot_ties);
+        const uint32_t tot_above = block_sum(above, s_scan32);
+        const long long need = k - (long long)tot_above;
+        if (threadIdx.x == 0) s_cutq = CUT_ALL;
+        __syncthreads();
+        if (need < (long long)tot_ties && (long long)ties_before < need && need <= (long long)(ties_before + ties)) {
+            uint32_t acc = ties_before;
+#pragma unroll
+            for (int j = 0; j < BFE; ++j)
+                if (key_of(tau[j]) == tk && (long long)(++acc) == need) s_cutq = ea + j + 1;
+        }
+        double g = 0.0;
+        if (want_gamma) {
+            // squares of the entries above t as binary32 two-sum pairs, then binary64 over the block
+            float sg = 0.0f, eg = 0.0f;
+#pragma unroll
+            for (int j = 0; j < BFE; ++j)
+                if (key_of(tau[j]) > tk) two_sum_add(sg, eg, __fmul_rn(tau[j], tau[j]));
+            g = block_sum((double)sg + (double)eg, s_dred);
+        }
+        __syncthreads();
+        const long long cut = s_cutq;
+        if (threadIdx.x == 0) {
+            U.n = n; U.k = k; U.t = tk; U.cut = cut;
+            U.count_above = tot_above; U.ties = tot_ties; U.need = need;
+            U.state = ST_DONE;
+            if (want_gamma) {
+                const double ft = (double)__uint_as_float(tk);
+                atomicAdd(&P.gram[t], g + (double)need * ft * ft);
+            }
+            stats(tk, k, tot_above, tot_ties, need);
+        }
+        if (P.fuse_block) {
+#pragma unroll
+            for (int gq = 0; gq < BFE / VEC; ++gq) {
+                const long long e = ea + gq * VEC;
+                float th0[VEC], o[VEC];
+                load8_tail<BT>(d.base, e, d.numel, th0);
+#pragma unroll
+                for (int j = 0; j < VEC; ++j) {
+                    const float tv = tau[gq * VEC + j];
+                    const uint32_t kk = key_of(tv);
+                    const bool kept = kk > tk || (kk == tk && e + j < cut);
+                    o[j] = kept ? out_of(th0[j], tv, P.lambda) : th0[j];
+                }
+                store8(d.out, e, d.numel, o, obf);
+            }
+        }
+        return;
+    }
     // keys in block order (row-major inside the block)
     bool bad = false;
     uint32_t kor = 0;                        // OR of the keys: trailing zero bits need no radix level
     if (threadIdx.x == 0) s_or = 0;
     __syncthreads();
-    const bool vec = (w % VEC == 0) && (d.cols % VEC == 0) && (c0 % VEC == 0);
     if (vec) {
         const int w8 = (int)(w / VEC);
         for (int q8 = threadIdx.x; q8 < n / VEC; q8 += blockDim.x) {
@@ -158,7 +303,6 @@ __global__ void __launch_bounds__(BLOCK_TPB) k_block_select(Plan P) {
     // counts above / at the threshold, and the squared norm of the kept entries
     const int per = (n + blockDim.x - 1) / blockDim.x;
     const int q0 = threadIdx.x * per;
-    const bool want_gamma = (P.op == ISO_OP_ISO) && (P.K == 1);
     uint32_t above = 0, ties = 0;
     double gsum = 0.0;
     for (int q = q0; q < q0 + per && q < n; ++q) {
@@ -186,12 +330,12 @@ __global__ void __launch_bounds__(BLOCK_TPB) k_block_select(Plan P) {
     __syncthreads();
     double g = 0.0;
     if (want_gamma) g = block_sum(gsum, s_dred);
+    long long cut = CUT_ALL;
+    if (s_cutq >= 0) {
+        const long long rr = s_cutq / w, cc = s_cutq - rr * w;
+        cut = (r0 + rr) * d.cols + c0 + cc + 1;
+    }
     if (threadIdx.x == 0) {
-        long long cut = CUT_ALL;
-        if (s_cutq >= 0) {
-            const long long rr = s_cutq / w, cc = s_cutq - rr * w;
-            cut = (r0 + rr) * d.cols + c0 + cc + 1;
-        }
         U.n = n; U.k = k; U.t = tk; U.cut = cut;
         U.count_above = tot_above; U.ties = tot_ties; U.need = need;
         U.state = ST_DONE;
@@ -201,6 +345,7 @@ __global__ void __launch_bounds__(BLOCK_TPB) k_block_select(Plan P) {
         }
         stats(tk, k, tot_above, tot_ties, need);
     }
+    if (P.fuse_block) apply_block(tk, cut, false);
 }
 
 #define ISO_BLOCK_INST(XT, BT, CK) template __global__ void k_block_select<XT, BT, CK>(Plan);

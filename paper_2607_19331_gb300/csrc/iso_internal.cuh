@@ -173,6 +173,7 @@ struct Plan {
     int32_t ckpt;           // experts are checkpoints (tau = x - base)
     int32_t op;
     int32_t fused;          // the K = 1 update runs the fused single pass
+    int32_t fuse_block;     // BLOCK scope, K = 1 TIES: k_block_select writes the outputs
     int32_t block_rows, block_cols;
     float lambda;
     double density, ridge, c_min, c_max;

@@ -21,7 +21,7 @@ template <typename XT, typename BT, bool CK> __global__ void k_tie(Plan P);
 template <typename XT, typename BT, bool CK> __global__ void k_cut(Plan P);
 
 // select (BLOCK scope)
-constexpr int BLOCK_TPB = 512;
+constexpr int BLOCK_TPB = 1024;
 template <typename XT, typename BT, bool CK> __global__ void k_block_select(Plan P);
 
 // fused K = 1 pass (bf16 base and update)
