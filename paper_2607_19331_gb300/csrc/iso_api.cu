@@ -120,6 +120,26 @@ int smem_optin(K kernel, int bytes) {
     return ISO_OK;
 }
 
+// A grid of exactly the blocks that are resident at once (one wave), for
+// latency-bound kernels that split their work evenly over the warps.
+template <typename K>
+int resident_grid(K kernel, int tpb, int smem, int sms, int* grid) {
+    int d = 0;
+    if (cudaGetDevice(&d) != cudaSuccess) return ISO_ERR_CUDA;
+    static std::mutex mu;
+    static std::unordered_map<long long, int> per_sm;
+    const long long key = ((long long)d << 48) ^ (long long)(uintptr_t)(const void*)kernel;
+    std::lock_guard<std::mutex> lk(mu);
+    auto it = per_sm.find(key);
+    if (it == per_sm.end()) {
+        int b = 0;
+        if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&b, kernel, tpb, smem) != cudaSuccess) return ISO_ERR_CUDA;
+        it = per_sm.emplace(key, b < 1 ? 1 : b).first;
+    }
+    *grid = sms * it->second;
+    return ISO_OK;
+}
+
 // ---------------------------------------------------------------------------
 // validation
 // ---------------------------------------------------------------------------
@@ -250,7 +270,7 @@ size_t al256(size_t v) { return (v + 255) & ~(size_t)255; }
 struct Layout {
     size_t hdr, units, tcand, teq_lo, teq_hi, tcnt, hist, hmxc, hmx, gram, coef, zero_end;
     size_t tens, xptr, mptr, table_end;
-    size_t tband, repair, cand, brec, total;
+    size_t tband, repair, csamp, cand, brec, total;
     unsigned long long brec_total = 0;
     long long n_tiles = 0;
     int n_units = 0;
@@ -310,6 +330,7 @@ Layout layout_of(const Call& c, int t0, int t1) {
     L.table_end = o;
     L.tband = o;  o = al256(o + (fused ? (size_t)tiles * 8 : 0));
     L.repair = o; o = al256(o + (fused ? (size_t)T * 4 : 0));
+    L.csamp = o;  o = al256(o + (fused ? (size_t)K * units * COUNT_CHUNKS * 4 : 0));
     L.cand = o;   o = al256(o + (size_t)L.cand_total * 4);
     L.brec = o;   o = al256(o + (size_t)L.brec_total * 8);
     L.total = o;
@@ -453,6 +474,7 @@ int run_group(const Call& c, int t0, int t1, char* ws, cudaStream_t s, const iso
     P.brec = reinterpret_cast<uint2*>(ws + L.brec);
     P.tband = reinterpret_cast<uint2*>(ws + L.tband);
     P.repair = fused ? reinterpret_cast<int32_t*>(ws + L.repair) : nullptr;
+    P.csamp = fused ? reinterpret_cast<uint32_t*>(ws + L.csamp) : nullptr;
     P.gram = reinterpret_cast<double*>(ws + L.gram);
     P.coef = reinterpret_cast<double*>(ws + L.coef);
     P.n_tensors = T;
@@ -505,9 +527,11 @@ int run_group(const Call& c, int t0, int t1, char* ws, cudaStream_t s, const iso
             using XT = std::remove_pointer_t<decltype(xt)>;
             using BT = std::remove_pointer_t<decltype(bt)>;
             constexpr bool CK = decltype(ck)::value;
-            const int smem = (SAMPLE_MAX + 2 * RADIX_BINS) * 4;
+            const int smem = (SAMPLE_MAX + SAMPLE_SEL_R * 256) * 4;
             ISO_TRY(smem_optin(k_sample<XT, BT, CK>, smem));
             ISO_TRY(launch(KD_SAMPLE, s, [&] { k_sample<XT, BT, CK><<<KU, SAMPLE_TPB, smem, s>>>(P); }));
+            if (fused)
+                ISO_TRY(launch(KD_SAMPLE, s, [&] { k_csample<XT, BT, CK><<<KU * CS_SPLIT, CS_TPB, 0, s>>>(P); }));
             if (fused) {
                 if (CK) {
                     ISO_TRY(smem_optin(k_count_apply<true>, FUSED_SMEM));
@@ -525,7 +549,7 @@ int run_group(const Call& c, int t0, int t1, char* ws, cudaStream_t s, const iso
                 ISO_TRY(launch(KD_RADIX_PICK, s, [&] { k_radix_pick<<<KU, TPB, 0, s>>>(P); }));
             }
             ISO_TRY(launch(KD_TIE, s, [&] { k_tie<XT, BT, CK><<<pgrid, TPB, 0, s>>>(P); }));
-            ISO_TRY(launch(KD_CUT, s, [&] { k_cut<XT, BT, CK><<<KU, 1024, 0, s>>>(P); }));
+            ISO_TRY(launch(KD_CUT, s, [&] { k_cut<XT, BT, CK><<<KU, CUT_TPB, 0, s>>>(P); }));
             return ISO_OK;
         });
         ISO_TRY(rc);
@@ -557,12 +581,17 @@ int run_group(const Call& c, int t0, int t1, char* ws, cudaStream_t s, const iso
         // the full exact apply of any flagged tensor
         ISO_TRY(launch(KD_SOLVE, s, [&] { k_solve<<<(T + 127) / 128, 128, 0, s>>>(P, gram_mode); }));
         ISO_TRY(launch(KD_REPAIR, s, [&] { k_fix_plan<<<1, 1024, 0, s>>>(P); }));
+        int ggrid = 0, fgrid = 0;
         if (c.ckpt) {
-            ISO_TRY(launch(KD_PATCH, s, [&] { k_patch<true><<<pgrid, TPB, 0, s>>>(P); }));
-            ISO_TRY(launch(KD_REPAIR, s, [&] { k_fix<true><<<pgrid, TPB, 0, s>>>(P); }));
+            ISO_TRY(resident_grid(k_patch<true>, TPB, 0, sms, &ggrid));
+            ISO_TRY(resident_grid(k_fix<true>, TPB, 0, sms, &fgrid));
+            ISO_TRY(launch(KD_PATCH, s, [&] { k_patch<true><<<ggrid, TPB, 0, s>>>(P); }));
+            ISO_TRY(launch(KD_REPAIR, s, [&] { k_fix<true><<<fgrid, TPB, 0, s>>>(P); }));
         } else {
-            ISO_TRY(launch(KD_PATCH, s, [&] { k_patch<false><<<pgrid, TPB, 0, s>>>(P); }));
-            ISO_TRY(launch(KD_REPAIR, s, [&] { k_fix<false><<<pgrid, TPB, 0, s>>>(P); }));
+            ISO_TRY(resident_grid(k_patch<false>, TPB, 0, sms, &ggrid));
+            ISO_TRY(resident_grid(k_fix<false>, TPB, 0, sms, &fgrid));
+            ISO_TRY(launch(KD_PATCH, s, [&] { k_patch<false><<<ggrid, TPB, 0, s>>>(P); }));
+            ISO_TRY(launch(KD_REPAIR, s, [&] { k_fix<false><<<fgrid, TPB, 0, s>>>(P); }));
         }
         return ISO_OK;
     }

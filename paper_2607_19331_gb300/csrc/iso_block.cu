@@ -123,7 +123,11 @@ __global__ void __launch_bounds__(BLOCK_TPB, 1) k_block_select(Plan P) {
         if (P.fuse_block) apply_block(0u, CUT_ALL, true);
         return;
     }
-    const long long k = k_of_density_b(P.density, n);
+    // k in binary64 by one thread (binary64 is slow on this GPU), then shared
+    __shared__ long long s_k;
+    if (threadIdx.x == 0) s_k = k_of_density_b(P.density, n);
+    __syncthreads();
+    const long long k = s_k;
     if (k == 0) {
         if (threadIdx.x == 0) {
             U.state = ST_NONE; U.k = 0; U.t = KEY_NONE; U.cut = 0;

@@ -203,22 +203,32 @@ __global__ void __launch_bounds__(TPB, FUSED_BLOCKS_PER_SM) k_count_apply(Plan P
             for (int v = 0; v < WVEC; ++v) {
                 float th0[VEC], tau[VEC], o[VEC];
                 raw_to_f32<__nv_bfloat16>(rt.b[v], th0);
-                if (CK) rt.tau(v, tau); else raw_to_f32<__nv_bfloat16>(rt.x[v], tau);
+                raw_to_f32<__nv_bfloat16>(rt.x[v], tau);
+                if (CK) {
+#pragma unroll
+                    for (int j = 0; j < VEC; j += 2) sub_rn2(tau[j], tau[j + 1], tau[j], tau[j + 1], th0[j], th0[j + 1]);
+                }
                 // keep the step's raw words for the band entries, then reuse the registers
                 s_raw[(2 * v) * 32] = rt.x[v][0];
                 s_raw[(2 * v + 1) * 32] = rt.b[v][0];
                 if (more) rt.load_step(v, nxp, nbp, ne0, nrem, lane);
                 const uint32_t o8 = (uint32_t)(v * (32 * VEC) + lane * VEC);
 #pragma unroll
-                for (int j = 0; j < VEC; ++j) {
-                    const uint32_t kk = key_of(tau[j]);
-                    const bool gt = kk > hi, eq = kk == th;
-                    const bool kept = (int)kk > (int)T;
-                    n_gt += gt;
-                    n_eq += eq;
-                    if (gt) f_gg = __fmaf_rn(tau[j], tau[j], f_gg);
-                    if ((kk - lo <= span) & !eq) tbm |= 1u << (v * VEC + j);
-                    o[j] = __fadd_rn(th0[j], kept ? __fmul_rn(a, tau[j]) : -0.0f);
+                for (int j = 0; j < VEC; j += 2) {
+                    bool kept[2];
+#pragma unroll
+                    for (int h = 0; h < 2; ++h) {
+                        const uint32_t kk = key_of(tau[j + h]);
+                        const bool gt = kk > hi, eq = kk == th;
+                        kept[h] = (int)kk > (int)T;
+                        n_gt += gt;
+                        n_eq += eq;
+                        if (gt) f_gg = __fmaf_rn(tau[j + h], tau[j + h], f_gg);
+                        if ((kk - lo <= span) & !eq) tbm |= 1u << (v * VEC + j + h);
+                    }
+                    float m0, m1;
+                    mul_rn2(m0, m1, a, a, tau[j], tau[j + 1]);
+                    add_rn2(o[j], o[j + 1], th0[j], th0[j + 1], kept[0] ? m0 : -0.0f, kept[1] ? m1 : -0.0f);
                 }
                 store8(op, (long long)e0 + o8, n, o, true);
             }
@@ -366,17 +376,25 @@ __global__ void __launch_bounds__(TPB) k_patch(Plan P) {
             const uint32_t c32 = (cut >= 0xFFFFFFFFLL) ? 0xFFFFFFFFu : (uint32_t)cut;
             thr = ((unsigned long long)U->t << 32) | (uint32_t)~c32;
         }
-        // 32 tiles at a time, one per lane
+        // 32 tiles at a time, one per lane; a lane's records eight at a time,
+        // their loads in flight together
         const uint32_t nt = min(32u, min(run_end, end) - it);
-        const uint2 r = (lane < (int)nt) ? P.tband[it + lane] : make_uint2(0u, 0u);
-        for (uint32_t q = 0; q < r.y; ++q) {
-            const uint2 rec = bseg[r.x + q];
-            const float xv = __uint_as_float(rec.y << 16);
-            const float bv = __uint_as_float(rec.y & 0xFFFF0000u);
-            const float tau = CK ? __fsub_rn(xv, bv) : xv;
-            const uint32_t kk = key_of(tau);
-            const bool kept = (((unsigned long long)kk << 32) | (uint32_t)~rec.x) > thr;
-            if (kept != (kk > th)) op[rec.x] = __float2bfloat16_rn(kept ? out_of(bv, tau, a) : bv);
+        const uint2 r = (lane < (int)nt) ? __ldg(&P.tband[it + lane]) : make_uint2(0u, 0u);
+        for (uint32_t q0 = 0; q0 < r.y; q0 += 8) {
+            uint2 rec[8];
+#pragma unroll
+            for (int u = 0; u < 8; ++u)
+                rec[u] = (q0 + u < r.y) ? __ldg(&bseg[r.x + q0 + u]) : make_uint2(0u, 0u);
+#pragma unroll
+            for (int u = 0; u < 8; ++u) {
+                if (q0 + u >= r.y) break;
+                const float xv = __uint_as_float(rec[u].y << 16);
+                const float bv = __uint_as_float(rec[u].y & 0xFFFF0000u);
+                const float tau = CK ? __fsub_rn(xv, bv) : xv;
+                const uint32_t kk = key_of(tau);
+                const bool kept = (((unsigned long long)kk << 32) | (uint32_t)~rec[u].x) > thr;
+                if (kept != (kk > th)) op[rec[u].x] = __float2bfloat16_rn(kept ? out_of(bv, tau, a) : bv);
+            }
         }
         it += nt;
     }
@@ -432,6 +450,24 @@ __global__ void __launch_bounds__(1024) k_fix_plan(Plan P) {
 // start when t > t^), the only entries the fused pass can have decided the
 // wrong way besides the recorded band entries.  The ranges' tiles are split
 // evenly over the warps.
+// flattened fix tiles [off, off + nt) of tensor t start at tensor tile g_lo
+struct FixRange {
+    int t;
+    long long off, nt, g_lo;
+    __device__ __forceinline__ void load(const Plan& P, int tt) {
+        t = tt;
+        const Unit& U = P.units[P.tens[tt].unit];
+        off = U.fix_off;
+        g_lo = U.fix0 / TILE;
+        nt = (U.fix1 > U.fix0) ? (U.fix1 + TILE - 1) / TILE - g_lo : 0;
+    }
+    // the range holding flattened tile f (>= off)
+    __device__ __forceinline__ void seek(const Plan& P, long long f) {
+        while (f >= off + nt) load(P, t + 1);
+    }
+    __device__ __forceinline__ uint32_t e0_of(long long f) const { return (uint32_t)(g_lo + (f - off)) * TILE; }
+};
+
 template <bool CK>
 __global__ void __launch_bounds__(TPB) k_fix(Plan P) {
     const int lane = threadIdx.x & 31;
@@ -441,56 +477,80 @@ __global__ void __launch_bounds__(TPB) k_fix(Plan P) {
     const long long per = (total + W - 1) / W;
     const long long fb = wid * per, fe = min(total, fb + per);
     if (fb >= fe) return;
-    // the unit holding flattened tile fb: last tensor with fix_off <= fb and tiles to fix
-    int t = 0;
+    // the tensor holding flattened tile fb: last tensor with fix_off <= fb
+    int t0 = 0;
     {
         int lo = 0, hi = P.n_tensors - 1;
         while (lo < hi) {
             const int mid = (lo + hi + 1) >> 1;
             if (P.units[P.tens[mid].unit].fix_off <= fb) lo = mid; else hi = mid - 1;
         }
-        t = lo;
+        t0 = lo;
     }
-    long long f = fb;
-    while (f < fe) {
-        const TensorDesc& d = P.tens[t];
-        const Unit& U = P.units[d.unit];
-        const long long r0 = U.fix0, r1 = U.fix1;
-        const long long g_lo = r0 / TILE, nt = (r1 > r0) ? (r1 + TILE - 1) / TILE - g_lo : 0;
-        if (f >= U.fix_off + nt) { ++t; continue; }
-        const bool all = P.repair[t] != 0;
-        const uint32_t n = (uint32_t)d.numel;
-        const uint32_t th = U.that;
-        const void* xp = P.xptr[t];
-        const void* bp = d.base;
-        __nv_bfloat16* q = static_cast<__nv_bfloat16*>(d.out);
-        const float a = (P.op == ISO_OP_ISO) ? (float)P.coef[t] : P.lambda;
-        const long long cut = U.cut;
-        const uint32_t c32 = (cut >= 0xFFFFFFFFLL) ? 0xFFFFFFFFu : (uint32_t)cut;
-        const unsigned long long thr = ((unsigned long long)U.t << 32) | (uint32_t)~c32;
-        const long long f_end = min(fe, U.fix_off + nt);
-        for (; f < f_end; ++f) {
-            const uint32_t e0 = (uint32_t)(g_lo + (f - U.fix_off)) * TILE;
-            RawTile<__nv_bfloat16, __nv_bfloat16, true> rt;
-            rt.load(xp, bp, e0, n, lane);
+    FixRange cur, nxt;          // the current tile's range, and the next tile's
+    cur.load(P, t0);
+    cur.seek(P, fb);
+    nxt = cur;
+    // the current range's parameters, reloaded when the range changes
+    int pt = -1;
+    long long r0 = 0, r1 = 0;
+    bool all = false;
+    uint32_t n = 0, th = 0;
+    __nv_bfloat16* q = nullptr;
+    float a = 0.0f;
+    unsigned long long thr = 0;
+    uint32_t e0 = cur.e0_of(fb);
+    RawTile<__nv_bfloat16, __nv_bfloat16, true> rt;   // x in rt.x, theta_0 in rt.b
 #pragma unroll
-            for (int v = 0; v < WVEC; ++v) {
-                const uint32_t e = e0 + v * (32 * VEC) + lane * VEC;
-                if (e >= n) continue;
-                float th0[VEC], tau[VEC];
-                raw_to_f32<__nv_bfloat16>(rt.b[v], th0);
-                if (CK) rt.tau(v, tau); else raw_to_f32<__nv_bfloat16>(rt.x[v], tau);
+    for (int v = 0; v < WVEC; ++v)
+        rt.load_step(v, P.xptr[cur.t], P.tens[cur.t].base, e0, (uint32_t)P.tens[cur.t].numel - e0, lane);
+    for (long long f = fb; f < fe; ++f) {
+        if (cur.t != pt) {
+            pt = cur.t;
+            const TensorDesc& d = P.tens[pt];
+            const Unit& U = P.units[d.unit];
+            r0 = U.fix0;
+            r1 = U.fix1;
+            all = P.repair[pt] != 0;
+            n = (uint32_t)d.numel;
+            th = U.that;
+            q = static_cast<__nv_bfloat16*>(d.out);
+            a = (P.op == ISO_OP_ISO) ? (float)P.coef[pt] : P.lambda;
+            const long long cut = U.cut;
+            const uint32_t c32 = (cut >= 0xFFFFFFFFLL) ? 0xFFFFFFFFu : (uint32_t)cut;
+            thr = ((unsigned long long)U.t << 32) | (uint32_t)~c32;
+        }
+        // the next tile's loads replace each step as it is consumed
+        const bool more = f + 1 < fe;
+        uint32_t ne0 = 0, nrem = 0;
+        const void* nxp = nullptr;
+        const void* nbp = nullptr;
+        if (more) {
+            nxt.seek(P, f + 1);
+            ne0 = nxt.e0_of(f + 1);
+            nxp = P.xptr[nxt.t];
+            nbp = P.tens[nxt.t].base;
+            nrem = (uint32_t)P.tens[nxt.t].numel - ne0;
+        }
 #pragma unroll
-                for (int j = 0; j < VEC; ++j) {
-                    const long long pos = (long long)e + j;
-                    const uint32_t kk = key_of(tau[j]);
-                    if (pos >= n || pos < r0 || pos >= r1 || !(all || kk == th)) continue;
-                    const unsigned long long kp = ((unsigned long long)kk << 32) | (uint32_t)~(uint32_t)pos;
-                    q[pos] = __float2bfloat16_rn((kp > thr) ? out_of(th0[j], tau[j], a) : th0[j]);
-                }
+        for (int v = 0; v < WVEC; ++v) {
+            const uint32_t e = e0 + v * (32 * VEC) + lane * VEC;
+            float th0[VEC], tau[VEC];
+            raw_to_f32<__nv_bfloat16>(rt.b[v], th0);
+            if (CK) rt.tau(v, tau); else raw_to_f32<__nv_bfloat16>(rt.x[v], tau);
+            if (more) rt.load_step(v, nxp, nbp, ne0, nrem, lane);
+            if (e >= n) continue;
+#pragma unroll
+            for (int j = 0; j < VEC; ++j) {
+                const long long pos = (long long)e + j;
+                const uint32_t kk = key_of(tau[j]);
+                if (pos >= n || pos < r0 || pos >= r1 || !(all || kk == th)) continue;
+                const unsigned long long kp = ((unsigned long long)kk << 32) | (uint32_t)~(uint32_t)pos;
+                q[pos] = __float2bfloat16_rn((kp > thr) ? out_of(th0[j], tau[j], a) : th0[j]);
             }
         }
-        ++t;
+        cur = nxt;
+        e0 = ne0;
     }
 }
 

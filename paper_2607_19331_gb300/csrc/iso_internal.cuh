@@ -32,7 +32,11 @@ constexpr int CHUNK_MAX = 1024;             // candidate slots a warp reserves a
 
 constexpr int SAMPLE_MAX = 24576;           // sampled keys per unit (96 KB of smem: two blocks per SM)
 constexpr int SAMPLE_CHUNK = 256;           // contiguous entries per sample chunk
-constexpr int SAMPLE_TPB = 1024;
+constexpr int SAMPLE_TPB = 512;             // two sample blocks per SM
+constexpr int SAMPLE_SEL_R = 5;             // ranks selected at once from the sample
+constexpr int CUT_TPB = 1024;
+constexpr int CS_SPLIT = 8;                 // count-sample blocks per unit
+constexpr int CS_TPB = 256;
 constexpr double SAMPLE_Z = 5.0;            // band half-width in sample standard deviations
 constexpr int COUNT_CHUNKS = 512;           // fused K = 1 pass: 256-entry chunks counted for the cut estimate
 
@@ -129,6 +133,9 @@ struct Unit {
     unsigned long long c_abv;           // candidates above t^
     long long fix0, fix1;               // positions k_fix re-applies (k_fix_plan)
     long long fix_off;                  // tiles to fix in the units before this one
+    unsigned long long cs_gt;           // count sample: keys above t^
+    uint32_t cs_done;                   // count-sample blocks finished
+    int32_t pad2;
 };
 
 // Per (expert, tile) records of the count pass, as separate arrays:
@@ -160,6 +167,7 @@ struct Plan {
     uint32_t*     cand;     // candidate pool
     uint2*        brec;     // fused K = 1 pass: band records (position, theta_0 bits << 16 | x bits)
     uint2*        tband;    // fused K = 1 pass: [n_tiles] (start, count) of the tile's band records
+    uint32_t*     csamp;    // fused K = 1 pass: [n_units][COUNT_CHUNKS] sampled ties of t^ per chunk
     int32_t*      repair;   // fused K = 1 pass: [n_tensors] tensor needs the full exact apply
     double*       gram;     // [n_tensors][K][K]
     double*       coef;     // [n_tensors][K]
@@ -572,6 +580,25 @@ __device__ __forceinline__ void store8(void* p, long long e, long long n, const 
 __device__ __forceinline__ float k1_spec_coef(const Plan& P) {
     if (P.op == ISO_OP_ISO) return (float)fmin(fmax(1.0, P.c_min), P.c_max);
     return P.lambda;
+}
+
+// Two binary32 operations in one packed instruction (sm_100 and later): each
+// half rounds to nearest like the scalar __fsub_rn / __fmul_rn / __fadd_rn,
+// subnormals kept.
+__device__ __forceinline__ void sub_rn2(float& d0, float& d1, float a0, float a1, float b0, float b1) {
+    asm("{\n\t.reg .b64 pa, pb, pd;\n\tmov.b64 pa, {%2, %3};\n\tmov.b64 pb, {%4, %5};\n\t"
+        "sub.rn.f32x2 pd, pa, pb;\n\tmov.b64 {%0, %1}, pd;\n\t}"
+        : "=f"(d0), "=f"(d1) : "f"(a0), "f"(a1), "f"(b0), "f"(b1));
+}
+__device__ __forceinline__ void mul_rn2(float& d0, float& d1, float a0, float a1, float b0, float b1) {
+    asm("{\n\t.reg .b64 pa, pb, pd;\n\tmov.b64 pa, {%2, %3};\n\tmov.b64 pb, {%4, %5};\n\t"
+        "mul.rn.f32x2 pd, pa, pb;\n\tmov.b64 {%0, %1}, pd;\n\t}"
+        : "=f"(d0), "=f"(d1) : "f"(a0), "f"(a1), "f"(b0), "f"(b1));
+}
+__device__ __forceinline__ void add_rn2(float& d0, float& d1, float a0, float a1, float b0, float b1) {
+    asm("{\n\t.reg .b64 pa, pb, pd;\n\tmov.b64 pa, {%2, %3};\n\tmov.b64 pb, {%4, %5};\n\t"
+        "add.rn.f32x2 pd, pa, pb;\n\tmov.b64 {%0, %1}, pd;\n\t}"
+        : "=f"(d0), "=f"(d1) : "f"(a0), "f"(a1), "f"(b0), "f"(b1));
 }
 
 __device__ __forceinline__ float out_of(float th0, float tau, float a) {

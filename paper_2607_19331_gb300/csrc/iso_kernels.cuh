@@ -17,6 +17,7 @@ template <typename XT, typename BT, bool CK> __global__ void k_count(Plan P);
 __global__ void k_decide(Plan P);
 template <typename XT, typename BT, bool CK> __global__ void k_radix_hist(Plan P);
 __global__ void k_radix_pick(Plan P);
+template <typename XT, typename BT, bool CK> __global__ void k_csample(Plan P);
 template <typename XT, typename BT, bool CK> __global__ void k_tie(Plan P);
 template <typename XT, typename BT, bool CK> __global__ void k_cut(Plan P);
 

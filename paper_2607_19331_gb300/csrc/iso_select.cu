@@ -95,38 +95,96 @@ __device__ void block_find_from_top(const uint32_t* hist, int nb, long long rank
     __syncthreads();
 }
 
-// The ra-th and rb-th largest (1-based) of n keys in shared memory, one
-// histogram pass per radix level for both ranks.
-__device__ void block_kth_largest2(const uint32_t* keys, int n, long long ra, long long rb,
-                                   uint32_t* ha, uint32_t* hb, long long* sm_scan, int* sm_bin,
-                                   long long* sm_above, uint32_t* ka, uint32_t* kb) {
-    uint32_t pa = 0, pb = 0;
-    int pshift = 31;
-    for (;;) {
-        const int shift = pshift > RADIX_BITS ? pshift - RADIX_BITS : 0;
-        const int nb = 1 << (pshift - shift);
-        for (int b = threadIdx.x; b < nb; b += blockDim.x) { ha[b] = 0; hb[b] = 0; }
-        __syncthreads();
-        for (int p = threadIdx.x; p < n; p += blockDim.x) {
-            const uint32_t v = keys[p];
-            const uint32_t top = v >> pshift, dig = (v >> shift) & (nb - 1);
-            if (top == pa) atomicAdd(&ha[dig], 1u);
-            if (top == pb) atomicAdd(&hb[dig], 1u);
+// The rank[r]-th largest (1-based, 1 <= rank[r] <= n) of n keys in shared
+// memory for R <= SEL_R ranks at once.  The key is found one 8-bit digit at
+// a time from the top; ranks whose prefixes agree share a histogram, so one
+// pass over the keys per digit serves every rank (at most one histogram bin
+// per key), and each histogram is scanned by one warp.  `hist` holds
+// SEL_R * 256 zeroed counters on entry and is zero again on return.
+constexpr int SEL_R = SAMPLE_SEL_R;
+__device__ void block_select_ranks(const uint32_t* keys, int n, int R, const long long* rank,
+                                   uint32_t* hist, uint32_t* out) {
+    __shared__ uint32_t s_pref[SEL_R];
+    __shared__ long long s_rem[SEL_R];
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    if (threadIdx.x < R) { s_pref[threadIdx.x] = 0; s_rem[threadIdx.x] = rank[threadIdx.x]; }
+    __syncthreads();
+#pragma unroll 1
+    for (int lvl = 0; lvl < 4; ++lvl) {
+        const int dsh = 24 - 8 * lvl;                    // the digit's shift
+        // distinct prefixes in rank order (every thread alike)
+        uint32_t gp[SEL_R];
+        int grp[SEL_R];
+        int ng = 0;
+#pragma unroll
+        for (int r = 0; r < SEL_R; ++r) {
+            gp[r] = 0;
+            grp[r] = -1;
+        }
+#pragma unroll
+        for (int r = 0; r < SEL_R; ++r) {
+            if (r < R) {
+                const uint32_t pr = s_pref[r];
+                int g = ng;
+#pragma unroll
+                for (int j = SEL_R - 1; j >= 0; --j)
+                    if (j < ng && gp[j] == pr) g = j;
+#pragma unroll
+                for (int j = 0; j < SEL_R; ++j)
+                    if (j == ng && g == ng) gp[j] = pr;
+                if (g == ng) ++ng;
+                grp[r] = g;
+            }
+        }
+        // one histogram per distinct prefix
+        for (int q = threadIdx.x; q < n; q += blockDim.x) {
+            const uint32_t v = keys[q];
+            const uint32_t top = lvl == 0 ? 0u : v >> (dsh + 8);
+            int g = -1;
+#pragma unroll
+            for (int j = SEL_R - 1; j >= 0; --j)
+                if (j < ng && gp[j] == top) g = j;
+            if (g >= 0) atomicAdd(&hist[(uint32_t)g * 256u + ((v >> dsh) & 255u)], 1u);
         }
         __syncthreads();
-        block_find_from_top(ha, nb, ra, sm_scan, sm_bin, sm_above);
-        ra -= *sm_above;
-        pa = (pa << (pshift - shift)) | (uint32_t)*sm_bin;
+        // warp g scans histogram g from the top bin: lane L holds bins 255-8L .. 248-8L
+        if (warp < ng) {
+            uint32_t h[8];
+            uint32_t* hg = hist + warp * 256;
+            uint32_t sum = 0;
+#pragma unroll
+            for (int j = 0; j < 8; ++j) { h[j] = hg[255 - 8 * lane - j]; sum += h[j]; }
+            uint32_t incl = sum;
+#pragma unroll
+            for (int o = 1; o < 32; o <<= 1) {
+                const uint32_t y = __shfl_up_sync(0xFFFFFFFFu, incl, o);
+                if (lane >= o) incl += y;
+            }
+            const long long excl = (long long)(incl - sum);
+#pragma unroll
+            for (int r = 0; r < SEL_R; ++r) {
+                if (r >= R || grp[r] != warp) continue;
+                const long long rr = s_rem[r];
+                if (excl < rr && rr <= excl + (long long)sum) {
+                    long long acc = excl;
+#pragma unroll
+                    for (int j = 0; j < 8; ++j) {
+                        if (rr <= acc + (long long)h[j]) {
+                            s_pref[r] = (s_pref[r] << 8) | (uint32_t)(255 - 8 * lane - j);
+                            s_rem[r] = rr - acc;
+                            break;
+                        }
+                        acc += h[j];
+                    }
+                }
+            }
+#pragma unroll
+            for (int j = 0; j < 8; ++j) hg[255 - 8 * lane - j] = 0;
+        }
         __syncthreads();
-        block_find_from_top(hb, nb, rb, sm_scan, sm_bin, sm_above);
-        rb -= *sm_above;
-        pb = (pb << (pshift - shift)) | (uint32_t)*sm_bin;
-        __syncthreads();
-        if (shift == 0) break;
-        pshift = shift;
     }
-    *ka = pa;
-    *kb = pb;
+    if (threadIdx.x < R) out[threadIdx.x] = s_pref[threadIdx.x];
+    __syncthreads();
 }
 
 // ---------------------------------------------------------------------------
@@ -144,20 +202,17 @@ __device__ __forceinline__ int tensor_of_upos(const TensorDesc* tens, int n_tens
 }
 
 template <typename XT, typename BT, bool CKPT>
-__global__ void __launch_bounds__(SAMPLE_TPB) k_sample(Plan P) {
+__global__ void __launch_bounds__(SAMPLE_TPB, 2) k_sample(Plan P) {
     extern __shared__ __align__(16) uint32_t s_keys[];
-    uint32_t* s_ha = s_keys + SAMPLE_MAX;
-    uint32_t* s_hb = s_ha + RADIX_BINS;
+    uint32_t* s_hist = s_keys + SAMPLE_MAX;          // SEL_R * 256 counters
     __shared__ long long s_scan[33];
-    __shared__ int s_bin;
-    __shared__ long long s_above;
 
     Unit& U = P.units[blockIdx.x];
     if (U.state != ST_SAMPLE) return;
     const int i = U.expert;
     const long long n = U.n;
     const int S = (int)(n < SAMPLE_MAX ? n : SAMPLE_MAX);
-    const int nch = SAMPLE_MAX / SAMPLE_CHUNK;
+    constexpr int nch = SAMPLE_MAX / SAMPLE_CHUNK;
     if (S < n && P.scope != ISO_SCOPE_GLOBAL) {
         // chunks of 256 contiguous entries at evenly spaced, 8-aligned starts:
         // one chunk per warp step, 8 entries per lane
@@ -165,14 +220,27 @@ __global__ void __launch_bounds__(SAMPLE_TPB) k_sample(Plan P) {
         const void* x = P.xptr[i * P.n_tensors + t];
         const void* b = P.tens[t].base;
         const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nw = blockDim.x >> 5;
-        for (int c = warp; c < nch; c += nw) {
-            // (n - 256) c / 95, rounded down (exact: integer arithmetic)
-            const long long start = (long long)(((unsigned long long)(n - SAMPLE_CHUNK) * (unsigned long long)c) /
-                                               (unsigned long long)(nch - 1)) & ~7LL;
-            float tau[VEC];
-            TauSrc<XT, BT, CKPT>::load8(x, b, start + lane * VEC, n, tau);
+        // three chunks per warp at a time: their loads are in flight together
+        constexpr int CB = 3;
+        for (int c0 = warp; c0 < nch; c0 += CB * nw) {
+            float tau[CB][VEC];
 #pragma unroll
-            for (int j = 0; j < VEC; ++j) s_keys[c * SAMPLE_CHUNK + lane * VEC + j] = key_of(tau[j]);
+            for (int m = 0; m < CB; ++m) {
+                const int c = c0 + m * nw;
+                // (n - 256) c / 95, rounded down (exact: integer arithmetic)
+                const long long start = (long long)(((unsigned long long)(n - SAMPLE_CHUNK) *
+                                                     (unsigned long long)(c < nch ? c : 0)) /
+                                                    (unsigned long long)(nch - 1)) & ~7LL;
+                TauSrc<XT, BT, CKPT>::load8(x, b, start + lane * VEC, n, tau[m]);
+            }
+#pragma unroll
+            for (int m = 0; m < CB; ++m) {
+                const int c = c0 + m * nw;
+                if (c < nch) {
+#pragma unroll
+                    for (int j = 0; j < VEC; ++j) s_keys[c * SAMPLE_CHUNK + lane * VEC + j] = key_of(tau[m][j]);
+                }
+            }
         }
     } else {
         for (int q = threadIdx.x; q < S; q += blockDim.x) {
@@ -181,7 +249,8 @@ __global__ void __launch_bounds__(SAMPLE_TPB) k_sample(Plan P) {
                 pos = q;
             } else {
                 const int c = q / SAMPLE_CHUNK, j = q % SAMPLE_CHUNK;
-                pos = (long long)((double)(n - SAMPLE_CHUNK) * c / (nch - 1)) + j;
+                pos = (long long)(((unsigned long long)(n - SAMPLE_CHUNK) * (unsigned long long)c) /
+                                  (unsigned long long)(nch - 1)) + j;
             }
             int t;
             long long e;
@@ -196,53 +265,55 @@ __global__ void __launch_bounds__(SAMPLE_TPB) k_sample(Plan P) {
             s_keys[q] = key_of(tau);
         }
     }
+    for (int q = threadIdx.x; q < SEL_R * 256; q += blockDim.x) s_hist[q] = 0;
     __syncthreads();
     uint32_t lo, hi;
     uint32_t that = 0;                       // fused pass: the estimate of the threshold
+    const bool fused_t = P.fused && P.scope == ISO_SCOPE_TENSOR;
+    __shared__ long long s_rk[SEL_R];
+    __shared__ uint32_t s_kv[SEL_R];
+    __shared__ int s_edge[2];
     if (S == n) {
         // the sample is the whole unit: the band is the exact threshold
-        block_kth_largest2(s_keys, S, U.k, U.k, s_ha, s_hb, s_scan, &s_bin, &s_above, &hi, &lo);
-        that = hi;
+        if (threadIdx.x == 0) s_rk[0] = U.k;
+        __syncthreads();
+        block_select_ranks(s_keys, S, 1, s_rk, s_hist, s_kv);
+        hi = lo = that = s_kv[0];
     } else {
-        // the band's sample ranks, by one thread (binary64 is slow on this GPU)
-        __shared__ long long s_r[4];
+        // the band's sample ranks, by one thread (binary64 is slow on this
+        // GPU), then every rank in one selection: the band edges and, for
+        // the fused pass, the rank of k and halfway to either edge
         if (threadIdx.x == 0) {
             const double q = (double)U.k / (double)n;
             const double r = (double)U.k * (double)S / (double)n;
             const double delta = SAMPLE_Z * sqrt((double)S * q * (1.0 - q)) + 2.0;
-            s_r[0] = (long long)floor(r - delta);
-            s_r[1] = (long long)ceil(r + delta);
-            s_r[2] = (long long)floor(r + 0.5);
-            s_r[3] = (long long)floor(delta / 2.0);
+            const long long ra = (long long)floor(r - delta), rb = (long long)ceil(r + delta);
+            const long long rk = (long long)floor(r + 0.5), h = (long long)floor(delta / 2.0);
+            auto clampr = [&](long long x) { return x < 1 ? 1LL : (x > S ? (long long)S : x); };
+            s_rk[0] = clampr(ra);
+            s_rk[1] = clampr(rb);
+            s_rk[2] = clampr(rk - h);
+            s_rk[3] = clampr(rk);
+            s_rk[4] = clampr(rk + h);
+            s_edge[0] = ra >= 1;
+            s_edge[1] = rb <= S;
         }
         __syncthreads();
-        const long long ra = s_r[0], rb = s_r[1];
-        uint32_t ka, kb;
-        block_kth_largest2(s_keys, S, ra >= 1 ? ra : 1, rb <= S ? rb : S, s_ha, s_hb, s_scan,
-                           &s_bin, &s_above, &ka, &kb);
-        hi = (ra >= 1) ? ka : KEY_MAX;
-        lo = (rb <= S) ? kb : 0u;
-        if (P.fused && P.scope == ISO_SCOPE_TENSOR) {
+        block_select_ranks(s_keys, S, fused_t ? 5 : 2, s_rk, s_hist, s_kv);
+        hi = s_edge[0] ? s_kv[0] : KEY_MAX;
+        lo = s_edge[1] ? s_kv[1] : 0u;
+        if (fused_t) {
             // t^: of the sampled keys at five ranks across the band (the band
             // edges, the rank of k and halfway between), the one that occurs
             // most often in the sample -- a run of ties wider than a fifth
             // of the band is always among them.  The corrections are then
             // small whichever side of that run rank k falls on.
-            const long long rk = s_r[2];
-            const long long h = s_r[3];
-            auto clampr = [&](long long x) { return x < 1 ? 1LL : (x > S ? (long long)S : x); };
             uint32_t pv[5];
-            pv[0] = ka;
-            pv[4] = kb;
-            block_kth_largest2(s_keys, S, clampr(rk - h), clampr(rk + h), s_ha, s_hb, s_scan, &s_bin, &s_above,
-                               &pv[1], &pv[3]);
-            if (pv[1] == pv[3]) {
-                pv[2] = pv[1];
-            } else {
-                uint32_t dummy;
-                block_kth_largest2(s_keys, S, clampr(rk), clampr(rk), s_ha, s_hb, s_scan, &s_bin, &s_above,
-                                   &pv[2], &dummy);
-            }
+            pv[0] = s_kv[0];
+            pv[1] = s_kv[2];
+            pv[2] = s_kv[3];
+            pv[3] = s_kv[4];
+            pv[4] = s_kv[1];
             unsigned cnt[5] = {0, 0, 0, 0, 0};
             for (int q = threadIdx.x; q < S; q += blockDim.x) {
                 const uint32_t v = s_keys[q];
@@ -274,19 +345,17 @@ __global__ void __launch_bounds__(SAMPLE_TPB) k_sample(Plan P) {
     }
     // Fused K = 1 pass: the estimate t^ of the threshold (the sample's key at
     // the rank of k; bf16-derived task vectors hold long runs of ties there)
-    // and of the position before which its ties are kept: exact when the
-    // sample is the whole unit, else interpolated from the sampled ties
-    // chunk by chunk.
+    // and of the position before which its ties are kept: exact here when
+    // the sample is the whole unit, else interpolated from a larger count
+    // sample by k_csample.
     long long chat = -1;
-    if (P.fused && P.scope == ISO_SCOPE_TENSOR) {
-        __shared__ unsigned long long s_cgt;
-        __shared__ unsigned s_ties[COUNT_CHUNKS];
+    if (fused_t) {
         __shared__ long long s_chat;
-        if (threadIdx.x == 0) { s_cgt = 0; s_chat = n; }
+        if (threadIdx.x == 0) s_chat = n;
         __syncthreads();
-        const uint32_t tk = that;
         if (S == n) {
             // keys in position order: the need-th tie
+            const uint32_t tk = that;
             const int per = (S + blockDim.x - 1) / blockDim.x;
             const int q0 = threadIdx.x * per;
             long long gt = 0, eq = 0;
@@ -301,61 +370,6 @@ __global__ void __launch_bounds__(SAMPLE_TPB) k_sample(Plan P) {
                     if (s_keys[q] == tk && ++acc == need) { s_chat = q + 1; break; }
             }
             __syncthreads();
-        } else {
-            // a larger count sample for the cut: CX chunks of 256 entries,
-            // contiguous when they cover the unit, else evenly spaced; per
-            // chunk the keys equal to t^, overall the keys above it
-            const long long nchunks = (n + SAMPLE_CHUNK - 1) / SAMPLE_CHUNK;
-            const bool whole = nchunks <= COUNT_CHUNKS;
-            const int CX = whole ? (int)nchunks : COUNT_CHUNKS;
-            auto chunk_start = [&](int c) -> long long {
-                if (whole) return (long long)c * SAMPLE_CHUNK;
-                return (long long)(((unsigned long long)(n - SAMPLE_CHUNK) * (unsigned long long)c) /
-                                   (unsigned long long)(CX - 1)) & ~7LL;
-            };
-            const int t = U.tensor;
-            const void* x = P.xptr[U.expert * P.n_tensors + t];
-            const void* b = P.tens[t].base;
-            const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nw = blockDim.x >> 5;
-            for (int c = warp; c < CX; c += nw) {
-                const long long st = chunk_start(c);
-                const long long e = st + lane * VEC;
-                float tau[VEC];
-                TauSrc<XT, BT, CKPT>::load8(x, b, e, n, tau);
-                unsigned gt = 0, eq = 0;
-#pragma unroll
-                for (int j = 0; j < VEC; ++j) {
-                    const uint32_t v = key_of(tau[j]);
-                    const bool in = e + j < n;
-                    gt += in && v > tk;
-                    eq += in && v == tk;
-                }
-                gt = __reduce_add_sync(0xFFFFFFFFu, gt);
-                eq = __reduce_add_sync(0xFFFFFFFFu, eq);
-                if (lane == 0) { s_ties[c] = eq; atomicAdd(&s_cgt, (unsigned long long)gt); }
-            }
-            __syncthreads();
-            // the chunk where the sampled ties reach the sampled need, one
-            // thread per chunk (a scan over the chunks' tie counts)
-            __shared__ double s_need;
-            if (threadIdx.x == 0) {
-                const long long SX = whole ? n : (long long)CX * SAMPLE_CHUNK;
-                s_need = (double)U.k * (double)SX / (double)n - (double)s_cgt;
-            }
-            __syncthreads();
-            const double need_s = s_need;
-            const int c = threadIdx.x;
-            const long long tcl = (c < CX) ? (long long)s_ties[c] : 0;
-            long long tot_ties;
-            const long long cum = block_excl_scan(tcl, s_scan, &tot_ties);
-            if (c < CX && tcl > 0 && (double)cum < need_s && need_s <= (double)(cum + tcl)) {
-                const long long a = chunk_start(c);
-                const long long bb = (c + 1 == CX) ? n : chunk_start(c + 1);
-                const long long ch = a + (long long)((need_s - (double)cum) / (double)tcl * (double)(bb - a));
-                s_chat = ch < 0 ? 0 : (ch > n ? n : ch);
-            }
-            if (c == 0 && need_s <= 0.0) s_chat = 0;
-            __syncthreads();
         }
         chat = s_chat;
     }
@@ -365,6 +379,125 @@ __global__ void __launch_bounds__(SAMPLE_TPB) k_sample(Plan P) {
         if (chat >= 0) { U.mode_t = 1; U.that = that; U.chat = chat; }
         U.state = ST_BAND;
     }
+}
+
+// Fused pass, units larger than the sample: the cut among the ties of t^
+// estimated from a count sample of up to COUNT_CHUNKS chunks of 256 entries
+// -- contiguous when they cover the unit (then the estimate is exact), else
+// evenly spaced -- counting per chunk the keys equal to t^ and overall the
+// keys above it.  CS_SPLIT blocks share a unit; the last of them to finish
+// finds the chunk where the sampled ties reach the sampled need and
+// interpolates inside it.
+template <typename XT, typename BT, bool CKPT>
+__global__ void __launch_bounds__(CS_TPB) k_csample(Plan P) {
+    const int u = blockIdx.x / CS_SPLIT, part = blockIdx.x % CS_SPLIT;
+    Unit& U = P.units[u];
+    // uniform over the unit's blocks: all of them return here, or none
+    if (U.state != ST_BAND || !U.mode_t || U.n <= SAMPLE_MAX) return;
+    const long long n = U.n;
+    const uint32_t tk = U.that;
+    const long long nchunks = (n + SAMPLE_CHUNK - 1) / SAMPLE_CHUNK;
+    const bool whole = nchunks <= COUNT_CHUNKS;
+    const int CX = whole ? (int)nchunks : COUNT_CHUNKS;
+    // (the divisor is a constant: no 64-bit division routine per chunk)
+    auto chunk_start = [&](int c) -> long long {
+        if (whole) return (long long)c * SAMPLE_CHUNK;
+        return (long long)(((unsigned long long)(n - SAMPLE_CHUNK) * (unsigned long long)c) /
+                           (unsigned long long)(COUNT_CHUNKS - 1)) & ~7LL;
+    };
+    uint32_t* ties = P.csamp + (size_t)u * COUNT_CHUNKS;
+    const int t = U.tensor;
+    const void* x = P.xptr[U.expert * P.n_tensors + t];
+    const void* b = P.tens[t].base;
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nw = blockDim.x >> 5;
+    constexpr int PER_PART = COUNT_CHUNKS / CS_SPLIT;
+    const int c_lo = part * PER_PART, c_hi = min(CX, c_lo + PER_PART);
+    // several chunks per warp at a time: their loads are in flight together
+    constexpr int CB = sizeof(XT) == 2 ? 4 : 2;
+    unsigned long long gt_w = 0;
+    for (int c0 = c_lo + warp; c0 < c_hi; c0 += CB * nw) {
+        float tau[CB][VEC];
+        long long ec[CB];
+#pragma unroll
+        for (int m = 0; m < CB; ++m) {
+            const int c = c0 + m * nw;
+            ec[m] = (c < c_hi) ? chunk_start(c) + lane * VEC : n;
+            TauSrc<XT, BT, CKPT>::load8(x, b, ec[m] < n ? ec[m] : 0, n, tau[m]);
+        }
+#pragma unroll
+        for (int m = 0; m < CB; ++m) {
+            const int c = c0 + m * nw;
+            unsigned gt = 0, eq = 0;
+#pragma unroll
+            for (int j = 0; j < VEC; ++j) {
+                const uint32_t v = key_of(tau[m][j]);
+                const bool in = ec[m] + j < n;
+                gt += in && v > tk;
+                eq += in && v == tk;
+            }
+            gt = __reduce_add_sync(0xFFFFFFFFu, gt);
+            eq = __reduce_add_sync(0xFFFFFFFFu, eq);
+            if (c < c_hi) {
+                if (lane == 0) ties[c] = eq;
+                gt_w += gt;
+            }
+        }
+    }
+    __shared__ unsigned long long s_gt;
+    __shared__ int s_last;
+    if (threadIdx.x == 0) s_gt = 0;
+    __syncthreads();
+    if (lane == 0 && gt_w) atomicAdd(&s_gt, gt_w);
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        if (s_gt) atomicAdd(&U.cs_gt, s_gt);
+        __threadfence();
+        s_last = atomicAdd(&U.cs_done, 1u) == (unsigned)(CS_SPLIT - 1);
+    }
+    __syncthreads();
+    if (!s_last) return;
+    __threadfence();
+    // the unit's last block: the sampled need, then the chunk where the
+    // sampled ties reach it (integer comparisons against ceil(need))
+    __shared__ double s_need;
+    __shared__ long long s_nc, s_chat;
+    __shared__ long long s_scan[33];
+    if (threadIdx.x == 0) {
+        const long long SX = whole ? n : (long long)CX * SAMPLE_CHUNK;
+        const unsigned long long cgt = atomicAdd(&U.cs_gt, 0ULL);
+        const double need = (double)U.k * (double)SX / (double)n - (double)cgt;
+        s_need = need;
+        s_nc = need <= 0.0 ? 0 : (long long)ceil(need);
+        s_chat = need <= 0.0 ? 0 : n;
+    }
+    __syncthreads();
+    const long long nc = s_nc;
+    constexpr int CPT = (COUNT_CHUNKS + CS_TPB - 1) / CS_TPB;   // chunks per thread
+    const int cb = threadIdx.x * CPT;
+    long long tcl[CPT];
+    long long local = 0;
+#pragma unroll
+    for (int j = 0; j < CPT; ++j) {
+        tcl[j] = (cb + j < CX) ? (long long)__ldcg(ties + cb + j) : 0;
+        local += tcl[j];
+    }
+    long long tot;
+    long long cum = block_excl_scan(local, s_scan, &tot);
+    if (nc > 0) {
+#pragma unroll
+        for (int j = 0; j < CPT; ++j) {
+            const int c = cb + j;
+            if (tcl[j] > 0 && cum < nc && nc <= cum + tcl[j]) {
+                const long long a0 = chunk_start(c);
+                const long long bb = (c + 1 == CX) ? n : chunk_start(c + 1);
+                const long long ch = a0 + (long long)((s_need - (double)cum) / (double)tcl[j] * (double)(bb - a0));
+                s_chat = ch < 0 ? 0 : (ch > n ? n : ch);
+            }
+            cum += tcl[j];
+        }
+    }
+    __syncthreads();
+    if (threadIdx.x == 0) U.chat = s_chat;
 }
 
 // ---------------------------------------------------------------------------
@@ -935,8 +1068,6 @@ __device__ __forceinline__ void write_unit_stats(const Plan& P, int idx, const U
     P.st_units[(long long)i * P.st_units_stride + P.st_unit_base + u] = s;
 }
 
-constexpr int CUT_TPB = 1024;
-
 template <typename XT, typename BT, bool CKPT>
 __global__ void __launch_bounds__(CUT_TPB) k_cut(Plan P) {
     __shared__ long long s_scan[33];
@@ -967,6 +1098,15 @@ __global__ void __launch_bounds__(CUT_TPB) k_cut(Plan P) {
             // 16-byte loads where the chunk allows
             long long g = j0;
             for (; g < j1 && ((uintptr_t)(src + g) & 15); ++g) local += src[g];
+            // eight 16-byte loads in flight at a time (a large unit gives a
+            // thread a hundred tiles and more)
+            for (; g + 32 <= j1; g += 32) {
+                uint4 v[8];
+#pragma unroll
+                for (int q = 0; q < 8; ++q) v[q] = *reinterpret_cast<const uint4*>(src + g + 4 * q);
+#pragma unroll
+                for (int q = 0; q < 8; ++q) local += (long long)v[q].x + v[q].y + v[q].z + v[q].w;
+            }
             for (; g + 4 <= j1; g += 4) {
                 const uint4 v = *reinterpret_cast<const uint4*>(src + g);
                 local += (long long)v.x + v.y + v.z + v.w;
@@ -1051,6 +1191,7 @@ __global__ void __launch_bounds__(CUT_TPB) k_cut(Plan P) {
 // ---------------------------------------------------------------------------
 #define ISO_SELECT_INST(XT, BT, CK)                                            \
     template __global__ void k_sample<XT, BT, CK>(Plan);                      \
+    template __global__ void k_csample<XT, BT, CK>(Plan);                     \
     template __global__ void k_count<XT, BT, CK>(Plan);                       \
     template __global__ void k_radix_hist<XT, BT, CK>(Plan);                  \
     template __global__ void k_tie<XT, BT, CK>(Plan);                         \
