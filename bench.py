@@ -64,7 +64,10 @@ def algorithmic_bytes(shapes, K, inputs, op, scope="tensor", two_pass=False):
     count:        (per-tensor scope) read the K task vectors once; in the fused
                   K = 1 pass this kernel is the whole update (read theta_0 and
                   the expert, write the output) and there is no apply pass
-    block_select: (per-block scope) read the K task vectors once
+    block_select: (per-block scope) read the K task vectors once; for the
+                  K = 1 TIES update this kernel writes the outputs itself (read
+                  theta_0 and the expert, write the output) and there is no
+                  apply pass
     gram:         (ISO, K >= 2) read the K task vectors once
     """
     n_all = sum(r * c for r, c, _ in shapes)
@@ -73,6 +76,8 @@ def algorithmic_bytes(shapes, K, inputs, op, scope="tensor", two_pass=False):
     per_base, per_out = 2, 2
     if fused_pass(K, inputs, op, scope, two_pass):
         return {"count": n_all * (per_base + per_x + per_out)}
+    if K == 1 and scope == "block" and op == "ties":
+        return {"block_select": n_all * (per_base + per_x + per_out)}
     read_tau = n_trim * (K * per_x + (per_base if inputs == "ckpt_bf16" else 0))
     out = {"apply": n_all * (per_base + K * per_x + per_out)}
     if op != "ta":

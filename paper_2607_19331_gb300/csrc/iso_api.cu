@@ -558,7 +558,7 @@ int run_group(const Call& c, int t0, int t1, char* ws, cudaStream_t s, const iso
             using XT = std::remove_pointer_t<decltype(xt)>;
             using BT = std::remove_pointer_t<decltype(bt)>;
             constexpr bool CK = decltype(ck)::value;
-            const int smem = (BLOCK_MAX_ENTRIES + BLOCK_MAX_ENTRIES / 32) * 4;
+            const int smem = BLOCK_KEYS_WORDS * 4;
             ISO_TRY(smem_optin(k_block_select<XT, BT, CK>, smem));
             if (KU > 0)
                 ISO_TRY(launch(KD_BLOCK_SELECT, s, [&] { k_block_select<XT, BT, CK><<<KU, BLOCK_TPB, smem, s>>>(P); }));

@@ -35,7 +35,7 @@ constexpr int SAMPLE_CHUNK = 256;           // contiguous entries per sample chu
 constexpr int SAMPLE_TPB = 512;             // two sample blocks per SM
 constexpr int SAMPLE_SEL_R = 5;             // ranks selected at once from the sample
 constexpr int CUT_TPB = 1024;
-constexpr int CS_SPLIT = 8;                 // count-sample blocks per unit
+constexpr int CS_SPLIT = 4;                 // count-sample blocks per unit
 constexpr int CS_TPB = 256;
 constexpr double SAMPLE_Z = 5.0;            // band half-width in sample standard deviations
 constexpr int COUNT_CHUNKS = 512;           // fused K = 1 pass: 256-entry chunks counted for the cut estimate
@@ -43,6 +43,7 @@ constexpr int COUNT_CHUNKS = 512;           // fused K = 1 pass: 256-entry chunk
 constexpr int RADIX_BITS = 11;
 constexpr int RADIX_BINS = 1 << RADIX_BITS;
 constexpr int BLOCK_MAX_ENTRIES = 16384;    // BLOCK scope: entries per unit held on chip
+constexpr int BLOCK_KEYS_WORDS = BLOCK_MAX_ENTRIES + BLOCK_MAX_ENTRIES / 32;   // padded key array
 
 constexpr int MAXK = ISO_MAX_EXPERTS;
 constexpr uint32_t KEY_NONE = 0xFFFFFFFFu;  // threshold of a unit that selects nothing

@@ -48,7 +48,7 @@ constexpr int merge_blocks_per_sm(int KC, int OPF) { return (KC >= 8 && OPF != 0
 // k_merge's dynamic shared memory (its per-warp staging ring)
 template <typename XT, typename BT, int KC, int OPF> int merge_smem_bytes();
 template <typename XT, typename BT, int KC> int gram_smem_bytes();
-constexpr int gram_blocks_per_sm(int KC) { return KC >= 8 ? 1 : 2; }
+constexpr int gram_blocks_per_sm(int KC) { return 2; }
 __global__ void k_solve(Plan P, int gram_mode);
 template <typename XT> __global__ void k_mask(Plan P, uint32_t* const* mptr);
 __global__ void k_status(const Header* h, int32_t* out);

@@ -593,8 +593,10 @@ __global__ void __launch_bounds__(TPB, gram_blocks_per_sm(KC)) k_gramk(Plan P) {
     char* ring = s_stage + warp * D * G::BYTES;
     const uint32_t ring_s = (uint32_t)__cvta_generic_to_shared(ring);
     const long long NS = (wr.end - wr.beg) * SPT;
-    constexpr bool SP = false;
+    constexpr bool SP = KC >= 8;   // eight experts: their pointers in shared memory (two blocks per SM)
     IssueCursor<KC, SP> ic;
+    __shared__ const void* s_xs[WPB][KC];
+    if constexpr (SP) ic.xs = s_xs[warp];
 #pragma unroll
     for (int p = 0; p < D - 1; ++p) {
         if (p < NS) issue_step<XT, BT, KC, SP>(P, K, ic, wr.beg + p / SPT, p % SPT, ring_s + p * G::BYTES, lane);
@@ -644,9 +646,22 @@ __global__ void __launch_bounds__(TPB, gram_blocks_per_sm(KC)) k_gramk(Plan P) {
             for (int q = 0; q < NP; ++q) acc[q] = 0.0f;
         }
         cp_async_wait<D - 2>();
-        Words<XT, E> x[KC];
-        Words<BT, E> b;
-        read_step<XT, BT, KC>(ring + (int)(i % D) * G::BYTES, K, lane, x, b);
+        // the step's words are read from the stage entry by entry (the stage is
+        // the lane's own and is refilled only after this step): fewer live
+        // registers than a whole step's words, two blocks per SM
+        const char* stg = ring + (int)(i % D) * G::BYTES;
+        auto xw = [&](int q, int j) -> float {
+            const char* p = stg + q * 512 + lane * 16;
+            if (sizeof(XT) == 4) return *reinterpret_cast<const float*>(p + 4 * j);
+            const uint32_t w = *reinterpret_cast<const uint32_t*>(p + 4 * (j >> 1));
+            return __uint_as_float((j & 1) ? (w & 0xFFFF0000u) : (w << 16));
+        };
+        auto bw = [&](int j) -> float {
+            const char* p = stg + KC * 512 + lane * G::BB;
+            if (sizeof(BT) == 4) return *reinterpret_cast<const float*>(p + 4 * j);
+            const uint32_t w = *reinterpret_cast<const uint32_t*>(p + 4 * (j >> 1));
+            return __uint_as_float((j & 1) ? (w & 0xFFFF0000u) : (w << 16));
+        };
         const long long ni = i + D - 1;
         if (ni < NS) issue_step<XT, BT, KC, SP>(P, K, ic, wr.beg + ni / SPT, (int)(ni % SPT), ring_s + (int)(ni % D) * G::BYTES, lane);
         cp_async_commit();
@@ -657,10 +672,10 @@ __global__ void __launch_bounds__(TPB, gram_blocks_per_sm(KC)) k_gramk(Plan P) {
 #pragma unroll
             for (int j = 0; j < E; ++j) {
                 float tau[KC];
-                const float th0 = CK ? word_f32<BT, E>(b, j) : 0.0f;
+                const float th0 = CK ? bw(j) : 0.0f;
 #pragma unroll
                 for (int q = 0; q < KC; ++q) {
-                    tau[q] = (q < K) ? word_f32<XT, E>(x[q], j) : 0.0f;
+                    tau[q] = (q < K) ? xw(q, j) : 0.0f;
                     if (CK) tau[q] = __fsub_rn(tau[q], th0);
                 }
                 float m[KC];

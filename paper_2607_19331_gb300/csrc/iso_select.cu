@@ -136,7 +136,9 @@ __device__ void block_select_ranks(const uint32_t* keys, int n, int R, const lon
                 grp[r] = g;
             }
         }
-        // one histogram per distinct prefix
+        // one histogram per distinct prefix; a thread's run of keys in one
+        // bin adds once (the keys near the threshold crowd into a few bins)
+        uint32_t run_slot = 0, run_cnt = 0;
         for (int q = threadIdx.x; q < n; q += blockDim.x) {
             const uint32_t v = keys[q];
             const uint32_t top = lvl == 0 ? 0u : v >> (dsh + 8);
@@ -144,8 +146,16 @@ __device__ void block_select_ranks(const uint32_t* keys, int n, int R, const lon
 #pragma unroll
             for (int j = SEL_R - 1; j >= 0; --j)
                 if (j < ng && gp[j] == top) g = j;
-            if (g >= 0) atomicAdd(&hist[(uint32_t)g * 256u + ((v >> dsh) & 255u)], 1u);
+            if (g < 0) continue;
+            const uint32_t slot = (uint32_t)g * 256u + ((v >> dsh) & 255u);
+            if (slot != run_slot) {
+                if (run_cnt) atomicAdd(&hist[run_slot], run_cnt);
+                run_slot = slot;
+                run_cnt = 0;
+            }
+            ++run_cnt;
         }
+        if (run_cnt) atomicAdd(&hist[run_slot], run_cnt);
         __syncthreads();
         // warp g scans histogram g from the top bin: lane L holds bins 255-8L .. 248-8L
         if (warp < ng) {
@@ -389,7 +399,7 @@ __global__ void __launch_bounds__(SAMPLE_TPB, 2) k_sample(Plan P) {
 // finds the chunk where the sampled ties reach the sampled need and
 // interpolates inside it.
 template <typename XT, typename BT, bool CKPT>
-__global__ void __launch_bounds__(CS_TPB) k_csample(Plan P) {
+__global__ void __launch_bounds__(CS_TPB, 4) k_csample(Plan P) {
     const int u = blockIdx.x / CS_SPLIT, part = blockIdx.x % CS_SPLIT;
     Unit& U = P.units[u];
     // uniform over the unit's blocks: all of them return here, or none

@@ -152,6 +152,23 @@ def test_update_checkpoint_bf16(scope, op):
     _check_merge(out, st, r, th0, OPS[op], 1, what=f"update {op} {scope}")
 
 
+@pytest.mark.parametrize("op", ["iso", "ties"])
+def test_block_update_many_full_units(op):
+    # more 128 x 128 units than SMs: each persistent block-select CTA walks
+    # several consecutive units, prefetching the next full unit, across tensor
+    # boundaries, partial edge units and a 1-D tensor
+    shapes = [(1024, 2048, False), (300, 1000, False), (2048, 1024, False), (1, 2048, True),
+              (640, 768, False)]
+    th0, th1 = synth.rl_update_set(shapes, seed=3)
+    d0, d1 = [t.to(DEV) for t in th0], [t.to(DEV) for t in th1]
+    out, st = iso.iso_update(d0, d1, op=op, update_is_delta=False, density=0.05, scope="block",
+                             lam=1.0, stats=True)
+    torch.cuda.synchronize()
+    r = oracle.update(_np_list(th0), _np_list(th1), OPS[op], update_is_delta=False, density=0.05,
+                      scope=oracle.SCOPE_BLOCK, lam=1.0, shapes=_shapes(shapes), is_1d=_is1d(shapes))
+    _check_merge(out, st, r, th0, OPS[op], 1, what=f"block update {op}")
+
+
 @pytest.mark.parametrize("op", ["ta", "ties", "iso"])
 def test_tiny_fp32_k2(op):
     # 1024 x 1024 fp32 base, K = 2 fp32 task vectors, density 10 %, lambda 1, seed 0
