@@ -44,7 +44,7 @@ template <typename XT, typename BT, bool CK, int KC, int OPF> __global__ void k_
 template <typename XT, typename BT, bool CK, int KC> __global__ void k_gramk(Plan P);
 // k_merge: resident blocks of TPB threads per SM
 // (eight experts and the coefficient-carrying family need more registers: one block)
-constexpr int merge_blocks_per_sm(int KC, int OPF) { return (KC >= 8 && OPF != 0) ? 1 : 2; }
+constexpr int merge_blocks_per_sm(int KC, int OPF) { return 2; }
 // k_merge's dynamic shared memory (its per-warp staging ring)
 template <typename XT, typename BT, int KC, int OPF> int merge_smem_bytes();
 template <typename XT, typename BT, int KC> int gram_smem_bytes();

@@ -536,9 +536,29 @@ __global__ void __launch_bounds__(TPB, merge_blocks_per_sm(KC, OPF)) k_merge(Pla
             op = dp->out;
         }
         cp_async_wait<D - 2>();
-        Words<XT, E> x[KC];
+        // eight experts: the step's words are read from the stage entry by
+        // entry (the stage is the lane's own and is refilled only after this
+        // step) -- fewer live registers, two blocks per SM without spills;
+        // fewer experts read the whole step at once
+        constexpr bool LAZY = KC >= 8;
+        Words<XT, E> x[LAZY ? 1 : KC];
         Words<BT, E> b;
-        read_step<XT, BT, KC>(ring + (int)(i % D) * G::BYTES, K, lane, x, b);
+        const char* stg = ring + (int)(i % D) * G::BYTES;
+        if constexpr (!LAZY) read_step<XT, BT, KC>(stg, K, lane, x, b);
+        auto xw = [&](int q, int j) -> float {
+            if constexpr (!LAZY) return word_f32<XT, E>(x[q], j);
+            const char* p = stg + q * 512 + lane * 16;
+            if (sizeof(XT) == 4) return *reinterpret_cast<const float*>(p + 4 * j);
+            const uint32_t w = *reinterpret_cast<const uint32_t*>(p + 4 * (j >> 1));
+            return __uint_as_float((j & 1) ? (w & 0xFFFF0000u) : (w << 16));
+        };
+        auto bw = [&](int j) -> float {
+            if constexpr (!LAZY) return word_f32<BT, E>(b, j);
+            const char* p = stg + KC * 512 + lane * G::BB;
+            if (sizeof(BT) == 4) return *reinterpret_cast<const float*>(p + 4 * j);
+            const uint32_t w = *reinterpret_cast<const uint32_t*>(p + 4 * (j >> 1));
+            return __uint_as_float((j & 1) ? (w & 0xFFFF0000u) : (w << 16));
+        };
         const long long ni = i + D - 1;
         if (ni < NS) issue_step<XT, BT, KC, SP>(P, K, ic, wr.beg + ni / SPT, (int)(ni % SPT), ring_s + (int)(ni % D) * G::BYTES, lane);
         cp_async_commit();
@@ -549,11 +569,11 @@ __global__ void __launch_bounds__(TPB, merge_blocks_per_sm(KC, OPF)) k_merge(Pla
         float o[E];
 #pragma unroll
         for (int j = 0; j < E; ++j) {
-            const float th0 = word_f32<BT, E>(b, j);
+            const float th0 = bw(j);
             float tau[KC];
 #pragma unroll
             for (int q = 0; q < KC; ++q) {
-                tau[q] = (q < K) ? word_f32<XT, E>(x[q], j) : 0.0f;
+                tau[q] = (q < K) ? xw(q, j) : 0.0f;
                 if (CK) tau[q] = __fsub_rn(tau[q], th0);
             }
             if (exact) {
