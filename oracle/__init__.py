@@ -11,6 +11,8 @@ unit, calls the C routines and scatters the results back.
 * TIES: sign election, agreeing set, disjoint mean, ``theta_0 + lambda tau``
                                                                    (App. F)
 * Task Arithmetic ``theta_0 + lambda sum_i tau_i``                 (App. F)
+* RAM: active set ``|tau_i| > eps_act``, unique values kept, shared ones
+  averaged over the active experts                                 (App. F)
 * ISO retention combiner (Gram, ridge solve, clip) applied to the trimmed
   task vectors, and the 1-D task-vector average    (Sec. 4.2, App. E, Alg. 1)
 
@@ -35,7 +37,7 @@ _SO = os.path.join(_BUILD, "liboracle.so")
 _SRC = os.path.join(_HERE, "iso_oracle.c")
 
 BF16, F32 = 0, 1
-TA, TIES, ISO = 0, 1, 2
+TA, TIES, ISO, RAM = 0, 1, 2, 3
 SCOPE_TENSOR, SCOPE_BLOCK, SCOPE_GLOBAL = 0, 1, 2
 
 KEY_NONE = 0xFFFFFFFF  # threshold key reported for a unit that selects nothing
@@ -85,6 +87,7 @@ def _lib():
             lib.orc_merge_tensor.argtypes = [i32, i32, i64, i32, P, P, P, P,
                                              f64, f64, f64, f64, P, P, P]
             lib.orc_retention.argtypes = [i32, P, f64, f64, f64, P]
+            lib.orc_merge_ram.argtypes = [i32, i64, P, P, P, f64, f64, P]
             lib.orc_f64_to_bf16.restype = ctypes.c_uint16
             lib.orc_f64_to_bf16.argtypes = [f64]
             lib.orc_f32_to_bf16.restype = ctypes.c_uint16
@@ -269,13 +272,17 @@ def retention(gram: np.ndarray, ridge=1e-12, c_min=0.0, c_max=1.5) -> np.ndarray
 
 def merge(theta0, experts, op, *, experts_are_deltas=True, density=0.2,
           scope=SCOPE_TENSOR, block=(128, 128), lam=1.0, ridge=1e-12, c_min=0.0,
-          c_max=1.5, mask_1d=True, shapes=None, is_1d=None, method="select"):
+          c_max=1.5, mask_1d=True, shapes=None, is_1d=None, method="select",
+          eps_act=1e-5):
     """Merge K experts into the base, tensor by tensor.
 
     theta0       list of base tensors (uint16 bfloat16 bits or float32)
     experts      list of K lists of tensors: task vectors (experts_are_deltas)
                  or fine-tuned checkpoints
-    op           TA / TIES / ISO
+    op           TA / TIES / ISO / RAM
+    eps_act      RAM activity threshold (the paper uses 1e-5); the library
+                 takes it as a binary32 value, so pass a value that float32
+                 represents (e.g. ``float(np.float32(1e-5))``) to compare
     shapes       list of (rows, cols); defaults to each array's 2-D shape
     is_1d        list of flags; defaults to rows == 1 for 1-row tensors
 
@@ -300,7 +307,7 @@ def merge(theta0, experts, op, *, experts_are_deltas=True, density=0.2,
             else:
                 tau32[i][t], tau64[i][t] = delta(experts[i][t], theta0[t])
 
-    if op == TA:
+    if op in (TA, RAM):
         participate = [False] * n_t
     elif op == TIES:
         participate = [True if mask_1d else not is_1d[t] for t in range(n_t)]
@@ -309,7 +316,7 @@ def merge(theta0, experts, op, *, experts_are_deltas=True, density=0.2,
 
     masks = [None] * K
     units = []
-    if op != TA:   # every trimming operator reports one row per unit (k = -1: not trimmed)
+    if op not in (TA, RAM):   # every trimming operator reports one row per unit (k = -1: not trimmed)
         for i in range(K):
             masks[i], st = topk_masks(tau32[i], shapes, density, scope, block, method, participate)
             units.append(st)
@@ -324,16 +331,19 @@ def merge(theta0, experts, op, *, experts_are_deltas=True, density=0.2,
         t64 = [np.ascontiguousarray(tau64[i][t]) for i in range(K)]
         P32 = (ctypes.c_void_p * K)(*[a.ctypes.data for a in t32])
         P64 = (ctypes.c_void_p * K)(*[a.ctypes.data for a in t64])
-        use_mask = participate[t] and op != TA
+        use_mask = participate[t] and op not in (TA, RAM)
         if use_mask:
             mk = [np.ascontiguousarray(masks[i][t]) for i in range(K)]
             PM = (ctypes.c_void_p * K)(*[a.ctypes.data for a in mk])
         else:
             mk = None
             PM = None
-        lib.orc_merge_tensor(op, K, n, int(bool(is_1d[t])), _ptr(th64), P32, P64, PM,
-                             float(lam), float(ridge), float(c_min), float(c_max),
-                             _ptr(o64), _ptr(g), _ptr(c))
+        if op == RAM:
+            lib.orc_merge_ram(K, n, _ptr(th64), P32, P64, float(eps_act), float(lam), _ptr(o64))
+        else:
+            lib.orc_merge_tensor(op, K, n, int(bool(is_1d[t])), _ptr(th64), P32, P64, PM,
+                                 float(lam), float(ridge), float(c_min), float(c_max),
+                                 _ptr(o64), _ptr(g), _ptr(c))
         code = dtype_code(np.asarray(theta0[t]))
         out.append(to_dtype(o64, code).reshape(np.shape(theta0[t])))
         out64.append(o64)

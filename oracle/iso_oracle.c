@@ -351,3 +351,32 @@ void orc_merge_tensor(int32_t op, int32_t K, int64_t n, int32_t is_1d,
         out[p] = add_update(theta0[p], s);
     }
 }
+
+/* ------------------------------------------------------------------------ */
+/* RAM (App. F): inactive coordinates are dropped, a coordinate that one
+ * expert updates keeps that expert's value, a coordinate that several update
+ * takes the mean over those experts only. */
+
+void orc_merge_ram(int32_t K, int64_t n, const double* theta0,
+                   const float* const* tau32, const double* const* tau64,
+                   double eps_act, double lambda, double* out) {
+    for (int64_t p = 0; p < n; ++p) {
+        /* A_p and c^p */
+        int active[64];
+        int c = 0;
+        for (int i = 0; i < K; ++i) {
+            if (fabs((double)tau32[i][p]) > eps_act) active[c++] = i;
+        }
+        double tau_ram;
+        if (c == 0) {
+            tau_ram = 0.0;
+        } else if (c == 1) {
+            tau_ram = tau64[active[0]][p];
+        } else {
+            double s = 0.0;
+            for (int a = 0; a < c; ++a) s += tau64[active[a]][p];
+            tau_ram = s / (double)c;
+        }
+        out[p] = add_update(theta0[p], lambda * tau_ram);
+    }
+}

@@ -3,8 +3,8 @@
  *
  * TEST INFRASTRUCTURE ONLY.  This is a plain, slow, single-threaded C
  * restatement of the definitions in "ISO: An RLVR-Native Optimization Stack"
- * (App. F: task vectors, TopKMask, Task Arithmetic, TIES; Sec. 4.2, App. E and
- * Algorithm 1: the retention combiner and the 1-D average).  Only tests/,
+ * (App. F: task vectors, TopKMask, Task Arithmetic, TIES, RAM; Sec. 4.2, App. E
+ * and Algorithm 1: the retention combiner and the 1-D average).  Only tests/,
  * __graft_entry__.smoke() and bench.py's CPU-baseline leg may call it.  It
  * shares no code, header, table or helper with the CUDA library.
  *
@@ -21,7 +21,7 @@ extern "C" {
 #endif
 
 enum { ORC_BF16 = 0, ORC_F32 = 1 };
-enum { ORC_TA = 0, ORC_TIES = 1, ORC_ISO = 2 };
+enum { ORC_TA = 0, ORC_TIES = 1, ORC_ISO = 2, ORC_RAM = 3 };
 
 /* per selection unit, as defined by the oracle's TopKMask */
 typedef struct {
@@ -71,6 +71,16 @@ void orc_merge_tensor(int32_t op, int32_t K, int64_t n, int32_t is_1d,
                       const uint8_t* const* mask,
                       double lambda, double ridge, double c_min, double c_max,
                       double* out, double* gram, double* coef);
+
+/* RAM merge of one tensor (App. F, the RAM coordinate rule): per entry p the
+ * active set A_p = { i : |tau_i^p| > eps_act } and c^p = |A_p|; the merged
+ * coordinate is 0 for c^p = 0, tau_j^p for A_p = {j}, and the mean of the
+ * active values for c^p >= 2; out = theta_0 + lambda tau_RAM (the paper's
+ * RAM has no scale: lambda = 1 is the paper's rule).  Activity is decided on
+ * tau32 (decision precision); the values come from tau64.  No trim. */
+void orc_merge_ram(int32_t K, int64_t n, const double* theta0,
+                   const float* const* tau32, const double* const* tau64,
+                   double eps_act, double lambda, double* out);
 
 /* retention coefficients from a K x K Gram matrix (App. E / Algorithm 1):
  * drop zero-norm experts, solve (G + ridge I) c = diag G, clip. */

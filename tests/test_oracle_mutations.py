@@ -32,6 +32,13 @@ MUTATIONS = {
     "iso_1d_no_average": ("out[p] = add_update(theta0[p], s / (double)K);", "out[p] = add_update(theta0[p], s);"),
     "bf16_round_half_up": ("u += 0x7FFFu + lsb;", "u += 0x8000u;"),
     "bf16_f64_truncates": ("double q = round_half_even(ldexp(a, -q_exp));", "double q = floor(ldexp(a, -q_exp));"),
+    "ram_threshold_inclusive": ("if (fabs((double)tau32[i][p]) > eps_act) active[c++] = i;",
+                                "if (fabs((double)tau32[i][p]) >= eps_act) active[c++] = i;"),
+    "ram_mean_over_all_experts": ("tau_ram = s / (double)c;", "tau_ram = s / (double)K;"),
+    "ram_unique_value_divided": ("tau_ram = tau64[active[0]][p];", "tau_ram = tau64[active[0]][p] / (double)K;"),
+    "ram_drops_lambda": ("out[p] = add_update(theta0[p], lambda * tau_ram);", "out[p] = add_update(theta0[p], tau_ram);"),
+    "ram_inactive_kept": ("if (c == 0) {\n            tau_ram = 0.0;",
+                          "if (c == 0) {\n            tau_ram = tau64[0][p];"),
     "zero_update_normalises_sign": ("return (upd == 0.0) ? theta0 : theta0 + upd;", "return theta0 + upd;"),
 }
 

@@ -405,3 +405,119 @@ def test_ties_untrimmed_tensor_keeps_every_entry():
     np.testing.assert_array_equal(r["out64"][0], th0.astype(np.float64) + tau.astype(np.float64))
     r = oracle.merge([th0], [[tau]], oracle.TIES, density=0.1, lam=1.0, mask_1d=True, is_1d=[True])
     assert (r["out64"][0] != th0.astype(np.float64)).sum() == oracle.k_of(0.1, 64)
+
+
+# ---------------------------------------------------------------------------
+# RAM (App. F): activity threshold, unique values kept, shared ones averaged
+# over the active experts only
+# ---------------------------------------------------------------------------
+
+class TestRamHandWorked:
+    g = _golden("handworked_ram_k3_1x8.json")
+
+    def _run(self, op, **kw):
+        th0 = _f32(self.g["theta0"]).reshape(1, 8)
+        taus = [[_f32(_fr(self.g[f"tau{i}"])).reshape(1, 8)] for i in (1, 2, 3)]
+        return oracle.merge([th0], taus, op, lam=1.0, is_1d=[False],
+                            eps_act=float(Fraction(self.g["eps_act"])), **kw)
+
+    def test_ram(self):
+        r = self._run(oracle.RAM)
+        want = [Fraction(x) for x in self.g["ram"]]
+        got = r["out64"][0]
+        for p, w in enumerate(want):
+            # binary64 mean of at most three dyadic values: exact except the
+            # one division by c, which rounds once
+            assert got[p] == pytest.approx(float(w), rel=2 ** -52, abs=0), p
+        # the entries with a dyadic result are exact
+        for p in (0, 1, 2, 4, 5):
+            assert got[p] == float(want[p])
+        assert r["units"].size == 0   # RAM trims nothing
+
+    def test_ta_differs_where_ram_keeps_or_drops(self):
+        r = self._run(oracle.TA)
+        np.testing.assert_array_equal(r["out64"][0], _fr(self.g["ta"]))
+
+
+def _ram_exact(th0, taus, eps, lam):
+    """RAM evaluated in exact rationals, entry by entry (App. F coordinate rule)."""
+    out = []
+    for p in range(th0.size):
+        act = [Fraction(float(t[p])) for t in taus if abs(float(t[p])) > eps]
+        c = len(act)
+        m = Fraction(0) if c == 0 else (act[0] if c == 1 else sum(act, Fraction(0)) / c)
+        out.append(Fraction(float(th0[p])) + Fraction(lam) * m)
+    return out
+
+
+@pytest.mark.parametrize("K,lam", [(2, 1.0), (3, 0.5), (5, 1.0), (8, 0.75)])
+def test_ram_brute_force_rationals(K, lam):
+    rng = np.random.default_rng(100 + K)
+    n = 300
+    eps = float(np.float32(1e-3))
+    th0 = rng.normal(0, 0.02, n).astype(np.float32)
+    taus = []
+    for i in range(K):
+        t = rng.normal(0, 1e-3, n).astype(np.float32)
+        t[rng.random(n) < 0.3] = 0.0
+        t[rng.random(n) < 0.05] = np.float32(eps) * rng.choice([-1, 1], n)[0]   # on the threshold
+        taus.append(t)
+    r = oracle.merge([th0.reshape(1, n)], [[t.reshape(1, n)] for t in taus], oracle.RAM,
+                     lam=lam, is_1d=[False], eps_act=eps)
+    want = _ram_exact(th0, taus, eps, lam)
+    got = r["out64"][0]
+    for p in range(n):
+        assert got[p] == pytest.approx(float(want[p]), rel=4e-16, abs=1e-300), p
+
+
+def test_ram_disjoint_supports_is_task_arithmetic():
+    rng = np.random.default_rng(110)
+    n, K = 512, 4
+    th0 = rng.normal(0, 0.02, n).astype(np.float32).reshape(1, n)
+    owner = rng.integers(0, K, n)
+    taus = []
+    for i in range(K):
+        t = np.zeros(n, np.float32)
+        sel = owner == i
+        # every owned entry well above the threshold, either sign
+        t[sel] = np.sign(rng.normal(size=sel.sum())) * (np.abs(rng.normal(0, 1e-3, sel.sum())) + 1e-4)
+        taus.append(t.reshape(1, n))
+    r = oracle.merge([th0], [[t] for t in taus], oracle.RAM, lam=1.0, is_1d=[False],
+                     eps_act=float(np.float32(1e-5)))
+    ra = oracle.merge([th0], [[t] for t in taus], oracle.TA, lam=1.0, is_1d=[False])
+    # one active expert per entry: its value is kept whole, as TA's sum gives it
+    np.testing.assert_array_equal(r["out64"][0], ra["out64"][0])
+
+
+@pytest.mark.parametrize("K", [2, 4, 8])
+def test_ram_identical_experts_keep_the_task_vector(K):
+    rng = np.random.default_rng(120 + K)
+    th0, tau = _rand_set(rng, [(16, 40)], dtype="f32")
+    r = oracle.merge(th0, [tau] * K, oracle.RAM, lam=1.0, is_1d=[False], eps_act=0.0)
+    t = tau[0].ravel().astype(np.float64)
+    want = np.where(t == 0.0, th0[0].ravel().astype(np.float64), th0[0].ravel().astype(np.float64) + t)
+    # K copies of one value sum exactly for K a power of two; the mean is the value
+    np.testing.assert_array_equal(r["out64"][0], want)
+
+
+def test_ram_threshold_above_every_update_is_fixed_point():
+    rng = np.random.default_rng(130)
+    th0, tau = _rand_set(rng, [(8, 32), (1, 32)])
+    th0[0].ravel()[3] = 0x8000   # -0.0 keeps its sign
+    eps = max(float(np.abs(oracle.load(t)[0]).max()) for t in tau)
+    r = oracle.merge(th0, [tau, tau], oracle.RAM, is_1d=[False, True], eps_act=eps)
+    for a, b in zip(r["out"], th0):
+        np.testing.assert_array_equal(a, b)
+
+
+def test_ram_single_expert_is_a_threshold_mask():
+    rng = np.random.default_rng(140)
+    n = 2000
+    th0 = rng.normal(0, 0.02, n).astype(np.float32).reshape(1, n)
+    t = rng.normal(0, 1e-5, n).astype(np.float32).reshape(1, n)
+    eps = float(np.float32(1e-5))
+    r = oracle.update([th0], [t], oracle.RAM, update_is_delta=True, is_1d=[False], eps_act=eps)
+    tt = t.ravel().astype(np.float64)
+    want = np.where(np.abs(tt) > eps, th0.ravel().astype(np.float64) + tt, th0.ravel().astype(np.float64))
+    np.testing.assert_array_equal(r["out64"][0], want)
+    assert 0 < np.sum(np.abs(tt) > eps) < n
