@@ -41,6 +41,8 @@ WORKLOADS = {
                        "Qwen2.5-7B-shaped bf16 base, 8 fp32 RL deltas, TopKMask 10% + TIES"),
     "qwen7b_iso_k8": ("qwen7b", 8, "iso", "delta_f32", 0.10, "tensor",
                       "Qwen2.5-7B-shaped bf16 base, 8 fp32 RL deltas, TopKMask 10% + ISO retention"),
+    "qwen7b_ram_k8": ("qwen7b", 8, "ram", "delta_f32", 0.0, "tensor",
+                      "Qwen2.5-7B-shaped bf16 base, 8 fp32 RL deltas, RAM merge (eps_act 1e-5, no trim)"),
     "sweep_tensor": ("sweep", 1, "ties", "delta_bf16", 0.05, "tensor",
                      "bf16 4096x14336 delta N(0,1e-3^2)+1e-3 t_3 with 1000 threshold ties, "
                      "per-tensor TopKMask + masked update (--density)"),
@@ -53,7 +55,7 @@ WORKLOADS = {
 def fused_pass(K, inputs, op, scope, two_pass=False):
     """Whether the library runs the K = 1 update as its fused single pass
     (bf16 base and update, per-tensor TopKMask, a trimming operator)."""
-    return (not two_pass and K == 1 and scope == "tensor" and op != "ta"
+    return (not two_pass and K == 1 and scope == "tensor" and op not in ("ta", "ram")
             and inputs in ("ckpt_bf16", "delta_bf16"))
 
 
@@ -80,7 +82,7 @@ def algorithmic_bytes(shapes, K, inputs, op, scope="tensor", two_pass=False):
         return {"block_select": n_all * (per_base + per_x + per_out)}
     read_tau = n_trim * (K * per_x + (per_base if inputs == "ckpt_bf16" else 0))
     out = {"apply": n_all * (per_base + K * per_x + per_out)}
-    if op != "ta":
+    if op not in ("ta", "ram"):   # the trimming operators select first
         out["block_select" if scope == "block" else "count"] = read_tau
     if op == "iso" and K >= 2:
         out["gram"] = read_tau
@@ -391,7 +393,7 @@ def cpu_baseline(name, budget_s=15.0, seed=0, rho=None):
     if shapes_name == "sweep":
         return cpu_baseline_sweep(name, density, scope, seed)
     shapes, order = cpu_sample(name, seed)
-    orc_op = {"ta": oracle.TA, "ties": oracle.TIES, "iso": oracle.ISO}[op]
+    orc_op = {"ta": oracle.TA, "ties": oracle.TIES, "iso": oracle.ISO, "ram": oracle.RAM}[op]
     done, params, spent = [], 0, 0.0
     for q in order:
         s = shapes[q]

@@ -9,7 +9,7 @@
  *
  *     theta_merge = theta_0 + tau_merge                   (App. F, problem statement)
  *
- * for three operators:
+ * for four operators:
  *   ISO_OP_TA    Task Arithmetic   tau = lambda * sum_i tau_i                (App. F)
  *   ISO_OP_TIES  TIES              trim, sign election, disjoint mean,
  *                                  theta_0 + lambda * tau_TIES              (App. F)
@@ -18,6 +18,10 @@
  *                                  [c_min, c_max], theta_0 + sum_i c_i trimmed tau_i;
  *                                  1-D tensors take the plain task-vector
  *                                  average                (Sec. 4.2, App. E, Algorithm 1)
+ *   ISO_OP_RAM   RAM               per entry, the experts with |tau_i| > eps_act
+ *                                  are active; no active expert: theta_0, one:
+ *                                  its value kept whole, several: their mean;
+ *                                  theta_0 + lambda * tau_RAM  (App. F, RAM)
  *
  * TopKMask(|tau|, rho) (App. F, TIES trim) keeps the k = floor(rho n + 1/2)
  * entries of largest |tau| in each selection unit; entries with equal |tau|
@@ -42,7 +46,9 @@
  *     host before anything is enqueued.  ISO_ERR_CUDA means a launch failed.
  *     ISO_ERR_NONFINITE is detected on the device: it is written to
  *     stats->status (when given) and is valid once the stream has reached the
- *     end of the call; the outputs of such a call are unspecified.
+ *     end of the call; the outputs of such a call are unspecified.  The
+ *     operators that read every task-vector entry's magnitude (TIES, ISO,
+ *     RAM) check for it; TA does not.
  *   - No C++ exception crosses this interface.  The library keeps no state
  *     between calls apart from optional profiling counters.
  */
@@ -104,19 +110,23 @@ typedef struct {
     int32_t reserved;    /* must be 0 */
 } iso_topk_cfg;
 
-typedef enum { ISO_OP_TA = 0, ISO_OP_TIES = 1, ISO_OP_ISO = 2 } iso_op;
+typedef enum { ISO_OP_TA = 0, ISO_OP_TIES = 1, ISO_OP_ISO = 2, ISO_OP_RAM = 3 } iso_op;
 
 typedef struct {
     int32_t op;          /* iso_op */
     int32_t mask_1d;     /* TIES: 1 = 1-D tensors are trimmed like the rest of the task
                             vector, 0 = used untrimmed.  Ignored by TA (never trims) and
                             ISO (1-D tensors take the average) */
-    float   lambda;      /* TA / TIES scale (the paper uses 1.0) */
-    float   reserved;    /* must be 0 */
+    float   lambda;      /* TA / TIES / RAM scale (the paper uses 1.0; its RAM has no
+                            scale, which is lambda = 1) */
+    float   eps_act;     /* RAM active-update threshold, finite and >= 0: expert i is
+                            active at an entry when the binary32 |tau_i| > eps_act
+                            (strict; the paper uses 1e-5).  Ignored by the other
+                            operators */
     double  ridge;       /* ISO lambda_ridge (the paper uses 1e-12), >= 0 */
     double  c_min;       /* ISO clip range (the paper uses [0, 1.5]) */
     double  c_max;
-    iso_topk_cfg topk;   /* TopKMask of TIES and ISO; ignored by TA */
+    iso_topk_cfg topk;   /* TopKMask of TIES and ISO; ignored by TA and RAM */
 } iso_merge_cfg;
 
 /* Per selection unit, written by the device. */
@@ -138,7 +148,8 @@ typedef struct {
 typedef struct {
     int32_t*        status;  /* 1 value: ISO_OK or ISO_ERR_NONFINITE, valid after the stream
                                 reaches the end of the call */
-    iso_unit_stats* units;   /* [K][n_units], n_units from iso_num_units */
+    iso_unit_stats* units;   /* [K][n_units], n_units from iso_num_units; not written by
+                                TA and RAM, which trim nothing */
     double*         gram;    /* ISO: [n_tensors][K][K] Gram of the trimmed task vectors
                                 (zero for 1-D tensors) */
     double*         coef;    /* ISO: [n_tensors][K] retention coefficients c* */
@@ -179,7 +190,9 @@ int32_t iso_topk_mask(const iso_tensor* tau, int32_t n_tensors, const iso_topk_c
  *                                               or update - theta_0 (a checkpoint)
  * with c = lambda for TIES, c = clip(Gamma / (Gamma + ridge)) for ISO (Gamma the
  * squared norm of the trimmed tensor); ISO leaves 1-D tensors at theta_0 + tau.
- * TA applies lambda * tau untrimmed.  out has the base's dtype and may alias
+ * TA applies lambda * tau untrimmed; RAM with one expert keeps theta_0 +
+ * lambda * tau where |tau| > eps_act and theta_0 elsewhere (no TopKMask).
+ * out has the base's dtype and may alias
  * theta_0 (each entry is read before it is written by the same thread); it may
  * not alias update. */
 int32_t iso_update(const iso_tensor* theta_0, const iso_tensor* update, int32_t update_is_delta,

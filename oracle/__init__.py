@@ -273,16 +273,15 @@ def retention(gram: np.ndarray, ridge=1e-12, c_min=0.0, c_max=1.5) -> np.ndarray
 def merge(theta0, experts, op, *, experts_are_deltas=True, density=0.2,
           scope=SCOPE_TENSOR, block=(128, 128), lam=1.0, ridge=1e-12, c_min=0.0,
           c_max=1.5, mask_1d=True, shapes=None, is_1d=None, method="select",
-          eps_act=1e-5):
+          eps_act=float(np.float32(1e-5))):
     """Merge K experts into the base, tensor by tensor.
 
     theta0       list of base tensors (uint16 bfloat16 bits or float32)
     experts      list of K lists of tensors: task vectors (experts_are_deltas)
                  or fine-tuned checkpoints
     op           TA / TIES / ISO / RAM
-    eps_act      RAM activity threshold (the paper uses 1e-5); the library
-                 takes it as a binary32 value, so pass a value that float32
-                 represents (e.g. ``float(np.float32(1e-5))``) to compare
+    eps_act      RAM activity threshold; the default is the paper's 1e-5 as
+                 a binary32 value (the library takes the threshold in binary32)
     shapes       list of (rows, cols); defaults to each array's 2-D shape
     is_1d        list of flags; defaults to rows == 1 for 1-row tensors
 

@@ -26,7 +26,7 @@ ISO_NOALLOC_SCRATCH_BYTES = 32 << 20
 
 ISO_BF16, ISO_F32 = 0, 1
 ISO_SCOPE_TENSOR, ISO_SCOPE_BLOCK, ISO_SCOPE_GLOBAL = 0, 1, 2
-ISO_OP_TA, ISO_OP_TIES, ISO_OP_ISO = 0, 1, 2
+ISO_OP_TA, ISO_OP_TIES, ISO_OP_ISO, ISO_OP_RAM = 0, 1, 2, 3
 
 
 class IsoTensor(ctypes.Structure):
@@ -42,7 +42,7 @@ class IsoTopkCfg(ctypes.Structure):
 
 class IsoMergeCfg(ctypes.Structure):
     _fields_ = [("op", ctypes.c_int32), ("mask_1d", ctypes.c_int32), ("lam", ctypes.c_float),
-                ("reserved", ctypes.c_float), ("ridge", ctypes.c_double),
+                ("eps_act", ctypes.c_float), ("ridge", ctypes.c_double),
                 ("c_min", ctypes.c_double), ("c_max", ctypes.c_double), ("topk", IsoTopkCfg)]
 
 

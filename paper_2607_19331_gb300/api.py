@@ -17,7 +17,7 @@ import torch
 from . import _abi
 from ._abi import (IsoMergeCfg, IsoMergeStats, IsoTensor, IsoTopkCfg, check, lib)
 
-OPS = {"ta": _abi.ISO_OP_TA, "ties": _abi.ISO_OP_TIES, "iso": _abi.ISO_OP_ISO}
+OPS = {"ta": _abi.ISO_OP_TA, "ties": _abi.ISO_OP_TIES, "iso": _abi.ISO_OP_ISO, "ram": _abi.ISO_OP_RAM}
 SCOPES = {"tensor": _abi.ISO_SCOPE_TENSOR, "block": _abi.ISO_SCOPE_BLOCK,
           "global": _abi.ISO_SCOPE_GLOBAL}
 UNIT_STATS_DTYPE = np.dtype([
@@ -61,9 +61,10 @@ def topk_cfg(density=0.05, scope="tensor", block=(128, 128)) -> IsoTopkCfg:
 
 
 def merge_cfg(op="ties", density=0.2, scope="tensor", block=(128, 128), lam=1.0, ridge=1e-12,
-              c_min=0.0, c_max=1.5, mask_1d=True) -> IsoMergeCfg:
-    return IsoMergeCfg(OPS[op], int(bool(mask_1d)), float(lam), 0.0, float(ridge), float(c_min),
-                       float(c_max), topk_cfg(density, scope, block))
+              c_min=0.0, c_max=1.5, mask_1d=True, eps_act=1e-5) -> IsoMergeCfg:
+    """eps_act (RAM) is passed as a binary32 value."""
+    return IsoMergeCfg(OPS[op], int(bool(mask_1d)), float(lam), float(eps_act), float(ridge),
+                       float(c_min), float(c_max), topk_cfg(density, scope, block))
 
 
 def _stream(stream) -> ctypes.c_void_p:
@@ -184,13 +185,13 @@ def iso_merge(theta_0: List[torch.Tensor], experts: List[List[torch.Tensor]], op
               experts_are_deltas=True, out=None, density=0.2, scope="tensor", block=(128, 128),
               lam=1.0, ridge=1e-12, c_min=0.0, c_max=1.5, mask_1d=True, is_1d=None,
               workspace: Optional[Workspace] = None, stats=False, stream=None,
-              ws_bytes: Optional[int] = None):
+              ws_bytes: Optional[int] = None, eps_act=1e-5):
     K = len(experts)
     n = len(theta_0)
     dev = theta_0[0].device
     if out is None:
         out = [torch.empty_like(t) for t in theta_0]
-    cfg = merge_cfg(op, density, scope, block, lam, ridge, c_min, c_max, mask_1d)
+    cfg = merge_cfg(op, density, scope, block, lam, ridge, c_min, c_max, mask_1d, eps_act)
     flat = [x for e in experts for x in e]
     d0 = describe(theta_0, is_1d)
     dx = describe(flat, None if is_1d is None else list(is_1d) * K)
@@ -275,7 +276,7 @@ def profile_read():
 def iso_update_noalloc(theta_0: List[torch.Tensor], update: List[torch.Tensor], op="iso",
                        update_is_delta=False, out=None, density=0.05, scope="tensor",
                        block=(128, 128), lam=1.0, ridge=1e-12, c_min=0.0, c_max=1.5,
-                       mask_1d=True, stats=False, stream=None):
+                       mask_1d=True, stats=False, stream=None, eps_act=1e-5):
     """iso_update for callers that cannot allocate device memory: the library
     runs the update in its own fixed per-device scratch (no workspace
     argument).  Make the first call on a device before any stream capture;
@@ -283,7 +284,7 @@ def iso_update_noalloc(theta_0: List[torch.Tensor], update: List[torch.Tensor], 
     dev = theta_0[0].device
     if out is None:
         out = [torch.empty_like(t) for t in theta_0]
-    cfg = merge_cfg(op, density, scope, block, lam, ridge, c_min, c_max, mask_1d)
+    cfg = merge_cfg(op, density, scope, block, lam, ridge, c_min, c_max, mask_1d, eps_act)
     st = make_stats(theta_0, 1, cfg.topk, dev) if stats else None
     check(lib().iso_update_noalloc(describe(theta_0), describe(update), int(bool(update_is_delta)),
                                    describe(out), len(theta_0), ctypes.byref(cfg),

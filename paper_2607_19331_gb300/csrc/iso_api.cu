@@ -174,12 +174,13 @@ int check_topk(const iso_topk_cfg& c) {
 }
 
 int check_merge_cfg(const iso_merge_cfg& c) {
-    if (c.op < ISO_OP_TA || c.op > ISO_OP_ISO) return ISO_ERR_ARG;
+    if (c.op < ISO_OP_TA || c.op > ISO_OP_RAM) return ISO_ERR_ARG;
     if (c.mask_1d != 0 && c.mask_1d != 1) return ISO_ERR_ARG;
-    if (!std::isfinite(c.lambda) || c.reserved != 0.0f) return ISO_ERR_ARG;
+    if (!std::isfinite(c.lambda)) return ISO_ERR_ARG;
+    if (!std::isfinite(c.eps_act) || c.eps_act < 0.0f) return ISO_ERR_ARG;
     if (!std::isfinite(c.ridge) || c.ridge < 0.0) return ISO_ERR_ARG;
     if (!std::isfinite(c.c_min) || !std::isfinite(c.c_max) || c.c_min > c.c_max) return ISO_ERR_ARG;
-    if (c.op != ISO_OP_TA) return check_topk(c.topk);
+    if (c.op != ISO_OP_TA && c.op != ISO_OP_RAM) return check_topk(c.topk);
     return ISO_OK;
 }
 
@@ -197,6 +198,7 @@ struct Call {
     bool mask_only = false;
     bool mask_1d = true;
     float lambda = 1.0f;
+    float eps_act = 0.0f;                 // RAM threshold, +0 for a zero
     double ridge = 1e-12, c_min = 0.0, c_max = 1.5;
     iso_topk_cfg topk{};
     bool trims = true;                    // some tensor is trimmed
@@ -494,6 +496,7 @@ int run_group(const Call& c, int t0, int t1, char* ws, cudaStream_t s, const iso
     P.block_rows = c.topk.block_rows;
     P.block_cols = c.topk.block_cols;
     P.lambda = c.lambda;
+    P.eps_act = c.eps_act;
     P.density = c.topk.density;
     P.ridge = c.ridge;
     P.c_min = c.c_min;
@@ -631,7 +634,9 @@ int run_group(const Call& c, int t0, int t1, char* ws, cudaStream_t s, const iso
             return launch(KD_APPLY, s, [&] { k_merge<XT, BT, CK, KC, OPF_OTHER><<<mgrid, TPB, smem, s>>>(P); });
         };
         if (K == 1 && fuse_block) return ISO_OK;
-        if (K == 1) ISO_TRY(launch(KD_APPLY, s, [&] { k_apply<XT, BT, CK, 1><<<pgrid, TPB, 0, s>>>(P); }));
+        // RAM with one expert: the merge pass (its activity test lives there)
+        if (K == 1 && c.op == ISO_OP_RAM) ISO_TRY(merge(std::integral_constant<int, 2>{}));
+        else if (K == 1) ISO_TRY(launch(KD_APPLY, s, [&] { k_apply<XT, BT, CK, 1><<<pgrid, TPB, 0, s>>>(P); }));
         else if (K == 2) ISO_TRY(merge(std::integral_constant<int, 2>{}));
         else if (K <= 4) ISO_TRY(merge(std::integral_constant<int, 4>{}));
         else ISO_TRY(merge(std::integral_constant<int, 8>{}));
@@ -687,7 +692,7 @@ void set_trim(Call& c, const iso_tensor* tens) {
     for (int t = 0; t < c.n; ++t) {
         bool tr;
         if (c.mask_only) tr = true;
-        else if (c.op == ISO_OP_TA) tr = false;
+        else if (c.op == ISO_OP_TA || c.op == ISO_OP_RAM) tr = false;
         else if (c.op == ISO_OP_TIES) tr = c.mask_1d || !tens[t].is_1d;
         else tr = !tens[t].is_1d;
         c.trim[t] = tr ? 1 : 0;
@@ -727,11 +732,12 @@ int build_merge_call(Call& c, const iso_tensor* theta_0, const iso_tensor* exper
     c.op = cfg->op;
     c.mask_1d = cfg->mask_1d != 0;
     c.lambda = cfg->lambda;
+    c.eps_act = (cfg->eps_act == 0.0f) ? 0.0f : cfg->eps_act;   // -0 -> +0: |tau| > 0 keeps zeros out
     c.ridge = cfg->ridge;
     c.c_min = cfg->c_min;
     c.c_max = cfg->c_max;
     c.topk = cfg->topk;
-    if (c.op == ISO_OP_TA) { c.topk.scope = ISO_SCOPE_TENSOR; c.topk.density = 1.0; }
+    if (c.op == ISO_OP_TA || c.op == ISO_OP_RAM) { c.topk.scope = ISO_SCOPE_TENSOR; c.topk.density = 1.0; }
     c.xdt = n > 0 ? experts[0].dtype : ISO_F32;
     c.bdt = n > 0 ? theta_0[0].dtype : ISO_F32;
     set_trim(c, theta_0);
@@ -779,7 +785,7 @@ int32_t iso_workspace_size(const iso_tensor* tensors, int32_t n_tensors, int32_t
     c.op = cfg->op;
     c.mask_1d = cfg->mask_1d != 0;
     c.topk = cfg->topk;
-    if (c.op == ISO_OP_TA) { c.topk.scope = ISO_SCOPE_TENSOR; c.topk.density = 1.0; }
+    if (c.op == ISO_OP_TA || c.op == ISO_OP_RAM) { c.topk.scope = ISO_SCOPE_TENSOR; c.topk.density = 1.0; }
     // experts are taken to share the base's dtype: for other combinations the
     // size reported is an upper bound
     c.xdt = c.bdt = n_tensors ? tensors[0].dtype : ISO_F32;

@@ -185,6 +185,7 @@ struct Plan {
     int32_t fuse_block;     // BLOCK scope, K = 1 TIES: k_block_select writes the outputs
     int32_t block_rows, block_cols;
     float lambda;
+    float eps_act;          // RAM: expert active where the binary32 |tau| > eps_act (>= +0)
     double density, ridge, c_min, c_max;
     // stats destinations (device, may be NULL) and the unit offset of this group
     iso_unit_stats* st_units;

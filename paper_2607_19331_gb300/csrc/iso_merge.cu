@@ -123,7 +123,7 @@ enum SelMode : int {
     SEL_BLOCK = 2,    // BLOCK scope: the unit of each entry's block
 };
 
-enum OpKind : int { OPK_SUM = 0, OPK_TIES = 1, OPK_ISO = 2 };
+enum OpKind : int { OPK_SUM = 0, OPK_TIES = 1, OPK_ISO = 2, OPK_RAM = 3 };
 
 template <int KC>
 struct MergeParams {
@@ -131,6 +131,7 @@ struct MergeParams {
     unsigned long long thr[KC];   // SEL_PACKED, tensor-local positions
     float cf[KC];                 // ISO 2-D coefficients
     int sel, opk;
+    int teps;                     // RAM: key of eps_act (active: key > teps)
     bool iso1d, trimmed2d;
 };
 
@@ -145,8 +146,10 @@ __device__ __forceinline__ void merge_params(const Plan& P, int t, int K, MergeP
     const bool trim = (d.flags & TF_TRIM) != 0;
     mp.iso1d = (P.op == ISO_OP_ISO) && is1d;
     mp.trimmed2d = trim && !is1d;
-    mp.opk = (P.op == ISO_OP_TA || mp.iso1d) ? OPK_SUM : (P.op == ISO_OP_TIES ? OPK_TIES : OPK_ISO);
-    if (mp.opk == OPK_SUM) mp.sel = SEL_ALL;
+    mp.opk = (P.op == ISO_OP_TA || mp.iso1d) ? OPK_SUM
+           : (P.op == ISO_OP_TIES ? OPK_TIES : (P.op == ISO_OP_RAM ? OPK_RAM : OPK_ISO));
+    mp.teps = (int)__float_as_uint(P.eps_act);   // eps_act >= +0 and finite: below 2^31
+    if (mp.opk == OPK_SUM || mp.opk == OPK_RAM) mp.sel = SEL_ALL;
     else if (trim && P.scope == ISO_SCOPE_BLOCK) mp.sel = SEL_BLOCK;
     else mp.sel = SEL_PACKED;
     // GLOBAL scope: the unit's cut is a position in the concatenation; entry
@@ -204,7 +207,9 @@ __device__ __forceinline__ uint32_t select_bits(const Plan& P, const TensorDesc&
     return bits;
 }
 
-// the merged output of one entry; every argument is in registers
+// the merged output of one entry; every argument is in registers.  RAM never
+// comes here: its tensors are untrimmed (SEL_ALL), so every tile takes the
+// per-tile form below.
 template <int KC>
 __device__ __forceinline__ float merged_value(int opk, bool iso1d, float lambda, int K, float th0,
                                               const float (&tau)[KC], const float (&cf)[KC], uint32_t bits) {
@@ -258,6 +263,7 @@ __device__ __forceinline__ bool tile_thresholds(const MergeParams<KC>& mp, int K
 #pragma unroll
     for (int i = 0; i < KC; ++i) {
         T[i] = (i < K) ? -1 : 0x7FFFFFFF;                      // experts past K: nothing kept
+        if (i < K && mp.opk == OPK_RAM) T[i] = mp.teps;        // RAM: active where |tau| > eps_act
         if (i < K && mp.sel == SEL_PACKED) {
             const unsigned long long th = mp.thr[i];
             const uint32_t tk = (uint32_t)(th >> 32), c32 = ~(uint32_t)th;
@@ -276,9 +282,27 @@ __device__ __forceinline__ bool tile_thresholds(const MergeParams<KC>& mp, int K
 // skipping form gives them
 template <int KC>
 __device__ __forceinline__ float merged_fast(int opk, bool iso1d, float lambda, int K, float th0,
-                                             const float (&tau)[KC], const float (&cf)[KC], const int (&T)[KC]) {
+                                             const float (&tau)[KC], const float (&cf)[KC], const int (&T)[KC],
+                                             uint32_t& kmax) {
     float upd;
-    if (opk == OPK_TIES) {
+    if (opk == OPK_RAM) {
+        // RAM (App. F): active experts key > T (|tau| > eps_act; T is past
+        // every key for q >= K); the active values summed in expert order,
+        // divided by their count -- one active value is kept whole (0 + v
+        // and v / 1 are exact), none leaves theta_0
+        float s = 0.0f;
+        int cnt = 0;
+#pragma unroll
+        for (int q = 0; q < KC; ++q) {
+            const uint32_t k = key_of(tau[q]);
+            kmax = (q < K && k > kmax) ? k : kmax;
+            const bool a = (int)k > T[q];
+            s = __fadd_rn(s, a ? tau[q] : 0.0f);
+            cnt += a;
+        }
+        const float m = cnt ? __fdiv_rn(s, (float)cnt) : 0.0f;
+        upd = __fmul_rn(lambda, m);
+    } else if (opk == OPK_TIES) {
         // gamma = sign of the trimmed sum; the agreeing set: the non-zero
         // trimmed values of that sign.  u = tt with the sign of the sum
         // cleared is |tt| exactly for the agreeing ones, so their sum in
@@ -408,8 +432,9 @@ struct IssueCursor<KC, true> {
     const void* bp = nullptr;
 };
 
-// copy step (g, s) of lane `lane` into stage `st` (shared-space address)
-template <typename XT, typename BT, int KC, bool SP>
+// copy step (g, s) of lane `lane` into stage `st` (shared-space address);
+// NB = false leaves the base out (a pass over task vectors that never reads it)
+template <typename XT, typename BT, int KC, bool SP, bool NB = true>
 __device__ __forceinline__ void issue_step(const Plan& P, int K, IssueCursor<KC, SP>& ic, long long g, int s,
                                            uint32_t st, int lane) {
     using G = StageGeom<XT, BT, KC>;
@@ -438,6 +463,7 @@ __device__ __forceinline__ void issue_step(const Plan& P, int K, IssueCursor<KC,
             cp_async16(st + i * 512 + lane * 16, src, xb);
         }
     }
+    if (!NB) return;
     const uint32_t bdst = st + KC * 512 + lane * G::BB;
     const char* bsrc = static_cast<const char*>(ic.bp) + (in ? e * (long long)sizeof(BT) : 0);
     const long long bavail = (ic.n - e) * (long long)sizeof(BT);
@@ -509,6 +535,7 @@ __global__ void __launch_bounds__(TPB, merge_blocks_per_sm(KC, OPF)) k_merge(Pla
     merge_params<KC>(P, t, K, mp);
     float cf[KC];
     int T[KC];
+    uint32_t kmax = 0;   // RAM: largest key seen (non-finite inputs)
     bool exact = false;
     int opk = 0;
     bool iso1d = false;
@@ -580,12 +607,15 @@ __global__ void __launch_bounds__(TPB, merge_blocks_per_sm(KC, OPF)) k_merge(Pla
                 const uint32_t bits = select_bits<KC>(P, *dp, mp, K, tau, e + j, r, c);
                 o[j] = merged_value<KC>(opk, iso1d, P.lambda, K, th0, tau, cf, bits);
             } else {
-                o[j] = merged_fast<KC>(opk, iso1d, P.lambda, K, th0, tau, cf, T);
+                o[j] = merged_fast<KC>(opk, iso1d, P.lambda, K, th0, tau, cf, T, kmax);
             }
         }
         store_out<BT, E>(op, e, n, o);
     }
     cp_async_wait<0>();
+    // RAM reads every entry's magnitude: a NaN or infinity is reported
+    // (entries past a tensor's end are staged as zeros)
+    if (__any_sync(0xFFFFFFFFu, kmax >= KEY_INF) && lane == 0) set_status(P.hdr, ISO_ERR_NONFINITE);
 }
 
 // Gram of the trimmed task vectors, upper triangle, per 2-D trimmed tensor.
@@ -619,7 +649,7 @@ __global__ void __launch_bounds__(TPB, gram_blocks_per_sm(KC)) k_gramk(Plan P) {
     if constexpr (SP) ic.xs = s_xs[warp];
 #pragma unroll
     for (int p = 0; p < D - 1; ++p) {
-        if (p < NS) issue_step<XT, BT, KC, SP>(P, K, ic, wr.beg + p / SPT, p % SPT, ring_s + p * G::BYTES, lane);
+        if (p < NS) issue_step<XT, BT, KC, SP, CK>(P, K, ic, wr.beg + p / SPT, p % SPT, ring_s + p * G::BYTES, lane);
         cp_async_commit();
     }
     int t = tensor_of_tile(P.tens, P.n_tensors, wr.beg);
@@ -683,7 +713,7 @@ __global__ void __launch_bounds__(TPB, gram_blocks_per_sm(KC)) k_gramk(Plan P) {
             return __uint_as_float((j & 1) ? (w & 0xFFFF0000u) : (w << 16));
         };
         const long long ni = i + D - 1;
-        if (ni < NS) issue_step<XT, BT, KC, SP>(P, K, ic, wr.beg + ni / SPT, (int)(ni % SPT), ring_s + (int)(ni % D) * G::BYTES, lane);
+        if (ni < NS) issue_step<XT, BT, KC, SP, CK>(P, K, ic, wr.beg + ni / SPT, (int)(ni % SPT), ring_s + (int)(ni % D) * G::BYTES, lane);
         cp_async_commit();
         const long long e = e0 + (long long)s * (32 * E) + lane * E;
         if (active && e < n) {

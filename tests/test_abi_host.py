@@ -63,12 +63,12 @@ def test_num_units_and_workspace():
         assert L.iso_num_units(ts, 3, ctypes.byref(cfg), ctypes.byref(n)) == 0
         assert n.value == want, (scope, n.value)
     mn, full = ctypes.c_size_t(), ctypes.c_size_t()
-    for op in ("ta", "ties", "iso"):
+    for op in ("ta", "ties", "iso", "ram"):
         for scope in ("tensor", "block", "global"):
             cfg = iso.merge_cfg(op, 0.05, scope)
             assert L.iso_workspace_size(ts, 3, 2, ctypes.byref(cfg), ctypes.byref(mn), ctypes.byref(full)) == 0
             assert 0 < mn.value <= full.value
-            if scope == "global" and op != "ta":
+            if scope == "global" and op not in ("ta", "ram"):
                 assert mn.value == full.value
     cfg = iso.merge_cfg("ties", 0.05)
     assert L.iso_workspace_size(ts, 3, 9, ctypes.byref(cfg), None, None) == _abi.ISO_ERR_UNSUPPORTED
@@ -97,6 +97,15 @@ def test_validation_rejects_before_launch():
     assert upd(a, b, o, cfg_=bad) == _abi.ISO_ERR_ARG
     bad = iso.merge_cfg("iso", 0.2, c_min=2.0, c_max=1.0)
     assert upd(a, b, o, cfg_=bad) == _abi.ISO_ERR_ARG
+    for eps in (-1e-5, float("nan"), float("inf")):       # RAM threshold: finite, >= 0
+        bad = iso.merge_cfg("ram", eps_act=eps)
+        assert upd(a, b, o, cfg_=bad) == _abi.ISO_ERR_ARG
+    bad = iso.merge_cfg("ties", 0.2)
+    bad.op = 4
+    assert upd(a, b, o, cfg_=bad) == _abi.ISO_ERR_ARG
+    # RAM ignores the TopKMask settings (host-only sizing call)
+    ram = iso.merge_cfg("ram", 0.2, "block", block=(128, 12))
+    assert L.iso_workspace_size(a, 1, 2, ctypes.byref(ram), None, None) == 0
     bad = iso.merge_cfg("ties", 0.2, "block", block=(128, 12))
     assert upd(a, b, o, cfg_=bad) == _abi.ISO_ERR_ARG
     bad = iso.merge_cfg("ties", 0.2, "block", block=(256, 256))

@@ -7,8 +7,8 @@ configuration, checked against the oracle on sampled tensors.
   moved onto the threshold (per-tensor and per-128x128-block TopKMask at
   rho = 1, 5, 20, 50 %), every entry checked;
 * the Qwen2.5-7B-shaped merge of 8 fp32 RL deltas into a bf16 base (TopKMask
-  10 % per delta, TIES and the ISO retention rule), which holds ~274 GB of
-  inputs and outputs on the device.
+  10 % per delta, TIES and the ISO retention rule; RAM with eps_act = 1e-5),
+  which holds ~274 GB of inputs and outputs on the device.
 
 Each selection unit is an independent problem, so a tensor checked alone by
 the oracle must match the same tensor inside the whole-model call.
@@ -113,9 +113,11 @@ def test_full_size_qwen7b_merge_k8_sampled():
     ws.get(ws_bytes)
     picks = [_qwen7b_index(0, "k"), _qwen7b_index(0, "norm2"), _qwen7b_index(13, "q"),
              _qwen7b_index(27, "v")]
-    for op, oop in (("ties", oracle.TIES), ("iso", oracle.ISO)):
+    eps = float(np.float32(1e-5))   # RAM's active-update threshold (App. F)
+    for op, oop in (("ties", oracle.TIES), ("iso", oracle.ISO), ("ram", oracle.RAM)):
         out, st = iso.iso_merge(th0, taus, op=op, experts_are_deltas=True, out=out, density=0.1,
-                                scope="tensor", lam=1.0, stats=True, workspace=ws, ws_bytes=ws_bytes)
+                                scope="tensor", lam=1.0, stats=True, workspace=ws, ws_bytes=ws_bytes,
+                                eps_act=eps)
         torch.cuda.synchronize()
         assert int(st.status.item()) == 0
         units = st.units_numpy()
@@ -125,10 +127,11 @@ def test_full_size_qwen7b_merge_k8_sampled():
             a = to_np(th0[q]).reshape(r_, c_)
             ex = [[to_np(taus[i][q]).reshape(r_, c_)] for i in range(K)]
             r = oracle.merge([a], ex, oop, experts_are_deltas=True, density=0.1, lam=1.0,
-                             is_1d=[one])
+                             is_1d=[one], eps_act=eps)
             what = f"7B K=8 {op} tensor {q}"
             assert_values_close(to_np(out[q]), r["out64"][0], r["mag"][0], what)
-            assert_units_equal(units[:, q:q + 1], r["units"], what)
+            if op != "ram":   # RAM trims nothing: no unit records
+                assert_units_equal(units[:, q:q + 1], r["units"], what)
             if op == "iso" and not one:
                 np.testing.assert_allclose(coef[q], r["coef"][0], rtol=1e-5, atol=1e-9)
     del th0, taus, out, ws
