@@ -41,6 +41,10 @@ WORKLOADS = {
                        "Qwen2.5-7B-shaped bf16 base, 8 fp32 RL deltas, TopKMask 10% + TIES"),
     "qwen7b_iso_k8": ("qwen7b", 8, "iso", "delta_f32", 0.10, "tensor",
                       "Qwen2.5-7B-shaped bf16 base, 8 fp32 RL deltas, TopKMask 10% + ISO retention"),
+    "qwen7b_update_global": ("qwen7b", 1, "ties", "ckpt_bf16", 0.20, "global",
+                             "Qwen2.5-7B-shaped bf16 base + RL checkpoint, TIES update under one "
+                             "GLOBAL TopKMask at 20% over the whole task vector (the paper's TIES "
+                             "scope and density)"),
     "qwen7b_ram_k8": ("qwen7b", 8, "ram", "delta_f32", 0.0, "tensor",
                       "Qwen2.5-7B-shaped bf16 base, 8 fp32 RL deltas, RAM merge (eps_act 1e-5, no trim)"),
     "sweep_tensor": ("sweep", 1, "ties", "delta_bf16", 0.05, "tensor",
@@ -93,6 +97,7 @@ def algorithmic_bytes(shapes, K, inputs, op, scope="tensor", two_pass=False):
 KERNEL_SOURCES = {
     "count": ["iso_fused.cu", "iso_select.cu"],   # fused K = 1 pass, or the two-pass counting read
     "apply": ["iso_apply.cu", "iso_merge.cu"],
+    "merge": ["iso_merge.cu"],                    # the apply pass of K >= 2 (and RAM) runs k_merge alone
     "gram": ["iso_merge.cu"],
     "block_select": ["iso_block.cu"],
 }
@@ -306,7 +311,10 @@ def run_mine(args):
     achieved = per_launch_bytes / (avg_ms * 1e-3) / 1e9 if avg_ms > 0 else 0.0
     step_gbs = sum(algo.values()) / (ms * 1e-3) / 1e9
     small = args.layers is not None or args.scale != 1
-    tb = profiled_traffic(dom, name) if not small else None
+    # the apply pass of K >= 2 merges (and of RAM at any K) is k_merge alone:
+    # its traffic is tied to that kernel's sources
+    hkind = "merge" if dom == "apply" and (K >= 2 or op == "ram") else dom
+    tb = profiled_traffic(hkind, name) if not small else None
     traffic = None if tb is None else int(tb * n_params)
 
     # end to end through the public API from pinned host memory

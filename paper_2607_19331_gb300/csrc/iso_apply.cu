@@ -66,8 +66,12 @@ __device__ __forceinline__ void k1_params(const Plan& P, const TensorParams& tp,
     else if (tp.iso1d) { *a = 1.0f; *mask = false; }
     else if (tp.iso2d) { *a = tp.cf[0]; *mask = true; }
     else { *a = P.lambda; *mask = true; }
+    // GLOBAL scope: the cut is a position in the concatenation; entry e of
+    // this tensor sits at pos_off + e, so the tensor-local cut is cut - pos_off
+    // clamped to [0, 2^32 - 1] (numel < 2^32 keeps every local position below)
     const long long cut = tp.sp[0].cut;
-    const uint32_t c32 = (cut >= 0xFFFFFFFFLL) ? 0xFFFFFFFFu : (uint32_t)cut;
+    const long long lc = (cut == CUT_ALL) ? cut : cut - tp.pos_off;
+    const uint32_t c32 = (lc >= 0xFFFFFFFFLL) ? 0xFFFFFFFFu : (lc <= 0 ? 0u : (uint32_t)lc);
     *thr = ((unsigned long long)tp.sp[0].t << 32) | (uint32_t)~c32;
 }
 
@@ -143,7 +147,7 @@ __global__ void __launch_bounds__(TPB) k_apply(Plan P) {
                     raw_to_f32<XT>(cur.x[v], tau);
                 }
                 float o[VEC];
-                if (tp.blk || P.scope == ISO_SCOPE_GLOBAL) {
+                if (tp.blk) {
                     long long r = 0, cc = 0;
                     if (tp.blk) { r = e / d.cols; cc = e - r * d.cols; }
 #pragma unroll

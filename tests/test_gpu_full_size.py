@@ -3,6 +3,9 @@ configuration, checked against the oracle on sampled tensors.
 
 * Qwen2.5-7B-shaped masked ISO update (bf16 base + RL checkpoint, 254
   tensors, per-tensor TopKMask 5 %);
+* the same update as TIES under one GLOBAL TopKMask at 20 % over the whole
+  task vector (the paper's TIES scope), checked entry by entry against the
+  definition;
 * the density sweep on one bf16 4096 x 14336 task vector with 1000 entries
   moved onto the threshold (per-tensor and per-128x128-block TopKMask at
   rho = 1, 5, 20, 50 %), every entry checked;
@@ -70,6 +73,60 @@ def test_full_size_qwen7b_update_sampled():
                           density=0.05, is_1d=[one])
         assert_values_close(to_np(out[q]), r["out64"][0], r["mag"][0], f"7B tensor {q}")
         assert_units_equal(units[q:q + 1], r["units"][0], f"7B unit {q}")
+    del th0, th1, out, ws
+    torch.cuda.empty_cache()
+
+
+def test_full_size_qwen7b_global_ties_update():
+    """One GLOBAL TopKMask over the whole 7,615,483,904-entry task vector (the
+    paper's TIES scope) at rho = 20 %, TIES with lambda = 1, in the benchmark's
+    launch configuration.  The oracle cannot hold the concatenation in a
+    test's time, so the result is checked against what the definition fixes,
+    computed from the inputs with plain tensor operations on the device: k,
+    the threshold t as the k-th largest key (count above t < k <= count at or
+    above t), the tie counts, and every output bit (kept entries: key > t, or
+    key == t among the first k - count_above ties in tensor-then-index
+    order)."""
+    shapes = synth.qwen_shapes("qwen7b")
+    th0, th1 = synth.rl_update_set(shapes, seed=0, device=DEV)
+    rho = 0.2
+    cfg = iso.merge_cfg("ties", rho, "global")
+    mn, full = iso.iso_workspace_size(th0, 1, cfg)
+    assert mn == full   # one unit over every tensor: one group
+    ws = iso.Workspace(DEV)
+    ws.get(full)
+    out = [torch.empty_like(t) for t in th0]
+    out, st = iso.iso_update(th0, th1, op="ties", density=rho, scope="global", lam=1.0, stats=True,
+                             out=out, workspace=ws, ws_bytes=full)
+    torch.cuda.synchronize()
+    assert int(st.status.item()) == 0
+    u = st.units_numpy()[0][0]
+    n_all = sum(t.numel() for t in th0)
+    k = oracle.k_of(rho, n_all)
+    assert int(u["k"]) == k
+    t = int(u["thresh_key"])
+    above, eq = 0, 0
+    for a, b in zip(th0, th1):
+        key = (b.float() - a.float()).view(torch.int32) & 0x7FFFFFFF
+        above += int((key > t).sum())
+        eq += int((key == t).sum())
+    assert int(u["count_above"]) == above and int(u["ties_at_thresh"]) == eq
+    assert above < k <= above + eq
+    need = k - above
+    assert int(u["ties_taken"]) == need
+    seen = 0
+    for q, (a, b, o) in enumerate(zip(th0, th1, out)):
+        tau = (b.float() - a.float()).reshape(-1)
+        key = tau.view(torch.int32) & 0x7FFFFFFF
+        tie = key == t
+        rank = torch.cumsum(tie.to(torch.int64), 0) + seen
+        kept = (key > t) | (tie & (rank <= need))
+        seen += int(tie.sum())
+        upd = torch.where(kept, tau, torch.zeros_like(tau))
+        base = a.reshape(-1)
+        want = torch.where(upd == 0, base, (base.float() + upd).to(torch.bfloat16))
+        assert torch.equal(o.reshape(-1).view(torch.int16), want.view(torch.int16)), f"tensor {q}"
+    assert seen == eq
     del th0, th1, out, ws
     torch.cuda.empty_cache()
 
