@@ -8,8 +8,9 @@
  * every float operation below is one IEEE operation.
  *
  * Precision.  Values are computed in binary64.  The decisions that the GPU
- * takes in binary32 -- the magnitude key that TopKMask ranks, and the sign of
- * the TIES election sum -- are taken here in binary32 in the same order, so
+ * takes in binary32 -- the magnitude key that TopKMask ranks, the sign of the
+ * TIES election sum, and RAM's activity test |tau| > eps_act -- are taken here
+ * in binary32 in the same order, so
  * that both sides decide identically.
  *
  * Parity status: every function here is pinned by tests (hand-worked cases,
