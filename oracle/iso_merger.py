@@ -1,0 +1,144 @@
+"""Frame-space ISO-Merger (App. E, Algorithm 1) -- TEST INFRASTRUCTURE ONLY.
+
+A plain binary64 numpy restatement of the paper's merge of K expert weight
+matrices that share one base, taken step by step in the paper's order and
+notation.  Library routines serve as steps where the paper names the
+operation (the thin SVD, matrix products); nothing is blocked, fused or
+reordered.  Only ``tests/``, ``__graft_entry__.smoke()`` and ``bench.py``'s
+CPU-baseline leg may import it; it shares no code with the CUDA library.
+
+For each 2-D weight matrix (App. E "Setup" to "Retraction and
+reconstruction"):
+
+1. thin SVDs  W_0 = U_0 S_0 V_0^T  and  W_i = U_i S_i V_i^T  (q = min(m, n)
+   singular values, in descending order);
+2. joint sign canonicalisation of each expert's mode k against the base:
+   s_ik = sign(<u_0k, u_ik>) with sign(0) := 1, u_ik <- s_ik u_ik,
+   v_ik <- s_ik v_ik;
+3. frame displacements dU_i = U_i - U_0, dV_i = V_i - V_0 and their Stiefel
+   tangent projections  Pi_{U_0}(D) = D - U_0 sym(U_0^T D);
+4. top-k_keep mode mask: k_keep = round(rho_keep q), taken as
+   floor(rho_keep q + 1/2); the trailing columns of both tangents are zeroed;
+5. first-order effect proxies g_i = xi~_Ui S_0 V_0^T + U_0 S_0 xi~_Vi^T,
+   Gram Gamma_ij = <g_i, g_j>_F, retention coefficients from
+   (Gamma + ridge I) c = diag Gamma on the non-zero proxies, clipped to
+   [c_min, c_max] (the element-wise path's own pinned solve);
+6. aggregate tangents xi_U* = Pi_{U_0}(sum_i c_i xi~_Ui) (same for V),
+   polar retraction U* = polar(U_0 + xi_U*) with polar(X) = P Q^T from the
+   thin SVD X = P S Q^T, and W* = U* S_0 V*^T.
+
+One-dimensional parameters take the task-vector average (App. E "Merged
+parameter scope"), which the element-wise oracle already provides.
+
+Parity status: pinned (tests/test_oracle_iso_merger.py) by the identities the
+paper states -- the tangent condition, (U_0 + xi)^T (U_0 + xi) = I + xi^T xi,
+polar(X) = X (X^T X)^{-1/2} for full column rank -- and by the spectrum of
+W* equal to that of W_0, fixed points (experts equal to the base, zero
+coefficients), sign-flip invariance, the mode mask, the single-expert
+second-order accuracy of the retraction, and identical experts.
+"""
+from __future__ import annotations
+
+import numpy as np
+
+from . import retention as _retention
+
+
+def sym(A: np.ndarray) -> np.ndarray:
+    """sym(A) = (A + A^T) / 2."""
+    return 0.5 * (A + A.T)
+
+
+def tangent_project(U0: np.ndarray, D: np.ndarray) -> np.ndarray:
+    """Orthogonal projection onto the tangent space of the Stiefel manifold
+    at U0: Pi_{U0}(D) = D - U0 sym(U0^T D)."""
+    return D - U0 @ sym(U0.T @ D)
+
+
+def thin_svd(W: np.ndarray):
+    """W = U diag(S) V^T with q = min(m, n) singular values, descending."""
+    U, S, Vt = np.linalg.svd(np.asarray(W, np.float64), full_matrices=False)
+    return U, S, Vt.T
+
+
+def canonicalize_signs(U0: np.ndarray, U: np.ndarray, V: np.ndarray):
+    """Joint per-mode sign alignment of (U, V) against the base frame U0:
+    s_k = sign(<u0_k, u_k>), sign(0) := 1; both frames take the same sign,
+    which leaves U diag(S) V^T unchanged."""
+    s = np.sign(np.sum(U0 * U, axis=0))
+    s[s == 0] = 1.0
+    return U * s, V * s, s
+
+
+def k_keep_of(rho_keep: float, q: int) -> int:
+    """k_keep = round(rho_keep q), rounding halves up (floor(x + 1/2)),
+    clamped to [0, q]."""
+    k = int(np.floor(rho_keep * q + 0.5))
+    return max(0, min(q, k))
+
+
+def keep_mask(xi: np.ndarray, k_keep: int) -> np.ndarray:
+    """xi D_keep: the leading k_keep columns kept, the trailing ones zeroed."""
+    out = xi.copy()
+    out[:, k_keep:] = 0.0
+    return out
+
+
+def effect_proxy(xiU: np.ndarray, xiV: np.ndarray, U0: np.ndarray, S0: np.ndarray,
+                 V0: np.ndarray) -> np.ndarray:
+    """g = xi_U S_0 V_0^T + U_0 S_0 xi_V^T."""
+    return (xiU * S0) @ V0.T + (U0 * S0) @ xiV.T
+
+
+def polar(X: np.ndarray) -> np.ndarray:
+    """polar(X) = P Q^T from the thin SVD X = P S Q^T."""
+    P, _, Q = thin_svd(X)
+    return P @ Q.T
+
+
+def merge_matrix(W0, experts, rho_keep=0.9, ridge=1e-12, c_min=0.0, c_max=1.5):
+    """ISO-Merger of one 2-D weight matrix (Algorithm 1, inner loop).
+
+    W0       base matrix (m x n)
+    experts  list of K expert matrices of the same shape (checkpoints W_i)
+
+    Returns a dict: ``W`` (merged matrix, binary64), ``U``, ``V`` (merged
+    frames), ``S0``, ``U0``, ``V0``, ``k_keep``, ``coef`` (c*), ``gram``
+    (Gamma), ``g`` (proxies), ``xiU`` / ``xiV`` (masked tangents per expert),
+    ``xiU_star`` / ``xiV_star`` (aggregate tangents) and ``signs``.
+    """
+    W0 = np.asarray(W0, np.float64)
+    U0, S0, V0 = thin_svd(W0)
+    q = S0.size
+    kk = k_keep_of(rho_keep, q)
+    K = len(experts)
+    xiU, xiV, g, signs = [], [], [], []
+    for Wi in experts:
+        Ui, _, Vi = thin_svd(Wi)
+        Ui, Vi, s = canonicalize_signs(U0, Ui, Vi)
+        signs.append(s)
+        dU, dV = Ui - U0, Vi - V0
+        xu = keep_mask(tangent_project(U0, dU), kk)
+        xv = keep_mask(tangent_project(V0, dV), kk)
+        xiU.append(xu)
+        xiV.append(xv)
+        g.append(effect_proxy(xu, xv, U0, S0, V0))
+    gram = np.zeros((K, K), np.float64)
+    for i in range(K):
+        for j in range(K):
+            gram[i, j] = float(np.sum(g[i] * g[j]))
+    # zero-norm proxies are dropped inside the solve (coefficient 0)
+    coef = _retention(gram, ridge, c_min, c_max)
+    aggU = np.zeros_like(U0)
+    aggV = np.zeros_like(V0)
+    for i in range(K):
+        aggU += coef[i] * xiU[i]
+        aggV += coef[i] * xiV[i]
+    xiU_star = tangent_project(U0, aggU)
+    xiV_star = tangent_project(V0, aggV)
+    U_star = polar(U0 + xiU_star)
+    V_star = polar(V0 + xiV_star)
+    W_star = (U_star * S0) @ V_star.T
+    return {"W": W_star, "U": U_star, "V": V_star, "S0": S0, "U0": U0, "V0": V0,
+            "k_keep": kk, "coef": coef, "gram": gram, "g": g, "xiU": xiU, "xiV": xiV,
+            "xiU_star": xiU_star, "xiV_star": xiV_star, "signs": signs}

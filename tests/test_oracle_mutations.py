@@ -60,3 +60,37 @@ def test_pins_catch_mutation(name, tmp_path):
                         os.path.join(ROOT, "tests", "test_oracle_pins.py")],
                        cwd=ROOT, env=env, capture_output=True, text=True, timeout=600)
     assert r.returncode != 0, f"pins did not catch mutation {name}:\n{r.stdout[-2000:]}"
+
+
+# ---------------------------------------------------------------------------
+# the frame-space ISO-Merger oracle (numpy): the same scheme on its source
+# ---------------------------------------------------------------------------
+MERGER_SRC = os.path.join(ROOT, "oracle", "iso_merger.py")
+MERGER_MUTATIONS = {
+    "sym_drops_half": ("return 0.5 * (A + A.T)", "return (A + A.T)"),
+    "projection_skipped": ("return D - U0 @ sym(U0.T @ D)", "return D"),
+    "sign_zero_negative": ("s[s == 0] = 1.0", "s[s == 0] = -1.0"),
+    "no_sign_canonicalization": ("Ui, Vi, s = canonicalize_signs(U0, Ui, Vi)", "s = np.ones(Ui.shape[1])"),
+    "mask_keeps_every_mode": ("out[:, k_keep:] = 0.0", "out[:, k_keep:] *= 1.0"),
+    "k_keep_truncates": ("k = int(np.floor(rho_keep * q + 0.5))", "k = int(np.floor(rho_keep * q))"),
+    "proxy_drops_v_motion": ("return (xiU * S0) @ V0.T + (U0 * S0) @ xiV.T", "return (xiU * S0) @ V0.T"),
+    "aggregate_not_projected": ("xiU_star = tangent_project(U0, aggU)", "xiU_star = aggU"),
+    "retraction_without_polar": ("U_star = polar(U0 + xiU_star)", "U_star = U0 + xiU_star"),
+    "gram_diagonal_only": ("gram[i, j] = float(np.sum(g[i] * g[j]))", "gram[i, j] = float(np.sum(g[i] * g[i]))"),
+    "coefficients_unused": ("aggU += coef[i] * xiU[i]", "aggU += xiU[i]"),
+}
+
+
+@pytest.mark.parametrize("name", sorted(MERGER_MUTATIONS))
+def test_merger_pins_catch_mutation(name, tmp_path):
+    old, new = MERGER_MUTATIONS[name]
+    src = open(MERGER_SRC).read()
+    assert src.count(old) == 1, f"mutation anchor not found: {name}"
+    src = src.replace("from . import retention as _retention", "from oracle import retention as _retention")
+    path = tmp_path / "iso_merger_mut.py"
+    path.write_text(src.replace(old, new))
+    env = dict(os.environ, ISO_MERGER_PATH=str(path))
+    r = subprocess.run([sys.executable, "-m", "pytest", "-x", "-q", "-p", "no:cacheprovider",
+                        os.path.join(ROOT, "tests", "test_oracle_iso_merger.py")],
+                       cwd=ROOT, env=env, capture_output=True, text=True, timeout=600)
+    assert r.returncode != 0, f"pins did not catch mutation {name}:\n{r.stdout[-2000:]}"
