@@ -103,10 +103,20 @@ KERNEL_SOURCES = {
 }
 
 
+def _code_only(text: bytes) -> bytes:
+    """The source without comments and with whitespace collapsed: edits to
+    comments leave a kernel's hash, and so its profiled traffic, in place."""
+    import re
+    t = text.decode()
+    t = re.sub(r"/\*.*?\*/", " ", t, flags=re.S)
+    t = re.sub(r"//[^\n]*", " ", t)
+    return " ".join(t.split()).encode()
+
+
 def kernel_source_hash(kind=None):
     """sha1 of a kernel kind's sources and the shared headers (all sources
-    when kind is None): a profile's traffic applies only to the kernels it
-    measured."""
+    when kind is None), comments and whitespace left out: a profile's traffic
+    applies only to the kernels it measured."""
     import hashlib
     csrc = os.path.join(ROOT, "paper_2607_19331_gb300", "csrc")
     names = KERNEL_SOURCES.get(kind) if kind else None
@@ -118,7 +128,7 @@ def kernel_source_hash(kind=None):
     for f in files:
         h.update(os.path.basename(f).encode())
         with open(f, "rb") as fh:
-            h.update(fh.read())
+            h.update(_code_only(fh.read()))
     return h.hexdigest()[:16]
 
 

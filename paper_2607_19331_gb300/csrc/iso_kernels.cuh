@@ -38,12 +38,12 @@ template <bool CK> __global__ void k_fix(Plan P);
 // the expert count, and the Gram pass for any K (iso_merge.cu)
 template <typename XT, typename BT, bool CK, int KC> __global__ void k_apply(Plan P);
 // k_merge is compiled for TIES alone and for the other operators (ISO, whose
-// 1-D tensors take the plain average, and TA): TIES needs no coefficients
+// 1-D tensors take the plain average, TA and RAM): TIES needs no coefficients
 enum MergeOpFamily : int { OPF_TIES = 0, OPF_OTHER = 1 };
 template <typename XT, typename BT, bool CK, int KC, int OPF> __global__ void k_merge(Plan P);
 template <typename XT, typename BT, bool CK, int KC> __global__ void k_gramk(Plan P);
-// k_merge: resident blocks of TPB threads per SM
-// (eight experts and the coefficient-carrying family need more registers: one block)
+// k_merge: resident blocks of TPB threads per SM, two for every expert bound
+// and family (eight experts read their step from the stage entry by entry)
 constexpr int merge_blocks_per_sm(int KC, int OPF) { return 2; }
 // k_merge's dynamic shared memory (its per-warp staging ring)
 template <typename XT, typename BT, int KC, int OPF> int merge_smem_bytes();

@@ -400,9 +400,8 @@ struct StageGeom {
     static constexpr int SPT = TILE / (32 * E);              // steps per tile
     static constexpr int BB = E * (int)sizeof(BT);           // base bytes per lane per step (8, 16, 32)
     static constexpr int BYTES = KC * 512 + 32 * BB;         // one stage of one warp
-    // up to four experts: about 108 KB per block, two blocks per SM; eight
-    // experts: one block per SM (its registers hold the eight vectors of a
-    // step without spilling) with about 216 KB, a deeper ring
+    // two blocks per SM: about 108 KB of ring per block; a kernel run at one
+    // block per SM (BLK = 1) gets about 216 KB, a deeper ring
     static constexpr int BUDGET = BLK == 1 ? 221184 : 110592;
     static constexpr int DMAX = BLK == 1 ? 6 : 4;
     static constexpr int D0 = BUDGET / (WPB * BYTES);
