@@ -1,13 +1,17 @@
-"""The host logic of runs on several GPUs, as world-size-2 gloo process
-groups on the CPU: whole-tensor sharding (no data-path collective) and the
-step time taken as the maximum over ranks."""
+"""The host logic of runs on several GPUs, as gloo process groups on the
+CPU: whole-tensor sharding (no data-path collective), the step time taken as
+the maximum over ranks, and the exchange step of a selection unit split over
+ranks (histogram all-reduce per radix level, tie-count all-gather), whose
+stitched masks must equal the oracle's TopKMask of the whole unit."""
 import os
 import socket
 
 import pytest
 import torch.multiprocessing as mp
 
-from paper_2607_19331_gb300.shard import job_throughput, reduce_step_ms, shard_tensors
+import numpy as np
+
+from paper_2607_19331_gb300.shard import job_throughput, reduce_step_ms, shard_tensors, split_unit_select
 import synth
 
 
@@ -75,3 +79,72 @@ def test_two_ranks_gloo_step_time_is_the_maximum():
     assert not set(res[0][4]) & set(res[1][4])
     assert job_throughput(2 * 10**9, 2.0) == pytest.approx(1000.0)
     assert reduce_step_ms(3.5) == 3.5        # no process group in this process
+
+
+def _unit_keys(seed, n):
+    """A task vector with bf16-quantised values (long runs of exact ties) and
+    some exact zeros, as binary32; its magnitude keys."""
+    rng = np.random.default_rng(seed)
+    x = rng.normal(0, 1e-3, n).astype(np.float32)
+    x = np.round(x * 2 ** 14) / 2 ** 14            # few distinct magnitudes
+    x[rng.random(n) < 0.05] = 0.0
+    return x.astype(np.float32), x.astype(np.float32).view(np.uint32) & np.uint32(0x7FFFFFFF)
+
+
+def _split_worker(rank, world, port, q, seed, n, bounds, densities):
+    import torch.distributed as dist
+    os.environ["MASTER_ADDR"] = "127.0.0.1"
+    os.environ["MASTER_PORT"] = str(port)
+    dist.init_process_group("gloo", rank=rank, world_size=world)
+    try:
+        _, keys = _unit_keys(seed, n)
+        mine = keys[bounds[rank]:bounds[rank + 1]].astype(np.int64)
+
+        def local_hist(prefix, pshift, shift, nb):
+            sel = mine[(mine >> pshift) == prefix]
+            return np.bincount((sel >> shift) & (nb - 1), minlength=nb).tolist()
+
+        def local_ties(t):
+            return int(np.sum(mine == t))
+
+        out = []
+        for rho in densities:
+            s = split_unit_select(mine.size, rho, local_hist, local_ties)
+            tie = mine == s.t
+            mask = (mine > s.t) | (tie & (np.cumsum(tie) <= s.take))
+            out.append((rho, s, mask.astype(np.uint8)))
+        q.put((rank, out))
+    finally:
+        dist.destroy_process_group()
+
+
+@pytest.mark.parametrize("world,bounds", [(2, [0, 3000, 7001]), (3, [0, 2500, 2500, 7001]),
+                                          (4, [0, 1, 4000, 6999, 7001])])
+def test_split_unit_select_matches_whole_unit(world, bounds):
+    import oracle
+    n, seed = 7001, 5
+    densities = [0.0, 0.05, 0.2, 0.5, 1.0, 1.0 / 7001]
+    ctx = mp.get_context("spawn")
+    q = ctx.Queue()
+    port = _free_port()
+    procs = [ctx.Process(target=_split_worker, args=(r, world, port, q, seed, n, bounds, densities))
+             for r in range(world)]
+    for p in procs:
+        p.start()
+    res = dict(q.get(timeout=180) for _ in procs)
+    for p in procs:
+        p.join(timeout=60)
+        assert p.exitcode == 0
+    tau, _ = _unit_keys(seed, n)
+    for j, rho in enumerate(densities):
+        m_want, st = oracle.topk_unit(tau, oracle.k_of(rho, n))
+        stitched = np.concatenate([res[r][j][2] for r in range(world)])
+        assert np.array_equal(stitched, m_want), f"rho={rho}"
+        for r in range(world):
+            s = res[r][j][1]
+            assert s.k == st["k"] and s.t == st["thresh_key"]
+            assert s.count_above == st["count_above"]
+            if s.k:
+                assert s.ties_at_thresh == st["ties_at_thresh"] and s.ties_taken == st["ties_taken"]
+        if 0.0 < rho < 1.0 and rho * n > 100:
+            assert st["ties_at_thresh"] > st["ties_taken"] > 0      # the tie rule really splits ties
