@@ -257,3 +257,52 @@ def test_merge_ignores_the_svd_sign_choice(monkeypatch):
     assert calls["n"] >= 4
     np.testing.assert_allclose(got["coef"], ref["coef"], rtol=1e-12)
     np.testing.assert_allclose(got["W"], ref["W"], atol=1e-13)
+
+
+def test_gram_from_frame_products():
+    # <g_i, g_j>_F without the m x n proxies: with P_i = U0^T xi~_Ui and
+    # Q_i = V0^T xi~_Vi (U0, V0 orthonormal),
+    #   Gamma_ij = sum_k s_k^2 [(xi~_Ui^T xi~_Uj)_kk + (xi~_Vi^T xi~_Vj)_kk]
+    #              + tr(S P_i S Q_j) + tr(S P_j S Q_i)
+    rng = np.random.default_rng(70)
+    for m, n in ((30, 18), (18, 30)):
+        W0, *_ = _matrix(rng, m, n)
+        experts = [W0 + 0.05 * rng.normal(size=W0.shape) for _ in range(3)]
+        r = M.merge_matrix(W0, experts)
+        U0, V0, s = r["U0"], r["V0"], r["S0"]
+        P = [U0.T @ x for x in r["xiU"]]
+        Q = [V0.T @ x for x in r["xiV"]]
+        K = len(experts)
+        G = np.zeros((K, K))
+        for i in range(K):
+            for j in range(K):
+                d = np.sum(r["xiU"][i] * r["xiU"][j], axis=0) + np.sum(r["xiV"][i] * r["xiV"][j], axis=0)
+                G[i, j] = (np.sum(s * s * d) + np.trace((s[:, None] * P[i] * s[None, :]) @ Q[j])
+                           + np.trace((s[:, None] * P[j] * s[None, :]) @ Q[i]))
+        np.testing.assert_allclose(r["gram"], G, rtol=1e-11, atol=1e-14 * np.abs(G).max())
+
+
+def test_masked_tangent_base_coordinates_are_skew():
+    # U0^T xi_U = skew(U0^T dU) for the projected displacement, so
+    # U0^T xi~_U = skew(U0^T dU) D_keep: the aggregate's projection needs only
+    # q x q algebra, and the merged frame argument satisfies
+    # (U0 + xi*)^T (U0 + xi*) = I + xi*^T xi*
+    rng = np.random.default_rng(71)
+    W0, *_ = _matrix(rng, 26, 20)
+    experts = [W0 + 0.05 * rng.normal(size=W0.shape) for _ in range(2)]
+    r = M.merge_matrix(W0, experts)
+    U0, kk = r["U0"], r["k_keep"]
+    for i, E in enumerate(experts):
+        Ui, _, Vi = M.thin_svd(E)
+        Ui, Vi, _ = M.canonicalize_signs(U0, Ui, Vi)
+        A = U0.T @ (Ui - U0)
+        skew = 0.5 * (A - A.T)
+        skew[:, kk:] = 0.0
+        np.testing.assert_allclose(U0.T @ r["xiU"][i], skew, atol=1e-13)
+    agg = sum(c * x for c, x in zip(r["coef"], r["xiU"]))
+    B = sum(c * (U0.T @ x) for c, x in zip(r["coef"], r["xiU"]))
+    xi_star = agg - U0 @ (0.5 * (B + B.T))
+    np.testing.assert_allclose(r["xiU_star"], xi_star, atol=1e-13)
+    X = U0 + r["xiU_star"]
+    w, Ev = np.linalg.eigh(np.eye(U0.shape[1]) + r["xiU_star"].T @ r["xiU_star"])
+    np.testing.assert_allclose(r["U"], X @ (Ev / np.sqrt(w)) @ Ev.T, atol=1e-12)
