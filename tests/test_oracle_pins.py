@@ -521,3 +521,27 @@ def test_ram_single_expert_is_a_threshold_mask():
     want = np.where(np.abs(tt) > eps, th0.ravel().astype(np.float64) + tt, th0.ravel().astype(np.float64))
     np.testing.assert_array_equal(r["out64"][0], want)
     assert 0 < np.sum(np.abs(tt) > eps) < n
+
+
+def test_f32_to_bf16_exhaustive():
+    """Every binary32 bit pattern but the NaNs: the oracle's bit-level
+    round-to-nearest-even against torch's conversion, 2^24 patterns at a
+    time in reused buffers."""
+    import ctypes
+    lib = oracle._lib()
+    CH = 1 << 24
+    idx = np.arange(CH, dtype=np.uint32)
+    bits = np.empty(CH, np.uint32)
+    got = np.empty(CH, np.uint16)
+    want = torch.empty(CH, dtype=torch.bfloat16)
+    P = ctypes.c_void_p
+    for c in range(1 << 8):
+        np.add(idx, np.uint32(c * CH), out=bits)
+        x = bits.view(np.float32)
+        lib.orc_f32_to_bf16_array(P(x.ctypes.data), CH, P(got.ctypes.data))
+        want.copy_(torch.from_numpy(x))
+        w = want.view(torch.int16).numpy().view(np.uint16)
+        ok = (got == w) | np.isnan(x)
+        if not ok.all():
+            i = int(np.flatnonzero(~ok)[0])
+            raise AssertionError(f"pattern {bits[i]:#010x}: oracle {got[i]:#06x}, torch {w[i]:#06x}")
