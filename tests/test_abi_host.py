@@ -124,3 +124,43 @@ def test_missing_library_fails_loudly(monkeypatch):
     monkeypatch.setattr(_abi, "_lib", None)
     with pytest.raises(RuntimeError, match="not found"):
         _abi.lib()
+
+
+C_CLIENT = r"""
+#include "iso.h"
+#include <stdio.h>
+int main(void) {
+    iso_tensor t = {0};
+    t.data = (void*)0x10000; t.rows = 300; t.cols = 1000; t.dtype = ISO_BF16; t.is_1d = 0;
+    iso_merge_cfg c = {0};
+    c.op = ISO_OP_RAM; c.lambda = 1.0f; c.eps_act = 1e-5f; c.ridge = 1e-12; c.c_min = 0.0; c.c_max = 1.5;
+    c.topk.density = 0.2; c.topk.scope = ISO_SCOPE_BLOCK; c.topk.block_rows = 128; c.topk.block_cols = 128;
+    size_t mn = 0, full = 0;
+    int rc = iso_workspace_size(&t, 1, 2, &c, &mn, &full);
+    int64_t nu = 0;
+    int rc2 = iso_num_units(&t, 1, &c.topk, &nu);
+    c.eps_act = -1.0f;
+    int rc3 = iso_workspace_size(&t, 1, 2, &c, &mn, &full);
+    printf("%d %d %lld %d\n", rc, rc2, (long long)nu, rc3);
+    return (rc == ISO_OK && rc2 == ISO_OK && nu == 3 * 8 && rc3 == ISO_ERR_ARG && full >= mn && mn > 0) ? 0 : 1;
+}
+"""
+
+
+def test_header_is_plain_c(tmp_path):
+    """include/iso.h compiles as strict C99 and a C program links against the
+    library and calls its host-only entry points (no device work)."""
+    import shutil
+    import subprocess
+    gcc = shutil.which("gcc")
+    if gcc is None:
+        pytest.skip("gcc not available")
+    src = tmp_path / "client.c"
+    src.write_text(C_CLIENT)
+    exe = tmp_path / "client"
+    libdir = os.path.dirname(_abi.LIB_PATH)
+    subprocess.check_call([gcc, "-std=c99", "-Wall", "-Wextra", "-pedantic", "-Werror",
+                           "-I", os.path.join(ROOT, "include"), "-o", str(exe), str(src),
+                           "-L", libdir, "-liso_gb300", f"-Wl,-rpath,{libdir}"])
+    r = subprocess.run([str(exe)], capture_output=True, text=True, timeout=60)
+    assert r.returncode == 0, r.stdout + r.stderr
