@@ -186,6 +186,15 @@ def iso_merge(theta_0: List[torch.Tensor], experts: List[List[torch.Tensor]], op
               lam=1.0, ridge=1e-12, c_min=0.0, c_max=1.5, mask_1d=True, is_1d=None,
               workspace: Optional[Workspace] = None, stats=False, stream=None,
               ws_bytes: Optional[int] = None, eps_act=1e-5):
+    """Merge K experts into the base (iso_merge; iso_update for K = 1).
+
+    op is "ta", "ties", "iso" or "ram"; experts holds K lists of tensors
+    shaped like theta_0 (task vectors, or checkpoints when
+    experts_are_deltas is False).  density / scope / block configure the
+    TopKMask of TIES and ISO; lam scales TA, TIES and RAM; ridge / c_min /
+    c_max configure ISO's retention solve; eps_act is RAM's activity
+    threshold.  Returns the outputs (and the device-side stats when
+    stats=True)."""
     K = len(experts)
     n = len(theta_0)
     dev = theta_0[0].device
