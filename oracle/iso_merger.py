@@ -28,14 +28,17 @@ reconstruction"):
    thin SVD X = P S Q^T, and W* = U* S_0 V*^T.
 
 One-dimensional parameters take the task-vector average (App. E "Merged
-parameter scope"), which the element-wise oracle already provides.
+parameter scope"); ``merge_model`` runs Algorithm 1's loop over a parameter
+list and rounds each result once to the base's encoding.
 
 Parity status: pinned (tests/test_oracle_iso_merger.py) by the identities the
 paper states -- the tangent condition, (U_0 + xi)^T (U_0 + xi) = I + xi^T xi,
 polar(X) = X (X^T X)^{-1/2} for full column rank -- and by the spectrum of
 W* equal to that of W_0, fixed points (experts equal to the base, zero
 coefficients), sign-flip invariance, the mode mask, the single-expert
-second-order accuracy of the retraction, and identical experts.
+third-order accuracy of the retraction, identical experts, the Gram and the
+aggregate projection in their q x q forms, and the model loop against the
+element-wise oracle's 1-D rule.
 """
 from __future__ import annotations
 
@@ -142,3 +145,41 @@ def merge_matrix(W0, experts, rho_keep=0.9, ridge=1e-12, c_min=0.0, c_max=1.5):
     return {"W": W_star, "U": U_star, "V": V_star, "S0": S0, "U0": U0, "V0": V0,
             "k_keep": kk, "coef": coef, "gram": gram, "g": g, "xiU": xiU, "xiV": xiV,
             "xiU_star": xiU_star, "xiV_star": xiV_star, "signs": signs}
+
+
+def merge_model(theta0, experts, is_1d=None, rho_keep=0.9, ridge=1e-12, c_min=0.0, c_max=1.5):
+    """Algorithm 1 over a parameter list.
+
+    theta0   list of base tensors (uint16 bfloat16 bits or float32), 2-D
+             matrices as (m, n) arrays
+    experts  K lists of checkpoints in the same encoding
+    is_1d    per tensor: 1-D parameters take the task-vector average
+             w_0 + (1/K) sum_i (w_i - w_0); every other tensor is merged as a
+             matrix with ``merge_matrix``
+
+    Returns the merged tensors in the base encoding (one rounding from
+    binary64) and the per-matrix results (None for 1-D tensors)."""
+    from . import BF16, F32, load, to_dtype
+    K = len(experts)
+    if is_1d is None:
+        is_1d = [np.asarray(a).ndim == 1 for a in theta0]
+    out, detail = [], []
+    for t, a in enumerate(theta0):
+        a = np.asarray(a)
+        code = F32 if a.dtype == np.float32 else BF16
+        _, w0 = load(a)
+        ws = [load(np.asarray(experts[i][t]))[1] for i in range(K)]
+        if is_1d[t]:
+            s = np.zeros_like(w0)
+            for w in ws:
+                s += w - w0
+            # an update of exactly zero keeps the base's bits (a -0 stays -0)
+            merged = np.where(s == 0.0, w0, w0 + s / K)
+            detail.append(None)
+        else:
+            r = merge_matrix(w0.reshape(a.shape), [w.reshape(a.shape) for w in ws],
+                             rho_keep, ridge, c_min, c_max)
+            merged = r["W"].reshape(-1)
+            detail.append(r)
+        out.append(to_dtype(merged, code).reshape(a.shape))
+    return out, detail

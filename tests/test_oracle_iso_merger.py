@@ -306,3 +306,40 @@ def test_masked_tangent_base_coordinates_are_skew():
     X = U0 + r["xiU_star"]
     w, Ev = np.linalg.eigh(np.eye(U0.shape[1]) + r["xiU_star"].T @ r["xiU_star"])
     np.testing.assert_allclose(r["U"], X @ (Ev / np.sqrt(w)) @ Ev.T, atol=1e-12)
+
+
+def test_model_loop_matrices_and_vectors():
+    # Algorithm 1's outer loop: matrices through the frame-space merge, 1-D
+    # parameters through the task-vector average (the element-wise oracle's
+    # ISO 1-D rule), each rounded once to the base's encoding
+    import oracle
+    rng = np.random.default_rng(80)
+    W0, *_ = _matrix(rng, 24, 16, spread=0.02)
+    b0 = rng.normal(0, 0.02, 16)
+    b0[3] = -0.0                                  # kept as -0 where every expert agrees
+    theta0 = [oracle.f64_to_bf16(W0), oracle.f64_to_bf16(b0), W0.astype(np.float32)]
+    experts = []
+    for i in range(3):
+        b = b0 + 1e-3 * rng.normal(size=16)
+        b[3] = -0.0
+        experts.append([oracle.f64_to_bf16(W0 + 1e-3 * rng.normal(size=W0.shape)),
+                        oracle.f64_to_bf16(b),
+                        (W0 + 1e-3 * rng.normal(size=W0.shape)).astype(np.float32)])
+    out, detail = M.merge_model(theta0, experts, is_1d=[False, True, False])
+    assert out[0].dtype == np.uint16 and out[1].dtype == np.uint16 and out[2].dtype == np.float32
+    assert detail[1] is None
+    # the 1-D rule: the element-wise oracle's ISO 1-D average, bit for bit
+    r1 = oracle.merge([theta0[1]], [[e[1]] for e in experts], oracle.ISO, experts_are_deltas=False,
+                      is_1d=[True])
+    np.testing.assert_array_equal(out[1], r1["out"][0])
+    assert out[1][3] == 0x8000
+    # matrices: the per-matrix merge of the decoded values, rounded once
+    for t in (0, 2):
+        w0 = oracle.load(theta0[t])[1].reshape(theta0[t].shape)
+        ws = [oracle.load(e[t])[1].reshape(theta0[t].shape) for e in experts]
+        r = M.merge_matrix(w0, ws)
+        np.testing.assert_array_equal(out[t], oracle.to_dtype(r["W"].reshape(-1),
+                                                              oracle.F32 if t == 2 else oracle.BF16)
+                                      .reshape(theta0[t].shape))
+        s = np.linalg.svd(detail[t]["W"], compute_uv=False)
+        np.testing.assert_allclose(s, np.linalg.svd(w0, compute_uv=False), rtol=1e-12)
