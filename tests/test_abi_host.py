@@ -164,3 +164,34 @@ def test_header_is_plain_c(tmp_path):
                            "-L", libdir, "-liso_gb300", f"-Wl,-rpath,{libdir}"])
     r = subprocess.run([str(exe)], capture_output=True, text=True, timeout=60)
     assert r.returncode == 0, r.stdout + r.stderr
+
+
+def test_workspace_at_full_model_sizes():
+    """Host-only sizing at the Qwen2.5-7B shapes (254 tensors, 7.6e9 entries):
+    one GLOBAL unit over the whole task vector plans as one group of a few
+    GB; per-tensor scopes can run in groups down to the largest tensor; RAM,
+    which selects nothing, needs only the tables; a tensor of 2^32 entries is
+    refused."""
+    import synth
+    L = _abi.lib()
+    shapes = synth.qwen_shapes("qwen7b")
+    mn, full = ctypes.c_size_t(), ctypes.c_size_t()
+
+    def size(op, scope, K, dtype, density):
+        ts = _arr(*[_fake(r, c, dtype=dtype, is_1d=int(o)) for r, c, o in shapes])
+        cfg = iso.merge_cfg(op, density, scope)
+        rc = L.iso_workspace_size(ts, len(shapes), K, ctypes.byref(cfg), ctypes.byref(mn), ctypes.byref(full))
+        assert rc == 0, (op, scope, rc)
+        return mn.value, full.value
+
+    g_mn, g_full = size("ties", "global", 1, _abi.ISO_BF16, 0.2)
+    assert g_mn == g_full and 1e9 < g_full < 8e9
+    t_mn, t_full = size("iso", "tensor", 1, _abi.ISO_BF16, 0.05)
+    assert t_mn < t_full < 20e9
+    k_mn, k_full = size("ties", "tensor", 8, _abi.ISO_F32, 0.1)
+    assert k_mn < k_full < 20e9
+    r_mn, r_full = size("ram", "tensor", 8, _abi.ISO_F32, 0.0)
+    assert r_full < (1 << 20)
+    cfg = iso.merge_cfg("ties", 0.1)
+    big = _arr(_fake(1 << 16, 1 << 16))
+    assert L.iso_workspace_size(big, 1, 1, ctypes.byref(cfg), None, None) == _abi.ISO_ERR_UNSUPPORTED
