@@ -51,9 +51,17 @@ __device__ __forceinline__ void tensor_params(const Plan& P, int t, int K, Tenso
         tp.xs[i] = P.xptr[i * P.n_tensors + t];
         tp.cf[i] = tp.iso2d ? (float)P.coef[(long long)t * K + i] : 0.0f;
         if (!tp.blk) {
-            const Unit& U = P.units[(long long)i * P.n_units + ((P.scope == ISO_SCOPE_GLOBAL) ? 0 : d.unit)];
-            tp.sp[i].t = U.t;
-            tp.sp[i].cut = U.cut;
+            if (P.scope == ISO_SCOPE_GLOBAL && !(d.flags & TF_TRIM)) {
+                // outside the one GLOBAL unit (a 1-D tensor TIES leaves
+                // untrimmed): every entry kept, as an untrimmed tensor's own
+                // unit record says in the other scopes
+                tp.sp[i].t = 0;
+                tp.sp[i].cut = CUT_ALL;
+            } else {
+                const Unit& U = P.units[(long long)i * P.n_units + ((P.scope == ISO_SCOPE_GLOBAL) ? 0 : d.unit)];
+                tp.sp[i].t = U.t;
+                tp.sp[i].cut = U.cut;
+            }
         }
     }
 }
