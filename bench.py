@@ -412,6 +412,8 @@ def cpu_baseline(name, budget_s=15.0, seed=0, rho=None):
         return cpu_baseline_sweep(name, density, scope, seed)
     shapes, order = cpu_sample(name, seed)
     orc_op = {"ta": oracle.TA, "ties": oracle.TIES, "iso": oracle.ISO, "ram": oracle.RAM}[op]
+    orc_scope = {"tensor": oracle.SCOPE_TENSOR, "block": oracle.SCOPE_BLOCK,
+                 "global": oracle.SCOPE_GLOBAL}[scope]
     done, params, spent = [], 0, 0.0
     for q in order:
         s = shapes[q]
@@ -425,8 +427,9 @@ def cpu_baseline(name, budget_s=15.0, seed=0, rho=None):
             a = [th0[0].view(-1).view(__import__("torch").int16).numpy().view(np.uint16).reshape(s[0], s[1])]
             ex = [[e[0].reshape(s[0], s[1]).numpy()] for e in taus]
         t = time.perf_counter()
+        # the workload's scope on the sampled tensor (GLOBAL: the sample's own unit)
         oracle.merge(a, ex, orc_op, experts_are_deltas=(inputs != "ckpt_bf16"), density=density,
-                     is_1d=[s[2]])
+                     scope=orc_scope, is_1d=[s[2]])
         spent += time.perf_counter() - t
         params += s[0] * s[1]
         done.append(q)
