@@ -1,9 +1,10 @@
 """Benchmark of the whole-model delta -> TopKMask -> update/merge pass.
 
 One step = one pass of the hot path over a full synthetic parameter set held
-in HBM.  Default workload: the Qwen2.5-1.5B-shaped masked ISO update (bf16
-base and RL checkpoint, 253 tensors, 1,543,655,424 parameters, per-tensor
-TopKMask density 5 %).  Other workloads (--workload) are for investigation.
+in HBM.  Default workload: the Qwen2.5-7B-shaped fused delta + mask + update
+(bf16 base and RL checkpoint, 254 tensors, 7,615,483,904 parameters,
+per-tensor TopKMask density 5 %, masked ISO update).  Other workloads
+(--workload) are for investigation.
 
     python bench.py [--gpus N] [--steps K] [--warmup W] [--impl mine|reference]
 
@@ -282,8 +283,12 @@ def run_mine(args):
         step()
     torch.cuda.synchronize()
     barrier()
-    os.makedirs(os.path.join(ROOT, "gpurun_out"), exist_ok=True)
-    clocks = Clocks(local, os.path.join(ROOT, "gpurun_out", f"clocks_rank{rank}.csv")) if rank == 0 else None
+    clocks = None
+    if rank == 0:
+        import tempfile
+        fd, clock_path = tempfile.mkstemp(prefix="iso_clocks_", suffix=".csv")
+        os.close(fd)
+        clocks = Clocks(local, args.clock_log or clock_path)
     time.sleep(0.3 if clocks else 0)
     l0 = iso.launch_count()
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
@@ -493,7 +498,7 @@ def main():
     ap.add_argument("--steps", type=int, default=30)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", choices=["mine", "reference"], default="mine")
-    ap.add_argument("--workload", choices=sorted(WORKLOADS), default="qwen1.5b_update")
+    ap.add_argument("--workload", choices=sorted(WORKLOADS), default="qwen7b_update")
     ap.add_argument("--two-pass", action="store_true",
                     help="run the K = 1 update as its two-pass form (count, then apply) "
                          "instead of the fused single pass")
@@ -505,6 +510,9 @@ def main():
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-budget", type=float, default=12.0)
+    ap.add_argument("--clock-log", default=None,
+                    help="keep the nvidia-smi clock samples of the timed region in this CSV "
+                         "(default: a temporary file)")
     ap.add_argument("--layers", type=int, default=None,
                     help="decoder layers of the shape set (default: the model's own); "
                          "smaller cases are for profiling only")

@@ -185,7 +185,10 @@ int32_t iso_topk_mask(const iso_tensor* tau, int32_t n_tensors, const iso_topk_c
                       uint32_t* const* mask_bits, const iso_merge_stats* stats,
                       void* workspace, size_t ws_bytes, void* stream);
 
-/* The K = 1 masked update of a base by one expert:
+/* The K = 1 masked update of a base by one expert, the single-expert case of
+ * the merge operators (App. F: TIES trim and scale; Sec. 4.2 and App. E:
+ * the retention system with K = 1; App. E "Merged parameter scope" for 1-D
+ * tensors):
  *   out = theta_0 + c * TopKMask(|tau|) * tau,   tau = update (update_is_delta = 1)
  *                                               or update - theta_0 (a checkpoint)
  * with c = lambda for TIES, c = clip(Gamma / (Gamma + ridge)) for ISO (Gamma the

@@ -33,7 +33,10 @@ static float bits_f32(uint32_t u) { float f; memcpy(&f, &u, 4); return f; }
 float orc_bf16_to_f32(uint16_t b) { return bits_f32((uint32_t)b << 16); }
 
 /* Round a binary32 to bfloat16, nearest with ties to even (IEEE 754
- * roundTiesToEven): add half an ulp minus one, plus the kept LSB. */
+ * roundTiesToEven).  The integer form is the standard rounding-bias method
+ * for truncating formats (as in TensorFlow's float-to-bfloat16 rounding):
+ * add half an ulp of the result minus one, plus the kept least-significant
+ * bit, so an exact half rounds up only when that bit is odd; then truncate. */
 uint16_t orc_f32_to_bf16(float f) {
     uint32_t u = f32_bits(f);
     if ((u & 0x7FFFFFFFu) > 0x7F800000u) return (uint16_t)((u >> 16) | 0x0040u); /* quiet NaN */

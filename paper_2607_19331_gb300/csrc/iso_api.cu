@@ -145,13 +145,17 @@ int resident_grid(K kernel, int tpb, int smem, int sms, int* grid) {
 // ---------------------------------------------------------------------------
 bool aligned16(const void* p) { return ((uintptr_t)p & 15u) == 0; }
 
+// rows * cols; only called on descriptors that check_tensor accepted, whose
+// extents are each below 2^32 and whose product is below 2^32
 long long numel_of(const iso_tensor& t) { return t.rows * t.cols; }
 
 int check_tensor(const iso_tensor& t) {
     if (t.rows < 0 || t.cols < 0) return ISO_ERR_SHAPE;
     if (t.dtype != ISO_BF16 && t.dtype != ISO_F32) return ISO_ERR_DTYPE;
     if (t.is_1d != 0 && t.is_1d != 1) return ISO_ERR_ARG;
-    if (t.rows > 0 && t.cols > (long long)1 << 40) return ISO_ERR_SHAPE;
+    // each extent below 2^32 before the product is formed, so rows * cols
+    // cannot overflow 64 bits
+    if (t.rows >= (1LL << 32) || t.cols >= (1LL << 32)) return ISO_ERR_UNSUPPORTED;
     const long long n = numel_of(t);
     if (n >= (1LL << 32)) return ISO_ERR_UNSUPPORTED;
     if (n > 0 && t.data == nullptr) return ISO_ERR_ARG;
@@ -686,6 +690,40 @@ int run_call(Call& c, void* workspace, size_t ws_bytes, const iso_merge_stats* s
     return ISO_OK;
 }
 
+// out[t] may coincide with theta_0[t] exactly (an in-place update) and must
+// share no byte with any other tensor of the call: another base tensor, any
+// expert or another output.  The passes read inputs after outputs have been
+// written (the fused pass's corrections, the K >= 2 staging), so a partial or
+// cross-tensor overlap would give wrong results without an error.
+int check_out_overlap(const iso_tensor* theta_0, const iso_tensor* experts, int K,
+                      const iso_tensor* out, int n) {
+    struct Span { uintptr_t a, b; int kind, t; };   // kind 0: output, 1: base, 2: expert
+    std::vector<Span> v;
+    v.reserve((size_t)n * (K + 2));
+    auto add = [&](const iso_tensor& d, int kind, int t) {
+        const long long bytes = numel_of(d) * (d.dtype == ISO_BF16 ? 2 : 4);
+        if (bytes > 0) v.push_back({(uintptr_t)d.data, (uintptr_t)d.data + (uintptr_t)bytes, kind, t});
+    };
+    for (int t = 0; t < n; ++t) {
+        add(out[t], 0, t);
+        add(theta_0[t], 1, t);
+        for (int i = 0; i < K; ++i) add(experts[(size_t)i * n + t], 2, t);
+    }
+    std::sort(v.begin(), v.end(), [](const Span& x, const Span& y) { return x.a < y.a; });
+    for (size_t p = 0; p < v.size(); ++p) {
+        for (size_t q = p + 1; q < v.size() && v[q].a < v[p].b; ++q) {
+            const Span& x = v[p];
+            const Span& y = v[q];
+            if (x.kind != 0 && y.kind != 0) continue;            // inputs may share memory
+            const Span& o = x.kind == 0 ? x : y;
+            const Span& w = x.kind == 0 ? y : x;
+            if (w.kind == 1 && w.t == o.t && w.a == o.a && w.b == o.b) continue;   // in place
+            return ISO_ERR_ARG;
+        }
+    }
+    return ISO_OK;
+}
+
 void set_trim(Call& c, const iso_tensor* tens) {
     c.trim.assign(c.n, 0);
     c.trims = false;
@@ -720,9 +758,9 @@ int build_merge_call(Call& c, const iso_tensor* theta_0, const iso_tensor* exper
             ISO_TRY(check_tensor(x));
             if (!same_shape(x, theta_0[t])) return ISO_ERR_SHAPE;
             if (x.dtype != experts[0].dtype) return ISO_ERR_DTYPE;
-            if (numel_of(x) > 0 && x.data == out[t].data) return ISO_ERR_ARG;   // out may alias the base only
         }
     }
+    ISO_TRY(check_out_overlap(theta_0, experts, K, out, n));
     c.base = theta_0;
     c.x = experts;
     c.out = out;

@@ -9,3 +9,21 @@ if ROOT not in sys.path:
 def pytest_configure(config):
     config.addinivalue_line("markers", "gpu: needs a CUDA GPU (sm_103a) and the built library")
     config.addinivalue_line("markers", "slow: long-running")
+
+
+def pytest_terminal_summary(terminalreporter, exitstatus, config):
+    """The worst value error each parity check observed against the oracle:
+    relative error for binary32 outputs, bfloat16 ulps for bfloat16 outputs,
+    and the entries that needed the cancellation bound of parity_util."""
+    try:
+        from parity_util import WORST
+    except ImportError:
+        return
+    if not WORST:
+        return
+    tr = terminalreporter
+    tr.section("worst observed value error against the oracle")
+    for what, (worst, n, n_cancel, kind) in sorted(WORST.items()):
+        unit = "ulp (bf16)" if kind == "ulp" else "relative (f32)"
+        tr.write_line(f"{what}: {worst:.3g} {unit} over {n} entries; "
+                      f"{n_cancel} on the cancellation bound")

@@ -113,6 +113,24 @@ def test_validation_rejects_before_launch():
     huge = _arr(_fake(1 << 16, 1 << 16))
     assert upd(huge, _arr(_fake(1 << 16, 1 << 16, ptr=0x20000)), _arr(_fake(1 << 16, 1 << 16, ptr=0x30000))) \
         == _abi.ISO_ERR_UNSUPPORTED
+    # extents whose product wraps 64 bits (2^33 x 2^31 = 2^64 -> 0) are rejected
+    # before the product is formed
+    wrap = _arr(_fake(1 << 33, 1 << 31))
+    assert upd(wrap, _arr(_fake(1 << 33, 1 << 31, ptr=0x20000)), _arr(_fake(1 << 33, 1 << 31, ptr=0x30000))) \
+        == _abi.ISO_ERR_UNSUPPORTED
+    assert upd(_arr(_fake(1, 1 << 32)), _arr(_fake(1, 1 << 32, ptr=0x20000)),
+               _arr(_fake(1, 1 << 32, ptr=0x30000))) == _abi.ISO_ERR_UNSUPPORTED
+    # out may coincide with its own base (in place; tested on the GPU), and overlap nothing else
+    assert upd(a, b, _arr(_fake(8, 8, ptr=0x10010))) == _abi.ISO_ERR_ARG            # partial overlap with the base
+    assert upd(a, b, _arr(_fake(8, 8, ptr=0x20000 + 64))) == _abi.ISO_ERR_ARG       # partial overlap with the expert
+    two_b = _arr(_fake(8, 8), _fake(8, 8, ptr=0x11000))
+    two_x = _arr(_fake(8, 8, ptr=0x20000), _fake(8, 8, ptr=0x21000))
+    assert upd(two_b, two_x, _arr(_fake(8, 8, ptr=0x30000), _fake(8, 8, ptr=0x20000 + 96)), n=2) \
+        == _abi.ISO_ERR_ARG                                                          # out[1] inside expert 0
+    assert upd(two_b, two_x, _arr(_fake(8, 8, ptr=0x30000), _fake(8, 8, ptr=0x10000)), n=2) \
+        == _abi.ISO_ERR_ARG                                                          # out[1] on base[0]
+    assert upd(two_b, two_x, _arr(_fake(8, 8, ptr=0x30000), _fake(8, 8, ptr=0x30040)), n=2) \
+        == _abi.ISO_ERR_ARG                                                          # outputs overlap
     K9 = (IsoTensor * 9)(*[_fake(8, 8, ptr=0x50000 + 0x1000 * i) for i in range(9)])
     assert L.iso_merge(a, K9, 9, 1, o, 1, ctypes.byref(cfg), ws, 1 << 20, None, None) == _abi.ISO_ERR_UNSUPPORTED
     # an empty list is a no-op that needs no workspace and no device

@@ -64,14 +64,17 @@ def test_full_size_qwen7b_update_sampled():
     torch.cuda.synchronize()
     assert int(st.status.item()) == 0
     units = st.units_numpy()[0]
-    picks = [_qwen7b_index(0, "k"), _qwen7b_index(0, "norm1"), _qwen7b_index(13, "v"),
-             _qwen7b_index(27, "down"), _qwen7b_index(27, "o")]
+    # the embedding and lm_head (152064 x 3584, 545 M entries each) are the
+    # largest units: the most tiles, band records and tie-scan work per unit
+    picks = [0, len(shapes) - 1, _qwen7b_index(0, "k"), _qwen7b_index(0, "norm1"),
+             _qwen7b_index(13, "v"), _qwen7b_index(27, "down"), _qwen7b_index(27, "o")]
     for q in picks:
         r_, c_, one = shapes[q]
         a, b = to_np(th0[q]), to_np(th1[q])
         r = oracle.update([a.reshape(r_, c_)], [b.reshape(r_, c_)], oracle.ISO, update_is_delta=False,
                           density=0.05, is_1d=[one])
-        assert_values_close(to_np(out[q]), r["out64"][0], r["mag"][0], f"7B tensor {q}")
+        assert_values_close(to_np(out[q]), r["out64"][0], r["mag"][0], f"7B tensor {q}",
+                            op="iso", K=1)
         assert_units_equal(units[q:q + 1], r["units"][0], f"7B unit {q}")
     del th0, th1, out, ws
     torch.cuda.empty_cache()
@@ -149,7 +152,7 @@ def test_density_sweep_full_size(rho):
         assert np.array_equal(unpack_mask(masks[0], delta.numel()), r["masks"][0][0]), what + " mask"
         assert_units_equal(mst.units_numpy()[0], r["units"][0], what + " mask units")
         assert_units_equal(st.units_numpy()[0], r["units"][0], what + " update units")
-        assert_values_close(to_np(out[0]), r["out64"][0], r["mag"][0], what)
+        assert_values_close(to_np(out[0]), r["out64"][0], r["mag"][0], what, op="ties", K=1)
         if scope == "tensor":
             u = r["units"][0][0]
             assert u["ties_at_thresh"] >= 1001, "the injected ties sit at the threshold"
@@ -186,7 +189,7 @@ def test_full_size_qwen7b_merge_k8_sampled():
             r = oracle.merge([a], ex, oop, experts_are_deltas=True, density=0.1, lam=1.0,
                              is_1d=[one], eps_act=eps)
             what = f"7B K=8 {op} tensor {q}"
-            assert_values_close(to_np(out[q]), r["out64"][0], r["mag"][0], what)
+            assert_values_close(to_np(out[q]), r["out64"][0], r["mag"][0], what, op=op, K=K)
             if op != "ram":   # RAM trims nothing: no unit records
                 assert_units_equal(units[:, q:q + 1], r["units"], what)
             if op == "iso" and not one:

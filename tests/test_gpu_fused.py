@@ -59,7 +59,8 @@ def check_fused(th0, th1, op, density, is_delta=False, what=""):
     r = oracle.update([to_np(t) for t in th0], [to_np(t) for t in th1], OPS[op],
                       update_is_delta=is_delta, density=density, shapes=shapes, is_1d=is1d)
     for q in range(len(th0)):
-        assert_values_close(to_np(out_f[q]), r["out64"][q], r["mag"][q], f"{what} fused tensor {q}")
+        assert_values_close(to_np(out_f[q]), r["out64"][q], r["mag"][q], f"{what} fused tensor {q}",
+                            op=op, K=1)
         assert np.array_equal(to_np(out_f[q]), to_np(out_t[q])), f"{what}: fused and two-pass differ, tensor {q}"
     uf = st_f.units_numpy()
     assert_units_equal(uf, r["units"], what)

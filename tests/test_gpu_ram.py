@@ -36,14 +36,14 @@ def _np(ts):
     return [to_np(t) for t in ts]
 
 
-def _check(out, st, r, theta0, what):
+def _check(out, st, r, theta0, what, K=8):
     torch.cuda.synchronize()
     if st is not None:
         assert int(st.status.item()) == 0, what
     for q, (o, b) in enumerate(zip(out, theta0)):
         g = to_np(o)
         assert g.dtype == (np.uint16 if b.dtype == torch.bfloat16 else np.float32)
-        assert_values_close(g, r["out64"][q], r["mag"][q], f"{what} tensor {q}")
+        assert_values_close(g, r["out64"][q], r["mag"][q], f"{what} tensor {q}", op="ram", K=K)
 
 
 MINI = synth.qwen_shapes("qwen1.5b", layers=2, scale=8)
@@ -80,7 +80,7 @@ def test_ram_merge_bf16_checkpoints(K, lam):
                             stats=True)
     r = oracle.merge(_np(th0), [_np(e) for e in cks], oracle.RAM, experts_are_deltas=False,
                      lam=lam, eps_act=EPS, shapes=_shapes(shapes), is_1d=_is1d(shapes))
-    _check(out, st, r, th0, f"RAM K={K} checkpoints")
+    _check(out, st, r, th0, f"RAM K={K} checkpoints", K=K)
     # the quantised deltas really are sparse: some entries have no active expert
     t = (cks[0][1].float() - th0[1].float()).abs()
     assert 0.0 < float((t <= EPS).float().mean()) < 0.9
@@ -109,7 +109,7 @@ def test_ram_merge_task_vectors(K, base_dtype, x_dtype):
         out, st = iso.iso_merge(d0, dx, op="ram", eps_act=eps, stats=True)
     r = oracle.merge(_np(th0), [_np(e) for e in taus], oracle.RAM, eps_act=eps,
                      shapes=_shapes(MIXED), is_1d=_is1d(MIXED))
-    _check(out, st, r, th0, f"RAM K={K} {base_dtype} {x_dtype}")
+    _check(out, st, r, th0, f"RAM K={K} {base_dtype} {x_dtype}", K=K)
 
 
 @pytest.mark.parametrize("K", [3, 8])
@@ -132,7 +132,7 @@ def test_ram_threshold_ties_exact(K):
     out, st = iso.iso_merge(d0, dx, op="ram", eps_act=eps, stats=True)
     r = oracle.merge(_np(th0), [_np(e) for e in taus], oracle.RAM, eps_act=eps,
                      shapes=_shapes(shapes), is_1d=_is1d(shapes))
-    _check(out, st, r, th0, f"RAM ties K={K}")
+    _check(out, st, r, th0, f"RAM ties K={K}", K=K)
     # dyadic inputs and power-of-two-free counts aside, every kept or dropped
     # decision shows: entries with no active expert are theta_0 bit for bit
     for q in range(len(shapes)):

@@ -18,7 +18,6 @@ import paper_2607_19331_gb300 as iso
 import synth
 from paper_2607_19331_gb300 import _abi
 from paper_2607_19331_gb300.api import describe, make_stats, merge_cfg
-from parity_util import assert_values_close, bf16_value, to_np
 
 pytestmark = pytest.mark.gpu
 DEV = "cuda:0"
@@ -47,9 +46,9 @@ def test_noalloc_matches_workspace_update_on_two_calls():
         torch.cuda.synchronize()
         assert int(st.status.item()) == 0
         for q, (a, b) in enumerate(zip(out, ref)):
-            ga, gb = to_np(a), to_np(b)
-            # the tolerance of the parity tests, measured against the workspace path
-            assert_values_close(ga, bf16_value(gb), bf16_value(gb) * 0.0, f"noalloc {op} tensor {q}")
+            # the same kernels on the same inputs: identical bits, so a value
+            # left in the shared scratch by the first call cannot hide
+            assert torch.equal(a.view(torch.int16), b.view(torch.int16)), f"noalloc {op} tensor {q}"
         assert torch.equal(st.units, st_ref.units)
         assert torch.equal(st.coef, st_ref.coef)
 
