@@ -44,9 +44,10 @@
  *   - The return value is ISO_OK or a negative iso_status.  Argument errors
  *     (ARG, SHAPE, DTYPE, ALIGN, WORKSPACE, UNSUPPORTED) are detected on the
  *     host before anything is enqueued.  ISO_ERR_CUDA means a launch failed.
- *     ISO_ERR_NONFINITE is detected on the device: it is written to
- *     stats->status (when given) and is valid once the stream has reached the
- *     end of the call; the outputs of such a call are unspecified.  The
+ *     ISO_ERR_NONFINITE and ISO_ERR_TIMEOUT are detected on the device: they
+ *     are written to stats->status (when given) and are valid once the stream
+ *     has reached the end of the call; the outputs of such a call are
+ *     unspecified.  The
  *     operators that read every task-vector entry's magnitude (TIES, ISO,
  *     RAM) check for it; TA does not.
  *   - No C++ exception crosses this interface.  The library keeps no state
@@ -76,9 +77,11 @@ typedef enum {
                                   minimum reported by iso_workspace_size */
     ISO_ERR_CUDA = -6,         /* a CUDA launch or runtime call failed */
     ISO_ERR_NONFINITE = -7,    /* (device) an input held NaN or +-Inf */
-    ISO_ERR_UNSUPPORTED = -8   /* valid request outside this build: K > ISO_MAX_EXPERTS,
+    ISO_ERR_UNSUPPORTED = -8,  /* valid request outside this build: K > ISO_MAX_EXPERTS,
                                   a tensor with 2^32 or more entries, GLOBAL scope larger
                                   than the workspace allows */
+    ISO_ERR_TIMEOUT = -9       /* (device) a kernel's wait for its own bulk copies gave up
+                                  after its iteration limit; the outputs are unspecified */
 } iso_status;
 
 #define ISO_MAX_EXPERTS 8
@@ -146,7 +149,7 @@ typedef struct {
 
 /* Optional device-side outputs of a call; every pointer may be NULL. */
 typedef struct {
-    int32_t*        status;  /* 1 value: ISO_OK or ISO_ERR_NONFINITE, valid after the stream
+    int32_t*        status;  /* 1 value: ISO_OK, ISO_ERR_NONFINITE or ISO_ERR_TIMEOUT, valid after the stream
                                 reaches the end of the call */
     iso_unit_stats* units;   /* [K][n_units], n_units from iso_num_units; not written by
                                 TA and RAM, which trim nothing */

@@ -21,6 +21,7 @@ ISO_ERR_WORKSPACE = -5
 ISO_ERR_CUDA = -6
 ISO_ERR_NONFINITE = -7
 ISO_ERR_UNSUPPORTED = -8
+ISO_ERR_TIMEOUT = -9
 ISO_MAX_EXPERTS = 8
 ISO_NOALLOC_SCRATCH_BYTES = 32 << 20
 

@@ -936,6 +936,7 @@ const char* iso_error_string(int32_t status) {
         case ISO_ERR_CUDA: return "ISO_ERR_CUDA: a CUDA launch or runtime call failed";
         case ISO_ERR_NONFINITE: return "ISO_ERR_NONFINITE: an input held NaN or Inf";
         case ISO_ERR_UNSUPPORTED: return "ISO_ERR_UNSUPPORTED: request outside this build's limits";
+        case ISO_ERR_TIMEOUT: return "ISO_ERR_TIMEOUT: a kernel's wait for its own copies gave up";
         default: return "unknown iso_status";
     }
 }

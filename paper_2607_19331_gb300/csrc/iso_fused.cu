@@ -29,18 +29,69 @@
 
 namespace iso {
 
+// One full tile of the fast form, read from the warp's stage in shared memory:
+// out = theta_0 + (key > T ? a tau : -0) for every entry, counting the keys
+// above hi and equal to t^ and, outside run mode, marking the band entries
+// other than t^ (bit 8 v + j of tbm: entry v * 256 + 8 lane + j).
+// RUN: the band is the single key t^ (no band entries besides its ties).
+// A1: a == 1, so a tau == tau.
+template <bool CK, bool RUN, bool A1>
+__device__ __forceinline__ void fused_fast_tile(const unsigned char* sx, const unsigned char* sb,
+                                                __nv_bfloat16* q, int lane, uint32_t T, uint32_t lo,
+                                                uint32_t span, uint32_t hi, uint32_t th, float a,
+                                                uint32_t& n_gt, uint32_t& n_eq, float& f_gg,
+                                                uint32_t& tbm) {
+#pragma unroll
+    for (int v = 0; v < WVEC; ++v) {
+        const uint32_t off = (uint32_t)(v * (32 * VEC) + lane * VEC);
+        const uint4 xr = *reinterpret_cast<const uint4*>(sx + 2 * off);
+        const uint4 br = *reinterpret_cast<const uint4*>(sb + 2 * off);
+        const uint32_t xw[4] = {xr.x, xr.y, xr.z, xr.w};
+        const uint32_t bw[4] = {br.x, br.y, br.z, br.w};
+        uint32_t ow[4];
+#pragma unroll
+        for (int w = 0; w < 4; ++w) {
+            const float b0 = __uint_as_float(bw[w] << 16), b1 = __uint_as_float(bw[w] & 0xFFFF0000u);
+            float t0 = __uint_as_float(xw[w] << 16), t1 = __uint_as_float(xw[w] & 0xFFFF0000u);
+            if (CK) sub_rn2(t0, t1, t0, t1, b0, b1);
+            const uint32_t k0 = key_of(t0), k1 = key_of(t1);
+            const bool kp0 = (int)k0 > (int)T, kp1 = (int)k1 > (int)T;
+            const bool gt0 = k0 > hi, gt1 = k1 > hi;
+            const bool eq0 = k0 == th, eq1 = k1 == th;
+            n_gt += (uint32_t)gt0 + (uint32_t)gt1;
+            n_eq += (uint32_t)eq0 + (uint32_t)eq1;
+            if (gt0) f_gg = __fmaf_rn(t0, t0, f_gg);
+            if (gt1) f_gg = __fmaf_rn(t1, t1, f_gg);
+            if (!RUN) {
+                if ((k0 - lo <= span) & !eq0) tbm |= 1u << (v * VEC + 2 * w);
+                if ((k1 - lo <= span) & !eq1) tbm |= 1u << (v * VEC + 2 * w + 1);
+            }
+            float u0 = t0, u1 = t1;
+            if (!A1) mul_rn2(u0, u1, a, a, t0, t1);
+            float o0, o1;
+            add_rn2(o0, o1, b0, b1, kp0 ? u0 : -0.0f, kp1 ? u1 : -0.0f);
+            __nv_bfloat162 h = __floats2bfloat162_rn(o0, o1);
+            ow[w] = *reinterpret_cast<uint32_t*>(&h);
+        }
+        __stcs(reinterpret_cast<uint4*>(q + off), make_uint4(ow[0], ow[1], ow[2], ow[3]));
+    }
+}
+
+// The fused pass.  Each warp walks a contiguous range of tiles; a ring of
+// FUSED_STAGES tile stages per warp in shared memory is filled by bulk copies
+// (cp.async.bulk, completion counted on one mbarrier per stage) issued by the
+// warp's lane 0 FUSED_STAGES - 1 tiles ahead of the tile being decided, so
+// several tiles of both inputs are in flight per warp without registers.  A
+// partial tile (a tensor's last) is not copied: its stage's barrier is
+// arrived on without transactions and the tile is read from global memory.
 template <bool CK>
 __global__ void __launch_bounds__(TPB, FUSED_BLOCKS_PER_SM) k_count_apply(Plan P) {
-    // per lane, its band entries other than t^ as (tile offset, theta_0 bits
-    // << 16 | x bits), lane L's j-th at j*32 + L; FUSED_SMEM bytes of dynamic
-    // shared memory
-    extern __shared__ uint2 s_stage[];
+    extern __shared__ __align__(128) unsigned char s_ring[];
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-    uint2* const sbl = s_stage + warp * (TILE + 32) + lane;
-    // the raw words of the tile being decided, per lane and step (x then theta_0)
-    // step v's x words of lane L at uint4 (2 v * 32 + L), its theta_0 words at ((2 v + 1) * 32 + L):
-    // each warp-wide store is 512 contiguous bytes
-    uint4* const s_raw = reinterpret_cast<uint4*>(s_stage + WPB * (TILE + 32)) + warp * (WVEC * 2 * 32) + lane;
+    unsigned char* const ring = s_ring + (size_t)warp * FUSED_STAGES * FUSED_STAGE_BYTES;
+    const uint32_t ring_s = smem_u32(ring);
+    const uint32_t bar_s = smem_u32(s_ring + (size_t)WPB * FUSED_STAGES * FUSED_STAGE_BYTES) +
+                           8u * (uint32_t)(warp * FUSED_STAGES);
     const uint32_t W = gridDim.x * WPB;
     const uint32_t wid = blockIdx.x * WPB + warp;
     const uint32_t items = (uint32_t)P.n_tiles;
@@ -50,6 +101,35 @@ __global__ void __launch_bounds__(TPB, FUSED_BLOCKS_PER_SM) k_count_apply(Plan P
     if (beg >= end) return;
     const unsigned FULL = 0xFFFFFFFFu;
     const float a_spec = k1_spec_coef(P);
+
+    if (lane == 0) {
+        for (int s = 0; s < FUSED_STAGES; ++s) mbar_init(bar_s + 8u * s, 1);
+        mbar_fence_init();
+    }
+    __syncwarp();
+
+    // the copy cursor: the tensor of the next tile whose copy is issued
+    int ct = tensor_of_tile(P.tens, P.n_tensors, beg);
+    uint32_t ct_end = (uint32_t)(P.tens[ct].tile_base + (P.tens[ct].numel + TILE - 1) / TILE);
+    auto issue = [&](uint32_t g, int s) {
+        while (g >= ct_end) {
+            ++ct;
+            ct_end = (uint32_t)(P.tens[ct].tile_base + (P.tens[ct].numel + TILE - 1) / TILE);
+        }
+        if (lane == 0) {
+            const TensorDesc& d = P.tens[ct];
+            const uint32_t e0 = (g - (uint32_t)d.tile_base) * TILE;
+            const uint32_t bar = bar_s + 8u * s;
+            if ((uint32_t)d.numel - e0 >= (uint32_t)TILE) {
+                const uint32_t dst = ring_s + (uint32_t)s * FUSED_STAGE_BYTES;
+                mbar_arrive_tx(bar, 2 * TILE * 2);
+                bulk_g2s(dst, static_cast<const char*>(P.xptr[ct]) + (size_t)e0 * 2, TILE * 2, bar);
+                bulk_g2s(dst + TILE * 2, static_cast<const char*>(d.base) + (size_t)e0 * 2, TILE * 2, bar);
+            } else {
+                mbar_arrive(bar);
+            }
+        }
+    };
 
     // the current tensor and its unit
     int t = tensor_of_tile(P.tens, P.n_tensors, beg);
@@ -141,121 +221,107 @@ __global__ void __launch_bounds__(TPB, FUSED_BLOCKS_PER_SM) k_count_apply(Plan P
         return true;
     };
 
-    RawTile<__nv_bfloat16, __nv_bfloat16, true> rt;   // x in rt.x, theta_0 in rt.b
+    // the first tiles' copies
+    for (int s = 0; s < FUSED_STAGES; ++s)
+        if (beg + (uint32_t)s < end) issue(beg + s, s);
 
-    // first tile's loads
     enter_tensor(t);
-    {
-        const TensorDesc& d = P.tens[t];
-        const uint32_t e0 = (uint32_t)(beg - d.tile_base) * TILE;
-#pragma unroll
-        for (int v = 0; v < WVEC; ++v) rt.load_step(v, P.xptr[t], d.base, e0, (uint32_t)d.numel - e0, lane);
-    }
-    int nt = t;                               // tensor of the next tile
-    uint32_t nt_end = t_end;
+    uint32_t phases = 0;                      // bit s: parity of stage s's next phase
+    int s = 0;
     for (uint32_t g = beg; g < end; ++g) {
+        {
+            const uint32_t bar = bar_s + 8u * s;
+            const uint32_t par = (phases >> s) & 1u;
+            int spin = 0;
+            while (!mbar_try_wait(bar, par)) {
+                if (++spin >= MBAR_SPIN_LIMIT) {
+                    // give up: report, then wait (bounded) for the copies this
+                    // warp still has in flight before the block may exit
+                    if (lane == 0) set_status(P.hdr, ISO_ERR_TIMEOUT);
+                    const uint32_t pend = min(end - g, (uint32_t)FUSED_STAGES);
+                    for (uint32_t j = 0; j < pend; ++j) {
+                        const int sj = (s + (int)j) % FUSED_STAGES;
+                        for (int r = 0; r < MBAR_SPIN_LIMIT; ++r)
+                            if (mbar_try_wait(bar_s + 8u * sj, (phases >> sj) & 1u)) break;
+                    }
+                    return;
+                }
+            }
+            phases ^= 1u << s;
+        }
         if (g >= t_end) {
             while (g >= (uint32_t)(P.tens[t].tile_base + (P.tens[t].numel + TILE - 1) / TILE)) ++t;
             enter_tensor(t);
         }
         const TensorDesc& d = P.tens[t];
-        void* op = d.out;
+        __nv_bfloat16* const q16 = static_cast<__nv_bfloat16*>(d.out);
         const uint32_t n = (uint32_t)d.numel;
         const uint32_t e0 = (uint32_t)(g - d.tile_base) * TILE;
         const uint32_t rem = n - e0;
-        // the next tile: its loads replace each step as it is consumed
-        const bool more = g + 1 < end;
-        const void* nxp = nullptr;
-        const void* nbp = nullptr;
-        uint32_t ne0 = 0, nrem = 0;
-        if (more) {
-            while (g + 1 >= nt_end) {
-                ++nt;
-                nt_end = (uint32_t)(P.tens[nt].tile_base + (P.tens[nt].numel + TILE - 1) / TILE);
-            }
-            const TensorDesc& nd = P.tens[nt];
-            nxp = P.xptr[nt];
-            nbp = nd.base;
-            ne0 = (uint32_t)(g + 1 - nd.tile_base) * TILE;
-            nrem = (uint32_t)nd.numel - ne0;
-        }
+        const bool full = rem >= (uint32_t)TILE;
+        const unsigned char* const sx = ring + (size_t)s * FUSED_STAGE_BYTES;
+        const unsigned char* const sb = sx + TILE * 2;
+        // a partial tile was not copied: it is read from global memory
+        const unsigned short* const xs16 = full ? reinterpret_cast<const unsigned short*>(sx)
+                                                : static_cast<const unsigned short*>(P.xptr[t]) + e0;
+        const unsigned short* const bs16 = full ? reinterpret_cast<const unsigned short*>(sb)
+                                                : static_cast<const unsigned short*>(d.base) + e0;
 
         // speculative selection: kept <=> key > t^, or key == t^ at a
         // position before chat.  In a whole tile on one side of chat that is
-        // one comparison, key > T, on the tile held in registers.  A tile of a
-        // tensor whose selection is already final, a tile holding chat and a
-        // tensor's last tile (a few per tensor) take a compact per-entry loop
-        // that reads the tile again from L2.  Band keys other than t^ are
-        // rare: their lanes stage them while the step's words are in registers.
+        // one comparison, key > T.  A tile of a tensor whose selection is
+        // already final, a tile holding chat and a tensor's last tile (a few
+        // per tensor) take a per-entry loop.  Band keys other than t^ are
+        // rare: a per-lane bit marks them for the second step below.
         const uint32_t tile_hi = e0 + min(rem, (uint32_t)TILE);
         // the fast form writes theta_0 + (kept ? a tau : -0): exact (theta_0 bits
         // kept for an update of 0) because every kept |tau| is at least t^'s and
         // a times that stays a normal number
-        const bool fast = sel && rem >= TILE && (tile_hi <= chat || e0 >= chat) && a_t_normal;
+        const bool fast = sel && full && (tile_hi <= chat || e0 >= chat) && a_t_normal;
         uint32_t n_gt = 0, n_eq = 0;
         float f_gg = 0.0f;                     // tau^2 above hi (also the non-finite detector)
-        uint2* sp = sbl;
+        uint32_t tbm = 0;                      // the lane's band entries of the tile
+        bool slow_map = false;                 // tbm bit j: entry lane + 32 j (else v * 256 + 8 lane + j)
         if (fast) {
             const uint32_t T = (tile_hi <= chat) ? th - 1u : th;     // th >= 1 whenever ties are kept here
             const uint32_t span = hi - lo;     // band: key - lo <= span (unsigned), key != t^
-            uint32_t tbm = 0;                  // band entries of the tile: bit 8 v + j
+            __nv_bfloat16* const qo = q16 + e0;
+            const bool run = lo == hi, a1 = a == 1.0f;
+            if (run) {
+                if (a1) fused_fast_tile<CK, true, true>(sx, sb, qo, lane, T, lo, span, hi, th, a, n_gt, n_eq, f_gg, tbm);
+                else    fused_fast_tile<CK, true, false>(sx, sb, qo, lane, T, lo, span, hi, th, a, n_gt, n_eq, f_gg, tbm);
+            } else {
+                if (a1) fused_fast_tile<CK, false, true>(sx, sb, qo, lane, T, lo, span, hi, th, a, n_gt, n_eq, f_gg, tbm);
+                else    fused_fast_tile<CK, false, false>(sx, sb, qo, lane, T, lo, span, hi, th, a, n_gt, n_eq, f_gg, tbm);
+            }
+        } else if (!sel && full) {
+            // a tensor whose selection is already final: every entry kept
+            // (untrimmed) or none (k == 0)
 #pragma unroll
             for (int v = 0; v < WVEC; ++v) {
+                const uint32_t off = (uint32_t)(v * (32 * VEC) + lane * VEC);
+                const uint4 xr = *reinterpret_cast<const uint4*>(sx + 2 * off);
+                const uint4 br = *reinterpret_cast<const uint4*>(sb + 2 * off);
                 float th0[VEC], tau[VEC], o[VEC];
-                raw_to_f32<__nv_bfloat16>(rt.b[v], th0);
-                raw_to_f32<__nv_bfloat16>(rt.x[v], tau);
-                if (CK) {
+                raw_to_f32<__nv_bfloat16>(reinterpret_cast<const uint4(&)[1]>(br), th0);
+                raw_to_f32<__nv_bfloat16>(reinterpret_cast<const uint4(&)[1]>(xr), tau);
 #pragma unroll
-                    for (int j = 0; j < VEC; j += 2) sub_rn2(tau[j], tau[j + 1], tau[j], tau[j + 1], th0[j], th0[j + 1]);
+                for (int j = 0; j < VEC; ++j) {
+                    const float tv = CK ? __fsub_rn(tau[j], th0[j]) : tau[j];
+                    o[j] = keep_all ? out_of(th0[j], tv, a) : th0[j];
                 }
-                // keep the step's raw words for the band entries, then reuse the registers
-                s_raw[(2 * v) * 32] = rt.x[v][0];
-                s_raw[(2 * v + 1) * 32] = rt.b[v][0];
-                if (more) rt.load_step(v, nxp, nbp, ne0, nrem, lane);
-                const uint32_t o8 = (uint32_t)(v * (32 * VEC) + lane * VEC);
-#pragma unroll
-                for (int j = 0; j < VEC; j += 2) {
-                    bool kept[2];
-#pragma unroll
-                    for (int h = 0; h < 2; ++h) {
-                        const uint32_t kk = key_of(tau[j + h]);
-                        const bool gt = kk > hi, eq = kk == th;
-                        kept[h] = (int)kk > (int)T;
-                        n_gt += gt;
-                        n_eq += eq;
-                        if (gt) f_gg = __fmaf_rn(tau[j + h], tau[j + h], f_gg);
-                        if ((kk - lo <= span) & !eq) tbm |= 1u << (v * VEC + j + h);
-                    }
-                    float m0, m1;
-                    mul_rn2(m0, m1, a, a, tau[j], tau[j + 1]);
-                    add_rn2(o[j], o[j + 1], th0[j], th0[j + 1], kept[0] ? m0 : -0.0f, kept[1] ? m1 : -0.0f);
-                }
-                store8(op, (long long)e0 + o8, n, o, true);
-            }
-            // the lane's band entries into its staging list, raw bits from shared memory
-            while (tbm) {
-                const int b = __ffs(tbm) - 1;
-                tbm &= tbm - 1;
-                const int v = b >> 3, j = b & 7;
-                const uint32_t sh = 16u * (uint32_t)(j & 1);
-                const uint32_t rx = (reinterpret_cast<const uint32_t*>(s_raw + (2 * v) * 32)[j >> 1] >> sh) & 0xFFFFu;
-                const uint32_t rb = (reinterpret_cast<const uint32_t*>(s_raw + (2 * v + 1) * 32)[j >> 1] >> sh) & 0xFFFFu;
-                *sp = make_uint2((uint32_t)(v * (32 * VEC) + lane * VEC + j), (rb << 16) | rx);
-                sp += 32;
+                store8(q16, (long long)e0 + off, n, o, true);
             }
         } else {
-            // the next tile's loads first, then this tile entry by entry from L2
-#pragma unroll
-            for (int v = 0; v < WVEC; ++v)
-                if (more) rt.load_step(v, nxp, nbp, ne0, nrem, lane);
-            const unsigned short* xs16 = static_cast<const unsigned short*>(P.xptr[t]);
-            const unsigned short* bs16 = static_cast<const unsigned short*>(d.base);
-            __nv_bfloat16* q16 = static_cast<__nv_bfloat16*>(op);
+            // entry by entry: lane L takes entries L + 32 j
+            slow_map = true;
             const uint32_t cnt = min(rem, (uint32_t)TILE);
 #pragma unroll 1
-            for (uint32_t o1 = lane; o1 < cnt; o1 += 32) {
+            for (uint32_t j = 0; j < 32; ++j) {
+                const uint32_t o1 = (uint32_t)lane + 32u * j;
+                if (o1 >= cnt) break;
                 const uint32_t pos = e0 + o1;
-                const uint32_t xr = __ldg(xs16 + pos), br = __ldg(bs16 + pos);
+                const uint32_t xr = xs16[o1], br = bs16[o1];
                 const float bv = __uint_as_float(br << 16), xv = __uint_as_float(xr << 16);
                 const float tv = CK ? __fsub_rn(xv, bv) : xv;
                 float ov;
@@ -268,75 +334,86 @@ __global__ void __launch_bounds__(TPB, FUSED_BLOCKS_PER_SM) k_count_apply(Plan P
                     n_gt += gt;
                     n_eq += eq;
                     if (gt) f_gg = __fmaf_rn(tv, tv, f_gg);
-                    if (kk >= lo && !gt && !eq) { *sp = make_uint2(o1, (br << 16) | xr); sp += 32; }
+                    if (kk >= lo && !gt && !eq) tbm |= 1u << j;
                     ov = kept ? out_of(bv, tv, a) : bv;
                 }
                 q16[pos] = __float2bfloat16_rn(ov);
             }
-            if (!sel) continue;
         }
-        if (__any_sync(FULL, !(fabsf(f_gg) <= 3.402823466e38f))) {
-            // a non-finite (or overflowing) sum: read the tile's keys again
-            uint32_t kmax = 0;
-            for (int v = 0; v < WVEC; ++v) {
-                const uint32_t o8 = (uint32_t)(v * (32 * VEC) + lane * VEC);
-                if (o8 >= rem) break;
-                float tau[VEC];
-                TauSrc<__nv_bfloat16, __nv_bfloat16, CK>::load8(P.xptr[t], d.base, (long long)e0 + o8, (long long)n, tau);
+        if (sel) {
+            if (__any_sync(FULL, !(fabsf(f_gg) <= 3.402823466e38f))) {
+                // a non-finite (or overflowing) sum: read the tile's keys again
+                uint32_t kmax = 0;
+                for (int v = 0; v < WVEC; ++v) {
+                    const uint32_t o8 = (uint32_t)(v * (32 * VEC) + lane * VEC);
+                    if (o8 >= rem) break;
+                    float tau[VEC];
+                    TauSrc<__nv_bfloat16, __nv_bfloat16, CK>::load8(P.xptr[t], d.base, (long long)e0 + o8, (long long)n, tau);
 #pragma unroll
-                for (int j = 0; j < VEC; ++j)
-                    if (o8 + j < rem) kmax = max(kmax, key_of(tau[j]));
+                    for (int j = 0; j < VEC; ++j)
+                        if (o8 + j < rem) kmax = max(kmax, key_of(tau[j]));
+                }
+                if (__any_sync(FULL, kmax >= KEY_INF) && lane == 0) set_status(P.hdr, ISO_ERR_NONFINITE);
             }
-            if (__any_sync(FULL, kmax >= KEY_INF) && lane == 0) set_status(P.hdr, ISO_ERR_NONFINITE);
-        }
-        if (want_gamma) two_sum_add(s_gg, e_gg, f_gg);
-        const uint32_t t_gt = __reduce_add_sync(FULL, n_gt);
-        const uint32_t t_eq = __reduce_add_sync(FULL, n_eq);
-        a_gt += t_gt;
-        a_eq += t_eq;
+            if (want_gamma) two_sum_add(s_gg, e_gg, f_gg);
+            const uint32_t t_gt = __reduce_add_sync(FULL, n_gt);
+            const uint32_t t_eq = __reduce_add_sync(FULL, n_eq);
+            a_gt += t_gt;
+            a_eq += t_eq;
 
-        // pass 2: the staged band entries (keys other than t^, a fraction of a
-        // per cent) go to the unit's candidate segment (keys) and its band
-        // records (position and raw values), read again from L2
-        const uint32_t nb = (uint32_t)(sp - sbl) >> 5;
-        uint32_t nb_tot;
-        const uint32_t nb_off = warp_excl_scan(nb, &nb_tot);
-        const uint32_t left_tiles = min(t_end, end) - g;   // this warp's tiles left in the unit
-        if (nb_tot && !c_ovf && nb_tot > c_left) c_ovf = !reserve(&au->n_alloc, nb_tot, c_cap, left_tiles, c_pos, c_left);
-        if (nb_tot && !b_ovf && nb_tot > b_left) b_ovf = !reserve(&au->b_alloc, nb_tot, b_cap, left_tiles, b_pos, b_left);
-        const bool c_store = nb_tot && !c_ovf;
-        const bool b_store = nb_tot && !b_ovf;
-        uint32_t n_abv = 0, kbad = 0;
-        float f_band = 0.0f;                   // tau^2 over the candidates above t^
-        if (nb_tot) {
-            uint32_t wi = c_pos + nb_off, wb = b_pos + nb_off;
-            for (uint32_t q = 0; q < nb; ++q) {
-                const uint2 st = sbl[q * 32];
-                const uint32_t pos = e0 + st.x;
-                const float xv = __uint_as_float(st.y << 16), bv = __uint_as_float(st.y & 0xFFFF0000u);
-                const float tv = CK ? __fsub_rn(xv, bv) : xv;
-                const uint32_t kk = key_of(tv);
-                if (b_store) bseg[wb++] = make_uint2(pos, st.y);
-                if (c_store) cseg[wi++] = kk;
-                const bool ab = kk > th;
-                n_abv += ab;
-                kbad |= (kk >= KEY_INF);
-                if (want_gamma && ab) f_band = __fmaf_rn(tv, tv, f_band);
+            // the marked band entries (keys other than t^, a fraction of a
+            // per cent) go to the unit's candidate segment (keys) and its band
+            // records (position and raw values), read again from the stage
+            const uint32_t nb = __popc(tbm);
+            uint32_t nb_tot;
+            const uint32_t nb_off = warp_excl_scan(nb, &nb_tot);
+            const uint32_t left_tiles = min(t_end, end) - g;   // this warp's tiles left in the unit
+            if (nb_tot && !c_ovf && nb_tot > c_left) c_ovf = !reserve(&au->n_alloc, nb_tot, c_cap, left_tiles, c_pos, c_left);
+            if (nb_tot && !b_ovf && nb_tot > b_left) b_ovf = !reserve(&au->b_alloc, nb_tot, b_cap, left_tiles, b_pos, b_left);
+            const bool c_store = nb_tot && !c_ovf;
+            const bool b_store = nb_tot && !b_ovf;
+            uint32_t n_abv = 0, kbad = 0;
+            float f_band = 0.0f;               // tau^2 over the candidates above t^
+            if (nb_tot) {
+                uint32_t wi = c_pos + nb_off, wb = b_pos + nb_off;
+                uint32_t m = tbm;
+                while (m) {
+                    const int b = __ffs(m) - 1;
+                    m &= m - 1;
+                    const uint32_t o1 = slow_map ? (uint32_t)lane + 32u * (uint32_t)b
+                                                 : (uint32_t)((b >> 3) * (32 * VEC) + lane * VEC + (b & 7));
+                    const uint32_t xr = xs16[o1], br = bs16[o1];
+                    const float xv = __uint_as_float(xr << 16), bv = __uint_as_float(br << 16);
+                    const float tv = CK ? __fsub_rn(xv, bv) : xv;
+                    const uint32_t kk = key_of(tv);
+                    if (b_store) bseg[wb++] = make_uint2(e0 + o1, (br << 16) | xr);
+                    if (c_store) cseg[wi++] = kk;
+                    const bool ab = kk > th;
+                    n_abv += ab;
+                    kbad |= (kk >= KEY_INF);
+                    if (want_gamma && ab) f_band = __fmaf_rn(tv, tv, f_band);
+                }
             }
+            if (__any_sync(FULL, kbad) && lane == 0) set_status(P.hdr, ISO_ERR_NONFINITE);
+            if (want_gamma) two_sum_add(s_gb, e_gb, f_band);
+            const uint32_t t_abv = __reduce_add_sync(FULL, n_abv);
+            if (lane == 0) {
+                P.tcand[g] = make_uint2(c_store ? c_pos : 0u, c_store ? nb_tot : 0u);
+                P.tband[g] = make_uint2(b_store ? b_pos : 0u, b_store ? nb_tot : 0u);
+                P.teq_hi[g] = t_eq;             // teq_lo stays 0 (zeroed with the group's state)
+            }
+            if (c_store) { c_pos += nb_tot; c_left -= nb_tot; }
+            if (b_store) { b_pos += nb_tot; b_left -= nb_tot; }
+            a_int += nb_tot;
+            a_abv += t_abv;
         }
-        if (__any_sync(FULL, kbad) && lane == 0) set_status(P.hdr, ISO_ERR_NONFINITE);
-        if (want_gamma) two_sum_add(s_gb, e_gb, f_band);
-        const uint32_t t_abv = __reduce_add_sync(FULL, n_abv);
-        if (lane == 0) {
-            P.tcand[g] = make_uint2(c_store ? c_pos : 0u, c_store ? nb_tot : 0u);
-            P.tband[g] = make_uint2(b_store ? b_pos : 0u, b_store ? nb_tot : 0u);
-            P.teq_hi[g] = t_eq;                 // teq_lo stays 0 (zeroed with the group's state)
-        }
-        if (c_store) { c_pos += nb_tot; c_left -= nb_tot; }
-        if (b_store) { b_pos += nb_tot; b_left -= nb_tot; }
-        a_int += nb_tot;
-        a_abv += t_abv;
+        // the stage is free again: the copy of the tile FUSED_STAGES ahead
         __syncwarp();
+        if (g + FUSED_STAGES < end) {
+            if (lane == 0) fence_proxy_async_smem();
+            issue(g + FUSED_STAGES, s);
+        }
+        s = (s + 1 == FUSED_STAGES) ? 0 : s + 1;
     }
     flush();
 }

@@ -26,9 +26,18 @@ constexpr int BLOCK_TPB = 1024;
 template <typename XT, typename BT, bool CK> __global__ void k_block_select(Plan P);
 
 // fused K = 1 pass (bf16 base and update)
-constexpr int FUSED_BLOCKS_PER_SM = 2;
-// dynamic shared memory: band staging (8 B per slot) and the raw words of a tile (4 KB per warp)
-constexpr int FUSED_SMEM = WPB * (TILE + 32) * 8 + WPB * TILE * 4;
+#ifndef ISO_FUSED_BLOCKS_PER_SM
+#define ISO_FUSED_BLOCKS_PER_SM 2
+#endif
+#ifndef ISO_FUSED_STAGES
+#define ISO_FUSED_STAGES 3
+#endif
+constexpr int FUSED_BLOCKS_PER_SM = ISO_FUSED_BLOCKS_PER_SM;
+constexpr int FUSED_STAGES = ISO_FUSED_STAGES;          // tile stages per warp in the copy ring
+constexpr int FUSED_STAGE_BYTES = 2 * TILE * 2;         // one tile of the update and of theta_0 (bf16)
+// dynamic shared memory: the warps' stage rings, then one 8-byte mbarrier per stage
+constexpr int FUSED_SMEM = WPB * FUSED_STAGES * (FUSED_STAGE_BYTES + 8);
+static_assert(FUSED_STAGES >= 2 && FUSED_STAGES <= 8, "stage ring");
 template <bool CK> __global__ void k_count_apply(Plan P);
 template <bool CK> __global__ void k_patch(Plan P);
 __global__ void k_fix_plan(Plan P);

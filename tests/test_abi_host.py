@@ -37,7 +37,7 @@ def test_every_declared_symbol_is_exported():
 
 def test_error_strings():
     L = _abi.lib()
-    for code in range(0, -9, -1):
+    for code in range(0, -10, -1):
         s = L.iso_error_string(code).decode()
         assert s.startswith("ISO_"), s
     assert "unknown" in L.iso_error_string(-99).decode()

@@ -171,8 +171,9 @@ def test_full_size_qwen7b_merge_k8_sampled():
     ws = iso.Workspace(DEV)
     ws_bytes = _workspace_bytes(th0, K, "iso", 0.1)
     ws.get(ws_bytes)
-    picks = [_qwen7b_index(0, "k"), _qwen7b_index(0, "norm2"), _qwen7b_index(13, "q"),
-             _qwen7b_index(27, "v")]
+    # the embedding and lm_head (545 M entries each: the largest units) first
+    picks = [0, len(shapes) - 1, _qwen7b_index(0, "k"), _qwen7b_index(0, "norm2"),
+             _qwen7b_index(13, "q"), _qwen7b_index(27, "v")]
     eps = float(np.float32(1e-5))   # RAM's active-update threshold (App. F)
     for op, oop in (("ties", oracle.TIES), ("iso", oracle.ISO), ("ram", oracle.RAM)):
         out, st = iso.iso_merge(th0, taus, op=op, experts_are_deltas=True, out=out, density=0.1,

@@ -55,8 +55,9 @@ def test_noalloc_matches_workspace_update_on_two_calls():
 
 def test_noalloc_rejects_requests_beyond_the_scratch():
     cfg = merge_cfg("iso", 0.05)
-    big = (_abi.IsoTensor * 1)(_abi.IsoTensor(0x10000, 20000, 20000, _abi.ISO_BF16, 0))
-    upd = (_abi.IsoTensor * 1)(_abi.IsoTensor(0x20000, 20000, 20000, _abi.ISO_BF16, 0))
-    out = (_abi.IsoTensor * 1)(_abi.IsoTensor(0x30000, 20000, 20000, _abi.ISO_BF16, 0))
+    # descriptors only (nothing is launched): three disjoint 800 MB ranges
+    big = (_abi.IsoTensor * 1)(_abi.IsoTensor(1 << 40, 20000, 20000, _abi.ISO_BF16, 0))
+    upd = (_abi.IsoTensor * 1)(_abi.IsoTensor(2 << 40, 20000, 20000, _abi.ISO_BF16, 0))
+    out = (_abi.IsoTensor * 1)(_abi.IsoTensor(3 << 40, 20000, 20000, _abi.ISO_BF16, 0))
     rc = _abi.lib().iso_update_noalloc(big, upd, 0, out, 1, ctypes.byref(cfg), None, None)
     assert rc == _abi.ISO_ERR_WORKSPACE
