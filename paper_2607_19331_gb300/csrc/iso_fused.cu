@@ -95,9 +95,20 @@ __global__ void __launch_bounds__(TPB, FUSED_BLOCKS_PER_SM) k_count_apply(Plan P
     const uint32_t W = gridDim.x * WPB;
     const uint32_t wid = blockIdx.x * WPB + warp;
     const uint32_t items = (uint32_t)P.n_tiles;
-    const uint32_t per = (items + W - 1) / W;
-    const uint32_t beg = wid * per;
-    const uint32_t end = min(items, beg + per);
+    // the warp's tiles: g = beg, beg + step, ... below end -- interleaved over
+    // the warps (all warps sweep one window of the tensors together) or one
+    // contiguous range per warp
+    uint32_t beg, end, step;
+    if (FUSED_INTERLEAVE) {
+        beg = wid;
+        end = items;
+        step = W;
+    } else {
+        const uint32_t per = (items + W - 1) / W;
+        beg = wid * per;
+        end = min(items, beg + per);
+        step = 1;
+    }
     if (beg >= end) return;
     const unsigned FULL = 0xFFFFFFFFu;
     const float a_spec = k1_spec_coef(P);
@@ -222,13 +233,15 @@ __global__ void __launch_bounds__(TPB, FUSED_BLOCKS_PER_SM) k_count_apply(Plan P
     };
 
     // the first tiles' copies
-    for (int s = 0; s < FUSED_STAGES; ++s)
-        if (beg + (uint32_t)s < end) issue(beg + s, s);
+    for (int s = 0; s < FUSED_STAGES; ++s) {
+        const unsigned long long gs = beg + (unsigned long long)s * step;
+        if (gs < end) issue((uint32_t)gs, s);
+    }
 
     enter_tensor(t);
     uint32_t phases = 0;                      // bit s: parity of stage s's next phase
     int s = 0;
-    for (uint32_t g = beg; g < end; ++g) {
+    for (uint32_t g = beg; g < end; g += step) {
         {
             const uint32_t bar = bar_s + 8u * s;
             const uint32_t par = (phases >> s) & 1u;
@@ -238,7 +251,7 @@ __global__ void __launch_bounds__(TPB, FUSED_BLOCKS_PER_SM) k_count_apply(Plan P
                     // give up: report, then wait (bounded) for the copies this
                     // warp still has in flight before the block may exit
                     if (lane == 0) set_status(P.hdr, ISO_ERR_TIMEOUT);
-                    const uint32_t pend = min(end - g, (uint32_t)FUSED_STAGES);
+                    const uint32_t pend = min((end - g + step - 1) / step, (uint32_t)FUSED_STAGES);
                     for (uint32_t j = 0; j < pend; ++j) {
                         const int sj = (s + (int)j) % FUSED_STAGES;
                         for (int r = 0; r < MBAR_SPIN_LIMIT; ++r)
@@ -367,7 +380,7 @@ __global__ void __launch_bounds__(TPB, FUSED_BLOCKS_PER_SM) k_count_apply(Plan P
             const uint32_t nb = __popc(tbm);
             uint32_t nb_tot;
             const uint32_t nb_off = warp_excl_scan(nb, &nb_tot);
-            const uint32_t left_tiles = min(t_end, end) - g;   // this warp's tiles left in the unit
+            const uint32_t left_tiles = (min(t_end, end) - g + step - 1) / step;   // this warp's tiles left in the unit
             if (nb_tot && !c_ovf && nb_tot > c_left) c_ovf = !reserve(&au->n_alloc, nb_tot, c_cap, left_tiles, c_pos, c_left);
             if (nb_tot && !b_ovf && nb_tot > b_left) b_ovf = !reserve(&au->b_alloc, nb_tot, b_cap, left_tiles, b_pos, b_left);
             const bool c_store = nb_tot && !c_ovf;
@@ -409,9 +422,10 @@ __global__ void __launch_bounds__(TPB, FUSED_BLOCKS_PER_SM) k_count_apply(Plan P
         }
         // the stage is free again: the copy of the tile FUSED_STAGES ahead
         __syncwarp();
-        if (g + FUSED_STAGES < end) {
+        const unsigned long long gn = g + (unsigned long long)FUSED_STAGES * step;
+        if (gn < end) {
             if (lane == 0) fence_proxy_async_smem();
-            issue(g + FUSED_STAGES, s);
+            issue((uint32_t)gn, s);
         }
         s = (s + 1 == FUSED_STAGES) ? 0 : s + 1;
     }

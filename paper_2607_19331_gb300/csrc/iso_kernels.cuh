@@ -30,9 +30,13 @@ template <typename XT, typename BT, bool CK> __global__ void k_block_select(Plan
 #define ISO_FUSED_BLOCKS_PER_SM 2
 #endif
 #ifndef ISO_FUSED_STAGES
-#define ISO_FUSED_STAGES 3
+#define ISO_FUSED_STAGES 2
+#endif
+#ifndef ISO_FUSED_INTERLEAVE
+#define ISO_FUSED_INTERLEAVE 1
 #endif
 constexpr int FUSED_BLOCKS_PER_SM = ISO_FUSED_BLOCKS_PER_SM;
+constexpr bool FUSED_INTERLEAVE = ISO_FUSED_INTERLEAVE != 0;   // tiles dealt round-robin over the warps
 constexpr int FUSED_STAGES = ISO_FUSED_STAGES;          // tile stages per warp in the copy ring
 constexpr int FUSED_STAGE_BYTES = 2 * TILE * 2;         // one tile of the update and of theta_0 (bf16)
 // dynamic shared memory: the warps' stage rings, then one 8-byte mbarrier per stage
