@@ -1,35 +1,38 @@
-"""Frame-space ISO-Merger (App. E, Algorithm 1) -- TEST INFRASTRUCTURE ONLY.
+"""Frame-space ISO-Merger (App. E) -- TEST INFRASTRUCTURE ONLY.
 
-A plain binary64 numpy restatement of the paper's merge of K expert weight
-matrices that share one base, taken step by step in the paper's order and
-notation.  Library routines serve as steps where the paper names the
-operation (the thin SVD, matrix products); nothing is blocked, fused or
-reordered.  Only ``tests/``, ``__graft_entry__.smoke()`` and ``bench.py``'s
-CPU-baseline leg may import it; it shares no code with the CUDA library.
+A plain binary64 numpy restatement of the definitions of App. E, one small
+function per definition, each citing the subsection that defines it; the
+merge of one matrix composes them.  Library routines serve where the paper
+names the operation (the thin SVD, matrix products); nothing is blocked,
+fused or reordered.  Only ``tests/``, ``__graft_entry__.smoke()`` and
+``bench.py``'s CPU-baseline leg may import it; it shares no code with the
+CUDA library.
 
-For each 2-D weight matrix (App. E "Setup" to "Retraction and
-reconstruction"):
+Definitions (App. E):
 
-1. thin SVDs  W_0 = U_0 S_0 V_0^T  and  W_i = U_i S_i V_i^T  (q = min(m, n)
-   singular values, in descending order);
-2. joint sign canonicalisation of each expert's mode k against the base:
-   s_ik = sign(<u_0k, u_ik>) with sign(0) := 1, u_ik <- s_ik u_ik,
-   v_ik <- s_ik v_ik;
-3. frame displacements dU_i = U_i - U_0, dV_i = V_i - V_0 and their Stiefel
-   tangent projections  Pi_{U_0}(D) = D - U_0 sym(U_0^T D);
-4. top-k_keep mode mask: k_keep = round(rho_keep q), taken as
-   floor(rho_keep q + 1/2); the trailing columns of both tangents are zeroed;
-5. first-order effect proxies g_i = xi~_Ui S_0 V_0^T + U_0 S_0 xi~_Vi^T,
-   Gram Gamma_ij = <g_i, g_j>_F, retention coefficients from
-   (Gamma + ridge I) c = diag Gamma on the non-zero proxies, clipped to
-   [c_min, c_max] (the element-wise path's own pinned solve);
-6. aggregate tangents xi_U* = Pi_{U_0}(sum_i c_i xi~_Ui) (same for V),
-   polar retraction U* = polar(U_0 + xi_U*) with polar(X) = P Q^T from the
-   thin SVD X = P S Q^T, and W* = U* S_0 V*^T.
-
-One-dimensional parameters take the task-vector average (App. E "Merged
-parameter scope"); ``merge_model`` runs Algorithm 1's loop over a parameter
-list and rounds each result once to the base's encoding.
+* Setup: the shared base and every expert as thin SVDs W = U S V^T with
+  q = min(m, n) singular values in descending order; the merged matrix keeps
+  the base spectrum S_0 and moves only the frames.
+* Sign canonicalization: an SVD fixes each mode (u_k, v_k) only up to a joint
+  sign, so each expert mode takes s_k = sign(<u_0k, u_k>), sign(0) := 1, on
+  both of its frames.
+* Stiefel tangent projection: the tangent space at U_0 is
+  {xi : U_0^T xi + xi^T U_0 = 0} and the orthogonal projection onto it is
+  Pi_{U_0}(D) = D - U_0 sym(U_0^T D); an expert's frame motion is the
+  projected displacement of its aligned frames from the base's.
+* Top-k_keep singular-mode masking: D_keep keeps the leading
+  k_keep = round(rho_keep q) modes (halves rounded up) of each displacement.
+* Retention coefficients: the effect proxy g_i = xi~_Ui S_0 V_0^T +
+  U_0 S_0 xi~_Vi^T, its Gram matrix Gamma_ij = <g_i, g_j>_F and the clipped
+  solution of (Gamma + ridge I) c = diag Gamma on the non-zero proxies (the
+  element-wise oracle's pinned solve).
+* Retraction and reconstruction: the aggregate xi_* = Pi_{U_0}(sum_i c_i
+  xi~_Ui) (same for V), the polar factor polar(X) = P Q^T of the thin SVD
+  X = P S Q^T, U_* = polar(U_0 + xi_U*), and W_* = U_* S_0 V_*^T.
+* Merged parameter scope: one-dimensional parameters take the task-vector
+  average w_0 + (1/K) sum_i (w_i - w_0); ``merge_model`` applies the matrix
+  merge or the average to each tensor of a list and rounds each result once
+  to the base's encoding.
 
 Parity status: pinned (tests/test_oracle_iso_merger.py) by the identities the
 paper states -- the tangent condition, (U_0 + xi)^T (U_0 + xi) = I + xi^T xi,
@@ -99,8 +102,44 @@ def polar(X: np.ndarray) -> np.ndarray:
     return P @ Q.T
 
 
+def expert_motion(U0: np.ndarray, V0: np.ndarray, Wi: np.ndarray, k_keep: int):
+    """One expert's masked frame motion (App. E, Sign canonicalization,
+    Stiefel tangent projection and Top-k_keep masking): its thin-SVD frames
+    in the base's sign gauge, their displacements from (U0, V0) projected
+    onto the tangent spaces there, the trailing modes zeroed.  Returns
+    (xi~_U, xi~_V, signs)."""
+    Ui, _, Vi = thin_svd(Wi)
+    Ui, Vi, s = canonicalize_signs(U0, Ui, Vi)
+    xu = keep_mask(tangent_project(U0, Ui - U0), k_keep)
+    xv = keep_mask(tangent_project(V0, Vi - V0), k_keep)
+    return xu, xv, s
+
+
+def gram_matrix(g) -> np.ndarray:
+    """Gamma_ij = <g_i, g_j>_F (App. E, Retention coefficients)."""
+    K = len(g)
+    gram = np.zeros((K, K), np.float64)
+    for i in range(K):
+        for j in range(K):
+            gram[i, j] = float(np.sum(g[i] * g[j]))
+    return gram
+
+
+def aggregate_tangent(U0: np.ndarray, xis, c) -> np.ndarray:
+    """xi_* = Pi_{U0}(sum_i c_i xi~_i) (App. E, Retraction and reconstruction)."""
+    agg = np.zeros_like(U0)
+    for i in range(len(xis)):
+        agg += c[i] * xis[i]
+    return tangent_project(U0, agg)
+
+
+def retract(U0: np.ndarray, xi: np.ndarray) -> np.ndarray:
+    """The merged frame polar(U0 + xi) (App. E, Retraction and reconstruction)."""
+    return polar(U0 + xi)
+
+
 def merge_matrix(W0, experts, rho_keep=0.9, ridge=1e-12, c_min=0.0, c_max=1.5):
-    """ISO-Merger of one 2-D weight matrix (Algorithm 1, inner loop).
+    """ISO-Merger of one 2-D weight matrix (App. E).
 
     W0       base matrix (m x n)
     experts  list of K expert matrices of the same shape (checkpoints W_i)
@@ -112,35 +151,19 @@ def merge_matrix(W0, experts, rho_keep=0.9, ridge=1e-12, c_min=0.0, c_max=1.5):
     """
     W0 = np.asarray(W0, np.float64)
     U0, S0, V0 = thin_svd(W0)
-    q = S0.size
-    kk = k_keep_of(rho_keep, q)
-    K = len(experts)
-    xiU, xiV, g, signs = [], [], [], []
-    for Wi in experts:
-        Ui, _, Vi = thin_svd(Wi)
-        Ui, Vi, s = canonicalize_signs(U0, Ui, Vi)
-        signs.append(s)
-        dU, dV = Ui - U0, Vi - V0
-        xu = keep_mask(tangent_project(U0, dU), kk)
-        xv = keep_mask(tangent_project(V0, dV), kk)
-        xiU.append(xu)
-        xiV.append(xv)
-        g.append(effect_proxy(xu, xv, U0, S0, V0))
-    gram = np.zeros((K, K), np.float64)
-    for i in range(K):
-        for j in range(K):
-            gram[i, j] = float(np.sum(g[i] * g[j]))
+    kk = k_keep_of(rho_keep, S0.size)
+    motion = [expert_motion(U0, V0, np.asarray(Wi, np.float64), kk) for Wi in experts]
+    xiU = [m[0] for m in motion]
+    xiV = [m[1] for m in motion]
+    signs = [m[2] for m in motion]
+    g = [effect_proxy(xu, xv, U0, S0, V0) for xu, xv in zip(xiU, xiV)]
+    gram = gram_matrix(g)
     # zero-norm proxies are dropped inside the solve (coefficient 0)
     coef = _retention(gram, ridge, c_min, c_max)
-    aggU = np.zeros_like(U0)
-    aggV = np.zeros_like(V0)
-    for i in range(K):
-        aggU += coef[i] * xiU[i]
-        aggV += coef[i] * xiV[i]
-    xiU_star = tangent_project(U0, aggU)
-    xiV_star = tangent_project(V0, aggV)
-    U_star = polar(U0 + xiU_star)
-    V_star = polar(V0 + xiV_star)
+    xiU_star = aggregate_tangent(U0, xiU, coef)
+    xiV_star = aggregate_tangent(V0, xiV, coef)
+    U_star = retract(U0, xiU_star)
+    V_star = retract(V0, xiV_star)
     W_star = (U_star * S0) @ V_star.T
     return {"W": W_star, "U": U_star, "V": V_star, "S0": S0, "U0": U0, "V0": V0,
             "k_keep": kk, "coef": coef, "gram": gram, "g": g, "xiU": xiU, "xiV": xiV,
@@ -148,7 +171,7 @@ def merge_matrix(W0, experts, rho_keep=0.9, ridge=1e-12, c_min=0.0, c_max=1.5):
 
 
 def merge_model(theta0, experts, is_1d=None, rho_keep=0.9, ridge=1e-12, c_min=0.0, c_max=1.5):
-    """Algorithm 1 over a parameter list.
+    """The merge of a parameter list (App. E, Merged parameter scope).
 
     theta0   list of base tensors (uint16 bfloat16 bits or float32), 2-D
              matrices as (m, n) arrays

@@ -1,4 +1,4 @@
-"""Pins of the frame-space ISO-Merger oracle (App. E, Algorithm 1).
+"""Pins of the frame-space ISO-Merger oracle (App. E).
 
 Each test ties the oracle to a fact fixed outside its code: an identity the
 paper states (the Stiefel tangent condition, (U_0 + xi)^T (U_0 + xi) =
@@ -309,7 +309,7 @@ def test_masked_tangent_base_coordinates_are_skew():
 
 
 def test_model_loop_matrices_and_vectors():
-    # Algorithm 1's outer loop: matrices through the frame-space merge, 1-D
+    # the parameter-list merge: matrices through the frame-space merge, 1-D
     # parameters through the task-vector average (the element-wise oracle's
     # ISO 1-D rule), each rounded once to the base's encoding
     import oracle

@@ -74,10 +74,10 @@ MERGER_MUTATIONS = {
     "mask_keeps_every_mode": ("out[:, k_keep:] = 0.0", "out[:, k_keep:] *= 1.0"),
     "k_keep_truncates": ("k = int(np.floor(rho_keep * q + 0.5))", "k = int(np.floor(rho_keep * q))"),
     "proxy_drops_v_motion": ("return (xiU * S0) @ V0.T + (U0 * S0) @ xiV.T", "return (xiU * S0) @ V0.T"),
-    "aggregate_not_projected": ("xiU_star = tangent_project(U0, aggU)", "xiU_star = aggU"),
-    "retraction_without_polar": ("U_star = polar(U0 + xiU_star)", "U_star = U0 + xiU_star"),
+    "aggregate_not_projected": ("return tangent_project(U0, agg)", "return agg"),
+    "retraction_without_polar": ("return polar(U0 + xi)", "return U0 + xi"),
     "gram_diagonal_only": ("gram[i, j] = float(np.sum(g[i] * g[j]))", "gram[i, j] = float(np.sum(g[i] * g[i]))"),
-    "coefficients_unused": ("aggU += coef[i] * xiU[i]", "aggU += xiU[i]"),
+    "coefficients_unused": ("agg += c[i] * xis[i]", "agg += xis[i]"),
 }
 
 
