@@ -239,6 +239,63 @@ int32_t iso_update_noalloc(const iso_tensor* theta_0, const iso_tensor* update, 
                            const iso_tensor* out, int32_t n_tensors, const iso_merge_cfg* cfg,
                            const iso_merge_stats* stats, void* stream);
 
+/* ---- Frame-space ISO-Merger of one weight matrix (App. E) ----------------
+ *
+ * The paper's merge of K experts fine-tuned from one base, per 2-D weight
+ * matrix (App. E, Setup to Retraction and reconstruction): experts' singular
+ * frames aligned to the base's sign gauge (Sign canonicalization), their
+ * displacements projected onto the Stiefel tangent spaces at the base frames
+ * (Stiefel tangent projection) and masked to the leading k_keep modes
+ * (Top-k_keep singular-mode masking), retention coefficients from the Gram of
+ * the first-order effect proxies (Retention coefficients), the aggregate
+ * tangent retracted by the polar factor, and W* = U* S_0 V*^T carrying the
+ * base spectrum (Retraction and reconstruction). */
+typedef struct {
+    double  rho_keep;   /* (0, 1]: k_keep = floor(rho_keep q + 1/2) leading modes, q = min(m, n)
+                           (the paper uses 0.9) */
+    double  ridge;      /* lambda_ridge >= 0 (the paper uses 1e-12) */
+    double  c_min;      /* clip range (the paper uses [0, 1.5]) */
+    double  c_max;
+    int32_t ns_iters;   /* iteration limit of the inverse square root in the polar factor;
+                           0 = the default (16); the iteration stops at convergence */
+    int32_t reserved;   /* must be 0 */
+} iso_frame_cfg;
+
+/* Host-only.  Workspace bytes of iso_frame_merge for an m x n matrix and K
+ * experts (1 <= K <= ISO_MAX_EXPERTS, min(m, n) <= 32768, m, n < 2^24). */
+int32_t iso_frame_workspace_size(int64_t m, int64_t n, int32_t K, size_t* bytes);
+
+/* Merge one m x n matrix.  Inputs are thin SVDs, binary64, row-major, on the
+ * device, singular values in descending order (q = min(m, n)):
+ *   U0 (m x q), S0 (q), Vt0 (q x n)      the base, W_0 = U0 diag(S0) Vt0
+ *   U[i] (m x q), Vt[i] (q x n)          expert i's frames (host array of K
+ *                                        device pointers); its singular values
+ *                                        are not needed
+ * W0 is the base matrix itself (ISO_BF16 or ISO_F32, m x n); out (same dtype
+ * and shape, may coincide with W0 but share no other byte with it) receives
+ *   W* = W0 + (U* S0 V*^T - U0 S0 V0^T),
+ * i.e. the paper's U* S0 V*^T with the base's own entries in place of their
+ * reconstruction from the factors.  stats (may be NULL): status (ISO_OK or
+ * ISO_ERR_TIMEOUT), gram [K][K] (Gamma), coef [K] (c*); units is not used.
+ * The workspace (256-byte aligned, iso_frame_workspace_size bytes) is
+ * scratch for the duration of the call.  Precision: the large contractions
+ * run on the tensor cores as three tf32 products per pair (binary32
+ * accumulation, about 2^-21 relative each), the rest in binary64.  Argument
+ * errors are returned before anything is enqueued. */
+int32_t iso_frame_merge(const double* U0, const double* S0, const double* Vt0, const double* const* U,
+                        const double* const* Vt, int32_t K, int64_t m, int64_t n, const iso_tensor* W0,
+                        const iso_tensor* out, const iso_frame_cfg* cfg, void* workspace, size_t ws_bytes,
+                        const iso_merge_stats* stats, void* stream);
+
+/* The frame merge's dense product on the tensor cores, for tests of the
+ * contraction alone: C (M x N, row stride ldc) = A[:, a_k0 : a_k0 + Kc]
+ * B[:, b_k0 : b_k0 + Kc]^T, A (M rows, stride lda) and B (N rows, stride
+ * ldb) row-major binary32 read as tf32, binary32 accumulation.  M and N
+ * multiples of 128; Kc, a_k0 and b_k0 multiples of 32; strides multiples of
+ * 4; pointers 16-byte aligned.  Device pointers; enqueued on stream. */
+int32_t iso_gemm_tf32(const float* A, int64_t lda, const float* B, int64_t ldb, float* C, int64_t ldc, int64_t M,
+                      int64_t N, int64_t Kc, int64_t a_k0, int64_t b_k0, void* stream);
+
 /* Static description of a status code. */
 const char* iso_error_string(int32_t status);
 

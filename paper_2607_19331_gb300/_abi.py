@@ -58,6 +58,11 @@ class IsoMergeStats(ctypes.Structure):
                 ("gram", ctypes.c_void_p), ("coef", ctypes.c_void_p)]
 
 
+class IsoFrameCfg(ctypes.Structure):
+    _fields_ = [("rho_keep", ctypes.c_double), ("ridge", ctypes.c_double), ("c_min", ctypes.c_double),
+                ("c_max", ctypes.c_double), ("ns_iters", ctypes.c_int32), ("reserved", ctypes.c_int32)]
+
+
 # (name, restype, argtypes) for every entry point of include/iso.h
 P = ctypes.c_void_p
 PT = ctypes.POINTER(IsoTensor)
@@ -75,6 +80,10 @@ PROTOTYPES = [
                         ctypes.POINTER(IsoMergeStats), P]),
     ("iso_update_noalloc", I32, [PT, PT, I32, PT, I32, ctypes.POINTER(IsoMergeCfg),
                                  ctypes.POINTER(IsoMergeStats), P]),
+    ("iso_frame_workspace_size", I32, [I64, I64, I32, ctypes.POINTER(SZ)]),
+    ("iso_frame_merge", I32, [P, P, P, P, P, I32, I64, I64, PT, PT, ctypes.POINTER(IsoFrameCfg), P, SZ,
+                              ctypes.POINTER(IsoMergeStats), P]),
+    ("iso_gemm_tf32", I32, [P, I64, P, I64, P, I64, I64, I64, I64, I64, I64, P]),
     ("iso_error_string", ctypes.c_char_p, [I32]),
     ("iso_launch_count", ctypes.c_uint64, []),
     ("iso_force_two_pass", ctypes.c_int32, [ctypes.c_int32]),

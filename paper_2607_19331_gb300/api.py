@@ -300,3 +300,88 @@ def iso_update_noalloc(theta_0: List[torch.Tensor], update: List[torch.Tensor], 
                                    ctypes.byref(st.abi()) if st else None, _stream(stream)),
           "iso_update_noalloc")
     return (out, st) if stats else out
+
+
+# ---------------------------------------------------------------------------
+# frame-space ISO-Merger of one matrix (App. E)
+# ---------------------------------------------------------------------------
+@dataclass
+class FrameStats:
+    """Device-side outputs of iso_frame_merge."""
+    status: torch.Tensor   # int32[1]
+    gram: torch.Tensor     # float64[K, K]
+    coef: torch.Tensor     # float64[K]
+
+    def abi(self) -> IsoMergeStats:
+        return IsoMergeStats(self.status.data_ptr(), None, self.gram.data_ptr(), self.coef.data_ptr())
+
+
+def frame_workspace_size(m: int, n: int, K: int) -> int:
+    b = ctypes.c_size_t(0)
+    check(lib().iso_frame_workspace_size(int(m), int(n), int(K), ctypes.byref(b)), "iso_frame_workspace_size")
+    return int(b.value)
+
+
+def frame_merge_factors(U0, S0, Vt0, Us, Vts, W0, out=None, rho_keep=0.9, ridge=1e-12, c_min=0.0, c_max=1.5,
+                        ns_iters=0, workspace=None, stats=False, stream=None):
+    """iso_frame_merge: the ISO-Merger of one m x n matrix from the thin SVD
+    factors of the base (U0 m x q, S0 q, Vt0 q x n) and of the K experts (Us,
+    Vts), binary64 and contiguous on the device; W0 is the base matrix (bf16
+    or fp32).  Returns out (and FrameStats with stats=True)."""
+    m, n = int(W0.shape[0]), int(W0.shape[1])
+    K = len(Us)
+    if len(Vts) != K:
+        raise ValueError("one U and one Vt per expert")
+    for t in [U0, S0, Vt0, *Us, *Vts]:
+        if t.dtype != torch.float64 or not t.is_contiguous():
+            raise ValueError("SVD factors must be contiguous float64 tensors")
+    if out is None:
+        out = torch.empty_like(W0)
+    dev = W0.device
+    cfg = _abi.IsoFrameCfg(float(rho_keep), float(ridge), float(c_min), float(c_max), int(ns_iters), 0)
+    need = frame_workspace_size(m, n, K)
+    ws = _workspace(workspace, dev)
+    wptr, wlen = ws.get(need)
+    up = (ctypes.c_void_p * K)(*[u.data_ptr() for u in Us])
+    vp = (ctypes.c_void_p * K)(*[v.data_ptr() for v in Vts])
+    st = None
+    if stats:
+        st = FrameStats(torch.zeros(1, dtype=torch.int32, device=dev),
+                        torch.zeros(K, K, dtype=torch.float64, device=dev),
+                        torch.zeros(K, dtype=torch.float64, device=dev))
+    rc = lib().iso_frame_merge(U0.data_ptr(), S0.data_ptr(), Vt0.data_ptr(), up, vp, K, m, n,
+                               describe([W0]), describe([out]), ctypes.byref(cfg), wptr, wlen,
+                               ctypes.byref(st.abi()) if st else None, _stream(stream))
+    check(rc, "iso_frame_merge")
+    return (out, st) if stats else out
+
+
+def thin_svd(W: torch.Tensor):
+    """The thin SVD W = U diag(S) Vt in binary64 on W's device (the library
+    SVD of torch.linalg; the frame merge's one step that is not this
+    library's own code)."""
+    U, S, Vt = torch.linalg.svd(W.to(torch.float64), full_matrices=False)
+    return U.contiguous(), S.contiguous(), Vt.contiguous()
+
+
+def frame_merge(W0: torch.Tensor, experts: Sequence[torch.Tensor], **kw):
+    """ISO-Merger of one matrix from the base and K expert checkpoints: the
+    thin SVDs (thin_svd), then iso_frame_merge."""
+    U0, S0, Vt0 = thin_svd(W0)
+    Us, Vts = [], []
+    for E in experts:
+        U, _, Vt = thin_svd(E)
+        Us.append(U)
+        Vts.append(Vt)
+    return frame_merge_factors(U0, S0, Vt0, Us, Vts, W0, **kw)
+
+
+def gemm_tf32(A: torch.Tensor, B: torch.Tensor, C: torch.Tensor, Kc: int, a_k0=0, b_k0=0, stream=None):
+    """iso_gemm_tf32: C = A[:, a_k0:a_k0+Kc] B[:, b_k0:b_k0+Kc]^T on the tensor cores (tf32)."""
+    for t in (A, B, C):
+        if t.dtype != torch.float32 or not t.is_contiguous() or t.dim() != 2:
+            raise ValueError("gemm_tf32 takes contiguous 2-D float32 tensors")
+    rc = lib().iso_gemm_tf32(A.data_ptr(), A.shape[1], B.data_ptr(), B.shape[1], C.data_ptr(), C.shape[1],
+                             A.shape[0], B.shape[0], int(Kc), int(a_k0), int(b_k0), _stream(stream))
+    check(rc, "iso_gemm_tf32")
+    return C

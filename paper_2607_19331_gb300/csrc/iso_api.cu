@@ -27,12 +27,12 @@ constexpr int FUSED_GRID_PER_SM = FUSED_BLOCKS_PER_SM;
 enum Kind {
     KD_UPLOAD, KD_INIT, KD_SAMPLE, KD_COUNT, KD_DECIDE, KD_RADIX_HIST, KD_RADIX_PICK, KD_TIE,
     KD_CUT, KD_BLOCK_SELECT, KD_GRAM, KD_SOLVE, KD_APPLY, KD_MASK, KD_DELTA, KD_STATUS, KD_MEMSET,
-    KD_PATCH, KD_REPAIR, KD_COUNT_KINDS
+    KD_PATCH, KD_REPAIR, KD_FRAME_GEMM, KD_FRAME, KD_COUNT_KINDS
 };
 const char* kKindNames[KD_COUNT_KINDS] = {
     "upload", "init_units", "sample", "count", "decide", "radix_hist", "radix_pick", "tie",
     "cut", "block_select", "gram", "solve", "apply", "mask", "delta", "status", "memset",
-    "patch", "repair"};
+    "patch", "repair", "frame_gemm", "frame"};
 
 std::atomic<uint64_t> g_launches{0};
 
@@ -82,7 +82,9 @@ int launch(int kind, cudaStream_t s, F&& f) {
     return (cudaGetLastError() == cudaSuccess) ? ISO_OK : ISO_ERR_CUDA;
 }
 
+#ifndef ISO_TRY
 #define ISO_TRY(x) do { int _r = (x); if (_r != ISO_OK) return _r; } while (0)
+#endif
 
 // ---------------------------------------------------------------------------
 // device properties (cached per device)
@@ -783,6 +785,32 @@ int build_merge_call(Call& c, const iso_tensor* theta_0, const iso_tensor* exper
 }
 
 }  // namespace
+
+// Launch accounting and profiling for the frame-space merge (iso_frame.cu).
+int prof_begin(int frame_kind, cudaStream_t s) {
+    if (!g_prof.on) return -1;
+    const int kind = frame_kind == 0 ? KD_FRAME_GEMM : KD_FRAME;
+    std::lock_guard<std::mutex> lk(g_prof_mu);
+    if (g_prof.used >= Prof::CAP) return -1;
+    const int slot = g_prof.used;
+    if ((int)g_prof.ev.size() < 2 * (slot + 1)) {
+        cudaEvent_t a, b;
+        if (cudaEventCreate(&a) != cudaSuccess) return -1;
+        if (cudaEventCreate(&b) != cudaSuccess) { cudaEventDestroy(a); return -1; }
+        g_prof.ev.push_back(a);
+        g_prof.ev.push_back(b);
+        g_prof.kind.push_back(kind);
+    } else {
+        g_prof.kind[slot] = kind;
+    }
+    g_prof.used++;
+    cudaEventRecord(g_prof.ev[2 * slot], s);
+    return slot;
+}
+void prof_end(int slot, cudaStream_t s) {
+    if (slot >= 0) cudaEventRecord(g_prof.ev[2 * slot + 1], s);
+    g_launches.fetch_add(1, std::memory_order_relaxed);
+}
 }  // namespace iso
 
 // ===========================================================================

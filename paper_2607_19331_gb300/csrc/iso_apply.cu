@@ -212,43 +212,7 @@ __global__ void k_solve(Plan P, int gram_mode) {
                     G[b * K + a] = v;
                 }
         }
-        // I = {i : Gamma_ii > 0}; (Gamma_II + ridge I) c_I = diag(Gamma)_I; clip
-        int idx[MAXK];
-        int m = 0;
-        for (int i = 0; i < K; ++i)
-            if (G[i * K + i] > 0.0) idx[m++] = i;
-        double A[MAXK * MAXK], rhs[MAXK], x[MAXK];
-        for (int r = 0; r < m; ++r) {
-            for (int q = 0; q < m; ++q) A[r * m + q] = G[idx[r] * K + idx[q]];
-            A[r * m + r] = __dadd_rn(A[r * m + r], P.ridge);
-            rhs[r] = G[idx[r] * K + idx[r]];
-        }
-        // Gaussian elimination with partial pivoting
-        for (int col = 0; col < m; ++col) {
-            int piv = col;
-            for (int r = col + 1; r < m; ++r)
-                if (fabs(A[r * m + col]) > fabs(A[piv * m + col])) piv = r;
-            if (piv != col) {
-                for (int q = 0; q < m; ++q) { double s = A[col * m + q]; A[col * m + q] = A[piv * m + q]; A[piv * m + q] = s; }
-                double s = rhs[col]; rhs[col] = rhs[piv]; rhs[piv] = s;
-            }
-            for (int r = col + 1; r < m; ++r) {
-                const double f = A[r * m + col] / A[col * m + col];
-                for (int q = col; q < m; ++q) A[r * m + q] = __dadd_rn(A[r * m + q], -__dmul_rn(f, A[col * m + q]));
-                rhs[r] = __dadd_rn(rhs[r], -__dmul_rn(f, rhs[col]));
-            }
-        }
-        for (int r = m - 1; r >= 0; --r) {
-            double s = rhs[r];
-            for (int q = r + 1; q < m; ++q) s = __dadd_rn(s, -__dmul_rn(A[r * m + q], x[q]));
-            x[r] = s / A[r * m + r];
-        }
-        for (int r = 0; r < m; ++r) {
-            double v = x[r];
-            if (v < P.c_min) v = P.c_min;
-            if (v > P.c_max) v = P.c_max;
-            c[idx[r]] = v;
-        }
+        retention_solve(G, K, P.ridge, P.c_min, P.c_max, c);
     }
     for (int i = 0; i < K; ++i) P.coef[(long long)t * K + i] = c[i];
     if (P.repair) {

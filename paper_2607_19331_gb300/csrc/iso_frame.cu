@@ -1,0 +1,778 @@
+// iso_frame.cu -- the frame-space ISO-Merger of one weight matrix (App. E)
+// on one GPU.
+//
+// Given the thin SVDs W_0 = U_0 S_0 V_0^T (base) and W_i = U_i S_i V_i^T
+// (experts, i = 1..K; their spectra are not used), the merge is
+//   s_ik   = sign(<u_0k, u_ik>), sign(0) := 1                  (Sign canonicalization)
+//   xi_Fi  = Pi_{F_0}(s_i F_i - F_0) D_keep,  F in {U, V}       (Stiefel tangent projection,
+//            Pi_{F_0}(X) = X - F_0 sym(F_0^T X)                  Top-k_keep masking)
+//   g_i    = xi_Ui S_0 V_0^T + U_0 S_0 xi_Vi^T, Gamma_ij = <g_i, g_j>_F
+//   c*     = clip((Gamma + ridge I)^-1 diag Gamma)              (Retention coefficients)
+//   xi_F*  = Pi_{F_0}(sum_i c*_i xi_Fi),  F* = polar(F_0 + xi_F*) (Retraction and
+//   W*     = U* S_0 V*^T                                          reconstruction)
+//
+// How it is computed here (every identity below is pinned against the binary64
+// oracle of the same definitions):
+// * Nothing of size m x n is formed but the output.  With A_i = F_0^T dF_i
+//   (dF_i = s_i F_i - F_0), Sym_i = sym(A_i), Kw_i = A_i - Sym_i:
+//     F_0^T xi_Fi = Kw_i D,
+//     (xi_Fi^T xi_Fj)_kk = D_k [(dF_i^T dF_j)_kk - (A_i^T Sym_j)_kk - (Sym_i A_j)_kk + (Sym_i Sym_j)_kk],
+//     Gamma_ij = sum_k s_k^2 [(xi_Ui^T xi_Uj)_kk + (xi_Vi^T xi_Vj)_kk]
+//                - sum_kl s_k s_l D_k D_l (KwU_i KwV_j + KwU_j KwV_i)[k, l],
+//     xi_F* = D dF_c - F_0 Y,  dF_c = sum_i c*_i dF_i,
+//     Y = (sum_i c*_i Sym_i) D + sym((sum_i c*_i Kw_i) D).
+// * polar(F_0 + xi) = (F_0 + xi)(I + xi^T xi)^(-1/2), since F_0^T xi is skew;
+//   the inverse square root comes from the coupled Newton-Schulz iteration
+//   written in differences from the identity (Y = I + y, Z = I + z), so that
+//   every product is of small matrices, scaled when ||xi^T xi||_F >= 0.9.
+// * W* = W_0 + [E_U S_0 | U_0 S_0] [V* | E_V]^T with E_F = F* - F_0: the
+//   difference form keeps the low-precision products on the small motion;
+//   W_0 itself (the caller's matrix) replaces U_0 S_0 V_0^T.
+// * The large contractions run on the tensor cores (k_gemm_tf32) in three tf32
+//   products per pair (hi hi + hi lo + lo hi, x = hi + lo split in binary64),
+//   binary32 accumulation: about 2^-21 relative per product.  Everything else
+//   is binary64 on the CUDA cores.
+#include "iso_gemm.cuh"
+#include "iso_internal.cuh"
+
+#include <algorithm>
+#include <cmath>
+#include <vector>
+
+namespace iso {
+
+namespace {
+
+constexpr int FR_PAD = 128;        // operand arrays padded to whole GEMM tiles
+constexpr int FR_MAX_NS = 64;      // Newton-Schulz iteration limit
+constexpr int FR_DEFAULT_NS = 16;
+constexpr double FR_NS_TOL = 1e-9; // max |y + z + z y| at which the iteration has converged
+
+long long pad_up(long long x) { return (x + FR_PAD - 1) / FR_PAD * FR_PAD; }
+
+struct FrameHeader {
+    int32_t status;
+    int32_t conv[2];                // per side: the Newton-Schulz iteration has converged
+    int32_t pad;
+    double nu2[2];                  // per side: ||xi^T xi||_F^2
+    double cs[2];                   // per side: the scaling of I + xi^T xi
+    uint32_t wmax[2][FR_MAX_NS];    // per side and iteration: max |w| as binary32 bits
+};
+
+// binary64 -> (hi, lo) with hi a tf32 value (round to nearest, ties away) and
+// lo the binary32 rest, so that hi + lo = x to about 2^-22 |x|
+__device__ __forceinline__ void split_tf32(double x, float& hi, float& lo) {
+    const float x32 = (float)x;
+    uint32_t h;
+    asm("cvt.rna.tf32.f32 %0, %1;" : "=r"(h) : "f"(x32));
+    hi = __uint_as_float(h);
+    const float l32 = (float)(x - (double)hi);
+    uint32_t l;
+    asm("cvt.rna.tf32.f32 %0, %1;" : "=r"(l) : "f"(l32));
+    lo = __uint_as_float(l);
+}
+
+// An operand row of contraction length L (padded) is stored in four segments
+// [hi | lo | hi | hi]: read from segment 0 it is (hi, lo, hi), from segment 1
+// (lo, hi, hi); A from 0 and B from 1 pair up as hi lo + lo hi + hi hi.
+__device__ __forceinline__ void put_split(float* row, long long L, long long k, double x) {
+    float hi, lo;
+    split_tf32(x, hi, lo);
+    row[k] = hi;
+    row[L + k] = lo;
+    row[2 * L + k] = hi;
+    row[3 * L + k] = hi;
+}
+
+struct Frames {                     // one side (U: d = m; V: d = n), d x q row-major binary64
+    const double* F0;
+    const double* F[MAXK];
+    int K;
+    long long d, q;
+};
+
+// ---------------------------------------------------------------------------
+// layout helpers
+// ---------------------------------------------------------------------------
+// out (C x R) = in (R x C)^T, binary64, 32 x 32 tiles
+__global__ void __launch_bounds__(256) k_fr_transpose(const double* in, double* out, long long R, long long C) {
+    __shared__ double t[32][33];
+    const long long r0 = (long long)blockIdx.y * 32, c0 = (long long)blockIdx.x * 32;
+    for (int y = threadIdx.y; y < 32; y += 8) {
+        const long long r = r0 + y, c = c0 + threadIdx.x;
+        t[y][threadIdx.x] = (r < R && c < C) ? in[r * C + c] : 0.0;
+    }
+    __syncthreads();
+    for (int y = threadIdx.y; y < 32; y += 8) {
+        const long long c = c0 + y, r = r0 + threadIdx.x;
+        if (c < C && r < R) out[c * R + r] = t[threadIdx.x][y];
+    }
+}
+
+// s_ik = sign(<u_0k, u_ik>): the column dot products (U side), summed into dots[i][k]
+__global__ void __launch_bounds__(256) k_fr_signdots(Frames f, double* dots, int row_chunks) {
+    __shared__ double red[8][33];
+    const long long k = (long long)blockIdx.x * 32 + threadIdx.x;
+    const int i = blockIdx.y;
+    const long long per = (f.d + row_chunks - 1) / row_chunks;
+    const long long r0 = (long long)blockIdx.z * per, r1 = min(f.d, r0 + per);
+    double acc = 0.0;
+    if (k < f.q)
+        for (long long r = r0 + threadIdx.y; r < r1; r += 8) acc = fma(f.F0[r * f.q + k], f.F[i][r * f.q + k], acc);
+    red[threadIdx.y][threadIdx.x] = acc;
+    __syncthreads();
+    if (threadIdx.y == 0 && k < f.q) {
+        double s = 0.0;
+        for (int y = 0; y < 8; ++y) s += red[y][threadIdx.x];
+        atomicAdd(&dots[(long long)i * f.q + k], s);
+    }
+}
+
+__device__ __forceinline__ double sign_of(const double* dots, long long q, int i, long long k) {
+    return dots[(long long)i * q + k] < 0.0 ? -1.0 : 1.0;
+}
+
+// (dF_i^T dF_j)_kk for i <= j, summed into cd[i][j][k]
+__global__ void __launch_bounds__(256) k_fr_coldots(Frames f, const double* dots, double* cd, int row_chunks) {
+    __shared__ double red[8][33];
+    const long long k = (long long)blockIdx.x * 32 + threadIdx.x;
+    const int K = f.K;
+    const long long per = (f.d + row_chunks - 1) / row_chunks;
+    const long long r0 = (long long)blockIdx.y * per, r1 = min(f.d, r0 + per);
+    double acc[MAXK * (MAXK + 1) / 2];
+#pragma unroll
+    for (int p = 0; p < MAXK * (MAXK + 1) / 2; ++p) acc[p] = 0.0;
+    double sg[MAXK];
+#pragma unroll
+    for (int i = 0; i < MAXK; ++i) sg[i] = (i < K && k < f.q) ? sign_of(dots, f.q, i, k) : 0.0;
+    if (k < f.q) {
+        for (long long r = r0 + threadIdx.y; r < r1; r += 8) {
+            const double f0 = f.F0[r * f.q + k];
+            double dv[MAXK];
+#pragma unroll
+            for (int i = 0; i < MAXK; ++i) dv[i] = (i < K) ? fma(sg[i], f.F[i][r * f.q + k], -f0) : 0.0;
+            int p = 0;
+#pragma unroll
+            for (int i = 0; i < MAXK; ++i)
+#pragma unroll
+                for (int j = i; j < MAXK; ++j) acc[p] = fma(dv[i], dv[j], acc[p]), ++p;
+        }
+    }
+    int p = 0;
+    for (int i = 0; i < MAXK; ++i)
+        for (int j = i; j < MAXK; ++j, ++p) {
+            if (i >= K || j >= K) continue;
+            red[threadIdx.y][threadIdx.x] = acc[p];
+            __syncthreads();
+            if (threadIdx.y == 0 && k < f.q) {
+                double s = 0.0;
+                for (int y = 0; y < 8; ++y) s += red[y][threadIdx.x];
+                atomicAdd(&cd[((long long)i * K + j) * f.q + k], s);
+            }
+            __syncthreads();
+        }
+}
+
+// Transposed split operand out[k][seg][r] (Qp rows of 4 Dp) of a d x q source:
+// mode 0: F_0; mode 1: dF_i = s_i F_i - F_0; mode 2: the binary64 array X
+struct SplitT {
+    Frames f;
+    const double* dots;
+    const double* X;
+    int mode, i;
+    float* out;
+    long long Dp, Qp;
+};
+__global__ void __launch_bounds__(256) k_fr_split_t(SplitT a) {
+    __shared__ double t[32][33];
+    const long long r0 = (long long)blockIdx.x * 32, k0 = (long long)blockIdx.y * 32;
+    const long long d = a.f.d, q = a.f.q;
+    for (int y = threadIdx.y; y < 32; y += 8) {
+        const long long r = r0 + y, k = k0 + threadIdx.x;
+        double v = 0.0;
+        if (r < d && k < q) {
+            const long long e = r * q + k;
+            if (a.mode == 0) v = a.f.F0[e];
+            else if (a.mode == 1) v = fma(sign_of(a.dots, q, a.i, k), a.f.F[a.i][e], -a.f.F0[e]);
+            else v = a.X[e];
+        }
+        t[y][threadIdx.x] = v;
+    }
+    __syncthreads();
+    for (int y = threadIdx.y; y < 32; y += 8) {
+        const long long k = k0 + y, r = r0 + threadIdx.x;
+        if (k < a.Qp && r < a.Dp) put_split(a.out + k * 4 * a.Dp, a.Dp, r, t[threadIdx.x][y]);
+    }
+}
+
+// Row-major split operand out[r][seg][c] (rows_p rows of 4 Lp), element value by mode:
+//   0  F_0[r, c]                          (d x q)
+//   1  F_0[r, c] + X[r, c]                (d x q)
+//   2  M[r, c]                            (q x q binary64)
+//   3  Y^T[r, c] of the aggregate          (q x q)
+//   4  [E_U S_0 | U_0 S_0]                (m x 2 Qp: c < Qp from X = E_U, else U_0)
+//   5  [V_0 + E_V | E_V]                  (n x 2 Qp: X = E_V)
+//   6  R = (z + (1 - sqrt cs) I) / sqrt cs (q x q, M = z)
+struct SplitR {
+    Frames f;
+    const double* X;
+    const double* M;
+    const double* S0;
+    const double* sym;     // mode 3: K arrays q x q (Sym_i), then K arrays (Kw_i)
+    const double* kw;
+    const double* coef;
+    const FrameHeader* hdr;
+    int side;
+    long long k_keep;
+    int mode;
+    float* out;
+    long long rows, rows_p, Lp;
+};
+__global__ void __launch_bounds__(256) k_fr_split_r(SplitR a) {
+    const long long total = a.rows_p * a.Lp;
+    const long long q = a.f.q;
+    for (long long e = (long long)blockIdx.x * blockDim.x + threadIdx.x; e < total; e += (long long)gridDim.x * blockDim.x) {
+        const long long r = e / a.Lp, c = e - r * a.Lp;
+        double v = 0.0;
+        if (r < a.rows) {
+            switch (a.mode) {
+                case 0: if (c < q) v = a.f.F0[r * q + c]; break;
+                case 1: if (c < q) v = a.f.F0[r * q + c] + a.X[r * q + c]; break;
+                case 2: if (c < q) v = a.M[r * q + c]; break;
+                case 3:
+                    if (c < q) {
+                        // Y^T[j, k] = Y[k, j] = Sc[j, k] D_j - Kwc[j, k] (D_j - D_k) / 2
+                        const double Dj = r < a.k_keep ? 1.0 : 0.0, Dk = c < a.k_keep ? 1.0 : 0.0;
+                        double sc = 0.0, kc = 0.0;
+                        for (int i = 0; i < a.f.K; ++i) {
+                            sc = fma(a.coef[i], a.sym[((long long)i * q + r) * q + c], sc);
+                            kc = fma(a.coef[i], a.kw[((long long)i * q + r) * q + c], kc);
+                        }
+                        v = sc * Dj - 0.5 * kc * (Dj - Dk);
+                    }
+                    break;
+                case 4: {
+                    const long long Qp = a.Lp / 2;
+                    if (c < Qp) { if (c < q) v = a.X[r * q + c] * a.S0[c]; }
+                    else if (c - Qp < q) v = a.f.F0[r * q + (c - Qp)] * a.S0[c - Qp];
+                    break;
+                }
+                case 5: {
+                    const long long Qp = a.Lp / 2;
+                    if (c < Qp) { if (c < q) v = a.f.F0[r * q + c] + a.X[r * q + c]; }
+                    else if (c - Qp < q) v = a.X[r * q + (c - Qp)];
+                    break;
+                }
+                case 6:
+                    if (c < q) {
+                        const double sc = sqrt(a.hdr->cs[a.side]);
+                        v = (a.M[r * q + c] + (r == c ? 1.0 - sc : 0.0)) / sc;
+                    }
+                    break;
+            }
+        }
+        put_split(a.out + r * 4 * a.Lp, a.Lp, c, v);
+    }
+}
+
+// Sym_i = sym(A_i), Kw_i = A_i - Sym_i (binary64) from the GEMM's A_i (binary32, ld Qp)
+__global__ void __launch_bounds__(256) k_fr_symskew(const float* A, long long Qp, long long q, double* sym, double* kw) {
+    __shared__ float ta[32][33], tb[32][33];
+    const int i = blockIdx.z;
+    const float* Ai = A + (long long)i * Qp * Qp;
+    const long long r0 = (long long)blockIdx.y * 32, c0 = (long long)blockIdx.x * 32;
+    for (int y = threadIdx.y; y < 32; y += 8) {
+        ta[y][threadIdx.x] = Ai[(r0 + y) * Qp + c0 + threadIdx.x];   // A[r0 + y, c0 + x]
+        tb[y][threadIdx.x] = Ai[(c0 + y) * Qp + r0 + threadIdx.x];   // A[c0 + y, r0 + x]
+    }
+    __syncthreads();
+    for (int y = threadIdx.y; y < 32; y += 8) {
+        const long long r = r0 + y, c = c0 + threadIdx.x;
+        if (r < q && c < q) {
+            const double a = ta[y][threadIdx.x], b = tb[threadIdx.x][y];   // A[r, c], A[c, r]
+            sym[((long long)i * q + r) * q + c] = 0.5 * (a + b);
+            kw[((long long)i * q + r) * q + c] = 0.5 * (a - b);
+        }
+    }
+}
+
+// Gamma_ij (i <= j), summed into gram[i][j]; block y covers a slice of the q x q entries
+struct GramArgs {
+    const float* A[2];          // per side: K arrays Qp x Qp
+    const double* sym[2];
+    const double* kw[2];
+    const double* cd[2];        // per side: K x K x q
+    const double* S0;
+    double* gram;
+    long long q, Qp, k_keep;
+    int K;
+};
+__global__ void __launch_bounds__(256) k_fr_gram(GramArgs g) {
+    __shared__ double red[32];
+    // pair (i, j), i <= j, from blockIdx.x
+    int i = 0, j = 0, p = blockIdx.x;
+    for (i = 0; i < g.K; ++i) {
+        if (p < g.K - i) { j = i + p; break; }
+        p -= g.K - i;
+    }
+    const long long q = g.q, qq = q * q;
+    const long long per = (qq + gridDim.y - 1) / gridDim.y;
+    const long long e0 = (long long)blockIdx.y * per, e1 = min(qq, e0 + per);
+    double acc = 0.0;
+    for (long long e = e0 + threadIdx.x; e < e1; e += blockDim.x) {
+        const long long r = e / q, c = e - r * q;
+        const double sr = g.S0[r], sc = g.S0[c];
+        const double Dr = r < g.k_keep ? 1.0 : 0.0, Dc = c < g.k_keep ? 1.0 : 0.0;
+        // column terms (row l = r, column k = c), both sides
+        double colt = 0.0;
+#pragma unroll
+        for (int s = 0; s < 2; ++s) {
+            const double ai = g.A[s][(long long)i * g.Qp * g.Qp + r * g.Qp + c];
+            const double aj = g.A[s][(long long)j * g.Qp * g.Qp + r * g.Qp + c];
+            const double si = g.sym[s][(long long)i * qq + e], sj = g.sym[s][(long long)j * qq + e];
+            colt += ai * sj + si * aj - si * sj;
+        }
+        acc -= sc * sc * Dc * colt;
+        // cross terms (k = r, l = c)
+        const double kui = g.kw[0][(long long)i * qq + e], kuj = g.kw[0][(long long)j * qq + e];
+        const double kvi = g.kw[1][(long long)i * qq + e], kvj = g.kw[1][(long long)j * qq + e];
+        acc -= sr * sc * Dr * Dc * (kui * kvj + kuj * kvi);
+    }
+    if (blockIdx.y == 0)
+        for (long long k = threadIdx.x; k < min(q, g.k_keep); k += blockDim.x)
+            acc += g.S0[k] * g.S0[k] *
+                   (g.cd[0][((long long)i * g.K + j) * q + k] + g.cd[1][((long long)i * g.K + j) * q + k]);
+    acc = block_sum(acc, red);
+    if (threadIdx.x == 0) atomicAdd(&g.gram[i * g.K + j], acc);
+}
+
+// c* from Gamma (upper triangle), then the caller's stats
+__global__ void k_fr_solve(double* gram, double* coef, int K, double ridge, double c_min, double c_max,
+                           double* st_gram, double* st_coef) {
+    if (threadIdx.x != 0 || blockIdx.x != 0) return;
+    double G[MAXK * MAXK], c[MAXK];
+    for (int a = 0; a < K; ++a)
+        for (int b = a; b < K; ++b) {
+            G[a * K + b] = gram[a * K + b];
+            G[b * K + a] = gram[a * K + b];
+        }
+    for (int a = 0; a < K * K; ++a) gram[a] = G[a];
+    retention_solve(G, K, ridge, c_min, c_max, c);
+    for (int a = 0; a < K; ++a) coef[a] = c[a];
+    if (st_gram) for (int a = 0; a < K * K; ++a) st_gram[a] = G[a];
+    if (st_coef) for (int a = 0; a < K; ++a) st_coef[a] = c[a];
+}
+
+// xi* = D dF_c - E (E = F_0 Y from the GEMM, ld Qp)
+__global__ void __launch_bounds__(256) k_fr_xi(Frames f, const double* dots, const double* coef, const float* E,
+                                               long long Qp, long long k_keep, double* xi) {
+    const long long total = f.d * f.q;
+    for (long long e = (long long)blockIdx.x * blockDim.x + threadIdx.x; e < total; e += (long long)gridDim.x * blockDim.x) {
+        const long long r = e / f.q, k = e - r * f.q;
+        double v = 0.0;
+        if (k < k_keep) {
+            const double f0 = f.F0[e];
+            for (int i = 0; i < f.K; ++i) v = fma(coef[i], fma(sign_of(dots, f.q, i, k), f.F[i][e], -f0), v);
+        }
+        xi[e] = v - (double)E[r * Qp + k];
+    }
+}
+
+// ||N||_F^2 of N = xi^T xi (binary32, ld Qp), summed into the header
+__global__ void __launch_bounds__(256) k_fr_norm(const float* N, long long Qp, long long q, FrameHeader* h, int side) {
+    __shared__ double red[32];
+    double acc = 0.0;
+    for (long long e = (long long)blockIdx.x * blockDim.x + threadIdx.x; e < q * q; e += (long long)gridDim.x * blockDim.x) {
+        const long long r = e / q, c = e - r * q;
+        const double v = N[r * Qp + c];
+        acc += v * v;
+    }
+    acc = block_sum(acc, red);
+    if (threadIdx.x == 0) atomicAdd(&h->nu2[side], acc);
+}
+
+// Newton-Schulz start: Y_0 = (I + N) / cs = I + y, Z_0 = I (z = 0)
+__global__ void __launch_bounds__(256) k_fr_ns_init(const float* N, long long Qp, long long q, FrameHeader* h,
+                                                    int side, double* y, double* z) {
+    const double nu = sqrt(h->nu2[side]);
+    const double cs = nu < 0.9 ? 1.0 : 1.0 + 0.5 * nu;
+    if (blockIdx.x == 0 && threadIdx.x == 0) {
+        h->cs[side] = cs;
+        h->conv[side] = 0;
+    }
+    for (long long e = (long long)blockIdx.x * blockDim.x + threadIdx.x; e < q * q; e += (long long)gridDim.x * blockDim.x) {
+        const long long r = e / q, c = e - r * q;
+        const double id = r == c ? 1.0 : 0.0;
+        y[e] = (id + (double)N[r * Qp + c]) / cs - id;
+        z[e] = 0.0;
+    }
+}
+
+// w = y + z + z y, m = -w / 2; the largest |w| of the iteration into the header
+__global__ void __launch_bounds__(256) k_fr_ns_m(const double* y, const double* z, const float* zy, long long Qp,
+                                                 long long q, double* m, FrameHeader* h, int side, int it) {
+    if (*reinterpret_cast<volatile int32_t*>(&h->conv[side])) return;
+    float wm = 0.0f;
+    for (long long e = (long long)blockIdx.x * blockDim.x + threadIdx.x; e < q * q; e += (long long)gridDim.x * blockDim.x) {
+        const long long r = e / q, c = e - r * q;
+        const double w = y[e] + z[e] + (double)zy[r * Qp + c];
+        m[e] = -0.5 * w;
+        wm = fmaxf(wm, (float)fabs(w));
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) wm = fmaxf(wm, __shfl_xor_sync(0xFFFFFFFFu, wm, o));
+    if ((threadIdx.x & 31) == 0) atomicMax(&h->wmax[side][it], __float_as_uint(wm));
+}
+
+// y += m + y m, z += m + m z; converged once max |w| <= FR_NS_TOL
+__global__ void __launch_bounds__(256) k_fr_ns_update(double* y, double* z, const double* m, const float* ym,
+                                                      const float* mz, long long Qp, long long q, FrameHeader* h,
+                                                      int side, int it) {
+    if (*reinterpret_cast<volatile int32_t*>(&h->conv[side])) return;
+    for (long long e = (long long)blockIdx.x * blockDim.x + threadIdx.x; e < q * q; e += (long long)gridDim.x * blockDim.x) {
+        const long long r = e / q, c = e - r * q;
+        y[e] += m[e] + (double)ym[r * Qp + c];
+        z[e] += m[e] + (double)mz[r * Qp + c];
+    }
+    if (blockIdx.x == 0 && threadIdx.x == 0 && (double)__uint_as_float(h->wmax[side][it]) <= FR_NS_TOL)
+        h->conv[side] = 1;
+}
+
+// E_F = xi* + (F_0 + xi*) R (P from the GEMM, ld Qp), in place over xi*
+__global__ void __launch_bounds__(256) k_fr_motion(double* xi, const float* P, long long Qp, long long d, long long q) {
+    for (long long e = (long long)blockIdx.x * blockDim.x + threadIdx.x; e < d * q; e += (long long)gridDim.x * blockDim.x) {
+        const long long r = e / q, c = e - r * q;
+        xi[e] += (double)P[r * Qp + c];
+    }
+}
+
+__global__ void k_fr_status(const FrameHeader* h, int32_t* out) {
+    if (threadIdx.x == 0 && blockIdx.x == 0) *out = h->status;
+}
+
+// ---------------------------------------------------------------------------
+// host
+// ---------------------------------------------------------------------------
+size_t al256(size_t v) { return (v + 255) & ~(size_t)255; }
+
+struct FrameLayout {
+    long long m, n, q, Mp, Np, Qp, K;
+    size_t hdr, gram, coef, dots, vcopy;
+    size_t cd[2], ft4[2], dft4[2], aq[2], sym[2], kw[2], fr4[2], y4[2], e[2], xi[2], nq[2];
+    size_t ns_y, ns_z, ns_m, ns_y4, ns_z4, ns_m4, ns_t1, ns_t2, ns_t3;
+    size_t a6, b6, total;
+};
+
+FrameLayout frame_layout(long long m, long long n, int K) {
+    FrameLayout L;
+    L.m = m; L.n = n; L.K = K;
+    L.q = std::min(m, n);
+    L.Mp = pad_up(m); L.Np = pad_up(n); L.Qp = pad_up(L.q);
+    const long long q = L.q, Qp = L.Qp;
+    size_t o = 0;
+    auto take = [&](size_t bytes) { const size_t at = o; o = al256(o + bytes); return at; };
+    L.hdr = take(sizeof(FrameHeader));
+    L.gram = take(sizeof(double) * K * K);
+    L.coef = take(sizeof(double) * K);
+    L.dots = take(sizeof(double) * K * q);
+    for (int s = 0; s < 2; ++s) L.cd[s] = take(sizeof(double) * K * K * q);
+    L.vcopy = take(sizeof(double) * (K + 1) * n * q);
+    for (int s = 0; s < 2; ++s) {
+        const long long Dp = s == 0 ? L.Mp : L.Np, d = s == 0 ? m : n;
+        L.ft4[s] = take(sizeof(float) * Qp * 4 * Dp);      // F_0^T split, later xi*^T split
+        L.dft4[s] = take(sizeof(float) * Qp * 4 * Dp);     // dF_i^T split (one expert at a time)
+        L.aq[s] = take(sizeof(float) * K * Qp * Qp);
+        L.sym[s] = take(sizeof(double) * K * q * q);
+        L.kw[s] = take(sizeof(double) * K * q * q);
+        L.fr4[s] = take(sizeof(float) * Dp * 4 * Qp);      // F_0 split, later (F_0 + xi*) split
+        L.y4[s] = take(sizeof(float) * Qp * 4 * Qp);       // Y^T split, later R split
+        L.e[s] = take(sizeof(float) * Dp * Qp);            // F_0 Y, later (F_0 + xi*) R
+        L.xi[s] = take(sizeof(double) * d * q);            // xi*, later E_F
+        L.nq[s] = take(sizeof(float) * Qp * Qp);
+    }
+    L.ns_y = take(sizeof(double) * q * q);
+    L.ns_z = take(sizeof(double) * q * q);
+    L.ns_m = take(sizeof(double) * q * q);
+    L.ns_y4 = take(sizeof(float) * Qp * 4 * Qp);
+    L.ns_z4 = take(sizeof(float) * Qp * 4 * Qp);
+    L.ns_m4 = take(sizeof(float) * Qp * 4 * Qp);
+    L.ns_t1 = take(sizeof(float) * Qp * Qp);
+    L.ns_t2 = take(sizeof(float) * Qp * Qp);
+    L.ns_t3 = take(sizeof(float) * Qp * Qp);
+    L.a6 = take(sizeof(float) * L.Mp * 4 * 2 * Qp);
+    L.b6 = take(sizeof(float) * L.Np * 4 * 2 * Qp);
+    L.total = o;
+    return L;
+}
+
+int grid_of(long long work, int sms) {
+    const long long b = (work + 255) / 256;
+    return (int)std::max(1LL, std::min(b, (long long)sms * 8));
+}
+
+int gemm_smem_optin() {
+    static int done = 0;
+    if (done) return ISO_OK;
+    if (cudaFuncSetAttribute(k_gemm_tf32, cudaFuncAttributeMaxDynamicSharedMemorySize, GEMM_SMEM) != cudaSuccess)
+        return ISO_ERR_CUDA;
+    done = 1;
+    return ISO_OK;
+}
+
+// C (a_rows x b_rows) = A B^T over the three-product split: A and B are
+// four-segment operand arrays of segment length L (rows a_rows / b_rows,
+// multiples of 128).
+int frame_gemm(cudaStream_t s, const float* A, long long a_rows, const float* B, long long b_rows, long long L,
+               GemmArgs g) {
+    CUtensorMap ta, tb;
+    ISO_TRY(gemm_tensor_map(&ta, A, a_rows, 4 * L, 4 * L));
+    ISO_TRY(gemm_tensor_map(&tb, B, b_rows, 4 * L, 4 * L));
+    g.k_tiles = (int)(3 * L / GEMM_BK);
+    g.a_k0 = 0;
+    g.b_k0 = (int)L;
+    ISO_TRY(gemm_smem_optin());
+    const dim3 grid((unsigned)(b_rows / GEMM_BN), (unsigned)(a_rows / GEMM_BM));
+    const int slot = prof_begin(0, s);
+    k_gemm_tf32<<<grid, GEMM_THREADS, GEMM_SMEM, s>>>(ta, tb, g);
+    prof_end(slot, s);
+    return cudaGetLastError() == cudaSuccess ? ISO_OK : ISO_ERR_CUDA;
+}
+
+}  // namespace
+}  // namespace iso
+
+using namespace iso;
+
+extern "C" {
+
+int32_t iso_frame_workspace_size(int64_t m, int64_t n, int32_t K, size_t* bytes) {
+    if (!bytes || m < 1 || n < 1 || K < 1) return ISO_ERR_ARG;
+    if (K > ISO_MAX_EXPERTS) return ISO_ERR_UNSUPPORTED;
+    if (m >= (1LL << 24) || n >= (1LL << 24) || std::min(m, n) > 32768) return ISO_ERR_UNSUPPORTED;
+    *bytes = frame_layout(m, n, K).total;
+    return ISO_OK;
+}
+
+int32_t iso_frame_merge(const double* U0, const double* S0, const double* Vt0, const double* const* U,
+                        const double* const* Vt, int32_t K, int64_t m, int64_t n, const iso_tensor* W0,
+                        const iso_tensor* out, const iso_frame_cfg* cfg, void* workspace, size_t ws_bytes,
+                        const iso_merge_stats* stats, void* stream) {
+    size_t need = 0;
+    ISO_TRY(iso_frame_workspace_size(m, n, K, &need));
+    if (!U0 || !S0 || !Vt0 || !U || !Vt || !W0 || !out || !cfg) return ISO_ERR_ARG;
+    for (int i = 0; i < K; ++i)
+        if (!U[i] || !Vt[i]) return ISO_ERR_ARG;
+    auto al8 = [](const void* p) { return ((uintptr_t)p & 7u) == 0; };
+    if (!al8(U0) || !al8(S0) || !al8(Vt0)) return ISO_ERR_ALIGN;
+    for (int i = 0; i < K; ++i)
+        if (!al8(U[i]) || !al8(Vt[i])) return ISO_ERR_ALIGN;
+    if (!(cfg->rho_keep > 0.0 && cfg->rho_keep <= 1.0)) return ISO_ERR_ARG;
+    if (!(cfg->ridge >= 0.0) || !std::isfinite(cfg->ridge)) return ISO_ERR_ARG;
+    if (!std::isfinite(cfg->c_min) || !std::isfinite(cfg->c_max) || cfg->c_min > cfg->c_max) return ISO_ERR_ARG;
+    if (cfg->ns_iters < 0 || cfg->ns_iters > FR_MAX_NS || cfg->reserved != 0) return ISO_ERR_ARG;
+    if (W0->rows != m || W0->cols != n || out->rows != m || out->cols != n) return ISO_ERR_SHAPE;
+    if ((W0->dtype != ISO_BF16 && W0->dtype != ISO_F32) || out->dtype != W0->dtype) return ISO_ERR_DTYPE;
+    if (!W0->data || !out->data) return ISO_ERR_ARG;
+    if (((uintptr_t)W0->data & 15u) || ((uintptr_t)out->data & 15u)) return ISO_ERR_ALIGN;
+    if (!workspace || ((uintptr_t)workspace & 255u)) return ISO_ERR_WORKSPACE;
+    if (ws_bytes < need) return ISO_ERR_WORKSPACE;
+    // out may coincide with W0 (each entry is read and written by one thread);
+    // it may share no other byte with an input
+    {
+        const size_t es = W0->dtype == ISO_BF16 ? 2 : 4;
+        const uintptr_t o0 = (uintptr_t)out->data, o1 = o0 + (uintptr_t)(m * n) * es;
+        const uintptr_t w0 = (uintptr_t)W0->data;
+        if (o0 != w0 && o0 < w0 + (uintptr_t)(m * n) * es && w0 < o1) return ISO_ERR_ARG;
+    }
+    const FrameLayout L = frame_layout(m, n, K);
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    char* ws = static_cast<char*>(workspace);
+    int dev = 0, sms = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess ||
+        cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
+        return ISO_ERR_CUDA;
+    const long long q = L.q, Qp = L.Qp;
+    long long k_keep = (long long)std::floor(cfg->rho_keep * (double)q + 0.5);
+    k_keep = std::max(0LL, std::min(q, k_keep));
+    const int ns_iters = cfg->ns_iters ? cfg->ns_iters : FR_DEFAULT_NS;
+    FrameHeader* hdr = reinterpret_cast<FrameHeader*>(ws + L.hdr);
+    double* gram = reinterpret_cast<double*>(ws + L.gram);
+    double* coef = reinterpret_cast<double*>(ws + L.coef);
+    double* dots = reinterpret_cast<double*>(ws + L.dots);
+    auto F = [&](size_t off) { return reinterpret_cast<float*>(ws + off); };
+    auto D = [&](size_t off) { return reinterpret_cast<double*>(ws + off); };
+#define FR_LAUNCH(...) do { const int _slot = prof_begin(1, s); __VA_ARGS__; prof_end(_slot, s); \
+                                if (cudaGetLastError() != cudaSuccess) return ISO_ERR_CUDA; } while (0)
+
+    // header, Gamma, c*, the sign dots and the column dots start at zero
+    if (cudaMemsetAsync(ws, 0, L.cd[1] + sizeof(double) * K * K * q, s) != cudaSuccess) return ISO_ERR_CUDA;
+
+    // the V side as n x q row-major frames
+    Frames fr[2];
+    fr[0].F0 = U0; fr[0].K = K; fr[0].d = m; fr[0].q = q;
+    fr[1].F0 = D(L.vcopy); fr[1].K = K; fr[1].d = n; fr[1].q = q;
+    for (int i = 0; i < MAXK; ++i) {
+        fr[0].F[i] = i < K ? U[i] : nullptr;
+        fr[1].F[i] = i < K ? D(L.vcopy) + (size_t)(i + 1) * n * q : nullptr;
+    }
+    {
+        const dim3 blk(32, 8), grd((unsigned)((n + 31) / 32), (unsigned)((q + 31) / 32));
+        FR_LAUNCH((k_fr_transpose<<<grd, blk, 0, s>>>(Vt0, D(L.vcopy), q, n)));
+        for (int i = 0; i < K; ++i)
+            FR_LAUNCH((k_fr_transpose<<<grd, blk, 0, s>>>(Vt[i], D(L.vcopy) + (size_t)(i + 1) * n * q, q, n)));
+    }
+    // signs (from the U frames), then the column dot products of each side
+    {
+        const int rc = (int)std::max(1LL, std::min(64LL, ((long long)m + 511) / 512));
+        FR_LAUNCH((k_fr_signdots<<<dim3((unsigned)((q + 31) / 32), K, rc), dim3(32, 8), 0, s>>>(fr[0], dots, rc)));
+        for (int sd = 0; sd < 2; ++sd) {
+            const int r2 = (int)std::max(1LL, std::min(256LL, (fr[sd].d + 255) / 256));
+            FR_LAUNCH((k_fr_coldots<<<dim3((unsigned)((q + 31) / 32), r2), dim3(32, 8), 0, s>>>(
+                fr[sd], dots, D(L.cd[sd]), r2)));
+        }
+    }
+    // A_i = F_0^T dF_i on the tensor cores, then Sym_i and Kw_i
+    for (int sd = 0; sd < 2; ++sd) {
+        const long long Dp = sd == 0 ? L.Mp : L.Np;
+        SplitT st{};
+        st.f = fr[sd]; st.dots = dots; st.X = nullptr; st.Dp = Dp; st.Qp = Qp;
+        const dim3 blk(32, 8), grd((unsigned)(Dp / 32), (unsigned)(Qp / 32));
+        st.mode = 0; st.i = 0; st.out = F(L.ft4[sd]);
+        FR_LAUNCH((k_fr_split_t<<<grd, blk, 0, s>>>(st)));
+        for (int i = 0; i < K; ++i) {
+            st.mode = 1; st.i = i; st.out = F(L.dft4[sd]);
+            FR_LAUNCH((k_fr_split_t<<<grd, blk, 0, s>>>(st)));
+            GemmArgs g{};
+            g.mode = GEMM_STORE_F32; g.C = F(L.aq[sd]) + (size_t)i * Qp * Qp; g.ldc = Qp; g.M = (int)Qp; g.N = (int)Qp;
+            g.status = &hdr->status;
+            ISO_TRY(frame_gemm(s, F(L.ft4[sd]), Qp, F(L.dft4[sd]), Qp, Dp, g));
+        }
+        FR_LAUNCH((k_fr_symskew<<<dim3((unsigned)(Qp / 32), (unsigned)(Qp / 32), K), dim3(32, 8), 0, s>>>(
+            F(L.aq[sd]), Qp, q, D(L.sym[sd]), D(L.kw[sd]))));
+    }
+    // Gamma and c*
+    {
+        GramArgs ga{};
+        for (int sd = 0; sd < 2; ++sd) {
+            ga.A[sd] = F(L.aq[sd]); ga.sym[sd] = D(L.sym[sd]); ga.kw[sd] = D(L.kw[sd]); ga.cd[sd] = D(L.cd[sd]);
+        }
+        ga.S0 = S0; ga.gram = gram; ga.q = q; ga.Qp = Qp; ga.k_keep = k_keep; ga.K = K;
+        const int pairs = K * (K + 1) / 2;
+        const int slices = (int)std::max(1LL, std::min((long long)sms * 4, (q * q + 4095) / 4096));
+        FR_LAUNCH((k_fr_gram<<<dim3(pairs, slices), 256, 0, s>>>(ga)));
+        FR_LAUNCH((k_fr_solve<<<1, 32, 0, s>>>(gram, coef, K, cfg->ridge, cfg->c_min, cfg->c_max,
+                                                stats ? stats->gram : nullptr, stats ? stats->coef : nullptr)));
+    }
+    // per side: aggregate tangent, polar factor, motion E_F
+    for (int sd = 0; sd < 2; ++sd) {
+        const long long Dp = sd == 0 ? L.Mp : L.Np, d = fr[sd].d;
+        SplitR sr{};
+        sr.f = fr[sd]; sr.S0 = S0; sr.sym = D(L.sym[sd]); sr.kw = D(L.kw[sd]); sr.coef = coef; sr.hdr = hdr;
+        sr.side = sd; sr.k_keep = k_keep;
+        // Y^T, F_0, then E = F_0 Y
+        sr.mode = 3; sr.out = F(L.y4[sd]); sr.rows = q; sr.rows_p = Qp; sr.Lp = Qp;
+        FR_LAUNCH((k_fr_split_r<<<grid_of(Qp * Qp, sms), 256, 0, s>>>(sr)));
+        sr.mode = 0; sr.out = F(L.fr4[sd]); sr.rows = d; sr.rows_p = Dp; sr.Lp = Qp;
+        FR_LAUNCH((k_fr_split_r<<<grid_of(Dp * Qp, sms), 256, 0, s>>>(sr)));
+        {
+            GemmArgs g{};
+            g.mode = GEMM_STORE_F32; g.C = F(L.e[sd]); g.ldc = Qp; g.M = (int)Dp; g.N = (int)Qp; g.status = &hdr->status;
+            ISO_TRY(frame_gemm(s, F(L.fr4[sd]), Dp, F(L.y4[sd]), Qp, Qp, g));
+        }
+        FR_LAUNCH((k_fr_xi<<<grid_of(d * q, sms), 256, 0, s>>>(fr[sd], dots, coef, F(L.e[sd]), Qp, k_keep, D(L.xi[sd]))));
+        // N = xi*^T xi*
+        {
+            SplitT st{};
+            st.f = fr[sd]; st.dots = dots; st.X = D(L.xi[sd]); st.mode = 2; st.out = F(L.ft4[sd]); st.Dp = Dp; st.Qp = Qp;
+            FR_LAUNCH((k_fr_split_t<<<dim3((unsigned)(Dp / 32), (unsigned)(Qp / 32)), dim3(32, 8), 0, s>>>(st)));
+            GemmArgs g{};
+            g.mode = GEMM_STORE_F32; g.C = F(L.nq[sd]); g.ldc = Qp; g.M = (int)Qp; g.N = (int)Qp; g.status = &hdr->status;
+            ISO_TRY(frame_gemm(s, F(L.ft4[sd]), Qp, F(L.ft4[sd]), Qp, Dp, g));
+        }
+        // (I + N)^(-1/2) = I + R by the difference-form Newton-Schulz iteration
+        FR_LAUNCH((k_fr_norm<<<grid_of(q * q, sms), 256, 0, s>>>(F(L.nq[sd]), Qp, q, hdr, sd)));
+        FR_LAUNCH((k_fr_ns_init<<<grid_of(q * q, sms), 256, 0, s>>>(F(L.nq[sd]), Qp, q, hdr, sd, D(L.ns_y), D(L.ns_z))));
+        SplitR sq{};
+        sq.f = fr[sd]; sq.hdr = hdr; sq.side = sd; sq.mode = 2; sq.rows = q; sq.rows_p = Qp; sq.Lp = Qp;
+        auto split_q = [&](const double* M_, size_t out_off) -> int {
+            sq.M = M_; sq.out = F(out_off);
+            FR_LAUNCH((k_fr_split_r<<<grid_of(Qp * Qp, sms), 256, 0, s>>>(sq)));
+            return ISO_OK;
+        };
+        ISO_TRY(split_q(D(L.ns_y), L.ns_y4));
+        ISO_TRY(split_q(D(L.ns_z), L.ns_z4));
+        for (int it = 0; it < ns_iters; ++it) {
+            GemmArgs g{};
+            g.mode = GEMM_STORE_F32; g.ldc = Qp; g.M = (int)Qp; g.N = (int)Qp; g.status = &hdr->status;
+            g.skip = &hdr->conv[sd];
+            g.C = F(L.ns_t1);
+            ISO_TRY(frame_gemm(s, F(L.ns_z4), Qp, F(L.ns_y4), Qp, Qp, g));     // z y
+            FR_LAUNCH((k_fr_ns_m<<<grid_of(q * q, sms), 256, 0, s>>>(D(L.ns_y), D(L.ns_z), F(L.ns_t1), Qp, q,
+                                                                      D(L.ns_m), hdr, sd, it)));
+            sq.M = D(L.ns_m); sq.out = F(L.ns_m4);
+            FR_LAUNCH((k_fr_split_r<<<grid_of(Qp * Qp, sms), 256, 0, s>>>(sq)));
+            g.C = F(L.ns_t2);
+            ISO_TRY(frame_gemm(s, F(L.ns_y4), Qp, F(L.ns_m4), Qp, Qp, g));     // y m
+            g.C = F(L.ns_t3);
+            ISO_TRY(frame_gemm(s, F(L.ns_m4), Qp, F(L.ns_z4), Qp, Qp, g));     // m z
+            FR_LAUNCH((k_fr_ns_update<<<grid_of(q * q, sms), 256, 0, s>>>(D(L.ns_y), D(L.ns_z), D(L.ns_m), F(L.ns_t2),
+                                                                           F(L.ns_t3), Qp, q, hdr, sd, it)));
+            ISO_TRY(split_q(D(L.ns_y), L.ns_y4));
+            ISO_TRY(split_q(D(L.ns_z), L.ns_z4));
+        }
+        // R, F_0 + xi*, then E_F = xi* + (F_0 + xi*) R
+        sr.mode = 6; sr.M = D(L.ns_z); sr.out = F(L.y4[sd]); sr.rows = q; sr.rows_p = Qp; sr.Lp = Qp;
+        FR_LAUNCH((k_fr_split_r<<<grid_of(Qp * Qp, sms), 256, 0, s>>>(sr)));
+        sr.mode = 1; sr.X = D(L.xi[sd]); sr.out = F(L.fr4[sd]); sr.rows = d; sr.rows_p = Dp; sr.Lp = Qp;
+        FR_LAUNCH((k_fr_split_r<<<grid_of(Dp * Qp, sms), 256, 0, s>>>(sr)));
+        {
+            GemmArgs g{};
+            g.mode = GEMM_STORE_F32; g.C = F(L.e[sd]); g.ldc = Qp; g.M = (int)Dp; g.N = (int)Qp; g.status = &hdr->status;
+            ISO_TRY(frame_gemm(s, F(L.fr4[sd]), Dp, F(L.y4[sd]), Qp, Qp, g));
+        }
+        FR_LAUNCH((k_fr_motion<<<grid_of(d * q, sms), 256, 0, s>>>(D(L.xi[sd]), F(L.e[sd]), Qp, d, q)));
+        // the reconstruction's operand of this side
+        sr.X = D(L.xi[sd]);
+        sr.mode = sd == 0 ? 4 : 5;
+        sr.out = F(sd == 0 ? L.a6 : L.b6);
+        sr.rows = d; sr.rows_p = Dp; sr.Lp = 2 * Qp;
+        FR_LAUNCH((k_fr_split_r<<<grid_of(Dp * 2 * Qp, sms), 256, 0, s>>>(sr)));
+    }
+    // W* = W_0 + [E_U S_0 | U_0 S_0] [V* | E_V]^T
+    {
+        GemmArgs g{};
+        g.mode = GEMM_ADD_BASE; g.M = (int)m; g.N = (int)n; g.out = out->data; g.w0 = W0->data; g.ldo = n;
+        g.out_dtype = W0->dtype; g.status = &hdr->status;
+        ISO_TRY(frame_gemm(s, F(L.a6), L.Mp, F(L.b6), L.Np, 2 * Qp, g));
+    }
+    if (stats && stats->status) FR_LAUNCH((k_fr_status<<<1, 32, 0, s>>>(hdr, stats->status)));
+#undef FR_LAUNCH
+    return ISO_OK;
+}
+
+// The tcgen05 product on its own, for tests of the contraction: C (M x N,
+// ldc) = A[:, a_k0 : a_k0 + Kc] B[:, b_k0 : b_k0 + Kc]^T with A (M x lda) and
+// B (N x ldb) row-major binary32 read as tf32.
+int32_t iso_gemm_tf32(const float* A, int64_t lda, const float* B, int64_t ldb, float* C, int64_t ldc, int64_t M,
+                      int64_t N, int64_t Kc, int64_t a_k0, int64_t b_k0, void* stream) {
+    if (!A || !B || !C) return ISO_ERR_ARG;
+    if (M <= 0 || N <= 0 || Kc <= 0 || a_k0 < 0 || b_k0 < 0) return ISO_ERR_ARG;
+    if (M % GEMM_BM || N % GEMM_BN || Kc % GEMM_BK || a_k0 % GEMM_BK || b_k0 % GEMM_BK) return ISO_ERR_SHAPE;
+    if (a_k0 + Kc > lda || b_k0 + Kc > ldb || ldc < N || lda % 4 || ldb % 4 || ldc % 4) return ISO_ERR_SHAPE;
+    if (M >= (1LL << 31) || N >= (1LL << 31) || lda >= (1LL << 31) || ldb >= (1LL << 31)) return ISO_ERR_UNSUPPORTED;
+    if (((uintptr_t)A & 15u) || ((uintptr_t)B & 15u) || ((uintptr_t)C & 15u)) return ISO_ERR_ALIGN;
+    CUtensorMap ta, tb;
+    ISO_TRY(gemm_tensor_map(&ta, A, M, lda, lda));
+    ISO_TRY(gemm_tensor_map(&tb, B, N, ldb, ldb));
+    ISO_TRY(gemm_smem_optin());
+    GemmArgs g{};
+    g.mode = GEMM_STORE_F32; g.C = C; g.ldc = ldc; g.M = (int)M; g.N = (int)N;
+    g.k_tiles = (int)(Kc / GEMM_BK); g.a_k0 = (int)a_k0; g.b_k0 = (int)b_k0;
+    const int slot = prof_begin(0, static_cast<cudaStream_t>(stream));
+    k_gemm_tf32<<<dim3((unsigned)(N / GEMM_BN), (unsigned)(M / GEMM_BM)), GEMM_THREADS, GEMM_SMEM,
+                  static_cast<cudaStream_t>(stream)>>>(ta, tb, g);
+    prof_end(slot, static_cast<cudaStream_t>(stream));
+    return cudaGetLastError() == cudaSuccess ? ISO_OK : ISO_ERR_CUDA;
+}
+
+}  // extern "C"

@@ -623,12 +623,15 @@ __device__ __forceinline__ void mbar_arrive_tx(uint32_t bar, uint32_t bytes) {
 __device__ __forceinline__ void mbar_arrive(uint32_t bar) {
     asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" :: "r"(bar) : "memory");
 }
-// true once the phase with the given parity has completed (one bounded probe)
+// true once the phase with the given parity has completed; one probe, which
+// may suspend the thread for at most MBAR_PROBE_NS nanoseconds (the thread is
+// resumed early when the phase completes)
+constexpr uint32_t MBAR_PROBE_NS = 1000;
 __device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
     uint32_t ok;
-    asm volatile("{\n\t.reg .pred p;\n\tmbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+    asm volatile("{\n\t.reg .pred p;\n\tmbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3;\n\t"
                  "selp.u32 %0, 1, 0, p;\n\t}"
-                 : "=r"(ok) : "r"(bar), "r"(parity) : "memory");
+                 : "=r"(ok) : "r"(bar), "r"(parity), "n"(MBAR_PROBE_NS) : "memory");
     return ok != 0;
 }
 // bytes (a multiple of 16) from global memory of this GPU to shared memory,
@@ -642,9 +645,53 @@ __device__ __forceinline__ void bulk_g2s(uint32_t dst, const void* src, uint32_t
 __device__ __forceinline__ void fence_proxy_async_smem() {
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
 }
-// probes of one barrier phase before a wait gives up (each probe blocks for
-// up to a hardware time limit; well over a second in all)
+// probes of one barrier phase before a wait gives up: at most about four
+// seconds of suspension in all
 constexpr int MBAR_SPIN_LIMIT = 1 << 22;
+
+// Retention coefficients (Sec. 4.2; App. E, Retention coefficients): on the
+// experts with Gamma_ii > 0, (Gamma + ridge I) c = diag(Gamma) by Gaussian
+// elimination with partial pivoting in binary64, clipped to [c_min, c_max];
+// an expert with Gamma_ii = 0 gets c = 0.  G is K x K row-major (K <= MAXK).
+__device__ __forceinline__ void retention_solve(const double* G, int K, double ridge, double c_min,
+                                                double c_max, double* c) {
+    for (int i = 0; i < K; ++i) c[i] = 0.0;
+    int idx[MAXK];
+    int m = 0;
+    for (int i = 0; i < K; ++i)
+        if (G[i * K + i] > 0.0) idx[m++] = i;
+    double A[MAXK * MAXK], rhs[MAXK], x[MAXK];
+    for (int r = 0; r < m; ++r) {
+        for (int q = 0; q < m; ++q) A[r * m + q] = G[idx[r] * K + idx[q]];
+        A[r * m + r] = __dadd_rn(A[r * m + r], ridge);
+        rhs[r] = G[idx[r] * K + idx[r]];
+    }
+    for (int col = 0; col < m; ++col) {
+        int piv = col;
+        for (int r = col + 1; r < m; ++r)
+            if (fabs(A[r * m + col]) > fabs(A[piv * m + col])) piv = r;
+        if (piv != col) {
+            for (int q = 0; q < m; ++q) { double s = A[col * m + q]; A[col * m + q] = A[piv * m + q]; A[piv * m + q] = s; }
+            double s = rhs[col]; rhs[col] = rhs[piv]; rhs[piv] = s;
+        }
+        for (int r = col + 1; r < m; ++r) {
+            const double f = A[r * m + col] / A[col * m + col];
+            for (int q = col; q < m; ++q) A[r * m + q] = __dadd_rn(A[r * m + q], -__dmul_rn(f, A[col * m + q]));
+            rhs[r] = __dadd_rn(rhs[r], -__dmul_rn(f, rhs[col]));
+        }
+    }
+    for (int r = m - 1; r >= 0; --r) {
+        double s = rhs[r];
+        for (int q = r + 1; q < m; ++q) s = __dadd_rn(s, -__dmul_rn(A[r * m + q], x[q]));
+        x[r] = s / A[r * m + r];
+    }
+    for (int r = 0; r < m; ++r) {
+        double v = x[r];
+        if (v < c_min) v = c_min;
+        if (v > c_max) v = c_max;
+        c[idx[r]] = v;
+    }
+}
 
 __device__ __forceinline__ float out_of(float th0, float tau, float a) {
     const float upd = __fmul_rn(a, tau);

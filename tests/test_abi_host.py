@@ -23,7 +23,7 @@ def _built():
 def _declared():
     src = open(os.path.join(ROOT, "include", "iso.h")).read()
     src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
-    return sorted(set(re.findall(r"\b(iso_[a-z_]+)\s*\(", src)))
+    return sorted(set(re.findall(r"\b(iso_[a-z_0-9]+)\s*\(", src)))
 
 
 def test_every_declared_symbol_is_exported():
@@ -213,3 +213,51 @@ def test_workspace_at_full_model_sizes():
     cfg = iso.merge_cfg("ties", 0.1)
     big = _arr(_fake(1 << 16, 1 << 16))
     assert L.iso_workspace_size(big, 1, 1, ctypes.byref(cfg), None, None) == _abi.ISO_ERR_UNSUPPORTED
+
+
+def test_frame_merge_sizes_and_argument_errors():
+    # iso_frame_merge: sizing and the checks made before anything is enqueued
+    # (descriptors and fake device pointers only; nothing is launched)
+    L = _abi.lib()
+    b = ctypes.c_size_t()
+    assert L.iso_frame_workspace_size(3584, 18944, 8, ctypes.byref(b)) == 0
+    assert 10e9 < b.value < 40e9           # the 7B gate/up projection fits the device several times
+    small = ctypes.c_size_t()
+    assert L.iso_frame_workspace_size(96, 64, 3, ctypes.byref(small)) == 0
+    assert 0 < small.value < b.value
+    assert L.iso_frame_workspace_size(96, 64, 9, ctypes.byref(small)) == _abi.ISO_ERR_UNSUPPORTED
+    assert L.iso_frame_workspace_size(0, 64, 1, ctypes.byref(small)) == _abi.ISO_ERR_ARG
+    cfg = _abi.IsoFrameCfg(0.9, 1e-12, 0.0, 1.5, 0, 0)
+    P = ctypes.c_void_p
+    U = (P * 2)(0x100000, 0x200000)
+    V = (P * 2)(0x300000, 0x400000)
+    W = _arr(_fake(96, 64, dtype=_abi.ISO_F32, ptr=0x1000000))
+    O = _arr(_fake(96, 64, dtype=_abi.ISO_F32, ptr=0x2000000))
+    ws = P(0x4000000)
+
+    def fm(W_=W, O_=O, cfg_=cfg, ws_=ws, wsb=1 << 30, m=96, n=64, K=2, U_=U):
+        return L.iso_frame_merge(P(0x10000), P(0x20000), P(0x30000), U_, V, K, m, n, W_, O_,
+                                 ctypes.byref(cfg_) if cfg_ is not None else None, ws_, wsb, None, None)
+    assert fm(W_=_arr(_fake(96, 65, dtype=_abi.ISO_F32, ptr=0x1000000))) == _abi.ISO_ERR_SHAPE
+    assert fm(O_=_arr(_fake(96, 64, dtype=_abi.ISO_BF16, ptr=0x2000000))) == _abi.ISO_ERR_DTYPE
+    assert fm(O_=_arr(_fake(96, 64, dtype=_abi.ISO_F32, ptr=0x1000040))) == _abi.ISO_ERR_ARG   # overlaps W0
+    assert fm(cfg_=None) == _abi.ISO_ERR_ARG
+    assert fm(cfg_=_abi.IsoFrameCfg(0.0, 1e-12, 0.0, 1.5, 0, 0)) == _abi.ISO_ERR_ARG           # rho_keep
+    assert fm(cfg_=_abi.IsoFrameCfg(0.9, 1e-12, 2.0, 1.5, 0, 0)) == _abi.ISO_ERR_ARG           # clip range
+    assert fm(cfg_=_abi.IsoFrameCfg(0.9, 1e-12, 0.0, 1.5, 65, 0)) == _abi.ISO_ERR_ARG          # iterations
+    assert fm(ws_=P(0x4000010)) == _abi.ISO_ERR_WORKSPACE                                       # misaligned
+    assert fm(wsb=1024) == _abi.ISO_ERR_WORKSPACE
+    assert fm(U_=(P * 2)(0x100000, 0)) == _abi.ISO_ERR_ARG
+    assert fm(U_=(P * 2)(0x100000, 0x200004)) == _abi.ISO_ERR_ALIGN
+    assert fm(K=9) == _abi.ISO_ERR_UNSUPPORTED
+
+
+def test_gemm_argument_errors():
+    L = _abi.lib()
+    P = ctypes.c_void_p
+    A, B, C = P(0x100000), P(0x200000), P(0x300000)
+    assert L.iso_gemm_tf32(A, 32, B, 32, C, 128, 100, 128, 32, 0, 0, None) == _abi.ISO_ERR_SHAPE   # M
+    assert L.iso_gemm_tf32(A, 32, B, 32, C, 128, 128, 128, 40, 0, 0, None) == _abi.ISO_ERR_SHAPE   # Kc
+    assert L.iso_gemm_tf32(A, 32, B, 32, C, 128, 128, 128, 32, 32, 0, None) == _abi.ISO_ERR_SHAPE  # past lda
+    assert L.iso_gemm_tf32(P(0x100004), 32, B, 32, C, 128, 128, 128, 32, 0, 0, None) == _abi.ISO_ERR_ALIGN
+    assert L.iso_gemm_tf32(None, 32, B, 32, C, 128, 128, 128, 32, 0, 0, None) == _abi.ISO_ERR_ARG

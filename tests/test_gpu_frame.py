@@ -1,0 +1,185 @@
+"""GPU parity of the frame-space ISO-Merger (App. E) and of its tensor-core
+product, through the C ABI.
+
+* iso_gemm_tf32 (tcgen05.mma, operands staged by TMA, accumulator in tensor
+  memory): on operands whose products and sums are exact in binary32 (small
+  multiples of 1/8) the result must equal the binary64 product bit for bit,
+  over several output tiles, a ring of stages that wraps many times and
+  contraction offsets.
+* iso_frame_merge against oracle/iso_merger.py on tall, wide and square
+  matrices, K = 1 ... 8 experts, rho_keep 0.5 / 0.9 / 1, binary32 and
+  bfloat16 weights.  The GPU is given the oracle's own thin-SVD factors, so
+  the comparison isolates the merge.  Tolerances (derived in the module's
+  DESIGN section and from the three-product tf32 scheme, about 2^-21 per
+  product, binary32 accumulation): Gamma within 1e-4 of max |Gamma|; c* within
+  1e-4 (absolute, the coefficients are O(1)); binary32 W* within 1e-4 of the
+  largest entry of W* - W_0 plus 2^-22 |W*|; bfloat16 W* within one ulp of
+  the oracle's value.  The spectrum of W* equals the base's (the paper's
+  fixed-spectrum property) and experts equal to the base leave W_0 bit for
+  bit.
+"""
+import numpy as np
+import pytest
+import torch
+
+import paper_2607_19331_gb300 as iso
+from oracle import iso_merger as M
+from paper_2607_19331_gb300 import _abi
+from parity_util import bf16_ulp
+
+pytestmark = pytest.mark.gpu
+DEV = "cuda:0"
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _cuda():
+    assert torch.cuda.is_available(), "GPU tests need CUDA"
+    torch.cuda.set_device(0)
+    _abi.lib()
+
+
+# ---------------------------------------------------------------------------
+# the tensor-core product
+# ---------------------------------------------------------------------------
+@pytest.mark.parametrize("M_,N_,Kc,a_k0,b_k0,lda,ldb", [
+    (128, 128, 32, 0, 0, 32, 32),            # one tile, one stage
+    (256, 384, 1024, 0, 64, 1024, 1088),     # 6 tiles, the six-stage ring wraps five times
+    (384, 128, 224, 32, 0, 256, 224),        # offsets, a contraction of seven stages
+    (128, 256, 3072, 1024, 0, 4096, 3072),   # the split layout's segment offsets
+])
+def test_gemm_tf32_exact(M_, N_, Kc, a_k0, b_k0, lda, ldb):
+    g = torch.Generator().manual_seed(M_ * 7 + Kc)
+    A = (torch.randint(-8, 9, (M_, lda), generator=g).float() / 8).to(DEV)
+    B = (torch.randint(-8, 9, (N_, ldb), generator=g).float() / 8).to(DEV)
+    C = torch.full((M_, N_), float("nan"), device=DEV)
+    iso.gemm_tf32(A, B, C, Kc, a_k0, b_k0)
+    torch.cuda.synchronize()
+    ref = A[:, a_k0:a_k0 + Kc].double() @ B[:, b_k0:b_k0 + Kc].double().T
+    assert torch.equal(C.double(), ref), float((C.double() - ref).abs().max())
+
+
+def test_gemm_tf32_rounding_of_general_operands():
+    # general binary32 operands are read as tf32 (10 mantissa bits): the error
+    # stays within the tf32 bound of the product's magnitude
+    g = torch.Generator().manual_seed(5)
+    A = torch.randn(256, 512, generator=g).to(DEV)
+    B = torch.randn(128, 512, generator=g).to(DEV)
+    C = torch.empty(256, 128, device=DEV)
+    iso.gemm_tf32(A, B, C, 512)
+    torch.cuda.synchronize()
+    ref = A.double() @ B.double().T
+    mag = A.double().abs() @ B.double().abs().T
+    assert ((C.double() - ref).abs() <= 2.0 ** -10 * mag).all()
+
+
+# ---------------------------------------------------------------------------
+# the frame-space merge
+# ---------------------------------------------------------------------------
+def _orth(rng, m, q):
+    Q, R = np.linalg.qr(rng.normal(size=(m, q)))
+    return Q * np.sign(np.diag(R))
+
+
+def _case(seed, m, n, K, dtype=np.float32, motion=0.05):
+    """A base with a well-separated spectrum and K experts moved by `motion`
+    (relative), stored in `dtype` (the oracle sees the stored values)."""
+    rng = np.random.default_rng(seed)
+    q = min(m, n)
+    U, V = _orth(rng, m, q), _orth(rng, n, q)
+    S = np.linspace(2.0, 0.2, q) * 0.05
+    W0 = (U * S) @ V.T
+    ex = [W0 + motion * 0.05 * rng.normal(size=(m, n)) / np.sqrt(max(m, n)) for _ in range(K)]
+    if dtype == "bf16":
+        cast = lambda a: torch.from_numpy(a).to(torch.bfloat16)
+    else:
+        cast = lambda a: torch.from_numpy(a.astype(np.float32))
+    W0_t, ex_t = cast(W0), [cast(e) for e in ex]
+    return W0_t, ex_t, W0_t.double().numpy(), [e.double().numpy() for e in ex_t]
+
+
+def _factors_on_gpu(W):
+    U, S, V = M.thin_svd(W)
+    to = lambda a: torch.from_numpy(np.ascontiguousarray(a)).to(DEV)
+    return to(U), to(S), to(V.T)
+
+
+def _run(W0_t, W0, experts, **kw):
+    U0, S0, Vt0 = _factors_on_gpu(W0)
+    Us, Vts = [], []
+    for E in experts:
+        U, _, Vt = _factors_on_gpu(E)
+        Us.append(U)
+        Vts.append(Vt)
+    out, st = iso.frame_merge_factors(U0, S0, Vt0, Us, Vts, W0_t.to(DEV), stats=True, **kw)
+    torch.cuda.synchronize()
+    assert int(st.status.item()) == 0
+    return out.cpu(), st
+
+
+def _check(out, st, r, W0, what):
+    K = r["coef"].size
+    gram = st.gram.cpu().numpy()
+    coef = st.coef.cpu().numpy()
+    gmax = np.abs(r["gram"]).max()
+    assert np.abs(gram - r["gram"]).max() <= 1e-4 * gmax + 1e-300, (what, gram, r["gram"])
+    assert np.abs(coef - r["coef"]).max() <= 1e-4, (what, coef, r["coef"])
+    want = r["W"]
+    if out.dtype == torch.bfloat16:
+        got = out.float().double().numpy()
+        ulp = bf16_ulp(np.maximum(np.abs(got), np.abs(want)))
+        assert (np.abs(got - want) <= ulp).all(), what
+    else:
+        got = out.double().numpy()
+        scale = np.abs(want - W0).max()
+        tol = 1e-4 * scale + 2.0 ** -22 * np.abs(want)
+        err = np.abs(got - want)
+        assert (err <= tol).all(), (what, float(err.max()), float(scale))
+    return K
+
+
+@pytest.mark.parametrize("m,n,K,rho", [
+    (96, 64, 3, 0.9),       # tall, one tile
+    (64, 160, 2, 0.9),      # wide
+    (80, 80, 4, 0.9),       # square
+    (300, 200, 1, 0.9),     # one expert, ragged padding
+    (200, 520, 8, 0.9),     # eight experts, wide, several tiles along n
+    (384, 256, 2, 0.5),     # half the modes masked, several tiles along q
+    (160, 144, 3, 1.0),     # no mode masked
+])
+def test_frame_merge_matches_oracle(m, n, K, rho):
+    W0_t, ex_t, W0, ex = _case(m * 1000 + n + K, m, n, K)
+    r = M.merge_matrix(W0, ex, rho_keep=rho)
+    out, st = _run(W0_t, W0, ex, rho_keep=rho)
+    _check(out, st, r, W0, f"{m}x{n} K={K} rho={rho}")
+    # the fixed-spectrum property: W* keeps the base's singular values
+    s0 = np.linalg.svd(W0, compute_uv=False)
+    s1 = np.linalg.svd(out.double().numpy(), compute_uv=False)
+    assert np.abs(s1 - s0).max() <= 1e-5 * s0.max()
+
+
+def test_frame_merge_bf16_weights():
+    W0_t, ex_t, W0, ex = _case(11, 192, 320, 3, dtype="bf16")
+    r = M.merge_matrix(W0, ex)
+    out, st = _run(W0_t, W0, ex)
+    assert out.dtype == torch.bfloat16
+    _check(out, st, r, W0, "bf16 192x320")
+
+
+def test_frame_merge_experts_equal_to_base_is_a_fixed_point():
+    W0_t, _, W0, _ = _case(12, 130, 90, 1)
+    out, st = _run(W0_t, W0, [W0, W0])
+    assert torch.equal(out, W0_t)
+    assert (st.coef.cpu().numpy() == 0).all()
+
+
+def test_frame_merge_in_place_and_through_gpu_svds():
+    # the GPU's own thin SVDs (torch.linalg in binary64) instead of the oracle's
+    # factors: the singular vectors differ by rounding and by sign, which the
+    # sign gauge absorbs; and out may coincide with W0
+    W0_t, ex_t, W0, ex = _case(13, 144, 208, 2)
+    r = M.merge_matrix(W0, ex)
+    W = W0_t.to(DEV)
+    out, st = iso.frame_merge(W, [e.to(DEV) for e in ex_t], out=W, stats=True)
+    torch.cuda.synchronize()
+    assert out.data_ptr() == W.data_ptr()
+    _check(out.cpu(), st, r, W0, "torch SVDs, in place")
