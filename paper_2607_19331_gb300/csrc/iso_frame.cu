@@ -227,8 +227,10 @@ struct SplitR {
     int mode;
     float* out;
     long long rows, rows_p, Lp;
+    const int32_t* skip;   // optional: nothing to do while *skip != 0
 };
 __global__ void __launch_bounds__(256) k_fr_split_r(SplitR a) {
+    if (a.skip && *reinterpret_cast<const volatile int32_t*>(a.skip)) return;
     const long long total = a.rows_p * a.Lp;
     const long long q = a.f.q;
     for (long long e = (long long)blockIdx.x * blockDim.x + threadIdx.x; e < total; e += (long long)gridDim.x * blockDim.x) {
@@ -391,51 +393,145 @@ __global__ void __launch_bounds__(256) k_fr_norm(const float* N, long long Qp, l
     if (threadIdx.x == 0) atomicAdd(&h->nu2[side], acc);
 }
 
-// Newton-Schulz start: Y_0 = (I + N) / cs = I + y, Z_0 = I (z = 0)
-__global__ void __launch_bounds__(256) k_fr_ns_init(const float* N, long long Qp, long long q, FrameHeader* h,
-                                                    int side, double* y, double* z) {
-    const double nu = sqrt(h->nu2[side]);
+// The Newton-Schulz iterates y, z and the step m are symmetric in exact
+// arithmetic (functions of N); the products treat them so (B = M^T = M).  Each
+// kernel below symmetrises what it writes, one 32 x 32 tile and its mirror
+// per block (blocks below the diagonal return), so that rounding cannot
+// build an asymmetric component from one iteration to the next.  Reading
+// both tiles before writing either makes the update safe in place.
+struct NsArgs {
+    const float* N;     // init: N = xi^T xi (ld Qp)
+    const float* T1;    // m: z y;  update: y m
+    const float* T2;    // update: m z
+    double* y;
+    double* z;
+    double* m;
+    FrameHeader* h;
+    long long q, Qp;
+    int side, it;
+};
+
+__device__ __forceinline__ bool ns_tile(long long q, long long& r0, long long& c0) {
+    if (blockIdx.x < blockIdx.y) return false;
+    r0 = (long long)blockIdx.y * 32;
+    c0 = (long long)blockIdx.x * 32;
+    return true;
+}
+
+// Y_0 = (I + N) / cs = I + y, Z_0 = I (z = 0); cs = 1 while ||N||_F < 0.9,
+// else 1 + ||N||_F / 2, so that the eigenvalues of Y_0 lie in (0, 2)
+__global__ void __launch_bounds__(256) k_fr_ns_init(NsArgs a) {
+    __shared__ double ta[32][33], tb[32][33];
+    long long r0, c0;
+    if (!ns_tile(a.q, r0, c0)) return;
+    const double nu = sqrt(a.h->nu2[a.side]);
     const double cs = nu < 0.9 ? 1.0 : 1.0 + 0.5 * nu;
-    if (blockIdx.x == 0 && threadIdx.x == 0) {
-        h->cs[side] = cs;
-        h->conv[side] = 0;
+    if (blockIdx.x == 0 && blockIdx.y == 0 && threadIdx.x == 0 && threadIdx.y == 0) {
+        a.h->cs[a.side] = cs;
+        a.h->conv[a.side] = 0;
     }
-    for (long long e = (long long)blockIdx.x * blockDim.x + threadIdx.x; e < q * q; e += (long long)gridDim.x * blockDim.x) {
-        const long long r = e / q, c = e - r * q;
+    auto f = [&](long long r, long long c) -> double {
+        if (r >= a.q || c >= a.q) return 0.0;
         const double id = r == c ? 1.0 : 0.0;
-        y[e] = (id + (double)N[r * Qp + c]) / cs - id;
-        z[e] = 0.0;
+        return (id + (double)a.N[r * a.Qp + c]) / cs - id;
+    };
+    for (int y = threadIdx.y; y < 32; y += 8) {
+        ta[y][threadIdx.x] = f(r0 + y, c0 + threadIdx.x);
+        tb[y][threadIdx.x] = f(c0 + y, r0 + threadIdx.x);
+    }
+    __syncthreads();
+    for (int y = threadIdx.y; y < 32; y += 8) {
+        const long long r = r0 + y, c = c0 + threadIdx.x;
+        if (r < a.q && c < a.q) {
+            a.y[r * a.q + c] = 0.5 * (ta[y][threadIdx.x] + tb[threadIdx.x][y]);
+            a.z[r * a.q + c] = 0.0;
+        }
+        const long long r2 = c0 + y, c2 = r0 + threadIdx.x;
+        if (r2 < a.q && c2 < a.q) {
+            a.y[r2 * a.q + c2] = 0.5 * (tb[y][threadIdx.x] + ta[threadIdx.x][y]);
+            a.z[r2 * a.q + c2] = 0.0;
+        }
     }
 }
 
-// w = y + z + z y, m = -w / 2; the largest |w| of the iteration into the header
-__global__ void __launch_bounds__(256) k_fr_ns_m(const double* y, const double* z, const float* zy, long long Qp,
-                                                 long long q, double* m, FrameHeader* h, int side, int it) {
-    if (*reinterpret_cast<volatile int32_t*>(&h->conv[side])) return;
+// w = y + z + z y (the residual Z Y - I), m = -w / 2; the largest |w| of the
+// iteration goes to the header
+__global__ void __launch_bounds__(256) k_fr_ns_m(NsArgs a) {
+    __shared__ double ta[32][33], tb[32][33];
+    if (*reinterpret_cast<volatile int32_t*>(&a.h->conv[a.side])) return;
+    long long r0, c0;
+    if (!ns_tile(a.q, r0, c0)) return;
+    auto w = [&](long long r, long long c) -> double {
+        if (r >= a.q || c >= a.q) return 0.0;
+        const long long e = r * a.q + c;
+        return a.y[e] + a.z[e] + (double)a.T1[r * a.Qp + c];
+    };
+    for (int y = threadIdx.y; y < 32; y += 8) {
+        ta[y][threadIdx.x] = w(r0 + y, c0 + threadIdx.x);
+        tb[y][threadIdx.x] = w(c0 + y, r0 + threadIdx.x);
+    }
+    __syncthreads();
     float wm = 0.0f;
-    for (long long e = (long long)blockIdx.x * blockDim.x + threadIdx.x; e < q * q; e += (long long)gridDim.x * blockDim.x) {
-        const long long r = e / q, c = e - r * q;
-        const double w = y[e] + z[e] + (double)zy[r * Qp + c];
-        m[e] = -0.5 * w;
-        wm = fmaxf(wm, (float)fabs(w));
+    for (int y = threadIdx.y; y < 32; y += 8) {
+        const long long r = r0 + y, c = c0 + threadIdx.x;
+        if (r < a.q && c < a.q) {
+            const double v = 0.5 * (ta[y][threadIdx.x] + tb[threadIdx.x][y]);
+            a.m[r * a.q + c] = -0.5 * v;
+            wm = fmaxf(wm, (float)fabs(v));
+        }
+        const long long r2 = c0 + y, c2 = r0 + threadIdx.x;
+        if (r2 < a.q && c2 < a.q) a.m[r2 * a.q + c2] = -0.25 * (tb[y][threadIdx.x] + ta[threadIdx.x][y]);
     }
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) wm = fmaxf(wm, __shfl_xor_sync(0xFFFFFFFFu, wm, o));
-    if ((threadIdx.x & 31) == 0) atomicMax(&h->wmax[side][it], __float_as_uint(wm));
+    if ((threadIdx.x & 31) == 0) atomicMax(&a.h->wmax[a.side][a.it], __float_as_uint(wm));
 }
 
-// y += m + y m, z += m + m z; converged once max |w| <= FR_NS_TOL
-__global__ void __launch_bounds__(256) k_fr_ns_update(double* y, double* z, const double* m, const float* ym,
-                                                      const float* mz, long long Qp, long long q, FrameHeader* h,
-                                                      int side, int it) {
-    if (*reinterpret_cast<volatile int32_t*>(&h->conv[side])) return;
-    for (long long e = (long long)blockIdx.x * blockDim.x + threadIdx.x; e < q * q; e += (long long)gridDim.x * blockDim.x) {
-        const long long r = e / q, c = e - r * q;
-        y[e] += m[e] + (double)ym[r * Qp + c];
-        z[e] += m[e] + (double)mz[r * Qp + c];
+// y += m + y m, z += m + m z, in place.  The iteration stops (this update and
+// every later one skipped) once the residual is at the tolerance, or has
+// stopped its quadratic fall below 1e-2 (the rounding floor of the products),
+// or has grown.
+__global__ void __launch_bounds__(256) k_fr_ns_update(NsArgs a) {
+    __shared__ double ya[32][33], yb[32][33], za[32][33], zb[32][33];
+    if (*reinterpret_cast<volatile int32_t*>(&a.h->conv[a.side])) return;
+    const double wc = (double)__uint_as_float(a.h->wmax[a.side][a.it]);
+    const double wp = a.it > 0 ? (double)__uint_as_float(a.h->wmax[a.side][a.it - 1]) : 1e300;
+    const bool stop = !(wc > FR_NS_TOL) || wc >= wp || (wc < 1e-2 && wc > 0.25 * wp);
+    if (stop) {
+        if (blockIdx.x == 0 && blockIdx.y == 0 && threadIdx.x == 0 && threadIdx.y == 0) a.h->conv[a.side] = 1;
+        return;
     }
-    if (blockIdx.x == 0 && threadIdx.x == 0 && (double)__uint_as_float(h->wmax[side][it]) <= FR_NS_TOL)
-        h->conv[side] = 1;
+    long long r0, c0;
+    if (!ns_tile(a.q, r0, c0)) return;
+    auto fy = [&](long long r, long long c) -> double {
+        if (r >= a.q || c >= a.q) return 0.0;
+        const long long e = r * a.q + c;
+        return a.y[e] + a.m[e] + (double)a.T1[r * a.Qp + c];
+    };
+    auto fz = [&](long long r, long long c) -> double {
+        if (r >= a.q || c >= a.q) return 0.0;
+        const long long e = r * a.q + c;
+        return a.z[e] + a.m[e] + (double)a.T2[r * a.Qp + c];
+    };
+    for (int y = threadIdx.y; y < 32; y += 8) {
+        ya[y][threadIdx.x] = fy(r0 + y, c0 + threadIdx.x);
+        yb[y][threadIdx.x] = fy(c0 + y, r0 + threadIdx.x);
+        za[y][threadIdx.x] = fz(r0 + y, c0 + threadIdx.x);
+        zb[y][threadIdx.x] = fz(c0 + y, r0 + threadIdx.x);
+    }
+    __syncthreads();
+    for (int y = threadIdx.y; y < 32; y += 8) {
+        const long long r = r0 + y, c = c0 + threadIdx.x;
+        if (r < a.q && c < a.q) {
+            a.y[r * a.q + c] = 0.5 * (ya[y][threadIdx.x] + yb[threadIdx.x][y]);
+            a.z[r * a.q + c] = 0.5 * (za[y][threadIdx.x] + zb[threadIdx.x][y]);
+        }
+        const long long r2 = c0 + y, c2 = r0 + threadIdx.x;
+        if (r2 < a.q && c2 < a.q) {
+            a.y[r2 * a.q + c2] = 0.5 * (yb[y][threadIdx.x] + ya[threadIdx.x][y]);
+            a.z[r2 * a.q + c2] = 0.5 * (zb[y][threadIdx.x] + za[threadIdx.x][y]);
+        }
+    }
 }
 
 // E_F = xi* + (F_0 + xi*) R (P from the GEMM, ld Qp), in place over xi*
@@ -691,9 +787,14 @@ int32_t iso_frame_merge(const double* U0, const double* S0, const double* Vt0, c
         }
         // (I + N)^(-1/2) = I + R by the difference-form Newton-Schulz iteration
         FR_LAUNCH((k_fr_norm<<<grid_of(q * q, sms), 256, 0, s>>>(F(L.nq[sd]), Qp, q, hdr, sd)));
-        FR_LAUNCH((k_fr_ns_init<<<grid_of(q * q, sms), 256, 0, s>>>(F(L.nq[sd]), Qp, q, hdr, sd, D(L.ns_y), D(L.ns_z))));
+        NsArgs na{};
+        na.N = F(L.nq[sd]); na.y = D(L.ns_y); na.z = D(L.ns_z); na.m = D(L.ns_m); na.h = hdr;
+        na.q = q; na.Qp = Qp; na.side = sd;
+        const dim3 tiles((unsigned)((q + 31) / 32), (unsigned)((q + 31) / 32)), tb(32, 8);
+        FR_LAUNCH((k_fr_ns_init<<<tiles, tb, 0, s>>>(na)));
         SplitR sq{};
         sq.f = fr[sd]; sq.hdr = hdr; sq.side = sd; sq.mode = 2; sq.rows = q; sq.rows_p = Qp; sq.Lp = Qp;
+        sq.skip = &hdr->conv[sd];
         auto split_q = [&](const double* M_, size_t out_off) -> int {
             sq.M = M_; sq.out = F(out_off);
             FR_LAUNCH((k_fr_split_r<<<grid_of(Qp * Qp, sms), 256, 0, s>>>(sq)));
@@ -707,16 +808,17 @@ int32_t iso_frame_merge(const double* U0, const double* S0, const double* Vt0, c
             g.skip = &hdr->conv[sd];
             g.C = F(L.ns_t1);
             ISO_TRY(frame_gemm(s, F(L.ns_z4), Qp, F(L.ns_y4), Qp, Qp, g));     // z y
-            FR_LAUNCH((k_fr_ns_m<<<grid_of(q * q, sms), 256, 0, s>>>(D(L.ns_y), D(L.ns_z), F(L.ns_t1), Qp, q,
-                                                                      D(L.ns_m), hdr, sd, it)));
-            sq.M = D(L.ns_m); sq.out = F(L.ns_m4);
-            FR_LAUNCH((k_fr_split_r<<<grid_of(Qp * Qp, sms), 256, 0, s>>>(sq)));
+            na.it = it;
+            na.T1 = F(L.ns_t1);
+            FR_LAUNCH((k_fr_ns_m<<<tiles, tb, 0, s>>>(na)));
+            ISO_TRY(split_q(D(L.ns_m), L.ns_m4));
             g.C = F(L.ns_t2);
             ISO_TRY(frame_gemm(s, F(L.ns_y4), Qp, F(L.ns_m4), Qp, Qp, g));     // y m
             g.C = F(L.ns_t3);
             ISO_TRY(frame_gemm(s, F(L.ns_m4), Qp, F(L.ns_z4), Qp, Qp, g));     // m z
-            FR_LAUNCH((k_fr_ns_update<<<grid_of(q * q, sms), 256, 0, s>>>(D(L.ns_y), D(L.ns_z), D(L.ns_m), F(L.ns_t2),
-                                                                           F(L.ns_t3), Qp, q, hdr, sd, it)));
+            na.T1 = F(L.ns_t2);
+            na.T2 = F(L.ns_t3);
+            FR_LAUNCH((k_fr_ns_update<<<tiles, tb, 0, s>>>(na)));
             ISO_TRY(split_q(D(L.ns_y), L.ns_y4));
             ISO_TRY(split_q(D(L.ns_z), L.ns_z4));
         }

@@ -226,3 +226,20 @@ def test_frame_merge_in_place_and_through_gpu_svds():
     torch.cuda.synchronize()
     assert out.data_ptr() == W.data_ptr()
     _check(out.cpu(), st, r, W0, "torch SVDs, in place")
+
+
+def test_frame_merge_full_size_projection():
+    # one Qwen2.5-7B gate/up projection (3584 x 18944, bf16), two RL experts,
+    # through the GPU's own thin SVDs, against the oracle in binary64
+    m, n, K = 3584, 18944, 2
+    g = torch.Generator().manual_seed(7)
+    W0 = (torch.randn(m, n, generator=g) * 0.02).to(torch.bfloat16)
+    ex = [(W0.float() + torch.randn(m, n, generator=g) * 5e-4).to(torch.bfloat16) for _ in range(K)]
+    W0n = W0.double().numpy()
+    r = M.merge_matrix(W0n, [e.double().numpy() for e in ex])
+    out, st = iso.frame_merge(W0.to(DEV), [e.to(DEV) for e in ex], stats=True)
+    torch.cuda.synchronize()
+    assert int(st.status.item()) == 0
+    _check(out.cpu(), st, r, W0n, "Qwen2.5-7B gate 3584x18944 K=2 bf16 (GPU SVDs)")
+    del out, st
+    torch.cuda.empty_cache()
