@@ -28,10 +28,17 @@
 // * W* = W_0 + [E_U S_0 | U_0 S_0] [V* | E_V]^T with E_F = F* - F_0: the
 //   difference form keeps the low-precision products on the small motion;
 //   W_0 itself (the caller's matrix) replaces U_0 S_0 V_0^T.
-// * The large contractions run on the tensor cores (k_gemm_tf32) in three tf32
-//   products per pair (hi hi + hi lo + lo hi, x = hi + lo split in binary64),
-//   binary32 accumulation: about 2^-21 relative per product.  Everything else
-//   is binary64 on the CUDA cores.
+// * Precision.  A_i = F_0^T dF_i is binary64 on the CUDA cores: on dense
+//   spectra the frames rotate far inside near-degenerate singular subspaces
+//   while the proxies stay small, so Gamma is a difference of terms up to
+//   thousands of times larger than itself (the paper takes the merge in
+//   binary64 throughout).  The other large contractions (F_0 Y, xi*^T xi*,
+//   the Newton-Schulz products, (F_0 + xi*) R and the reconstruction) run on
+//   the tensor cores (k_gemm_tf32) as three tf32 products per pair (hi hi +
+//   hi lo + lo hi, x = hi + lo split in binary64) with binary32 accumulation,
+//   about 2^-22 relative per product; what they feed is the merged frame,
+//   whose error reaches W* only through products with the small motion.
+//   Everything else is binary64 on the CUDA cores.
 #include "iso_gemm.cuh"
 #include "iso_internal.cuh"
 
@@ -277,15 +284,69 @@ __global__ void __launch_bounds__(256) k_fr_split_r(SplitR a) {
     }
 }
 
-// Sym_i = sym(A_i), Kw_i = A_i - Sym_i (binary64) from the GEMM's A_i (binary32, ld Qp)
-__global__ void __launch_bounds__(256) k_fr_symskew(const float* A, long long Qp, long long q, double* sym, double* kw) {
-    __shared__ float ta[32][33], tb[32][33];
+// A_i = F_0^T dF_i in binary64 on the CUDA cores (dF_i = s_i F_i - F_0 formed
+// on the fly).  The Gram is a small difference of large terms whenever
+// frames rotate inside near-degenerate singular subspaces while the proxies
+// stay small, so this contraction (and only this one) is carried at the
+// paper's binary64 precision.  64 x 64 output tile per block, 16 rows of the
+// contraction per step, a 4 x 4 register tile per thread.
+__global__ void __launch_bounds__(256) k_fr_ftdf(Frames f, const double* dots, int i, double* A) {
+    __shared__ double sa[16][64], sb[16][64];
+    __shared__ double sg[64];
+    const long long q = f.q, d = f.d;
+    const long long k0 = (long long)blockIdx.y * 64, l0 = (long long)blockIdx.x * 64;
+    const int tx = threadIdx.x & 15, ty = threadIdx.x >> 4;
+    if (threadIdx.x < 64) sg[threadIdx.x] = (l0 + threadIdx.x < q) ? sign_of(dots, q, i, l0 + threadIdx.x) : 0.0;
+    double acc[4][4];
+#pragma unroll
+    for (int a = 0; a < 4; ++a)
+#pragma unroll
+        for (int b = 0; b < 4; ++b) acc[a][b] = 0.0;
+    const double* F0 = f.F0;
+    const double* Fi = f.F[i];
+    __syncthreads();
+    for (long long r0 = 0; r0 < d; r0 += 16) {
+        for (int e = threadIdx.x; e < 16 * 64; e += 256) {
+            const int rr = e >> 6, cc = e & 63;
+            const long long r = r0 + rr;
+            const long long ka = k0 + cc, lb = l0 + cc;
+            sa[rr][cc] = (r < d && ka < q) ? F0[r * q + ka] : 0.0;
+            sb[rr][cc] = (r < d && lb < q) ? fma(sg[cc], Fi[r * q + lb], -F0[r * q + lb]) : 0.0;
+        }
+        __syncthreads();
+#pragma unroll
+        for (int kk = 0; kk < 16; ++kk) {
+            double av[4], bv[4];
+#pragma unroll
+            for (int a = 0; a < 4; ++a) av[a] = sa[kk][ty * 4 + a];
+#pragma unroll
+            for (int b = 0; b < 4; ++b) bv[b] = sb[kk][tx * 4 + b];
+#pragma unroll
+            for (int a = 0; a < 4; ++a)
+#pragma unroll
+                for (int b = 0; b < 4; ++b) acc[a][b] = fma(av[a], bv[b], acc[a][b]);
+        }
+        __syncthreads();
+    }
+#pragma unroll
+    for (int a = 0; a < 4; ++a)
+#pragma unroll
+        for (int b = 0; b < 4; ++b) {
+            const long long k = k0 + ty * 4 + a, l = l0 + tx * 4 + b;
+            if (k < q && l < q) A[((long long)i * q + k) * q + l] = acc[a][b];
+        }
+}
+
+// Sym_i = sym(A_i), Kw_i = A_i - Sym_i (binary64; A is K arrays q x q)
+__global__ void __launch_bounds__(256) k_fr_symskew(const double* A, long long Qp, long long q, double* sym, double* kw) {
+    __shared__ double ta[32][33], tb[32][33];
     const int i = blockIdx.z;
-    const float* Ai = A + (long long)i * Qp * Qp;
+    const double* Ai = A + (long long)i * q * q;
     const long long r0 = (long long)blockIdx.y * 32, c0 = (long long)blockIdx.x * 32;
     for (int y = threadIdx.y; y < 32; y += 8) {
-        ta[y][threadIdx.x] = Ai[(r0 + y) * Qp + c0 + threadIdx.x];   // A[r0 + y, c0 + x]
-        tb[y][threadIdx.x] = Ai[(c0 + y) * Qp + r0 + threadIdx.x];   // A[c0 + y, r0 + x]
+        const long long ra = r0 + y, ca = c0 + threadIdx.x, rb = c0 + y, cb = r0 + threadIdx.x;
+        ta[y][threadIdx.x] = (ra < q && ca < q) ? Ai[ra * q + ca] : 0.0;   // A[r0 + y, c0 + x]
+        tb[y][threadIdx.x] = (rb < q && cb < q) ? Ai[rb * q + cb] : 0.0;   // A[c0 + y, r0 + x]
     }
     __syncthreads();
     for (int y = threadIdx.y; y < 32; y += 8) {
@@ -300,7 +361,7 @@ __global__ void __launch_bounds__(256) k_fr_symskew(const float* A, long long Qp
 
 // Gamma_ij (i <= j), summed into gram[i][j]; block y covers a slice of the q x q entries
 struct GramArgs {
-    const float* A[2];          // per side: K arrays Qp x Qp
+    const double* A[2];         // per side: K arrays q x q
     const double* sym[2];
     const double* kw[2];
     const double* cd[2];        // per side: K x K x q
@@ -329,8 +390,8 @@ __global__ void __launch_bounds__(256) k_fr_gram(GramArgs g) {
         double colt = 0.0;
 #pragma unroll
         for (int s = 0; s < 2; ++s) {
-            const double ai = g.A[s][(long long)i * g.Qp * g.Qp + r * g.Qp + c];
-            const double aj = g.A[s][(long long)j * g.Qp * g.Qp + r * g.Qp + c];
+            const double ai = g.A[s][(long long)i * qq + e];
+            const double aj = g.A[s][(long long)j * qq + e];
             const double si = g.sym[s][(long long)i * qq + e], sj = g.sym[s][(long long)j * qq + e];
             colt += ai * sj + si * aj - si * sj;
         }
@@ -554,7 +615,7 @@ size_t al256(size_t v) { return (v + 255) & ~(size_t)255; }
 struct FrameLayout {
     long long m, n, q, Mp, Np, Qp, K;
     size_t hdr, gram, coef, dots, vcopy;
-    size_t cd[2], ft4[2], dft4[2], aq[2], sym[2], kw[2], fr4[2], y4[2], e[2], xi[2], nq[2];
+    size_t cd[2], ft4[2], aq[2], sym[2], kw[2], fr4[2], y4[2], e[2], xi[2], nq[2];
     size_t ns_y, ns_z, ns_m, ns_y4, ns_z4, ns_m4, ns_t1, ns_t2, ns_t3;
     size_t a6, b6, total;
 };
@@ -575,9 +636,8 @@ FrameLayout frame_layout(long long m, long long n, int K) {
     L.vcopy = take(sizeof(double) * (K + 1) * n * q);
     for (int s = 0; s < 2; ++s) {
         const long long Dp = s == 0 ? L.Mp : L.Np, d = s == 0 ? m : n;
-        L.ft4[s] = take(sizeof(float) * Qp * 4 * Dp);      // F_0^T split, later xi*^T split
-        L.dft4[s] = take(sizeof(float) * Qp * 4 * Dp);     // dF_i^T split (one expert at a time)
-        L.aq[s] = take(sizeof(float) * K * Qp * Qp);
+        L.ft4[s] = take(sizeof(float) * Qp * 4 * Dp);      // xi*^T split
+        L.aq[s] = take(sizeof(double) * K * q * q);        // A_i = F_0^T dF_i (binary64)
         L.sym[s] = take(sizeof(double) * K * q * q);
         L.kw[s] = take(sizeof(double) * K * q * q);
         L.fr4[s] = take(sizeof(float) * Dp * 4 * Qp);      // F_0 split, later (F_0 + xi*) split
@@ -727,30 +787,19 @@ int32_t iso_frame_merge(const double* U0, const double* S0, const double* Vt0, c
                 fr[sd], dots, D(L.cd[sd]), r2)));
         }
     }
-    // A_i = F_0^T dF_i on the tensor cores, then Sym_i and Kw_i
+    // A_i = F_0^T dF_i (binary64), then Sym_i and Kw_i
     for (int sd = 0; sd < 2; ++sd) {
-        const long long Dp = sd == 0 ? L.Mp : L.Np;
-        SplitT st{};
-        st.f = fr[sd]; st.dots = dots; st.X = nullptr; st.Dp = Dp; st.Qp = Qp;
-        const dim3 blk(32, 8), grd((unsigned)(Dp / 32), (unsigned)(Qp / 32));
-        st.mode = 0; st.i = 0; st.out = F(L.ft4[sd]);
-        FR_LAUNCH((k_fr_split_t<<<grd, blk, 0, s>>>(st)));
-        for (int i = 0; i < K; ++i) {
-            st.mode = 1; st.i = i; st.out = F(L.dft4[sd]);
-            FR_LAUNCH((k_fr_split_t<<<grd, blk, 0, s>>>(st)));
-            GemmArgs g{};
-            g.mode = GEMM_STORE_F32; g.C = F(L.aq[sd]) + (size_t)i * Qp * Qp; g.ldc = Qp; g.M = (int)Qp; g.N = (int)Qp;
-            g.status = &hdr->status;
-            ISO_TRY(frame_gemm(s, F(L.ft4[sd]), Qp, F(L.dft4[sd]), Qp, Dp, g));
-        }
+        const dim3 grd((unsigned)((q + 63) / 64), (unsigned)((q + 63) / 64));
+        for (int i = 0; i < K; ++i)
+            FR_LAUNCH((k_fr_ftdf<<<grd, 256, 0, s>>>(fr[sd], dots, i, D(L.aq[sd]))));
         FR_LAUNCH((k_fr_symskew<<<dim3((unsigned)(Qp / 32), (unsigned)(Qp / 32), K), dim3(32, 8), 0, s>>>(
-            F(L.aq[sd]), Qp, q, D(L.sym[sd]), D(L.kw[sd]))));
+            D(L.aq[sd]), Qp, q, D(L.sym[sd]), D(L.kw[sd]))));
     }
     // Gamma and c*
     {
         GramArgs ga{};
         for (int sd = 0; sd < 2; ++sd) {
-            ga.A[sd] = F(L.aq[sd]); ga.sym[sd] = D(L.sym[sd]); ga.kw[sd] = D(L.kw[sd]); ga.cd[sd] = D(L.cd[sd]);
+            ga.A[sd] = D(L.aq[sd]); ga.sym[sd] = D(L.sym[sd]); ga.kw[sd] = D(L.kw[sd]); ga.cd[sd] = D(L.cd[sd]);
         }
         ga.S0 = S0; ga.gram = gram; ga.q = q; ga.Qp = Qp; ga.k_keep = k_keep; ga.K = K;
         const int pairs = K * (K + 1) / 2;
