@@ -360,8 +360,21 @@ def thin_svd(W: torch.Tensor):
     """The thin SVD W = U diag(S) Vt in binary64 on W's device (the library
     SVD of torch.linalg; the frame merge's one step that is not this
     library's own code)."""
+    _load_torch_linalg()
     U, S, Vt = torch.linalg.svd(W.to(torch.float64), full_matrices=False)
     return U.contiguous(), S.contiguous(), Vt.contiguous()
+
+
+def _load_torch_linalg():
+    """torch opens its GPU linear-algebra library lazily by name; under a
+    profiler that rewrites the library search path that lookup fails, so it is
+    loaded once here by its full path when the file is present."""
+    import os
+    lib_dir = os.path.join(os.path.dirname(torch.__file__), "lib")
+    path = os.path.join(lib_dir, "libtorch_cuda_linalg.so")
+    if os.path.exists(path) and not getattr(_load_torch_linalg, "done", False):
+        ctypes.CDLL(path, mode=ctypes.RTLD_GLOBAL)
+        _load_torch_linalg.done = True
 
 
 def frame_merge(W0: torch.Tensor, experts: Sequence[torch.Tensor], **kw):
