@@ -94,3 +94,33 @@ def test_merger_pins_catch_mutation(name, tmp_path):
                         os.path.join(ROOT, "tests", "test_oracle_iso_merger.py")],
                        cwd=ROOT, env=env, capture_output=True, text=True, timeout=600)
     assert r.returncode != 0, f"pins did not catch mutation {name}:\n{r.stdout[-2000:]}"
+
+
+# ---------------------------------------------------------------------------
+# the ISO-Optimizer oracle (numpy): the same scheme on its source
+# ---------------------------------------------------------------------------
+OPT_SRC = os.path.join(ROOT, "oracle", "iso_optimizer.py")
+OPT_MUTATIONS = {
+    "grad_u_without_sigma": ("return (G_W @ V) * S0[None, :], (G_W.T @ U) * S0[None, :]",
+                             "return (G_W @ V), (G_W.T @ U) * S0[None, :]"),
+    "grad_v_from_v": ("(G_W.T @ U) * S0[None, :]", "(G_W.T @ U[:, ::-1]) * S0[None, :]"),
+    "no_bias_correction": ("bc1 = 1.0 - beta1 ** step", "bc1 = 1.0"),
+    "eps_inside_sqrt": ("np.sqrt(v / bc2) + eps", "np.sqrt(v / bc2 + eps)"),
+    "coupled_decay": ("X - lr * weight_decay * X", "X - weight_decay * X"),
+    "second_moment_of_abs": ("(1.0 - beta2) * g * g", "(1.0 - beta2) * np.abs(g)"),
+    "no_retraction": ("    return P @ Qt", "    return np.asarray(X, np.float64)"),
+}
+
+
+@pytest.mark.parametrize("name", sorted(OPT_MUTATIONS))
+def test_optimizer_pins_catch_mutation(name, tmp_path):
+    old, new = OPT_MUTATIONS[name]
+    src = open(OPT_SRC).read()
+    assert src.count(old) == 1, f"mutation anchor not found: {name}"
+    path = tmp_path / "iso_optimizer_mut.py"
+    path.write_text(src.replace(old, new))
+    env = dict(os.environ, ISO_OPTIMIZER_PATH=str(path))
+    r = subprocess.run([sys.executable, "-m", "pytest", "-x", "-q", "-p", "no:cacheprovider",
+                        os.path.join(ROOT, "tests", "test_oracle_iso_optimizer.py")],
+                       cwd=ROOT, env=env, capture_output=True, text=True, timeout=600)
+    assert r.returncode != 0, f"pins did not catch mutation {name}:\n{r.stdout[-2000:]}"
