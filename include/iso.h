@@ -287,6 +287,49 @@ int32_t iso_frame_merge(const double* U0, const double* S0, const double* Vt0, c
                         const iso_tensor* out, const iso_frame_cfg* cfg, void* workspace, size_t ws_bytes,
                         const iso_merge_stats* stats, void* stream);
 
+/* ---- ISO-Optimizer step ISO[AdamW] on one weight matrix (Sec. 4.3) -------
+ *
+ * The fixed-spectrum parameterisation W(U, V) = U S0 V^T with AdamW applied
+ * to the frames: the factor gradients G_U = G_W V S0 and G_V = G_W^T U S0
+ * (Sec. 4.3, factor gradients), AdamW on U and on V with their own moments
+ * (the base optimizer on the factors; decoupled weight decay, bias-corrected
+ * moments), the polar retraction U+ = polar(U_bar), V+ = polar(V_bar) and
+ * W+ = U+ S0 V+^T (Sec. 4.3 with the polar factor of App. E). */
+typedef struct {
+    double  lr;            /* learning rate >= 0 */
+    double  beta1, beta2;  /* moment decays in [0, 1) */
+    double  eps;           /* > 0 */
+    double  weight_decay;  /* >= 0 (decoupled; the paper uses 0) */
+    int64_t step;          /* this update's step number, from 1 (bias correction) */
+    int32_t ns_iters;      /* iteration limit of the polar factor's inverse square root;
+                              0 = the default (16); it stops at convergence */
+    int32_t reserved;      /* must be 0 */
+} iso_adamw_cfg;
+
+/* Host-only.  Workspace bytes of iso_opt_step for an m x n matrix
+ * (m, n < 2^24, min(m, n) <= 32768). */
+int32_t iso_opt_workspace_size(int64_t m, int64_t n, size_t* bytes);
+
+/* One ISO[AdamW] step of an m x n matrix, q = min(m, n).  Device pointers:
+ *   U (m x q), V (n x q)   binary64 frames with orthonormal columns, updated in place
+ *   S0 (q)                 the fixed spectrum
+ *   G_W                    the gradient with respect to W (m x n, ISO_BF16 or ISO_F32)
+ *   mU, vU (m x q), mV, vV (n x q)  binary32 AdamW moments, updated in place
+ *                          (zero before the first step)
+ *   W                      the current weight matrix U S0 V^T as stored (bf16 / fp32)
+ *   W_out                  receives W + (U+ S0 V+^T - U S0 V^T); same dtype, may
+ *                          coincide with W (each entry read and written by one
+ *                          thread) but share no other byte with it
+ * The retraction assumes U^T U = I (and V^T V = I) to the working precision.
+ * Precision: the factor gradients and the retraction's products are three tf32
+ * products per pair with binary32 accumulation; the AdamW arithmetic and the
+ * frames are binary64.  stats->status (may be NULL) receives ISO_OK or
+ * ISO_ERR_TIMEOUT.  Argument errors are returned before anything is enqueued. */
+int32_t iso_opt_step(double* U, double* V, const double* S0, const iso_tensor* G_W, float* mU, float* vU,
+                     float* mV, float* vV, const iso_tensor* W, const iso_tensor* W_out, int64_t m, int64_t n,
+                     const iso_adamw_cfg* cfg, void* workspace, size_t ws_bytes, const iso_merge_stats* stats,
+                     void* stream);
+
 /* The frame merge's dense product on the tensor cores, for tests of the
  * contraction alone: C (M x N, row stride ldc) = A[:, a_k0 : a_k0 + Kc]
  * B[:, b_k0 : b_k0 + Kc]^T, A (M rows, stride lda) and B (N rows, stride

@@ -63,6 +63,12 @@ class IsoFrameCfg(ctypes.Structure):
                 ("c_max", ctypes.c_double), ("ns_iters", ctypes.c_int32), ("reserved", ctypes.c_int32)]
 
 
+class IsoAdamwCfg(ctypes.Structure):
+    _fields_ = [("lr", ctypes.c_double), ("beta1", ctypes.c_double), ("beta2", ctypes.c_double),
+                ("eps", ctypes.c_double), ("weight_decay", ctypes.c_double), ("step", ctypes.c_int64),
+                ("ns_iters", ctypes.c_int32), ("reserved", ctypes.c_int32)]
+
+
 # (name, restype, argtypes) for every entry point of include/iso.h
 P = ctypes.c_void_p
 PT = ctypes.POINTER(IsoTensor)
@@ -84,6 +90,9 @@ PROTOTYPES = [
     ("iso_frame_merge", I32, [P, P, P, P, P, I32, I64, I64, PT, PT, ctypes.POINTER(IsoFrameCfg), P, SZ,
                               ctypes.POINTER(IsoMergeStats), P]),
     ("iso_gemm_tf32", I32, [P, I64, P, I64, P, I64, I64, I64, I64, I64, I64, P]),
+    ("iso_opt_workspace_size", I32, [I64, I64, ctypes.POINTER(SZ)]),
+    ("iso_opt_step", I32, [P, P, P, PT, P, P, P, P, PT, PT, I64, I64, ctypes.POINTER(IsoAdamwCfg), P, SZ,
+                           ctypes.POINTER(IsoMergeStats), P]),
     ("iso_error_string", ctypes.c_char_p, [I32]),
     ("iso_launch_count", ctypes.c_uint64, []),
     ("iso_force_two_pass", ctypes.c_int32, [ctypes.c_int32]),

@@ -398,3 +398,40 @@ def gemm_tf32(A: torch.Tensor, B: torch.Tensor, C: torch.Tensor, Kc: int, a_k0=0
                              A.shape[0], B.shape[0], int(Kc), int(a_k0), int(b_k0), _stream(stream))
     check(rc, "iso_gemm_tf32")
     return C
+
+
+# ---------------------------------------------------------------------------
+# ISO-Optimizer step ISO[AdamW] on one matrix (Sec. 4.3)
+# ---------------------------------------------------------------------------
+def opt_workspace_size(m: int, n: int) -> int:
+    b = ctypes.c_size_t(0)
+    check(lib().iso_opt_workspace_size(int(m), int(n), ctypes.byref(b)), "iso_opt_workspace_size")
+    return int(b.value)
+
+
+def opt_step(U, V, S0, G_W, mU, vU, mV, vV, W, W_out=None, lr=1e-6, beta1=0.9, beta2=0.999, eps=1e-8,
+             weight_decay=0.0, step=1, ns_iters=0, workspace=None, stats=False, stream=None):
+    """iso_opt_step: one ISO[AdamW] step of an m x n matrix.  U (m x q) and V
+    (n x q) are contiguous float64 frames and mU, vU, mV, vV float32 moments
+    of the same shapes, all updated in place; S0 (q) float64; G_W, W (m x n,
+    bf16 or fp32).  Returns W_out (and a status tensor with stats=True)."""
+    m, n = int(W.shape[0]), int(W.shape[1])
+    for t in (U, V, S0):
+        if t.dtype != torch.float64 or not t.is_contiguous():
+            raise ValueError("frames and spectrum must be contiguous float64 tensors")
+    for t in (mU, vU, mV, vV):
+        if t.dtype != torch.float32 or not t.is_contiguous():
+            raise ValueError("moments must be contiguous float32 tensors")
+    if W_out is None:
+        W_out = torch.empty_like(W)
+    cfg = _abi.IsoAdamwCfg(float(lr), float(beta1), float(beta2), float(eps), float(weight_decay), int(step),
+                           int(ns_iters), 0)
+    ws = _workspace(workspace, W.device)
+    wptr, wlen = ws.get(opt_workspace_size(m, n))
+    st = torch.zeros(1, dtype=torch.int32, device=W.device) if stats else None
+    abi_st = IsoMergeStats(st.data_ptr(), None, None, None) if stats else None
+    rc = lib().iso_opt_step(U.data_ptr(), V.data_ptr(), S0.data_ptr(), describe([G_W]), mU.data_ptr(),
+                            vU.data_ptr(), mV.data_ptr(), vV.data_ptr(), describe([W]), describe([W_out]), m, n,
+                            ctypes.byref(cfg), wptr, wlen, ctypes.byref(abi_st) if stats else None, _stream(stream))
+    check(rc, "iso_opt_step")
+    return (W_out, st) if stats else W_out

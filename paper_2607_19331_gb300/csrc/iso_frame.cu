@@ -180,35 +180,48 @@ __global__ void __launch_bounds__(256) k_fr_coldots(Frames f, const double* dots
         }
 }
 
-// Transposed split operand out[k][seg][r] (Qp rows of 4 Dp) of a d x q source:
-// mode 0: F_0; mode 1: dF_i = s_i F_i - F_0; mode 2: the binary64 array X
+// Transposed split operand out[k][seg][j] (Qp rows of 4 Lr) of a d x q source,
+// j the source row (Lr = Dp; the stacked modes 4 and 5 put two d-row sources
+// one above the other, Lr = 2 Dp):
+//   0  F_0[j, k];  1  dF_i = s_i F_i - F_0;  2  X[j, k];  3  X[j, k] S_0[k]
+//   4  [F_0 ; X];  5  [X ; F_0 + X]
 struct SplitT {
     Frames f;
     const double* dots;
     const double* X;
+    const double* S0;
     int mode, i;
     float* out;
     long long Dp, Qp;
 };
 __global__ void __launch_bounds__(256) k_fr_split_t(SplitT a) {
     __shared__ double t[32][33];
+    const long long Lr = (a.mode >= 4) ? 2 * a.Dp : a.Dp;
     const long long r0 = (long long)blockIdx.x * 32, k0 = (long long)blockIdx.y * 32;
     const long long d = a.f.d, q = a.f.q;
     for (int y = threadIdx.y; y < 32; y += 8) {
-        const long long r = r0 + y, k = k0 + threadIdx.x;
+        long long r = r0 + y;
+        const long long k = k0 + threadIdx.x;
+        int half = 0;
+        if (a.mode >= 4 && r >= a.Dp) { half = 1; r -= a.Dp; }
         double v = 0.0;
         if (r < d && k < q) {
             const long long e = r * q + k;
-            if (a.mode == 0) v = a.f.F0[e];
-            else if (a.mode == 1) v = fma(sign_of(a.dots, q, a.i, k), a.f.F[a.i][e], -a.f.F0[e]);
-            else v = a.X[e];
+            switch (a.mode) {
+                case 0: v = a.f.F0[e]; break;
+                case 1: v = fma(sign_of(a.dots, q, a.i, k), a.f.F[a.i][e], -a.f.F0[e]); break;
+                case 2: v = a.X[e]; break;
+                case 3: v = a.X[e] * a.S0[k]; break;
+                case 4: v = half ? a.X[e] : a.f.F0[e]; break;
+                case 5: v = half ? a.f.F0[e] + a.X[e] : a.X[e]; break;
+            }
         }
         t[y][threadIdx.x] = v;
     }
     __syncthreads();
     for (int y = threadIdx.y; y < 32; y += 8) {
         const long long k = k0 + y, r = r0 + threadIdx.x;
-        if (k < a.Qp && r < a.Dp) put_split(a.out + k * 4 * a.Dp, a.Dp, r, t[threadIdx.x][y]);
+        if (k < a.Qp && r < Lr) put_split(a.out + k * 4 * Lr, Lr, r, t[threadIdx.x][y]);
     }
 }
 
@@ -335,6 +348,43 @@ __global__ void __launch_bounds__(256) k_fr_ftdf(Frames f, const double* dots, i
             const long long k = k0 + ty * 4 + a, l = l0 + tx * 4 + b;
             if (k < q && l < q) A[((long long)i * q + k) * q + l] = acc[a][b];
         }
+}
+
+// Split operands of an m x n bf16 / fp32 matrix G (row stride n): row-major
+// (rows Mp of 4 Np, element G[r, c]) or transposed (rows Np of 4 Mp, element
+// G[r, c] at row c, position r)
+__device__ __forceinline__ double load_typed(const void* p, int dtype, long long e) {
+    if (dtype == ISO_BF16) return (double)__uint_as_float((uint32_t)static_cast<const unsigned short*>(p)[e] << 16);
+    return (double)static_cast<const float*>(p)[e];
+}
+__global__ void __launch_bounds__(256) k_op_split_g(const void* G, int dtype, long long m, long long n, long long Mp,
+                                                    long long Np, float* out) {
+    const long long total = Mp * Np;
+    for (long long e = (long long)blockIdx.x * blockDim.x + threadIdx.x; e < total; e += (long long)gridDim.x * blockDim.x) {
+        const long long r = e / Np, c = e - r * Np;
+        const double v = (r < m && c < n) ? load_typed(G, dtype, r * n + c) : 0.0;
+        put_split(out + r * 4 * Np, Np, c, v);
+    }
+}
+__global__ void __launch_bounds__(256) k_op_split_gt(const void* G, int dtype, long long m, long long n, long long Mp,
+                                                     long long Np, float* out) {
+    __shared__ double t[32][33];
+    const long long r0 = (long long)blockIdx.x * 32, c0 = (long long)blockIdx.y * 32;
+    for (int y = threadIdx.y; y < 32; y += 8) {
+        const long long r = r0 + y, c = c0 + threadIdx.x;
+        t[y][threadIdx.x] = (r < m && c < n) ? load_typed(G, dtype, r * n + c) : 0.0;
+    }
+    __syncthreads();
+    for (int y = threadIdx.y; y < 32; y += 8) {
+        const long long c = c0 + y, r = r0 + threadIdx.x;
+        if (c < Np && r < Mp) put_split(out + c * 4 * Mp, Mp, r, t[threadIdx.x][y]);
+    }
+}
+
+// F += E (binary64, d x q)
+__global__ void __launch_bounds__(256) k_op_add(double* F, const double* E, long long total) {
+    for (long long e = (long long)blockIdx.x * blockDim.x + threadIdx.x; e < total; e += (long long)gridDim.x * blockDim.x)
+        F[e] += E[e];
 }
 
 // Sym_i = sym(A_i), Kw_i = A_i - Sym_i (binary64; A is K arrays q x q)
@@ -694,6 +744,107 @@ int frame_gemm(cudaStream_t s, const float* A, long long a_rows, const float* B,
     return cudaGetLastError() == cudaSuccess ? ISO_OK : ISO_ERR_CUDA;
 }
 
+struct OptLayout {
+    long long m, n, q, Mp, Np, Qp, Dmax;
+    size_t hdr, gw4, gwt4, su4, sv4, dF[2], na4, nb4, nq, xb4, r4, p, a6, b6;
+    size_t ns_y, ns_z, ns_m, ns_y4, ns_z4, ns_m4, ns_t1, ns_t2, ns_t3, total;
+};
+
+OptLayout opt_layout(long long m, long long n) {
+    OptLayout L;
+    L.m = m; L.n = n; L.q = std::min(m, n);
+    L.Mp = pad_up(m); L.Np = pad_up(n); L.Qp = pad_up(L.q);
+    L.Dmax = std::max(L.Mp, L.Np);
+    const long long q = L.q, Qp = L.Qp;
+    size_t o = 0;
+    auto take = [&](size_t bytes) { const size_t at = o; o = al256(o + bytes); return at; };
+    L.hdr = take(sizeof(FrameHeader));
+    L.gw4 = take(sizeof(float) * L.Mp * 4 * L.Np);      // G_W, rows m, contraction n
+    L.gwt4 = take(sizeof(float) * L.Np * 4 * L.Mp);     // G_W^T, rows n, contraction m
+    L.su4 = take(sizeof(float) * Qp * 4 * L.Mp);        // (U S_0)^T
+    L.sv4 = take(sizeof(float) * Qp * 4 * L.Np);        // (V S_0)^T
+    L.dF[0] = take(sizeof(double) * m * q);             // U_bar - U, later E_U
+    L.dF[1] = take(sizeof(double) * n * q);             // V_bar - V, later E_V
+    L.na4 = take(sizeof(float) * Qp * 4 * 2 * L.Dmax);  // [F ; dF]^T
+    L.nb4 = take(sizeof(float) * Qp * 4 * 2 * L.Dmax);  // [dF ; F + dF]^T
+    L.nq = take(sizeof(float) * Qp * Qp);
+    L.xb4 = take(sizeof(float) * L.Dmax * 4 * Qp);      // F + dF
+    L.r4 = take(sizeof(float) * Qp * 4 * Qp);
+    L.p = take(sizeof(float) * L.Dmax * Qp);
+    L.a6 = take(sizeof(float) * L.Mp * 4 * 2 * Qp);
+    L.b6 = take(sizeof(float) * L.Np * 4 * 2 * Qp);
+    L.ns_y = take(sizeof(double) * q * q);
+    L.ns_z = take(sizeof(double) * q * q);
+    L.ns_m = take(sizeof(double) * q * q);
+    L.ns_y4 = take(sizeof(float) * Qp * 4 * Qp);
+    L.ns_z4 = take(sizeof(float) * Qp * 4 * Qp);
+    L.ns_m4 = take(sizeof(float) * Qp * 4 * Qp);
+    L.ns_t1 = take(sizeof(float) * Qp * Qp);
+    L.ns_t2 = take(sizeof(float) * Qp * Qp);
+    L.ns_t3 = take(sizeof(float) * Qp * Qp);
+    L.total = o;
+    return L;
+}
+
+// launch one CUDA-core kernel of the frame merge / optimizer step on stream s
+#define FR_LAUNCH(...) do { const int _slot = prof_begin(1, s); __VA_ARGS__; prof_end(_slot, s); \
+                                if (cudaGetLastError() != cudaSuccess) return ISO_ERR_CUDA; } while (0)
+
+// Scratch of the inverse square root
+struct NsBufs {
+    double *y, *z, *m;
+    float *y4, *z4, *m4, *t1, *t2, *t3;
+};
+
+// R = (I + N)^(-1/2) - I for N = X^T X (binary32, ld Qp) with X^T F_0 skew,
+// by the difference-form Newton-Schulz iteration (k_fr_ns_*), written as
+// the split operand R4 (Qp rows of 4 Qp; R is symmetric, so it serves as B
+// of (F_0 + X) R).  Header slot `side` holds its scaling and state.
+int ns_root(cudaStream_t s, int sms, FrameHeader* hdr, int side, const float* Nq, long long q, long long Qp,
+            const NsBufs& b, int ns_iters, float* R4) {
+    FR_LAUNCH((k_fr_norm<<<grid_of(q * q, sms), 256, 0, s>>>(Nq, Qp, q, hdr, side)));
+    NsArgs na{};
+    na.N = Nq; na.y = b.y; na.z = b.z; na.m = b.m; na.h = hdr;
+    na.q = q; na.Qp = Qp; na.side = side;
+    const dim3 tiles((unsigned)((q + 31) / 32), (unsigned)((q + 31) / 32)), tb(32, 8);
+    FR_LAUNCH((k_fr_ns_init<<<tiles, tb, 0, s>>>(na)));
+    SplitR sq{};
+    sq.f.q = q; sq.hdr = hdr; sq.side = side; sq.mode = 2; sq.rows = q; sq.rows_p = Qp; sq.Lp = Qp;
+    sq.skip = &hdr->conv[side];
+    auto split_q = [&](const double* M_, float* out) -> int {
+        sq.M = M_; sq.out = out;
+        FR_LAUNCH((k_fr_split_r<<<grid_of(Qp * Qp, sms), 256, 0, s>>>(sq)));
+        return ISO_OK;
+    };
+    ISO_TRY(split_q(b.y, b.y4));
+    ISO_TRY(split_q(b.z, b.z4));
+    for (int it = 0; it < ns_iters; ++it) {
+        GemmArgs g{};
+        g.mode = GEMM_STORE_F32; g.ldc = Qp; g.M = (int)Qp; g.N = (int)Qp; g.status = &hdr->status;
+        g.skip = &hdr->conv[side];
+        g.C = b.t1;
+        ISO_TRY(frame_gemm(s, b.z4, Qp, b.y4, Qp, Qp, g));     // z y
+        na.it = it;
+        na.T1 = b.t1;
+        FR_LAUNCH((k_fr_ns_m<<<tiles, tb, 0, s>>>(na)));
+        ISO_TRY(split_q(b.m, b.m4));
+        g.C = b.t2;
+        ISO_TRY(frame_gemm(s, b.y4, Qp, b.m4, Qp, Qp, g));     // y m
+        g.C = b.t3;
+        ISO_TRY(frame_gemm(s, b.m4, Qp, b.z4, Qp, Qp, g));     // m z
+        na.T1 = b.t2;
+        na.T2 = b.t3;
+        FR_LAUNCH((k_fr_ns_update<<<tiles, tb, 0, s>>>(na)));
+        ISO_TRY(split_q(b.y, b.y4));
+        ISO_TRY(split_q(b.z, b.z4));
+    }
+    SplitR sr{};
+    sr.f.q = q; sr.hdr = hdr; sr.side = side; sr.mode = 6; sr.M = b.z; sr.out = R4;
+    sr.rows = q; sr.rows_p = Qp; sr.Lp = Qp;
+    FR_LAUNCH((k_fr_split_r<<<grid_of(Qp * Qp, sms), 256, 0, s>>>(sr)));
+    return ISO_OK;
+}
+
 }  // namespace
 }  // namespace iso
 
@@ -757,8 +908,6 @@ int32_t iso_frame_merge(const double* U0, const double* S0, const double* Vt0, c
     double* dots = reinterpret_cast<double*>(ws + L.dots);
     auto F = [&](size_t off) { return reinterpret_cast<float*>(ws + off); };
     auto D = [&](size_t off) { return reinterpret_cast<double*>(ws + off); };
-#define FR_LAUNCH(...) do { const int _slot = prof_begin(1, s); __VA_ARGS__; prof_end(_slot, s); \
-                                if (cudaGetLastError() != cudaSuccess) return ISO_ERR_CUDA; } while (0)
 
     // header, Gamma, c*, the sign dots and the column dots start at zero
     if (cudaMemsetAsync(ws, 0, L.cd[1] + sizeof(double) * K * K * q, s) != cudaSuccess) return ISO_ERR_CUDA;
@@ -834,46 +983,13 @@ int32_t iso_frame_merge(const double* U0, const double* S0, const double* Vt0, c
             g.mode = GEMM_STORE_F32; g.C = F(L.nq[sd]); g.ldc = Qp; g.M = (int)Qp; g.N = (int)Qp; g.status = &hdr->status;
             ISO_TRY(frame_gemm(s, F(L.ft4[sd]), Qp, F(L.ft4[sd]), Qp, Dp, g));
         }
-        // (I + N)^(-1/2) = I + R by the difference-form Newton-Schulz iteration
-        FR_LAUNCH((k_fr_norm<<<grid_of(q * q, sms), 256, 0, s>>>(F(L.nq[sd]), Qp, q, hdr, sd)));
-        NsArgs na{};
-        na.N = F(L.nq[sd]); na.y = D(L.ns_y); na.z = D(L.ns_z); na.m = D(L.ns_m); na.h = hdr;
-        na.q = q; na.Qp = Qp; na.side = sd;
-        const dim3 tiles((unsigned)((q + 31) / 32), (unsigned)((q + 31) / 32)), tb(32, 8);
-        FR_LAUNCH((k_fr_ns_init<<<tiles, tb, 0, s>>>(na)));
-        SplitR sq{};
-        sq.f = fr[sd]; sq.hdr = hdr; sq.side = sd; sq.mode = 2; sq.rows = q; sq.rows_p = Qp; sq.Lp = Qp;
-        sq.skip = &hdr->conv[sd];
-        auto split_q = [&](const double* M_, size_t out_off) -> int {
-            sq.M = M_; sq.out = F(out_off);
-            FR_LAUNCH((k_fr_split_r<<<grid_of(Qp * Qp, sms), 256, 0, s>>>(sq)));
-            return ISO_OK;
-        };
-        ISO_TRY(split_q(D(L.ns_y), L.ns_y4));
-        ISO_TRY(split_q(D(L.ns_z), L.ns_z4));
-        for (int it = 0; it < ns_iters; ++it) {
-            GemmArgs g{};
-            g.mode = GEMM_STORE_F32; g.ldc = Qp; g.M = (int)Qp; g.N = (int)Qp; g.status = &hdr->status;
-            g.skip = &hdr->conv[sd];
-            g.C = F(L.ns_t1);
-            ISO_TRY(frame_gemm(s, F(L.ns_z4), Qp, F(L.ns_y4), Qp, Qp, g));     // z y
-            na.it = it;
-            na.T1 = F(L.ns_t1);
-            FR_LAUNCH((k_fr_ns_m<<<tiles, tb, 0, s>>>(na)));
-            ISO_TRY(split_q(D(L.ns_m), L.ns_m4));
-            g.C = F(L.ns_t2);
-            ISO_TRY(frame_gemm(s, F(L.ns_y4), Qp, F(L.ns_m4), Qp, Qp, g));     // y m
-            g.C = F(L.ns_t3);
-            ISO_TRY(frame_gemm(s, F(L.ns_m4), Qp, F(L.ns_z4), Qp, Qp, g));     // m z
-            na.T1 = F(L.ns_t2);
-            na.T2 = F(L.ns_t3);
-            FR_LAUNCH((k_fr_ns_update<<<tiles, tb, 0, s>>>(na)));
-            ISO_TRY(split_q(D(L.ns_y), L.ns_y4));
-            ISO_TRY(split_q(D(L.ns_z), L.ns_z4));
+        // (I + N)^(-1/2) = I + R by the difference-form Newton-Schulz iteration,
+        // then F_0 + xi*, and E_F = xi* + (F_0 + xi*) R
+        {
+            NsBufs nb{D(L.ns_y), D(L.ns_z), D(L.ns_m), F(L.ns_y4), F(L.ns_z4), F(L.ns_m4), F(L.ns_t1),
+                      F(L.ns_t2), F(L.ns_t3)};
+            ISO_TRY(ns_root(s, sms, hdr, sd, F(L.nq[sd]), q, Qp, nb, ns_iters, F(L.y4[sd])));
         }
-        // R, F_0 + xi*, then E_F = xi* + (F_0 + xi*) R
-        sr.mode = 6; sr.M = D(L.ns_z); sr.out = F(L.y4[sd]); sr.rows = q; sr.rows_p = Qp; sr.Lp = Qp;
-        FR_LAUNCH((k_fr_split_r<<<grid_of(Qp * Qp, sms), 256, 0, s>>>(sr)));
         sr.mode = 1; sr.X = D(L.xi[sd]); sr.out = F(L.fr4[sd]); sr.rows = d; sr.rows_p = Dp; sr.Lp = Qp;
         FR_LAUNCH((k_fr_split_r<<<grid_of(Dp * Qp, sms), 256, 0, s>>>(sr)));
         {
@@ -897,7 +1013,129 @@ int32_t iso_frame_merge(const double* U0, const double* S0, const double* Vt0, c
         ISO_TRY(frame_gemm(s, F(L.a6), L.Mp, F(L.b6), L.Np, 2 * Qp, g));
     }
     if (stats && stats->status) FR_LAUNCH((k_fr_status<<<1, 32, 0, s>>>(hdr, stats->status)));
-#undef FR_LAUNCH
+    return ISO_OK;
+}
+
+int32_t iso_opt_workspace_size(int64_t m, int64_t n, size_t* bytes) {
+    if (!bytes || m < 1 || n < 1) return ISO_ERR_ARG;
+    if (m >= (1LL << 24) || n >= (1LL << 24) || std::min(m, n) > 32768) return ISO_ERR_UNSUPPORTED;
+    *bytes = opt_layout(m, n).total;
+    return ISO_OK;
+}
+
+int32_t iso_opt_step(double* U, double* V, const double* S0, const iso_tensor* G_W, float* mU, float* vU,
+                     float* mV, float* vV, const iso_tensor* W, const iso_tensor* W_out, int64_t m, int64_t n,
+                     const iso_adamw_cfg* cfg, void* workspace, size_t ws_bytes, const iso_merge_stats* stats,
+                     void* stream) {
+    size_t need = 0;
+    ISO_TRY(iso_opt_workspace_size(m, n, &need));
+    if (!U || !V || !S0 || !G_W || !mU || !vU || !mV || !vV || !W || !W_out || !cfg) return ISO_ERR_ARG;
+    auto al8 = [](const void* p) { return ((uintptr_t)p & 7u) == 0; };
+    auto al4 = [](const void* p) { return ((uintptr_t)p & 3u) == 0; };
+    if (!al8(U) || !al8(V) || !al8(S0) || !al4(mU) || !al4(vU) || !al4(mV) || !al4(vV)) return ISO_ERR_ALIGN;
+    if (!(cfg->lr >= 0.0) || !std::isfinite(cfg->lr)) return ISO_ERR_ARG;
+    if (!(cfg->beta1 >= 0.0 && cfg->beta1 < 1.0) || !(cfg->beta2 >= 0.0 && cfg->beta2 < 1.0)) return ISO_ERR_ARG;
+    if (!(cfg->eps > 0.0) || !std::isfinite(cfg->eps)) return ISO_ERR_ARG;
+    if (!(cfg->weight_decay >= 0.0) || !std::isfinite(cfg->weight_decay)) return ISO_ERR_ARG;
+    if (cfg->step < 1 || cfg->ns_iters < 0 || cfg->ns_iters > FR_MAX_NS || cfg->reserved != 0) return ISO_ERR_ARG;
+    for (const iso_tensor* t : {G_W, W, W_out}) {
+        if (t->rows != m || t->cols != n) return ISO_ERR_SHAPE;
+        if (t->dtype != ISO_BF16 && t->dtype != ISO_F32) return ISO_ERR_DTYPE;
+        if (!t->data) return ISO_ERR_ARG;
+        if ((uintptr_t)t->data & 15u) return ISO_ERR_ALIGN;
+    }
+    if (W_out->dtype != W->dtype) return ISO_ERR_DTYPE;
+    {
+        const size_t es = W->dtype == ISO_BF16 ? 2 : 4;
+        const uintptr_t o0 = (uintptr_t)W_out->data, o1 = o0 + (uintptr_t)(m * n) * es, w0 = (uintptr_t)W->data;
+        if (o0 != w0 && o0 < w0 + (uintptr_t)(m * n) * es && w0 < o1) return ISO_ERR_ARG;
+    }
+    if (!workspace || ((uintptr_t)workspace & 255u)) return ISO_ERR_WORKSPACE;
+    if (ws_bytes < need) return ISO_ERR_WORKSPACE;
+    const OptLayout L = opt_layout(m, n);
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    char* ws = static_cast<char*>(workspace);
+    int dev = 0, sms = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess ||
+        cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
+        return ISO_ERR_CUDA;
+    const long long q = L.q, Qp = L.Qp;
+    const int ns_iters = cfg->ns_iters ? cfg->ns_iters : FR_DEFAULT_NS;
+    FrameHeader* hdr = reinterpret_cast<FrameHeader*>(ws + L.hdr);
+    auto F = [&](size_t off) { return reinterpret_cast<float*>(ws + off); };
+    auto D = [&](size_t off) { return reinterpret_cast<double*>(ws + off); };
+    if (cudaMemsetAsync(ws + L.hdr, 0, sizeof(FrameHeader), s) != cudaSuccess) return ISO_ERR_CUDA;
+
+    Frames fr[2];
+    fr[0] = Frames{}; fr[0].F0 = U; fr[0].d = m; fr[0].q = q;
+    fr[1] = Frames{}; fr[1].F0 = V; fr[1].d = n; fr[1].q = q;
+    // operands of the factor gradients G_U = G_W (V S_0), G_V = G_W^T (U S_0)
+    FR_LAUNCH((k_op_split_g<<<grid_of(L.Mp * L.Np, sms), 256, 0, s>>>(G_W->data, G_W->dtype, m, n, L.Mp, L.Np,
+                                                                      F(L.gw4))));
+    FR_LAUNCH((k_op_split_gt<<<dim3((unsigned)(L.Mp / 32), (unsigned)(L.Np / 32)), dim3(32, 8), 0, s>>>(
+        G_W->data, G_W->dtype, m, n, L.Mp, L.Np, F(L.gwt4))));
+    for (int sd = 0; sd < 2; ++sd) {
+        SplitT st{};
+        st.f = fr[sd]; st.X = sd == 0 ? U : V; st.S0 = S0; st.mode = 3; st.Dp = sd == 0 ? L.Mp : L.Np; st.Qp = Qp;
+        st.out = F(sd == 0 ? L.su4 : L.sv4);
+        FR_LAUNCH((k_fr_split_t<<<dim3((unsigned)(st.Dp / 32), (unsigned)(Qp / 32)), dim3(32, 8), 0, s>>>(st)));
+    }
+    // the factor gradients on the tensor cores with AdamW in the epilogue:
+    // dF = F_bar - F, the moments updated in place
+    const double bc1 = 1.0 - std::pow(cfg->beta1, (double)cfg->step);
+    const double bc2 = 1.0 - std::pow(cfg->beta2, (double)cfg->step);
+    for (int sd = 0; sd < 2; ++sd) {
+        GemmArgs g{};
+        g.mode = GEMM_ADAMW; g.M = (int)(sd == 0 ? m : n); g.N = (int)q; g.ldo = q; g.status = &hdr->status;
+        g.adam = AdamwArgs{sd == 0 ? U : V, sd == 0 ? mU : mV, sd == 0 ? vU : vV, D(L.dF[sd]),
+                           cfg->lr, cfg->beta1, cfg->beta2, cfg->eps, cfg->weight_decay, bc1, bc2};
+        if (sd == 0) ISO_TRY(frame_gemm(s, F(L.gw4), L.Mp, F(L.sv4), Qp, L.Np, g));
+        else ISO_TRY(frame_gemm(s, F(L.gwt4), L.Np, F(L.su4), Qp, L.Mp, g));
+    }
+    // the polar retraction of each side: N = F^T dF + dF^T (F + dF) (F^T F = I),
+    // R = (I + N)^(-1/2) - I, E_F = dF + (F + dF) R
+    for (int sd = 0; sd < 2; ++sd) {
+        const long long Dp = sd == 0 ? L.Mp : L.Np, d = fr[sd].d;
+        SplitT st{};
+        st.f = fr[sd]; st.X = D(L.dF[sd]); st.Dp = Dp; st.Qp = Qp;
+        const dim3 grd((unsigned)(2 * Dp / 32), (unsigned)(Qp / 32));
+        st.mode = 4; st.out = F(L.na4);
+        FR_LAUNCH((k_fr_split_t<<<grd, dim3(32, 8), 0, s>>>(st)));
+        st.mode = 5; st.out = F(L.nb4);
+        FR_LAUNCH((k_fr_split_t<<<grd, dim3(32, 8), 0, s>>>(st)));
+        {
+            // contraction of 2 Dp: A = [F ; dF]^T read from segment 0, B = [dF ; F + dF]^T from segment 1
+            GemmArgs g{};
+            g.mode = GEMM_STORE_F32; g.C = F(L.nq); g.ldc = Qp; g.M = (int)Qp; g.N = (int)Qp; g.status = &hdr->status;
+            ISO_TRY(frame_gemm(s, F(L.na4), Qp, F(L.nb4), Qp, 2 * Dp, g));
+        }
+        NsBufs nb{D(L.ns_y), D(L.ns_z), D(L.ns_m), F(L.ns_y4), F(L.ns_z4), F(L.ns_m4), F(L.ns_t1),
+                  F(L.ns_t2), F(L.ns_t3)};
+        ISO_TRY(ns_root(s, sms, hdr, sd, F(L.nq), q, Qp, nb, ns_iters, F(L.r4)));
+        SplitR sr{};
+        sr.f = fr[sd]; sr.X = D(L.dF[sd]); sr.mode = 1; sr.out = F(L.xb4); sr.rows = d; sr.rows_p = Dp; sr.Lp = Qp;
+        FR_LAUNCH((k_fr_split_r<<<grid_of(Dp * Qp, sms), 256, 0, s>>>(sr)));
+        {
+            GemmArgs g{};
+            g.mode = GEMM_STORE_F32; g.C = F(L.p); g.ldc = Qp; g.M = (int)Dp; g.N = (int)Qp; g.status = &hdr->status;
+            ISO_TRY(frame_gemm(s, F(L.xb4), Dp, F(L.r4), Qp, Qp, g));
+        }
+        FR_LAUNCH((k_fr_motion<<<grid_of(d * q, sms), 256, 0, s>>>(D(L.dF[sd]), F(L.p), Qp, d, q)));
+        // the reconstruction's operand of this side ([E_U S_0 | U S_0] or [V + E_V | E_V])
+        sr.S0 = S0; sr.X = D(L.dF[sd]); sr.mode = sd == 0 ? 4 : 5; sr.out = F(sd == 0 ? L.a6 : L.b6);
+        sr.rows = d; sr.rows_p = Dp; sr.Lp = 2 * Qp;
+        FR_LAUNCH((k_fr_split_r<<<grid_of(Dp * 2 * Qp, sms), 256, 0, s>>>(sr)));
+    }
+    // F+ = F + E_F, then W+ = W + [E_U S_0 | U S_0] [V+ | E_V]^T
+    FR_LAUNCH((k_op_add<<<grid_of(m * q, sms), 256, 0, s>>>(U, D(L.dF[0]), m * q)));
+    FR_LAUNCH((k_op_add<<<grid_of(n * q, sms), 256, 0, s>>>(V, D(L.dF[1]), n * q)));
+    {
+        GemmArgs g{};
+        g.mode = GEMM_ADD_BASE; g.M = (int)m; g.N = (int)n; g.out = W_out->data; g.w0 = W->data; g.ldo = n;
+        g.out_dtype = W->dtype; g.status = &hdr->status;
+        ISO_TRY(frame_gemm(s, F(L.a6), L.Mp, F(L.b6), L.Np, 2 * Qp, g));
+    }
+    if (stats && stats->status) FR_LAUNCH((k_fr_status<<<1, 32, 0, s>>>(hdr, stats->status)));
     return ISO_OK;
 }
 

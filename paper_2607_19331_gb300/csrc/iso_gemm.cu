@@ -175,6 +175,22 @@ k_gemm_tf32(const __grid_constant__ CUtensorMap ta, const __grid_constant__ CUte
                 float4* dst = reinterpret_cast<float4*>(g.C + row * g.ldc + col0);
 #pragma unroll
                 for (int j = 0; j < 8; ++j) dst[j] = make_float4(v[4 * j], v[4 * j + 1], v[4 * j + 2], v[4 * j + 3]);
+            } else if (g.mode == GEMM_ADAMW) {
+                if (row < g.M) {
+                    const AdamwArgs& a = g.adam;
+#pragma unroll 4
+                    for (int j = 0; j < 32; ++j) {
+                        const int col = col0 + j;
+                        if (col >= g.N) break;
+                        const long long e = row * g.ldo + col;
+                        const double gr = (double)v[j];
+                        const double mm = a.beta1 * (double)a.m[e] + (1.0 - a.beta1) * gr;
+                        const double vv = a.beta2 * (double)a.v[e] + (1.0 - a.beta2) * gr * gr;
+                        a.m[e] = (float)mm;
+                        a.v[e] = (float)vv;
+                        a.dX[e] = -a.lr * a.wd * a.X[e] - (a.lr / a.bc1) * mm / (sqrt(vv / a.bc2) + a.eps);
+                    }
+                }
             } else if (row < g.M) {
                 if (g.out_dtype == ISO_BF16) {
                     const unsigned short* w = static_cast<const unsigned short*>(g.w0) + row * g.ldo;

@@ -33,7 +33,19 @@ constexpr int GEMM_THREADS = 128;
 
 enum GemmEpilogue : int32_t {
     GEMM_STORE_F32 = 0,   // C[row * ldc + col] = acc (the tile is inside C's padded extents)
-    GEMM_ADD_BASE = 1     // out[row * ldo + col] = W0[row * ldo + col] + acc for row < M, col < N
+    GEMM_ADD_BASE = 1,    // out[row * ldo + col] = W0[row * ldo + col] + acc for row < M, col < N
+    GEMM_ADAMW = 2        // acc is the gradient of the binary64 variable X (row < M, col < N, row
+                          // stride ldo): AdamW moments updated in place, the step X_bar - X stored
+};
+
+// AdamW on a binary64 variable in the product's epilogue (decoupled weight
+// decay, bias-corrected moments kept in binary32, arithmetic in binary64)
+struct AdamwArgs {
+    const double* X;      // the variable (read)
+    float* m;             // first moment (in place)
+    float* v;             // second moment (in place)
+    double* dX;           // out: X_bar - X = -lr wd X - lr / bc1 * m / (sqrt(v / bc2) + eps)
+    double lr, beta1, beta2, eps, wd, bc1, bc2;
 };
 
 struct GemmArgs {
@@ -50,6 +62,7 @@ struct GemmArgs {
     int32_t pad;
     const int32_t* skip;  // optional: the whole grid returns at once while *skip != 0
     int32_t* status;      // header status word for ISO_ERR_TIMEOUT
+    AdamwArgs adam;       // GEMM_ADAMW
 };
 
 __global__ void k_gemm_tf32(const __grid_constant__ CUtensorMap ta, const __grid_constant__ CUtensorMap tb,

@@ -16,6 +16,11 @@ def pytest_terminal_summary(terminalreporter, exitstatus, config):
     relative error for binary32 outputs, bfloat16 ulps for bfloat16 outputs,
     and the entries that needed the cancellation bound of parity_util."""
     tr = terminalreporter
+    opt = getattr(sys.modules.get("test_gpu_optimizer"), "WORST_OPT", None)
+    if opt:
+        tr.section("ISO-Optimizer step: worst error / derived bound")
+        for what, ratio in sorted(opt.items()):
+            tr.write_line(f"{what}: " + ", ".join(f"{k} {v:.3g}" for k, v in ratio.items()))
     frame = getattr(sys.modules.get("test_gpu_frame"), "WORST_FRAME", None)
     if frame:
         tr.section("frame-space merge: worst error / derived bound")

@@ -261,3 +261,38 @@ def test_gemm_argument_errors():
     assert L.iso_gemm_tf32(A, 32, B, 32, C, 128, 128, 128, 32, 32, 0, None) == _abi.ISO_ERR_SHAPE  # past lda
     assert L.iso_gemm_tf32(P(0x100004), 32, B, 32, C, 128, 128, 128, 32, 0, 0, None) == _abi.ISO_ERR_ALIGN
     assert L.iso_gemm_tf32(None, 32, B, 32, C, 128, 128, 128, 32, 0, 0, None) == _abi.ISO_ERR_ARG
+
+
+def test_opt_step_sizes_and_argument_errors():
+    # iso_opt_step: sizing and the checks made before anything is enqueued
+    L = _abi.lib()
+    b = ctypes.c_size_t()
+    assert L.iso_opt_workspace_size(3584, 18944, ctypes.byref(b)) == 0
+    assert 5e9 < b.value < 40e9
+    assert L.iso_opt_workspace_size(0, 5, ctypes.byref(b)) == _abi.ISO_ERR_ARG
+    P = ctypes.c_void_p
+    G = _arr(_fake(96, 64, dtype=_abi.ISO_F32, ptr=0x1000000))
+    W = _arr(_fake(96, 64, dtype=_abi.ISO_BF16, ptr=0x2000000))
+    O = _arr(_fake(96, 64, dtype=_abi.ISO_BF16, ptr=0x3000000))
+
+    def cfg(**kw):
+        d = dict(lr=1e-3, beta1=0.9, beta2=0.999, eps=1e-8, weight_decay=0.0, step=1, ns_iters=0, reserved=0)
+        d.update(kw)
+        return _abi.IsoAdamwCfg(**d)
+
+    def st(c=None, G_=G, W_=W, O_=O, wsb=1 << 30, U=0x100000, mU=0x500000):
+        c = cfg() if c is None else c
+        return L.iso_opt_step(P(U), P(0x200000), P(0x300000), G_, P(mU), P(0x600000), P(0x700000),
+                              P(0x800000), W_, O_, 96, 64, ctypes.byref(c), P(0x4000000), wsb, None, None)
+    assert st(G_=_arr(_fake(96, 65, dtype=_abi.ISO_F32, ptr=0x1000000))) == _abi.ISO_ERR_SHAPE
+    assert st(O_=_arr(_fake(96, 64, dtype=_abi.ISO_F32, ptr=0x3000000))) == _abi.ISO_ERR_DTYPE
+    assert st(O_=_arr(_fake(96, 64, dtype=_abi.ISO_BF16, ptr=0x2000010))) == _abi.ISO_ERR_ARG     # overlaps W
+    assert st(cfg(step=0)) == _abi.ISO_ERR_ARG
+    assert st(cfg(beta1=1.0)) == _abi.ISO_ERR_ARG
+    assert st(cfg(eps=0.0)) == _abi.ISO_ERR_ARG
+    assert st(cfg(lr=float("nan"))) == _abi.ISO_ERR_ARG
+    assert st(cfg(ns_iters=65)) == _abi.ISO_ERR_ARG
+    assert st(wsb=1024) == _abi.ISO_ERR_WORKSPACE
+    assert st(U=0x100004) == _abi.ISO_ERR_ALIGN
+    assert st(mU=0x500002) == _abi.ISO_ERR_ALIGN
+    assert st(U=0) == _abi.ISO_ERR_ARG
