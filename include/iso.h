@@ -320,10 +320,12 @@ int32_t iso_opt_workspace_size(int64_t m, int64_t n, size_t* bytes);
  *   W_out                  receives W + (U+ S0 V+^T - U S0 V^T); same dtype, may
  *                          coincide with W (each entry read and written by one
  *                          thread) but share no other byte with it
- * The retraction assumes U^T U = I (and V^T V = I) to the working precision.
- * Precision: the factor gradients and the retraction's products are three tf32
- * products per pair with binary32 accumulation; the AdamW arithmetic and the
- * frames are binary64.  stats->status (may be NULL) receives ISO_OK or
+ * The retraction takes polar(F_bar) = F_bar (F_bar^T F_bar)^(-1/2) with
+ * F_bar^T F_bar formed in binary64, so it also restores orthonormality lost
+ * to rounding in earlier steps.  Precision: the factor gradients and the
+ * retraction's remaining products are three tf32 products per pair with
+ * binary32 accumulation (about 2^-22 relative each); the AdamW arithmetic,
+ * F_bar^T F_bar and the frames are binary64.  stats->status (may be NULL) receives ISO_OK or
  * ISO_ERR_TIMEOUT.  Argument errors are returned before anything is enqueued. */
 int32_t iso_opt_step(double* U, double* V, const double* S0, const iso_tensor* G_W, float* mU, float* vU,
                      float* mV, float* vV, const iso_tensor* W, const iso_tensor* W_out, int64_t m, int64_t n,

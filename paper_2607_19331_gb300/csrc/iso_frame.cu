@@ -350,6 +350,51 @@ __global__ void __launch_bounds__(256) k_fr_ftdf(Frames f, const double* dots, i
         }
 }
 
+// N = (F + dF)^T (F + dF) - I in binary64, the polar retraction's argument
+// (any departure of F^T F from I included, so the retraction also restores
+// orthonormality lost to rounding); tiling as in k_fr_ftdf
+__global__ void __launch_bounds__(256) k_op_gram64(const double* F, const double* dF, long long d, long long q,
+                                                   double* N) {
+    __shared__ double sa[16][64], sb[16][64];
+    const long long k0 = (long long)blockIdx.y * 64, l0 = (long long)blockIdx.x * 64;
+    const int tx = threadIdx.x & 15, ty = threadIdx.x >> 4;
+    double acc[4][4];
+#pragma unroll
+    for (int a = 0; a < 4; ++a)
+#pragma unroll
+        for (int b = 0; b < 4; ++b) acc[a][b] = 0.0;
+    for (long long r0 = 0; r0 < d; r0 += 16) {
+        for (int e = threadIdx.x; e < 16 * 64; e += 256) {
+            const int rr = e >> 6, cc = e & 63;
+            const long long r = r0 + rr;
+            const long long ka = k0 + cc, lb = l0 + cc;
+            sa[rr][cc] = (r < d && ka < q) ? F[r * q + ka] + dF[r * q + ka] : 0.0;
+            sb[rr][cc] = (r < d && lb < q) ? F[r * q + lb] + dF[r * q + lb] : 0.0;
+        }
+        __syncthreads();
+#pragma unroll
+        for (int kk = 0; kk < 16; ++kk) {
+            double av[4], bv[4];
+#pragma unroll
+            for (int a = 0; a < 4; ++a) av[a] = sa[kk][ty * 4 + a];
+#pragma unroll
+            for (int b = 0; b < 4; ++b) bv[b] = sb[kk][tx * 4 + b];
+#pragma unroll
+            for (int a = 0; a < 4; ++a)
+#pragma unroll
+                for (int b = 0; b < 4; ++b) acc[a][b] = fma(av[a], bv[b], acc[a][b]);
+        }
+        __syncthreads();
+    }
+#pragma unroll
+    for (int a = 0; a < 4; ++a)
+#pragma unroll
+        for (int b = 0; b < 4; ++b) {
+            const long long k = k0 + ty * 4 + a, l = l0 + tx * 4 + b;
+            if (k < q && l < q) N[k * q + l] = acc[a][b] - (k == l ? 1.0 : 0.0);
+        }
+}
+
 // Split operands of an m x n bf16 / fp32 matrix G (row stride n): row-major
 // (rows Mp of 4 Np, element G[r, c]) or transposed (rows Np of 4 Mp, element
 // G[r, c] at row c, position r)
@@ -491,13 +536,14 @@ __global__ void __launch_bounds__(256) k_fr_xi(Frames f, const double* dots, con
     }
 }
 
-// ||N||_F^2 of N = xi^T xi (binary32, ld Qp), summed into the header
-__global__ void __launch_bounds__(256) k_fr_norm(const float* N, long long Qp, long long q, FrameHeader* h, int side) {
+// ||N||_F^2 of N = xi^T xi (binary32, ld Qp; or binary64, ld q), summed into the header
+__global__ void __launch_bounds__(256) k_fr_norm(const float* N, const double* N64, long long Qp, long long q,
+                                                 FrameHeader* h, int side) {
     __shared__ double red[32];
     double acc = 0.0;
     for (long long e = (long long)blockIdx.x * blockDim.x + threadIdx.x; e < q * q; e += (long long)gridDim.x * blockDim.x) {
         const long long r = e / q, c = e - r * q;
-        const double v = N[r * Qp + c];
+        const double v = N64 ? N64[e] : (double)N[r * Qp + c];
         acc += v * v;
     }
     acc = block_sum(acc, red);
@@ -511,7 +557,8 @@ __global__ void __launch_bounds__(256) k_fr_norm(const float* N, long long Qp, l
 // build an asymmetric component from one iteration to the next.  Reading
 // both tiles before writing either makes the update safe in place.
 struct NsArgs {
-    const float* N;     // init: N = xi^T xi (ld Qp)
+    const float* N;     // init: N = xi^T xi (binary32, ld Qp), unless N64 is given
+    const double* N64;  // init: N in binary64 (ld q)
     const float* T1;    // m: z y;  update: y m
     const float* T2;    // update: m z
     double* y;
@@ -544,7 +591,8 @@ __global__ void __launch_bounds__(256) k_fr_ns_init(NsArgs a) {
     auto f = [&](long long r, long long c) -> double {
         if (r >= a.q || c >= a.q) return 0.0;
         const double id = r == c ? 1.0 : 0.0;
-        return (id + (double)a.N[r * a.Qp + c]) / cs - id;
+        const double nv = a.N64 ? a.N64[r * a.q + c] : (double)a.N[r * a.Qp + c];
+        return (id + nv) / cs - id;
     };
     for (int y = threadIdx.y; y < 32; y += 8) {
         ta[y][threadIdx.x] = f(r0 + y, c0 + threadIdx.x);
@@ -746,7 +794,7 @@ int frame_gemm(cudaStream_t s, const float* A, long long a_rows, const float* B,
 
 struct OptLayout {
     long long m, n, q, Mp, Np, Qp, Dmax;
-    size_t hdr, gw4, gwt4, su4, sv4, dF[2], na4, nb4, nq, xb4, r4, p, a6, b6;
+    size_t hdr, gw4, gwt4, su4, sv4, dF[2], n64, xb4, r4, p, a6, b6;
     size_t ns_y, ns_z, ns_m, ns_y4, ns_z4, ns_m4, ns_t1, ns_t2, ns_t3, total;
 };
 
@@ -765,9 +813,7 @@ OptLayout opt_layout(long long m, long long n) {
     L.sv4 = take(sizeof(float) * Qp * 4 * L.Np);        // (V S_0)^T
     L.dF[0] = take(sizeof(double) * m * q);             // U_bar - U, later E_U
     L.dF[1] = take(sizeof(double) * n * q);             // V_bar - V, later E_V
-    L.na4 = take(sizeof(float) * Qp * 4 * 2 * L.Dmax);  // [F ; dF]^T
-    L.nb4 = take(sizeof(float) * Qp * 4 * 2 * L.Dmax);  // [dF ; F + dF]^T
-    L.nq = take(sizeof(float) * Qp * Qp);
+    L.n64 = take(sizeof(double) * q * q);               // (F + dF)^T (F + dF) - I
     L.xb4 = take(sizeof(float) * L.Dmax * 4 * Qp);      // F + dF
     L.r4 = take(sizeof(float) * Qp * 4 * Qp);
     L.p = take(sizeof(float) * L.Dmax * Qp);
@@ -800,11 +846,11 @@ struct NsBufs {
 // by the difference-form Newton-Schulz iteration (k_fr_ns_*), written as
 // the split operand R4 (Qp rows of 4 Qp; R is symmetric, so it serves as B
 // of (F_0 + X) R).  Header slot `side` holds its scaling and state.
-int ns_root(cudaStream_t s, int sms, FrameHeader* hdr, int side, const float* Nq, long long q, long long Qp,
-            const NsBufs& b, int ns_iters, float* R4) {
-    FR_LAUNCH((k_fr_norm<<<grid_of(q * q, sms), 256, 0, s>>>(Nq, Qp, q, hdr, side)));
+int ns_root(cudaStream_t s, int sms, FrameHeader* hdr, int side, const float* Nq, const double* N64, long long q,
+            long long Qp, const NsBufs& b, int ns_iters, float* R4) {
+    FR_LAUNCH((k_fr_norm<<<grid_of(q * q, sms), 256, 0, s>>>(Nq, N64, Qp, q, hdr, side)));
     NsArgs na{};
-    na.N = Nq; na.y = b.y; na.z = b.z; na.m = b.m; na.h = hdr;
+    na.N = Nq; na.N64 = N64; na.y = b.y; na.z = b.z; na.m = b.m; na.h = hdr;
     na.q = q; na.Qp = Qp; na.side = side;
     const dim3 tiles((unsigned)((q + 31) / 32), (unsigned)((q + 31) / 32)), tb(32, 8);
     FR_LAUNCH((k_fr_ns_init<<<tiles, tb, 0, s>>>(na)));
@@ -988,7 +1034,7 @@ int32_t iso_frame_merge(const double* U0, const double* S0, const double* Vt0, c
         {
             NsBufs nb{D(L.ns_y), D(L.ns_z), D(L.ns_m), F(L.ns_y4), F(L.ns_z4), F(L.ns_m4), F(L.ns_t1),
                       F(L.ns_t2), F(L.ns_t3)};
-            ISO_TRY(ns_root(s, sms, hdr, sd, F(L.nq[sd]), q, Qp, nb, ns_iters, F(L.y4[sd])));
+            ISO_TRY(ns_root(s, sms, hdr, sd, F(L.nq[sd]), nullptr, q, Qp, nb, ns_iters, F(L.y4[sd])));
         }
         sr.mode = 1; sr.X = D(L.xi[sd]); sr.out = F(L.fr4[sd]); sr.rows = d; sr.rows_p = Dp; sr.Lp = Qp;
         FR_LAUNCH((k_fr_split_r<<<grid_of(Dp * Qp, sms), 256, 0, s>>>(sr)));
@@ -1092,26 +1138,15 @@ int32_t iso_opt_step(double* U, double* V, const double* S0, const iso_tensor* G
         if (sd == 0) ISO_TRY(frame_gemm(s, F(L.gw4), L.Mp, F(L.sv4), Qp, L.Np, g));
         else ISO_TRY(frame_gemm(s, F(L.gwt4), L.Np, F(L.su4), Qp, L.Mp, g));
     }
-    // the polar retraction of each side: N = F^T dF + dF^T (F + dF) (F^T F = I),
-    // R = (I + N)^(-1/2) - I, E_F = dF + (F + dF) R
+    // the polar retraction of each side: N = (F + dF)^T (F + dF) - I in
+    // binary64, R = (I + N)^(-1/2) - I, E_F = dF + (F + dF) R
     for (int sd = 0; sd < 2; ++sd) {
         const long long Dp = sd == 0 ? L.Mp : L.Np, d = fr[sd].d;
-        SplitT st{};
-        st.f = fr[sd]; st.X = D(L.dF[sd]); st.Dp = Dp; st.Qp = Qp;
-        const dim3 grd((unsigned)(2 * Dp / 32), (unsigned)(Qp / 32));
-        st.mode = 4; st.out = F(L.na4);
-        FR_LAUNCH((k_fr_split_t<<<grd, dim3(32, 8), 0, s>>>(st)));
-        st.mode = 5; st.out = F(L.nb4);
-        FR_LAUNCH((k_fr_split_t<<<grd, dim3(32, 8), 0, s>>>(st)));
-        {
-            // contraction of 2 Dp: A = [F ; dF]^T read from segment 0, B = [dF ; F + dF]^T from segment 1
-            GemmArgs g{};
-            g.mode = GEMM_STORE_F32; g.C = F(L.nq); g.ldc = Qp; g.M = (int)Qp; g.N = (int)Qp; g.status = &hdr->status;
-            ISO_TRY(frame_gemm(s, F(L.na4), Qp, F(L.nb4), Qp, 2 * Dp, g));
-        }
+        FR_LAUNCH((k_op_gram64<<<dim3((unsigned)((q + 63) / 64), (unsigned)((q + 63) / 64)), 256, 0, s>>>(
+            sd == 0 ? U : V, D(L.dF[sd]), d, q, D(L.n64))));
         NsBufs nb{D(L.ns_y), D(L.ns_z), D(L.ns_m), F(L.ns_y4), F(L.ns_z4), F(L.ns_m4), F(L.ns_t1),
                   F(L.ns_t2), F(L.ns_t3)};
-        ISO_TRY(ns_root(s, sms, hdr, sd, F(L.nq), q, Qp, nb, ns_iters, F(L.r4)));
+        ISO_TRY(ns_root(s, sms, hdr, sd, nullptr, D(L.n64), q, Qp, nb, ns_iters, F(L.r4)));
         SplitR sr{};
         sr.f = fr[sd]; sr.X = D(L.dF[sd]); sr.mode = 1; sr.out = F(L.xb4); sr.rows = d; sr.rows_p = Dp; sr.Lp = Qp;
         FR_LAUNCH((k_fr_split_r<<<grid_of(Dp * Qp, sms), 256, 0, s>>>(sr)));
