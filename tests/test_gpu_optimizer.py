@@ -12,8 +12,12 @@ W+ = W + (U+ S0 V+^T - U S0 V^T).  Bounds, derived from that arithmetic:
 * the second moment within (1 - b2)(2 |g| dg + dg^2) plus its rounding;
 * the frames: ||U+ - U+_oracle||_F within 1.5 ||d step||_F plus the
   retraction's products, where d step is the AdamW step's change over the
-  gradient interval g +- dg (evaluated with the oracle's AdamW); U+ has
-  orthonormal columns to 1e-12;
+  gradient interval g +- dg (evaluated with the oracle's AdamW);
+  |U+^T U+ - I| within 2 |U_bar|^T (eps |U_bar| |R|), R = (U_bar^T
+  U_bar)^(-1/2) - I: the retraction's argument U_bar^T U_bar is binary64 and
+  only the product U_bar R is tf32 x 3 (the departure is of the order of the
+  step times 1e-6 and does not accumulate over steps: each retraction is
+  built from the exact U_bar^T U_bar);
 * W+ within one bf16 ulp of the oracle's value (bf16 weights), or the change
   the frames' own differences and the products' rounding explain (fp32).
 """
@@ -121,8 +125,17 @@ def _run_and_check(m, n, t, wd, wdtype, lr=1e-3, b1=0.9, b2=0.999, eps=1e-8, gsc
         tol_F = 1.5 * np.linalg.norm(d_step) + 8 * _eps(2 * max(m, n)) * np.linalg.norm(dF) + 1e-13
         ratio[side] = float(np.linalg.norm(F_gpu - r[side]) / tol_F)
         assert ratio[side] <= 1.0, (what, side, ratio)
-        ortho = np.abs(F_gpu.T @ F_gpu - np.eye(q)).max()
-        assert ortho <= 1e-12, (what, side, ortho)
+        # orthonormality: the retraction's argument is binary64, its product
+        # P = F_bar R is tf32 x 3, so F+^T F+ - I is bounded by
+        # 2 |F_bar|^T (eps |F_bar| |R|) with R = (F_bar^T F_bar)^(-1/2) - I
+        Fb = r[side + "_bar"]
+        w, E = np.linalg.eigh(Fb.T @ Fb)
+        R = (E / np.sqrt(w)) @ E.T - np.eye(q)
+        ortho_bound = 2 * np.abs(Fb).T @ (_eps(q) * (np.abs(Fb) @ np.abs(R))) + 1e-13
+        ortho = np.abs(F_gpu.T @ F_gpu - np.eye(q))
+        ratio["ortho" + side] = float(np.max(ortho / ortho_bound))
+        assert ratio["ortho" + side] <= 1.0, (what, side, ratio)
+        ratio["ortho" + side + "_abs"] = float(ortho.max())
     # weights: the oracle's W+ shifted by the stored W's own rounding
     W_store = W_t.double().numpy()
     want = r["W"] + (W_store - (U * S) @ V.T)
@@ -139,9 +152,11 @@ def _run_and_check(m, n, t, wd, wdtype, lr=1e-3, b1=0.9, b2=0.999, eps=1e-8, gsc
         bound = bound + 2 * U32 * np.abs(want)
     ratio["W"] = float(np.max(np.abs(got - want) / bound))
     assert ratio["W"] <= 1.0, (what, ratio)
-    # the fixed spectrum of the new frames' weights
+    # the fixed spectrum of the new frames' weights, to first order in their
+    # departure from orthonormality
     s_new = np.linalg.svd((U_g * S) @ V_g.T, compute_uv=False)
-    np.testing.assert_allclose(s_new, S, rtol=0, atol=1e-12)
+    dev = np.linalg.norm(U_g.T @ U_g - np.eye(q), 2) + np.linalg.norm(V_g.T @ V_g - np.eye(q), 2)
+    np.testing.assert_allclose(s_new, S, rtol=0, atol=2 * dev * S.max() + 1e-13)
     WORST_OPT[what] = ratio
 
 
