@@ -100,9 +100,18 @@ __global__ void __launch_bounds__(TPB) k_apply(Plan P) {
     const int lane = threadIdx.x & 31;
     const long long W = (long long)gridDim.x * WPB;
     const long long wid = (long long)blockIdx.x * WPB + (threadIdx.x >> 5);
-    const long long per = (P.n_tiles + W - 1) / W;
-    const long long beg = wid * per;
-    const long long end = (beg + per < P.n_tiles) ? beg + per : P.n_tiles;
+    // round-robin tiles (all warps sweep one window together) or one range per warp
+    long long beg, end, step;
+    if (PASS_INTERLEAVE) {
+        beg = wid;
+        end = P.n_tiles;
+        step = W;
+    } else {
+        const long long per = (P.n_tiles + W - 1) / W;
+        beg = wid * per;
+        end = (beg + per < P.n_tiles) ? beg + per : P.n_tiles;
+        step = 1;
+    }
     if (beg >= end) return;
     const bool obf = sizeof(BT) == 2;
     int t = tensor_of_tile(P.tens, P.n_tensors, beg);
@@ -125,15 +134,15 @@ __global__ void __launch_bounds__(TPB) k_apply(Plan P) {
         float k1_a = 1.0f;
         bool k1_mask = true;
         unsigned long long k1_thr = 0;
-        for (long long g = beg; g < end; ++g) {
-            // prefetch tile g + 1
-            if (g + 1 < end) {
-                while (g + 1 >= nt_end) {
+        for (long long g = beg; g < end; g += step) {
+            // prefetch the warp's next tile
+            if (g + step < end) {
+                while (g + step >= nt_end) {
                     ++nt;
                     nt_end = P.tens[nt].tile_base + (P.tens[nt].numel + TILE - 1) / TILE;
                 }
                 const TensorDesc& nd = P.tens[nt];
-                nxt.load(P.xptr[nt], nd.base, (g + 1 - nd.tile_base) * TILE, nd.numel, lane);
+                nxt.load(P.xptr[nt], nd.base, (g + step - nd.tile_base) * TILE, nd.numel, lane);
             }
             if (g >= t_end || g == beg) {
                 while (g >= t_end) { ++t; t_end = P.tens[t].tile_base + (P.tens[t].numel + TILE - 1) / TILE; }

@@ -9,6 +9,13 @@ namespace iso {
 
 
 
+// the streaming passes over (expert, tile) items deal them round-robin over
+// the warps (1) or give each warp one contiguous range (0)
+#ifndef ISO_PASS_INTERLEAVE
+#define ISO_PASS_INTERLEAVE 1
+#endif
+constexpr bool PASS_INTERLEAVE = ISO_PASS_INTERLEAVE != 0;
+
 // select (TENSOR / GLOBAL scope)
 constexpr int COUNT_BLOCKS_PER_SM = 2;      // k_count: resident blocks of TPB threads per SM
 __global__ void k_init_units(Plan P, long long global_n);

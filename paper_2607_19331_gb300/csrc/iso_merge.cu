@@ -353,15 +353,28 @@ __device__ __forceinline__ uint32_t fast_bits(const int (&T)[KC], int K, const f
     return bits;
 }
 
-// the warp's contiguous tile range
-struct WarpRange { long long beg, end; };
+// the warp's tiles: beg, beg + step, ... below end -- dealt round-robin over
+// the warps (all warps sweep one window of the tensors together, for DRAM
+// page locality) or one contiguous range per warp
+struct WarpRange {
+    long long beg, end, step;
+    __device__ __forceinline__ long long count() const { return beg < end ? (end - beg + step - 1) / step : 0; }
+    __device__ __forceinline__ long long tile(long long j) const { return beg + j * step; }
+};
 __device__ __forceinline__ WarpRange warp_range(const Plan& P) {
     const long long W = (long long)gridDim.x * WPB;
     const long long wid = (long long)blockIdx.x * WPB + (threadIdx.x >> 5);
-    const long long per = (P.n_tiles + W - 1) / W;
     WarpRange r;
-    r.beg = wid * per;
-    r.end = (r.beg + per < P.n_tiles) ? r.beg + per : P.n_tiles;
+    if (PASS_INTERLEAVE) {
+        r.beg = wid;
+        r.end = P.n_tiles;
+        r.step = W;
+    } else {
+        const long long per = (P.n_tiles + W - 1) / W;
+        r.beg = wid * per;
+        r.end = (r.beg + per < P.n_tiles) ? r.beg + per : P.n_tiles;
+        r.step = 1;
+    }
     return r;
 }
 
@@ -517,14 +530,14 @@ __global__ void __launch_bounds__(TPB, merge_blocks_per_sm(KC, OPF)) k_merge(Pla
     if (wr.beg >= wr.end) return;
     char* ring = s_stage + warp * D * G::BYTES;
     const uint32_t ring_s = (uint32_t)__cvta_generic_to_shared(ring);
-    const long long NS = (wr.end - wr.beg) * SPT;
+    const long long NS = wr.count() * SPT;
     constexpr bool SP = merge_blocks_per_sm(KC, OPF) == 2 && KC >= 8;
     __shared__ const void* s_xs[WPB][KC];
     IssueCursor<KC, SP> ic;
     if constexpr (SP) ic.xs = s_xs[warp];
 #pragma unroll
     for (int p = 0; p < D - 1; ++p) {
-        if (p < NS) issue_step<XT, BT, KC, SP>(P, K, ic, wr.beg + p / SPT, p % SPT, ring_s + p * G::BYTES, lane);
+        if (p < NS) issue_step<XT, BT, KC, SP>(P, K, ic, wr.tile(p / SPT), p % SPT, ring_s + p * G::BYTES, lane);
         cp_async_commit();
     }
     int t = tensor_of_tile(P.tens, P.n_tensors, wr.beg);
@@ -543,7 +556,7 @@ __global__ void __launch_bounds__(TPB, merge_blocks_per_sm(KC, OPF)) k_merge(Pla
     const TensorDesc* dp = nullptr;
 #pragma unroll 1
     for (long long i = 0; i < NS; ++i) {
-        const long long g = wr.beg + i / SPT;
+        const long long g = wr.tile(i / SPT);
         const int s = (int)(i % SPT);
         if (s == 0) {
             if (g >= t_end) {
@@ -586,7 +599,7 @@ __global__ void __launch_bounds__(TPB, merge_blocks_per_sm(KC, OPF)) k_merge(Pla
             return __uint_as_float((j & 1) ? (w & 0xFFFF0000u) : (w << 16));
         };
         const long long ni = i + D - 1;
-        if (ni < NS) issue_step<XT, BT, KC, SP>(P, K, ic, wr.beg + ni / SPT, (int)(ni % SPT), ring_s + (int)(ni % D) * G::BYTES, lane);
+        if (ni < NS) issue_step<XT, BT, KC, SP>(P, K, ic, wr.tile(ni / SPT), (int)(ni % SPT), ring_s + (int)(ni % D) * G::BYTES, lane);
         cp_async_commit();
         const long long e = e0 + (long long)s * (32 * E) + lane * E;
         if (e >= n) continue;
@@ -641,14 +654,14 @@ __global__ void __launch_bounds__(TPB, gram_blocks_per_sm(KC)) k_gramk(Plan P) {
     if (wr.beg >= wr.end) return;
     char* ring = s_stage + warp * D * G::BYTES;
     const uint32_t ring_s = (uint32_t)__cvta_generic_to_shared(ring);
-    const long long NS = (wr.end - wr.beg) * SPT;
+    const long long NS = wr.count() * SPT;
     constexpr bool SP = KC >= 8;   // eight experts: their pointers in shared memory (two blocks per SM)
     IssueCursor<KC, SP> ic;
     __shared__ const void* s_xs[WPB][KC];
     if constexpr (SP) ic.xs = s_xs[warp];
 #pragma unroll
     for (int p = 0; p < D - 1; ++p) {
-        if (p < NS) issue_step<XT, BT, KC, SP, CK>(P, K, ic, wr.beg + p / SPT, p % SPT, ring_s + p * G::BYTES, lane);
+        if (p < NS) issue_step<XT, BT, KC, SP, CK>(P, K, ic, wr.tile(p / SPT), p % SPT, ring_s + p * G::BYTES, lane);
         cp_async_commit();
     }
     int t = tensor_of_tile(P.tens, P.n_tensors, wr.beg);
@@ -677,7 +690,7 @@ __global__ void __launch_bounds__(TPB, gram_blocks_per_sm(KC)) k_gramk(Plan P) {
     float acc[NP];
 #pragma unroll 1
     for (long long i = 0; i < NS; ++i) {
-        const long long g = wr.beg + i / SPT;
+        const long long g = wr.tile(i / SPT);
         const int s = (int)(i % SPT);
         if (s == 0) {
             if (g >= t_end) {
@@ -712,7 +725,7 @@ __global__ void __launch_bounds__(TPB, gram_blocks_per_sm(KC)) k_gramk(Plan P) {
             return __uint_as_float((j & 1) ? (w & 0xFFFF0000u) : (w << 16));
         };
         const long long ni = i + D - 1;
-        if (ni < NS) issue_step<XT, BT, KC, SP, CK>(P, K, ic, wr.beg + ni / SPT, (int)(ni % SPT), ring_s + (int)(ni % D) * G::BYTES, lane);
+        if (ni < NS) issue_step<XT, BT, KC, SP, CK>(P, K, ic, wr.tile(ni / SPT), (int)(ni % SPT), ring_s + (int)(ni % D) * G::BYTES, lane);
         cp_async_commit();
         const long long e = e0 + (long long)s * (32 * E) + lane * E;
         if (active && e < n) {

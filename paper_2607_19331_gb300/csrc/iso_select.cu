@@ -527,19 +527,23 @@ __global__ void __launch_bounds__(CS_TPB, 4) k_csample(Plan P) {
 // or a band key, checked when the band keys are copied; lo itself is a sampled
 // key, so a non-finite lo is a band key of its own unit.
 
-// consecutive items of one (expert, tensor) that the count pass visits
+// consecutive items of one (expert, tensor) that the count pass visits (with
+// round-robin items, one item)
 struct CountRun {
     uint32_t it0, end;       // items [it0, end), end clipped to the warp's range
     uint32_t e0;             // tensor entry of item it0's first element
     uint32_t n;              // tensor entries
     uint32_t rec;            // index of item it0 in the per-(expert, tile) arrays
+    uint32_t left0;          // this warp's items of the unit from it0 on
     const void* xp;
     const void* bp;
     Unit* U;
 };
 
-// the first counted run at or after item it (< end); false if there is none
-__device__ __forceinline__ bool count_run_at(const Plan& P, uint32_t it, uint32_t end, CountRun& r) {
+// the first counted item at or after item it (< end) in steps of `step`: the
+// run of its (expert, tensor) with step 1, the item alone otherwise; false if
+// there is none
+__device__ __forceinline__ bool count_run_at(const Plan& P, uint32_t it, uint32_t end, uint32_t step, CountRun& r) {
     while (it < end) {
         Cursor c;
         cursor_at(P, it, c);
@@ -548,7 +552,8 @@ __device__ __forceinline__ bool count_run_at(const Plan& P, uint32_t it, uint32_
         if (U) {
             const TensorDesc& d = P.tens[c.t];
             r.it0 = it;
-            r.end = re;
+            r.end = step == 1 ? re : it + 1;
+            r.left0 = (re - it + step - 1) / step;
             r.e0 = (uint32_t)(c.g - d.tile_base) * TILE;
             r.n = (uint32_t)d.numel;
             r.rec = (uint32_t)((long long)c.i * P.n_tiles + c.g);
@@ -557,7 +562,7 @@ __device__ __forceinline__ bool count_run_at(const Plan& P, uint32_t it, uint32_
             r.U = U;
             return true;
         }
-        it = re;
+        it += (re - it + step - 1) / step * step;   // the warp's first item past the run
     }
     return false;
 }
@@ -571,14 +576,22 @@ __global__ void __launch_bounds__(TPB, COUNT_BLOCKS_PER_SM) k_count(Plan P) {
     const uint32_t W = gridDim.x * WPB;
     const uint32_t wid = blockIdx.x * WPB + warp;
     const uint32_t items = (uint32_t)(P.K * P.n_tiles);
-    const uint32_t per = (items + W - 1) / W;
-    const uint32_t beg = wid * per;
-    const uint32_t end = min(items, beg + per);
+    uint32_t beg, end, step;
+    if (PASS_INTERLEAVE) {
+        beg = wid;
+        end = items;
+        step = W;
+    } else {
+        const uint32_t per = (items + W - 1) / W;
+        beg = wid * per;
+        end = min(items, beg + per);
+        step = 1;
+    }
     if (beg >= end) return;
     const unsigned FULL = 0xFFFFFFFFu;
 
     CountRun r;
-    if (!count_run_at(P, beg, end, r)) return;
+    if (!count_run_at(P, beg, end, step, r)) return;
 
     // per-unit accumulators (warp-uniform) and the candidate chunk
     Unit* au = nullptr;
@@ -699,7 +712,7 @@ __global__ void __launch_bounds__(TPB, COUNT_BLOCKS_PER_SM) k_count(Plan P) {
             unsigned long long start = 0;
             uint32_t req = 0;
             if (lane == 0) {
-                const uint32_t left = rr.end - it;
+                const uint32_t left = rr.left0 - (it - rr.it0);   // this warp's items of the unit still to count
                 const unsigned long long want = (unsigned long long)t_int * (unsigned long long)left;
                 req = (uint32_t)max((unsigned long long)t_int, min((unsigned long long)CHUNK_MAX, want));
                 start = atomicAdd(&au->n_alloc, (unsigned long long)req);
@@ -750,7 +763,7 @@ __global__ void __launch_bounds__(TPB, COUNT_BLOCKS_PER_SM) k_count(Plan P) {
         CountRun r2 = r;
         bool more = true;
         if (it2 >= r.end) {
-            more = count_run_at(P, r.end, end, r2);
+            more = count_run_at(P, step == 1 ? r.end : it + step, end, step, r2);
             it2 = r2.it0;
         }
         count_tile(r, it, more, r2, it2);
