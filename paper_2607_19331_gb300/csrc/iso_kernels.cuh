@@ -10,9 +10,12 @@ namespace iso {
 
 
 // the streaming passes over (expert, tile) items deal them round-robin over
-// the warps (1) or give each warp one contiguous range (0)
+// the warps (1) or give each warp one contiguous range (0).  Contiguous ranges
+// measured faster for these passes on the 7B K = 8 merges (round-robin: every
+// warp visits every unit, and the warps flush a unit's counters together);
+// the fused K = 1 pass takes round-robin tiles (FUSED_INTERLEAVE)
 #ifndef ISO_PASS_INTERLEAVE
-#define ISO_PASS_INTERLEAVE 1
+#define ISO_PASS_INTERLEAVE 0
 #endif
 constexpr bool PASS_INTERLEAVE = ISO_PASS_INTERLEAVE != 0;
 
