@@ -239,6 +239,55 @@ int32_t iso_update_noalloc(const iso_tensor* theta_0, const iso_tensor* update, 
                            const iso_tensor* out, int32_t n_tensors, const iso_merge_cfg* cfg,
                            const iso_merge_stats* stats, void* stream);
 
+/* ---- The K = 1 update of a parameter set held in host memory --------------
+ *
+ * The update of iso_update (same operation, same configuration, same results
+ * bit for bit) for tensors that live in host memory: a model on the host that
+ * is fine-tuned, merged or corrected on the GPU and read back.  The paper has
+ * no counterpart; the call is an interface of this library.
+ *
+ * The tensor list is cut into groups of consecutive tensors of about
+ * group_bytes each (theta_0 + update + out bytes; a GLOBAL-scope TopKMask,
+ * one unit over every tensor, makes one group of the whole list).  Groups go
+ * through two device slots (one when the list forms one group) of the
+ * caller's staging buffer in a pipeline over
+ * three caller streams: streams[0] copies a group's theta_0 and update in,
+ * streams[1] runs iso_update on it, streams[2] copies its out back, so the
+ * copies of one group overlap the update of the next.  Tensors whose host
+ * copies follow one another in ascending order are moved by one copy (inputs
+ * may have gaps below 4096 bytes between them, which are read but not used;
+ * outputs only exactly adjacent runs, so no host byte outside an out tensor
+ * is written).
+ *
+ *   theta_0, update, out   host descriptors (16-byte aligned like every
+ *                          tensor); the overlap rules of iso_update apply to
+ *                          them.  Page-locked host memory (cudaHostAlloc or
+ *                          cudaHostRegister) lets the copies run
+ *                          asynchronously; with pageable memory the runtime
+ *                          makes them synchronous and the pipeline serialises.
+ *   staging                device buffer, 256-byte aligned, of at least the
+ *                          size iso_update_host_staging_size returns for the
+ *                          same descriptors, configuration and group_bytes;
+ *                          it holds the two slots, the update's workspace
+ *                          and a per-group status array.
+ *   stats                  device-side outputs as for iso_update (units, gram
+ *                          and coef for the whole list; status combined over
+ *                          the groups: the first group's error that is not
+ *                          ISO_OK).
+ *   streams                three CUDA streams (h2d, compute, d2h); they may
+ *                          be one and the same stream (no overlap).
+ * The call enqueues and returns.  The whole call has finished, out written
+ * in host memory included, once streams[1] reaches the point where the call
+ * returned.  Argument errors return before anything is enqueued; a CUDA error
+ * while enqueueing returns ISO_ERR_CUDA with earlier groups enqueued. */
+int32_t iso_update_host_staging_size(const iso_tensor* theta_0, const iso_tensor* update,
+                                     const iso_tensor* out, int32_t n_tensors, const iso_merge_cfg* cfg,
+                                     size_t group_bytes, size_t* bytes);
+int32_t iso_update_host(const iso_tensor* theta_0, const iso_tensor* update, int32_t update_is_delta,
+                        const iso_tensor* out, int32_t n_tensors, const iso_merge_cfg* cfg,
+                        size_t group_bytes, void* staging, size_t staging_bytes,
+                        const iso_merge_stats* stats, void* const* streams);
+
 /* ---- Frame-space ISO-Merger of one weight matrix (App. E) ----------------
  *
  * The paper's merge of K experts fine-tuned from one base, per 2-D weight

@@ -86,6 +86,10 @@ PROTOTYPES = [
                         ctypes.POINTER(IsoMergeStats), P]),
     ("iso_update_noalloc", I32, [PT, PT, I32, PT, I32, ctypes.POINTER(IsoMergeCfg),
                                  ctypes.POINTER(IsoMergeStats), P]),
+    ("iso_update_host_staging_size", I32, [PT, PT, PT, I32, ctypes.POINTER(IsoMergeCfg), SZ,
+                                           ctypes.POINTER(SZ)]),
+    ("iso_update_host", I32, [PT, PT, I32, PT, I32, ctypes.POINTER(IsoMergeCfg), SZ, P, SZ,
+                              ctypes.POINTER(IsoMergeStats), ctypes.POINTER(P)]),
     ("iso_frame_workspace_size", I32, [I64, I64, I32, ctypes.POINTER(SZ)]),
     ("iso_frame_merge", I32, [P, P, P, P, P, I32, I64, I64, PT, PT, ctypes.POINTER(IsoFrameCfg), P, SZ,
                               ctypes.POINTER(IsoMergeStats), P]),

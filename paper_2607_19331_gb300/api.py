@@ -229,29 +229,59 @@ def iso_update(theta_0: List[torch.Tensor], update: List[torch.Tensor], op="iso"
     return iso_merge(theta_0, [update], op=op, experts_are_deltas=update_is_delta, **kw)
 
 
-class HostStaging:
-    """End-to-end use from host memory: pinned host inputs are copied to the
-    device, the update runs through iso_update, and the result is copied back
-    into pinned host memory."""
+def iso_update_host_staging_size(theta_0, update, out, op="iso", density=0.05, scope="tensor",
+                                 block=(128, 128), lam=1.0, ridge=1e-12, c_min=0.0, c_max=1.5,
+                                 mask_1d=True, eps_act=1e-5, group_bytes=2 << 30) -> int:
+    cfg = merge_cfg(op, density, scope, block, lam, ridge, c_min, c_max, mask_1d, eps_act)
+    nb = ctypes.c_size_t(0)
+    check(lib().iso_update_host_staging_size(describe(theta_0), describe(update), describe(out),
+                                              len(theta_0), ctypes.byref(cfg), int(group_bytes),
+                                              ctypes.byref(nb)), "iso_update_host_staging_size")
+    return int(nb.value)
 
-    def __init__(self, theta_0_host, update_host, device="cuda"):
+
+class HostUpdate:
+    """The K = 1 update of tensors in host memory (iso_update_host): groups of
+    tensors are copied in, updated and copied back in a pipeline over three
+    CUDA streams.  Host tensors should be page-locked (pin_memory) for the
+    copies to overlap the update; out may be the theta_0 tensors themselves."""
+
+    def __init__(self, device="cuda", group_bytes=2 << 30):
         self.dev = torch.device(device)
-        self.theta_0 = [torch.empty(t.shape, dtype=t.dtype, device=self.dev) for t in theta_0_host]
-        self.update = [torch.empty(t.shape, dtype=t.dtype, device=self.dev) for t in update_host]
-        self.out = [torch.empty(t.shape, dtype=t.dtype, device=self.dev) for t in theta_0_host]
-        self.out_host = [torch.empty(t.shape, dtype=t.dtype, pin_memory=True) for t in theta_0_host]
-        self.h2d_bytes = sum(t.numel() * t.element_size() for t in list(theta_0_host) + list(update_host))
-        self.d2h_bytes = sum(t.numel() * t.element_size() for t in self.out_host)
+        self.group_bytes = int(group_bytes)
+        self.streams = [torch.cuda.Stream(self.dev) for _ in range(3)]
+        self.ws = Workspace(self.dev)
+        self.h2d_bytes = self.d2h_bytes = 0
 
-    def run(self, theta_0_host, update_host, **kw):
-        for d, h in zip(self.theta_0, theta_0_host):
-            d.copy_(h, non_blocking=True)
-        for d, h in zip(self.update, update_host):
-            d.copy_(h, non_blocking=True)
-        iso_update(self.theta_0, self.update, out=self.out, **kw)
-        for h, d in zip(self.out_host, self.out):
-            h.copy_(d, non_blocking=True)
-        return self.out_host
+    def run(self, theta_0, update, out=None, op="iso", update_is_delta=False, density=0.05,
+            scope="tensor", block=(128, 128), lam=1.0, ridge=1e-12, c_min=0.0, c_max=1.5, mask_1d=True,
+            eps_act=1e-5, stats=False, stream=None):
+        """Enqueue the update; it has finished once ``stream`` (default: the
+        current stream) reaches the point where this call returned."""
+        if out is None:
+            out = [torch.empty(t.shape, dtype=t.dtype, pin_memory=True) for t in theta_0]
+        cfg = merge_cfg(op, density, scope, block, lam, ridge, c_min, c_max, mask_1d, eps_act)
+        d0, d1, do = describe(theta_0), describe(update), describe(out)
+        nb = ctypes.c_size_t(0)
+        check(lib().iso_update_host_staging_size(d0, d1, do, len(theta_0), ctypes.byref(cfg),
+                                                  self.group_bytes, ctypes.byref(nb)),
+              "iso_update_host_staging_size")
+        wptr, wlen = self.ws.get(int(nb.value))
+        st = make_stats(theta_0, 1, cfg.topk, self.dev) if stats else None
+        cur = stream if stream is not None else torch.cuda.current_stream(self.dev)
+        h2d, comp, d2h = self.streams
+        # the pipeline starts after the caller's earlier work and ends on the
+        # caller's stream
+        for s_ in self.streams:
+            s_.wait_stream(cur)
+        ptrs = (ctypes.c_void_p * 3)(h2d.cuda_stream, comp.cuda_stream, d2h.cuda_stream)
+        check(lib().iso_update_host(d0, d1, int(bool(update_is_delta)), do, len(theta_0),
+                                    ctypes.byref(cfg), self.group_bytes, wptr, wlen,
+                                    ctypes.byref(st.abi()) if st else None, ptrs), "iso_update_host")
+        cur.wait_stream(comp)
+        self.h2d_bytes = sum(t.numel() * t.element_size() for t in list(theta_0) + list(update))
+        self.d2h_bytes = sum(t.numel() * t.element_size() for t in out)
+        return (out, st) if stats else out
 
 
 def launch_count() -> int:

@@ -13,6 +13,8 @@
 #include <unordered_map>
 #include <vector>
 
+#include <cuda.h>
+
 #include "iso_kernels.cuh"
 
 namespace iso {
@@ -530,6 +532,10 @@ int run_group(const Call& c, int t0, int t1, char* ws, cudaStream_t s, const iso
     const int KU = K * L.n_units;
 
     int rc = ISO_OK;
+    if (!select && !c.mask_only && (c.op == ISO_OP_TIES || c.op == ISO_OP_ISO) && P.st_units && KU > 0)
+        ISO_TRY(launch(KD_INIT, s, [&] {
+            k_units_off<<<(KU + 255) / 256, 256, 0, s>>>(P.st_units, P.st_units_stride, P.st_unit_base, L.n_units, K);
+        }));
     if (select && c.topk.scope != ISO_SCOPE_BLOCK) {
         ISO_TRY(launch(KD_INIT, s, [&] { k_init_units<<<(KU + 255) / 256, 256, 0, s>>>(P, L.global_n); }));
         rc = dispatch_src(c.xdt, c.bdt, c.ckpt, [&](auto* xt, auto* bt, auto ck) -> int {
@@ -1069,3 +1075,254 @@ extern "C" int32_t iso_update_noalloc(const iso_tensor* theta_0, const iso_tenso
     // region it uses before the group's kernels run
     return run_call(c, ws, NOALLOC_SCRATCH_BYTES, stats, s);
 }
+
+// ---------------------------------------------------------------------------
+// the K = 1 update of a parameter set in host memory, pipelined
+// ---------------------------------------------------------------------------
+namespace iso {
+namespace {
+
+__global__ void k_status_first(const int32_t* st, int n, int32_t* out) {
+    if (threadIdx.x != 0 || blockIdx.x != 0) return;
+    int32_t v = ISO_OK;
+    for (int g = 0; g < n && v == ISO_OK; ++g) v = st[g];
+    *out = v;
+}
+
+size_t bytes_of(const iso_tensor& t) { return (size_t)numel_of(t) * (t.dtype == ISO_BF16 ? 2 : 4); }
+
+// One group of consecutive tensors and where each of its three tensor lists
+// sits inside a slot's region.  The region is sized for the tensors packed
+// at 256-byte boundaries.  Tensors that follow one another in one host
+// allocation form a run, moved by one copy, and keep their host spacing
+// inside the region: for a list that is read (theta_0, update) the next
+// tensor starts at the first 16-byte boundary after the previous one, for a
+// list that is written back (out) right at its end, so no host byte outside
+// an out tensor is ever written.  Either spacing takes no more room than the
+// packed layout (a gap below 16 bytes never crosses a 256-byte boundary that
+// the packed layout would not).
+struct HostRun {
+    const char* host;                 // first byte of the run in host memory
+    size_t off, bytes;                // its offset inside the region, its length
+    uintptr_t alloc_end;              // end of the host allocation holding it (0: unknown)
+};
+struct HostList {
+    std::vector<size_t> off;          // per tensor, offset inside the region
+    std::vector<HostRun> runs;
+    size_t size = 0;                  // bytes of the region the list needs
+};
+struct HostGroup {
+    int t0, t1;
+    HostList l[3];                    // theta_0, update, out
+    long long unit0;                  // first unit of the group
+};
+
+using PtrAttrFn = CUresult (*)(void*, CUpointer_attribute, CUdeviceptr);
+PtrAttrFn ptr_attr_fn() {
+    static std::once_flag once;
+    static PtrAttrFn fn = nullptr;
+    std::call_once(once, [] {
+        void* p = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuPointerGetAttribute", &p, 12000, cudaEnableDefault, &q) == cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            fn = reinterpret_cast<PtrAttrFn>(p);
+    });
+    return fn;
+}
+
+// End of the page-locked allocation that holds host address p, or 0 when the
+// driver knows none (pageable memory): a copy may not cross from one
+// allocation into the next, so runs stay inside one.
+uintptr_t host_alloc_end(const void* p) {
+    PtrAttrFn fn = ptr_attr_fn();
+    if (!fn) return 0;
+    CUdeviceptr start = 0;
+    size_t size = 0;
+    if (fn(&start, CU_POINTER_ATTRIBUTE_RANGE_START_ADDR, (CUdeviceptr)(uintptr_t)p) != CUDA_SUCCESS) return 0;
+    if (fn(&size, CU_POINTER_ATTRIBUTE_RANGE_SIZE, (CUdeviceptr)(uintptr_t)p) != CUDA_SUCCESS) return 0;
+    if ((uintptr_t)p < (uintptr_t)start || (uintptr_t)p >= (uintptr_t)start + size) return 0;
+    return (uintptr_t)start + size;
+}
+
+size_t al16(size_t v) { return (v + 15) & ~(size_t)15; }
+
+// with_runs = false sizes the region only (no CUDA call)
+HostList place_list(const iso_tensor* h, int t0, int t1, bool written, bool with_runs) {
+    HostList L;
+    L.off.assign(t1 - t0, 0);
+    size_t packed = 0;
+    for (int t = t0; t < t1; ++t) packed += al256(bytes_of(h[t]));
+    L.size = packed;
+    if (!with_runs) return L;
+    size_t o = 0;
+    for (int t = t0; t < t1; ++t) {
+        const size_t b = bytes_of(h[t]);
+        if (b == 0) continue;
+        const char* p = static_cast<const char*>(h[t].data);   // 16-byte aligned (check_tensor)
+        if (!L.runs.empty()) {
+            HostRun& r = L.runs.back();
+            const uintptr_t end = (uintptr_t)r.host + r.bytes;
+            const uintptr_t next = written ? end : al16(end);
+            if ((uintptr_t)p == next && r.alloc_end != 0 && (uintptr_t)p + b <= r.alloc_end) {
+                L.off[t - t0] = r.off + (size_t)(p - r.host);
+                r.bytes = (size_t)(p - r.host) + b;
+                o = al256(r.off + r.bytes);
+                continue;
+            }
+        }
+        L.runs.push_back({p, o, b, host_alloc_end(p)});
+        L.off[t - t0] = o;
+        o = al256(o + b);
+    }
+    return L;
+}
+
+struct HostPlan {
+    std::vector<HostGroup> groups;
+    size_t region[3] = {0, 0, 0};     // per slot
+    size_t slot = 0, ws = 0, total = 0, st_off = 0, ws_off = 0;
+};
+
+int plan_host(const iso_tensor* th0, const iso_tensor* upd, const iso_tensor* out, int n,
+              const iso_merge_cfg* cfg, size_t group_bytes, bool with_runs, HostPlan& hp) {
+    const bool global = cfg->op != ISO_OP_TA && cfg->op != ISO_OP_RAM && cfg->topk.scope == ISO_SCOPE_GLOBAL;
+    long long units = 0;
+    int t = 0;
+    while (t < n) {
+        HostGroup g;
+        g.t0 = t;
+        size_t b = 0;
+        // GLOBAL scope has one unit over every tensor: one group
+        do { b += bytes_of(th0[t]) + bytes_of(upd[t]) + bytes_of(out[t]); ++t; }
+        while (t < n && (global || b < group_bytes));
+        g.t1 = t;
+        g.l[0] = place_list(th0, g.t0, g.t1, false, with_runs);
+        g.l[1] = place_list(upd, g.t0, g.t1, false, with_runs);
+        g.l[2] = place_list(out, g.t0, g.t1, true, with_runs);
+        size_t mn = 0, full = 0;
+        ISO_TRY(iso_workspace_size(th0 + g.t0, g.t1 - g.t0, 1, cfg, &mn, &full));
+        g.unit0 = units;
+        long long u = 0;
+        units_per_expert(th0 + g.t0, g.t1 - g.t0, cfg->topk, &u);
+        if (global) u = 1;
+        units += u;
+        for (int q = 0; q < 3; ++q) hp.region[q] = std::max(hp.region[q], g.l[q].size);
+        hp.ws = std::max(hp.ws, al256(full));
+        hp.groups.push_back(std::move(g));
+    }
+    hp.slot = hp.region[0] + hp.region[1] + hp.region[2];
+    hp.ws_off = (hp.groups.size() > 1 ? 2 : 1) * hp.slot;    // one group needs one slot
+    hp.st_off = hp.ws_off + hp.ws;
+    hp.total = hp.st_off + al256(sizeof(int32_t) * std::max<size_t>(1, hp.groups.size()));
+    return ISO_OK;
+}
+
+// copies of one tensor list between host and a slot region, one per run
+int copy_list(const HostList& L, char* dev, bool to_dev, cudaStream_t s) {
+    for (const HostRun& r : L.runs) {
+        const cudaError_t e = to_dev
+            ? cudaMemcpyAsync(dev + r.off, r.host, r.bytes, cudaMemcpyHostToDevice, s)
+            : cudaMemcpyAsync(const_cast<char*>(r.host), dev + r.off, r.bytes, cudaMemcpyDeviceToHost, s);
+        if (e != cudaSuccess) return ISO_ERR_CUDA;
+    }
+    return ISO_OK;
+}
+
+}  // namespace
+}  // namespace iso
+
+extern "C" {
+
+int32_t iso_update_host_staging_size(const iso_tensor* theta_0, const iso_tensor* update, const iso_tensor* out,
+                                     int32_t n_tensors, const iso_merge_cfg* cfg, size_t group_bytes,
+                                     size_t* bytes) {
+    if (!bytes || !cfg || n_tensors < 0 || (n_tensors > 0 && (!theta_0 || !update || !out))) return ISO_ERR_ARG;
+    if (group_bytes == 0) return ISO_ERR_ARG;
+    Call c;
+    ISO_TRY(build_merge_call(c, theta_0, update, 1, 1, out, n_tensors, cfg));
+    HostPlan hp;
+    ISO_TRY(plan_host(theta_0, update, out, n_tensors, cfg, group_bytes, false, hp));
+    *bytes = hp.total;
+    return ISO_OK;
+}
+
+int32_t iso_update_host(const iso_tensor* theta_0, const iso_tensor* update, int32_t update_is_delta,
+                        const iso_tensor* out, int32_t n_tensors, const iso_merge_cfg* cfg, size_t group_bytes,
+                        void* staging, size_t staging_bytes, const iso_merge_stats* stats, void* const* streams) {
+    if (!cfg || !streams || n_tensors < 0 || group_bytes == 0) return ISO_ERR_ARG;
+    Call c;
+    ISO_TRY(build_merge_call(c, theta_0, update, 1, update_is_delta, out, n_tensors, cfg));
+    if (n_tensors == 0) return ISO_OK;
+    HostPlan hp;
+    ISO_TRY(plan_host(theta_0, update, out, n_tensors, cfg, group_bytes, false, hp));
+    if (!staging || ((uintptr_t)staging & 255u)) return ISO_ERR_WORKSPACE;
+    if (staging_bytes < hp.total) return ISO_ERR_WORKSPACE;
+    hp = HostPlan{};                  // the same plan, with the host runs placed
+    ISO_TRY(plan_host(theta_0, update, out, n_tensors, cfg, group_bytes, true, hp));
+    cudaStream_t h2d = static_cast<cudaStream_t>(streams[0]);
+    cudaStream_t comp = static_cast<cudaStream_t>(streams[1]);
+    cudaStream_t d2h = static_cast<cudaStream_t>(streams[2]);
+    char* st = static_cast<char*>(staging);
+    int32_t* gstat = reinterpret_cast<int32_t*>(st + hp.st_off);
+    // per-slot events; destroyed when the call returns, released by the
+    // runtime once the work recorded on them completes
+    struct Events {
+        cudaEvent_t e[3][2] = {};
+        ~Events() {
+            for (auto& r : e)
+                for (cudaEvent_t x : r)
+                    if (x) cudaEventDestroy(x);
+        }
+    } evs;
+    auto& ev = evs.e;
+    for (int a = 0; a < 3; ++a)
+        for (int b = 0; b < 2; ++b)
+            if (cudaEventCreateWithFlags(&ev[a][b], cudaEventDisableTiming) != cudaSuccess) return ISO_ERR_CUDA;
+    enum { LOADED = 0, COMPUTED = 1, FREED = 2 };
+    const int G = (int)hp.groups.size();
+    std::vector<iso_tensor> d0, d1, d2;
+    for (int gi = 0; gi < G; ++gi) {
+        const HostGroup& g = hp.groups[gi];
+        const int slot = gi & 1;
+        char* base = st + (size_t)slot * hp.slot;
+        char* reg[3] = {base, base + hp.region[0], base + hp.region[0] + hp.region[1]};
+        // the slot's previous group has been copied out
+        if (gi >= 2 && cudaStreamWaitEvent(h2d, ev[FREED][slot], 0) != cudaSuccess) return ISO_ERR_CUDA;
+        for (int q = 0; q < 2; ++q)
+            if (copy_list(g.l[q], reg[q], true, h2d) != ISO_OK) return ISO_ERR_CUDA;
+        if (cudaEventRecord(ev[LOADED][slot], h2d) != cudaSuccess) return ISO_ERR_CUDA;
+        if (cudaStreamWaitEvent(comp, ev[LOADED][slot], 0) != cudaSuccess) return ISO_ERR_CUDA;
+        const int nt = g.t1 - g.t0;
+        d0.assign(theta_0 + g.t0, theta_0 + g.t1);
+        d1.assign(update + g.t0, update + g.t1);
+        d2.assign(out + g.t0, out + g.t1);
+        for (int t = 0; t < nt; ++t) {
+            d0[t].data = bytes_of(d0[t]) ? reg[0] + g.l[0].off[t] : nullptr;
+            d1[t].data = bytes_of(d1[t]) ? reg[1] + g.l[1].off[t] : nullptr;
+            d2[t].data = bytes_of(d2[t]) ? reg[2] + g.l[2].off[t] : nullptr;
+        }
+        iso_merge_stats gs{};
+        gs.status = gstat + gi;
+        if (stats) {
+            gs.units = stats->units ? stats->units + g.unit0 : nullptr;
+            gs.gram = stats->gram ? stats->gram + g.t0 : nullptr;
+            gs.coef = stats->coef ? stats->coef + g.t0 : nullptr;
+        }
+        const int rc = iso_update(d0.data(), d1.data(), update_is_delta, d2.data(), nt, cfg, st + hp.ws_off, hp.ws,
+                                  &gs, comp);
+        if (rc != ISO_OK) return rc;
+        if (cudaEventRecord(ev[COMPUTED][slot], comp) != cudaSuccess) return ISO_ERR_CUDA;
+        if (cudaStreamWaitEvent(d2h, ev[COMPUTED][slot], 0) != cudaSuccess) return ISO_ERR_CUDA;
+        if (copy_list(g.l[2], reg[2], false, d2h) != ISO_OK) return ISO_ERR_CUDA;
+        if (cudaEventRecord(ev[FREED][slot], d2h) != cudaSuccess) return ISO_ERR_CUDA;
+    }
+    // the call ends on the compute stream once every copy back has finished
+    for (int b = 0; b < 2 && b < G; ++b)
+        if (cudaStreamWaitEvent(comp, ev[FREED][(G - 1 - b) & 1], 0) != cudaSuccess) return ISO_ERR_CUDA;
+    if (stats && stats->status)
+        return launch(KD_STATUS, comp, [&] { k_status_first<<<1, 32, 0, comp>>>(gstat, G, stats->status); });
+    return ISO_OK;
+}
+
+}  // extern "C"

@@ -298,6 +298,26 @@ __global__ void k_status(const Header* h, int32_t* out) {
     if (threadIdx.x == 0 && blockIdx.x == 0) *out = h->status;
 }
 
+// The statistics of units that no tensor of a group trims (every tensor of
+// the group is a 1-D tensor that the operator leaves untrimmed, or empty): no
+// selection pass runs for such a group, so their records are written here,
+// the same record the selection writes for an untrimmed unit.
+__global__ void k_units_off(iso_unit_stats* st, long long stride, long long base, int n_units, int K) {
+    const long long n = (long long)K * n_units;
+    for (long long idx = blockIdx.x * (long long)blockDim.x + threadIdx.x; idx < n;
+         idx += (long long)gridDim.x * blockDim.x) {
+        const long long i = idx / n_units, u = idx % n_units;
+        iso_unit_stats s;
+        s.thresh_key = KEY_NONE;
+        s.flags = 0;
+        s.k = -1;
+        s.count_above = 0;
+        s.ties_at_thresh = 0;
+        s.ties_taken = 0;
+        st[i * stride + base + u] = s;
+    }
+}
+
 __global__ void k_upload(UploadChunk c) {
     uint4* dst = reinterpret_cast<uint4*>(c.dst);
     for (uint32_t q = threadIdx.x; q < c.nbytes / 16; q += blockDim.x) dst[q] = c.data[q];

@@ -75,6 +75,7 @@ constexpr int gram_blocks_per_sm(int KC) { return 2; }
 __global__ void k_solve(Plan P, int gram_mode);
 template <typename XT> __global__ void k_mask(Plan P, uint32_t* const* mptr);
 __global__ void k_status(const Header* h, int32_t* out);
+__global__ void k_units_off(iso_unit_stats* st, long long stride, long long base, int n_units, int K);
 
 // upload of host-built tables through kernel parameters (no host staging
 // buffer, capturable, ordered on the stream)

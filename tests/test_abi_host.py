@@ -296,3 +296,45 @@ def test_opt_step_sizes_and_argument_errors():
     assert st(U=0x100004) == _abi.ISO_ERR_ALIGN
     assert st(mU=0x500002) == _abi.ISO_ERR_ALIGN
     assert st(U=0) == _abi.ISO_ERR_ARG
+
+
+def test_host_update_sizes_and_argument_errors():
+    L = _abi.lib()
+    cfg = iso.merge_cfg("iso", 0.05)
+    # three 64 x 64 bf16 tensors per list, each list back to back in memory
+    th0 = _arr(*[_fake(64, 64, ptr=0x100000 + 8192 * i) for i in range(3)])
+    upd = _arr(*[_fake(64, 64, ptr=0x200000 + 8192 * i) for i in range(3)])
+    out = _arr(*[_fake(64, 64, ptr=0x300000 + 8192 * i) for i in range(3)])
+    nb = ctypes.c_size_t()
+
+    def size(group, cfg_=cfg, n=3):
+        rc = L.iso_update_host_staging_size(th0, upd, out, n, ctypes.byref(cfg_), group, ctypes.byref(nb))
+        return rc, nb.value
+
+    rc, one_group = size(1 << 30)
+    assert rc == 0 and one_group % 256 == 0
+    rc, per_tensor = size(1)                       # a group per tensor: slots hold one tensor
+    assert rc == 0 and per_tensor < one_group
+    assert one_group >= 2 * 3 * 3 * 8192           # two slots of three lists of three tensors
+    glob = iso.merge_cfg("ties", 0.2, "global")    # one unit over every tensor: one group
+    assert size(1, glob) == size(1 << 30, glob)
+    assert size(0)[0] == _abi.ISO_ERR_ARG
+    assert L.iso_update_host_staging_size(th0, upd, out, 3, ctypes.byref(cfg), 1 << 20, None) == _abi.ISO_ERR_ARG
+    bad_out = _arr(_fake(64, 64, ptr=0x300000), _fake(64, 64, ptr=0x200000), _fake(64, 64, ptr=0x300000 + 16384))
+    assert L.iso_update_host_staging_size(th0, upd, bad_out, 3, ctypes.byref(cfg), 1 << 20,
+                                          ctypes.byref(nb)) == _abi.ISO_ERR_ARG    # out on an update
+
+    streams = (ctypes.c_void_p * 3)()
+    _, need = size(1 << 20)
+
+    def run(staging, nbytes, streams_=streams, n=3, group=1 << 20):
+        return L.iso_update_host(th0, upd, 0, out, n, ctypes.byref(cfg), group, ctypes.c_void_p(staging),
+                                 nbytes, None, streams_)
+
+    # every rejection happens before anything is enqueued
+    assert run(0x4000000, need, streams_=None) == _abi.ISO_ERR_ARG
+    assert run(0x4000000, need, group=0) == _abi.ISO_ERR_ARG
+    assert run(0, need) == _abi.ISO_ERR_WORKSPACE
+    assert run(0x4000010, need) == _abi.ISO_ERR_WORKSPACE                   # not 256-byte aligned
+    assert run(0x4000000, need - 256) == _abi.ISO_ERR_WORKSPACE
+    assert run(0, 0, n=0) == 0                                              # an empty list is a no-op
