@@ -239,6 +239,46 @@ int32_t iso_update_noalloc(const iso_tensor* theta_0, const iso_tensor* update, 
                            const iso_tensor* out, int32_t n_tensors, const iso_merge_cfg* cfg,
                            const iso_merge_stats* stats, void* stream);
 
+/* ---- One selection unit split over several GPUs (App. F, TIES trim) -------
+ *
+ * A unit too large for one GPU (a GLOBAL-scope unit, or an embedding split
+ * with its tensor) is held as contiguous ranges of its positions, rank r's
+ * range before rank r + 1's.  The exact TopKMask of the whole unit is a radix
+ * descent over the magnitude keys whose per-digit counts are summed over the
+ * ranks; each rank runs the two calls below on its own range and the host
+ * exchanges the counts (paper_2607_19331_gb300/shard.py, split_unit_select).
+ * The threshold t and the ties each rank keeps follow the library's rules:
+ * k = floor(rho N + 1/2) over the unit's N entries, ties at t taken lowest
+ * position first over the whole unit.
+ *
+ * key_e is the binary32 bits of |tau_e| with the sign cleared, tau_e = x_e
+ * (base = NULL: x is a task vector) or x_e - base_e in binary32 (x a
+ * checkpoint of the base; same shape, either dtype).  [begin, end) is a range
+ * of x's flat (row-major) positions.  Device pointers; enqueued on stream;
+ * argument errors are returned before anything is enqueued.  Non-finite
+ * values are counted by their keys (above 0x7F800000) and not reported. */
+
+/* counts[b] (int64, nbins entries, overwritten) = the number of positions e
+ * in [begin, end) with key_e >> pshift == prefix and
+ * (key_e >> shift) & (nbins - 1) == b.  nbins a power of two <= 4096,
+ * 0 <= shift <= pshift <= 32.  With nbins = 1 and pshift = shift = 0 the one
+ * count is the number of keys equal to prefix. */
+int32_t iso_range_hist(const iso_tensor* x, const iso_tensor* base, int64_t begin, int64_t end,
+                       uint32_t prefix, int32_t pshift, int32_t shift, int32_t nbins, int64_t* counts,
+                       void* stream);
+
+/* Host-only.  Workspace bytes of iso_range_mask for a range of n positions. */
+int32_t iso_range_mask_workspace_size(int64_t n, size_t* bytes);
+
+/* mask_bits (ceil((end - begin) / 32) uint32 words, bit j of word w for
+ * position begin + 32 w + j, bits past end zero): set where key_e > t, or
+ * key_e == t and fewer than take keys equal to t lie in [begin, e).  t and
+ * take come from the unit's selection (take = this rank's share of the ties
+ * the unit keeps); t = 0xFFFFFFFF selects nothing.  The workspace (8-byte
+ * aligned) holds per-tile tie counts. */
+int32_t iso_range_mask(const iso_tensor* x, const iso_tensor* base, int64_t begin, int64_t end, uint32_t t,
+                       int64_t take, uint32_t* mask_bits, void* workspace, size_t ws_bytes, void* stream);
+
 /* ---- The K = 1 update of a parameter set held in host memory --------------
  *
  * The update of iso_update (same operation, same configuration, same results

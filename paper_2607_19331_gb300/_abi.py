@@ -86,6 +86,9 @@ PROTOTYPES = [
                         ctypes.POINTER(IsoMergeStats), P]),
     ("iso_update_noalloc", I32, [PT, PT, I32, PT, I32, ctypes.POINTER(IsoMergeCfg),
                                  ctypes.POINTER(IsoMergeStats), P]),
+    ("iso_range_hist", I32, [PT, PT, I64, I64, ctypes.c_uint32, I32, I32, I32, P, P]),
+    ("iso_range_mask_workspace_size", I32, [I64, ctypes.POINTER(SZ)]),
+    ("iso_range_mask", I32, [PT, PT, I64, I64, ctypes.c_uint32, I64, P, P, SZ, P]),
     ("iso_update_host_staging_size", I32, [PT, PT, PT, I32, ctypes.POINTER(IsoMergeCfg), SZ,
                                            ctypes.POINTER(SZ)]),
     ("iso_update_host", I32, [PT, PT, I32, PT, I32, ctypes.POINTER(IsoMergeCfg), SZ, P, SZ,

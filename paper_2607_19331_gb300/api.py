@@ -284,6 +284,65 @@ class HostUpdate:
         return (out, st) if stats else out
 
 
+# ---------------------------------------------------------------------------
+# one selection unit split over ranks (App. F, TIES trim)
+# ---------------------------------------------------------------------------
+def _range_args(x, base, begin, end):
+    n = x.numel()
+    end = n if end is None else int(end)
+    dx = describe([x])
+    db = describe([base]) if base is not None else None
+    return dx, db, int(begin), end
+
+
+def range_hist(x: torch.Tensor, base: Optional[torch.Tensor] = None, begin=0, end=None, prefix=0, pshift=32,
+               shift=21, nbins=2048, counts=None, stream=None) -> torch.Tensor:
+    """iso_range_hist: int64[nbins] device counts of the magnitude keys of
+    x[begin:end] (x - base for a checkpoint) with key >> pshift == prefix,
+    binned by (key >> shift) & (nbins - 1)."""
+    dx, db, b, e = _range_args(x, base, begin, end)
+    if counts is None:
+        counts = torch.empty(nbins, dtype=torch.int64, device=x.device)
+    check(lib().iso_range_hist(dx, db, b, e, int(prefix) & 0xFFFFFFFF, int(pshift), int(shift), int(nbins),
+                               ctypes.c_void_p(counts.data_ptr()), _stream(stream)), "iso_range_hist")
+    return counts
+
+
+def range_mask(x: torch.Tensor, t: int, take: int, base: Optional[torch.Tensor] = None, begin=0, end=None,
+               workspace: Optional[Workspace] = None, stream=None) -> torch.Tensor:
+    """iso_range_mask: packed int32 words of this range's share of a unit's
+    TopKMask (keys above t, and the first ``take`` keys equal to t)."""
+    dx, db, b, e = _range_args(x, base, begin, end)
+    words = torch.zeros(max(1, (e - b + 31) // 32), dtype=torch.int32, device=x.device)
+    nb = ctypes.c_size_t(0)
+    check(lib().iso_range_mask_workspace_size(e - b, ctypes.byref(nb)), "iso_range_mask_workspace_size")
+    ws = _workspace(workspace, x.device)
+    wptr, wlen = ws.get(int(nb.value))
+    check(lib().iso_range_mask(dx, db, b, e, int(t) & 0xFFFFFFFF, int(take), ctypes.c_void_p(words.data_ptr()),
+                               wptr, wlen, _stream(stream)), "iso_range_mask")
+    return words[: (e - b + 31) // 32]
+
+
+def split_unit_topk(x: torch.Tensor, density: float, base: Optional[torch.Tensor] = None, begin=0, end=None,
+                    group=None, workspace: Optional[Workspace] = None):
+    """This rank's part of the exact TopKMask of one unit split over the ranks
+    of ``group`` (rank order = position order): the radix counts come from
+    iso_range_hist on the device, summed over the ranks by
+    shard.split_unit_select; the mask words from iso_range_mask.  Returns
+    (SplitSelect, int32 mask words of x[begin:end])."""
+    from .shard import split_unit_select
+    dx, db, b, e = _range_args(x, base, begin, end)
+
+    def local_hist(prefix, pshift, shift, nb):
+        return range_hist(x, base, b, e, prefix, pshift, shift, nb).cpu().tolist()
+
+    def local_ties(t):
+        return int(range_hist(x, base, b, e, t, 0, 0, 1).cpu()[0])
+
+    sel = split_unit_select(e - b, density, local_hist, local_ties, group=group)
+    return sel, range_mask(x, sel.t, sel.take, base, b, e, workspace=workspace)
+
+
 def launch_count() -> int:
     return int(lib().iso_launch_count())
 

@@ -16,7 +16,7 @@ CSRC = os.path.join(HERE, "csrc")
 BUILD = os.path.join(HERE, "_build")
 LIB = os.path.join(BUILD, "libiso_gb300.so")
 SOURCES = ["iso_api.cu", "iso_select.cu", "iso_apply.cu", "iso_merge.cu", "iso_block.cu", "iso_fused.cu",
-           "iso_gemm.cu", "iso_frame.cu"]
+           "iso_gemm.cu", "iso_frame.cu", "iso_range.cu"]
 HEADERS = ["iso_internal.cuh", "iso_kernels.cuh", "iso_gemm.cuh"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-static-global-template-stub=false", "-Xcompiler", "-fPIC,-ffp-contract=off",

@@ -29,12 +29,12 @@ constexpr int FUSED_GRID_PER_SM = FUSED_BLOCKS_PER_SM;
 enum Kind {
     KD_UPLOAD, KD_INIT, KD_SAMPLE, KD_COUNT, KD_DECIDE, KD_RADIX_HIST, KD_RADIX_PICK, KD_TIE,
     KD_CUT, KD_BLOCK_SELECT, KD_GRAM, KD_SOLVE, KD_APPLY, KD_MASK, KD_DELTA, KD_STATUS, KD_MEMSET,
-    KD_PATCH, KD_REPAIR, KD_FRAME_GEMM, KD_FRAME, KD_COUNT_KINDS
+    KD_PATCH, KD_REPAIR, KD_FRAME_GEMM, KD_FRAME, KD_RANGE, KD_COUNT_KINDS
 };
 const char* kKindNames[KD_COUNT_KINDS] = {
     "upload", "init_units", "sample", "count", "decide", "radix_hist", "radix_pick", "tie",
     "cut", "block_select", "gram", "solve", "apply", "mask", "delta", "status", "memset",
-    "patch", "repair", "frame_gemm", "frame"};
+    "patch", "repair", "frame_gemm", "frame", "range"};
 
 std::atomic<uint64_t> g_launches{0};
 
@@ -792,10 +792,12 @@ int build_merge_call(Call& c, const iso_tensor* theta_0, const iso_tensor* exper
 
 }  // namespace
 
-// Launch accounting and profiling for the frame-space merge (iso_frame.cu).
+// Launch accounting and profiling for the kernels of other translation units
+// (0: the tensor-core product, 1: the frame-space merge and optimizer, 2: the
+// range selection of iso_range.cu).
 int prof_begin(int frame_kind, cudaStream_t s) {
     if (!g_prof.on) return -1;
-    const int kind = frame_kind == 0 ? KD_FRAME_GEMM : KD_FRAME;
+    const int kind = frame_kind == 0 ? KD_FRAME_GEMM : frame_kind == 1 ? KD_FRAME : KD_RANGE;
     std::lock_guard<std::mutex> lk(g_prof_mu);
     if (g_prof.used >= Prof::CAP) return -1;
     const int slot = g_prof.used;

@@ -352,11 +352,18 @@ __global__ void __launch_bounds__(256) k_fr_ftdf(Frames f, const double* dots, i
 
 // N = (F + dF)^T (F + dF) - I in binary64, the polar retraction's argument
 // (any departure of F^T F from I included, so the retraction also restores
-// orthonormality lost to rounding); tiling as in k_fr_ftdf
+// orthonormality lost to rounding).  N is symmetric: one block per 64 x 64
+// tile on or above the diagonal (nt (nt + 1) / 2 blocks for nt tiles a side),
+// written to both halves.  Entry (k, l) and entry (l, k) are the same sum of
+// the same products in the same order, so the two halves agree bit for bit
+// also inside a diagonal tile.  Tiling as in k_fr_ftdf.
 __global__ void __launch_bounds__(256) k_op_gram64(const double* F, const double* dF, long long d, long long q,
                                                    double* N) {
     __shared__ double sa[16][64], sb[16][64];
-    const long long k0 = (long long)blockIdx.y * 64, l0 = (long long)blockIdx.x * 64;
+    const long long nt = (q + 63) / 64;
+    long long rest = blockIdx.x, tr = 0;
+    while (rest >= nt - tr) { rest -= nt - tr; ++tr; }      // at most nt steps
+    const long long k0 = tr * 64, l0 = (tr + rest) * 64;
     const int tx = threadIdx.x & 15, ty = threadIdx.x >> 4;
     double acc[4][4];
 #pragma unroll
@@ -391,7 +398,11 @@ __global__ void __launch_bounds__(256) k_op_gram64(const double* F, const double
 #pragma unroll
         for (int b = 0; b < 4; ++b) {
             const long long k = k0 + ty * 4 + a, l = l0 + tx * 4 + b;
-            if (k < q && l < q) N[k * q + l] = acc[a][b] - (k == l ? 1.0 : 0.0);
+            if (k < q && l < q) {
+                const double v = acc[a][b] - (k == l ? 1.0 : 0.0);
+                N[k * q + l] = v;
+                if (k0 != l0) N[l * q + k] = v;
+            }
         }
 }
 
@@ -1142,8 +1153,8 @@ int32_t iso_opt_step(double* U, double* V, const double* S0, const iso_tensor* G
     // binary64, R = (I + N)^(-1/2) - I, E_F = dF + (F + dF) R
     for (int sd = 0; sd < 2; ++sd) {
         const long long Dp = sd == 0 ? L.Mp : L.Np, d = fr[sd].d;
-        FR_LAUNCH((k_op_gram64<<<dim3((unsigned)((q + 63) / 64), (unsigned)((q + 63) / 64)), 256, 0, s>>>(
-            sd == 0 ? U : V, D(L.dF[sd]), d, q, D(L.n64))));
+        const unsigned nt = (unsigned)((q + 63) / 64);
+        FR_LAUNCH((k_op_gram64<<<nt * (nt + 1) / 2, 256, 0, s>>>(sd == 0 ? U : V, D(L.dF[sd]), d, q, D(L.n64))));
         NsBufs nb{D(L.ns_y), D(L.ns_z), D(L.ns_m), F(L.ns_y4), F(L.ns_z4), F(L.ns_m4), F(L.ns_t1),
                   F(L.ns_t2), F(L.ns_t3)};
         ISO_TRY(ns_root(s, sms, hdr, sd, nullptr, D(L.n64), q, Qp, nb, ns_iters, F(L.r4)));

@@ -75,7 +75,8 @@ int gemm_tensor_map(CUtensorMap* map, const float* base, long long rows, long lo
 
 // Launch accounting and per-kind device timing shared with the rest of the
 // library (iso_api.cu): kind 0 = the tensor-core products, 1 = the other
-// frame-merge kernels.  prof_begin returns a slot (or -1 when profiling is
+// frame-merge and optimizer kernels, 2 = the range selection kernels
+// (iso_range.cu).  prof_begin returns a slot (or -1 when profiling is
 // off); prof_end records the end event and counts the launch.
 int prof_begin(int frame_kind, cudaStream_t s);
 void prof_end(int slot, cudaStream_t s);

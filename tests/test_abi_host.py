@@ -338,3 +338,33 @@ def test_host_update_sizes_and_argument_errors():
     assert run(0x4000010, need) == _abi.ISO_ERR_WORKSPACE                   # not 256-byte aligned
     assert run(0x4000000, need - 256) == _abi.ISO_ERR_WORKSPACE
     assert run(0, 0, n=0) == 0                                              # an empty list is a no-op
+
+
+def test_range_selection_argument_errors():
+    L = _abi.lib()
+    x = _arr(_fake(100, 100, ptr=0x100000))
+    base = _arr(_fake(100, 100, ptr=0x200000))
+    cnt = ctypes.c_void_p(0x300000)
+
+    def hist(b=0, e=10_000, prefix=0, pshift=31, shift=20, nb=2048, counts=cnt, base_=base, x_=x):
+        return L.iso_range_hist(x_, base_, b, e, prefix, pshift, shift, nb, counts, None)
+
+    # every rejection happens before anything is enqueued
+    assert hist(nb=3) == _abi.ISO_ERR_ARG                      # not a power of two
+    assert hist(nb=8192) == _abi.ISO_ERR_ARG
+    assert hist(shift=25, pshift=20) == _abi.ISO_ERR_ARG       # shift above pshift
+    assert hist(pshift=33) == _abi.ISO_ERR_ARG
+    assert hist(b=5, e=4) == _abi.ISO_ERR_ARG
+    assert hist(e=10_001) == _abi.ISO_ERR_ARG                  # past the tensor
+    assert hist(counts=None) == _abi.ISO_ERR_ARG
+    assert hist(base_=_arr(_fake(100, 99, ptr=0x200000))) == _abi.ISO_ERR_SHAPE
+    assert hist(x_=_arr(_fake(100, 100, ptr=0x100002))) == _abi.ISO_ERR_ARG      # misaligned
+    nb = ctypes.c_size_t()
+    assert L.iso_range_mask_workspace_size(10_000, ctypes.byref(nb)) == 0 and nb.value == 10 * 8
+    mask = ctypes.c_void_p(0x400000)
+    ws = ctypes.c_void_p(0x500000)
+    assert L.iso_range_mask(x, base, 0, 10_000, 5, -1, mask, ws, 80, None) == _abi.ISO_ERR_ARG
+    assert L.iso_range_mask(x, base, 0, 10_000, 5, 0, mask, ws, 72, None) == _abi.ISO_ERR_WORKSPACE
+    assert L.iso_range_mask(x, base, 0, 10_000, 5, 0, mask, None, 80, None) == _abi.ISO_ERR_WORKSPACE
+    assert L.iso_range_mask(x, base, 0, 10_000, 5, 0, None, ws, 80, None) == _abi.ISO_ERR_ARG
+    assert L.iso_range_mask(x, base, 7, 7, 5, 0, None, None, 0, None) == 0     # an empty range is a no-op
