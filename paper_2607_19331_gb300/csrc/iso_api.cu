@@ -29,12 +29,12 @@ constexpr int FUSED_GRID_PER_SM = FUSED_BLOCKS_PER_SM;
 enum Kind {
     KD_UPLOAD, KD_INIT, KD_SAMPLE, KD_COUNT, KD_DECIDE, KD_RADIX_HIST, KD_RADIX_PICK, KD_TIE,
     KD_CUT, KD_BLOCK_SELECT, KD_GRAM, KD_SOLVE, KD_APPLY, KD_MASK, KD_DELTA, KD_STATUS, KD_MEMSET,
-    KD_PATCH, KD_REPAIR, KD_FRAME_GEMM, KD_FRAME, KD_RANGE, KD_COUNT_KINDS
+    KD_PATCH, KD_REPAIR, KD_FRAME_GEMM, KD_FRAME, KD_RANGE, KD_RADIX_FLAT, KD_CUT_PART, KD_COUNT_KINDS
 };
 const char* kKindNames[KD_COUNT_KINDS] = {
     "upload", "init_units", "sample", "count", "decide", "radix_hist", "radix_pick", "tie",
     "cut", "block_select", "gram", "solve", "apply", "mask", "delta", "status", "memset",
-    "patch", "repair", "frame_gemm", "frame", "range"};
+    "patch", "repair", "frame_gemm", "frame", "range", "radix_flat", "cut_part"};
 
 std::atomic<uint64_t> g_launches{0};
 
@@ -559,11 +559,14 @@ int run_group(const Call& c, int t0, int t1, char* ws, cudaStream_t s, const iso
                 ISO_TRY(launch(KD_COUNT, s, [&] { k_count<XT, BT, CK><<<sms * COUNT_GRID_PER_SM, TPB, 0, s>>>(P); }));
             }
             ISO_TRY(launch(KD_DECIDE, s, [&] { k_decide<<<(KU + 255) / 256, 256, 0, s>>>(P); }));
+            ISO_TRY(smem_optin(k_radix_flat, RADIX_FLAT_SMEM));
             for (int level = 0; level < 3; ++level) {
+                ISO_TRY(launch(KD_RADIX_FLAT, s, [&] { k_radix_flat<<<sms * 2, TPB, RADIX_FLAT_SMEM, s>>>(P); }));
                 ISO_TRY(launch(KD_RADIX_HIST, s, [&] { k_radix_hist<XT, BT, CK><<<pgrid, TPB, 0, s>>>(P); }));
                 ISO_TRY(launch(KD_RADIX_PICK, s, [&] { k_radix_pick<<<KU, TPB, 0, s>>>(P); }));
             }
             ISO_TRY(launch(KD_TIE, s, [&] { k_tie<XT, BT, CK><<<pgrid, TPB, 0, s>>>(P); }));
+            ISO_TRY(launch(KD_CUT_PART, s, [&] { k_cut_part<<<pgrid, TPB, 0, s>>>(P); }));
             ISO_TRY(launch(KD_CUT, s, [&] { k_cut<XT, BT, CK><<<KU, CUT_TPB, 0, s>>>(P); }));
             return ISO_OK;
         });

@@ -42,6 +42,14 @@ constexpr int COUNT_CHUNKS = 512;           // fused K = 1 pass: 256-entry chunk
 
 constexpr int RADIX_BITS = 11;
 constexpr int RADIX_BINS = 1 << RADIX_BITS;
+// A unit whose candidate pool holds at least this many slots is histogrammed
+// as one flat array (the count pass seals the unused slots of its chunks with
+// KEY_NONE), not tile by tile.
+constexpr unsigned long long RADIX_FLAT_MIN = 1ull << 20;
+constexpr int RADIX_FLAT_SMEM = (WPB + 2) * RADIX_BINS * 4;   // k_radix_flat's dynamic shared memory
+// A unit with at least this many tiles finds the tile of its cut from
+// per-chunk tie sums (k_cut_part, RADIX_BINS chunks) before it scans tiles.
+constexpr long long CUT_SPLIT_MIN = 1ll << 16;
 constexpr int BLOCK_MAX_ENTRIES = 16384;    // BLOCK scope: entries per unit held on chip
 constexpr int BLOCK_KEYS_WORDS = BLOCK_MAX_ENTRIES + BLOCK_MAX_ENTRIES / 32;   // padded key array
 

@@ -30,6 +30,8 @@ __global__ void k_radix_pick(Plan P);
 template <typename XT, typename BT, bool CK> __global__ void k_csample(Plan P);
 template <typename XT, typename BT, bool CK> __global__ void k_tie(Plan P);
 template <typename XT, typename BT, bool CK> __global__ void k_cut(Plan P);
+__global__ void k_cut_part(Plan P);
+__global__ void k_radix_flat(Plan P);
 
 // select (BLOCK scope)
 constexpr int BLOCK_TPB = 1024;

@@ -629,8 +629,17 @@ __global__ void __launch_bounds__(TPB, COUNT_BLOCKS_PER_SM) k_count(Plan P) {
     // of the next tile (item it2 of run r2), so a whole tile of loads is in
     // flight while this one is counted.
     RawTile<XT, BT, CK> rt;
+    // the unused slots of the warp's chunk get KEY_NONE, so that a large
+    // unit's pool can be read as one flat array (k_radix_hist)
+    auto seal = [&]() {
+        if (au && !ovf)
+            for (uint32_t q = lane; q < ch_left; q += 32) cseg[ch_pos + q] = KEY_NONE;
+        ch_left = 0;
+    };
+
     auto count_tile = [&](const CountRun& rr, uint32_t it, bool more, const CountRun& r2, uint32_t it2) {
         if (rr.U != au) {
+            seal();
             flush();
             au = rr.U;
             lo = au->lo;
@@ -709,6 +718,8 @@ __global__ void __launch_bounds__(TPB, COUNT_BLOCKS_PER_SM) k_count(Plan P) {
         uint32_t t_int;
         const uint32_t off = warp_excl_scan(nb, &t_int);
         if (t_int && !ovf && t_int > ch_left) {
+            // the rest of the current chunk is too short: seal it, take a new one
+            for (uint32_t q = lane; q < ch_left; q += 32) cseg[ch_pos + q] = KEY_NONE;
             unsigned long long start = 0;
             uint32_t req = 0;
             if (lane == 0) {
@@ -771,6 +782,7 @@ __global__ void __launch_bounds__(TPB, COUNT_BLOCKS_PER_SM) k_count(Plan P) {
         it = it2;
         r = r2;
     }
+    seal();
     flush();
 }
 
@@ -871,18 +883,107 @@ __device__ __forceinline__ void hist_add(uint32_t* h, uint32_t* mxc, uint32_t* m
     }
 }
 
+// A unit in radix select over a pool filled by k_count (not the fused pass,
+// whose pool is not sealed) and large enough to scan as one flat array.
+__device__ __forceinline__ bool radix_flat(const Unit& U) {
+    return U.state == ST_RADIX && U.r_src == SRC_CAND && !U.mode_t && !U.overflow && U.n_alloc >= RADIX_FLAT_MIN;
+}
+
+// Large pools (radix_flat): every block takes a slice of the unit's pool
+// (sealed slots hold KEY_NONE), read consecutively by each warp.  A band
+// where a few keys hold most entries sends many keys to a few bins, so the
+// counts are kept per warp (no two warps add to one counter), and instead of
+// per-bin minima and maxima each bin records its first key and whether
+// another key was seen: what the pick needs to tell a single-key bin.  RADIX_FLAT_SMEM bytes of dynamic shared
+// memory: WPB count arrays, the first keys, the flags.
+__global__ void __launch_bounds__(TPB) k_radix_flat(Plan P) {
+    extern __shared__ uint32_t fsm[];
+    if (*(volatile int32_t*)&P.hdr->n_radix == 0) return;
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    uint32_t* const wc = fsm + warp * RADIX_BINS;
+    uint32_t* const bkey = fsm + WPB * RADIX_BINS;
+    uint32_t* const mixed = bkey + RADIX_BINS;
+    for (int b = threadIdx.x; b < (WPB + 2) * RADIX_BINS; b += blockDim.x)
+        fsm[b] = (b >= WPB * RADIX_BINS && b < (WPB + 1) * RADIX_BINS) ? KEY_NONE : 0u;
+    __syncthreads();
+    const int KU = P.K * P.n_units;
+    for (int u = 0; u < KU; ++u) {
+        const Unit& U = P.units[u];
+        if (!radix_flat(U)) continue;                  // the same for every thread
+        const int pshift = U.r_pshift;
+        const int shift = pshift > RADIX_BITS ? pshift - RADIX_BITS : 0;
+        const int nb = 1 << (pshift - shift);
+        const uint32_t base = U.r_base, prefix = U.r_prefix;
+        const uint32_t* cs = P.cand + U.cand_off;
+        const long long n = (long long)U.n_alloc;
+        // a warp takes FLAT_KEYS consecutive slots per step: four 16-byte
+        // loads per lane issued together, then one count per key into the
+        // warp's own array (lanes of one warp with equal bins are the only
+        // conflicts), and the bin's first key compared with each key
+        constexpr int FLAT_VEC = 4, FLAT_KEYS = 32 * 4 * FLAT_VEC;
+        const bool vec = (reinterpret_cast<uintptr_t>(cs) & 15u) == 0;
+        for (long long q0 = ((long long)blockIdx.x * WPB + warp) * FLAT_KEYS; q0 < n;
+             q0 += (long long)gridDim.x * WPB * FLAT_KEYS) {
+            uint32_t kk[4 * FLAT_VEC];
+#pragma unroll
+            for (int j = 0; j < FLAT_VEC; ++j) {
+                const long long q = q0 + (long long)(j * 32 + lane) * 4;
+                if (vec && q + 4 <= n) {
+                    const uint4 w = *reinterpret_cast<const uint4*>(cs + q);
+                    kk[4 * j] = w.x; kk[4 * j + 1] = w.y; kk[4 * j + 2] = w.z; kk[4 * j + 3] = w.w;
+                } else {
+#pragma unroll
+                    for (int i = 0; i < 4; ++i) kk[4 * j + i] = q + i < n ? cs[q + i] : KEY_NONE;
+                }
+            }
+#pragma unroll
+            for (int i = 0; i < 4 * FLAT_VEC; ++i) {
+                const uint32_t v = kk[i] - base;
+                if (kk[i] != KEY_NONE && (v >> pshift) == prefix) {
+                    const int bin = (int)((v >> shift) & (uint32_t)(nb - 1));
+                    atomicAdd(&wc[bin], 1u);
+                    uint32_t bk = bkey[bin];
+                    if (bk == KEY_NONE) {
+                        const uint32_t old = atomicCAS(&bkey[bin], KEY_NONE, kk[i]);
+                        bk = old == KEY_NONE ? kk[i] : old;
+                    }
+                    if (kk[i] != bk) mixed[bin] = 1u;
+                }
+            }
+        }
+        __syncthreads();
+        // a single key k: (max, max of complements) = (k, ~k); several: both
+        // all ones, so the pick's minimum (the complement) and maximum differ
+        for (int b = threadIdx.x; b < nb; b += blockDim.x) {
+            uint32_t c = 0;
+#pragma unroll
+            for (int w = 0; w < WPB; ++w) { c += fsm[w * RADIX_BINS + b]; fsm[w * RADIX_BINS + b] = 0; }
+            if (c) {
+                const bool mx = mixed[b] != 0;
+                const uint32_t bk = bkey[b];
+                atomicAdd(&P.hist[(long long)u * RADIX_BINS + b], c);
+                atomicMax(&P.hmx[(long long)u * RADIX_BINS + b], mx ? 0xFFFFFFFFu : bk);
+                atomicMax(&P.hmxc[(long long)u * RADIX_BINS + b], mx ? 0xFFFFFFFFu : ~bk);
+            }
+            bkey[b] = KEY_NONE;
+            mixed[b] = 0;
+        }
+        __syncthreads();
+    }
+}
+
 template <typename XT, typename BT, bool CK>
 __global__ void __launch_bounds__(TPB) k_radix_hist(Plan P) {
     __shared__ uint32_t s_hist[RADIX_BINS];
     __shared__ uint32_t s_mxc[RADIX_BINS];
     __shared__ uint32_t s_mx[RADIX_BINS];
     if (*(volatile int32_t*)&P.hdr->n_radix == 0) return;
+    for (int b = threadIdx.x; b < RADIX_BINS; b += blockDim.x) { s_hist[b] = 0; s_mxc[b] = 0; s_mx[b] = 0; }
+    __syncthreads();
     const long long items = (long long)P.K * P.n_tiles;
     const long long per = (items + gridDim.x - 1) / gridDim.x;
     const long long beg = blockIdx.x * per;
     const long long end = (beg + per < items) ? beg + per : items;
-    for (int b = threadIdx.x; b < RADIX_BINS; b += blockDim.x) { s_hist[b] = 0; s_mxc[b] = 0; s_mx[b] = 0; }
-    __syncthreads();
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     long long it = beg;
     while (it < end) {
@@ -891,7 +992,7 @@ __global__ void __launch_bounds__(TPB) k_radix_hist(Plan P) {
         const long long run_end = c.run_end < end ? c.run_end : end;
         const TensorDesc& d = P.tens[c.t];
         Unit* U = (d.flags & TF_TRIM) ? unit_of(P, c.i, d) : nullptr;
-        if (!U || U->state != ST_RADIX) { it = run_end; continue; }
+        if (!U || U->state != ST_RADIX || radix_flat(*U)) { it = run_end; continue; }
         const long long ui = U - P.units;
         const int pshift = U->r_pshift;
         const int shift = pshift > RADIX_BITS ? pshift - RADIX_BITS : 0;
@@ -1091,6 +1192,41 @@ __device__ __forceinline__ void write_unit_stats(const Plan& P, int idx, const U
     P.st_units[(long long)i * P.st_units_stride + P.st_unit_base + u] = s;
 }
 
+// The per-tile tie counts the cut of unit U scans.
+__device__ __forceinline__ const uint32_t* cut_src(const Plan& P, const Unit& U) {
+    return ((U.tie_src == TIE_EQ_HI) ? P.teq_hi : (U.tie_src == TIE_EQ_LO) ? P.teq_lo : P.tcnt) +
+           (long long)U.expert * P.n_tiles;
+}
+__device__ __forceinline__ bool cut_split(const Unit& U) {
+    return U.state == ST_TKNOWN && U.need < U.ties && U.tile_end - U.tile_begin >= CUT_SPLIT_MIN;
+}
+
+// For units with many tiles: the tie counts summed over RADIX_BINS chunks of
+// consecutive tiles (chunk c holds tiles tile_begin + c * per ...), into the
+// unit's histogram row (free once the radix select is over).  One warp per
+// chunk, consecutive loads.
+__global__ void __launch_bounds__(TPB) k_cut_part(Plan P) {
+    const int lane = threadIdx.x & 31;
+    const long long gw = ((long long)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+    const long long nw = ((long long)gridDim.x * blockDim.x) >> 5;
+    const int KU = P.K * P.n_units;
+    for (int u = 0; u < KU; ++u) {
+        const Unit& U = P.units[u];
+        if (!cut_split(U)) continue;
+        const long long nt = U.tile_end - U.tile_begin;
+        const long long per = (nt + RADIX_BINS - 1) / RADIX_BINS;
+        const uint32_t* src = cut_src(P, U);
+        for (long long c = gw; c < RADIX_BINS; c += nw) {
+            const long long g0 = U.tile_begin + c * per;
+            const long long g1 = min(U.tile_end, g0 + per);
+            uint32_t sum = 0;                      // <= per * TILE < 2^32
+            for (long long g = g0 + lane; g < g1; g += 32) sum += src[g];
+            sum = __reduce_add_sync(0xFFFFFFFFu, sum);
+            if (lane == 0) P.hist[(long long)u * RADIX_BINS + c] = sum;
+        }
+    }
+}
+
 template <typename XT, typename BT, bool CKPT>
 __global__ void __launch_bounds__(CUT_TPB) k_cut(Plan P) {
     __shared__ long long s_scan[33];
@@ -1108,13 +1244,42 @@ __global__ void __launch_bounds__(CUT_TPB) k_cut(Plan P) {
     const int i = U.expert;
     if (threadIdx.x == 0) { s_tile = -1; s_rem = 0; s_pos = -1; }   // ordered by the scan's barriers
     if (U.need < U.ties) {
-        // 1. the tile that holds the need-th tie (tiles in unit order)
-        const long long nt = U.tile_end - U.tile_begin;
+        // 1. the tile that holds the need-th tie (tiles in unit order); a
+        //    unit with many tiles first picks the chunk from k_cut_part's sums
+        const uint32_t* src = cut_src(P, U);
+        long long lo_t = U.tile_begin, hi_t = U.tile_end, need = U.need;
+        if (cut_split(U)) {
+            __shared__ long long s_c0, s_c1, s_before;
+            const long long nt = U.tile_end - U.tile_begin;
+            const long long per_c = (nt + RADIX_BINS - 1) / RADIX_BINS;
+            const uint32_t* cs = P.hist + (long long)idx * RADIX_BINS;
+            constexpr int CPT = RADIX_BINS / CUT_TPB;          // chunks per thread
+            long long local = 0;
+#pragma unroll
+            for (int q = 0; q < CPT; ++q) local += cs[threadIdx.x * CPT + q];
+            if (threadIdx.x == 0) { s_c0 = -1; s_c1 = -1; s_before = 0; }
+            long long tot;
+            const long long excl = block_excl_scan(local, s_scan, &tot);
+            if (excl < need && need <= excl + local) {
+                long long acc = excl;
+                for (int q = 0; q < CPT; ++q) {
+                    const long long c = threadIdx.x * CPT + q;
+                    if (need <= acc + cs[c]) {
+                        s_c0 = U.tile_begin + c * per_c;
+                        s_c1 = min(U.tile_end, s_c0 + per_c);
+                        s_before = acc;
+                        break;
+                    }
+                    acc += cs[c];
+                }
+            }
+            __syncthreads();
+            if (s_c0 >= 0) { lo_t = s_c0; hi_t = s_c1; need -= s_before; }
+        }
+        const long long nt = hi_t - lo_t;
         const long long per = (nt + blockDim.x - 1) / blockDim.x;
-        const long long j0 = U.tile_begin + threadIdx.x * per;
-        const long long j1 = (j0 + per < U.tile_end) ? j0 + per : U.tile_end;
-        const uint32_t* src = ((U.tie_src == TIE_EQ_HI) ? P.teq_hi : (U.tie_src == TIE_EQ_LO) ? P.teq_lo : P.tcnt) +
-                              (long long)i * P.n_tiles;
+        const long long j0 = lo_t + threadIdx.x * per;
+        const long long j1 = (j0 + per < hi_t) ? j0 + per : hi_t;
         auto tile_ties = [&](long long g) -> long long { return src[g]; };
         long long local = 0;
         {
@@ -1138,11 +1303,11 @@ __global__ void __launch_bounds__(CUT_TPB) k_cut(Plan P) {
         }
         long long total;
         const long long excl = block_excl_scan(local, s_scan, &total);
-        if (excl < U.need && U.need <= excl + local) {
+        if (excl < need && need <= excl + local) {
             long long acc = excl;
             for (long long g = j0; g < j1; ++g) {
                 const long long cnt = tile_ties(g);
-                if (U.need <= acc + cnt) { s_tile = g; s_rem = U.need - acc; break; }
+                if (need <= acc + cnt) { s_tile = g; s_rem = need - acc; break; }
                 acc += cnt;
             }
         }

@@ -422,3 +422,25 @@ def test_fused_bf16_delta_input_mixed_list():
     taus = [t.to(torch.bfloat16) for t in _taus(MIXED, 34, torch.float32)]
     for op in ("ties", "iso"):
         _update_vs_oracle(th0, taus, op, 0.05, is_delta=True, what=f"bf16 delta {op}")
+
+
+LARGE_GLOBAL = [(4096, 8192, False), (1, 4096, True), (4096, 8192, False), (3000, 7001, False)]
+
+
+@pytest.mark.parametrize("op,density", [("ties", 0.2), ("iso", 0.05), ("ties", 0.5)])
+def test_global_unit_with_a_large_pool_and_many_tiles(op, density):
+    # one GLOBAL unit of 88 M entries: more than 65536 tiles (the cut picks
+    # its chunk from per-chunk tie sums first) and a band of candidates above
+    # 2^20 keys (histogrammed as one flat pool, the count pass sealing the
+    # unused slots of its chunks); bf16 checkpoints give long runs of ties
+    th0, th1 = synth.rl_update_set(LARGE_GLOBAL, seed=43)
+    d0, d1 = [t.to(DEV) for t in th0], [t.to(DEV) for t in th1]
+    out, st = iso.iso_update(d0, d1, op=op, update_is_delta=False, density=density, scope="global",
+                             lam=1.0, stats=True)
+    torch.cuda.synchronize()
+    r = oracle.update(_np_list(th0), _np_list(th1), OPS[op], update_is_delta=False, density=density,
+                      scope=oracle.SCOPE_GLOBAL, lam=1.0, shapes=_shapes(LARGE_GLOBAL), is_1d=_is1d(LARGE_GLOBAL))
+    _check_merge(out, st, r, th0, OPS[op], 1, what=f"large global {op} {density}")
+    u = st.units_numpy()[0, 0]
+    if op == "ties":
+        assert u["ties_at_thresh"] > u["ties_taken"] > 0     # the cut splits a run of ties
