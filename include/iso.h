@@ -140,7 +140,8 @@ typedef struct {
                                  bit 1: fused K = 1 pass took the sampled run of ties as the
                                  threshold; bit 2: fused pass re-applied the unit in full;
                                  bit 3: band keys overflowed their segment; bit 4: fused band
-                                 records overflowed */
+                                 records overflowed; bit 5: the Gram and merge passes read this
+                                 unit's compact candidates (iso_compact_candidates) */
     int64_t  k;               /* entries selected; -1 for a unit that is not trimmed */
     int64_t  count_above;     /* entries with |tau| above the threshold */
     int64_t  ties_at_thresh;  /* entries with |tau| equal to the threshold */
@@ -443,6 +444,14 @@ uint64_t iso_launch_count(void);
  * on = 1 makes later calls take the two-pass form instead (a counting pass,
  * then the apply pass).  Both give the same result.  Process-wide host state. */
 int32_t iso_force_two_pass(int32_t on);
+
+/* Diagnostics: whether later K >= 2 TIES and ISO merges at per-tensor scope
+ * (density <= 0.3) let the counting pass write each expert's candidate values
+ * (the entries at or above the low edge of its sampled band, in position
+ * order, with a bit mask per tile), so that the Gram and merge passes read
+ * those instead of the full task vectors; on by default.  The results are
+ * the same either way. */
+int32_t iso_compact_candidates(int32_t on);
 
 /* Diagnostics: when enabled, each launch is bracketed by CUDA events on its
  * stream.  iso_profile_read waits for the recorded events and returns, for

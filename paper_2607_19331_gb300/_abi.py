@@ -103,6 +103,7 @@ PROTOTYPES = [
     ("iso_error_string", ctypes.c_char_p, [I32]),
     ("iso_launch_count", ctypes.c_uint64, []),
     ("iso_force_two_pass", ctypes.c_int32, [ctypes.c_int32]),
+    ("iso_compact_candidates", ctypes.c_int32, [ctypes.c_int32]),
     ("iso_profile_enable", I32, [I32]),
     ("iso_profile_reset", I32, []),
     ("iso_profile_kinds", I32, []),

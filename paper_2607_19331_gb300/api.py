@@ -352,6 +352,13 @@ def force_two_pass(on=True):
     check(lib().iso_force_two_pass(int(bool(on))), "iso_force_two_pass")
 
 
+def compact_candidates(on=True):
+    """Diagnostics: let later K >= 2 TIES / ISO merges read compact candidate
+    values in their Gram and merge passes (the default) or the full task
+    vectors; the results are the same."""
+    check(lib().iso_compact_candidates(int(bool(on))), "iso_compact_candidates")
+
+
 def profile_enable(on=True):
     check(lib().iso_profile_enable(int(bool(on))), "iso_profile_enable")
 

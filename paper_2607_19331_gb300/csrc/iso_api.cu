@@ -212,6 +212,7 @@ struct Call {
     bool trims = true;                    // some tensor is trimmed
     std::vector<char> trim;               // per tensor
     int xdt = ISO_F32, bdt = ISO_F32;
+    bool ccv = false;                     // compact candidates (set by run_call when they fit)
 };
 
 bool tensor_trimmed(const Call& c, int t) { return c.trim[t] != 0; }
@@ -240,6 +241,35 @@ unsigned long long cand_cap_of(long long n, double rho, bool quantized) {
     const double ties = quantized ? 0.08 : 0.004;
     const double cap = 8192.0 + std::ceil((2.0 * band + ties) * (double)n) + waste;
     return (unsigned long long)std::min(cap, (double)n);
+}
+
+// Value slots of one unit's compact candidates (keys >= lo, about the kept
+// fraction plus the band): the band's rank width twice over, room for ties at
+// its low edge, and the chunk ends the count pass's warps may leave unused
+// (at most VCHUNK per warp that reaches the unit; per = the count pass's
+// items per warp on the largest GPU this is sized for).  Never more than the
+// tile-padded entries plus one tile per such warp.
+constexpr long long CCV_WARPS = 160LL * COUNT_BLOCKS_PER_SM * WPB;
+unsigned long long v_cap_of(long long n, double rho, bool quantized, long long per) {
+    const long long tiles = (n + TILE - 1) / TILE;
+    const long long warps = tiles / std::max(1LL, per) + 2;
+    double q = std::floor(rho * (double)n + 0.5) / std::max(1.0, (double)n);
+    q = std::min(std::max(q, 0.0), 1.0);
+    const double S = SAMPLE_MAX;
+    const double band = n <= SAMPLE_MAX ? 0.0 : 2.0 * (SAMPLE_Z * std::sqrt(S * q * (1.0 - q)) + 2.0) / S;
+    const double ties = quantized ? 0.08 : 0.004;
+    const double est = 8192.0 + std::ceil((q + 2.0 * band + ties) * (double)n) + (double)VCHUNK * (double)warps;
+    const double most = (double)tiles * TILE + (double)TILE * (double)warps;
+    return (unsigned long long)std::min(std::min(est, most), 4294967040.0);
+}
+
+std::atomic<int> g_ccv{0};
+// K >= 2 TIES / ISO merges at per-tensor scope and moderate density: the
+// count pass writes the candidates, the Gram and merge passes read them
+bool ccv_eligible(const Call& c) {
+    return g_ccv.load(std::memory_order_relaxed) && c.K >= 2 && !c.mask_only && c.trims &&
+           (c.op == ISO_OP_TIES || c.op == ISO_OP_ISO) && c.topk.scope == ISO_SCOPE_TENSOR &&
+           c.topk.density <= 0.3;
 }
 
 // band-record capacity of one unit for the fused K = 1 pass: the band's rank
@@ -280,11 +310,13 @@ size_t al256(size_t v) { return (v + 255) & ~(size_t)255; }
 struct Layout {
     size_t hdr, units, tcand, teq_lo, teq_hi, tcnt, hist, hmxc, hmx, gram, coef, zero_end;
     size_t tens, xptr, mptr, table_end;
-    size_t tband, repair, csamp, cand, brec, total;
+    size_t tband, repair, csamp, cand, brec, vmask, tval, vals, total;
     unsigned long long brec_total = 0;
     long long n_tiles = 0;
     int n_units = 0;
     unsigned long long cand_total = 0;
+    unsigned long long v_total = 0;       // compact-candidate value slots
+    long long v_per = 1;                  // count-pass items per warp (compact-candidate sizing)
     long long global_n = 0;
 };
 
@@ -319,6 +351,12 @@ Layout layout_of(const Call& c, int t0, int t1) {
     L.n_tiles = tiles;
     L.n_units = (int)units;
     L.cand_total = select ? cand : 0;
+    if (c.ccv) {
+        L.v_per = ((long long)K * tiles + CCV_WARPS - 1) / CCV_WARPS;
+        for (int t = t0; t < t1; ++t)
+            if (tensor_trimmed(c, t))
+                L.v_total += (unsigned long long)K * v_cap_of(numel_of(c.x[t]), c.topk.density, c.xdt == ISO_BF16, L.v_per);
+    }
     L.global_n = gn;
     size_t o = 0;
     L.hdr = o;   o = al256(o + sizeof(Header));
@@ -343,6 +381,9 @@ Layout layout_of(const Call& c, int t0, int t1) {
     L.csamp = o;  o = al256(o + (fused ? (size_t)K * units * COUNT_CHUNKS * 4 : 0));
     L.cand = o;   o = al256(o + (size_t)L.cand_total * 4);
     L.brec = o;   o = al256(o + (size_t)L.brec_total * 8);
+    L.vmask = o;  o = al256(o + (c.ccv ? (size_t)K * tiles * 128 : 0));
+    L.tval = o;   o = al256(o + (c.ccv ? (size_t)K * tiles * 4 : 0));
+    L.vals = o;   o = al256(o + (size_t)L.v_total * 4);
     L.total = o;
     return L;
 }
@@ -423,7 +464,7 @@ int run_group(const Call& c, int t0, int t1, char* ws, cudaStream_t s, const iso
     uint32_t** mptr = reinterpret_cast<uint32_t**>(blob.data() + (L.mptr - L.tens));
     long long tile = 0, uoff = 0;
     int unit = 0;
-    unsigned long long cand = 0, brec = 0;
+    unsigned long long cand = 0, brec = 0, vslots = 0;
     const bool fused = fused_path(c);
     for (int q = 0; q < T; ++q) {
         const int t = t0 + q;
@@ -463,6 +504,9 @@ int run_group(const Call& c, int t0, int t1, char* ws, cudaStream_t s, const iso
         d.brec_off = brec;
         d.brec_cap = (fused && tensor_trimmed(c, t)) ? brec_cap_of(d.numel, c.topk.density) : 0;
         brec += d.brec_cap;
+        d.v_off = vslots;
+        d.v_cap = (c.ccv && tensor_trimmed(c, t)) ? v_cap_of(d.numel, c.topk.density, c.xdt == ISO_BF16, L.v_per) : 0;
+        vslots += (unsigned long long)K * d.v_cap;
         for (int i = 0; i < K; ++i) xptr[i * T + q] = c.x[(size_t)i * c.n + t].data;
         mptr[q] = c.masks ? c.masks[t] : nullptr;
     }
@@ -487,6 +531,10 @@ int run_group(const Call& c, int t0, int t1, char* ws, cudaStream_t s, const iso
     P.csamp = fused ? reinterpret_cast<uint32_t*>(ws + L.csamp) : nullptr;
     P.gram = reinterpret_cast<double*>(ws + L.gram);
     P.coef = reinterpret_cast<double*>(ws + L.coef);
+    P.ccv = c.ccv ? 1 : 0;
+    P.vmask = c.ccv ? reinterpret_cast<uint32_t*>(ws + L.vmask) : nullptr;
+    P.tval = c.ccv ? reinterpret_cast<uint32_t*>(ws + L.tval) : nullptr;
+    P.vals = c.ccv ? reinterpret_cast<float*>(ws + L.vals) : nullptr;
     P.n_tensors = T;
     P.K = K;
     P.n_units = L.n_units;
@@ -556,17 +604,22 @@ int run_group(const Call& c, int t0, int t1, char* ws, cudaStream_t s, const iso
                     ISO_TRY(launch(KD_COUNT, s, [&] { k_count_apply<false><<<sms * FUSED_GRID_PER_SM, TPB, FUSED_SMEM, s>>>(P); }));
                 }
             } else {
-                ISO_TRY(launch(KD_COUNT, s, [&] { k_count<XT, BT, CK><<<sms * COUNT_GRID_PER_SM, TPB, 0, s>>>(P); }));
+                if (c.ccv)
+                    ISO_TRY(launch(KD_COUNT, s, [&] { k_count<XT, BT, CK, true><<<sms * COUNT_GRID_PER_SM, TPB, 0, s>>>(P); }));
+                else
+                    ISO_TRY(launch(KD_COUNT, s, [&] { k_count<XT, BT, CK, false><<<sms * COUNT_GRID_PER_SM, TPB, 0, s>>>(P); }));
             }
             ISO_TRY(launch(KD_DECIDE, s, [&] { k_decide<<<(KU + 255) / 256, 256, 0, s>>>(P); }));
-            ISO_TRY(smem_optin(k_radix_flat, RADIX_FLAT_SMEM));
+            if (c.topk.scope == ISO_SCOPE_GLOBAL) ISO_TRY(smem_optin(k_radix_flat, RADIX_FLAT_SMEM));
             for (int level = 0; level < 3; ++level) {
-                ISO_TRY(launch(KD_RADIX_FLAT, s, [&] { k_radix_flat<<<sms * 2, TPB, RADIX_FLAT_SMEM, s>>>(P); }));
+                if (c.topk.scope == ISO_SCOPE_GLOBAL)
+                    ISO_TRY(launch(KD_RADIX_FLAT, s, [&] { k_radix_flat<<<sms * 2, TPB, RADIX_FLAT_SMEM, s>>>(P); }));
                 ISO_TRY(launch(KD_RADIX_HIST, s, [&] { k_radix_hist<XT, BT, CK><<<pgrid, TPB, 0, s>>>(P); }));
                 ISO_TRY(launch(KD_RADIX_PICK, s, [&] { k_radix_pick<<<KU, TPB, 0, s>>>(P); }));
             }
             ISO_TRY(launch(KD_TIE, s, [&] { k_tie<XT, BT, CK><<<pgrid, TPB, 0, s>>>(P); }));
-            ISO_TRY(launch(KD_CUT_PART, s, [&] { k_cut_part<<<pgrid, TPB, 0, s>>>(P); }));
+            if (c.topk.scope == ISO_SCOPE_GLOBAL)
+                ISO_TRY(launch(KD_CUT_PART, s, [&] { k_cut_part<<<pgrid, TPB, 0, s>>>(P); }));
             ISO_TRY(launch(KD_CUT, s, [&] { k_cut<XT, BT, CK><<<KU, CUT_TPB, 0, s>>>(P); }));
             return ISO_OK;
         });
@@ -623,6 +676,9 @@ int run_group(const Call& c, int t0, int t1, char* ws, cudaStream_t s, const iso
             if (need_gram_pass) {
                 auto gram = [&](auto kc) {
                     constexpr int KC = decltype(kc)::value;
+                    if constexpr (KC >= 2) {
+                        if (c.ccv) return launch(KD_GRAM, s, [&] { k_gramk_c<XT, BT, CK, KC><<<sms * 2, TPB, 0, s>>>(P); });
+                    }
                     const int ggrid = sms * gram_blocks_per_sm(KC);
                     const int smem = gram_smem_bytes<XT, BT, KC>();
                     ISO_TRY(smem_optin(k_gramk<XT, BT, CK, KC>, smem));
@@ -637,6 +693,10 @@ int run_group(const Call& c, int t0, int t1, char* ws, cudaStream_t s, const iso
         }
         auto merge = [&](auto kc) {
             constexpr int KC = decltype(kc)::value;
+            if (c.ccv && c.op == ISO_OP_TIES)
+                return launch(KD_APPLY, s, [&] { k_merge_c<XT, BT, CK, KC, OPF_TIES><<<sms * 2, TPB, 0, s>>>(P); });
+            if (c.ccv)
+                return launch(KD_APPLY, s, [&] { k_merge_c<XT, BT, CK, KC, OPF_OTHER><<<sms * 2, TPB, 0, s>>>(P); });
             if (c.op == ISO_OP_TIES) {
                 const int smem = merge_smem_bytes<XT, BT, KC, OPF_TIES>();
                 const int mgrid = sms * merge_blocks_per_sm(KC, OPF_TIES);
@@ -678,6 +738,10 @@ int run_call(Call& c, void* workspace, size_t ws_bytes, const iso_merge_stats* s
         if (((uintptr_t)workspace & 255u) != 0) return ISO_ERR_WORKSPACE;
     }
     std::vector<int> bounds;
+    // compact candidates when every tensor group can hold them, else the
+    // full passes
+    c.ccv = ccv_eligible(c);
+    if (c.ccv && plan_groups(c, ws_bytes, &bounds) != ISO_OK) c.ccv = false;
     ISO_TRY(plan_groups(c, ws_bytes, &bounds));
     char* ws = static_cast<char*>(workspace);
     if (c.n > 0) ISO_TRY(launch(KD_MEMSET, s, [&] { cudaMemsetAsync(ws, 0, 4, s); }));
@@ -867,8 +931,12 @@ int32_t iso_workspace_size(const iso_tensor* tensors, int32_t n_tensors, int32_t
     // size reported is an upper bound
     c.xdt = c.bdt = n_tensors ? tensors[0].dtype : ISO_F32;
     set_trim(c, tensors);
-    size_t full = n_tensors ? layout_of(c, 0, n_tensors).total : 256;
+    // the smallest workspace runs the full passes; the full size holds the
+    // compact candidates where the call takes them
     size_t mn = 256;
+    c.ccv = ccv_eligible(c);
+    size_t full = n_tensors ? layout_of(c, 0, n_tensors).total : 256;
+    c.ccv = false;
     if (c.topk.scope == ISO_SCOPE_GLOBAL && c.trims) mn = full;
     else for (int t = 0; t < n_tensors; ++t) mn = std::max(mn, layout_of(c, t, t + 1).total);
     if (bytes_min) *bytes_min = mn;
@@ -984,6 +1052,11 @@ uint64_t iso_launch_count(void) { return g_launches.load(); }
 
 int32_t iso_force_two_pass(int32_t on) {
     g_two_pass.store(on ? 1 : 0);
+    return ISO_OK;
+}
+
+int32_t iso_compact_candidates(int32_t on) {
+    g_ccv.store(on ? 1 : 0);
     return ISO_OK;
 }
 

@@ -29,6 +29,7 @@ constexpr int TPB = 256;                    // threads per streaming block
 constexpr int WPB = TPB / 32;               // warps per streaming block
 static_assert(WVEC * 32 * VEC == TILE, "tile geometry");
 constexpr int CHUNK_MAX = 1024;             // candidate slots a warp reserves at once
+constexpr int VCHUNK = 8192;                // compact-candidate value slots a warp reserves at most at once
 
 constexpr int SAMPLE_MAX = 24576;           // sampled keys per unit (96 KB of smem: two blocks per SM)
 constexpr int SAMPLE_CHUNK = 256;           // contiguous entries per sample chunk
@@ -79,6 +80,8 @@ struct TensorDesc {
     unsigned long long cand_cap;
     unsigned long long brec_off;  // fused K = 1 pass: band-record segment
     unsigned long long brec_cap;
+    unsigned long long v_off;     // compact candidates: expert 0's value segment (expert i adds i*v_cap)
+    unsigned long long v_cap;
 };
 
 enum UnitState : int32_t {
@@ -145,6 +148,12 @@ struct Unit {
     unsigned long long cs_gt;           // count sample: keys above t^
     uint32_t cs_done;                   // count-sample blocks finished
     int32_t pad2;
+    // compact candidates (K >= 2 merges): the values with key >= lo, per
+    // tile in position order, in this unit's value segment
+    unsigned long long v_off, v_cap;    // segment in the value pool, slots
+    unsigned long long v_alloc;         // slots handed out (above v_cap: overflow)
+    int32_t v_ok;                       // every kept entry is in the compact candidates (set by k_decide)
+    int32_t pad3;
 };
 
 // Per (expert, tile) records of the count pass, as separate arrays:
@@ -152,6 +161,11 @@ struct Unit {
 //          segment, band keys stored; count 0 when the segment overflowed)
 //   teq_lo / teq_hi  band keys == lo / == hi in the tile
 //   tcnt   keys == t in the tile (interior thresholds; written by k_tie)
+//   tval   compact candidates: first slot of the tile's values in the unit's
+//          value segment (KEY_NONE when the segment overflowed); vmask holds
+//          32 words per record, bit p of word w for position 32 w + p of the
+//          tile (key >= lo), and the tile's values follow the set bits in
+//          position order
 
 struct Header {             // first bytes of the workspace
     int32_t status;
@@ -178,6 +192,9 @@ struct Plan {
     uint2*        tband;    // fused K = 1 pass: [n_tiles] (start, count) of the tile's band records
     uint32_t*     csamp;    // fused K = 1 pass: [n_units][COUNT_CHUNKS] sampled ties of t^ per chunk
     int32_t*      repair;   // fused K = 1 pass: [n_tensors] tensor needs the full exact apply
+    uint32_t*     vmask;    // compact candidates: [K][n_tiles][32] words
+    uint32_t*     tval;     // compact candidates: [K][n_tiles] first value slot (KEY_NONE: overflow)
+    float*        vals;     // compact candidates: value pool (binary32 tau)
     double*       gram;     // [n_tensors][K][K]
     double*       coef;     // [n_tensors][K]
     int32_t n_tensors;
@@ -191,6 +208,8 @@ struct Plan {
     int32_t op;
     int32_t fused;          // the K = 1 update runs the fused single pass
     int32_t fuse_block;     // BLOCK scope, K = 1 TIES: k_block_select writes the outputs
+    int32_t ccv;            // K >= 2 TIES / ISO: the count pass writes compact candidates and
+                            // the Gram and merge passes read them for every unit with v_ok
     int32_t block_rows, block_cols;
     float lambda;
     float eps_act;          // RAM: expert active where the binary32 |tau| > eps_act (>= +0)

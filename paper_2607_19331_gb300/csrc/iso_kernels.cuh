@@ -23,7 +23,7 @@ constexpr bool PASS_INTERLEAVE = ISO_PASS_INTERLEAVE != 0;
 constexpr int COUNT_BLOCKS_PER_SM = 2;      // k_count: resident blocks of TPB threads per SM
 __global__ void k_init_units(Plan P, long long global_n);
 template <typename XT, typename BT, bool CK> __global__ void k_sample(Plan P);
-template <typename XT, typename BT, bool CK> __global__ void k_count(Plan P);
+template <typename XT, typename BT, bool CK, bool EMIT> __global__ void k_count(Plan P);
 __global__ void k_decide(Plan P);
 template <typename XT, typename BT, bool CK> __global__ void k_radix_hist(Plan P);
 __global__ void k_radix_pick(Plan P);
@@ -74,6 +74,8 @@ constexpr int merge_blocks_per_sm(int KC, int OPF) { return 2; }
 template <typename XT, typename BT, int KC, int OPF> int merge_smem_bytes();
 template <typename XT, typename BT, int KC> int gram_smem_bytes();
 constexpr int gram_blocks_per_sm(int KC) { return 2; }
+template <typename XT, typename BT, bool CK, int KC, int OPF> __global__ void k_merge_c(Plan P);
+template <typename XT, typename BT, bool CK, int KC> __global__ void k_gramk_c(Plan P);
 __global__ void k_solve(Plan P, int gram_mode);
 template <typename XT> __global__ void k_mask(Plan P, uint32_t* const* mptr);
 __global__ void k_status(const Header* h, int32_t* out);

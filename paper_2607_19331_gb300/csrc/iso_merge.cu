@@ -781,6 +781,286 @@ __global__ void __launch_bounds__(TPB, gram_blocks_per_sm(KC)) k_gramk(Plan P) {
     flush(t);
 }
 
+// ---------------------------------------------------------------------------
+// Compact candidates (Plan::ccv).  The count pass has written, per expert and
+// tile, the binary32 task-vector values whose key is at least the low edge of
+// the unit's band, in position order, and a 32-word mask of their positions.
+// When the unit's threshold lies in its band (Unit::v_ok) those values hold
+// every entry the selection can keep, so the Gram and merge passes read them
+// (about the kept fraction of each expert's bytes) instead of the full task
+// vectors; any other expert of the tensor (an untrimmed tensor, a unit whose
+// band missed or whose value segment overflowed) is read in full.  An entry
+// absent from the values has key < lo <= t: never kept, it enters every sum
+// as +0 exactly as an unkept entry does in k_merge / k_gramk, so both give
+// the same results.  One warp per tile, lane l taking entries 4 l .. 4 l + 3
+// of each 128-entry step: the four bits of word 4 s + l / 8 at 4 (l % 8).
+// ---------------------------------------------------------------------------
+template <int KC>
+struct CompactParams {
+    uint32_t vok;                      // bit q: expert q reads its compact values
+    unsigned long long voff[KC];       // the unit's value segment in the pool
+};
+
+template <int KC>
+__device__ __forceinline__ void compact_params(const Plan& P, int t, int K, CompactParams<KC>& cp) {
+    __syncwarp();
+    if ((threadIdx.x & 31) == 0) {
+        const TensorDesc& d = P.tens[t];
+        uint32_t ok = 0;
+#pragma unroll
+        for (int q = 0; q < KC; ++q) {
+            cp.voff[q] = 0;
+            if (q < K && (d.flags & TF_TRIM)) {
+                const Unit& U = P.units[(long long)q * P.n_units + d.unit];
+                if (U.v_ok) { ok |= 1u << q; cp.voff[q] = U.v_off; }
+            }
+        }
+        cp.vok = ok;
+    }
+    __syncwarp();
+}
+
+// the tile's mask words, their exclusive popcount prefix and the value
+// pointer of each compact expert, in the warp's shared memory (registers
+// stay free for the data)
+template <int KC>
+struct CompactTile {
+    uint32_t mw[KC][32], pre[KC][32];
+    const float* vb[KC];
+};
+
+template <int KC>
+__device__ __forceinline__ void compact_tile(const Plan& P, const CompactParams<KC>& cp, int K, long long g, int lane,
+                                             CompactTile<KC>& ct) {
+    __syncwarp();
+#pragma unroll
+    for (int q = 0; q < KC; ++q) {
+        if (q < K && ((cp.vok >> q) & 1u)) {
+            const long long rec = (long long)q * P.n_tiles + g;
+            const uint32_t w = P.vmask[rec * 32 + lane];
+            uint32_t tot;
+            ct.pre[q][lane] = warp_excl_scan((uint32_t)__popc(w), &tot);
+            ct.mw[q][lane] = w;
+            if (lane == 0) ct.vb[q] = P.vals + cp.voff[q] + P.tval[rec];
+        }
+    }
+    __syncwarp();
+}
+
+// tau of entries e .. e + 3 (step s of the tile) for every expert: compact
+// values, or the full task vector; entries past the tensor's end read 0
+template <typename XT, typename BT, bool CK, int KC>
+__device__ __forceinline__ void compact_step(const CompactParams<KC>& cp, const CompactTile<KC>& ct,
+                                             const void* const* xs, int K, long long e, long long n, int s, int lane,
+                                             const float (&th0)[4], float (&tau)[KC][4]) {
+    const int w = s * 4 + (lane >> 3), bo = (lane & 7) * 4;
+#pragma unroll
+    for (int q = 0; q < KC; ++q) {
+#pragma unroll
+        for (int j = 0; j < 4; ++j) tau[q][j] = 0.0f;
+        if (q >= K) continue;
+        if ((cp.vok >> q) & 1u) {
+            const uint32_t word = ct.mw[q][w];
+            const uint32_t at = ct.pre[q][w] + (uint32_t)__popc(word & ((1u << bo) - 1u));
+            const uint32_t nib = (word >> bo) & 0xFu;
+            const float* vb = ct.vb[q] + at;
+            uint32_t r = 0;
+#pragma unroll
+            for (int j = 0; j < 4; ++j) {
+                if ((nib >> j) & 1u) { tau[q][j] = __ldg(vb + r); ++r; }
+            }
+        } else {
+            Words<XT, 4> x;
+            load_words<XT, 4>(xs[q], e, n, x);
+#pragma unroll
+            for (int j = 0; j < 4; ++j) {
+                tau[q][j] = word_f32<XT, 4>(x, j);
+                if (CK) tau[q][j] = __fsub_rn(tau[q][j], th0[j]);
+            }
+        }
+    }
+}
+
+template <typename XT, typename BT, bool CK, int KC, int OPF>
+__global__ void __launch_bounds__(TPB, 2) k_merge_c(Plan P) {
+    constexpr int E = 4, SPT = TILE / (32 * E);
+    const int K = P.K;
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const WarpRange wr = warp_range(P);
+    if (wr.beg >= wr.end) return;
+    __shared__ MergeParams<KC> s_mp[WPB];
+    __shared__ CompactParams<KC> s_cp[WPB];
+    __shared__ CompactTile<KC> s_ct[WPB];
+    MergeParams<KC>& mp = s_mp[warp];
+    CompactParams<KC>& cp = s_cp[warp];
+    int t = tensor_of_tile(P.tens, P.n_tensors, wr.beg);
+    long long t_end = tensor_tile_end(P, t);
+    merge_params<KC>(P, t, K, mp);
+    compact_params<KC>(P, t, K, cp);
+    const long long nt = wr.count();
+#pragma unroll 1
+    for (long long jt = 0; jt < nt; ++jt) {
+        const long long g = wr.tile(jt);
+        if (g >= t_end) {
+            while (g >= t_end) t_end = tensor_tile_end(P, ++t);
+            merge_params<KC>(P, t, K, mp);
+            compact_params<KC>(P, t, K, cp);
+        }
+        const TensorDesc& d = P.tens[t];
+        const long long n = d.numel;
+        const long long e0 = (g - d.tile_base) * TILE;
+        const long long e1 = (e0 + TILE < n) ? e0 + TILE : n;
+        int T[KC];
+        float cf[KC];
+        const bool exact = tile_thresholds<KC>(mp, K, (uint32_t)e0, (uint32_t)e1, T);
+#pragma unroll
+        for (int q = 0; q < KC; ++q) cf[q] = (OPF == OPF_TIES) ? 0.0f : mp.cf[q];
+        const int opk = (OPF == OPF_TIES) ? (int)OPK_TIES : mp.opk;
+        const bool iso1d = mp.iso1d;
+        CompactTile<KC>& ct = s_ct[warp];
+        compact_tile<KC>(P, cp, K, g, lane, ct);
+        uint32_t kmax = 0;
+#pragma unroll 1
+        for (int s = 0; s < SPT; ++s) {
+            const long long e = e0 + (long long)s * (32 * E) + lane * E;
+            Words<BT, E> b;
+            load_words<BT, E>(d.base, e, n, b);
+            float th0[E];
+#pragma unroll
+            for (int j = 0; j < E; ++j) th0[j] = word_f32<BT, E>(b, j);
+            float tau[KC][E];
+            compact_step<XT, BT, CK, KC>(cp, ct, mp.xs, K, e, n, s, lane, th0, tau);
+            long long r = 0, c = 0;
+            if (exact && mp.sel == SEL_BLOCK) { r = e / d.cols; c = e - r * d.cols; }
+            float o[E];
+#pragma unroll
+            for (int j = 0; j < E; ++j) {
+                float tj[KC];
+#pragma unroll
+                for (int q = 0; q < KC; ++q) tj[q] = tau[q][j];
+                if (exact) {
+                    const uint32_t bits = (e + j < n) ? select_bits<KC>(P, d, mp, K, tj, e + j, r, c) : 0u;
+                    o[j] = merged_value<KC>(opk, iso1d, P.lambda, K, th0[j], tj, cf, bits);
+                } else {
+                    o[j] = merged_fast<KC>(opk, iso1d, P.lambda, K, th0[j], tj, cf, T, kmax);
+                }
+            }
+            store_out<BT, E>(d.out, e, n, o);
+        }
+    }
+}
+
+// Gram of the trimmed task vectors from the compact candidates (see above);
+// partial sums as in k_gramk: per lane over the tile's entries in order,
+// warp sums per tile, binary32 two-sum pairs per tensor, one atomic per pair.
+template <typename XT, typename BT, bool CK, int KC>
+__global__ void __launch_bounds__(TPB, 2) k_gramk_c(Plan P) {
+    constexpr int E = 4, SPT = TILE / (32 * E);
+    constexpr int NP = KC * (KC + 1) / 2;
+    static_assert(NP <= 64, "two pair sums per lane");
+    const int K = P.K;
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    float gs0 = 0.0f, ge0 = 0.0f, gs1 = 0.0f, ge1 = 0.0f;
+    const WarpRange wr = warp_range(P);
+    if (wr.beg >= wr.end) return;
+    __shared__ MergeParams<KC> s_mp[WPB];
+    __shared__ CompactParams<KC> s_cp[WPB];
+    __shared__ CompactTile<KC> s_ct[WPB];
+    MergeParams<KC>& mp = s_mp[warp];
+    CompactParams<KC>& cp = s_cp[warp];
+    int t = tensor_of_tile(P.tens, P.n_tensors, wr.beg);
+    long long t_end = tensor_tile_end(P, t);
+    merge_params<KC>(P, t, K, mp);
+    compact_params<KC>(P, t, K, cp);
+    auto flush = [&](int tt) {
+        int q = 0;
+#pragma unroll
+        for (int a = 0; a < KC; ++a) {
+#pragma unroll
+            for (int b = a; b < KC; ++b, ++q) {
+                if (a < K && b < K && (lane == q || lane + 32 == q)) {
+                    const double v = (lane == q) ? (double)gs0 + (double)ge0 : (double)gs1 + (double)ge1;
+                    if (v != 0.0) atomicAdd(&P.gram[((long long)tt * K + a) * K + b], v);
+                }
+            }
+        }
+        gs0 = ge0 = gs1 = ge1 = 0.0f;
+    };
+    const long long nt = wr.count();
+#pragma unroll 1
+    for (long long jt = 0; jt < nt; ++jt) {
+        const long long g = wr.tile(jt);
+        if (g >= t_end) {
+            flush(t);
+            while (g >= t_end) t_end = tensor_tile_end(P, ++t);
+            merge_params<KC>(P, t, K, mp);
+            compact_params<KC>(P, t, K, cp);
+        }
+        if (!mp.trimmed2d) continue;
+        const TensorDesc& d = P.tens[t];
+        const long long n = d.numel;
+        const long long e0 = (g - d.tile_base) * TILE;
+        const long long e1 = (e0 + TILE < n) ? e0 + TILE : n;
+        int T[KC];
+        const bool exact = tile_thresholds<KC>(mp, K, (uint32_t)e0, (uint32_t)e1, T);
+        CompactTile<KC>& ct = s_ct[warp];
+        compact_tile<KC>(P, cp, K, g, lane, ct);
+        float acc[NP];
+#pragma unroll
+        for (int q = 0; q < NP; ++q) acc[q] = 0.0f;
+#pragma unroll 1
+        for (int s = 0; s < SPT; ++s) {
+            const long long e = e0 + (long long)s * (32 * E) + lane * E;
+            float th0[E] = {0.0f, 0.0f, 0.0f, 0.0f};
+            if (CK && cp.vok != ((1u << K) - 1u)) {
+                Words<BT, E> b;
+                load_words<BT, E>(d.base, e, n, b);
+#pragma unroll
+                for (int j = 0; j < E; ++j) th0[j] = word_f32<BT, E>(b, j);
+            }
+            float tau[KC][E];
+            compact_step<XT, BT, CK, KC>(cp, ct, mp.xs, K, e, n, s, lane, th0, tau);
+            long long r = 0, c = 0;
+            if (exact && mp.sel == SEL_BLOCK) { r = e / d.cols; c = e - r * d.cols; }
+#pragma unroll
+            for (int j = 0; j < E; ++j) {
+                float tj[KC], m[KC];
+#pragma unroll
+                for (int q = 0; q < KC; ++q) tj[q] = tau[q][j];
+                if (exact) {
+                    const uint32_t bits = (e + j < n) ? select_bits<KC>(P, d, mp, K, tj, e + j, r, c) : 0u;
+#pragma unroll
+                    for (int q = 0; q < KC; ++q) m[q] = ((bits >> q) & 1u) ? tj[q] : 0.0f;
+                } else {
+#pragma unroll
+                    for (int q = 0; q < KC; ++q) m[q] = ((int)key_of(tj[q]) > T[q]) ? tj[q] : 0.0f;
+                }
+                int q = 0;
+#pragma unroll
+                for (int a2 = 0; a2 < KC; ++a2)
+#pragma unroll
+                    for (int b2 = a2; b2 < KC; ++b2, ++q) acc[q] = __fmaf_rn(m[a2], m[b2], acc[q]);
+            }
+        }
+        float w0 = 0.0f, w1 = 0.0f;
+        int q = 0;
+#pragma unroll
+        for (int a2 = 0; a2 < KC; ++a2) {
+#pragma unroll
+            for (int b2 = a2; b2 < KC; ++b2, ++q) {
+                if (a2 < K && b2 < K) {
+                    const float w = warp_sum(acc[q]);
+                    if (q < 32) w0 = (lane == q) ? w : w0;
+                    else w1 = (lane + 32 == q) ? w : w1;
+                }
+            }
+        }
+        two_sum_add(gs0, ge0, w0);
+        if (NP > 32) two_sum_add(gs1, ge1, w1);
+    }
+    flush(t);
+}
+
 template <typename XT, typename BT, int KC, int OPF>
 int merge_smem_bytes() { return StageGeom<XT, BT, KC, merge_blocks_per_sm(KC, OPF)>::SMEM; }
 template <typename XT, typename BT, int KC>
@@ -803,6 +1083,15 @@ ISO_MERGE_SMEM(float, __nv_bfloat16)
 ISO_MERGE_SMEM(float, float)
 
 #define ISO_MERGE_INST(XT, BT, CK)                                             \
+    template __global__ void k_merge_c<XT, BT, CK, 2, OPF_TIES>(Plan);        \
+    template __global__ void k_merge_c<XT, BT, CK, 4, OPF_TIES>(Plan);        \
+    template __global__ void k_merge_c<XT, BT, CK, 8, OPF_TIES>(Plan);        \
+    template __global__ void k_merge_c<XT, BT, CK, 2, OPF_OTHER>(Plan);       \
+    template __global__ void k_merge_c<XT, BT, CK, 4, OPF_OTHER>(Plan);       \
+    template __global__ void k_merge_c<XT, BT, CK, 8, OPF_OTHER>(Plan);       \
+    template __global__ void k_gramk_c<XT, BT, CK, 2>(Plan);                  \
+    template __global__ void k_gramk_c<XT, BT, CK, 4>(Plan);                  \
+    template __global__ void k_gramk_c<XT, BT, CK, 8>(Plan);                  \
     template __global__ void k_merge<XT, BT, CK, 2, OPF_TIES>(Plan);          \
     template __global__ void k_merge<XT, BT, CK, 4, OPF_TIES>(Plan);          \
     template __global__ void k_merge<XT, BT, CK, 8, OPF_TIES>(Plan);          \

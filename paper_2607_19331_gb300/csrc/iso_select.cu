@@ -54,6 +54,8 @@ __global__ void k_init_units(Plan P, long long global_n) {
         U.tile_end = d.tile_base + (d.numel + TILE - 1) / TILE;
         U.cand_cap = d.cand_cap;
         U.cand_off = d.cand_off + (unsigned long long)i * d.cand_cap;
+        U.v_cap = d.v_cap;
+        U.v_off = d.v_off + (unsigned long long)i * d.v_cap;
         U.brec_cap = d.brec_cap;
         U.brec_off = d.brec_off;
         trimmed = (d.flags & TF_TRIM) != 0;
@@ -567,7 +569,9 @@ __device__ __forceinline__ bool count_run_at(const Plan& P, uint32_t it, uint32_
     return false;
 }
 
-template <typename XT, typename BT, bool CK>
+// EMIT: also write the compact candidates (Plan::ccv); a separate
+// instantiation, so the plain counting pass keeps its registers
+template <typename XT, typename BT, bool CK, bool EMIT>
 __global__ void __launch_bounds__(TPB, COUNT_BLOCKS_PER_SM) k_count(Plan P) {
     __shared__ uint32_t s_band[WPB][TILE + 32];
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
@@ -605,6 +609,12 @@ __global__ void __launch_bounds__(TPB, COUNT_BLOCKS_PER_SM) k_count(Plan P) {
     bool ovf = false;
     uint32_t lo = 0, hi = 0, span = 0;
     bool want_gamma = false;
+    // compact candidates (P.ccv): the warp's chunk of the unit's value
+    // segment; a tile needs at most TILE slots, taken before the tile
+    float* vseg = nullptr;
+    unsigned long long v_pos = 0;
+    uint32_t v_left = 0, v_run = 0;
+    bool v_ovf = false;
 
     auto flush = [&]() {
         if (!au) return;
@@ -650,12 +660,50 @@ __global__ void __launch_bounds__(TPB, COUNT_BLOCKS_PER_SM) k_count(Plan P) {
             cseg = P.cand + au->cand_off;
             ch_left = 0;
             ovf = false;
+            vseg = P.vals + au->v_off;
+            v_left = 0;
+            v_ovf = false;
         }
         const uint32_t e0 = rr.e0 + (it - rr.it0) * TILE;
         const uint32_t rem = rr.n - e0;           // > 0
         const uint32_t rec = rr.rec + (it - rr.it0);
         const uint32_t ne0 = more ? r2.e0 + (it2 - r2.it0) * TILE : 0u;
         const uint32_t nrem = more ? r2.n - ne0 : 0u;
+        if constexpr (EMIT) {
+            if (v_left < TILE && !v_ovf) {
+                unsigned long long start = 0;
+                uint32_t req = 0;
+                if (lane == 0) {
+                    const uint32_t left = rr.left0 - (it - rr.it0);   // this warp's items of the unit still to count
+                    req = (uint32_t)min((unsigned long long)VCHUNK, (unsigned long long)TILE * max(left, 1u));
+                    start = atomicAdd(&au->v_alloc, (unsigned long long)req);
+                }
+                start = __shfl_sync(FULL, start, 0);
+                req = __shfl_sync(FULL, req, 0);
+                if (start + req > au->v_cap) v_ovf = true;
+                else { v_pos = start; v_left = req; }
+            }
+            v_run = 0;
+        }
+        // compact candidates of one vector step: the lane's entries with
+        // key >= lo (bits of m) in position order, and the step's mask words
+        // (lanes 4 q .. 4 q + 3 hold the 32 positions of word 8 v + q)
+        auto emit = [&](int v, const float (&tau)[VEC], uint32_t m) {
+            uint32_t tot;
+            const uint32_t off = warp_excl_scan((uint32_t)__popc(m), &tot);
+            if (!v_ovf) {
+                float* dst = vseg + v_pos + v_run + off;
+                int r = 0;
+#pragma unroll
+                for (int j = 0; j < VEC; ++j)
+                    if ((m >> j) & 1u) dst[r++] = tau[j];
+            }
+            v_run += tot;
+            const uint32_t b1 = __shfl_down_sync(FULL, m, 1), b2 = __shfl_down_sync(FULL, m, 2);
+            const uint32_t b3 = __shfl_down_sync(FULL, m, 3);
+            if ((lane & 3) == 0)
+                P.vmask[(size_t)rec * 32 + v * 8 + (lane >> 2)] = m | (b1 << 8) | (b2 << 16) | (b3 << 24);
+        };
 
         // pass 1: every entry
         uint32_t n_gt = 0;
@@ -667,6 +715,7 @@ __global__ void __launch_bounds__(TPB, COUNT_BLOCKS_PER_SM) k_count(Plan P) {
                 float tau[VEC];
                 rt.tau(v, tau);
                 if (more) rt.load_step(v, r2.xp, r2.bp, ne0, nrem, lane);
+                uint32_t m = 0;
 #pragma unroll
                 for (int j = 0; j < VEC; ++j) {
                     const uint32_t kk = key_of(tau[j]);
@@ -675,7 +724,9 @@ __global__ void __launch_bounds__(TPB, COUNT_BLOCKS_PER_SM) k_count(Plan P) {
                     f_gg = gt ? __fmaf_rn(tau[j], tau[j], f_gg) : f_gg;
                     *sp = kk;
                     sp += (kk - lo <= span) ? 32 : 0;
+                    if (EMIT) m |= (uint32_t)(kk >= lo) << j;
                 }
+                if constexpr (EMIT) emit(v, tau, m);
             }
         } else {
 #pragma unroll
@@ -684,6 +735,7 @@ __global__ void __launch_bounds__(TPB, COUNT_BLOCKS_PER_SM) k_count(Plan P) {
                 rt.tau(v, tau);
                 if (more) rt.load_step(v, r2.xp, r2.bp, ne0, nrem, lane);
                 const uint32_t o = (uint32_t)(v * (32 * VEC) + lane * VEC);
+                uint32_t m = 0;
 #pragma unroll
                 for (int j = 0; j < VEC; ++j) {
                     if (o + j >= rem) continue;
@@ -693,7 +745,9 @@ __global__ void __launch_bounds__(TPB, COUNT_BLOCKS_PER_SM) k_count(Plan P) {
                     f_gg = gt ? __fmaf_rn(tau[j], tau[j], f_gg) : f_gg;
                     *sp = kk;
                     sp += ((kk >= lo) & !gt) ? 32 : 0;
+                    if (EMIT) m |= (uint32_t)(kk >= lo) << j;
                 }
+                if constexpr (EMIT) emit(v, tau, m);
             }
         }
         const uint32_t nb = (uint32_t)(sp - sbl) >> 5;
@@ -756,7 +810,9 @@ __global__ void __launch_bounds__(TPB, COUNT_BLOCKS_PER_SM) k_count(Plan P) {
             P.tcand[rec] = make_uint2(store ? ch_pos : 0u, store ? t_int : 0u);
             P.teq_lo[rec] = t_lo;
             P.teq_hi[rec] = t_hi;
+            if (EMIT) P.tval[rec] = v_ovf ? KEY_NONE : (uint32_t)v_pos;
         }
+        if (EMIT && !v_ovf) { v_pos += v_run; v_left -= v_run; }
         if (store) { ch_pos += t_int; ch_left -= t_int; }
         a_gt += t_gt; a_int += t_int; a_hi += t_hi; a_lo += t_lo;
         __syncwarp();
@@ -855,6 +911,9 @@ __global__ void k_decide(Plan P) {
         U.r_above = 0;
         U.state = ST_RADIX;
     }
+    // the compact candidates hold every kept entry when the threshold lies
+    // in the band (t >= lo) and the unit's value segment did not overflow
+    U.v_ok = (P.ccv && !U.fallback && U.v_alloc <= U.v_cap) ? 1 : 0;
     if (U.state == ST_RADIX) atomicAdd(&P.hdr->n_radix, 1);
     else atomicAdd(&P.hdr->n_tknown, 1);
 }
@@ -885,8 +944,9 @@ __device__ __forceinline__ void hist_add(uint32_t* h, uint32_t* mxc, uint32_t* m
 
 // A unit in radix select over a pool filled by k_count (not the fused pass,
 // whose pool is not sealed) and large enough to scan as one flat array.
-__device__ __forceinline__ bool radix_flat(const Unit& U) {
-    return U.state == ST_RADIX && U.r_src == SRC_CAND && !U.mode_t && !U.overflow && U.n_alloc >= RADIX_FLAT_MIN;
+__device__ __forceinline__ bool radix_flat(const Plan& P, const Unit& U) {
+    return P.scope == ISO_SCOPE_GLOBAL && U.state == ST_RADIX && U.r_src == SRC_CAND && !U.mode_t && !U.overflow &&
+           U.n_alloc >= RADIX_FLAT_MIN;
 }
 
 // Large pools (radix_flat): every block takes a slice of the unit's pool
@@ -909,7 +969,7 @@ __global__ void __launch_bounds__(TPB) k_radix_flat(Plan P) {
     const int KU = P.K * P.n_units;
     for (int u = 0; u < KU; ++u) {
         const Unit& U = P.units[u];
-        if (!radix_flat(U)) continue;                  // the same for every thread
+        if (!radix_flat(P, U)) continue;                  // the same for every thread
         const int pshift = U.r_pshift;
         const int shift = pshift > RADIX_BITS ? pshift - RADIX_BITS : 0;
         const int nb = 1 << (pshift - shift);
@@ -992,7 +1052,7 @@ __global__ void __launch_bounds__(TPB) k_radix_hist(Plan P) {
         const long long run_end = c.run_end < end ? c.run_end : end;
         const TensorDesc& d = P.tens[c.t];
         Unit* U = (d.flags & TF_TRIM) ? unit_of(P, c.i, d) : nullptr;
-        if (!U || U->state != ST_RADIX || radix_flat(*U)) { it = run_end; continue; }
+        if (!U || U->state != ST_RADIX || radix_flat(P, *U)) { it = run_end; continue; }
         const long long ui = U - P.units;
         const int pshift = U->r_pshift;
         const int shift = pshift > RADIX_BITS ? pshift - RADIX_BITS : 0;
@@ -1184,7 +1244,7 @@ __device__ __forceinline__ void write_unit_stats(const Plan& P, int idx, const U
     const int i = idx / P.n_units, u = idx % P.n_units;
     iso_unit_stats s;
     s.thresh_key = (U.state == ST_OFF) ? KEY_NONE : U.t;
-    s.flags = (U.fallback ? 1u : 0u) | (U.mode_t ? 2u : 0u) | (U.overflow ? 8u : 0u);
+    s.flags = (U.fallback ? 1u : 0u) | (U.mode_t ? 2u : 0u) | (U.overflow ? 8u : 0u) | (U.v_ok ? 32u : 0u);
     s.k = U.k;
     s.count_above = (U.state == ST_DONE) ? U.count_above : 0;
     s.ties_at_thresh = (U.state == ST_DONE) ? U.ties : 0;
@@ -1197,8 +1257,9 @@ __device__ __forceinline__ const uint32_t* cut_src(const Plan& P, const Unit& U)
     return ((U.tie_src == TIE_EQ_HI) ? P.teq_hi : (U.tie_src == TIE_EQ_LO) ? P.teq_lo : P.tcnt) +
            (long long)U.expert * P.n_tiles;
 }
-__device__ __forceinline__ bool cut_split(const Unit& U) {
-    return U.state == ST_TKNOWN && U.need < U.ties && U.tile_end - U.tile_begin >= CUT_SPLIT_MIN;
+__device__ __forceinline__ bool cut_split(const Plan& P, const Unit& U) {
+    return P.scope == ISO_SCOPE_GLOBAL && U.state == ST_TKNOWN && U.need < U.ties &&
+           U.tile_end - U.tile_begin >= CUT_SPLIT_MIN;
 }
 
 // For units with many tiles: the tie counts summed over RADIX_BINS chunks of
@@ -1212,7 +1273,7 @@ __global__ void __launch_bounds__(TPB) k_cut_part(Plan P) {
     const int KU = P.K * P.n_units;
     for (int u = 0; u < KU; ++u) {
         const Unit& U = P.units[u];
-        if (!cut_split(U)) continue;
+        if (!cut_split(P, U)) continue;
         const long long nt = U.tile_end - U.tile_begin;
         const long long per = (nt + RADIX_BINS - 1) / RADIX_BINS;
         const uint32_t* src = cut_src(P, U);
@@ -1248,7 +1309,7 @@ __global__ void __launch_bounds__(CUT_TPB) k_cut(Plan P) {
         //    unit with many tiles first picks the chunk from k_cut_part's sums
         const uint32_t* src = cut_src(P, U);
         long long lo_t = U.tile_begin, hi_t = U.tile_end, need = U.need;
-        if (cut_split(U)) {
+        if (cut_split(P, U)) {
             __shared__ long long s_c0, s_c1, s_before;
             const long long nt = U.tile_end - U.tile_begin;
             const long long per_c = (nt + RADIX_BINS - 1) / RADIX_BINS;
@@ -1380,7 +1441,8 @@ __global__ void __launch_bounds__(CUT_TPB) k_cut(Plan P) {
 #define ISO_SELECT_INST(XT, BT, CK)                                            \
     template __global__ void k_sample<XT, BT, CK>(Plan);                      \
     template __global__ void k_csample<XT, BT, CK>(Plan);                     \
-    template __global__ void k_count<XT, BT, CK>(Plan);                       \
+    template __global__ void k_count<XT, BT, CK, false>(Plan);                \
+    template __global__ void k_count<XT, BT, CK, true>(Plan);                 \
     template __global__ void k_radix_hist<XT, BT, CK>(Plan);                  \
     template __global__ void k_tie<XT, BT, CK>(Plan);                         \
     template __global__ void k_cut<XT, BT, CK>(Plan);
