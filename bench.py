@@ -450,6 +450,7 @@ def run_mine(args):
     ckpt = inputs == "ckpt_bf16"
     out = [torch.empty_like(t) for t in th0]
     iso.force_two_pass(args.two_pass)
+    iso.compact_candidates(args.compact_candidates)
     cfg = iso.merge_cfg(op, density, scope)
     mn, full = iso.iso_workspace_size(th0, K, cfg)
     free = torch.cuda.mem_get_info(dev)[0]
@@ -775,6 +776,9 @@ def main():
                          "instead of a replica per rank (weak scaling)")
     ap.add_argument("--density", type=float, default=None,
                     help="TopKMask density (default: the workload's own)")
+    ap.add_argument("--compact-candidates", action="store_true",
+                    help="K >= 2 TIES / ISO: the Gram and merge passes read the counting pass's "
+                         "compact candidate values (iso_compact_candidates)")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--e2e-group-mb", type=int, default=2048,
                     help="end-to-end leg: bytes (MiB) of one tensor group of the host-staged pipeline")

@@ -604,8 +604,12 @@ int run_group(const Call& c, int t0, int t1, char* ws, cudaStream_t s, const iso
                     ISO_TRY(launch(KD_COUNT, s, [&] { k_count_apply<false><<<sms * FUSED_GRID_PER_SM, TPB, FUSED_SMEM, s>>>(P); }));
                 }
             } else {
-                if (c.ccv)
-                    ISO_TRY(launch(KD_COUNT, s, [&] { k_count<XT, BT, CK, true><<<sms * COUNT_GRID_PER_SM, TPB, 0, s>>>(P); }));
+                if (c.ccv) {
+                    ISO_TRY(smem_optin(k_count<XT, BT, CK, true>, COUNT_EMIT_SMEM));
+                    ISO_TRY(launch(KD_COUNT, s, [&] {
+                        k_count<XT, BT, CK, true><<<sms * COUNT_GRID_PER_SM, TPB, COUNT_EMIT_SMEM, s>>>(P);
+                    }));
+                }
                 else
                     ISO_TRY(launch(KD_COUNT, s, [&] { k_count<XT, BT, CK, false><<<sms * COUNT_GRID_PER_SM, TPB, 0, s>>>(P); }));
             }
@@ -677,7 +681,11 @@ int run_group(const Call& c, int t0, int t1, char* ws, cudaStream_t s, const iso
                 auto gram = [&](auto kc) {
                     constexpr int KC = decltype(kc)::value;
                     if constexpr (KC >= 2) {
-                        if (c.ccv) return launch(KD_GRAM, s, [&] { k_gramk_c<XT, BT, CK, KC><<<sms * 2, TPB, 0, s>>>(P); });
+                        if (c.ccv) {
+                            const int cs = compact_smem_bytes<BT, KC>();
+                            ISO_TRY(smem_optin(k_gramk_c<XT, BT, CK, KC>, cs));
+                            return launch(KD_GRAM, s, [&] { k_gramk_c<XT, BT, CK, KC><<<sms * 2, TPB, cs, s>>>(P); });
+                        }
                     }
                     const int ggrid = sms * gram_blocks_per_sm(KC);
                     const int smem = gram_smem_bytes<XT, BT, KC>();
@@ -693,10 +701,15 @@ int run_group(const Call& c, int t0, int t1, char* ws, cudaStream_t s, const iso
         }
         auto merge = [&](auto kc) {
             constexpr int KC = decltype(kc)::value;
-            if (c.ccv && c.op == ISO_OP_TIES)
-                return launch(KD_APPLY, s, [&] { k_merge_c<XT, BT, CK, KC, OPF_TIES><<<sms * 2, TPB, 0, s>>>(P); });
-            if (c.ccv)
-                return launch(KD_APPLY, s, [&] { k_merge_c<XT, BT, CK, KC, OPF_OTHER><<<sms * 2, TPB, 0, s>>>(P); });
+            if (c.ccv) {
+                const int cs = compact_smem_bytes<BT, KC>();
+                if (c.op == ISO_OP_TIES) {
+                    ISO_TRY(smem_optin(k_merge_c<XT, BT, CK, KC, OPF_TIES>, cs));
+                    return launch(KD_APPLY, s, [&] { k_merge_c<XT, BT, CK, KC, OPF_TIES><<<sms * 2, TPB, cs, s>>>(P); });
+                }
+                ISO_TRY(smem_optin(k_merge_c<XT, BT, CK, KC, OPF_OTHER>, cs));
+                return launch(KD_APPLY, s, [&] { k_merge_c<XT, BT, CK, KC, OPF_OTHER><<<sms * 2, TPB, cs, s>>>(P); });
+            }
             if (c.op == ISO_OP_TIES) {
                 const int smem = merge_smem_bytes<XT, BT, KC, OPF_TIES>();
                 const int mgrid = sms * merge_blocks_per_sm(KC, OPF_TIES);

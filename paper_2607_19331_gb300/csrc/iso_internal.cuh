@@ -48,6 +48,7 @@ constexpr int RADIX_BINS = 1 << RADIX_BITS;
 // KEY_NONE), not tile by tile.
 constexpr unsigned long long RADIX_FLAT_MIN = 1ull << 20;
 constexpr int RADIX_FLAT_SMEM = (WPB + 2) * RADIX_BINS * 4;   // k_radix_flat's dynamic shared memory
+constexpr int COUNT_EMIT_SMEM = WPB * 32 * 33 * 4;               // k_count<..., true>'s dynamic shared memory
 // A unit with at least this many tiles finds the tile of its cut from
 // per-chunk tie sums (k_cut_part, RADIX_BINS chunks) before it scans tiles.
 constexpr long long CUT_SPLIT_MIN = 1ll << 16;

@@ -76,6 +76,8 @@ template <typename XT, typename BT, int KC> int gram_smem_bytes();
 constexpr int gram_blocks_per_sm(int KC) { return 2; }
 template <typename XT, typename BT, bool CK, int KC, int OPF> __global__ void k_merge_c(Plan P);
 template <typename XT, typename BT, bool CK, int KC> __global__ void k_gramk_c(Plan P);
+// the compact kernels' dynamic shared memory (one stage per warp)
+template <typename BT, int KC> int compact_smem_bytes();
 __global__ void k_solve(Plan P, int gram_mode);
 template <typename XT> __global__ void k_mask(Plan P, uint32_t* const* mptr);
 __global__ void k_status(const Header* h, int32_t* out);

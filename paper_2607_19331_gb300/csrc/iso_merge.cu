@@ -822,35 +822,80 @@ __device__ __forceinline__ void compact_params(const Plan& P, int t, int K, Comp
 
 // the tile's mask words, their exclusive popcount prefix and the value
 // pointer of each compact expert, in the warp's shared memory (registers
-// stay free for the data)
-template <int KC>
+// stay free for the data); the tile's values of each expert (when they fit
+// CC_STAGE slots) and the tile's theta_0 are copied into the warp's stage
+// with cp.async before the tile is merged, so that the merge reads shared
+// memory only: two round trips to memory per tile (mask words, then values)
+// instead of one per step.
+constexpr int CC_STAGE = 256;
+template <int KC, typename BT>
 struct CompactTile {
     uint32_t mw[KC][32], pre[KC][32];
     const float* vb[KC];
+    uint32_t staged;                   // bit q: expert q's values are in sv[q]
+    float sv[KC][CC_STAGE];
+    __align__(16) char th0[TILE * sizeof(BT)];
 };
 
-template <int KC>
+__device__ __forceinline__ void cp_async4(uint32_t dst, const void* src) {
+    asm volatile("cp.async.ca.shared.global [%0], [%1], 4;" :: "r"(dst), "l"(src) : "memory");
+}
+
+template <int KC, typename BT>
 __device__ __forceinline__ void compact_tile(const Plan& P, const CompactParams<KC>& cp, int K, long long g, int lane,
-                                             CompactTile<KC>& ct) {
+                                             const void* base, long long e0, long long n, bool want_base,
+                                             CompactTile<KC, BT>& ct) {
     __syncwarp();
+    uint32_t cnt[KC];
 #pragma unroll
     for (int q = 0; q < KC; ++q) {
+        cnt[q] = 0;
         if (q < K && ((cp.vok >> q) & 1u)) {
             const long long rec = (long long)q * P.n_tiles + g;
             const uint32_t w = P.vmask[rec * 32 + lane];
-            uint32_t tot;
-            ct.pre[q][lane] = warp_excl_scan((uint32_t)__popc(w), &tot);
+            ct.pre[q][lane] = warp_excl_scan((uint32_t)__popc(w), &cnt[q]);
             ct.mw[q][lane] = w;
             if (lane == 0) ct.vb[q] = P.vals + cp.voff[q] + P.tval[rec];
         }
     }
     __syncwarp();
+    uint32_t staged = 0;
+#pragma unroll
+    for (int q = 0; q < KC; ++q) {
+        if (q < K && ((cp.vok >> q) & 1u) && cnt[q] <= (uint32_t)CC_STAGE) {
+            staged |= 1u << q;
+            const float* src = ct.vb[q];
+            const uint32_t dst = (uint32_t)__cvta_generic_to_shared(&ct.sv[q][0]);
+            for (uint32_t i = lane; i < cnt[q]; i += 32) cp_async4(dst + 4 * i, src + i);
+        }
+    }
+    if (want_base) {
+        // the tile's theta_0, 16 bytes per lane per copy, zero-filled past the tensor's end
+        const uint32_t dst = (uint32_t)__cvta_generic_to_shared(ct.th0);
+        const char* src = static_cast<const char*>(base) + e0 * (long long)sizeof(BT);
+        const long long avail = (n - e0) * (long long)sizeof(BT);
+#pragma unroll
+        for (int k = 0; k < (int)(TILE * sizeof(BT)) / 512; ++k) {
+            const long long off = (long long)k * 512 + lane * 16;
+            cp_async16(dst + (uint32_t)off, src + (avail > off ? off : 0), clamp_bytes(avail - off, 16));
+        }
+    }
+    cp_async_commit();
+    cp_async_wait<0>();
+    if (lane == 0) ct.staged = staged;
+    __syncwarp();
+}
+
+template <typename BT>
+__device__ __forceinline__ float staged_base(const char* th0, int p) {
+    if (sizeof(BT) == 4) return reinterpret_cast<const float*>(th0)[p];
+    return __uint_as_float((uint32_t)reinterpret_cast<const unsigned short*>(th0)[p] << 16);
 }
 
 // tau of entries e .. e + 3 (step s of the tile) for every expert: compact
 // values, or the full task vector; entries past the tensor's end read 0
 template <typename XT, typename BT, bool CK, int KC>
-__device__ __forceinline__ void compact_step(const CompactParams<KC>& cp, const CompactTile<KC>& ct,
+__device__ __forceinline__ void compact_step(const CompactParams<KC>& cp, const CompactTile<KC, BT>& ct,
                                              const void* const* xs, int K, long long e, long long n, int s, int lane,
                                              const float (&th0)[4], float (&tau)[KC][4]) {
     const int w = s * 4 + (lane >> 3), bo = (lane & 7) * 4;
@@ -863,11 +908,12 @@ __device__ __forceinline__ void compact_step(const CompactParams<KC>& cp, const 
             const uint32_t word = ct.mw[q][w];
             const uint32_t at = ct.pre[q][w] + (uint32_t)__popc(word & ((1u << bo) - 1u));
             const uint32_t nib = (word >> bo) & 0xFu;
-            const float* vb = ct.vb[q] + at;
+            const bool st = (ct.staged >> q) & 1u;
+            const float* vb = (st ? &ct.sv[q][0] : ct.vb[q]) + at;
             uint32_t r = 0;
 #pragma unroll
             for (int j = 0; j < 4; ++j) {
-                if ((nib >> j) & 1u) { tau[q][j] = __ldg(vb + r); ++r; }
+                if ((nib >> j) & 1u) { tau[q][j] = st ? vb[r] : __ldg(vb + r); ++r; }
             }
         } else {
             Words<XT, 4> x;
@@ -890,7 +936,8 @@ __global__ void __launch_bounds__(TPB, 2) k_merge_c(Plan P) {
     if (wr.beg >= wr.end) return;
     __shared__ MergeParams<KC> s_mp[WPB];
     __shared__ CompactParams<KC> s_cp[WPB];
-    __shared__ CompactTile<KC> s_ct[WPB];
+    extern __shared__ __align__(16) char s_cstage[];
+    CompactTile<KC, BT>& ct = reinterpret_cast<CompactTile<KC, BT>*>(s_cstage)[warp];
     MergeParams<KC>& mp = s_mp[warp];
     CompactParams<KC>& cp = s_cp[warp];
     int t = tensor_of_tile(P.tens, P.n_tensors, wr.beg);
@@ -917,17 +964,14 @@ __global__ void __launch_bounds__(TPB, 2) k_merge_c(Plan P) {
         for (int q = 0; q < KC; ++q) cf[q] = (OPF == OPF_TIES) ? 0.0f : mp.cf[q];
         const int opk = (OPF == OPF_TIES) ? (int)OPK_TIES : mp.opk;
         const bool iso1d = mp.iso1d;
-        CompactTile<KC>& ct = s_ct[warp];
-        compact_tile<KC>(P, cp, K, g, lane, ct);
+        compact_tile<KC, BT>(P, cp, K, g, lane, d.base, e0, n, true, ct);
         uint32_t kmax = 0;
 #pragma unroll 1
         for (int s = 0; s < SPT; ++s) {
             const long long e = e0 + (long long)s * (32 * E) + lane * E;
-            Words<BT, E> b;
-            load_words<BT, E>(d.base, e, n, b);
             float th0[E];
 #pragma unroll
-            for (int j = 0; j < E; ++j) th0[j] = word_f32<BT, E>(b, j);
+            for (int j = 0; j < E; ++j) th0[j] = staged_base<BT>(ct.th0, s * (32 * E) + lane * E + j);
             float tau[KC][E];
             compact_step<XT, BT, CK, KC>(cp, ct, mp.xs, K, e, n, s, lane, th0, tau);
             long long r = 0, c = 0;
@@ -965,7 +1009,8 @@ __global__ void __launch_bounds__(TPB, 2) k_gramk_c(Plan P) {
     if (wr.beg >= wr.end) return;
     __shared__ MergeParams<KC> s_mp[WPB];
     __shared__ CompactParams<KC> s_cp[WPB];
-    __shared__ CompactTile<KC> s_ct[WPB];
+    extern __shared__ __align__(16) char s_cstage[];
+    CompactTile<KC, BT>& ct = reinterpret_cast<CompactTile<KC, BT>*>(s_cstage)[warp];
     MergeParams<KC>& mp = s_mp[warp];
     CompactParams<KC>& cp = s_cp[warp];
     int t = tensor_of_tile(P.tens, P.n_tensors, wr.beg);
@@ -1003,8 +1048,8 @@ __global__ void __launch_bounds__(TPB, 2) k_gramk_c(Plan P) {
         const long long e1 = (e0 + TILE < n) ? e0 + TILE : n;
         int T[KC];
         const bool exact = tile_thresholds<KC>(mp, K, (uint32_t)e0, (uint32_t)e1, T);
-        CompactTile<KC>& ct = s_ct[warp];
-        compact_tile<KC>(P, cp, K, g, lane, ct);
+        const bool want_base = CK && cp.vok != ((1u << K) - 1u);
+        compact_tile<KC, BT>(P, cp, K, g, lane, d.base, e0, n, want_base, ct);
         float acc[NP];
 #pragma unroll
         for (int q = 0; q < NP; ++q) acc[q] = 0.0f;
@@ -1012,11 +1057,9 @@ __global__ void __launch_bounds__(TPB, 2) k_gramk_c(Plan P) {
         for (int s = 0; s < SPT; ++s) {
             const long long e = e0 + (long long)s * (32 * E) + lane * E;
             float th0[E] = {0.0f, 0.0f, 0.0f, 0.0f};
-            if (CK && cp.vok != ((1u << K) - 1u)) {
-                Words<BT, E> b;
-                load_words<BT, E>(d.base, e, n, b);
+            if (want_base) {
 #pragma unroll
-                for (int j = 0; j < E; ++j) th0[j] = word_f32<BT, E>(b, j);
+                for (int j = 0; j < E; ++j) th0[j] = staged_base<BT>(ct.th0, s * (32 * E) + lane * E + j);
             }
             float tau[KC][E];
             compact_step<XT, BT, CK, KC>(cp, ct, mp.xs, K, e, n, s, lane, th0, tau);
@@ -1063,6 +1106,8 @@ __global__ void __launch_bounds__(TPB, 2) k_gramk_c(Plan P) {
 
 template <typename XT, typename BT, int KC, int OPF>
 int merge_smem_bytes() { return StageGeom<XT, BT, KC, merge_blocks_per_sm(KC, OPF)>::SMEM; }
+template <typename BT, int KC>
+int compact_smem_bytes() { return WPB * (int)sizeof(CompactTile<KC, BT>); }
 template <typename XT, typename BT, int KC>
 int gram_smem_bytes() { return StageGeom<XT, BT, KC, gram_blocks_per_sm(KC)>::SMEM; }
 
@@ -1077,6 +1122,12 @@ int gram_smem_bytes() { return StageGeom<XT, BT, KC, gram_blocks_per_sm(KC)>::SM
     template int gram_smem_bytes<XT, BT, 2>();                                \
     template int gram_smem_bytes<XT, BT, 4>();                                \
     template int gram_smem_bytes<XT, BT, 8>();
+template int compact_smem_bytes<__nv_bfloat16, 2>();
+template int compact_smem_bytes<__nv_bfloat16, 4>();
+template int compact_smem_bytes<__nv_bfloat16, 8>();
+template int compact_smem_bytes<float, 2>();
+template int compact_smem_bytes<float, 4>();
+template int compact_smem_bytes<float, 8>();
 ISO_MERGE_SMEM(__nv_bfloat16, __nv_bfloat16)
 ISO_MERGE_SMEM(__nv_bfloat16, float)
 ISO_MERGE_SMEM(float, __nv_bfloat16)

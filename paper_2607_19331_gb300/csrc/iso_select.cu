@@ -570,11 +570,17 @@ __device__ __forceinline__ bool count_run_at(const Plan& P, uint32_t it, uint32_
 }
 
 // EMIT: also write the compact candidates (Plan::ccv); a separate
-// instantiation, so the plain counting pass keeps its registers
+// instantiation, so the plain counting pass keeps its registers.  The tile's
+// binary32 task vector is kept in COUNT_EMIT_SMEM bytes of dynamic shared
+// memory (32 rows of 33 words per warp, row w holding positions 32 w ..
+// 32 w + 31), and after the count each lane turns one row into its mask word
+// and writes the row's candidates in position order.
 template <typename XT, typename BT, bool CK, bool EMIT>
 __global__ void __launch_bounds__(TPB, COUNT_BLOCKS_PER_SM) k_count(Plan P) {
     __shared__ uint32_t s_band[WPB][TILE + 32];
+    extern __shared__ float s_vst[];
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    float* const vrow = s_vst + warp * (32 * 33);
     uint32_t* const sbl = s_band[warp] + lane;
     // item indices fit 32 bits (the host checks K * n_tiles < 2^31)
     const uint32_t W = gridDim.x * WPB;
@@ -613,7 +619,7 @@ __global__ void __launch_bounds__(TPB, COUNT_BLOCKS_PER_SM) k_count(Plan P) {
     // segment; a tile needs at most TILE slots, taken before the tile
     float* vseg = nullptr;
     unsigned long long v_pos = 0;
-    uint32_t v_left = 0, v_run = 0;
+    uint32_t v_left = 0;
     bool v_ovf = false;
 
     auto flush = [&]() {
@@ -683,26 +689,15 @@ __global__ void __launch_bounds__(TPB, COUNT_BLOCKS_PER_SM) k_count(Plan P) {
                 if (start + req > au->v_cap) v_ovf = true;
                 else { v_pos = start; v_left = req; }
             }
-            v_run = 0;
         }
-        // compact candidates of one vector step: the lane's entries with
-        // key >= lo (bits of m) in position order, and the step's mask words
-        // (lanes 4 q .. 4 q + 3 hold the 32 positions of word 8 v + q)
-        auto emit = [&](int v, const float (&tau)[VEC], uint32_t m) {
-            uint32_t tot;
-            const uint32_t off = warp_excl_scan((uint32_t)__popc(m), &tot);
-            if (!v_ovf) {
-                float* dst = vseg + v_pos + v_run + off;
-                int r = 0;
+        // the step's binary32 values into the warp's rows (position
+        // 256 v + 8 lane + j: row 8 v + lane / 4, column 8 (lane % 4) + j;
+        // the 33-word rows keep both this and the row-per-lane reads free of
+        // bank conflicts)
+        auto stash = [&](int v, const float (&tau)[VEC]) {
+            float* d = vrow + (8 * v + (lane >> 2)) * 33 + 8 * (lane & 3);
 #pragma unroll
-                for (int j = 0; j < VEC; ++j)
-                    if ((m >> j) & 1u) dst[r++] = tau[j];
-            }
-            v_run += tot;
-            const uint32_t b1 = __shfl_down_sync(FULL, m, 1), b2 = __shfl_down_sync(FULL, m, 2);
-            const uint32_t b3 = __shfl_down_sync(FULL, m, 3);
-            if ((lane & 3) == 0)
-                P.vmask[(size_t)rec * 32 + v * 8 + (lane >> 2)] = m | (b1 << 8) | (b2 << 16) | (b3 << 24);
+            for (int j = 0; j < VEC; ++j) d[j] = tau[j];
         };
 
         // pass 1: every entry
@@ -715,7 +710,6 @@ __global__ void __launch_bounds__(TPB, COUNT_BLOCKS_PER_SM) k_count(Plan P) {
                 float tau[VEC];
                 rt.tau(v, tau);
                 if (more) rt.load_step(v, r2.xp, r2.bp, ne0, nrem, lane);
-                uint32_t m = 0;
 #pragma unroll
                 for (int j = 0; j < VEC; ++j) {
                     const uint32_t kk = key_of(tau[j]);
@@ -724,9 +718,8 @@ __global__ void __launch_bounds__(TPB, COUNT_BLOCKS_PER_SM) k_count(Plan P) {
                     f_gg = gt ? __fmaf_rn(tau[j], tau[j], f_gg) : f_gg;
                     *sp = kk;
                     sp += (kk - lo <= span) ? 32 : 0;
-                    if (EMIT) m |= (uint32_t)(kk >= lo) << j;
                 }
-                if constexpr (EMIT) emit(v, tau, m);
+                if constexpr (EMIT) stash(v, tau);
             }
         } else {
 #pragma unroll
@@ -735,7 +728,6 @@ __global__ void __launch_bounds__(TPB, COUNT_BLOCKS_PER_SM) k_count(Plan P) {
                 rt.tau(v, tau);
                 if (more) rt.load_step(v, r2.xp, r2.bp, ne0, nrem, lane);
                 const uint32_t o = (uint32_t)(v * (32 * VEC) + lane * VEC);
-                uint32_t m = 0;
 #pragma unroll
                 for (int j = 0; j < VEC; ++j) {
                     if (o + j >= rem) continue;
@@ -745,9 +737,8 @@ __global__ void __launch_bounds__(TPB, COUNT_BLOCKS_PER_SM) k_count(Plan P) {
                     f_gg = gt ? __fmaf_rn(tau[j], tau[j], f_gg) : f_gg;
                     *sp = kk;
                     sp += ((kk >= lo) & !gt) ? 32 : 0;
-                    if (EMIT) m |= (uint32_t)(kk >= lo) << j;
                 }
-                if constexpr (EMIT) emit(v, tau, m);
+                if constexpr (EMIT) stash(v, tau);
             }
         }
         const uint32_t nb = (uint32_t)(sp - sbl) >> 5;
@@ -812,7 +803,31 @@ __global__ void __launch_bounds__(TPB, COUNT_BLOCKS_PER_SM) k_count(Plan P) {
             P.teq_hi[rec] = t_hi;
             if (EMIT) P.tval[rec] = v_ovf ? KEY_NONE : (uint32_t)v_pos;
         }
-        if (EMIT && !v_ovf) { v_pos += v_run; v_left -= v_run; }
+        if constexpr (EMIT) {
+            // lane l: row l (positions 32 l .. 32 l + 31) into mask word l and
+            // its values with key >= lo, in position order
+            __syncwarp();
+            const float* row = vrow + lane * 33;
+            uint32_t m = 0;
+#pragma unroll
+            for (int q = 0; q < 32; ++q)
+                m |= (uint32_t)(key_of(row[q]) >= lo && (uint32_t)(32 * lane + q) < rem) << q;
+            uint32_t tot;
+            const uint32_t off = warp_excl_scan((uint32_t)__popc(m), &tot);
+            if (!v_ovf) {
+                float* dst = vseg + v_pos + off;
+                uint32_t mm = m;
+                while (mm) {
+                    const int q = __ffs(mm) - 1;
+                    mm &= mm - 1;
+                    *dst++ = row[q];
+                }
+                v_pos += tot;
+                v_left -= tot;
+            }
+            P.vmask[(size_t)rec * 32 + lane] = m;
+            __syncwarp();
+        }
         if (store) { ch_pos += t_int; ch_left -= t_int; }
         a_gt += t_gt; a_int += t_int; a_hi += t_hi; a_lo += t_lo;
         __syncwarp();
