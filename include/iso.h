@@ -449,7 +449,7 @@ int32_t iso_force_two_pass(int32_t on);
  * (density <= 0.3) let the counting pass write each expert's candidate values
  * (the entries at or above the low edge of its sampled band, in position
  * order, with a bit mask per tile), so that the Gram and merge passes read
- * those instead of the full task vectors; on by default.  The results are
+ * those instead of the full task vectors; off by default.  The results are
  * the same either way. */
 int32_t iso_compact_candidates(int32_t on);
 

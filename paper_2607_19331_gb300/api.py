@@ -354,8 +354,8 @@ def force_two_pass(on=True):
 
 def compact_candidates(on=True):
     """Diagnostics: let later K >= 2 TIES / ISO merges read compact candidate
-    values in their Gram and merge passes (the default) or the full task
-    vectors; the results are the same."""
+    values in their Gram and merge passes, or the full task vectors (the
+    default); the results are the same."""
     check(lib().iso_compact_candidates(int(bool(on))), "iso_compact_candidates")
 
 

@@ -206,17 +206,18 @@ def test_workspace_at_full_model_sizes():
     assert g_mn == g_full and 1e9 < g_full < 8e9
     t_mn, t_full = size("iso", "tensor", 1, _abi.ISO_BF16, 0.05)
     assert t_mn < t_full < 20e9
-    # eight experts: the full size holds every expert's compact candidates
-    # (about 15 % of its entries as binary32 plus a bit per entry); without
-    # them the full passes need a fraction of that
+    # eight experts: the full passes (the default) need a few GB per group;
+    # with compact candidates the full size also holds every expert's
+    # candidate values (about 15 % of its entries as binary32 plus a bit per
+    # entry), while the smallest workspace stays that of the full passes
     k_mn, k_full = size("ties", "tensor", 8, _abi.ISO_F32, 0.1)
-    assert k_mn < k_full < 80e9
-    iso.compact_candidates(False)
+    assert k_mn < k_full < 20e9
+    iso.compact_candidates(True)
     try:
         k_mn2, k_full2 = size("ties", "tensor", 8, _abi.ISO_F32, 0.1)
     finally:
-        iso.compact_candidates(True)
-    assert k_mn2 == k_mn and k_full2 < 20e9 and k_full - k_full2 > 30e9
+        iso.compact_candidates(False)
+    assert k_mn2 == k_mn and k_full2 < 80e9 and k_full2 - k_full > 30e9
     r_mn, r_full = size("ram", "tensor", 8, _abi.ISO_F32, 0.0)
     assert r_full < (1 << 20)
     cfg = iso.merge_cfg("ties", 0.1)
