@@ -43,7 +43,7 @@ __device__ void block_find_from_top_b(const uint32_t* hist, int nb, long long ra
 __device__ __forceinline__ int kpad(int q) { return q + (q >> 5); }
 
 template <typename XT, typename BT, bool CK>
-__global__ void __launch_bounds__(BLOCK_TPB, 1) k_block_select(Plan P) {
+__global__ void __launch_bounds__(BLOCK_TPB, BLOCK_CTAS_PER_SM) k_block_select(Plan P) {
     extern __shared__ __align__(16) uint32_t s_keys[];      // kpad(BLOCK_MAX_ENTRIES)
     __shared__ uint32_t s_hist[RADIX_BINS];
     __shared__ long long s_scan[33];
@@ -138,8 +138,10 @@ __global__ void __launch_bounds__(BLOCK_TPB, 1) k_block_select(Plan P) {
     }
     const bool want_gamma = (P.op == ISO_OP_ISO) && (P.K == 1);
 
-    // Full block of BLOCK_TPB x 16 entries in rows of a multiple of 16: each
-    // thread holds 16 consecutive entries (block order) in registers, and the
+    // Full block of BLOCK_TPB x BFE entries in rows of a multiple of BFE: each
+    // thread holds BFE consecutive entries (block order) in registers -- their
+    // keys and one word of signs, from which each tau is rebuilt exactly --
+    // and the
     // threshold is found bit by bit from the top: t is the largest key value v
     // with #{key >= v} >= k, so a bit is kept when the block still counts k
     // keys at or above the prefix with that bit set.  No atomics, no bank
@@ -150,17 +152,24 @@ __global__ void __launch_bounds__(BLOCK_TPB, 1) k_block_select(Plan P) {
         const int tq = threadIdx.x * BFE;
         const int rr = tq / (int)w, cc = tq - rr * (int)w;
         const long long ea = (r0 + rr) * d.cols + c0 + cc;     // tensor position of the thread's first entry
-        float tau[BFE];
+        static_assert(BFE <= 32, "one sign word per thread");
+        uint32_t key[BFE];
+        uint32_t sgn = 0;
 #pragma unroll
         for (int g = 0; g < BFE / VEC; ++g) {
             float t8[VEC];
             TauSrc<XT, BT, CK>::load8(x, d.base, ea + g * VEC, d.numel, t8);
 #pragma unroll
-            for (int j = 0; j < VEC; ++j) tau[g * VEC + j] = t8[j];
+            for (int j = 0; j < VEC; ++j) {
+                const uint32_t b = __float_as_uint(t8[j]);
+                key[g * VEC + j] = b & 0x7FFFFFFFu;
+                sgn |= (b >> 31) << (g * VEC + j);
+            }
         }
+        auto tau_of = [&](int j) -> float { return __uint_as_float(key[j] | (((sgn >> j) & 1u) << 31)); };
         uint32_t kmax = 0, kor = 0;
 #pragma unroll
-        for (int j = 0; j < BFE; ++j) { const uint32_t kk = key_of(tau[j]); kmax = max(kmax, kk); kor |= kk; }
+        for (int j = 0; j < BFE; ++j) { kmax = max(kmax, key[j]); kor |= key[j]; }
         if (kmax >= KEY_INF) set_status(P.hdr, ISO_ERR_NONFINITE);
         kor = __reduce_or_sync(0xFFFFFFFFu, kor);
         if (threadIdx.x == 0) s_or = 0;
@@ -181,7 +190,7 @@ __global__ void __launch_bounds__(BLOCK_TPB, 1) k_block_select(Plan P) {
             const uint32_t cand = prefix | (1u << bit);
             uint32_t c = 0;
 #pragma unroll
-            for (int j = 0; j < BFE; ++j) c += key_of(tau[j]) >= cand;
+            for (int j = 0; j < BFE; ++j) c += key[j] >= cand;
             c = __reduce_add_sync(0xFFFFFFFFu, c);
             if ((threadIdx.x & 31) == 0 && c) atomicAdd(&s_cnt[cur], c);
             __syncthreads();
@@ -193,7 +202,7 @@ __global__ void __launch_bounds__(BLOCK_TPB, 1) k_block_select(Plan P) {
         const uint32_t tk = prefix;
         uint32_t above = 0, ties = 0;
 #pragma unroll
-        for (int j = 0; j < BFE; ++j) { const uint32_t kk = key_of(tau[j]); above += kk > tk; ties += kk == tk; }
+        for (int j = 0; j < BFE; ++j) { above += key[j] > tk; ties += key[j] == tk; }
         uint32_t tot_ties;
         const uint32_t ties_before = block_excl_scan(ties, s_scan32, &tot_ties);
         const uint32_t tot_above = block_sum(above, s_scan32);
@@ -204,15 +213,17 @@ __global__ void __launch_bounds__(BLOCK_TPB, 1) k_block_select(Plan P) {
             uint32_t acc = ties_before;
 #pragma unroll
             for (int j = 0; j < BFE; ++j)
-                if (key_of(tau[j]) == tk && (long long)(++acc) == need) s_cutq = ea + j + 1;
+                if (key[j] == tk && (long long)(++acc) == need) s_cutq = ea + j + 1;
         }
         double g = 0.0;
         if (want_gamma) {
             // squares of the entries above t as binary32 two-sum pairs, then binary64 over the block
             float sg = 0.0f, eg = 0.0f;
 #pragma unroll
-            for (int j = 0; j < BFE; ++j)
-                if (key_of(tau[j]) > tk) two_sum_add(sg, eg, __fmul_rn(tau[j], tau[j]));
+            for (int j = 0; j < BFE; ++j) {
+                const float f = __uint_as_float(key[j]);          // |tau|: the same square
+                if (key[j] > tk) two_sum_add(sg, eg, __fmul_rn(f, f));
+            }
             g = block_sum((double)sg + (double)eg, s_dred);
         }
         __syncthreads();
@@ -235,10 +246,9 @@ __global__ void __launch_bounds__(BLOCK_TPB, 1) k_block_select(Plan P) {
                 load8_tail<BT>(d.base, e, d.numel, th0);
 #pragma unroll
                 for (int j = 0; j < VEC; ++j) {
-                    const float tv = tau[gq * VEC + j];
-                    const uint32_t kk = key_of(tv);
+                    const uint32_t kk = key[gq * VEC + j];
                     const bool kept = kk > tk || (kk == tk && e + j < cut);
-                    o[j] = kept ? out_of(th0[j], tv, P.lambda) : th0[j];
+                    o[j] = kept ? out_of(th0[j], tau_of(gq * VEC + j), P.lambda) : th0[j];
                 }
                 store8(d.out, e, d.numel, o, obf);
             }

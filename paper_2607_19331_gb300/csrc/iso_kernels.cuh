@@ -34,7 +34,8 @@ __global__ void k_cut_part(Plan P);
 __global__ void k_radix_flat(Plan P);
 
 // select (BLOCK scope)
-constexpr int BLOCK_TPB = 1024;
+constexpr int BLOCK_TPB = 512;             // k_block_select: threads per unit (32 keys each on the fast path)
+constexpr int BLOCK_CTAS_PER_SM = 2;       // two units in flight per SM
 template <typename XT, typename BT, bool CK> __global__ void k_block_select(Plan P);
 
 // fused K = 1 pass (bf16 base and update)
